@@ -1,0 +1,407 @@
+"""Benchmark: block-restricted bidirectional selective scan, forward + backward.
+
+One step = the all-block forward (bdscan_forward) and backward
+(bdscan_backward) of one layer on one batch of synthetic input, through the
+C ABI, on the 87M-scale layer configuration: batch 8, clean and noisy streams
+of 2048 tokens, block 16, d_inner 1536, d_state 16, bf16 inputs/outputs with
+fp32 state. Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun each rank runs an independent replica on its own GPU (the
+scan needs no exchange between replicas); the elapsed time is the maximum
+over ranks and the value counts the tokens of all ranks. --impl reference
+times the fp64 CPU oracle (the reference arm of this method) on a bounded
+sample of the same workload, on rank 0 only.
+"""
+
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "block-bidir scan fwd+bwd tokens/sec on 1 GB300; achieved HBM GB/s vs ~8 TB/s"
+CFG = dict(batch=8, seq_len=2048, block=16, d_inner=1536, d_state=16)
+WORKLOAD = ("87M-scale layer: batch 8, clean+noisy streams of 2048 tokens each, block 16, d_inner 1536, "
+            "d_state 16, bf16 inputs/outputs, fp32 state; all-block forward + backward")
+KERNELS = ["chunk_local", "chunk_carry", "block_scan", "bwd_noisy", "bwd_carry", "bwd_clean", "reduce_tok",
+           "reduce_par"]
+
+
+def algorithmic_bytes(Bt, L, D, N, Bs, in_b=2, out_b=2):
+    """Bytes one forward+backward step must move at least: every input read
+    once per pass, every output written once, boundary states written by the
+    forward and read by the backward (no recompute or workspace traffic)."""
+    nb = L // Bs
+    td = Bt * L * D
+    tn = Bt * L * N
+    fwd = 5 * td * in_b + 6 * tn * in_b + 2 * td * out_b + Bt * nb * D * N * 4
+    bwd = (5 * td * in_b + 2 * td * in_b + 6 * tn * in_b + Bt * nb * D * N * 4
+           + 5 * td * out_b + 6 * tn * out_b)
+    return fwd, bwd
+
+
+def kernel_bytes(Bt, L, D, N, Bs, in_b=2, out_b=2):
+    """Per-kernel algorithmic bytes (the layer's own inputs and outputs each
+    kernel has to touch; workspace exchange between kernels excluded)."""
+    td, tn, nb = Bt * L * D, Bt * L * N, L // Bs
+    S = Bt * nb * D * N * 4
+    return {
+        "chunk_local": 2 * td * in_b + tn * in_b,
+        "chunk_carry": 0,
+        "block_scan": 5 * td * in_b + 6 * tn * in_b + 2 * td * out_b + S,
+        "bwd_noisy": 6 * td * in_b + 5 * tn * in_b + S + 3 * td * out_b,
+        "bwd_carry": 0,
+        "bwd_clean": 3 * td * in_b + 2 * tn * in_b + S + 2 * td * out_b,
+        "reduce_tok": 6 * tn * out_b,
+        "reduce_par": 0,
+    }
+
+
+# FP32 work per (token, channel, state) element of each scan kernel, counted
+# from the kernel's arithmetic (FMA = 2 flops; ex2, mul, add, reduction add = 1).
+KERNEL_FLOPS_PER_ELEM = {
+    "chunk_local": 6,     # dt*A, ex2, u*B, fma
+    "block_scan": 21,     # 3 directions x (dt*A, ex2, u*B, fma h, fma y)
+    "bwd_noisy": 47,      # clean local adjoint 5 + 2 directions x (recompute 7 + adjoint 14)
+    "bwd_clean": 21,      # recompute 7 + adjoint 14
+}
+
+
+def sample_clocks(stop, rows, bus_id):
+    cmd = ["nvidia-smi", "--query-gpu=pci.bus_id,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+           "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+           "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+           "--format=csv,noheader,nounits", "-lms", "200"]
+    try:
+        p = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+    except OSError:
+        return
+    try:
+        for line in p.stdout:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            if bus_id and bus_id.lower() not in f[0].lower() and f[0].lower() not in bus_id.lower():
+                continue
+            rows.append((time.time(), f))
+            if stop.is_set():
+                break
+    finally:
+        p.terminate()
+        try:
+            p.wait(timeout=2)
+        except Exception:
+            p.kill()
+
+
+def summarize_clocks(rows, t0, t1):
+    inside = [f for (ts, f) in rows if t0 <= ts <= t1]
+    used = inside if len(inside) >= 3 else [f for (_, f) in rows]
+    if not used:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"], "samples": 0}
+
+    def num(x):
+        try:
+            return float(x)
+        except ValueError:
+            return None
+
+    sm = [num(f[1]) for f in used if num(f[1]) is not None]
+    reasons = set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for f in used:
+        for name, v in zip(names, f[5:9]):
+            if v.strip().lower() == "active":
+                reasons.add(name)
+    return {"sm_mhz": statistics.median(sm) if sm else None,
+            "sm_max_mhz": max(num(f[2]) or 0 for f in used),
+            "power_w_max": max((num(f[3]) or 0) for f in used),
+            "reasons": sorted(reasons), "samples": len(used),
+            "window": "timed region" if len(inside) >= 3 else "warm-up and timed region"}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "sm_max_mhz": 2070.0}, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (reference arm and cpu_baseline)
+# ---------------------------------------------------------------------------
+def oracle_run(d_sample, seed=0, threads=None):
+    """fp64 oracle forward+backward on the configuration restricted to
+    `d_sample` channels (channels are independent, so the work is exactly
+    d_sample/d_inner of the full step). Returns (seconds, threads)."""
+    import oracle
+    from paper_2607_02805_gb300.inputs import Workload
+    oracle.build()
+    th = threads or max(1, min(os.cpu_count() or 1, 64))
+    oracle.set_threads(th)
+    wl = Workload(CFG["batch"], CFG["seq_len"], CFG["block"], d_sample, CFG["d_state"], dtype="bf16", seed=seed)
+    names = ("x_c", "dt_c", "B_c", "C_c", "x_n", "dt_f", "B_f", "C_f", "dt_r", "B_r", "C_r", "A_f", "D_f", "A_r",
+             "D_r")
+    d = {k: wl.f64(k) for k in wl.t32}
+    t0 = time.perf_counter()
+    y_c, y_n, st = oracle.forward(CFG["block"], *[d[k] for k in names])
+    oracle.backward(CFG["block"], *[d[k] for k in names], st, d["dy_c"], d["dy_n"], None)
+    return time.perf_counter() - t0, th
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    # size each step so the whole run stays within about 90 s of wall time
+    per_step = 90.0 / max(1, args.steps + args.warmup)
+    # measured: about 20 ns per (token, channel, state, stream) on one core, fwd+bwd
+    full_core_s = CFG["batch"] * CFG["seq_len"] * CFG["d_inner"] * CFG["d_state"] * 3 * 20e-9
+    th = max(1, min(os.cpu_count() or 1, 64))
+    eff = min(th, CFG["batch"])  # the oracle's backward runs one batch row per thread
+    d_s = int(max(8, min(CFG["d_inner"], CFG["d_inner"] * per_step * eff / full_core_s)))
+    for _ in range(args.warmup):
+        oracle_run(d_s, threads=th)
+    times = [oracle_run(d_s, threads=th)[0] for _ in range(args.steps)]
+    tok = CFG["batch"] * CFG["seq_len"] * d_s / CFG["d_inner"]
+    total = sum(times)
+    value = tok * args.steps / total
+    sample = (f"fp64 oracle fwd+bwd on {d_s} of {CFG['d_inner']} channels (batch 8, 2048 tokens, block 16, "
+              f"d_state 16); tokens scaled by {d_s}/{CFG['d_inner']}")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, **CFG, "parallelism": "cpu threads"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": th, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_02805_gb300 import binding
+    from paper_2607_02805_gb300.inputs import Workload
+    from paper_2607_02805_gb300.layer import Layer
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    Bt, L, Bs, D, N = CFG["batch"], CFG["seq_len"], CFG["block"], CFG["d_inner"], CFG["d_state"]
+    wl = Workload(Bt, L, Bs, D, N, dtype="bf16", seed=rank, with_grads=True)
+    lay = Layer(wl, device=dev)
+    lay.alloc_backward()
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        lay.forward(stream)
+        lay.backward(stream, use_dstates=False)
+
+    # per-kernel events through the library's timing hook
+    nk = len(KERNELS)
+    ev_start = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev_k = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(args.steps)]
+    arr_f = [(ctypes.c_void_p * 3)(*[e.cuda_event for e in evs[:3]]) for evs in ev_k]
+    arr_b = [(ctypes.c_void_p * (nk - 3))(*[e.cuda_event for e in evs[3:]]) for evs in ev_k]
+
+    def step_profiled(i):
+        ev_start[i].record(stream)
+        binding.bdscan_profile_events(arr_f[i], 3)
+        lay.forward(stream)
+        nf = binding.bdscan_last_launch_count()
+        binding.bdscan_profile_events(arr_b[i], nk - 3)
+        lay.backward(stream, use_dstates=False)
+        nb_ = binding.bdscan_last_launch_count()
+        binding.bdscan_profile_events(None, 0)
+        return nf + nb_
+
+    bus = ""
+    try:
+        bus = torch.cuda.get_device_properties(dev).pci_bus_id
+    except Exception:
+        pass
+    rows, stop = [], threading.Event()
+    sampler = threading.Thread(target=sample_clocks, args=(stop, rows, bus), daemon=True)
+    if rank == 0:
+        sampler.start()
+
+    # warm-up: at least W steps and about a second under load
+    t_w = time.time()
+    i = 0
+    while i < args.warmup or time.time() - t_w < 1.0:
+        step()
+        i += 1
+        if i % 50 == 0:
+            torch.cuda.synchronize(dev)
+    torch.cuda.synchronize(dev)
+    launches_per_step = 0
+
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t_start_wall = time.time()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.steps):
+        launches_per_step = step_profiled(i)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    t_end_wall = time.time()
+    ms = e0.elapsed_time(e1)
+    if launches_per_step != nk:
+        raise RuntimeError(f"expected {nk} kernel launches per step, the library reported {launches_per_step}")
+
+    # per-kernel average durations (event after kernel i minus event after kernel i-1)
+    per = [[] for _ in range(nk)]
+    for i in range(args.steps):
+        prev = ev_start[i]
+        for j in range(nk):
+            per[j].append(prev.elapsed_time(ev_k[i][j]))
+            prev = ev_k[i][j]
+    avg_us = [1e3 * statistics.mean(p) for p in per]
+
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # end-to-end through the public API with host buffers
+    e2e = run_e2e(lay, wl, stream, dev, args)
+    if world > 1:
+        t = torch.tensor([e2e["ms"]], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e["ms"] = float(t.item())
+    stop.set()
+
+    if rank != 0:
+        return
+    sampler.join(timeout=3)
+    clocks = summarize_clocks(rows, t_start_wall, t_end_wall)
+    ms_step = ms / args.steps
+    tokens = Bt * L * world
+    value = tokens / (ms_step / 1e3)
+    peaks, peak_kind = measured_peaks()
+    fb, bb = algorithmic_bytes(Bt, L, D, N, Bs)
+    kb = kernel_bytes(Bt, L, D, N, Bs)
+    total_us = sum(avg_us)
+    kernels = [{"name": k, "avg_us": round(u, 2), "share": round(u / total_us, 4),
+                "alg_bytes": kb[k], "alg_gbs": round(kb[k] / (u * 1e3), 1) if u > 0 else None}
+               for k, u in zip(KERNELS, avg_us)]
+    dom = max(range(nk), key=lambda j: avg_us[j])
+    dname = KERNELS[dom]
+    elems = Bt * L * D * N
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    fp32_peak_tflops = 152 * 128 * 2 * sm_max * 1e6 / 1e12
+    dom_flops = KERNEL_FLOPS_PER_ELEM.get(dname, 0) * elems
+    roofline = {"bound": "alu", "kernel": dname,
+                "achieved": round(dom_flops / (avg_us[dom] * 1e-6) / 1e12, 2),
+                "peak": round(fp32_peak_tflops, 1), "unit": "TFLOP/s",
+                "frac": round(dom_flops / (avg_us[dom] * 1e-6) / 1e12 / fp32_peak_tflops, 4),
+                "traffic": None,
+                "peak_kind": "derived: 152 SMs x 128 FP32 lanes x 2 flop/FMA x max SM clock",
+                "flops_per_launch": dom_flops}
+    hbm = {"bound": "hbm", "achieved": round((fb + bb) / (ms_step * 1e-3) / 1e9, 1),
+           "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
+           "frac": round((fb + bb) / (ms_step * 1e-3) / 1e9 / float(peaks.get("hbm_gbs", 6800.0)), 4),
+           "frac_of_8tbs": round((fb + bb) / (ms_step * 1e-3) / 8e12, 4),
+           "alg_bytes_per_step": fb + bb, "peak_kind": peak_kind,
+           "dominant_kernel_gbs": round(kb[dname] / (avg_us[dom] * 1e-6) / 1e9, 1)}
+
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        secs, th = oracle_run(CFG["d_inner"])
+        cpu = {"value": Bt * L / secs, "unit": "tokens/s", "cores": th, "kind": "oracle",
+               "sample": "fp64 oracle fwd+bwd of one full step of the same configuration (seed 0), "
+                         f"{th} OpenMP threads (the backward uses one per batch row)", "seconds": round(secs, 2)}
+
+    line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32 state, bf16 I/O", "data": "synthetic",
+            "config": {"workload": WORKLOAD, **CFG, "parallelism": "replicas" if world > 1 else "single",
+                       "l2": "inputs larger than L2 (about 0.36 GB of token tensors per step; no flush)"},
+            "roofline": roofline, "hbm": hbm, "cpu_baseline": cpu,
+            "e2e": {"value": tokens / (e2e["ms"] / 1e3), "unit": "tokens/s",
+                    "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"]},
+            "gpu_launches": launches_per_step * args.steps, "clocks": clocks, "kernels": kernels}
+    print(json.dumps(line), flush=True)
+
+
+def run_e2e(lay, wl, stream, dev, args):
+    """Forward + backward through the C ABI with host (pinned) inputs and a
+    device-to-host read of every output and gradient, timed per step."""
+    import torch
+    ins = [k for k in wl.t32]
+    host_in = {k: lay.t[k].detach().to("cpu").pin_memory() for k in ins}
+    outs = [lay.y_c, lay.y_n] + [lay.g[k] for k in lay.g]
+    host_out = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    steps = max(3, min(args.steps, 20))
+
+    def one():
+        for k in ins:
+            lay.t[k].copy_(host_in[k], non_blocking=True)
+        lay.forward(stream)
+        lay.backward(stream, use_dstates=False)
+        for o, h in zip(outs, host_out):
+            h.copy_(o, non_blocking=True)
+
+    for _ in range(3):
+        one()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    return {"ms": e0.elapsed_time(e1) / steps, "h2d": h2d, "d2h": d2h}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

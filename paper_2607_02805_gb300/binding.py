@@ -1,0 +1,256 @@
+"""ctypes binding of libbdscan (include/bdscan.h): argument marshalling only.
+
+Every function of the C ABI appears here under the same name and takes the
+same arguments; the ctypes structures mirror the C structs field by field.
+The tensor helpers at the bottom turn torch tensors into those structs (data
+pointers, the current CUDA stream) and raise on a non-zero return code. All
+computation happens in the CUDA library; if it cannot be loaded, every call
+raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "lib", "libbdscan.so")
+
+BDSCAN_OK = 0
+BDSCAN_ERR_ARG = -1
+BDSCAN_ERR_UNSUPPORTED = -2
+BDSCAN_ERR_CUDA = -3
+BDSCAN_F32 = 0
+BDSCAN_BF16 = 1
+
+c_void_p = ctypes.c_void_p
+
+
+class bdscan_dims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int64), ("len", ctypes.c_int64), ("block", ctypes.c_int64),
+                ("d_inner", ctypes.c_int64), ("d_state", ctypes.c_int64), ("dtype", ctypes.c_int32),
+                ("out_dtype", ctypes.c_int32)]
+
+
+class bdscan_clean(ctypes.Structure):
+    _fields_ = [("x", c_void_p), ("dt", c_void_p), ("B", c_void_p), ("C", c_void_p)]
+
+
+class bdscan_noisy(ctypes.Structure):
+    _fields_ = [("x", c_void_p), ("dt_f", c_void_p), ("B_f", c_void_p), ("C_f", c_void_p),
+                ("dt_r", c_void_p), ("B_r", c_void_p), ("C_r", c_void_p)]
+
+
+class bdscan_params(ctypes.Structure):
+    _fields_ = [("A_f", c_void_p), ("D_f", c_void_p), ("A_r", c_void_p), ("D_r", c_void_p)]
+
+
+class bdscan_clean_grads(ctypes.Structure):
+    _fields_ = [("dx", c_void_p), ("ddt", c_void_p), ("dB", c_void_p), ("dC", c_void_p)]
+
+
+class bdscan_noisy_grads(ctypes.Structure):
+    _fields_ = [("dx", c_void_p), ("ddt_f", c_void_p), ("dB_f", c_void_p), ("dC_f", c_void_p),
+                ("ddt_r", c_void_p), ("dB_r", c_void_p), ("dC_r", c_void_p)]
+
+
+class bdscan_param_grads(ctypes.Structure):
+    _fields_ = [("dA_f", c_void_p), ("dD_f", c_void_p), ("dA_r", c_void_p), ("dD_r", c_void_p)]
+
+
+# (name, restype, argtypes) of every exported function, in header order
+_P = ctypes.POINTER
+SIGNATURES = [
+    ("bdscan_last_error", ctypes.c_char_p, []),
+    ("bdscan_version", ctypes.c_int, []),
+    ("bdscan_chunk_tokens", ctypes.c_int64, [ctypes.c_int64]),
+    ("bdscan_profile_events", ctypes.c_int, [ctypes.POINTER(c_void_p), ctypes.c_int]),
+    ("bdscan_last_launch_count", ctypes.c_int, []),
+    ("bdscan_forward_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_forward", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_clean), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, c_void_p,
+      c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_backward_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_backward", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_clean), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, c_void_p,
+      c_void_p, _P(bdscan_clean_grads), _P(bdscan_noisy_grads), _P(bdscan_param_grads), c_void_p,
+      ctypes.c_size_t, c_void_p]),
+    ("bdscan_boundary_states_workspace_size", ctypes.c_size_t, [_P(bdscan_dims), ctypes.c_int]),
+    ("bdscan_boundary_states", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_clean), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, ctypes.c_int,
+      c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_active_block", ctypes.c_int,
+     [_P(bdscan_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
+]
+
+_lock = threading.Lock()
+_lib = None
+
+
+def load(build_if_missing: bool = True):
+    """Load the CUDA library (building it in-tree first if it is missing or stale)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if build_if_missing:
+                from . import build as _build
+                _build.build()
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(f"libbdscan is not built ({LIB_PATH} missing); run paper_2607_02805_gb300/build.py")
+            lib = ctypes.CDLL(LIB_PATH)
+            for name, res, args in SIGNATURES:
+                f = getattr(lib, name)
+                f.restype = res
+                f.argtypes = args
+            _lib = lib
+    return _lib
+
+
+class BdscanError(RuntimeError):
+    def __init__(self, fn, code, msg):
+        super().__init__(f"{fn} failed with code {code}: {msg}")
+        self.code = code
+
+
+def _call(name, *args):
+    lib = load()
+    rc = getattr(lib, name)(*args)
+    if rc != BDSCAN_OK:
+        raise BdscanError(name, rc, lib.bdscan_last_error().decode())
+    return rc
+
+
+def _ref(x):
+    return None if x is None else ctypes.byref(x)
+
+
+# raw functions, same names and arguments as the C ABI
+def bdscan_last_error() -> str:
+    return load().bdscan_last_error().decode()
+
+
+def bdscan_version() -> int:
+    return load().bdscan_version()
+
+
+def bdscan_chunk_tokens(block: int) -> int:
+    return load().bdscan_chunk_tokens(block)
+
+
+def bdscan_profile_events(events, n) -> int:
+    """events: a ctypes array of c_void_p (cudaEvent_t handles) or None."""
+    return load().bdscan_profile_events(events, int(n))
+
+
+def bdscan_last_launch_count() -> int:
+    return load().bdscan_last_launch_count()
+
+
+def bdscan_forward_workspace_size(dims) -> int:
+    return load().bdscan_forward_workspace_size(_ref(dims))
+
+
+def bdscan_backward_workspace_size(dims) -> int:
+    return load().bdscan_backward_workspace_size(_ref(dims))
+
+
+def bdscan_boundary_states_workspace_size(dims, emit_all) -> int:
+    return load().bdscan_boundary_states_workspace_size(_ref(dims), int(emit_all))
+
+
+def bdscan_forward(dims, clean, noisy, params, y_c, y_n, states, workspace, workspace_bytes, stream):
+    return load().bdscan_forward(_ref(dims), _ref(clean), _ref(noisy),
+                                 _ref(params), y_c, y_n, states, workspace, workspace_bytes, stream)
+
+
+def bdscan_backward(dims, clean, noisy, params, states, dy_c, dy_n, dstates, gclean, gnoisy, gparams,
+                    workspace, workspace_bytes, stream):
+    return load().bdscan_backward(_ref(dims), _ref(clean), _ref(noisy),
+                                  _ref(params), states, dy_c, dy_n, dstates, _ref(gclean),
+                                  _ref(gnoisy), _ref(gparams), workspace, workspace_bytes, stream)
+
+
+def bdscan_boundary_states(dims, clean, A_f, D_f, init_state, y_c, states, emit_all, workspace,
+                           workspace_bytes, stream):
+    return load().bdscan_boundary_states(_ref(dims), _ref(clean), A_f, D_f, init_state, y_c,
+                                         states, int(emit_all), workspace, workspace_bytes, stream)
+
+
+def bdscan_active_block(dims, seed, noisy, params, y_n, stream):
+    return load().bdscan_active_block(_ref(dims), seed, _ref(noisy), _ref(params),
+                                      y_n, stream)
+
+
+# ---------------------------------------------------------------------------
+# torch-tensor helpers (marshalling only)
+# ---------------------------------------------------------------------------
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("bdscan tensors must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def _dtype_code(t):
+    import torch
+    if t.dtype == torch.float32:
+        return BDSCAN_F32
+    if t.dtype == torch.bfloat16:
+        return BDSCAN_BF16
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def make_dims(batch, length, block, d_inner, d_state, dtype, out_dtype=None):
+    return bdscan_dims(int(batch), int(length), int(block), int(d_inner), int(d_state), int(dtype),
+                       int(dtype if out_dtype is None else out_dtype))
+
+
+def make_clean(t):
+    return bdscan_clean(_ptr(t["x_c"]), _ptr(t["dt_c"]), _ptr(t["B_c"]), _ptr(t["C_c"]))
+
+
+def make_noisy(t):
+    return bdscan_noisy(_ptr(t["x_n"]), _ptr(t["dt_f"]), _ptr(t["B_f"]), _ptr(t["C_f"]), _ptr(t["dt_r"]),
+                        _ptr(t["B_r"]), _ptr(t["C_r"]))
+
+
+def make_params(t):
+    return bdscan_params(_ptr(t["A_f"]), _ptr(t["D_f"]), _ptr(t["A_r"]), _ptr(t["D_r"]))
+
+
+def forward(dims, t, y_c, y_n, states, workspace, stream=None):
+    """t: dict of device tensors keyed like paper_2607_02805_gb300.inputs."""
+    _call("bdscan_forward", ctypes.byref(dims), ctypes.byref(make_clean(t)), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), _ptr(y_c), _ptr(y_n), _ptr(states), _ptr(workspace),
+          workspace.numel() * workspace.element_size(), _stream(stream))
+
+
+def backward(dims, t, states, dy_c, dy_n, dstates, g, workspace, stream=None):
+    """g: dict of gradient tensors keyed by input name (x_c, ..., D_r)."""
+    gc = bdscan_clean_grads(_ptr(g["x_c"]), _ptr(g["dt_c"]), _ptr(g["B_c"]), _ptr(g["C_c"]))
+    gn = bdscan_noisy_grads(_ptr(g["x_n"]), _ptr(g["dt_f"]), _ptr(g["B_f"]), _ptr(g["C_f"]), _ptr(g["dt_r"]),
+                            _ptr(g["B_r"]), _ptr(g["C_r"]))
+    gp = bdscan_param_grads(_ptr(g["A_f"]), _ptr(g["D_f"]), _ptr(g["A_r"]), _ptr(g["D_r"]))
+    _call("bdscan_backward", ctypes.byref(dims), ctypes.byref(make_clean(t)), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), _ptr(states), _ptr(dy_c), _ptr(dy_n), _ptr(dstates), ctypes.byref(gc),
+          ctypes.byref(gn), ctypes.byref(gp), _ptr(workspace), workspace.numel() * workspace.element_size(),
+          _stream(stream))
+
+
+def boundary_states(dims, t, init_state, y_c, states, emit_all, workspace, stream=None):
+    _call("bdscan_boundary_states", ctypes.byref(dims), ctypes.byref(make_clean(t)), _ptr(t["A_f"]),
+          _ptr(t["D_f"]), _ptr(init_state), _ptr(y_c), _ptr(states), int(emit_all), _ptr(workspace),
+          0 if workspace is None else workspace.numel() * workspace.element_size(), _stream(stream))
+
+
+def active_block(dims, seed, t, y_n, stream=None):
+    _call("bdscan_active_block", ctypes.byref(dims), _ptr(seed), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), _ptr(y_n), _stream(stream))

@@ -1,0 +1,468 @@
+// api.cu -- the C ABI of libbdscan: argument validation, workspace layout
+// and the launch sequence of each entry point. No exception crosses the ABI;
+// every error is a return code plus a thread-local message.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "bdscan.h"
+#include "params.h"
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+// timing hook state (per host thread)
+thread_local void* const* g_prof_ev = nullptr;
+thread_local int g_prof_n = 0;
+thread_local int g_launches = 0;
+thread_local int g_last_launches = 0;
+
+int ok() {
+  g_err[0] = '\0';
+  g_last_launches = g_launches;
+  return BDSCAN_OK;
+}
+
+// Called after every kernel launch of an entry point.
+cudaError_t launched(cudaError_t e, cudaStream_t s) {
+  if (e != cudaSuccess) return e;
+  if (g_prof_ev != nullptr && g_launches < g_prof_n) e = cudaEventRecord((cudaEvent_t)g_prof_ev[g_launches], s);
+  ++g_launches;
+  return e;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  return fail(BDSCAN_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int64_t blocks_per_chunk(int64_t Bs) { return Bs >= 128 ? 1 : 128 / Bs; }
+
+struct Call {
+  bds::Geo g;
+  int dt;  // 0 f32/f32, 1 bf16/bf16, 2 bf16/f32
+  int N;
+  size_t in_elt;
+};
+
+// Validates the dimensions common to every entry point.
+int check_dims(const bdscan_dims* dm, Call* c, const char* fn) {
+  g_launches = 0;
+  if (dm == nullptr) return fail(BDSCAN_ERR_ARG, "%s: dims is NULL", fn);
+  if (dm->batch < 0 || dm->len < 0) return fail(BDSCAN_ERR_ARG, "%s: negative batch or len", fn);
+  if (dm->block <= 0) return fail(BDSCAN_ERR_ARG, "%s: block must be positive", fn);
+  if (dm->d_inner <= 0 || dm->d_state <= 0) return fail(BDSCAN_ERR_ARG, "%s: d_inner and d_state must be positive", fn);
+  if (dm->len % dm->block != 0)
+    return fail(BDSCAN_ERR_ARG, "%s: len (%lld) is not a multiple of block (%lld)", fn, (long long)dm->len,
+                (long long)dm->block);
+  if (dm->dtype != BDSCAN_F32 && dm->dtype != BDSCAN_BF16) return fail(BDSCAN_ERR_ARG, "%s: bad dtype %d", fn, dm->dtype);
+  if (dm->out_dtype != BDSCAN_F32 && dm->out_dtype != BDSCAN_BF16)
+    return fail(BDSCAN_ERR_ARG, "%s: bad out_dtype %d", fn, dm->out_dtype);
+  if (dm->dtype == BDSCAN_F32 && dm->out_dtype == BDSCAN_BF16)
+    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: f32 inputs with bf16 outputs are not supported", fn);
+  if (dm->d_state != 8 && dm->d_state != 16)
+    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: d_state %lld not supported (8 or 16)", fn, (long long)dm->d_state);
+  const int64_t vec = dm->dtype == BDSCAN_BF16 ? 8 : 4;
+  if (dm->d_inner % vec != 0)
+    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: d_inner %lld must be a multiple of %lld for this dtype", fn,
+                (long long)dm->d_inner, (long long)vec);
+  if (dm->batch > 65535) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: batch above 65535", fn);
+  const int64_t nb = dm->len / dm->block;
+  if (nb > (int64_t)1 << 30) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: too many blocks", fn);
+  const int64_t m = blocks_per_chunk(dm->block);
+  const int64_t nc = (nb + m - 1) / m;
+  if (nc > 65535) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: len too long for one call (more than 65535 chunks)", fn);
+  c->g.Bt = dm->batch;
+  c->g.L = dm->len;
+  c->g.Bs = dm->block;
+  c->g.D = dm->d_inner;
+  c->g.nb = (int)nb;
+  c->g.m = (int)m;
+  c->g.nc = (int)nc;
+  c->g.nc_full = (int)(nb / m);
+  c->g.G = (int)((dm->d_inner + bds::kCtaHost - 1) / bds::kCtaHost);
+  c->dt = dm->dtype == BDSCAN_F32 ? 0 : (dm->out_dtype == BDSCAN_BF16 ? 1 : 2);
+  c->N = (int)dm->d_state;
+  c->in_elt = dm->dtype == BDSCAN_F32 ? 4 : 2;
+  return BDSCAN_OK;
+}
+
+#define REQ(ptr, fn, name)                                                              \
+  do {                                                                                  \
+    if ((ptr) == nullptr) return fail(BDSCAN_ERR_ARG, "%s: %s is NULL", fn, name);      \
+    if (!aligned16(ptr)) return fail(BDSCAN_ERR_ARG, "%s: %s is not 16-byte aligned", fn, name); \
+  } while (0)
+#define OPT(ptr, fn, name)                                                              \
+  do {                                                                                  \
+    if ((ptr) != nullptr && !aligned16(ptr))                                            \
+      return fail(BDSCAN_ERR_ARG, "%s: %s is not 16-byte aligned", fn, name);           \
+  } while (0)
+
+size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+size_t fwd_ws(const bds::Geo& g, int N) {
+  return al256((size_t)g.Bt * (g.nc + 1) * g.D * N * 4) + al256((size_t)g.Bt * g.nc * g.D * 4);
+}
+
+struct BwdWs {
+  size_t dS, Lc, sdtc, part_tok, part_A, part_D, total;
+};
+BwdWs bwd_ws(const bds::Geo& g, int N) {
+  BwdWs w;
+  size_t o = 0;
+  w.dS = o;
+  o += al256((size_t)g.Bt * g.nb * g.D * N * 4);
+  w.Lc = o;
+  o += al256((size_t)g.Bt * g.nc * g.D * N * 4);
+  w.sdtc = o;
+  o += al256((size_t)g.Bt * g.nc * g.D * 4);
+  w.part_tok = o;
+  o += al256((size_t)6 * g.Bt * g.L * g.G * N * 4);
+  w.part_A = o;
+  o += al256((size_t)3 * g.Bt * g.nc * g.D * N * 4);
+  w.part_D = o;
+  o += al256((size_t)2 * g.Bt * g.nc * g.D * 4);
+  w.total = o;
+  return w;
+}
+
+int check_block_limits(const Call& c, bool backward, const char* fn) {
+  if (c.g.Bs > 64) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: block %lld above 64", fn, (long long)c.g.Bs);
+  if (backward && c.g.Bs > 16 && c.g.Bs % 16 != 0)
+    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward needs block <= 16 or a multiple of 16", fn);
+  return BDSCAN_OK;
+}
+
+void fill_clean(bds::FwdParams& p, const bdscan_clean* cl) {
+  p.xc = cl->x;
+  p.dtc = cl->dt;
+  p.Bc = cl->B;
+  p.Cc = cl->C;
+}
+void fill_noisy(bds::FwdParams& p, const bdscan_noisy* nz) {
+  p.xn = nz->x;
+  p.dtf = nz->dt_f;
+  p.Bf = nz->B_f;
+  p.Cf = nz->C_f;
+  p.dtr = nz->dt_r;
+  p.Br = nz->B_r;
+  p.Cr = nz->C_r;
+}
+
+int check_clean(const bdscan_clean* cl, const char* fn) {
+  if (cl == nullptr) return fail(BDSCAN_ERR_ARG, "%s: clean is NULL", fn);
+  REQ(cl->x, fn, "clean.x");
+  REQ(cl->dt, fn, "clean.dt");
+  REQ(cl->B, fn, "clean.B");
+  REQ(cl->C, fn, "clean.C");
+  return BDSCAN_OK;
+}
+int check_noisy(const bdscan_noisy* nz, const char* fn) {
+  if (nz == nullptr) return fail(BDSCAN_ERR_ARG, "%s: noisy is NULL", fn);
+  REQ(nz->x, fn, "noisy.x");
+  REQ(nz->dt_f, fn, "noisy.dt_f");
+  REQ(nz->B_f, fn, "noisy.B_f");
+  REQ(nz->C_f, fn, "noisy.C_f");
+  REQ(nz->dt_r, fn, "noisy.dt_r");
+  REQ(nz->B_r, fn, "noisy.B_r");
+  REQ(nz->C_r, fn, "noisy.C_r");
+  return BDSCAN_OK;
+}
+int check_params(const bdscan_params* pr, const char* fn) {
+  if (pr == nullptr) return fail(BDSCAN_ERR_ARG, "%s: params is NULL", fn);
+  REQ(pr->A_f, fn, "params.A_f");
+  REQ(pr->D_f, fn, "params.D_f");
+  REQ(pr->A_r, fn, "params.A_r");
+  REQ(pr->D_r, fn, "params.D_r");
+  return BDSCAN_OK;
+}
+
+// Runs the chunk-local scan and the chunk carry: hst then holds every chunk
+// start state (slot nc_full: the state after the last full chunk).
+int run_chunk_states(const Call& c, bds::FwdParams& p, cudaStream_t s, const char* fn) {
+  cudaError_t e = cudaSuccess;
+  if (c.g.nc_full > 0) e = launched(bds::launch_chunk_local(c.dt, c.N, p, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  e = launched(bds::launch_chunk_carry(c.N, p, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return BDSCAN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* bdscan_last_error(void) { return g_err; }
+
+int bdscan_version(void) { return 100; }
+
+int bdscan_profile_events(void* const* events, int n) {
+  g_prof_ev = (n > 0) ? events : nullptr;
+  g_prof_n = (events != nullptr && n > 0) ? n : 0;
+  return BDSCAN_OK;
+}
+
+int bdscan_last_launch_count(void) { return g_last_launches; }
+
+int64_t bdscan_chunk_tokens(int64_t block) { return block <= 0 ? 0 : blocks_per_chunk(block) * block; }
+
+size_t bdscan_forward_workspace_size(const bdscan_dims* dims) {
+  Call c;
+  if (check_dims(dims, &c, "bdscan_forward_workspace_size") != BDSCAN_OK) return 0;
+  return fwd_ws(c.g, c.N);
+}
+
+size_t bdscan_boundary_states_workspace_size(const bdscan_dims* dims, int emit_all) {
+  (void)emit_all;
+  Call c;
+  if (check_dims(dims, &c, "bdscan_boundary_states_workspace_size") != BDSCAN_OK) return 0;
+  return fwd_ws(c.g, c.N);
+}
+
+size_t bdscan_backward_workspace_size(const bdscan_dims* dims) {
+  Call c;
+  if (check_dims(dims, &c, "bdscan_backward_workspace_size") != BDSCAN_OK) return 0;
+  return bwd_ws(c.g, c.N).total;
+}
+
+int bdscan_forward(const bdscan_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
+                   const bdscan_params* params, void* y_c, void* y_n, float* states, void* workspace,
+                   size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_forward";
+  Call c;
+  int rc = check_dims(dims, &c, fn);
+  if (rc) return rc;
+  if ((rc = check_block_limits(c, false, fn))) return rc;
+  if (c.g.Bt == 0 || c.g.L == 0) return ok();
+  if ((rc = check_clean(clean, fn)) || (rc = check_noisy(noisy, fn)) || (rc = check_params(params, fn))) return rc;
+  REQ(y_c, fn, "y_c");
+  REQ(y_n, fn, "y_n");
+  REQ(states, fn, "states");
+  const size_t need = fwd_ws(c.g, c.N);
+  REQ(workspace, fn, "workspace");
+  if (workspace_bytes < need)
+    return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
+  cudaStream_t s = (cudaStream_t)stream;
+  bds::FwdParams p;
+  memset(&p, 0, sizeof(p));
+  p.g = c.g;
+  fill_clean(p, clean);
+  fill_noisy(p, noisy);
+  p.Af = params->A_f;
+  p.Df = params->D_f;
+  p.Ar = params->A_r;
+  p.Dr = params->D_r;
+  p.yc = y_c;
+  p.yn = y_n;
+  p.states = states;
+  p.emit_all = 1;
+  p.hst = (float*)workspace;
+  p.sdt = (float*)((char*)workspace + al256((size_t)c.g.Bt * (c.g.nc + 1) * c.g.D * c.N * 4));
+  if ((rc = run_chunk_states(c, p, s, fn))) return rc;
+  cudaError_t e = launched(bds::launch_block_scan(c.dt, c.N, 0, c.g.nc, p, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
+int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, const float* A_f,
+                           const float* D_f, const float* init_state, void* y_c, float* states, int emit_all,
+                           void* workspace, size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_boundary_states";
+  Call c;
+  int rc = check_dims(dims, &c, fn);
+  if (rc) return rc;
+  if ((rc = check_block_limits(c, false, fn))) return rc;
+  if (c.g.Bt == 0) return ok();
+  cudaStream_t s = (cudaStream_t)stream;
+  OPT(init_state, fn, "init_state");
+  if (c.g.L == 0) {
+    if (emit_all) return ok();
+    REQ(states, fn, "states");
+    const size_t bytes = (size_t)c.g.Bt * c.g.D * c.N * 4;
+    cudaError_t e = init_state ? cudaMemcpyAsync(states, init_state, bytes, cudaMemcpyDeviceToDevice, s)
+                               : cudaMemsetAsync(states, 0, bytes, s);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+  }
+  if ((rc = check_clean(clean, fn))) return rc;
+  REQ(A_f, fn, "A_f");
+  REQ(D_f, fn, "D_f");
+  REQ(states, fn, "states");
+  OPT(y_c, fn, "y_c");
+  const size_t need = fwd_ws(c.g, c.N);
+  REQ(workspace, fn, "workspace");
+  if (workspace_bytes < need)
+    return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
+  bds::FwdParams p;
+  memset(&p, 0, sizeof(p));
+  p.g = c.g;
+  fill_clean(p, clean);
+  p.Af = A_f;
+  p.Df = D_f;
+  p.yc = y_c;
+  p.init = init_state;
+  p.hst = (float*)workspace;
+  p.sdt = (float*)((char*)workspace + al256((size_t)c.g.Bt * (c.g.nc + 1) * c.g.D * c.N * 4));
+  if ((rc = run_chunk_states(c, p, s, fn))) return rc;
+  cudaError_t e = cudaSuccess;
+  if (emit_all || y_c != nullptr) {
+    p.emit_all = emit_all ? 1 : 0;
+    p.states = emit_all ? states : nullptr;
+    p.final_state = emit_all ? nullptr : states;
+    e = launched(bds::launch_block_scan(c.dt, c.N, 1, c.g.nc, p, s), s);
+  } else if (c.g.nc_full == c.g.nc) {
+    // the state after the last chunk is the carry kernel's final value
+    const size_t row = (size_t)c.g.D * c.N * 4;
+    e = cudaMemcpy2DAsync(states, row, p.hst + (size_t)c.g.nc * c.g.D * c.N, (size_t)(c.g.nc + 1) * row, row,
+                          (size_t)c.g.Bt, cudaMemcpyDeviceToDevice, s);
+  } else {
+    // a partial last chunk: rescan it from its start state
+    p.emit_all = 0;
+    p.final_state = states;
+    p.c_begin = c.g.nc - 1;
+    e = launched(bds::launch_block_scan(c.dt, c.N, 1, 1, p, s), s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
+int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan_noisy* noisy,
+                        const bdscan_params* params, void* y_n, void* stream) {
+  const char* fn = "bdscan_active_block";
+  Call c;
+  int rc = check_dims(dims, &c, fn);
+  if (rc) return rc;
+  if (dims->len != dims->block && dims->len != 0)
+    return fail(BDSCAN_ERR_ARG, "%s: len (%lld) must equal block (%lld)", fn, (long long)dims->len,
+                (long long)dims->block);
+  if ((rc = check_block_limits(c, false, fn))) return rc;
+  if (c.g.Bt == 0 || c.g.L == 0) return ok();
+  REQ(seed, fn, "seed");
+  if ((rc = check_noisy(noisy, fn)) || (rc = check_params(params, fn))) return rc;
+  REQ(y_n, fn, "y_n");
+  bds::FwdParams p;
+  memset(&p, 0, sizeof(p));
+  p.g = c.g;
+  fill_noisy(p, noisy);
+  p.Af = params->A_f;
+  p.Df = params->D_f;
+  p.Ar = params->A_r;
+  p.Dr = params->D_r;
+  p.yn = y_n;
+  p.seed = seed;
+  cudaError_t e = launched(bds::launch_block_scan(c.dt, c.N, 2, 1, p, (cudaStream_t)stream), (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
+int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
+                    const bdscan_params* params, const float* states, const void* dy_c, const void* dy_n,
+                    const float* dstates, const bdscan_clean_grads* gclean, const bdscan_noisy_grads* gnoisy,
+                    const bdscan_param_grads* gparams, void* workspace, size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_backward";
+  Call c;
+  int rc = check_dims(dims, &c, fn);
+  if (rc) return rc;
+  if ((rc = check_block_limits(c, true, fn))) return rc;
+  if (gparams == nullptr) return fail(BDSCAN_ERR_ARG, "%s: gparams is NULL", fn);
+  REQ(gparams->dA_f, fn, "dA_f");
+  REQ(gparams->dD_f, fn, "dD_f");
+  REQ(gparams->dA_r, fn, "dA_r");
+  REQ(gparams->dD_r, fn, "dD_r");
+  cudaStream_t s = (cudaStream_t)stream;
+  if (c.g.Bt == 0 || c.g.L == 0) {
+    const size_t an = (size_t)c.g.D * c.N * 4, dn = (size_t)c.g.D * 4;
+    cudaError_t e = cudaMemsetAsync(gparams->dA_f, 0, an, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(gparams->dA_r, 0, an, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(gparams->dD_f, 0, dn, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(gparams->dD_r, 0, dn, s);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+  }
+  if ((rc = check_clean(clean, fn)) || (rc = check_noisy(noisy, fn)) || (rc = check_params(params, fn))) return rc;
+  REQ(states, fn, "states");
+  OPT(dy_c, fn, "dy_c");
+  REQ(dy_n, fn, "dy_n");
+  OPT(dstates, fn, "dstates");
+  if (gclean == nullptr || gnoisy == nullptr) return fail(BDSCAN_ERR_ARG, "%s: gradient struct is NULL", fn);
+  REQ(gclean->dx, fn, "gclean.dx");
+  REQ(gclean->ddt, fn, "gclean.ddt");
+  REQ(gclean->dB, fn, "gclean.dB");
+  REQ(gclean->dC, fn, "gclean.dC");
+  REQ(gnoisy->dx, fn, "gnoisy.dx");
+  REQ(gnoisy->ddt_f, fn, "gnoisy.ddt_f");
+  REQ(gnoisy->dB_f, fn, "gnoisy.dB_f");
+  REQ(gnoisy->dC_f, fn, "gnoisy.dC_f");
+  REQ(gnoisy->ddt_r, fn, "gnoisy.ddt_r");
+  REQ(gnoisy->dB_r, fn, "gnoisy.dB_r");
+  REQ(gnoisy->dC_r, fn, "gnoisy.dC_r");
+  const BwdWs w = bwd_ws(c.g, c.N);
+  REQ(workspace, fn, "workspace");
+  if (workspace_bytes < w.total)
+    return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, w.total);
+
+  bds::BwdParams p;
+  memset(&p, 0, sizeof(p));
+  p.g = c.g;
+  p.xc = clean->x;
+  p.dtc = clean->dt;
+  p.Bc = clean->B;
+  p.Cc = clean->C;
+  p.xn = noisy->x;
+  p.dtf = noisy->dt_f;
+  p.Bf = noisy->B_f;
+  p.Cf = noisy->C_f;
+  p.dtr = noisy->dt_r;
+  p.Br = noisy->B_r;
+  p.Cr = noisy->C_r;
+  p.Af = params->A_f;
+  p.Df = params->D_f;
+  p.Ar = params->A_r;
+  p.Dr = params->D_r;
+  p.states = states;
+  p.dyc = dy_c;
+  p.dyn = dy_n;
+  p.dstates = dstates;
+  p.dxc = gclean->dx;
+  p.ddtc = gclean->ddt;
+  p.dBc = gclean->dB;
+  p.dCc = gclean->dC;
+  p.dxn = gnoisy->dx;
+  p.ddtf = gnoisy->ddt_f;
+  p.dBf = gnoisy->dB_f;
+  p.dCf = gnoisy->dC_f;
+  p.ddtr = gnoisy->ddt_r;
+  p.dBr = gnoisy->dB_r;
+  p.dCr = gnoisy->dC_r;
+  p.dAf = gparams->dA_f;
+  p.dDf = gparams->dD_f;
+  p.dAr = gparams->dA_r;
+  p.dDr = gparams->dD_r;
+  char* ws = (char*)workspace;
+  p.dS = (float*)(ws + w.dS);
+  p.Lc = (float*)(ws + w.Lc);
+  p.sdtc = (float*)(ws + w.sdtc);
+  p.part_tok = (float*)(ws + w.part_tok);
+  p.part_A = (float*)(ws + w.part_A);
+  p.part_D = (float*)(ws + w.part_D);
+
+  cudaError_t e = launched(bds::launch_bwd_noisy(c.dt, c.N, p, s), s);
+  if (e == cudaSuccess) e = launched(bds::launch_bwd_carry(c.N, p, s), s);
+  if (e == cudaSuccess) e = launched(bds::launch_bwd_clean(c.dt, c.N, p, s), s);
+  if (e == cudaSuccess) e = launched(bds::launch_bwd_reduce_tok(c.dt, c.N, p, s), s);
+  if (e == cudaSuccess) e = launched(bds::launch_bwd_reduce_par(c.N, p, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
+}  // extern "C"

@@ -1,0 +1,330 @@
+// fwd.cu -- forward-side kernels of libbdscan (sm_103a).
+//
+// The clean prefix scan (eq. boundary-state) is split into time chunks of
+// m blocks (m = max(1, 128 / Bs)) so that Bt * D channels are not the only
+// source of parallelism:
+//   k_chunk_local  each (batch, chunk, 128 channels): scan the chunk from a
+//                  zero state; keep the end state and the sum of dt.
+//   k_chunk_carry  each (batch, channel, state): walk the chunks in order,
+//                  H_{c+1} = exp(A * sum_c dt) * H_c + local_c, giving the
+//                  exact state at every chunk start.
+//   k_block_scan   each (batch, chunk, 128 channels): rescan the chunk from
+//                  its start state, emitting y_c and the state at every
+//                  block end; for every noisy block of the chunk, continue
+//                  the state at its start through the noisy tokens (forward
+//                  direction, eq. partial-reverse first line) and run the
+//                  block-local reverse scan from zero (second line), and
+//                  write their sum (third line).
+// The state at the end of a chunk's last block is taken from the carry
+// kernel (the same value the next chunk starts from), so every consumer of
+// a boundary state sees one value, and boundary states of a prefix equal
+// those of any longer stream: chunking depends on Bs only.
+#include "device.cuh"
+#include "params.h"
+
+namespace bds {
+
+static_assert(kCta == kCtaHost, "host and device CTA widths differ");
+
+constexpr int kLocalSpan = 32;  // tokens staged per step of the chunk-local scan
+
+template <typename T, int N>
+__global__ void __launch_bounds__(kCta) k_chunk_local(const FwdParams p) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const Geo& g = p.g;
+  const int64_t b = blockIdx.z;
+  const int c = blockIdx.y;
+  const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
+  const bool act = d < g.D;
+  Stage<T, N, 2, 1> st;
+  st.carve(smem, kLocalSpan);
+  st.td_src[0] = (const T*)p.xc;
+  st.td_src[1] = (const T*)p.dtc;
+  st.row_src[0] = (const T*)p.Bc;
+
+  float A2[N];
+  if (act) {
+    vload(A2, p.Af + d * N);
+#pragma unroll
+    for (int n = 0; n < N; ++n) A2[n] = __fmul_rn(A2[n], kLog2e);
+  } else {
+    vzero(A2);
+  }
+  float h[N];
+  vzero(h);
+  float sdt = 0.f;
+  const int64_t tc = (int64_t)g.m * g.Bs;
+  const int64_t tbeg = (int64_t)c * tc;
+  for (int64_t t = 0; t < tc; t += kLocalSpan) {
+    const int ns = (int)((tc - t) < kLocalSpan ? (tc - t) : kLocalSpan);
+    st.load(b * g.L + tbeg + t, ns, g.D, d0);
+    for (int i = 0; i < ns; ++i) {
+      const float dt = st.at(1, i);
+      scan_state(h, A2, dt, st.at(0, i), st.row(0, i));
+      sdt = __fadd_rn(sdt, dt);
+    }
+  }
+  if (act) {
+    vstore(p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, h);
+    p.sdt[(b * g.nc + c) * g.D + d] = sdt;
+  }
+}
+
+template <int N>
+__global__ void __launch_bounds__(256) k_chunk_carry(const FwdParams p) {
+  const Geo& g = p.g;
+  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (idx >= g.Bt * g.D * N) return;
+  const int n = (int)(idx % N);
+  const int64_t d = (idx / N) % g.D, b = idx / ((int64_t)N * g.D);
+  const float A2 = __fmul_rn(p.Af[d * N + n], kLog2e);
+  float H = p.init ? p.init[(b * g.D + d) * N + n] : 0.f;
+  const int64_t hstride = g.D * N;
+  float* hs = p.hst + b * (g.nc + 1) * hstride + d * N + n;
+  const float* sd = p.sdt + b * g.nc * g.D + d;
+  constexpr int U = 8;
+  int c = 0;
+  for (; c + U <= g.nc_full; c += U) {
+    float hl[U], s[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      hl[j] = hs[(int64_t)(c + j) * hstride];
+      s[j] = sd[(int64_t)(c + j) * g.D];
+    }
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      hs[(int64_t)(c + j) * hstride] = H;
+      H = __fmaf_rn(ex2(__fmul_rn(A2, s[j])), H, hl[j]);
+    }
+  }
+  for (; c < g.nc_full; ++c) {
+    const float hl = hs[(int64_t)c * hstride], s = sd[(int64_t)c * g.D];
+    hs[(int64_t)c * hstride] = H;
+    H = __fmaf_rn(ex2(__fmul_rn(A2, s)), H, hl);
+  }
+  hs[(int64_t)g.nc_full * hstride] = H;
+}
+
+// MODE 0: all-block forward (clean + noisy). MODE 1: clean scan only (cache
+// build). MODE 2: one noisy block from a cached seed (active block).
+template <int MODE>
+struct ScanLayout {
+  static constexpr bool kClean = MODE != 2;
+  static constexpr bool kNoisy = MODE != 1;
+  static constexpr int NTD = MODE == 0 ? 5 : (MODE == 1 ? 2 : 3);
+  static constexpr int NROW = MODE == 0 ? 6 : (MODE == 1 ? 2 : 4);
+  // token-by-channel slots
+  static constexpr int XC = 0, DTC = 1;
+  static constexpr int XN = MODE == 0 ? 2 : 0, DTF = XN + 1, DTR = XN + 2;
+  // token-by-state slots
+  static constexpr int BC = 0, CC = 1;
+  static constexpr int BF = MODE == 0 ? 2 : 0, CF = BF + 1, BR = BF + 2, CR = BF + 3;
+};
+
+template <typename T, typename TO, int N, int MODE>
+__global__ void __launch_bounds__(kCta) k_block_scan(const FwdParams p) {
+  using Ly = ScanLayout<MODE>;
+  extern __shared__ __align__(16) unsigned char smem[];
+  const Geo& g = p.g;
+  const int64_t b = blockIdx.z;
+  const int c = p.c_begin + blockIdx.y;
+  const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
+  const bool act = d < g.D;
+  const int Bs = (int)g.Bs;
+  Stage<T, N, Ly::NTD, Ly::NROW> st;
+  st.carve(smem, Bs);
+  float* yfbuf = reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW>::bytes(Bs));
+  if (Ly::kClean) {
+    st.td_src[Ly::XC] = (const T*)p.xc;
+    st.td_src[Ly::DTC] = (const T*)p.dtc;
+    st.row_src[Ly::BC] = (const T*)p.Bc;
+    st.row_src[Ly::CC] = (const T*)p.Cc;
+  }
+  if (Ly::kNoisy) {
+    st.td_src[Ly::XN] = (const T*)p.xn;
+    st.td_src[Ly::DTF] = (const T*)p.dtf;
+    st.td_src[Ly::DTR] = (const T*)p.dtr;
+    st.row_src[Ly::BF] = (const T*)p.Bf;
+    st.row_src[Ly::CF] = (const T*)p.Cf;
+    st.row_src[Ly::BR] = (const T*)p.Br;
+    st.row_src[Ly::CR] = (const T*)p.Cr;
+  }
+
+  float A2f[N], A2r[N];
+  float Df = 0.f, Dr = 0.f;
+  vzero(A2f);
+  vzero(A2r);
+  if (act) {
+    vload(A2f, p.Af + d * N);
+    Df = p.Df[d];
+    if (Ly::kNoisy) {
+      vload(A2r, p.Ar + d * N);
+      Dr = p.Dr[d];
+    }
+#pragma unroll
+    for (int n = 0; n < N; ++n) {
+      A2f[n] = __fmul_rn(A2f[n], kLog2e);
+      A2r[n] = __fmul_rn(A2r[n], kLog2e);
+    }
+  }
+
+  int k_lo = 0, k_hi = 0;
+  bool full = false;
+  if (MODE != 2) {
+    k_lo = c * g.m;
+    k_hi = min(k_lo + g.m, g.nb) - 1;
+    full = c < g.nc_full;
+  }
+  float hc[N];
+  vzero(hc);
+  if (act) {
+    if (MODE == 2)
+      vload(hc, p.seed + (b * g.D + d) * N);
+    else
+      vload(hc, p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N);
+  }
+
+  for (int k = k_lo; k <= k_hi; ++k) {
+    const int64_t row0 = b * g.L + (int64_t)k * Bs;
+    st.load(row0, Bs, g.D, d0);
+    float hs[N];
+#pragma unroll
+    for (int n = 0; n < N; ++n) hs[n] = hc[n];  // the block's seed: state before its first token
+    for (int i = 0; i < Bs; ++i) {
+      const int64_t o = (row0 + i) * g.D + d;
+      if (Ly::kClean) {
+        const float x = st.at(Ly::XC, i), dt = st.at(Ly::DTC, i);
+        const float y = scan_step(hc, A2f, dt, x, st.row(Ly::BC, i), st.row(Ly::CC, i));
+        if (p.yc != nullptr && act) reinterpret_cast<TO*>(p.yc)[o] = to_out<TO>(with_skip(y, Df, x));
+      }
+      if (Ly::kNoisy) {
+        const float x = st.at(Ly::XN, i), dt = st.at(Ly::DTF, i);
+        const float y = scan_step(hs, A2f, dt, x, st.row(Ly::BF, i), st.row(Ly::CF, i));
+        yfbuf[i * kCta + threadIdx.x] = with_skip(y, Df, x);
+      }
+    }
+    if (Ly::kClean && p.emit_all && act) {
+      float* dst = p.states + ((b * g.nb + k) * g.D + d) * N;
+      if (k == k_hi && full) {
+        float e[N];
+        vload(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N);
+        vstore(dst, e);
+      } else {
+        vstore(dst, hc);
+      }
+    }
+    if (Ly::kNoisy) {
+      float hr[N];
+      vzero(hr);
+      for (int i = Bs - 1; i >= 0; --i) {
+        const int64_t o = (row0 + i) * g.D + d;
+        const float x = st.at(Ly::XN, i), dt = st.at(Ly::DTR, i);
+        const float y = scan_step(hr, A2r, dt, x, st.row(Ly::BR, i), st.row(Ly::CR, i));
+        if (act)
+          reinterpret_cast<TO*>(p.yn)[o] =
+              to_out<TO>(combine_dirs(yfbuf[i * kCta + threadIdx.x], with_skip(y, Dr, x)));
+      }
+    }
+  }
+  if (Ly::kClean && p.final_state != nullptr && c == g.nc - 1 && act) {
+    float* dst = p.final_state + (b * g.D + d) * N;
+    if (full) {
+      float e[N];
+      vload(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N);
+      vstore(dst, e);
+    } else {
+      vstore(dst, hc);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// launchers
+// ---------------------------------------------------------------------------
+namespace {
+
+template <typename T, int N>
+cudaError_t chunk_local_t(const FwdParams& p, cudaStream_t s) {
+  const size_t smem = Stage<T, N, 2, 1>::bytes(kLocalSpan);
+  dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc_full, (unsigned)p.g.Bt);
+  k_chunk_local<T, N><<<grid, kCta, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <typename T, typename TO, int N, int MODE>
+size_t block_scan_smem_t(int64_t Bs) {
+  using Ly = ScanLayout<MODE>;
+  size_t b = Stage<T, N, Ly::NTD, Ly::NROW>::bytes((int)Bs);
+  if (Ly::kNoisy) b += (size_t)Bs * kCta * sizeof(float);
+  return b;
+}
+
+template <typename T, typename TO, int N, int MODE>
+cudaError_t block_scan_t(int nchunks, const FwdParams& p, cudaStream_t s) {
+  const size_t smem = block_scan_smem_t<T, TO, N, MODE>(p.g.Bs);
+  cudaError_t e = cudaFuncSetAttribute(k_block_scan<T, TO, N, MODE>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((unsigned)p.g.G, (unsigned)nchunks, (unsigned)p.g.Bt);
+  k_block_scan<T, TO, N, MODE><<<grid, kCta, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <typename T, typename TO, int N>
+cudaError_t block_scan_mode(int mode, int nchunks, const FwdParams& p, cudaStream_t s) {
+  switch (mode) {
+    case 0: return block_scan_t<T, TO, N, 0>(nchunks, p, s);
+    case 1: return block_scan_t<T, TO, N, 1>(nchunks, p, s);
+    default: return block_scan_t<T, TO, N, 2>(nchunks, p, s);
+  }
+}
+
+template <typename T, typename TO, int N>
+size_t block_scan_smem_mode(int mode, int64_t Bs) {
+  switch (mode) {
+    case 0: return block_scan_smem_t<T, TO, N, 0>(Bs);
+    case 1: return block_scan_smem_t<T, TO, N, 1>(Bs);
+    default: return block_scan_smem_t<T, TO, N, 2>(Bs);
+  }
+}
+
+}  // namespace
+
+#define BDS_DISPATCH_N(N, ...)                      \
+  switch (N) {                                      \
+    case 8: { constexpr int NN = 8; __VA_ARGS__ }   \
+    case 16: { constexpr int NN = 16; __VA_ARGS__ } \
+    default: return cudaErrorInvalidValue;          \
+  }
+
+cudaError_t launch_chunk_local(int dt, int N, const FwdParams& p, cudaStream_t s) {
+  if (p.g.nc_full == 0 || p.g.Bt == 0) return cudaSuccess;
+  if (dt == 0) {
+    BDS_DISPATCH_N(N, return chunk_local_t<float, NN>(p, s);)
+  }
+  BDS_DISPATCH_N(N, return chunk_local_t<bf16, NN>(p, s);)
+}
+
+cudaError_t launch_chunk_carry(int N, const FwdParams& p, cudaStream_t s) {
+  const int64_t total = p.g.Bt * p.g.D * N;
+  if (total == 0) return cudaSuccess;
+  const unsigned blocks = (unsigned)((total + 255) / 256);
+  BDS_DISPATCH_N(N, k_chunk_carry<NN><<<blocks, 256, 0, s>>>(p); return cudaGetLastError();)
+}
+
+cudaError_t launch_block_scan(int dt, int N, int mode, int nchunks, const FwdParams& p, cudaStream_t s) {
+  if (nchunks == 0 || p.g.Bt == 0) return cudaSuccess;
+  switch (dt) {
+    case 0: BDS_DISPATCH_N(N, return block_scan_mode<float, float, NN>(mode, nchunks, p, s);)
+    case 1: BDS_DISPATCH_N(N, return block_scan_mode<bf16, bf16, NN>(mode, nchunks, p, s);)
+    default: BDS_DISPATCH_N(N, return block_scan_mode<bf16, float, NN>(mode, nchunks, p, s);)
+  }
+}
+
+size_t block_scan_smem(int dt, int N, int mode, int64_t Bs) {
+  if (N != 8 && N != 16) return 0;
+  if (dt == 0) return N == 8 ? block_scan_smem_mode<float, float, 8>(mode, Bs) : block_scan_smem_mode<float, float, 16>(mode, Bs);
+  return N == 8 ? block_scan_smem_mode<bf16, bf16, 8>(mode, Bs) : block_scan_smem_mode<bf16, bf16, 16>(mode, Bs);
+}
+
+}  // namespace bds

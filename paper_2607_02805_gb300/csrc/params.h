@@ -1,0 +1,75 @@
+// params.h -- kernel argument blocks and internal launcher declarations.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace bds {
+
+constexpr int kCtaHost = 128;  // channels per CTA (one per thread); equals kCta in device.cuh
+
+// Geometry shared by all kernels of one call.
+struct Geo {
+  int64_t Bt, L, Bs, D;
+  int nb;       // blocks per stream, L / Bs
+  int m;        // blocks per time chunk
+  int nc;       // chunks, ceil(nb / m)
+  int nc_full;  // chunks holding m blocks
+  int G;        // channel groups of 128, ceil(D / 128)
+};
+
+// Forward-side kernels: chunk-local scan, chunk carry, block scan.
+struct FwdParams {
+  Geo g;
+  const void *xc, *dtc, *Bc, *Cc;
+  const void *xn, *dtf, *Bf, *Cf, *dtr, *Br, *Cr;
+  const float *Af, *Df, *Ar, *Dr;
+  void *yc, *yn;
+  float* states;       // [Bt][nb][D][N] when emit_all
+  int emit_all;
+  float* final_state;  // [Bt][D][N] or null: state after the last token
+  float* hst;          // workspace [Bt][nc+1][D][N]: chunk-local states, then chunk start states
+  float* sdt;          // workspace [Bt][nc][D]: sum of dt over each chunk
+  const float* init;   // [Bt][D][N] or null: state before token 0
+  const float* seed;   // active block: [Bt][D][N]
+  int c_begin;         // first chunk handled by a block-scan launch
+};
+
+// Backward-side kernels.
+struct BwdParams {
+  Geo g;
+  const void *xc, *dtc, *Bc, *Cc;
+  const void *xn, *dtf, *Bf, *Cf, *dtr, *Br, *Cr;
+  const float *Af, *Df, *Ar, *Dr;
+  const float* states;
+  const void *dyc, *dyn;
+  const float* dstates;
+  void *dxc, *ddtc, *dBc, *dCc;
+  void *dxn, *ddtf, *dBf, *dCf, *ddtr, *dBr, *dCr;
+  float *dAf, *dDf, *dAr, *dDr;
+  // workspace
+  float* dS;        // [Bt][nb][D][N]  gradient of each noisy block's seed
+  float* Lc;        // [Bt][nc][D][N]  local clean adjoint carry, then the carry into each chunk end
+  float* sdtc;      // [Bt][nc][D]
+  float* part_tok;  // [6][Bt][L][G][N] per channel-group sums of dB_c, dC_c, dB_f, dC_f, dB_r, dC_r
+  float* part_A;    // [3][Bt*nc][D][N] dA partial sums: noisy fwd, noisy rev, clean
+  float* part_D;    // [2][Bt*nc][D]    dD partial sums: noisy, clean
+};
+
+// Launchers (fwd.cu / bwd.cu). dt: 0 = f32 in/out, 1 = bf16 in/out, 2 = bf16 in, f32 out.
+cudaError_t launch_chunk_local(int dt, int N, const FwdParams& p, cudaStream_t s);
+cudaError_t launch_chunk_carry(int N, const FwdParams& p, cudaStream_t s);
+// mode 0: all-block forward, 1: clean scan only, 2: active block
+cudaError_t launch_block_scan(int dt, int N, int mode, int nchunks, const FwdParams& p, cudaStream_t s);
+cudaError_t launch_bwd_noisy(int dt, int N, const BwdParams& p, cudaStream_t s);
+cudaError_t launch_bwd_carry(int N, const BwdParams& p, cudaStream_t s);
+cudaError_t launch_bwd_clean(int dt, int N, const BwdParams& p, cudaStream_t s);
+cudaError_t launch_bwd_reduce_tok(int dt, int N, const BwdParams& p, cudaStream_t s);
+cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s);
+
+size_t block_scan_smem(int dt, int N, int mode, int64_t Bs);
+size_t bwd_noisy_smem(int dt, int N, int64_t Bs);
+size_t bwd_clean_smem(int dt, int N, int64_t Bs);
+
+}  // namespace bds

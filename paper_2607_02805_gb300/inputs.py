@@ -43,15 +43,21 @@ TOKEN_N = ("B_c", "C_c", "B_f", "C_f", "B_r", "C_r")   # [Bt, L, N]
 PARAMS = ("A_f", "D_f", "A_r", "D_r")                  # fp32 always
 
 
-def _rng(seed: int, name: str) -> np.random.Generator:
-    return np.random.Generator(np.random.PCG64(np.random.SeedSequence([int(seed), STREAM_IDS[name]])))
+def _rng(seed: int, name: str, part: int = 0) -> np.random.Generator:
+    key = [int(seed), STREAM_IDS[name]] + ([int(part)] if part else [])
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence(key)))
 
 
 def f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
-    """Round fp32 to bf16 (round to nearest, ties to even); returns uint16 bits."""
-    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    r = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
-    return r.astype(np.uint16)
+    """Round finite fp32 values to bf16 (round to nearest, ties to even);
+    returns uint16 bits. (uint32 arithmetic cannot overflow for finite input.)"""
+    u = np.ascontiguousarray(a, dtype=np.float32).reshape(-1).view(np.uint32)
+    out = np.empty(u.shape, dtype=np.uint16)
+    step = 1 << 24
+    for i in range(0, u.size, step):
+        v = u[i:i + step]
+        out[i:i + step] = ((v + np.uint32(0x7FFF) + ((v >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)).astype(np.uint16)
+    return out.reshape(np.shape(a))
 
 
 def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
@@ -64,9 +70,11 @@ def _softplus32(z: np.ndarray) -> np.ndarray:
     return (np.maximum(z, 0) + np.log1p(np.exp(-np.abs(z)))).astype(np.float32)
 
 
-def draw(name: str, shape, seed: int) -> np.ndarray:
-    """fp32 draw for one named tensor, following the module recipe."""
-    g = _rng(seed, name)
+def draw(name: str, shape, seed: int, part: int = 0) -> np.ndarray:
+    """fp32 draw for one named tensor, following the module recipe. `part`
+    selects an independent draw of the same tensor (e.g. successive noisy
+    blocks of a denoising loop)."""
+    g = _rng(seed, name, part)
     if name in ("x_c", "x_n", "dy_c", "dy_n", "dstates", "init_state"):
         return g.standard_normal(shape, dtype=np.float32)
     if name in ("dt_c", "dt_f", "dt_r"):
@@ -92,7 +100,7 @@ class Workload:
     """
 
     def __init__(self, batch, length, block, d_inner, d_state, dtype="bf16", seed=0,
-                 with_grads=True, with_dstates=False, with_init=False):
+                 with_grads=True, with_dstates=False, with_init=False, parts=("clean", "noisy"), part=0):
         if dtype not in ("bf16", "f32"):
             raise ValueError(dtype)
         self.batch, self.len, self.block = int(batch), int(length), int(block)
@@ -101,9 +109,11 @@ class Workload:
         nb = L // self.block if self.block > 0 else 0
         shapes = {}
         for k in TOKEN_D:
-            shapes[k] = (Bt, L, D)
+            if ("clean" in parts and k.endswith("_c")) or ("noisy" in parts and not k.endswith("_c")):
+                shapes[k] = (Bt, L, D)
         for k in TOKEN_N:
-            shapes[k] = (Bt, L, N)
+            if ("clean" in parts and k.endswith("_c")) or ("noisy" in parts and not k.endswith("_c")):
+                shapes[k] = (Bt, L, N)
         shapes.update({"A_f": (D, N), "A_r": (D, N), "D_f": (D,), "D_r": (D,)})
         if with_grads:
             shapes.update({"dy_c": (Bt, L, D), "dy_n": (Bt, L, D)})
@@ -113,7 +123,7 @@ class Workload:
             shapes["init_state"] = (Bt, D, N)
         self.t32 = {}
         for k, shp in shapes.items():
-            a = draw(k, shp, self.seed)
+            a = draw(k, shp, self.seed, 0 if k in PARAMS else part)
             if dtype == "bf16" and k not in PARAMS and k not in ("dstates", "init_state"):
                 a = bf16_bits_to_f32(f32_to_bf16_bits(a)).reshape(shp)
             self.t32[k] = a

@@ -1,0 +1,145 @@
+"""The C ABI on the host: the library builds and loads, exports every function
+include/bdscan.h declares, and rejects bad arguments before touching a GPU."""
+
+import os
+import re
+
+import pytest
+
+from paper_2607_02805_gb300 import binding
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "bdscan.h")
+
+
+def header_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(bdscan_\w+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_function():
+    lib = binding.load()
+    names = header_functions()
+    assert len(names) >= 10
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(n for n, _, _ in binding.SIGNATURES) == names
+
+
+def test_version_and_chunking():
+    assert binding.bdscan_version() >= 100
+    # chunks are whole blocks, about 128 tokens, and depend on the block size only
+    assert binding.bdscan_chunk_tokens(16) == 128
+    assert binding.bdscan_chunk_tokens(4) == 128
+    assert binding.bdscan_chunk_tokens(48) == 96
+    assert binding.bdscan_chunk_tokens(5) == 125
+    assert binding.bdscan_chunk_tokens(256) == 256
+    assert binding.bdscan_chunk_tokens(0) == 0
+
+
+def _dims(**kw):
+    base = dict(batch=2, length=64, block=16, d_inner=32, d_state=16, dtype=binding.BDSCAN_BF16)
+    base.update(kw)
+    return binding.make_dims(base["batch"], base["length"], base["block"], base["d_inner"], base["d_state"],
+                             base["dtype"], base.get("out_dtype"))
+
+
+def test_workspace_sizes():
+    d = _dims(batch=8, length=2048, block=16, d_inner=1536, d_state=16)
+    nc = 2048 // 128
+    al = lambda x: (x + 255) // 256 * 256
+    assert binding.bdscan_forward_workspace_size(d) == al(8 * (nc + 1) * 1536 * 16 * 4) + al(8 * nc * 1536 * 4)
+    assert binding.bdscan_boundary_states_workspace_size(d, 1) == binding.bdscan_forward_workspace_size(d)
+    G = 1536 // 128
+    expect = (al(8 * 128 * 1536 * 16 * 4) + al(8 * nc * 1536 * 16 * 4) + al(8 * nc * 1536 * 4)
+              + al(6 * 8 * 2048 * G * 16 * 4) + al(3 * 8 * nc * 1536 * 16 * 4) + al(2 * 8 * nc * 1536 * 4))
+    assert binding.bdscan_backward_workspace_size(d) == expect
+    assert binding.bdscan_forward_workspace_size(_dims(length=60)) == 0  # invalid dims -> 0
+
+
+FAKE = 1 << 20  # an aligned address that is never dereferenced on the error paths
+
+
+def _structs(ptr=FAKE):
+    c = binding.bdscan_clean(ptr, ptr, ptr, ptr)
+    n = binding.bdscan_noisy(ptr, ptr, ptr, ptr, ptr, ptr, ptr)
+    p = binding.bdscan_params(ptr, ptr, ptr, ptr)
+    return c, n, p
+
+
+def _fwd(d, c=None, n=None, p=None, y=FAKE, ws=FAKE, wsb=1 << 40):
+    c0, n0, p0 = _structs()
+    return binding.bdscan_forward(d, c or c0, n or n0, p or p0, y, y, y, ws, wsb, None)
+
+
+@pytest.mark.parametrize("kw,code,msg", [
+    (dict(length=60), binding.BDSCAN_ERR_ARG, "not a multiple of block"),
+    (dict(block=0), binding.BDSCAN_ERR_ARG, "block must be positive"),
+    (dict(batch=-1), binding.BDSCAN_ERR_ARG, "negative"),
+    (dict(d_state=12), binding.BDSCAN_ERR_UNSUPPORTED, "d_state"),
+    (dict(d_inner=12), binding.BDSCAN_ERR_UNSUPPORTED, "multiple of 8"),
+    (dict(dtype=binding.BDSCAN_F32, out_dtype=binding.BDSCAN_BF16), binding.BDSCAN_ERR_UNSUPPORTED, "f32 inputs"),
+    (dict(dtype=7), binding.BDSCAN_ERR_ARG, "bad dtype"),
+    (dict(block=128, length=256), binding.BDSCAN_ERR_UNSUPPORTED, "above 64"),
+])
+def test_forward_rejects_bad_dims(kw, code, msg):
+    assert _fwd(_dims(**kw)) == code
+    assert msg in binding.bdscan_last_error()
+
+
+def test_forward_rejects_bad_pointers_and_small_workspace():
+    d = _dims()
+    c, n, p = _structs()
+    c.dt = None
+    assert _fwd(d, c=c) == binding.BDSCAN_ERR_ARG and "clean.dt is NULL" in binding.bdscan_last_error()
+    c, n, p = _structs()
+    n.C_r = FAKE + 8
+    assert _fwd(d, n=n) == binding.BDSCAN_ERR_ARG and "noisy.C_r is not 16-byte aligned" in binding.bdscan_last_error()
+    assert _fwd(d, y=FAKE + 4) == binding.BDSCAN_ERR_ARG
+    assert _fwd(d, wsb=16) == binding.BDSCAN_ERR_ARG and "workspace" in binding.bdscan_last_error()
+    assert binding.bdscan_forward(None, *_structs(), FAKE, FAKE, FAKE, FAKE, 1 << 40, None) == binding.BDSCAN_ERR_ARG
+
+
+def test_zero_batch_is_a_noop_without_pointers():
+    d = _dims(batch=0)
+    c, n, p = _structs(None)
+    assert binding.bdscan_forward(d, c, n, p, None, None, None, None, 0, None) == binding.BDSCAN_OK
+
+
+def test_backward_block_limits():
+    d = _dims(block=24, length=48)
+    c, n, p = _structs()
+    gc = binding.bdscan_clean_grads(FAKE, FAKE, FAKE, FAKE)
+    gn = binding.bdscan_noisy_grads(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE)
+    gp = binding.bdscan_param_grads(FAKE, FAKE, FAKE, FAKE)
+    rc = binding.bdscan_backward(d, c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "multiple of 16" in binding.bdscan_last_error()
+    gn.dB_r = None
+    rc = binding.bdscan_backward(_dims(), c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "gnoisy.dB_r is NULL" in binding.bdscan_last_error()
+
+
+def test_active_block_needs_one_block():
+    d = _dims(length=32, block=16)
+    _, n, p = _structs()
+    rc = binding.bdscan_active_block(d, FAKE, n, p, FAKE, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "must equal block" in binding.bdscan_last_error()
+
+
+def test_boundary_states_checks():
+    d = _dims()
+    c, _, _ = _structs()
+    rc = binding.bdscan_boundary_states(d, c, FAKE, FAKE, FAKE + 4, None, FAKE, 1, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "init_state" in binding.bdscan_last_error()
+    rc = binding.bdscan_boundary_states(d, c, None, FAKE, None, None, FAKE, 1, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "A_f is NULL" in binding.bdscan_last_error()
+
+
+def test_fails_loudly_without_a_gpu():
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    d = _dims()
+    rc = _fwd(d)
+    assert rc == binding.BDSCAN_ERR_CUDA
+    assert "bdscan_forward" in binding.bdscan_last_error()
