@@ -218,6 +218,10 @@ def run_ours(args, rank, world, local_rank):
     nk = len(KERNELS)
     ev_start = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ev_k = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(args.steps)]
+    for evs in ev_k:  # torch creates the CUDA event on its first record
+        for e in evs:
+            e.record(stream)
+    torch.cuda.synchronize(dev)
     arr_f = [(ctypes.c_void_p * 3)(*[e.cuda_event for e in evs[:3]]) for evs in ev_k]
     arr_b = [(ctypes.c_void_p * (nk - 3))(*[e.cuda_event for e in evs[3:]]) for evs in ev_k]
 
@@ -245,7 +249,7 @@ def run_ours(args, rank, world, local_rank):
     # warm-up: at least W steps and about a second under load
     t_w = time.time()
     i = 0
-    while i < args.warmup or time.time() - t_w < 1.0:
+    while i < args.warmup or time.time() - t_w < args.warmup_seconds:
         step()
         i += 1
         if i % 50 == 0:
@@ -385,7 +389,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--warmup-seconds", type=float, default=1.0,
+                    help="keep warming up for at least this long (clock sampling under load)")
+    ap.add_argument("--batch", type=int, default=None, help="override the batch (smaller profiling case)")
     args = ap.parse_args()
+    if args.batch:
+        CFG["batch"] = args.batch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
