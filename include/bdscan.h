@@ -219,6 +219,37 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
 int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan_noisy* noisy,
                         const bdscan_params* params, void* y_n, void* stream);
 
+/* ---------------------------------------------------------------------- */
+/* Cache build for callers that cannot allocate device memory. The paper    */
+/* has no counterpart: this is a deployment convenience of this library.   */
+/* ---------------------------------------------------------------------- */
+/* Some callers are not allowed to allocate device memory at the point
+ * where they build or extend the cache: a plugin inside another inference
+ * engine whose execution step may only use memory that engine planned
+ * ahead of time, or a latency-critical serving loop where a cudaMalloc
+ * (which can synchronise the device) is not acceptable. This entry point
+ * takes the same arguments as bdscan_boundary_states minus the workspace
+ * and computes the same result (bit for bit). Its scratch is a static device
+ * array of BDSCAN_NOALLOC_SCRATCH_BYTES inside the library; every GPU on
+ * which the library is used keeps that array until the process exits.
+ *
+ * Size limit: the call needs bdscan_boundary_states_workspace_size(dims,
+ * emit_all) bytes of scratch; larger problems are rejected with
+ * BDSCAN_ERR_UNSUPPORTED (use bdscan_boundary_states with a workspace).
+ * First call per device: it looks up the array's device address with the
+ * device current; make that first call before any stream capture begins.
+ * Sharing: all calls use the same array. Calls whose GPU work overlaps (on
+ * different streams or from different threads without ordering between
+ * them) race on it and give wrong results; order them on one stream or with
+ * events. Nothing in the array has to start at zero: each call writes every
+ * scratch value before it reads it, so leftovers of a previous call are
+ * never used. No allocation happens in this call (no cudaMalloc, cudaFree,
+ * or allocating library routine). */
+#define BDSCAN_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+int bdscan_boundary_states_noalloc(const bdscan_dims* dims, const bdscan_clean* clean, const float* A_f,
+                                   const float* D_f, const float* init_state, void* y_c, float* states,
+                                   int emit_all, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

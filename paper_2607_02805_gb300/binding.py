@@ -82,7 +82,11 @@ SIGNATURES = [
       c_void_p, ctypes.c_size_t, c_void_p]),
     ("bdscan_active_block", ctypes.c_int,
      [_P(bdscan_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
+    ("bdscan_boundary_states_noalloc", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_clean), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, ctypes.c_int, c_void_p]),
 ]
+
+BDSCAN_NOALLOC_SCRATCH_BYTES = 32 << 20
 
 _lock = threading.Lock()
 _lib = None
@@ -180,6 +184,11 @@ def bdscan_boundary_states(dims, clean, A_f, D_f, init_state, y_c, states, emit_
 def bdscan_active_block(dims, seed, noisy, params, y_n, stream):
     return load().bdscan_active_block(_ref(dims), seed, _ref(noisy), _ref(params),
                                       y_n, stream)
+
+
+def bdscan_boundary_states_noalloc(dims, clean, A_f, D_f, init_state, y_c, states, emit_all, stream):
+    return load().bdscan_boundary_states_noalloc(_ref(dims), _ref(clean), A_f, D_f, init_state, y_c, states,
+                                                 int(emit_all), stream)
 
 
 # ---------------------------------------------------------------------------

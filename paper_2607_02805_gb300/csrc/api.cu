@@ -466,3 +466,25 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
 }
 
 }  // extern "C"
+
+namespace bds {
+
+int api_fail(int code, const char* msg) { return fail(code, "%s", msg); }
+
+int api_ok() { return ok(); }
+
+// Validation shared with other entry points that take forward-side dims.
+int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn) {
+  Call c;
+  int rc = check_dims((const bdscan_dims*)dims, &c, fn);
+  if (rc) return rc;
+  if ((rc = check_block_limits(c, false, fn))) return rc;
+  *g = c.g;
+  *dt = c.dt;
+  *N = c.N;
+  return BDSCAN_OK;
+}
+
+size_t api_fwd_workspace(const Geo& g, int N) { return fwd_ws(g, N); }
+
+}  // namespace bds

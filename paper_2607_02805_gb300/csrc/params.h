@@ -69,6 +69,12 @@ cudaError_t launch_bwd_reduce_tok(int dt, int N, const BwdParams& p, cudaStream_
 cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s);
 
 size_t block_scan_smem(int dt, int N, int mode, int64_t Bs);
+
+// Helpers of api.cu for other translation units of the library.
+int api_fail(int code, const char* msg);
+int api_ok();
+int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn);
+size_t api_fwd_workspace(const Geo& g, int N);
 size_t bwd_noisy_smem(int dt, int N, int64_t Bs);
 size_t bwd_clean_smem(int dt, int N, int64_t Bs);
 
