@@ -232,7 +232,9 @@ size_t bdscan_boundary_states_workspace_size(const bdscan_dims* dims, int emit_a
 size_t bdscan_backward_workspace_size(const bdscan_dims* dims) {
   Call c;
   if (check_dims(dims, &c, "bdscan_backward_workspace_size") != BDSCAN_OK) return 0;
-  return bwd_ws(c.g, c.N).total;
+  bds::Geo gmax = c.g;
+  gmax.nc = bds::bwd_max_chunks(c.g);
+  return bwd_ws(gmax, c.N).total;
 }
 
 int bdscan_forward(const bdscan_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
@@ -406,14 +408,19 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
   REQ(gnoisy->ddt_r, fn, "gnoisy.ddt_r");
   REQ(gnoisy->dB_r, fn, "gnoisy.dB_r");
   REQ(gnoisy->dC_r, fn, "gnoisy.dC_r");
-  const BwdWs w = bwd_ws(c.g, c.N);
+  bds::Geo gmax = c.g;
+  gmax.nc = bds::bwd_max_chunks(c.g);
+  const size_t need = bwd_ws(gmax, c.N).total;
   REQ(workspace, fn, "workspace");
-  if (workspace_bytes < w.total)
-    return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, w.total);
+  if (workspace_bytes < need)
+    return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
+  bds::Geo gb = c.g;  // the backward's own chunking of each batch row
+  gb.nc = bds::bwd_chunk_count(c.dt, c.N, c.g);
+  const BwdWs w = bwd_ws(gb, c.N);
 
   bds::BwdParams p;
   memset(&p, 0, sizeof(p));
-  p.g = c.g;
+  p.g = gb;
   p.xc = clean->x;
   p.dtc = clean->dt;
   p.Bc = clean->B;

@@ -30,6 +30,10 @@
 // (TMEM): 16 x N fp32 per thread would not fit in registers next to the
 // scan state, and TMEM is otherwise idle in this path. Blocks longer than 16
 // tokens are processed in 16-token segments from checkpointed states.
+//
+// Arithmetic is packed two state indices per FFMA2/FMUL2/FADD2, and per-thread
+// state vectors use the group-swizzled order of device.cuh, which makes the
+// channel reductions of dB and dC mostly select-free.
 #include "device.cuh"
 #include "params.h"
 
@@ -37,15 +41,21 @@ namespace bds {
 
 namespace {
 
+// checkpoint slots in shared memory: ck[slot][N][kCta], any (private) order
 template <int N>
-__device__ __forceinline__ void ck_store(float* ck, int slot, const float (&h)[N]) {
+__device__ __forceinline__ void ck_store(float* ck, int slot, const float2 (&h)[N / 2]) {
 #pragma unroll
-  for (int n = 0; n < N; ++n) ck[((size_t)slot * N + n) * kCta + threadIdx.x] = h[n];
+  for (int j = 0; j < N / 2; ++j) {
+    ck[((size_t)slot * N + 2 * j) * kCta + threadIdx.x] = h[j].x;
+    ck[((size_t)slot * N + 2 * j + 1) * kCta + threadIdx.x] = h[j].y;
+  }
 }
 template <int N>
-__device__ __forceinline__ void ck_load(float (&h)[N], const float* ck, int slot) {
+__device__ __forceinline__ void ck_load(float2 (&h)[N / 2], const float* ck, int slot) {
 #pragma unroll
-  for (int n = 0; n < N; ++n) h[n] = ck[((size_t)slot * N + n) * kCta + threadIdx.x];
+  for (int j = 0; j < N / 2; ++j)
+    h[j] = make_float2(ck[((size_t)slot * N + 2 * j) * kCta + threadIdx.x],
+                       ck[((size_t)slot * N + 2 * j + 1) * kCta + threadIdx.x]);
 }
 
 // red[which][i][warp][n]: which 0 = dB (adjoint pass), 1 = dC (recompute pass).
@@ -76,11 +86,86 @@ __device__ void red_flush(const BwdParams& p, const float* red, int tensB, int t
 
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 
-// TMEM columns per CTA and the residency that allows (512 columns per SM).
+// The backward splits each batch row's blocks into g.nc nearly equal chunks
+// (its own partition, chosen per call so the last wave of CTAs is nearly
+// full); chunk c holds blocks [chunk_lo(c), chunk_lo(c+1)).
+__host__ __device__ inline int chunk_lo(const Geo& g, int c) { return (int)(((int64_t)c * g.nb) / g.nc); }
+
 __host__ __device__ inline uint32_t tcols_host(int TS, int N) {
   uint32_t need = (uint32_t)(TS * N), c = 32;
   while (c < need) c <<= 1;
   return c;
+}
+
+// The state update alone on a group-swizzled packed state (checkpoint passes).
+template <int N>
+__device__ __forceinline__ void scan_state_swz(float2 (&h)[N / 2], const float2 (&A2)[N / 2], float dt, float x,
+                                               const float* Brow, int sw) {
+  const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x));
+  float2 B[N / 2];
+  vload2<N>(B, Brow, sw);
+#pragma unroll
+  for (int j = 0; j < N / 2; ++j) h[j] = fma2(ex2x2(mul2(dt2, A2[j])), h[j], mul2(u2, B[j]));
+}
+
+// Backward of one scan direction over one segment of TS tokens.
+// FWDDIR: the scan runs left to right (recompute i = 0..TS-1, adjoint
+// i = TS-1..0); otherwise right to left.
+//   h   the state the segment's first scanned token continues (clobbered)
+//   g   a_next gbar_next entering the segment's last scanned token (in/out)
+//   dA  accumulated sum of dt * gbar * p (in/out)
+//   epi(i, dt, x, dy, sum_n gbar B, sum_n A2 gbar p) writes the per-token results.
+// Channel sums of dy*h (dC) and gbar*dt*x (dB) go to red[1] and red[0].
+template <int N, bool FWDDIR, typename St, typename Epi>
+__device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, int jdy, int rB, int rC,
+                                        const float2 (&A2)[N / 2], int sw, float2 (&h)[N / 2],
+                                        float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* red,
+                                        Epi epi) {
+#pragma unroll 2
+  for (int k = 0; k < TS; ++k) {  // recompute, in scan order
+    const int i = FWDDIR ? k : TS - 1 - k;
+    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
+    float2 B[N / 2], pv[N / 2], w[N / 2];
+    vload2<N>(B, st.row(rB, i), sw);
+#pragma unroll
+    for (int j = 0; j < N / 2; ++j) {
+      const float2 a = ex2x2(mul2(dt2, A2[j]));
+      pv[j] = mul2(a, h[j]);
+      h[j] = fma2(u2, B[j], pv[j]);
+      w[j] = mul2(dy2, h[j]);
+    }
+    tmem_st2<N>(tb + (uint32_t)(i * N), pv);
+    red_put<N>(red, 1, TS, i, warp_reduce_swz<N>(w));
+  }
+  tmem_wait_st();
+#pragma unroll 2
+  for (int k = 0; k < TS; ++k) {  // adjoint, against scan order
+    const int i = FWDDIR ? TS - 1 - k : k;
+    float2 pv[N / 2];
+    tmem_ld2<N>(tb + (uint32_t)(i * N), pv);
+    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
+    float2 B[N / 2], C[N / 2], w[N / 2];
+    vload2<N>(B, st.row(rB, i), sw);
+    vload2<N>(C, st.row(rC, i), sw);
+    float2 sg[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    float2 sa[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+    for (int j = 0; j < N / 2; ++j) {
+      const float2 a = ex2x2(mul2(dt2, A2[j]));
+      const float2 gb = fma2(C[j], dy2, g[j]);
+      g[j] = mul2(a, gb);
+      const float2 q = mul2(gb, pv[j]);
+      sa[j & 1] = fma2(A2[j], q, sa[j & 1]);
+      dA[j] = fma2(dt2, q, dA[j]);
+      sg[j & 1] = fma2(gb, B[j], sg[j & 1]);
+      w[j] = mul2(gb, u2);
+    }
+    red_put<N>(red, 0, TS, i, warp_reduce_swz<N>(w));
+    const float2 sgs = add2(sg[0], sg[1]), sas = add2(sa[0], sa[1]);
+    epi(i, dt, x, dy, __fadd_rn(sgs.x, sgs.y), __fadd_rn(sas.x, sas.y));
+  }
 }
 
 }  // namespace
@@ -91,10 +176,10 @@ __host__ __device__ inline uint32_t tcols_host(int TS, int N) {
 template <typename T, int N>
 struct NoisyBwdSmem {
   // token-by-channel: x_n, dt_f, dt_r, dy_n, dt_c, dy_c; token-by-state: B_f, C_f, B_r, C_r, C_c
-  using St = Stage<T, N, 6, 5>;
-  static __host__ __device__ size_t stage_off() { return 0; }
-  static __host__ __device__ size_t dx_off(int TS) { return align16(St::bytes(TS)); }
-  static __host__ __device__ size_t red_off(int TS, int Bs) { return dx_off(TS) + (size_t)Bs * kCta * 4; }
+  using St = Stage<T, N, 6, 5, 2>;
+  // two staging buffers when a block is a single segment (prefetch of the next block)
+  static __host__ __device__ size_t dx_off(int TS, int Bs) { return align16(St::buf_bytes(TS) * (Bs / TS == 1 ? 2 : 1)); }
+  static __host__ __device__ size_t red_off(int TS, int Bs) { return dx_off(TS, Bs) + (size_t)Bs * kCta * 4; }
   static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * TS * kWarps * N * 4; }
   static __host__ __device__ size_t slot_off(int TS, int Bs) {
     const int nseg = Bs / TS;
@@ -108,14 +193,14 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   extern __shared__ __align__(16) unsigned char smem[];
   using L = NoisyBwdSmem<T, N>;
   const Geo& g = p.g;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  (void)lane;
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int sw = swz_of_lane<N>();
   const int64_t b = blockIdx.z;
   const int c = blockIdx.y;
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + tid;
   const bool act = d < g.D;
   const int Bs = (int)g.Bs, TS = Bs < 16 ? Bs : 16, NSEG = Bs / TS;
-  const int k_lo = c * g.m, k_hi = min(k_lo + g.m, g.nb) - 1;
+  const int k_lo = chunk_lo(g, c), k_hi = chunk_lo(g, c + 1) - 1;
 
   enum { XN = 0, DTF = 1, DTR = 2, DYN = 3, DTC = 4, DYC = 5 };
   enum { BF = 0, CF = 1, BR = 2, CR = 3, CC = 4 };
@@ -132,7 +217,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   st.row_src[BR] = (const T*)p.Br;
   st.row_src[CR] = (const T*)p.Cr;
   st.row_src[CC] = (const T*)p.Cc;
-  float* dxbuf = reinterpret_cast<float*>(smem + L::dx_off(TS));
+  float* dxbuf = reinterpret_cast<float*>(smem + L::dx_off(TS, Bs));
   float* red = reinterpret_cast<float*>(smem + L::red_off(TS, Bs));
   float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
@@ -143,212 +228,151 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   const uint32_t tbase = *tslot;
   const uint32_t tb = tbase + ((uint32_t)(warp * 32) << 16);
 
-  float A2f[N], A2r[N];
-  vzero(A2f);
-  vzero(A2r);
+  float2 A2f[N / 2], A2r[N / 2];
+  vzero2<N>(A2f);
+  vzero2<N>(A2r);
   float Dsum = 0.f;
   if (act) {
-    vload(A2f, p.Af + d * N);
-    vload(A2r, p.Ar + d * N);
+    vload2<N>(A2f, p.Af + d * N, sw);
+    vload2<N>(A2r, p.Ar + d * N, sw);
 #pragma unroll
-    for (int n = 0; n < N; ++n) {
-      A2f[n] = __fmul_rn(A2f[n], kLog2e);
-      A2r[n] = __fmul_rn(A2r[n], kLog2e);
+    for (int j = 0; j < N / 2; ++j) {
+      A2f[j] = mul2(A2f[j], f2(kLog2e));
+      A2r[j] = mul2(A2r[j], f2(kLog2e));
     }
     Dsum = __fadd_rn(p.Df[d], p.Dr[d]);
   }
-  float dAf[N], dAr[N];
-  vzero(dAf);
-  vzero(dAr);
+  float2 dAf[N / 2], dAr[N / 2];
+  vzero2<N>(dAf);
+  vzero2<N>(dAr);
   float dDn = 0.f, sdt = 0.f;
-  float carry[N];  // clean stream: a_{t+1} gbar_{t+1} (+ injections) entering token t from the right
-  vzero(carry);
-  float dSn[N];  // seed gradient of the block to the right of the current one
-  vzero(dSn);
+  float2 carry[N / 2];  // clean stream: a_{t+1} gbar_{t+1} (+ injections) entering token t from the right
+  vzero2<N>(carry);
+  float2 dSn[N / 2];  // seed gradient of the block to the right of the current one
+  vzero2<N>(dSn);
 
+  // one-segment blocks: block k-1 is copied while block k is processed
+  if (NSEG == 1) st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
   for (int k = k_hi; k >= k_lo; --k) {
     const int64_t t0 = (int64_t)k * Bs;
     const int64_t row0 = b * g.L + t0;
-    if (NSEG == 1) st.load(row0, TS, g.D, d0);
+    if (NSEG == 1) {
+      const int buf = (k_hi - k) & 1;
+      __syncthreads();  // the other buffer is no longer read
+      if (k > k_lo) st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
+      st.complete(buf, TS, k > k_lo ? 1 : 0);
+    }
 
     // ---- clean stream: chunk-local adjoint over block k ----
     if (k < k_hi) {
 #pragma unroll
-      for (int n = 0; n < N; ++n) carry[n] = __fadd_rn(carry[n], dSn[n]);
+      for (int j = 0; j < N / 2; ++j) carry[j] = add2(carry[j], dSn[j]);
       if (p.dstates != nullptr && act) {
-        float e[N];
-        vload(e, p.dstates + ((b * g.nb + k) * g.D + d) * N);
+        float2 e[N / 2];
+        vload2<N>(e, p.dstates + ((b * g.nb + k) * g.D + d) * N, sw);
 #pragma unroll
-        for (int n = 0; n < N; ++n) carry[n] = __fadd_rn(carry[n], e[n]);
+        for (int j = 0; j < N / 2; ++j) carry[j] = add2(carry[j], e[j]);
       }
     }
     for (int s = NSEG - 1; s >= 0; --s) {
       if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+#pragma unroll 2
       for (int i = TS - 1; i >= 0; --i) {
         const float dt = st.at(DTC, i), dy = st.at(DYC, i);
-        float C[N];
-        vload_row(C, st.row(CC, i));
+        const float2 dt2 = f2(dt), dy2 = f2(dy);
+        float2 C[N / 2];
+        vload2<N>(C, st.row(CC, i), sw);
 #pragma unroll
-        for (int n = 0; n < N; ++n) {
-          const float gb = __fmaf_rn(C[n], dy, carry[n]);
-          carry[n] = __fmul_rn(ex2(__fmul_rn(dt, A2f[n])), gb);
-        }
+        for (int j = 0; j < N / 2; ++j) carry[j] = mul2(ex2x2(mul2(dt2, A2f[j])), fma2(C[j], dy2, carry[j]));
         sdt = __fadd_rn(sdt, dt);
       }
     }
 
-    // ---- noisy block k, reverse direction ----
+    // ---- noisy block k, reverse direction (zero state at the block end) ----
     {
       if (NSEG > 1) {
-        float h[N];
-        vzero(h);
+        float2 h[N / 2];
+        vzero2<N>(h);
         for (int s = NSEG - 1; s >= 1; --s) {
           st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
-          for (int i = TS - 1; i >= 0; --i) scan_state(h, A2r, st.at(DTR, i), st.at(XN, i), st.row(BR, i));
-          ck_store(ck, s - 1, h);
+          for (int i = TS - 1; i >= 0; --i) scan_state_swz<N>(h, A2r, st.at(DTR, i), st.at(XN, i), st.row(BR, i), sw);
+          ck_store<N>(ck, s - 1, h);
         }
       }
-      float gr[N];  // a_{t-1} gbar_{t-1}, entering token t from the left
-      vzero(gr);
+      float2 gr[N / 2];  // a_{t-1} gbar_{t-1}, entering token t from the left
+      vzero2<N>(gr);
       for (int s = 0; s < NSEG; ++s) {
         if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
-        float h[N];
+        float2 h[N / 2];
         if (s == NSEG - 1)
-          vzero(h);
+          vzero2<N>(h);
         else
-          ck_load(h, ck, s);
-        for (int i = TS - 1; i >= 0; --i) {  // recompute, right to left
-          const float dt = st.at(DTR, i), x = st.at(XN, i), dy = st.at(DYN, i);
-          const float u = __fmul_rn(dt, x);
-          float B[N], pv[N], w[N];
-          vload_row(B, st.row(BR, i));
-#pragma unroll
-          for (int n = 0; n < N; ++n) {
-            const float a = ex2(__fmul_rn(dt, A2r[n]));
-            pv[n] = __fmul_rn(a, h[n]);
-            h[n] = __fmaf_rn(u, B[n], pv[n]);
-            w[n] = __fmul_rn(dy, h[n]);
-          }
-          Tmem<N>::st(tb + (uint32_t)(i * N), pv);
-          red_put<N>(red, 1, TS, i, warp_reduce_scatter<N>(w));
-        }
-        tmem_wait_st();
-        for (int i = 0; i < TS; ++i) {  // adjoint, left to right
-          const float dt = st.at(DTR, i), x = st.at(XN, i), dy = st.at(DYN, i);
-          const float u = __fmul_rn(dt, x);
-          float B[N], C[N], pv[N], w[N];
-          vload_row(B, st.row(BR, i));
-          vload_row(C, st.row(CR, i));
-          Tmem<N>::ld(tb + (uint32_t)(i * N), pv);
-          float sgB = 0.f, sAq = 0.f;
-#pragma unroll
-          for (int n = 0; n < N; ++n) {
-            const float a = ex2(__fmul_rn(dt, A2r[n]));
-            const float gb = __fmaf_rn(C[n], dy, gr[n]);
-            gr[n] = __fmul_rn(a, gb);
-            const float q = __fmul_rn(gb, pv[n]);
-            sAq = __fmaf_rn(A2r[n], q, sAq);
-            dAr[n] = __fmaf_rn(dt, q, dAr[n]);
-            sgB = __fmaf_rn(gb, B[n], sgB);
-            w[n] = __fmul_rn(gb, u);
-          }
-          red_put<N>(red, 0, TS, i, warp_reduce_scatter<N>(w));
-          const int ib = s * TS + i;
-          if (act)
-            reinterpret_cast<TO*>(p.ddtr)[(row0 + ib) * g.D + d] =
-                to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
-          dxbuf[ib * kCta + tid] = __fmul_rn(dt, sgB);
-        }
+          ck_load<N>(h, ck, s);
+        seg_bwd<N, false>(st, TS, XN, DTR, DYN, BR, CR, A2r, sw, h, gr, dAr, tb, red,
+                          [&](int i, float dt, float x, float dy, float sgB, float sAq) {
+                            const int ib = s * TS + i;
+                            if (act)
+                              reinterpret_cast<TO*>(p.ddtr)[(row0 + ib) * g.D + d] =
+                                  to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
+                            dxbuf[ib * kCta + tid] = __fmul_rn(dt, sgB);
+                          });
         red_flush<N>(p, red, 4, 5, b, t0 + (int64_t)s * TS, TS);
       }
     }
 
     // ---- noisy block k, forward direction (seeded with states[k-1]) ----
     {
-      float seed[N];
-      vzero(seed);
-      if (k > 0 && act) vload(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N);
+      float2 seed[N / 2];
+      vzero2<N>(seed);
+      if (k > 0 && act) vload2<N>(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N, sw);
       if (NSEG > 1) {
-        float h[N];
+        float2 h[N / 2];
 #pragma unroll
-        for (int n = 0; n < N; ++n) h[n] = seed[n];
+        for (int j = 0; j < N / 2; ++j) h[j] = seed[j];
         for (int s = 0; s < NSEG - 1; ++s) {
           st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
-          for (int i = 0; i < TS; ++i) scan_state(h, A2f, st.at(DTF, i), st.at(XN, i), st.row(BF, i));
-          ck_store(ck, s, h);
+          for (int i = 0; i < TS; ++i) scan_state_swz<N>(h, A2f, st.at(DTF, i), st.at(XN, i), st.row(BF, i), sw);
+          ck_store<N>(ck, s, h);
         }
       }
-      float gf[N];  // a_{t+1} gbar_{t+1}, entering token t from the right
-      vzero(gf);
+      float2 gf[N / 2];  // a_{t+1} gbar_{t+1}, entering token t from the right
+      vzero2<N>(gf);
       for (int s = NSEG - 1; s >= 0; --s) {
         if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
-        float h[N];
+        float2 h[N / 2];
         if (s == 0) {
 #pragma unroll
-          for (int n = 0; n < N; ++n) h[n] = seed[n];
+          for (int j = 0; j < N / 2; ++j) h[j] = seed[j];
         } else {
-          ck_load(h, ck, s - 1);
+          ck_load<N>(h, ck, s - 1);
         }
-        for (int i = 0; i < TS; ++i) {  // recompute, left to right
-          const float dt = st.at(DTF, i), x = st.at(XN, i), dy = st.at(DYN, i);
-          const float u = __fmul_rn(dt, x);
-          float B[N], pv[N], w[N];
-          vload_row(B, st.row(BF, i));
-#pragma unroll
-          for (int n = 0; n < N; ++n) {
-            const float a = ex2(__fmul_rn(dt, A2f[n]));
-            pv[n] = __fmul_rn(a, h[n]);
-            h[n] = __fmaf_rn(u, B[n], pv[n]);
-            w[n] = __fmul_rn(dy, h[n]);
-          }
-          Tmem<N>::st(tb + (uint32_t)(i * N), pv);
-          red_put<N>(red, 1, TS, i, warp_reduce_scatter<N>(w));
-        }
-        tmem_wait_st();
-        for (int i = TS - 1; i >= 0; --i) {  // adjoint, right to left
-          const float dt = st.at(DTF, i), x = st.at(XN, i), dy = st.at(DYN, i);
-          const float u = __fmul_rn(dt, x);
-          float B[N], C[N], pv[N], w[N];
-          vload_row(B, st.row(BF, i));
-          vload_row(C, st.row(CF, i));
-          Tmem<N>::ld(tb + (uint32_t)(i * N), pv);
-          float sgB = 0.f, sAq = 0.f;
-#pragma unroll
-          for (int n = 0; n < N; ++n) {
-            const float a = ex2(__fmul_rn(dt, A2f[n]));
-            const float gb = __fmaf_rn(C[n], dy, gf[n]);
-            gf[n] = __fmul_rn(a, gb);
-            const float q = __fmul_rn(gb, pv[n]);
-            sAq = __fmaf_rn(A2f[n], q, sAq);
-            dAf[n] = __fmaf_rn(dt, q, dAf[n]);
-            sgB = __fmaf_rn(gb, B[n], sgB);
-            w[n] = __fmul_rn(gb, u);
-          }
-          red_put<N>(red, 0, TS, i, warp_reduce_scatter<N>(w));
-          const int ib = s * TS + i;
-          const int64_t o = (row0 + ib) * g.D + d;
-          if (act) {
-            reinterpret_cast<TO*>(p.ddtf)[o] = to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
-            const float dxv = __fmaf_rn(Dsum, dy, __fadd_rn(dxbuf[ib * kCta + tid], __fmul_rn(dt, sgB)));
-            reinterpret_cast<TO*>(p.dxn)[o] = to_out<TO>(dxv);
-          }
-          dDn = __fmaf_rn(dy, x, dDn);
-        }
+        seg_bwd<N, true>(st, TS, XN, DTF, DYN, BF, CF, A2f, sw, h, gf, dAf, tb, red,
+                         [&](int i, float dt, float x, float dy, float sgB, float sAq) {
+                           const int ib = s * TS + i;
+                           const int64_t o = (row0 + ib) * g.D + d;
+                           if (act) {
+                             reinterpret_cast<TO*>(p.ddtf)[o] = to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
+                             const float dxv =
+                                 __fmaf_rn(Dsum, dy, __fadd_rn(dxbuf[ib * kCta + tid], __fmul_rn(dt, sgB)));
+                             reinterpret_cast<TO*>(p.dxn)[o] = to_out<TO>(dxv);
+                           }
+                           dDn = __fmaf_rn(dy, x, dDn);
+                         });
         red_flush<N>(p, red, 2, 3, b, t0 + (int64_t)s * TS, TS);
       }
       // gradient of this block's seed, states[k-1]: a_{t0} gbar_{t0}
 #pragma unroll
-      for (int n = 0; n < N; ++n) dSn[n] = gf[n];
-      if (k > 0 && act) vstore(p.dS + ((b * g.nb + (k - 1)) * g.D + d) * N, gf);
+      for (int j = 0; j < N / 2; ++j) dSn[j] = gf[j];
+      if (k > 0 && act) vstore2<N>(p.dS + ((b * g.nb + (k - 1)) * g.D + d) * N, gf, sw);
     }
   }
 
   if (act) {
-    vstore(p.Lc + ((b * g.nc + c) * g.D + d) * N, carry);
+    vstore2<N>(p.Lc + ((b * g.nc + c) * g.D + d) * N, carry, sw);
     p.sdtc[(b * g.nc + c) * g.D + d] = sdt;
     const int64_t u = b * g.nc + c, U = g.Bt * g.nc;
-    vstore(p.part_A + ((0 * U + u) * g.D + d) * N, dAf);
-    vstore(p.part_A + ((1 * U + u) * g.D + d) * N, dAr);
+    vstore2<N>(p.part_A + ((0 * U + u) * g.D + d) * N, dAf, sw);
+    vstore2<N>(p.part_A + ((1 * U + u) * g.D + d) * N, dAr, sw);
     p.part_D[(0 * U + u) * g.D + d] = dDn;
   }
   tmem_sync();
@@ -367,16 +391,32 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
   const int64_t d = (idx / N) % g.D, b = idx / ((int64_t)N * g.D);
   const float A2 = __fmul_rn(p.Af[d * N + n], kLog2e);
   float G = 0.f;  // a_{t+1} gbar_{t+1} entering the current chunk's last token from the right
-  for (int c = g.nc - 1; c >= 0; --c) {
-    const int kl = min((c + 1) * g.m, g.nb) - 1;
-    float gin = G;
-    if (kl + 1 < g.nb) gin = __fadd_rn(gin, p.dS[((b * g.nb + kl) * g.D + d) * N + n]);
-    if (p.dstates != nullptr) gin = __fadd_rn(gin, p.dstates[((b * g.nb + kl) * g.D + d) * N + n]);
-    const int64_t o = ((b * g.nc + c) * g.D + d) * N + n;
-    const float loc = p.Lc[o];
-    const float s = p.sdtc[(b * g.nc + c) * g.D + d];
-    p.Lc[o] = gin;
-    G = __fmaf_rn(ex2(__fmul_rn(A2, s)), gin, loc);
+  constexpr int U = 8;
+  for (int c0 = g.nc - 1; c0 >= 0; c0 -= U) {
+    // loads of up to U chunks first (they do not depend on the carry)
+    float inj[U], loc[U], sd[U];
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const int c = c0 - j;
+      inj[j] = 0.f;
+      loc[j] = 0.f;
+      sd[j] = 0.f;
+      if (c >= 0) {
+        const int kl = chunk_lo(g, c + 1) - 1;
+        if (kl + 1 < g.nb) inj[j] = p.dS[((b * g.nb + kl) * g.D + d) * N + n];
+        if (p.dstates != nullptr) inj[j] = __fadd_rn(inj[j], p.dstates[((b * g.nb + kl) * g.D + d) * N + n]);
+        loc[j] = p.Lc[((b * g.nc + c) * g.D + d) * N + n];
+        sd[j] = p.sdtc[(b * g.nc + c) * g.D + d];
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < U; ++j) {
+      const int c = c0 - j;
+      if (c < 0) break;
+      const float gin = __fadd_rn(G, inj[j]);
+      p.Lc[((b * g.nc + c) * g.D + d) * N + n] = gin;
+      G = __fmaf_rn(ex2(__fmul_rn(A2, sd[j])), gin, loc[j]);
+    }
   }
 }
 
@@ -385,12 +425,12 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
 // ---------------------------------------------------------------------------
 template <typename T, int N>
 struct CleanBwdSmem {
-  using St = Stage<T, N, 3, 2>;  // x_c, dt_c, dy_c; B_c, C_c
-  static __host__ __device__ size_t red_off(int TS) { return align16(St::bytes(TS)); }
-  static __host__ __device__ size_t ck_off(int TS) { return red_off(TS) + (size_t)2 * TS * kWarps * N * 4; }
+  using St = Stage<T, N, 3, 2, 2>;  // x_c, dt_c, dy_c; B_c, C_c
+  static __host__ __device__ size_t red_off(int TS, int Bs) { return align16(St::buf_bytes(TS) * (Bs / TS == 1 ? 2 : 1)); }
+  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * TS * kWarps * N * 4; }
   static __host__ __device__ size_t slot_off(int TS, int Bs) {
     const int nseg = Bs / TS;
-    return ck_off(TS) + (size_t)(nseg > 1 ? nseg - 1 : 1) * N * kCta * 4;
+    return ck_off(TS, Bs) + (size_t)(nseg > 1 ? nseg - 1 : 1) * N * kCta * 4;
   }
   static __host__ __device__ size_t bytes(int TS, int Bs) { return slot_off(TS, Bs) + 16; }
 };
@@ -401,12 +441,13 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
   using L = CleanBwdSmem<T, N>;
   const Geo& g = p.g;
   const int tid = threadIdx.x, warp = tid >> 5;
+  const int sw = swz_of_lane<N>();
   const int64_t b = blockIdx.z;
   const int c = blockIdx.y;
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + tid;
   const bool act = d < g.D;
   const int Bs = (int)g.Bs, TS = Bs < 16 ? Bs : 16, NSEG = Bs / TS;
-  const int k_lo = c * g.m, k_hi = min(k_lo + g.m, g.nb) - 1;
+  const int k_lo = chunk_lo(g, c), k_hi = chunk_lo(g, c + 1) - 1;
 
   enum { XC = 0, DTC = 1, DYC = 2 };
   enum { BC = 0, CC = 1 };
@@ -417,8 +458,8 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
   st.td_src[DYC] = (const T*)p.dyc;
   st.row_src[BC] = (const T*)p.Bc;
   st.row_src[CC] = (const T*)p.Cc;
-  float* red = reinterpret_cast<float*>(smem + L::red_off(TS));
-  float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS));
+  float* red = reinterpret_cast<float*>(smem + L::red_off(TS, Bs));
+  float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
 
   const uint32_t tcols = tmem_cols_for((uint32_t)(TS * N));
@@ -427,109 +468,82 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
   const uint32_t tbase = *tslot;
   const uint32_t tb = tbase + ((uint32_t)(warp * 32) << 16);
 
-  float A2[N];
-  vzero(A2);
+  float2 A2[N / 2];
+  vzero2<N>(A2);
   float Df = 0.f;
   if (act) {
-    vload(A2, p.Af + d * N);
+    vload2<N>(A2, p.Af + d * N, sw);
 #pragma unroll
-    for (int n = 0; n < N; ++n) A2[n] = __fmul_rn(A2[n], kLog2e);
+    for (int j = 0; j < N / 2; ++j) A2[j] = mul2(A2[j], f2(kLog2e));
     Df = p.Df[d];
   }
-  float dA[N];
-  vzero(dA);
+  float2 dA[N / 2];
+  vzero2<N>(dA);
   float dDc = 0.f;
-  float gc[N];  // a_{t+1} gbar_{t+1} (+ injections) entering token t from the right
-  vzero(gc);
+  float2 gc[N / 2];  // a_{t+1} gbar_{t+1} (+ injections) entering token t from the right
+  vzero2<N>(gc);
 
+  // one-segment blocks: block k-1 is copied while block k is processed
+  if (NSEG == 1) st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
   for (int k = k_hi; k >= k_lo; --k) {
     const int64_t t0 = (int64_t)k * Bs;
     const int64_t row0 = b * g.L + t0;
-    if (NSEG == 1) st.load(row0, TS, g.D, d0);
+    if (NSEG == 1) {
+      const int buf = (k_hi - k) & 1;
+      __syncthreads();  // the other buffer is no longer read
+      if (k > k_lo) st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
+      st.complete(buf, TS, k > k_lo ? 1 : 0);
+    }
     if (k == k_hi) {
-      if (act) vload(gc, p.Lc + ((b * g.nc + c) * g.D + d) * N);
+      if (act) vload2<N>(gc, p.Lc + ((b * g.nc + c) * g.D + d) * N, sw);
     } else if (act) {
-      float e[N];
-      vload(e, p.dS + ((b * g.nb + k) * g.D + d) * N);
+      float2 e[N / 2];
+      vload2<N>(e, p.dS + ((b * g.nb + k) * g.D + d) * N, sw);
 #pragma unroll
-      for (int n = 0; n < N; ++n) gc[n] = __fadd_rn(gc[n], e[n]);
+      for (int j = 0; j < N / 2; ++j) gc[j] = add2(gc[j], e[j]);
       if (p.dstates != nullptr) {
-        vload(e, p.dstates + ((b * g.nb + k) * g.D + d) * N);
+        vload2<N>(e, p.dstates + ((b * g.nb + k) * g.D + d) * N, sw);
 #pragma unroll
-        for (int n = 0; n < N; ++n) gc[n] = __fadd_rn(gc[n], e[n]);
+        for (int j = 0; j < N / 2; ++j) gc[j] = add2(gc[j], e[j]);
       }
     }
-    float seed[N];
-    vzero(seed);
-    if (k > 0 && act) vload(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N);
+    float2 seed[N / 2];
+    vzero2<N>(seed);
+    if (k > 0 && act) vload2<N>(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N, sw);
     if (NSEG > 1) {
-      float h[N];
+      float2 h[N / 2];
 #pragma unroll
-      for (int n = 0; n < N; ++n) h[n] = seed[n];
+      for (int j = 0; j < N / 2; ++j) h[j] = seed[j];
       for (int s = 0; s < NSEG - 1; ++s) {
         st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
-        for (int i = 0; i < TS; ++i) scan_state(h, A2, st.at(DTC, i), st.at(XC, i), st.row(BC, i));
-        ck_store(ck, s, h);
+        for (int i = 0; i < TS; ++i) scan_state_swz<N>(h, A2, st.at(DTC, i), st.at(XC, i), st.row(BC, i), sw);
+        ck_store<N>(ck, s, h);
       }
     }
     for (int s = NSEG - 1; s >= 0; --s) {
       if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
-      float h[N];
+      float2 h[N / 2];
       if (s == 0) {
 #pragma unroll
-        for (int n = 0; n < N; ++n) h[n] = seed[n];
+        for (int j = 0; j < N / 2; ++j) h[j] = seed[j];
       } else {
-        ck_load(h, ck, s - 1);
+        ck_load<N>(h, ck, s - 1);
       }
-      for (int i = 0; i < TS; ++i) {  // recompute, left to right
-        const float dt = st.at(DTC, i), x = st.at(XC, i), dy = st.at(DYC, i);
-        const float u = __fmul_rn(dt, x);
-        float B[N], pv[N], w[N];
-        vload_row(B, st.row(BC, i));
-#pragma unroll
-        for (int n = 0; n < N; ++n) {
-          const float a = ex2(__fmul_rn(dt, A2[n]));
-          pv[n] = __fmul_rn(a, h[n]);
-          h[n] = __fmaf_rn(u, B[n], pv[n]);
-          w[n] = __fmul_rn(dy, h[n]);
-        }
-        Tmem<N>::st(tb + (uint32_t)(i * N), pv);
-        red_put<N>(red, 1, TS, i, warp_reduce_scatter<N>(w));
-      }
-      tmem_wait_st();
-      for (int i = TS - 1; i >= 0; --i) {  // adjoint, right to left
-        const float dt = st.at(DTC, i), x = st.at(XC, i), dy = st.at(DYC, i);
-        const float u = __fmul_rn(dt, x);
-        float B[N], C[N], pv[N], w[N];
-        vload_row(B, st.row(BC, i));
-        vload_row(C, st.row(CC, i));
-        Tmem<N>::ld(tb + (uint32_t)(i * N), pv);
-        float sgB = 0.f, sAq = 0.f;
-#pragma unroll
-        for (int n = 0; n < N; ++n) {
-          const float a = ex2(__fmul_rn(dt, A2[n]));
-          const float gb = __fmaf_rn(C[n], dy, gc[n]);
-          gc[n] = __fmul_rn(a, gb);
-          const float q = __fmul_rn(gb, pv[n]);
-          sAq = __fmaf_rn(A2[n], q, sAq);
-          dA[n] = __fmaf_rn(dt, q, dA[n]);
-          sgB = __fmaf_rn(gb, B[n], sgB);
-          w[n] = __fmul_rn(gb, u);
-        }
-        red_put<N>(red, 0, TS, i, warp_reduce_scatter<N>(w));
-        const int64_t o = (row0 + s * TS + i) * g.D + d;
-        if (act) {
-          reinterpret_cast<TO*>(p.ddtc)[o] = to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
-          reinterpret_cast<TO*>(p.dxc)[o] = to_out<TO>(__fmaf_rn(Df, dy, __fmul_rn(dt, sgB)));
-        }
-        dDc = __fmaf_rn(dy, x, dDc);
-      }
+      seg_bwd<N, true>(st, TS, XC, DTC, DYC, BC, CC, A2, sw, h, gc, dA, tb, red,
+                       [&](int i, float dt, float x, float dy, float sgB, float sAq) {
+                         const int64_t o = (row0 + s * TS + i) * g.D + d;
+                         if (act) {
+                           reinterpret_cast<TO*>(p.ddtc)[o] = to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
+                           reinterpret_cast<TO*>(p.dxc)[o] = to_out<TO>(__fmaf_rn(Df, dy, __fmul_rn(dt, sgB)));
+                         }
+                         dDc = __fmaf_rn(dy, x, dDc);
+                       });
       red_flush<N>(p, red, 0, 1, b, t0 + (int64_t)s * TS, TS);
     }
   }
   if (act) {
     const int64_t u = b * g.nc + c, U = g.Bt * g.nc;
-    vstore(p.part_A + ((2 * U + u) * g.D + d) * N, dA);
+    vstore2<N>(p.part_A + ((2 * U + u) * g.D + d) * N, dA, sw);
     p.part_D[(1 * U + u) * g.D + d] = dDc;
   }
   tmem_sync();
@@ -552,34 +566,60 @@ __global__ void __launch_bounds__(256) k_reduce_tok(const BwdParams p) {
   const float* src = p.part_tok + row * g.G * N + n;
   float s = 0.f;
   for (int gi = 0; gi < g.G; ++gi) s += src[(int64_t)gi * N];
-  void* dsts[6] = {p.dBc, p.dCc, p.dBf, p.dCf, p.dBr, p.dCr};
-  reinterpret_cast<TO*>(dsts[tensor])[bt * N + n] = to_out<TO>(s);
+  void* dst = tensor == 0 ? p.dBc : tensor == 1 ? p.dCc : tensor == 2 ? p.dBf : tensor == 3 ? p.dCf
+            : tensor == 4 ? p.dBr : p.dCr;
+  reinterpret_cast<TO*>(dst)[bt * N + n] = to_out<TO>(s);
 }
 
+// One CTA sums 32 columns of the per-chunk partials: 8 slices of threads
+// each add every 8th chunk (in order), then the slices are added in order.
 template <int N>
 __global__ void __launch_bounds__(256) k_reduce_par(const BwdParams p) {
+  __shared__ float part[5][8][32];
   const Geo& g = p.g;
   const int64_t U = g.Bt * g.nc;
   const int64_t DN = g.D * N;
-  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (idx < DN) {
-    float sf = 0.f, sc = 0.f, sr = 0.f;
-    for (int64_t u = 0; u < U; ++u) {
-      sf += p.part_A[(0 * U + u) * DN + idx];
-      sr += p.part_A[(1 * U + u) * DN + idx];
-      sc += p.part_A[(2 * U + u) * DN + idx];
+  const int lane = threadIdx.x & 31, slice = threadIdx.x >> 5;
+  const int64_t col = (int64_t)blockIdx.x * 32 + lane;
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f;
+  if (col < DN) {
+    const float* a0 = p.part_A + col;
+    const float* a1 = p.part_A + U * DN + col;
+    const float* a2 = p.part_A + 2 * U * DN + col;
+#pragma unroll 4
+    for (int64_t u = slice; u < U; u += 8) {
+      s0 += a0[u * DN];
+      s1 += a1[u * DN];
+      s2 += a2[u * DN];
     }
-    p.dAf[idx] = sf + sc;
-    p.dAr[idx] = sr;
-  } else if (idx < DN + g.D) {
-    const int64_t d = idx - DN;
-    float sn = 0.f, sc = 0.f;
-    for (int64_t u = 0; u < U; ++u) {
-      sn += p.part_D[(0 * U + u) * g.D + d];
-      sc += p.part_D[(1 * U + u) * g.D + d];
+  } else if (col < DN + g.D) {
+    const int64_t d = col - DN;
+#pragma unroll 4
+    for (int64_t u = slice; u < U; u += 8) {
+      s0 += p.part_D[u * g.D + d];
+      s1 += p.part_D[(U + u) * g.D + d];
     }
-    p.dDf[d] = sn + sc;
-    p.dDr[d] = sn;
+  }
+  part[0][slice][lane] = s0;
+  part[1][slice][lane] = s1;
+  part[2][slice][lane] = s2;
+  __syncthreads();
+  if (slice == 0) {
+    float t0 = part[0][0][lane], t1 = part[1][0][lane], t2 = part[2][0][lane];
+#pragma unroll
+    for (int k = 1; k < 8; ++k) {
+      t0 += part[0][k][lane];
+      t1 += part[1][k][lane];
+      t2 += part[2][k][lane];
+    }
+    if (col < DN) {
+      p.dAf[col] = t0 + t2;  // noisy forward direction + clean stream
+      p.dAr[col] = t1;
+    } else if (col < DN + g.D) {
+      const int64_t d = col - DN;
+      p.dDf[d] = t0 + t1;  // noisy + clean
+      p.dDr[d] = t0;
+    }
   }
 }
 
@@ -593,9 +633,9 @@ namespace {
 inline size_t pad_for_tmem(size_t smem, int TS, int N) {
   const uint32_t cols = tcols_host(TS, N);
   const int ctas = (int)(512 / cols);
+  if (ctas >= 16) return smem;  // the thread limit already bounds residency
   const size_t cap = (size_t)(220 * 1024) / (size_t)ctas;
-  size_t need = cap > 2048 ? cap - 2048 : cap;
-  if (ctas >= 16) need = 0;  // thread limit already bounds residency
+  const size_t need = cap > 2048 ? cap - 2048 : cap;
   return smem > need ? smem : need;
 }
 
@@ -664,7 +704,50 @@ cudaError_t launch_bwd_reduce_tok(int dt, int N, const BwdParams& p, cudaStream_
 
 cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s) {
   const int64_t npar = p.g.D * N + p.g.D;
-  BDS_DISPATCH_N(N, k_reduce_par<NN><<<(unsigned)((npar + 255) / 256), 256, 0, s>>>(p); return cudaGetLastError();)
+  BDS_DISPATCH_N(N, k_reduce_par<NN><<<(unsigned)((npar + 31) / 32), 256, 0, s>>>(p); return cudaGetLastError();)
+}
+
+// Backward chunks per batch row: the count whose grid (channel groups x
+// chunks x batch) fills the resident CTA slots best, between 1 and
+// bwd_max_chunks(). Falls back to the forward chunking if the occupancy
+// query fails.
+int bwd_chunk_count(int dt, int N, const Geo& g) {
+  int dev = 0, sms = 0, per_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return g.nc;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) return g.nc;
+  const int Bs = (int)g.Bs, TS = Bs < 16 ? Bs : 16;
+  const size_t smem = pad_for_tmem(dt == 0 ? (N == 8 ? NoisyBwdSmem<float, 8>::bytes(TS, Bs) : NoisyBwdSmem<float, 16>::bytes(TS, Bs))
+                                           : (N == 8 ? NoisyBwdSmem<bf16, 8>::bytes(TS, Bs) : NoisyBwdSmem<bf16, 16>::bytes(TS, Bs)),
+                                   TS, N);
+  cudaError_t e = cudaErrorInvalidValue;
+  if (dt == 0)
+    e = N == 8 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<float, float, 8>, kCta, smem)
+               : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<float, float, 16>, kCta, smem);
+  else if (dt == 1)
+    e = N == 8 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, bf16, 8>, kCta, smem)
+               : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, bf16, 16>, kCta, smem);
+  else
+    e = N == 8 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, float, 8>, kCta, smem)
+               : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, float, 16>, kCta, smem);
+  if (e != cudaSuccess || per_sm <= 0) {
+    cudaGetLastError();
+    return g.nc;
+  }
+  const int64_t slots = (int64_t)per_sm * sms;
+  const int64_t rows = g.Bt * g.G;
+  const int cmax = bwd_max_chunks(g);
+  int best = g.nc;
+  double best_cost = 1e300;
+  for (int nc = 1; nc <= cmax; ++nc) {
+    const int64_t waves = (rows * nc + slots - 1) / slots;
+    const int64_t blocks = (g.nb + nc - 1) / nc;  // longest chunk
+    const double cost = (double)waves * ((double)blocks + 0.25);  // + per-CTA set-up, in blocks
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best = nc;
+    }
+  }
+  return best;
 }
 
 size_t bwd_noisy_smem(int dt, int N, int64_t Bs) {

@@ -94,62 +94,88 @@ __device__ __forceinline__ void issue_rows(T* dst, const T* g, int64_t row0, int
   }
 }
 
-// A set of staged tensors for one span of up to `tsmax` tokens.
-template <typename T, int N, int NTD, int NROW>
+__device__ __forceinline__ void cp_async_wait_one() { asm volatile("cp.async.wait_group 1;\n" ::: "memory"); }
+
+// A set of staged tensors for one span of up to `tsmax` tokens, in NBUF
+// shared-memory buffers. With two buffers the next span is copied while the
+// current one is processed: issue(next) ... complete(current, pending = 1).
+template <typename T, int N, int NTD, int NROW, int NBUF = 1>
 struct Stage {
-  T* td;        // [NTD][tsmax][kCta]
-  T* raw;       // [NROW][tsmax][N] (bf16 inputs only)
-  float* rows;  // [NROW][tsmax][N] fp32
+  unsigned char* base;
   int tsmax;
+  const T* cur_td;       // token-by-channel tiles of the current buffer, this thread's channel
+  const float* cur_rows;  // fp32 rows of the current buffer
   const T* td_src[NTD];
   const T* row_src[NROW];
 
-  static __host__ __device__ size_t bytes(int tsmax) {
-    size_t b = (size_t)NTD * tsmax * kCta * sizeof(T);
-    b = (b + 15) & ~(size_t)15;
-    if (!is_f32<T>::value) b += ((size_t)NROW * tsmax * N * sizeof(T) + 15) & ~(size_t)15;
-    b += (size_t)NROW * tsmax * N * sizeof(float);
-    return b;
+  static __host__ __device__ size_t td_bytes(int ts) { return ((size_t)NTD * ts * kCta * sizeof(T) + 15) & ~(size_t)15; }
+  static __host__ __device__ size_t raw_bytes(int ts) {
+    return is_f32<T>::value ? 0 : (((size_t)NROW * ts * N * sizeof(T) + 15) & ~(size_t)15);
   }
-  __device__ void carve(unsigned char* base, int ts) {
+  static __host__ __device__ size_t rows_bytes(int ts) { return (size_t)NROW * ts * N * sizeof(float); }
+  static __host__ __device__ size_t buf_bytes(int ts) { return td_bytes(ts) + raw_bytes(ts) + rows_bytes(ts); }
+  static __host__ __device__ size_t bytes(int ts) { return (size_t)NBUF * buf_bytes(ts); }
+
+  __device__ void carve(unsigned char* b, int ts) {
+    base = b;
     tsmax = ts;
-    size_t o = (size_t)NTD * ts * kCta * sizeof(T);
-    o = (o + 15) & ~(size_t)15;
-    td = reinterpret_cast<T*>(base);
-    if (!is_f32<T>::value) {
-      raw = reinterpret_cast<T*>(base + o);
-      o += ((size_t)NROW * ts * N * sizeof(T) + 15) & ~(size_t)15;
-      rows = reinterpret_cast<float*>(base + o);
-    } else {
-      rows = reinterpret_cast<float*>(base + o);
-      raw = reinterpret_cast<T*>(rows);
-    }
+    select(0);
   }
-  // Loads tokens [row0, row0+nsteps) of this CTA's batch row and channels.
-  // Starts with a barrier so no thread still reads the previous contents.
-  __device__ void load(int64_t row0, int nsteps, int64_t D, int64_t d0) {
-    __syncthreads();
+  __device__ __forceinline__ void select(int buf) {
+    cur_td = td(buf) + threadIdx.x;
+    cur_rows = rows(buf);
+  }
+  __device__ __forceinline__ T* td(int buf) const { return reinterpret_cast<T*>(base + (size_t)buf * buf_bytes(tsmax)); }
+  __device__ __forceinline__ float* rows(int buf) const {
+    return reinterpret_cast<float*>(base + (size_t)buf * buf_bytes(tsmax) + td_bytes(tsmax) + raw_bytes(tsmax));
+  }
+  __device__ __forceinline__ T* raw(int buf) const {
+    return is_f32<T>::value ? reinterpret_cast<T*>(rows(buf))
+                            : reinterpret_cast<T*>(base + (size_t)buf * buf_bytes(tsmax) + td_bytes(tsmax));
+  }
+  // Starts the copies of tokens [row0, row0+nsteps) into buffer `buf` (one
+  // cp.async group per thread). The caller guarantees no thread still reads it.
+  __device__ void issue(int buf, int64_t row0, int nsteps, int64_t D, int64_t d0) {
+    T* t = td(buf);
+    T* r = raw(buf);
 #pragma unroll
-    for (int j = 0; j < NTD; ++j) issue_td<T>(td + (size_t)j * tsmax * kCta, td_src[j], row0, nsteps, D, d0);
+    for (int j = 0; j < NTD; ++j) issue_td<T>(t + (size_t)j * tsmax * kCta, td_src[j], row0, nsteps, D, d0);
 #pragma unroll
-    for (int j = 0; j < NROW; ++j) issue_rows<T, N>(raw + (size_t)j * tsmax * N, row_src[j], row0, nsteps);
+    for (int j = 0; j < NROW; ++j) issue_rows<T, N>(r + (size_t)j * tsmax * N, row_src[j], row0, nsteps);
     cp_async_commit();
-    cp_async_wait_all();
+  }
+  // Waits for the copies of buffer `buf` (with `pending` newer groups still in
+  // flight), widens its B/C rows to fp32 and makes it the current buffer.
+  __device__ void complete(int buf, int nsteps, int pending) {
+    if (pending)
+      cp_async_wait_one();
+    else
+      cp_async_wait_all();
     __syncthreads();
     if (!is_f32<T>::value) {
       const int per = nsteps * N;
+      const T* r = raw(buf);
+      float* f = rows(buf);
       for (int i = threadIdx.x; i < NROW * per; i += kCta) {
-        const int j = i / per, r = i - j * per;
-        rows[(size_t)j * tsmax * N + r] = cvt(raw[(size_t)j * tsmax * N + r]);
+        const int j = i / per, q = i - j * per;
+        f[(size_t)j * tsmax * N + q] = cvt(r[(size_t)j * tsmax * N + q]);
       }
       __syncthreads();
     }
+    select(buf);
+  }
+  // Synchronous load into buffer 0 (starts with a barrier so no thread still
+  // reads the previous contents).
+  __device__ void load(int64_t row0, int nsteps, int64_t D, int64_t d0) {
+    __syncthreads();
+    issue(0, row0, nsteps, D, d0);
+    complete(0, nsteps, 0);
   }
   __device__ __forceinline__ float at(int j, int step) const {
-    return cvt(td[((size_t)j * tsmax + step) * kCta + threadIdx.x]);
+    return cvt(cur_td[(j * tsmax + step) * kCta]);
   }
   __device__ __forceinline__ const float* row(int j, int step) const {
-    return rows + ((size_t)j * tsmax + step) * N;
+    return cur_rows + (j * tsmax + step) * N;
   }
 };
 
@@ -189,51 +215,6 @@ __device__ __forceinline__ void vload_row(float (&v)[N], const float* s) {  // s
   }
 }
 
-// ---------------------------------------------------------------------------
-// The selective-scan step (eq. mamba-scan-background with A_t = exp(dt A)):
-//     a[n] = 2^(dt * A2[n]),  h[n] = a[n] h[n] + (dt x) B[n],
-// returning sum_n C[n] h[n] (without the D term). The operation order is
-// fixed with explicit round-to-nearest intrinsics, so every kernel that uses
-// it (all-block forward, cache build, cache tail, active block) produces the
-// same bits from the same state and inputs.
-// ---------------------------------------------------------------------------
-template <int N>
-__device__ __forceinline__ float scan_step(float (&h)[N], const float (&A2)[N], float dt, float x,
-                                           const float* Bs, const float* Cs) {
-  const float u = __fmul_rn(dt, x);
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-  for (int n = 0; n < N; n += 4) {
-    const float4 b = *reinterpret_cast<const float4*>(Bs + n);
-    const float4 c = *reinterpret_cast<const float4*>(Cs + n);
-    const float bb[4] = {b.x, b.y, b.z, b.w}, cc[4] = {c.x, c.y, c.z, c.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float a = ex2(__fmul_rn(dt, A2[n + j]));
-      h[n + j] = __fmaf_rn(a, h[n + j], __fmul_rn(u, bb[j]));
-      acc[j] = __fmaf_rn(cc[j], h[n + j], acc[j]);
-    }
-  }
-  return __fadd_rn(__fadd_rn(acc[0], acc[1]), __fadd_rn(acc[2], acc[3]));
-}
-
-// The state update alone (no output), same arithmetic as scan_step.
-template <int N>
-__device__ __forceinline__ void scan_state(float (&h)[N], const float (&A2)[N], float dt, float x,
-                                           const float* Bs) {
-  const float u = __fmul_rn(dt, x);
-#pragma unroll
-  for (int n = 0; n < N; n += 4) {
-    const float4 b = *reinterpret_cast<const float4*>(Bs + n);
-    const float bb[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float a = ex2(__fmul_rn(dt, A2[n + j]));
-      h[n + j] = __fmaf_rn(a, h[n + j], __fmul_rn(u, bb[j]));
-    }
-  }
-}
-
 // y of one direction with its D term, and the two-direction sum of a noisy
 // token (eq. partial-reverse). Shared by the all-block forward and the
 // active-block step so both round identically.
@@ -265,6 +246,121 @@ __device__ __forceinline__ float warp_reduce_scatter(float (&v)[N]) {
 }
 
 // ---------------------------------------------------------------------------
+// Packed FP32: two state indices per FFMA2/FMUL2/FADD2 (sm_100 family). Each
+// half is rounded exactly as the scalar __fmaf_rn/__fmul_rn/__fadd_rn.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float2 f2(float v) { return make_float2(v, v); }
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
+__device__ __forceinline__ float2 add2(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 ex2x2(float2 v) { return make_float2(ex2(v.x), ex2(v.y)); }
+
+// Per-thread state vectors of N floats held as N/2 float2. In the backward
+// kernels the 4-float groups of a vector are stored in a lane-dependent
+// order: slot group j holds state group j ^ sw with sw = (lane >> 2) & (N/4 - 1).
+// This makes the first halving levels of the channel reduction select-free
+// (see warp_reduce_swz). The forward kernels use the natural order (sw = 0).
+template <int N>
+__device__ __forceinline__ int swz_of_lane() {
+  return (int)((threadIdx.x >> 2) & (N / 4 - 1));
+}
+// global or shared memory -> registers, group-swizzled
+template <int N>
+__device__ __forceinline__ void vload2(float2 (&v)[N / 2], const float* src, int sw) {
+#pragma unroll
+  for (int j = 0; j < N / 4; ++j) {
+    const float4 q = *reinterpret_cast<const float4*>(src + 4 * (j ^ sw));
+    v[2 * j] = make_float2(q.x, q.y);
+    v[2 * j + 1] = make_float2(q.z, q.w);
+  }
+}
+template <int N>
+__device__ __forceinline__ void vstore2(float* dst, const float2 (&v)[N / 2], int sw) {
+#pragma unroll
+  for (int j = 0; j < N / 4; ++j)
+    *reinterpret_cast<float4*>(dst + 4 * (j ^ sw)) = make_float4(v[2 * j].x, v[2 * j].y, v[2 * j + 1].x, v[2 * j + 1].y);
+}
+template <int N>
+__device__ __forceinline__ void vzero2(float2 (&v)[N / 2]) {
+#pragma unroll
+  for (int j = 0; j < N / 2; ++j) v[j] = make_float2(0.f, 0.f);
+}
+
+// Channel reduction of a group-swizzled vector: v summed over the 32 lanes;
+// afterwards every lane l holds the total for state index l % N. The levels
+// over lane bits 3 and 2 exchange whole slot halves without selects (the
+// partner's matching state sits in the complementary slot); the levels over
+// lane bits 1 and 0 exchange within a 4-group with selects; the remaining
+// lane bits are a butterfly. Fixed order: deterministic.
+template <int N>
+__device__ __forceinline__ float warp_reduce_swz(float2 (&v)[N / 2]) {
+  const int lane = threadIdx.x & 31;
+  // group levels: offsets N/2 ... 4 (in floats), i.e. N/4 ... 2 float2 slots
+#pragma unroll
+  for (int o = N / 4; o >= 2; o >>= 1) {
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const float2 r = make_float2(__shfl_xor_sync(0xffffffffu, v[i + o].x, 2 * o),
+                                   __shfl_xor_sync(0xffffffffu, v[i + o].y, 2 * o));
+      v[i] = add2(v[i], r);
+    }
+  }
+  // v[0], v[1] now hold the four states of group sw; lane bit 1 picks a pair
+  const bool up1 = (lane & 2) != 0;
+  float k0 = up1 ? v[1].x : v[0].x, k1 = up1 ? v[1].y : v[0].y;
+  const float s0 = up1 ? v[0].x : v[1].x, s1 = up1 ? v[0].y : v[1].y;
+  k0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+  k1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+  const bool up0 = (lane & 1) != 0;
+  float k = up0 ? k1 : k0;
+  const float s = up0 ? k0 : k1;
+  k += __shfl_xor_sync(0xffffffffu, s, 1);
+#pragma unroll
+  for (int o = N; o < 32; o <<= 1) k += __shfl_xor_sync(0xffffffffu, k, o);
+  return k;
+}
+
+// ---------------------------------------------------------------------------
+// The selective-scan step (eq. mamba-scan-background with A_t = exp(dt A)):
+//     a[n] = 2^(dt * A2[n]),  h[n] = a[n] h[n] + (dt x) B[n],
+// returning sum_n C[n] h[n] (without the D term), on a packed state in the
+// natural order. The operation order is fixed with explicit round-to-nearest
+// intrinsics, so every kernel that uses it (all-block forward, cache build,
+// cache tail, active block) produces the same bits from the same state and
+// inputs.
+// ---------------------------------------------------------------------------
+template <int N>
+__device__ __forceinline__ float scan_step(float2 (&h)[N / 2], const float2 (&A2)[N / 2], float dt, float x,
+                                           const float* Bs, const float* Cs) {
+  const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x));
+  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int q = 0; q < N / 4; ++q) {
+    const float4 b = *reinterpret_cast<const float4*>(Bs + 4 * q);
+    const float4 c = *reinterpret_cast<const float4*>(Cs + 4 * q);
+    h[2 * q] = fma2(ex2x2(mul2(dt2, A2[2 * q])), h[2 * q], mul2(u2, make_float2(b.x, b.y)));
+    acc0 = fma2(make_float2(c.x, c.y), h[2 * q], acc0);
+    h[2 * q + 1] = fma2(ex2x2(mul2(dt2, A2[2 * q + 1])), h[2 * q + 1], mul2(u2, make_float2(b.z, b.w)));
+    acc1 = fma2(make_float2(c.z, c.w), h[2 * q + 1], acc1);
+  }
+  const float2 s = add2(acc0, acc1);
+  return __fadd_rn(s.x, s.y);
+}
+
+// The state update alone (no output), same arithmetic as scan_step.
+template <int N>
+__device__ __forceinline__ void scan_state(float2 (&h)[N / 2], const float2 (&A2)[N / 2], float dt, float x,
+                                           const float* Bs) {
+  const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x));
+#pragma unroll
+  for (int q = 0; q < N / 4; ++q) {
+    const float4 b = *reinterpret_cast<const float4*>(Bs + 4 * q);
+    h[2 * q] = fma2(ex2x2(mul2(dt2, A2[2 * q])), h[2 * q], mul2(u2, make_float2(b.x, b.y)));
+    h[2 * q + 1] = fma2(ex2x2(mul2(dt2, A2[2 * q + 1])), h[2 * q + 1], mul2(u2, make_float2(b.z, b.w)));
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Tensor memory (TMEM) as per-thread scratch for the backward recompute.
 // A CTA of 4 warps allocates `cols` 32-bit columns; warp w owns TMEM lanes
 // 32w..32w+31 (one lane per thread), so each thread has `cols` private fp32
@@ -290,10 +386,32 @@ __device__ __forceinline__ void tmem_sync() {
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
 }
-__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::); }
 
 template <int N>
 struct Tmem;
+
+// float2-array views of the TMEM row copies
+template <int N>
+__device__ __forceinline__ void tmem_st2(uint32_t ta, const float2 (&v)[N / 2]) {
+  Tmem<N>::st(ta, *reinterpret_cast<const float(*)[N]>(&v[0]));
+}
+template <int N>
+__device__ __forceinline__ void tmem_ld2(uint32_t ta, float2 (&v)[N / 2]) {
+  Tmem<N>::ld(ta, *reinterpret_cast<float(*)[N]>(&v[0]));
+}
+// Split form: request a row into raw registers r, do other work, then wait.
+// r must not be read, written or copied between the two calls (the load
+// writes it asynchronously); the wait names r, so no use of it can be
+// scheduled before the wait.
+template <int N>
+__device__ __forceinline__ void tmem_ld_async(uint32_t ta, uint32_t (&r)[N]) {
+  Tmem<N>::ld_nowait(ta, r);
+}
+template <int N>
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[N]) {
+  Tmem<N>::wait(r);
+}
 
 template <>
 struct Tmem<16> {
@@ -306,8 +424,7 @@ struct Tmem<16> {
         "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
         "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
         "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
-        "r"(__float_as_uint(v[15]))
-        : "memory");
+        "r"(__float_as_uint(v[15])));
   }
   static __device__ __forceinline__ void ld(uint32_t ta, float (&v)[16]) {
     uint32_t r[16];
@@ -316,17 +433,30 @@ struct Tmem<16> {
         "%13, %14, %15}, [%16];\n"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
           "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(ta)
-        : "memory");
+        : "r"(ta));
     // the wait names the destination registers so no use moves above it
     asm volatile("tcgen05.wait::ld.sync.aligned;\n"
                  : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
                    "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
                    "+r"(r[14]), "+r"(r[15])
-                 :
-                 : "memory");
+                 :);
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+  }
+  static __device__ __forceinline__ void ld_nowait(uint32_t ta, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, "
+        "%13, %14, %15}, [%16];\n"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(ta));
+  }
+  static __device__ __forceinline__ void wait(uint32_t (&r)[16]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;\n"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+                   "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
+                   "+r"(r[14]), "+r"(r[15])
+                 :);
   }
 };
 
@@ -336,21 +466,28 @@ struct Tmem<8> {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"r"(ta),
                  "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
                  "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
-                 "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7]))
-                 : "memory");
+                 "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])));
   }
   static __device__ __forceinline__ void ld(uint32_t ta, float (&v)[8]) {
     uint32_t r[8];
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];\n"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                 : "r"(ta)
-                 : "memory");
+                 : "r"(ta));
     asm volatile("tcgen05.wait::ld.sync.aligned;\n"
                  : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7])
-                 :
-                 : "memory");
+                 :);
 #pragma unroll
     for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+  }
+  static __device__ __forceinline__ void ld_nowait(uint32_t ta, uint32_t (&r)[8]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(ta));
+  }
+  static __device__ __forceinline__ void wait(uint32_t (&r)[8]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;\n"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7])
+                 :);
   }
 };
 

@@ -36,36 +36,43 @@ __global__ void __launch_bounds__(kCta) k_chunk_local(const FwdParams p) {
   const int c = blockIdx.y;
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
   const bool act = d < g.D;
-  Stage<T, N, 2, 1> st;
+  Stage<T, N, 2, 1, 2> st;
   st.carve(smem, kLocalSpan);
   st.td_src[0] = (const T*)p.xc;
   st.td_src[1] = (const T*)p.dtc;
   st.row_src[0] = (const T*)p.Bc;
 
-  float A2[N];
+  float2 A2[N / 2], h[N / 2];
+  vzero2<N>(A2);
+  vzero2<N>(h);
   if (act) {
-    vload(A2, p.Af + d * N);
+    vload2<N>(A2, p.Af + d * N, 0);
 #pragma unroll
-    for (int n = 0; n < N; ++n) A2[n] = __fmul_rn(A2[n], kLog2e);
-  } else {
-    vzero(A2);
+    for (int j = 0; j < N / 2; ++j) A2[j] = mul2(A2[j], f2(kLog2e));
   }
-  float h[N];
-  vzero(h);
   float sdt = 0.f;
   const int64_t tc = (int64_t)g.m * g.Bs;
   const int64_t tbeg = (int64_t)c * tc;
-  for (int64_t t = 0; t < tc; t += kLocalSpan) {
+  const int nspan = (int)((tc + kLocalSpan - 1) / kLocalSpan);
+  st.issue(0, b * g.L + tbeg, (int)(tc < kLocalSpan ? tc : kLocalSpan), g.D, d0);
+  for (int sp = 0; sp < nspan; ++sp) {
+    const int64_t t = (int64_t)sp * kLocalSpan;
     const int ns = (int)((tc - t) < kLocalSpan ? (tc - t) : kLocalSpan);
-    st.load(b * g.L + tbeg + t, ns, g.D, d0);
+    __syncthreads();  // the other buffer is no longer read
+    if (sp + 1 < nspan) {
+      const int64_t tn = t + kLocalSpan;
+      st.issue((sp + 1) & 1, b * g.L + tbeg + tn, (int)((tc - tn) < kLocalSpan ? (tc - tn) : kLocalSpan), g.D, d0);
+    }
+    st.complete(sp & 1, ns, sp + 1 < nspan ? 1 : 0);
+#pragma unroll 4
     for (int i = 0; i < ns; ++i) {
       const float dt = st.at(1, i);
-      scan_state(h, A2, dt, st.at(0, i), st.row(0, i));
+      scan_state<N>(h, A2, dt, st.at(0, i), st.row(0, i));
       sdt = __fadd_rn(sdt, dt);
     }
   }
   if (act) {
-    vstore(p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, h);
+    vstore2<N>(p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, h, 0);
     p.sdt[(b * g.nc + c) * g.D + d] = sdt;
   }
 }
@@ -122,7 +129,7 @@ struct ScanLayout {
 };
 
 template <typename T, typename TO, int N, int MODE>
-__global__ void __launch_bounds__(kCta) k_block_scan(const FwdParams p) {
+__global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   using Ly = ScanLayout<MODE>;
   extern __shared__ __align__(16) unsigned char smem[];
   const Geo& g = p.g;
@@ -131,9 +138,11 @@ __global__ void __launch_bounds__(kCta) k_block_scan(const FwdParams p) {
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
   const bool act = d < g.D;
   const int Bs = (int)g.Bs;
-  Stage<T, N, Ly::NTD, Ly::NROW> st;
+  Stage<T, N, Ly::NTD, Ly::NROW, 2> st;
   st.carve(smem, Bs);
-  float* yfbuf = reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW>::bytes(Bs));
+  const bool dbuf = p.stage_bufs == 2;
+  float* yfbuf =
+      reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(Bs) * (dbuf ? 2 : 1));
   if (Ly::kClean) {
     st.td_src[Ly::XC] = (const T*)p.xc;
     st.td_src[Ly::DTC] = (const T*)p.dtc;
@@ -150,21 +159,21 @@ __global__ void __launch_bounds__(kCta) k_block_scan(const FwdParams p) {
     st.row_src[Ly::CR] = (const T*)p.Cr;
   }
 
-  float A2f[N], A2r[N];
+  float2 A2f[N / 2], A2r[N / 2];
   float Df = 0.f, Dr = 0.f;
-  vzero(A2f);
-  vzero(A2r);
+  vzero2<N>(A2f);
+  vzero2<N>(A2r);
   if (act) {
-    vload(A2f, p.Af + d * N);
+    vload2<N>(A2f, p.Af + d * N, 0);
     Df = p.Df[d];
     if (Ly::kNoisy) {
-      vload(A2r, p.Ar + d * N);
+      vload2<N>(A2r, p.Ar + d * N, 0);
       Dr = p.Dr[d];
     }
 #pragma unroll
-    for (int n = 0; n < N; ++n) {
-      A2f[n] = __fmul_rn(A2f[n], kLog2e);
-      A2r[n] = __fmul_rn(A2r[n], kLog2e);
+    for (int j = 0; j < N / 2; ++j) {
+      A2f[j] = mul2(A2f[j], f2(kLog2e));
+      A2r[j] = mul2(A2r[j], f2(kLog2e));
     }
   }
 
@@ -175,51 +184,60 @@ __global__ void __launch_bounds__(kCta) k_block_scan(const FwdParams p) {
     k_hi = min(k_lo + g.m, g.nb) - 1;
     full = c < g.nc_full;
   }
-  float hc[N];
-  vzero(hc);
+  float2 hc[N / 2];
+  vzero2<N>(hc);
   if (act) {
     if (MODE == 2)
-      vload(hc, p.seed + (b * g.D + d) * N);
+      vload2<N>(hc, p.seed + (b * g.D + d) * N, 0);
     else
-      vload(hc, p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N);
+      vload2<N>(hc, p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, 0);
   }
 
+  if (dbuf) st.issue(0, b * g.L + (int64_t)k_lo * Bs, Bs, g.D, d0);
   for (int k = k_lo; k <= k_hi; ++k) {
     const int64_t row0 = b * g.L + (int64_t)k * Bs;
-    st.load(row0, Bs, g.D, d0);
-    float hs[N];
+    if (dbuf) {
+      __syncthreads();  // the other buffer is no longer read
+      if (k < k_hi) st.issue((k - k_lo + 1) & 1, row0 + Bs, Bs, g.D, d0);
+      st.complete((k - k_lo) & 1, Bs, k < k_hi ? 1 : 0);
+    } else {
+      st.load(row0, Bs, g.D, d0);
+    }
+    float2 hs[N / 2];
 #pragma unroll
-    for (int n = 0; n < N; ++n) hs[n] = hc[n];  // the block's seed: state before its first token
+    for (int j = 0; j < N / 2; ++j) hs[j] = hc[j];  // the block's seed: state before its first token
+#pragma unroll 4
     for (int i = 0; i < Bs; ++i) {
       const int64_t o = (row0 + i) * g.D + d;
       if (Ly::kClean) {
         const float x = st.at(Ly::XC, i), dt = st.at(Ly::DTC, i);
-        const float y = scan_step(hc, A2f, dt, x, st.row(Ly::BC, i), st.row(Ly::CC, i));
+        const float y = scan_step<N>(hc, A2f, dt, x, st.row(Ly::BC, i), st.row(Ly::CC, i));
         if (p.yc != nullptr && act) reinterpret_cast<TO*>(p.yc)[o] = to_out<TO>(with_skip(y, Df, x));
       }
       if (Ly::kNoisy) {
         const float x = st.at(Ly::XN, i), dt = st.at(Ly::DTF, i);
-        const float y = scan_step(hs, A2f, dt, x, st.row(Ly::BF, i), st.row(Ly::CF, i));
+        const float y = scan_step<N>(hs, A2f, dt, x, st.row(Ly::BF, i), st.row(Ly::CF, i));
         yfbuf[i * kCta + threadIdx.x] = with_skip(y, Df, x);
       }
     }
     if (Ly::kClean && p.emit_all && act) {
       float* dst = p.states + ((b * g.nb + k) * g.D + d) * N;
       if (k == k_hi && full) {
-        float e[N];
-        vload(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N);
-        vstore(dst, e);
+        float2 e[N / 2];
+        vload2<N>(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N, 0);
+        vstore2<N>(dst, e, 0);
       } else {
-        vstore(dst, hc);
+        vstore2<N>(dst, hc, 0);
       }
     }
     if (Ly::kNoisy) {
-      float hr[N];
-      vzero(hr);
+      float2 hr[N / 2];
+      vzero2<N>(hr);
+#pragma unroll 4
       for (int i = Bs - 1; i >= 0; --i) {
         const int64_t o = (row0 + i) * g.D + d;
         const float x = st.at(Ly::XN, i), dt = st.at(Ly::DTR, i);
-        const float y = scan_step(hr, A2r, dt, x, st.row(Ly::BR, i), st.row(Ly::CR, i));
+        const float y = scan_step<N>(hr, A2r, dt, x, st.row(Ly::BR, i), st.row(Ly::CR, i));
         if (act)
           reinterpret_cast<TO*>(p.yn)[o] =
               to_out<TO>(combine_dirs(yfbuf[i * kCta + threadIdx.x], with_skip(y, Dr, x)));
@@ -229,11 +247,11 @@ __global__ void __launch_bounds__(kCta) k_block_scan(const FwdParams p) {
   if (Ly::kClean && p.final_state != nullptr && c == g.nc - 1 && act) {
     float* dst = p.final_state + (b * g.D + d) * N;
     if (full) {
-      float e[N];
-      vload(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N);
-      vstore(dst, e);
+      float2 e[N / 2];
+      vload2<N>(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N, 0);
+      vstore2<N>(dst, e, 0);
     } else {
-      vstore(dst, hc);
+      vstore2<N>(dst, hc, 0);
     }
   }
 }
@@ -245,22 +263,38 @@ namespace {
 
 template <typename T, int N>
 cudaError_t chunk_local_t(const FwdParams& p, cudaStream_t s) {
-  const size_t smem = Stage<T, N, 2, 1>::bytes(kLocalSpan);
+  const size_t smem = Stage<T, N, 2, 1, 2>::bytes(kLocalSpan);
+  cudaError_t e = cudaFuncSetAttribute(k_chunk_local<T, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc_full, (unsigned)p.g.Bt);
   k_chunk_local<T, N><<<grid, kCta, smem, s>>>(p);
   return cudaGetLastError();
 }
 
+// Above this much shared memory per CTA the block scan stages synchronously:
+// at 16-token blocks a second buffer would cost a resident CTA per SM, which
+// measured slower than the overlap it buys.
+constexpr size_t kDoubleBufferLimit = 48 * 1024;
+
+template <typename T, typename TO, int N, int MODE>
+int block_scan_bufs_t(int64_t Bs) {
+  using Ly = ScanLayout<MODE>;
+  const size_t extra = Ly::kNoisy ? (size_t)Bs * kCta * sizeof(float) : 0;
+  return 2 * Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes((int)Bs) + extra <= kDoubleBufferLimit ? 2 : 1;
+}
+
 template <typename T, typename TO, int N, int MODE>
 size_t block_scan_smem_t(int64_t Bs) {
   using Ly = ScanLayout<MODE>;
-  size_t b = Stage<T, N, Ly::NTD, Ly::NROW>::bytes((int)Bs);
+  size_t b = Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes((int)Bs) * block_scan_bufs_t<T, TO, N, MODE>(Bs);
   if (Ly::kNoisy) b += (size_t)Bs * kCta * sizeof(float);
   return b;
 }
 
 template <typename T, typename TO, int N, int MODE>
-cudaError_t block_scan_t(int nchunks, const FwdParams& p, cudaStream_t s) {
+cudaError_t block_scan_t(int nchunks, const FwdParams& p_in, cudaStream_t s) {
+  FwdParams p = p_in;
+  p.stage_bufs = block_scan_bufs_t<T, TO, N, MODE>(p.g.Bs);
   const size_t smem = block_scan_smem_t<T, TO, N, MODE>(p.g.Bs);
   cudaError_t e = cudaFuncSetAttribute(k_block_scan<T, TO, N, MODE>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -34,6 +34,7 @@ struct FwdParams {
   const float* init;   // [Bt][D][N] or null: state before token 0
   const float* seed;   // active block: [Bt][D][N]
   int c_begin;         // first chunk handled by a block-scan launch
+  int stage_bufs;      // block scan: 2 = copy the next block while computing, 1 = synchronous
 };
 
 // Backward-side kernels.
@@ -76,6 +77,11 @@ int api_ok();
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn);
 size_t api_fwd_workspace(const Geo& g, int N);
 size_t bwd_noisy_smem(int dt, int N, int64_t Bs);
+int bwd_chunk_count(int dt, int N, const Geo& g);
+// Upper bound of the backward's chunks per batch row (sizes its workspace
+// independently of the device): twice the forward chunking, at most one
+// chunk per block.
+inline int bwd_max_chunks(const Geo& g) { return g.nb < 2 * g.nc ? g.nb : 2 * g.nc; }
 size_t bwd_clean_smem(int dt, int N, int64_t Bs);
 
 }  // namespace bds

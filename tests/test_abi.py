@@ -51,8 +51,9 @@ def test_workspace_sizes():
     assert binding.bdscan_forward_workspace_size(d) == al(8 * (nc + 1) * 1536 * 16 * 4) + al(8 * nc * 1536 * 4)
     assert binding.bdscan_boundary_states_workspace_size(d, 1) == binding.bdscan_forward_workspace_size(d)
     G = 1536 // 128
-    expect = (al(8 * 128 * 1536 * 16 * 4) + al(8 * nc * 1536 * 16 * 4) + al(8 * nc * 1536 * 4)
-              + al(6 * 8 * 2048 * G * 16 * 4) + al(3 * 8 * nc * 1536 * 16 * 4) + al(2 * 8 * nc * 1536 * 4))
+    ncb = min(128, 2 * nc)  # the backward's own chunking is bounded by twice the forward's
+    expect = (al(8 * 128 * 1536 * 16 * 4) + al(8 * ncb * 1536 * 16 * 4) + al(8 * ncb * 1536 * 4)
+              + al(6 * 8 * 2048 * G * 16 * 4) + al(3 * 8 * ncb * 1536 * 16 * 4) + al(2 * 8 * ncb * 1536 * 4))
     assert binding.bdscan_backward_workspace_size(d) == expect
     assert binding.bdscan_forward_workspace_size(_dims(length=60)) == 0  # invalid dims -> 0
 
