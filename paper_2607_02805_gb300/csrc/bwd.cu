@@ -58,11 +58,20 @@ __device__ __forceinline__ void ck_load(float2 (&h)[N / 2], const float* ck, int
                        ck[((size_t)slot * N + 2 * j + 1) * kCta + threadIdx.x]);
 }
 
-// red[which][i][warp][n]: which 0 = dB (adjoint pass), 1 = dC (recompute pass).
+// Tokens per backward segment; also the fixed stride of the staged tiles and
+// of the reduction buffer, so that their addresses are immediates.
+constexpr int kBwdTS = 16;
+
+// red[which][i][warp][n] (i < kBwdTS): which 0 = dB (adjoint pass), 1 = dC
+// (recompute pass). `mine` is this thread's slot, red + warp * N + lane; only
+// lanes below N store.
 template <int N>
-__device__ __forceinline__ void red_put(float* red, int which, int TS, int i, float v) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (lane < N) red[(((size_t)which * TS + i) * kWarps + warp) * N + lane] = v;
+__device__ __forceinline__ float* red_slot(float* red) {
+  return red + (threadIdx.x >> 5) * N + (threadIdx.x & 31);
+}
+template <int N>
+__device__ __forceinline__ void red_put(float* mine, int which, int i, float v) {
+  if ((threadIdx.x & 31) < N) mine[(which * kBwdTS + i) * kWarps * N] = v;
 }
 
 // Sums the 4 warps' rows and stores the CTA's channel-group partials of two
@@ -72,14 +81,18 @@ __device__ void red_flush(const BwdParams& p, const float* red, int tensB, int t
                           int64_t tstart, int TS) {
   __syncthreads();
   const Geo& g = p.g;
-  for (int j = threadIdx.x; j < 2 * TS * N; j += kCta) {
-    const int which = j / (TS * N), r = j - which * TS * N, i = r / N, n = r - i * N;
-    const float* src = red + (((size_t)which * TS + i) * kWarps) * N + n;
-    float s = src[0];
 #pragma unroll
-    for (int w = 1; w < kWarps; ++w) s += src[w * N];
-    const int tensor = which == 0 ? tensB : tensC;
-    p.part_tok[((((int64_t)tensor * g.Bt + b) * g.L + tstart + i) * g.G + blockIdx.x) * N + n] = s;
+  for (int j0 = 0; j0 < 2 * kBwdTS * N; j0 += kCta) {
+    const int j = j0 + threadIdx.x;
+    const int which = j / (kBwdTS * N), i = (j / N) % kBwdTS, n = j % N;
+    if (i < TS) {
+      const float* src = red + ((which * kBwdTS + i) * kWarps) * N + n;
+      float s = src[0];
+#pragma unroll
+      for (int w = 1; w < kWarps; ++w) s += src[w * N];
+      const int tensor = which == 0 ? tensB : tensC;
+      p.part_tok[((((int64_t)tensor * g.Bt + b) * g.L + tstart + i) * g.G + blockIdx.x) * N + n] = s;
+    }
   }
   __syncthreads();
 }
@@ -115,11 +128,12 @@ __device__ __forceinline__ void scan_state_swz(float2 (&h)[N / 2], const float2 
 //   g   a_next gbar_next entering the segment's last scanned token (in/out)
 //   dA  accumulated sum of dt * gbar * p (in/out)
 //   epi(i, dt, x, dy, sum_n gbar B, sum_n A2 gbar p) writes the per-token results.
-// Channel sums of dy*h (dC) and gbar*dt*x (dB) go to red[1] and red[0].
+// Channel sums of dy*h (dC) and gbar*dt*x (dB) go to red[1] and red[0]
+// through this thread's slot `mine`.
 template <int N, bool FWDDIR, typename St, typename Epi>
 __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, int jdy, int rB, int rC,
                                         const float2 (&A2)[N / 2], int sw, float2 (&h)[N / 2],
-                                        float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* red,
+                                        float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* mine,
                                         Epi epi) {
 #pragma unroll 2
   for (int k = 0; k < TS; ++k) {  // recompute, in scan order
@@ -136,7 +150,7 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
       w[j] = mul2(dy2, h[j]);
     }
     tmem_st2<N>(tb + (uint32_t)(i * N), pv);
-    red_put<N>(red, 1, TS, i, warp_reduce_swz<N>(w));
+    red_put<N>(mine, 1, i, warp_reduce_swz<N>(w));
   }
   tmem_wait_st();
 #pragma unroll 2
@@ -162,7 +176,7 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
       sg[j & 1] = fma2(gb, B[j], sg[j & 1]);
       w[j] = mul2(gb, u2);
     }
-    red_put<N>(red, 0, TS, i, warp_reduce_swz<N>(w));
+    red_put<N>(mine, 0, i, warp_reduce_swz<N>(w));
     const float2 sgs = add2(sg[0], sg[1]), sas = add2(sa[0], sa[1]);
     epi(i, dt, x, dy, __fadd_rn(sgs.x, sgs.y), __fadd_rn(sas.x, sas.y));
   }
@@ -176,11 +190,11 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
 template <typename T, int N>
 struct NoisyBwdSmem {
   // token-by-channel: x_n, dt_f, dt_r, dy_n, dt_c, dy_c; token-by-state: B_f, C_f, B_r, C_r, C_c
-  using St = Stage<T, N, 6, 5, 2>;
+  using St = Stage<T, N, 6, 5, 2, kBwdTS>;
   // two staging buffers when a block is a single segment (prefetch of the next block)
-  static __host__ __device__ size_t dx_off(int TS, int Bs) { return align16(St::buf_bytes(TS) * (Bs / TS == 1 ? 2 : 1)); }
+  static __host__ __device__ size_t dx_off(int TS, int Bs) { return align16(St::buf_bytes(kBwdTS) * (Bs / TS == 1 ? 2 : 1)); }
   static __host__ __device__ size_t red_off(int TS, int Bs) { return dx_off(TS, Bs) + (size_t)Bs * kCta * 4; }
-  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * TS * kWarps * N * 4; }
+  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kWarps * N * 4; }
   static __host__ __device__ size_t slot_off(int TS, int Bs) {
     const int nseg = Bs / TS;
     return ck_off(TS, Bs) + (size_t)(nseg > 1 ? nseg - 1 : 1) * N * kCta * 4;
@@ -219,6 +233,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   st.row_src[CC] = (const T*)p.Cc;
   float* dxbuf = reinterpret_cast<float*>(smem + L::dx_off(TS, Bs));
   float* red = reinterpret_cast<float*>(smem + L::red_off(TS, Bs));
+  float* mine = red_slot<N>(red);
   float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
 
@@ -308,7 +323,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
           vzero2<N>(h);
         else
           ck_load<N>(h, ck, s);
-        seg_bwd<N, false>(st, TS, XN, DTR, DYN, BR, CR, A2r, sw, h, gr, dAr, tb, red,
+        seg_bwd<N, false>(st, TS, XN, DTR, DYN, BR, CR, A2r, sw, h, gr, dAr, tb, mine,
                           [&](int i, float dt, float x, float dy, float sgB, float sAq) {
                             const int ib = s * TS + i;
                             if (act)
@@ -346,7 +361,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
         } else {
           ck_load<N>(h, ck, s - 1);
         }
-        seg_bwd<N, true>(st, TS, XN, DTF, DYN, BF, CF, A2f, sw, h, gf, dAf, tb, red,
+        seg_bwd<N, true>(st, TS, XN, DTF, DYN, BF, CF, A2f, sw, h, gf, dAf, tb, mine,
                          [&](int i, float dt, float x, float dy, float sgB, float sAq) {
                            const int ib = s * TS + i;
                            const int64_t o = (row0 + ib) * g.D + d;
@@ -425,9 +440,9 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
 // ---------------------------------------------------------------------------
 template <typename T, int N>
 struct CleanBwdSmem {
-  using St = Stage<T, N, 3, 2, 2>;  // x_c, dt_c, dy_c; B_c, C_c
-  static __host__ __device__ size_t red_off(int TS, int Bs) { return align16(St::buf_bytes(TS) * (Bs / TS == 1 ? 2 : 1)); }
-  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * TS * kWarps * N * 4; }
+  using St = Stage<T, N, 3, 2, 2, kBwdTS>;  // x_c, dt_c, dy_c; B_c, C_c
+  static __host__ __device__ size_t red_off(int TS, int Bs) { return align16(St::buf_bytes(kBwdTS) * (Bs / TS == 1 ? 2 : 1)); }
+  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kWarps * N * 4; }
   static __host__ __device__ size_t slot_off(int TS, int Bs) {
     const int nseg = Bs / TS;
     return ck_off(TS, Bs) + (size_t)(nseg > 1 ? nseg - 1 : 1) * N * kCta * 4;
@@ -459,6 +474,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
   st.row_src[BC] = (const T*)p.Bc;
   st.row_src[CC] = (const T*)p.Cc;
   float* red = reinterpret_cast<float*>(smem + L::red_off(TS, Bs));
+  float* mine = red_slot<N>(red);
   float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
 
@@ -529,7 +545,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
       } else {
         ck_load<N>(h, ck, s - 1);
       }
-      seg_bwd<N, true>(st, TS, XC, DTC, DYC, BC, CC, A2, sw, h, gc, dA, tb, red,
+      seg_bwd<N, true>(st, TS, XC, DTC, DYC, BC, CC, A2, sw, h, gc, dA, tb, mine,
                        [&](int i, float dt, float x, float dy, float sgB, float sAq) {
                          const int64_t o = (row0 + s * TS + i) * g.D + d;
                          if (act) {
@@ -639,11 +655,55 @@ inline size_t pad_for_tmem(size_t smem, int TS, int N) {
   return smem > need ? smem : need;
 }
 
+// Both attributes are set before every launch and before the occupancy query:
+// the padded shared memory exceeds the 48 KB default, and without the largest
+// carveout the driver may configure an SM for one such CTA instead of the two
+// its TMEM can hold.
+template <typename K>
+cudaError_t set_bwd_attrs(K kernel, size_t smem) {
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, (int)cudaSharedmemCarveoutMaxShared);
+}
+
+// Resident CTAs per SM of k_bwd_noisy at this block size (0 on failure),
+// from the per-SM limits: TMEM columns, registers (each of the four SM
+// sub-partitions holds whole warps, registers allocated per thread in
+// multiples of 8), shared memory with the per-CTA reserve, and threads. The
+// runtime's occupancy calculator reports one CTA for this kernel where the
+// hardware admits two, so it is not used.
+template <typename T, typename TO, int N>
+int bwd_noisy_per_sm(int Bs, int dev) {
+  const int TS = Bs < 16 ? Bs : 16;
+  const size_t smem = pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), TS, N);
+  cudaFuncAttributes fa;
+  int sm_smem = 0, sm_regs = 0, sm_threads = 0, reserve = 0;
+  if (set_bwd_attrs(k_bwd_noisy<T, TO, N>, smem) != cudaSuccess ||
+      cudaFuncGetAttributes(&fa, k_bwd_noisy<T, TO, N>) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sm_smem, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sm_regs, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sm_threads, cudaDevAttrMaxThreadsPerMultiProcessor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&reserve, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  const int by_tmem = (int)(512 / tcols_host(TS, N));
+  const int warp_regs = ((fa.numRegs + 7) / 8 * 8) * 32;
+  const int by_regs = warp_regs > 0 ? (sm_regs / 4 / warp_regs) * 4 / kWarps : 0;
+  const int by_smem = (int)((size_t)sm_smem / (smem + fa.sharedSizeBytes + (size_t)reserve));
+  const int by_threads = sm_threads / kCta;
+  int n = by_tmem;
+  n = by_regs < n ? by_regs : n;
+  n = by_smem < n ? by_smem : n;
+  n = by_threads < n ? by_threads : n;
+  return n;
+}
+
 template <typename T, typename TO, int N>
 cudaError_t bwd_noisy_t(const BwdParams& p, cudaStream_t s) {
   const int Bs = (int)p.g.Bs, TS = Bs < 16 ? Bs : 16;
   const size_t smem = pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), TS, N);
-  cudaError_t e = cudaFuncSetAttribute(k_bwd_noisy<T, TO, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = set_bwd_attrs(k_bwd_noisy<T, TO, N>, smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
   k_bwd_noisy<T, TO, N><<<grid, kCta, smem, s>>>(p);
@@ -654,7 +714,7 @@ template <typename T, typename TO, int N>
 cudaError_t bwd_clean_t(const BwdParams& p, cudaStream_t s) {
   const int Bs = (int)p.g.Bs, TS = Bs < 16 ? Bs : 16;
   const size_t smem = pad_for_tmem(CleanBwdSmem<T, N>::bytes(TS, Bs), TS, N);
-  cudaError_t e = cudaFuncSetAttribute(k_bwd_clean<T, TO, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = set_bwd_attrs(k_bwd_clean<T, TO, N>, smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
   k_bwd_clean<T, TO, N><<<grid, kCta, smem, s>>>(p);
@@ -709,30 +769,21 @@ cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s) {
 
 // Backward chunks per batch row: the count whose grid (channel groups x
 // chunks x batch) fills the resident CTA slots best, between 1 and
-// bwd_max_chunks(). Falls back to the forward chunking if the occupancy
-// query fails.
+// bwd_max_chunks(). Falls back to the forward chunking if the attribute
+// queries fail.
 int bwd_chunk_count(int dt, int N, const Geo& g) {
-  int dev = 0, sms = 0, per_sm = 0;
+  int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return g.nc;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) return g.nc;
-  const int Bs = (int)g.Bs, TS = Bs < 16 ? Bs : 16;
-  const size_t smem = pad_for_tmem(dt == 0 ? (N == 8 ? NoisyBwdSmem<float, 8>::bytes(TS, Bs) : NoisyBwdSmem<float, 16>::bytes(TS, Bs))
-                                           : (N == 8 ? NoisyBwdSmem<bf16, 8>::bytes(TS, Bs) : NoisyBwdSmem<bf16, 16>::bytes(TS, Bs)),
-                                   TS, N);
-  cudaError_t e = cudaErrorInvalidValue;
+  const int Bs = (int)g.Bs;
+  int per_sm = 0;
   if (dt == 0)
-    e = N == 8 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<float, float, 8>, kCta, smem)
-               : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<float, float, 16>, kCta, smem);
+    per_sm = N == 8 ? bwd_noisy_per_sm<float, float, 8>(Bs, dev) : bwd_noisy_per_sm<float, float, 16>(Bs, dev);
   else if (dt == 1)
-    e = N == 8 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, bf16, 8>, kCta, smem)
-               : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, bf16, 16>, kCta, smem);
+    per_sm = N == 8 ? bwd_noisy_per_sm<bf16, bf16, 8>(Bs, dev) : bwd_noisy_per_sm<bf16, bf16, 16>(Bs, dev);
   else
-    e = N == 8 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, float, 8>, kCta, smem)
-               : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_bwd_noisy<bf16, float, 16>, kCta, smem);
-  if (e != cudaSuccess || per_sm <= 0) {
-    cudaGetLastError();
-    return g.nc;
-  }
+    per_sm = N == 8 ? bwd_noisy_per_sm<bf16, float, 8>(Bs, dev) : bwd_noisy_per_sm<bf16, float, 16>(Bs, dev);
+  if (per_sm <= 0) return g.nc;
   const int64_t slots = (int64_t)per_sm * sms;
   const int64_t rows = g.Bt * g.G;
   const int cmax = bwd_max_chunks(g);

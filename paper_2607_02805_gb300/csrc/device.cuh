@@ -99,7 +99,9 @@ __device__ __forceinline__ void cp_async_wait_one() { asm volatile("cp.async.wai
 // A set of staged tensors for one span of up to `tsmax` tokens, in NBUF
 // shared-memory buffers. With two buffers the next span is copied while the
 // current one is processed: issue(next) ... complete(current, pending = 1).
-template <typename T, int N, int NTD, int NROW, int NBUF = 1>
+// TSMAX > 0 fixes the span stride at compile time (every staged address is
+// then a base plus an immediate); 0 takes it from carve().
+template <typename T, int N, int NTD, int NROW, int NBUF = 1, int TSMAX = 0>
 struct Stage {
   unsigned char* base;
   int tsmax;
@@ -116,22 +118,23 @@ struct Stage {
   static __host__ __device__ size_t buf_bytes(int ts) { return td_bytes(ts) + raw_bytes(ts) + rows_bytes(ts); }
   static __host__ __device__ size_t bytes(int ts) { return (size_t)NBUF * buf_bytes(ts); }
 
+  __device__ __forceinline__ int stride() const { return TSMAX > 0 ? TSMAX : tsmax; }
   __device__ void carve(unsigned char* b, int ts) {
     base = b;
-    tsmax = ts;
+    tsmax = TSMAX > 0 ? TSMAX : ts;
     select(0);
   }
   __device__ __forceinline__ void select(int buf) {
     cur_td = td(buf) + threadIdx.x;
     cur_rows = rows(buf);
   }
-  __device__ __forceinline__ T* td(int buf) const { return reinterpret_cast<T*>(base + (size_t)buf * buf_bytes(tsmax)); }
+  __device__ __forceinline__ T* td(int buf) const { return reinterpret_cast<T*>(base + (size_t)buf * buf_bytes(stride())); }
   __device__ __forceinline__ float* rows(int buf) const {
-    return reinterpret_cast<float*>(base + (size_t)buf * buf_bytes(tsmax) + td_bytes(tsmax) + raw_bytes(tsmax));
+    return reinterpret_cast<float*>(base + (size_t)buf * buf_bytes(stride()) + td_bytes(stride()) + raw_bytes(stride()));
   }
   __device__ __forceinline__ T* raw(int buf) const {
     return is_f32<T>::value ? reinterpret_cast<T*>(rows(buf))
-                            : reinterpret_cast<T*>(base + (size_t)buf * buf_bytes(tsmax) + td_bytes(tsmax));
+                            : reinterpret_cast<T*>(base + (size_t)buf * buf_bytes(stride()) + td_bytes(stride()));
   }
   // Starts the copies of tokens [row0, row0+nsteps) into buffer `buf` (one
   // cp.async group per thread). The caller guarantees no thread still reads it.
@@ -139,9 +142,9 @@ struct Stage {
     T* t = td(buf);
     T* r = raw(buf);
 #pragma unroll
-    for (int j = 0; j < NTD; ++j) issue_td<T>(t + (size_t)j * tsmax * kCta, td_src[j], row0, nsteps, D, d0);
+    for (int j = 0; j < NTD; ++j) issue_td<T>(t + (size_t)j * stride() * kCta, td_src[j], row0, nsteps, D, d0);
 #pragma unroll
-    for (int j = 0; j < NROW; ++j) issue_rows<T, N>(r + (size_t)j * tsmax * N, row_src[j], row0, nsteps);
+    for (int j = 0; j < NROW; ++j) issue_rows<T, N>(r + (size_t)j * stride() * N, row_src[j], row0, nsteps);
     cp_async_commit();
   }
   // Waits for the copies of buffer `buf` (with `pending` newer groups still in
@@ -153,12 +156,15 @@ struct Stage {
       cp_async_wait_all();
     __syncthreads();
     if (!is_f32<T>::value) {
-      const int per = nsteps * N;
+      const int half = nsteps * N / 2;  // element pairs per row
       const T* r = raw(buf);
       float* f = rows(buf);
-      for (int i = threadIdx.x; i < NROW * per; i += kCta) {
-        const int j = i / per, q = i - j * per;
-        f[(size_t)j * tsmax * N + q] = cvt(r[(size_t)j * tsmax * N + q]);
+#pragma unroll
+      for (int j = 0; j < NROW; ++j) {
+        const T* rj = r + (size_t)j * stride() * N;
+        float* fj = f + (size_t)j * stride() * N;
+        for (int q = threadIdx.x; q < half; q += kCta)
+          reinterpret_cast<float2*>(fj)[q] = make_float2(cvt(rj[2 * q]), cvt(rj[2 * q + 1]));
       }
       __syncthreads();
     }
@@ -172,10 +178,10 @@ struct Stage {
     complete(0, nsteps, 0);
   }
   __device__ __forceinline__ float at(int j, int step) const {
-    return cvt(cur_td[(j * tsmax + step) * kCta]);
+    return cvt(cur_td[(j * stride() + step) * kCta]);
   }
   __device__ __forceinline__ const float* row(int j, int step) const {
-    return cur_rows + (j * tsmax + step) * N;
+    return cur_rows + (j * stride() + step) * N;
   }
 };
 
