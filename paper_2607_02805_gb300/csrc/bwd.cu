@@ -104,11 +104,15 @@ __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t
 // full); chunk c holds blocks [chunk_lo(c), chunk_lo(c+1)).
 __host__ __device__ inline int chunk_lo(const Geo& g, int c) { return (int)(((int64_t)c * g.nb) / g.nc); }
 
-__host__ __device__ inline uint32_t tcols_host(int TS, int N) {
-  uint32_t need = (uint32_t)(TS * N), c = 32;
+__host__ __device__ inline uint32_t pow2_cols(uint32_t need) {
+  uint32_t c = 32;
   while (c < need) c <<= 1;
   return c;
 }
+// TMEM columns of one segment's held values: every state (noisy kernel) or
+// every other one (clean kernel).
+__host__ __device__ inline uint32_t full_cols(int TS, int N) { return pow2_cols((uint32_t)(TS * N)); }
+__host__ __device__ inline uint32_t half_cols(int TS, int N) { return pow2_cols((uint32_t)(((TS + 1) / 2) * N)); }
 
 // The state update alone on a group-swizzled packed state (checkpoint passes).
 template <int N>
@@ -182,6 +186,99 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
   }
 }
 
+// seg_bwd holding half of the states, for the clean kernel: its smaller TMEM
+// footprint lets three CTAs share an SM. Arguments as for seg_bwd, except
+//   tb   TMEM, (TS+1)/2 slots of N columns: the state entering every even
+//        scan step.
+// The adjoint takes the steps two at a time from the end. For steps k and
+// k-1 it reloads the state entering k-1 and redoes step k-1 to get the state
+// entering k, with the operations of the recompute (so the same bits); the
+// decay a_{k-1} that this needs is the one the adjoint of step k-1 uses.
+template <int N, bool FWDDIR, typename St, typename Epi>
+__device__ __forceinline__ void seg_bwd_half(const St& st, int TS, int jx, int jdt, int jdy, int rB, int rC,
+                                             const float2 (&A2)[N / 2], int sw, float2 (&h)[N / 2],
+                                             float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* mine,
+                                             Epi epi) {
+#pragma unroll 2
+  for (int k = 0; k < TS; ++k) {  // recompute, in scan order
+    const int i = FWDDIR ? k : TS - 1 - k;
+    if ((k & 1) == 0) tmem_st2<N>(tb + (uint32_t)((k >> 1) * N), h);
+    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
+    float2 B[N / 2], w[N / 2];
+    vload2<N>(B, st.row(rB, i), sw);
+#pragma unroll
+    for (int j = 0; j < N / 2; ++j) {
+      const float2 a = ex2x2(mul2(dt2, A2[j]));
+      h[j] = fma2(u2, B[j], mul2(a, h[j]));
+      w[j] = mul2(dy2, h[j]);
+    }
+    red_put<N>(mine, 1, i, warp_reduce_swz<N>(w));
+  }
+  tmem_wait_st();
+
+  // one adjoint step at token i, given a = a_i and pv = a_i * (state entering i)
+  auto step = [&](int i, const float2 (&a)[N / 2], const float2 (&pv)[N / 2]) {
+    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
+    float2 B[N / 2], C[N / 2], w[N / 2];
+    vload2<N>(B, st.row(rB, i), sw);
+    vload2<N>(C, st.row(rC, i), sw);
+    float2 sg[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    float2 sa[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+    for (int j = 0; j < N / 2; ++j) {
+      const float2 gb = fma2(C[j], dy2, g[j]);
+      g[j] = mul2(a[j], gb);
+      const float2 q = mul2(gb, pv[j]);
+      sa[j & 1] = fma2(A2[j], q, sa[j & 1]);
+      dA[j] = fma2(dt2, q, dA[j]);
+      sg[j & 1] = fma2(gb, B[j], sg[j & 1]);
+      w[j] = mul2(gb, u2);
+    }
+    red_put<N>(mine, 0, i, warp_reduce_swz<N>(w));
+    const float2 sgs = add2(sg[0], sg[1]), sas = add2(sa[0], sa[1]);
+    epi(i, dt, x, dy, __fadd_rn(sgs.x, sgs.y), __fadd_rn(sas.x, sas.y));
+  };
+
+  int k = TS - 1;
+  if ((TS & 1) != 0) {  // an odd count: the last step alone, its entering state is held
+    const int i = FWDDIR ? k : TS - 1 - k;
+    float2 S[N / 2], a[N / 2], pv[N / 2];
+    tmem_ld2<N>(tb + (uint32_t)((k >> 1) * N), S);
+    const float2 dt2 = f2(st.at(jdt, i));
+#pragma unroll
+    for (int j = 0; j < N / 2; ++j) {
+      a[j] = ex2x2(mul2(dt2, A2[j]));
+      pv[j] = mul2(a[j], S[j]);
+    }
+    step(i, a, pv);
+    --k;
+  }
+#pragma unroll 1
+  for (; k > 0; k -= 2) {  // steps k (odd) and k-1
+    const int i0 = FWDDIR ? k : TS - 1 - k, i1 = FWDDIR ? k - 1 : TS - k;
+    float2 S[N / 2], a0[N / 2], pv0[N / 2], a1[N / 2], pv1[N / 2];
+    tmem_ld2<N>(tb + (uint32_t)(((k - 1) >> 1) * N), S);  // state entering step k-1
+    {
+      const float dt1 = st.at(jdt, i1), x1 = st.at(jx, i1);
+      const float2 dt12 = f2(dt1), u12 = f2(__fmul_rn(dt1, x1)), dt02 = f2(st.at(jdt, i0));
+      float2 B1[N / 2];
+      vload2<N>(B1, st.row(rB, i1), sw);
+#pragma unroll
+      for (int j = 0; j < N / 2; ++j) {
+        a1[j] = ex2x2(mul2(dt12, A2[j]));
+        pv1[j] = mul2(a1[j], S[j]);
+        const float2 hk = fma2(u12, B1[j], pv1[j]);  // state entering step k
+        a0[j] = ex2x2(mul2(dt02, A2[j]));
+        pv0[j] = mul2(a0[j], hk);
+      }
+    }
+    step(i0, a0, pv0);
+    step(i1, a1, pv1);
+  }
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -237,7 +334,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
 
-  const uint32_t tcols = tmem_cols_for((uint32_t)(TS * N));
+  const uint32_t tcols = full_cols(TS, N);
   if (warp == 0) tmem_alloc(tslot, tcols);
   tmem_sync();
   const uint32_t tbase = *tslot;
@@ -445,13 +542,13 @@ struct CleanBwdSmem {
   static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kWarps * N * 4; }
   static __host__ __device__ size_t slot_off(int TS, int Bs) {
     const int nseg = Bs / TS;
-    return ck_off(TS, Bs) + (size_t)(nseg > 1 ? nseg - 1 : 1) * N * kCta * 4;
+    return ck_off(TS, Bs) + (size_t)(nseg - 1) * N * kCta * 4;
   }
   static __host__ __device__ size_t bytes(int TS, int Bs) { return slot_off(TS, Bs) + 16; }
 };
 
 template <typename T, typename TO, int N>
-__global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
+__global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   extern __shared__ __align__(16) unsigned char smem[];
   using L = CleanBwdSmem<T, N>;
   const Geo& g = p.g;
@@ -478,7 +575,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
   float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
 
-  const uint32_t tcols = tmem_cols_for((uint32_t)(TS * N));
+  const uint32_t tcols = half_cols(TS, N);  // held states of a segment
   if (warp == 0) tmem_alloc(tslot, tcols);
   tmem_sync();
   const uint32_t tbase = *tslot;
@@ -545,7 +642,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_clean(const BwdParams p) {
       } else {
         ck_load<N>(h, ck, s - 1);
       }
-      seg_bwd<N, true>(st, TS, XC, DTC, DYC, BC, CC, A2, sw, h, gc, dA, tb, mine,
+      seg_bwd_half<N, true>(st, TS, XC, DTC, DYC, BC, CC, A2, sw, h, gc, dA, tb, mine,
                        [&](int i, float dt, float x, float dy, float sgB, float sAq) {
                          const int64_t o = (row0 + s * TS + i) * g.D + d;
                          if (act) {
@@ -646,8 +743,7 @@ namespace {
 
 // Dynamic shared memory is padded so that no more CTAs share an SM than its
 // 512 TMEM columns can hold at once.
-inline size_t pad_for_tmem(size_t smem, int TS, int N) {
-  const uint32_t cols = tcols_host(TS, N);
+inline size_t pad_for_tmem(size_t smem, uint32_t cols) {
   const int ctas = (int)(512 / cols);
   if (ctas >= 16) return smem;  // the thread limit already bounds residency
   const size_t cap = (size_t)(220 * 1024) / (size_t)ctas;
@@ -666,20 +762,17 @@ cudaError_t set_bwd_attrs(K kernel, size_t smem) {
   return cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, (int)cudaSharedmemCarveoutMaxShared);
 }
 
-// Resident CTAs per SM of k_bwd_noisy at this block size (0 on failure),
-// from the per-SM limits: TMEM columns, registers (each of the four SM
-// sub-partitions holds whole warps, registers allocated per thread in
-// multiples of 8), shared memory with the per-CTA reserve, and threads. The
-// runtime's occupancy calculator reports one CTA for this kernel where the
-// hardware admits two, so it is not used.
-template <typename T, typename TO, int N>
-int bwd_noisy_per_sm(int Bs, int dev) {
-  const int TS = Bs < 16 ? Bs : 16;
-  const size_t smem = pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), TS, N);
+// Resident CTAs per SM of a backward kernel (0 on failure), from the per-SM
+// limits: TMEM columns, registers (each of the four SM sub-partitions holds
+// whole warps, registers allocated per thread in multiples of 8), shared
+// memory with the per-CTA reserve, and threads. The runtime's occupancy
+// calculator reports one CTA for the noisy kernel where the hardware admits
+// two, so it is not used.
+template <typename K>
+int resident_ctas(K kernel, size_t smem, uint32_t tcols, int dev) {
   cudaFuncAttributes fa;
   int sm_smem = 0, sm_regs = 0, sm_threads = 0, reserve = 0;
-  if (set_bwd_attrs(k_bwd_noisy<T, TO, N>, smem) != cudaSuccess ||
-      cudaFuncGetAttributes(&fa, k_bwd_noisy<T, TO, N>) != cudaSuccess ||
+  if (set_bwd_attrs(kernel, smem) != cudaSuccess || cudaFuncGetAttributes(&fa, kernel) != cudaSuccess ||
       cudaDeviceGetAttribute(&sm_smem, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sm_regs, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sm_threads, cudaDevAttrMaxThreadsPerMultiProcessor, dev) != cudaSuccess ||
@@ -687,7 +780,7 @@ int bwd_noisy_per_sm(int Bs, int dev) {
     cudaGetLastError();
     return 0;
   }
-  const int by_tmem = (int)(512 / tcols_host(TS, N));
+  const int by_tmem = (int)(512 / tcols);
   const int warp_regs = ((fa.numRegs + 7) / 8 * 8) * 32;
   const int by_regs = warp_regs > 0 ? (sm_regs / 4 / warp_regs) * 4 / kWarps : 0;
   const int by_smem = (int)((size_t)sm_smem / (smem + fa.sharedSizeBytes + (size_t)reserve));
@@ -700,9 +793,18 @@ int bwd_noisy_per_sm(int Bs, int dev) {
 }
 
 template <typename T, typename TO, int N>
+void bwd_per_sm(int Bs, int dev, int& noisy, int& clean) {
+  const int TS = Bs < 16 ? Bs : 16;
+  noisy = resident_ctas(k_bwd_noisy<T, TO, N>, pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), full_cols(TS, N)),
+                        full_cols(TS, N), dev);
+  clean = resident_ctas(k_bwd_clean<T, TO, N>, pad_for_tmem(CleanBwdSmem<T, N>::bytes(TS, Bs), half_cols(TS, N)),
+                        half_cols(TS, N), dev);
+}
+
+template <typename T, typename TO, int N>
 cudaError_t bwd_noisy_t(const BwdParams& p, cudaStream_t s) {
   const int Bs = (int)p.g.Bs, TS = Bs < 16 ? Bs : 16;
-  const size_t smem = pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), TS, N);
+  const size_t smem = pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), full_cols(TS, N));
   cudaError_t e = set_bwd_attrs(k_bwd_noisy<T, TO, N>, smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
@@ -713,7 +815,7 @@ cudaError_t bwd_noisy_t(const BwdParams& p, cudaStream_t s) {
 template <typename T, typename TO, int N>
 cudaError_t bwd_clean_t(const BwdParams& p, cudaStream_t s) {
   const int Bs = (int)p.g.Bs, TS = Bs < 16 ? Bs : 16;
-  const size_t smem = pad_for_tmem(CleanBwdSmem<T, N>::bytes(TS, Bs), TS, N);
+  const size_t smem = pad_for_tmem(CleanBwdSmem<T, N>::bytes(TS, Bs), half_cols(TS, N));
   cudaError_t e = set_bwd_attrs(k_bwd_clean<T, TO, N>, smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
@@ -767,32 +869,38 @@ cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s) {
   BDS_DISPATCH_N(N, k_reduce_par<NN><<<(unsigned)((npar + 31) / 32), 256, 0, s>>>(p); return cudaGetLastError();)
 }
 
-// Backward chunks per batch row: the count whose grid (channel groups x
-// chunks x batch) fills the resident CTA slots best, between 1 and
-// bwd_max_chunks(). Falls back to the forward chunking if the attribute
-// queries fail.
+// Backward chunks per batch row, between 1 and bwd_max_chunks(); both
+// backward kernels use the same chunks. For each count, each kernel's time is
+// modelled as (waves of CTAs over its resident slots) x (blocks in the longest
+// chunk + a set-up of a quarter block) x (its work per block) x (CTAs sharing
+// an SM): per token the noisy kernel makes five scan passes and four channel
+// reductions, the clean kernel two and two. The count with the least modelled
+// sum is taken. Falls back to the forward chunking if the attribute queries
+// fail.
 int bwd_chunk_count(int dt, int N, const Geo& g) {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return g.nc;
   if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) return g.nc;
   const int Bs = (int)g.Bs;
-  int per_sm = 0;
-  if (dt == 0)
-    per_sm = N == 8 ? bwd_noisy_per_sm<float, float, 8>(Bs, dev) : bwd_noisy_per_sm<float, float, 16>(Bs, dev);
-  else if (dt == 1)
-    per_sm = N == 8 ? bwd_noisy_per_sm<bf16, bf16, 8>(Bs, dev) : bwd_noisy_per_sm<bf16, bf16, 16>(Bs, dev);
-  else
-    per_sm = N == 8 ? bwd_noisy_per_sm<bf16, float, 8>(Bs, dev) : bwd_noisy_per_sm<bf16, float, 16>(Bs, dev);
-  if (per_sm <= 0) return g.nc;
-  const int64_t slots = (int64_t)per_sm * sms;
+  int pn = 0, pc = 0;
+  if (dt == 0) {
+    if (N == 8) bwd_per_sm<float, float, 8>(Bs, dev, pn, pc); else bwd_per_sm<float, float, 16>(Bs, dev, pn, pc);
+  } else if (dt == 1) {
+    if (N == 8) bwd_per_sm<bf16, bf16, 8>(Bs, dev, pn, pc); else bwd_per_sm<bf16, bf16, 16>(Bs, dev, pn, pc);
+  } else {
+    if (N == 8) bwd_per_sm<bf16, float, 8>(Bs, dev, pn, pc); else bwd_per_sm<bf16, float, 16>(Bs, dev, pn, pc);
+  }
+  if (pn <= 0 || pc <= 0) return g.nc;
+  constexpr double kNoisyWork = 9.0, kCleanWork = 4.0;  // scan passes + reductions per token
   const int64_t rows = g.Bt * g.G;
   const int cmax = bwd_max_chunks(g);
   int best = g.nc;
   double best_cost = 1e300;
   for (int nc = 1; nc <= cmax; ++nc) {
-    const int64_t waves = (rows * nc + slots - 1) / slots;
-    const int64_t blocks = (g.nb + nc - 1) / nc;  // longest chunk
-    const double cost = (double)waves * ((double)blocks + 0.25);  // + per-CTA set-up, in blocks
+    const double blocks = (double)((g.nb + nc - 1) / nc) + 0.25;  // longest chunk + set-up
+    const double wn = (double)((rows * nc + (int64_t)pn * sms - 1) / ((int64_t)pn * sms));
+    const double wc = (double)((rows * nc + (int64_t)pc * sms - 1) / ((int64_t)pc * sms));
+    const double cost = blocks * (wn * kNoisyWork * pn + wc * kCleanWork * pc);
     if (cost < best_cost - 1e-9) {
       best_cost = cost;
       best = nc;
