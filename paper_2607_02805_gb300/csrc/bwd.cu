@@ -502,6 +502,15 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
   const int n = (int)(idx % N);
   const int64_t d = (idx / N) % g.D, b = idx / ((int64_t)N * g.D);
   const float A2 = __fmul_rn(p.Af[d * N + n], kLog2e);
+  const float* dS = p.dS + (b * g.nb * g.D + d) * N + n;  // block k at [k * D * N]
+  const float* ext = p.dstates != nullptr ? p.dstates + (b * g.nb * g.D + d) * N + n : nullptr;
+  float* Lc = p.Lc + (b * g.nc * g.D + d) * N + n;        // chunk c at [c * D * N]
+  const float* sdtc = p.sdtc + b * g.nc * g.D + d;         // chunk c at [c * D]
+  const int64_t DN = g.D * N;
+  // chunk_lo(c) = floor(c nb / nc), stepped down from c = nc by quotient and
+  // remainder (no division per chunk)
+  const int q0 = (int)(g.nb / g.nc), r0 = (int)(g.nb % g.nc);
+  int lo = (int)g.nb, rem = 0;  // chunk_lo(c0 + 1) and its remainder
   float G = 0.f;  // a_{t+1} gbar_{t+1} entering the current chunk's last token from the right
   constexpr int U = 8;
   for (int c0 = g.nc - 1; c0 >= 0; c0 -= U) {
@@ -510,23 +519,27 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
 #pragma unroll
     for (int j = 0; j < U; ++j) {
       const int c = c0 - j;
-      inj[j] = 0.f;
-      loc[j] = 0.f;
-      sd[j] = 0.f;
-      if (c >= 0) {
-        const int kl = chunk_lo(g, c + 1) - 1;
-        if (kl + 1 < g.nb) inj[j] = p.dS[((b * g.nb + kl) * g.D + d) * N + n];
-        if (p.dstates != nullptr) inj[j] = __fadd_rn(inj[j], p.dstates[((b * g.nb + kl) * g.D + d) * N + n]);
-        loc[j] = p.Lc[((b * g.nc + c) * g.D + d) * N + n];
-        sd[j] = p.sdtc[(b * g.nc + c) * g.D + d];
+      const int kl = lo - 1;  // last block of chunk c
+      lo -= q0;
+      rem -= r0;
+      if (rem < 0) {
+        rem += (int)g.nc;
+        lo -= 1;
       }
+      const int cc = c >= 0 ? c : 0;
+      const int64_t kk = c >= 0 ? kl : 0;
+      const float vS = dS[kk * DN], vE = ext != nullptr ? ext[kk * DN] : 0.f;
+      inj[j] = c >= 0 && kl + 1 < g.nb ? vS : 0.f;
+      if (ext != nullptr) inj[j] = __fadd_rn(inj[j], c >= 0 ? vE : 0.f);
+      loc[j] = Lc[cc * DN];
+      sd[j] = sdtc[(int64_t)cc * g.D];
     }
 #pragma unroll
     for (int j = 0; j < U; ++j) {
       const int c = c0 - j;
       if (c < 0) break;
       const float gin = __fadd_rn(G, inj[j]);
-      p.Lc[((b * g.nc + c) * g.D + d) * N + n] = gin;
+      Lc[c * DN] = gin;
       G = __fmaf_rn(ex2(__fmul_rn(A2, sd[j])), gin, loc[j]);
     }
   }
@@ -688,29 +701,37 @@ __global__ void __launch_bounds__(256) k_reduce_tok(const BwdParams p) {
 // each add every 8th chunk (in order), then the slices are added in order.
 template <int N>
 __global__ void __launch_bounds__(256) k_reduce_par(const BwdParams p) {
-  __shared__ float part[5][8][32];
+  // 8 slices (warps) of the chunk partials; each lane sums 4 adjacent columns
+  __shared__ float4 part[3][8][32];
   const Geo& g = p.g;
   const int64_t U = g.Bt * g.nc;
   const int64_t DN = g.D * N;
   const int lane = threadIdx.x & 31, slice = threadIdx.x >> 5;
-  const int64_t col = (int64_t)blockIdx.x * 32 + lane;
-  float s0 = 0.f, s1 = 0.f, s2 = 0.f;
+  const int64_t col = ((int64_t)blockIdx.x * 32 + lane) * 4;  // D and D*N are multiples of 4
+  float4 s0 = make_float4(0.f, 0.f, 0.f, 0.f), s1 = s0, s2 = s0;
+  auto acc = [](float4& s, const float* src) {
+    const float4 v = *reinterpret_cast<const float4*>(src);
+    s.x += v.x;
+    s.y += v.y;
+    s.z += v.z;
+    s.w += v.w;
+  };
   if (col < DN) {
     const float* a0 = p.part_A + col;
     const float* a1 = p.part_A + U * DN + col;
     const float* a2 = p.part_A + 2 * U * DN + col;
 #pragma unroll 4
     for (int64_t u = slice; u < U; u += 8) {
-      s0 += a0[u * DN];
-      s1 += a1[u * DN];
-      s2 += a2[u * DN];
+      acc(s0, a0 + u * DN);
+      acc(s1, a1 + u * DN);
+      acc(s2, a2 + u * DN);
     }
   } else if (col < DN + g.D) {
     const int64_t d = col - DN;
 #pragma unroll 4
     for (int64_t u = slice; u < U; u += 8) {
-      s0 += p.part_D[u * g.D + d];
-      s1 += p.part_D[(U + u) * g.D + d];
+      acc(s0, p.part_D + u * g.D + d);
+      acc(s1, p.part_D + (U + u) * g.D + d);
     }
   }
   part[0][slice][lane] = s0;
@@ -718,20 +739,22 @@ __global__ void __launch_bounds__(256) k_reduce_par(const BwdParams p) {
   part[2][slice][lane] = s2;
   __syncthreads();
   if (slice == 0) {
-    float t0 = part[0][0][lane], t1 = part[1][0][lane], t2 = part[2][0][lane];
+    float4 t0 = part[0][0][lane], t1 = part[1][0][lane], t2 = part[2][0][lane];
 #pragma unroll
     for (int k = 1; k < 8; ++k) {
-      t0 += part[0][k][lane];
-      t1 += part[1][k][lane];
-      t2 += part[2][k][lane];
+      const float4 v0 = part[0][k][lane], v1 = part[1][k][lane], v2 = part[2][k][lane];
+      t0 = make_float4(t0.x + v0.x, t0.y + v0.y, t0.z + v0.z, t0.w + v0.w);
+      t1 = make_float4(t1.x + v1.x, t1.y + v1.y, t1.z + v1.z, t1.w + v1.w);
+      t2 = make_float4(t2.x + v2.x, t2.y + v2.y, t2.z + v2.z, t2.w + v2.w);
     }
     if (col < DN) {
-      p.dAf[col] = t0 + t2;  // noisy forward direction + clean stream
-      p.dAr[col] = t1;
+      // noisy forward direction + clean stream
+      *reinterpret_cast<float4*>(p.dAf + col) = make_float4(t0.x + t2.x, t0.y + t2.y, t0.z + t2.z, t0.w + t2.w);
+      *reinterpret_cast<float4*>(p.dAr + col) = t1;
     } else if (col < DN + g.D) {
       const int64_t d = col - DN;
-      p.dDf[d] = t0 + t1;  // noisy + clean
-      p.dDr[d] = t0;
+      *reinterpret_cast<float4*>(p.dDf + d) = make_float4(t0.x + t1.x, t0.y + t1.y, t0.z + t1.z, t0.w + t1.w);  // noisy + clean
+      *reinterpret_cast<float4*>(p.dDr + d) = t0;
     }
   }
 }
@@ -865,8 +888,8 @@ cudaError_t launch_bwd_reduce_tok(int dt, int N, const BwdParams& p, cudaStream_
 }
 
 cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s) {
-  const int64_t npar = p.g.D * N + p.g.D;
-  BDS_DISPATCH_N(N, k_reduce_par<NN><<<(unsigned)((npar + 31) / 32), 256, 0, s>>>(p); return cudaGetLastError();)
+  const int64_t npar4 = (p.g.D * N + p.g.D) / 4;  // float4 columns
+  BDS_DISPATCH_N(N, k_reduce_par<NN><<<(unsigned)((npar4 + 31) / 32), 256, 0, s>>>(p); return cudaGetLastError();)
 }
 
 // Backward chunks per batch row, between 1 and bwd_max_chunks(); both
