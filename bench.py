@@ -7,6 +7,14 @@ of 2048 tokens, block 16, d_inner 1536, d_state 16, bf16 inputs/outputs with
 fp32 state. Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py --workload sweep|prefill65k|prefill262k   (one GPU; extra lines)
+
+The extra workloads print one JSON line per measurement instead of the
+step line: the block-size sweep at d_inner 2048 (forward+backward for block
+4, 8, 16, 32, 64), and the inference cache path: boundary_states over a
+65,536-token prefix (block 32) or a 262,144-token prefix (block 16), then
+active-block calls from the cached state, each call timed on its own and all
+calls replayed as one CUDA graph.
 
 Under torchrun each rank runs an independent replica on its own GPU (the
 scan needs no exchange between replicas); the elapsed time is the maximum
@@ -350,6 +358,180 @@ def run_ours(args, rank, world, local_rank):
     print(json.dumps(line), flush=True)
 
 
+def time_layer_steps(lay, stream, steps, warmup):
+    """Average ms of one forward+backward step and per-kernel averages (us)."""
+    import torch
+    from paper_2607_02805_gb300 import binding
+    nk = len(KERNELS)
+    for _ in range(warmup):
+        lay.forward(stream)
+        lay.backward(stream, use_dstates=False)
+    ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ev_k = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(steps)]
+    for evs in ev_k:
+        for e in evs:
+            e.record(stream)
+    torch.cuda.synchronize()
+    arr_f = [(ctypes.c_void_p * 3)(*[e.cuda_event for e in evs[:3]]) for evs in ev_k]
+    arr_b = [(ctypes.c_void_p * (nk - 3))(*[e.cuda_event for e in evs[3:]]) for evs in ev_k]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(steps):
+        ev_s[i].record(stream)
+        binding.bdscan_profile_events(arr_f[i], 3)
+        lay.forward(stream)
+        binding.bdscan_profile_events(arr_b[i], nk - 3)
+        lay.backward(stream, use_dstates=False)
+        binding.bdscan_profile_events(None, 0)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    per = [[] for _ in range(nk)]
+    for i in range(steps):
+        prev = ev_s[i]
+        for j in range(nk):
+            per[j].append(prev.elapsed_time(ev_k[i][j]))
+            prev = ev_k[i][j]
+    return e0.elapsed_time(e1) / steps, {k: round(1e3 * statistics.mean(v), 2) for k, v in zip(KERNELS, per)}
+
+
+def run_sweep(args):
+    """Forward+backward at batch 8, 2048 tokens, d_inner 2048, d_state 16 for
+    each block size (the 350M-scale layer), one line per block size."""
+    import torch
+    from paper_2607_02805_gb300.inputs import Workload
+    from paper_2607_02805_gb300.layer import Layer
+    peaks, peak_kind = measured_peaks()
+    Bt, L, D, N = 8, 2048, 2048, 16
+    for Bs in (4, 8, 16, 32, 64):
+        wl = Workload(Bt, L, Bs, D, N, dtype="bf16", seed=1, with_grads=True)
+        lay = Layer(wl)
+        lay.alloc_backward()
+        stream = torch.cuda.current_stream()
+        ms, kern = time_layer_steps(lay, stream, args.steps, max(3, args.warmup))
+        fb, bb = algorithmic_bytes(Bt, L, D, N, Bs)
+        gbs = (fb + bb) / (ms * 1e-3) / 1e9
+        print(json.dumps({
+            "metric": METRIC, "value": Bt * L / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": args.steps,
+            "ms_per_step": ms, "higher_is_better": True, "dtype": "f32 state, bf16 I/O", "data": "synthetic",
+            "config": {"workload": f"350M-scale layer block sweep: batch 8, 2048 tokens per stream, block {Bs}, "
+                                   "d_inner 2048, d_state 16; all-block forward + backward",
+                       "batch": Bt, "seq_len": L, "block": Bs, "d_inner": D, "d_state": N},
+            "hbm": {"achieved": round(gbs, 1), "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
+                    "frac": round(gbs / float(peaks.get("hbm_gbs", 6800.0)), 4), "alg_bytes_per_step": fb + bb,
+                    "peak_kind": peak_kind},
+            "kernels_us": kern}), flush=True)
+        del lay
+        torch.cuda.empty_cache()
+
+
+def run_prefill(args, L, Bs, calls):
+    """Inference cache path at d_inner 2048, d_state 16, batch 1: the cache
+    build over an L-token clean prefix (final state only, and every block-end
+    state plus the clean outputs), then `calls` active-block calls from the
+    cached state, each timed on its own and all replayed as one CUDA graph."""
+    import torch
+    from paper_2607_02805_gb300 import binding
+    from paper_2607_02805_gb300.inputs import Workload
+    from paper_2607_02805_gb300.layer import to_device
+    peaks, peak_kind = measured_peaks()
+    D, N = 2048, 16
+    code = binding.BDSCAN_BF16
+    wl = Workload(1, L, Bs, D, N, dtype="bf16", seed=5, with_grads=False, parts=("clean",))
+    t = {k: to_device(wl.dev_bits(k), code, "cuda") for k in wl.t32}
+    dims = binding.make_dims(1, L, Bs, D, N, code)
+    stream = torch.cuda.current_stream()
+    nb = L // Bs
+    fin = torch.empty((1, 1, D, N), dtype=torch.float32, device="cuda")
+    allst = torch.empty((1, nb, D, N), dtype=torch.float32, device="cuda")
+    y_c = torch.empty((1, L, D), dtype=torch.bfloat16, device="cuda")
+    ws = {}
+    for emit_all in (0, 1):
+        nbytes = binding.bdscan_boundary_states_workspace_size(dims, emit_all)
+        ws[emit_all] = torch.empty(max(1, (nbytes + 3) // 4), dtype=torch.float32, device="cuda")
+    read_b = L * (2 * D * 2 + 2 * N * 2)  # x, dt [L, D] and B, C [L, N], bf16
+    modes = [("final state only", 0, None, fin, 0),
+             ("every block-end state and the clean outputs", 1, y_c, allst, nb * D * N * 4 + L * D * 2)]
+    for name, emit_all, y, st, extra_b in modes:
+        def one():
+            binding.boundary_states(dims, t, None, y, st, emit_all, ws[emit_all], stream)
+        for _ in range(max(3, args.warmup)):
+            one()
+        reps = max(3, min(args.steps, 20))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            one()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        gbs = (read_b + extra_b) / (ms * 1e-3) / 1e9
+        print(json.dumps({
+            "metric": "cache build (bdscan_boundary_states) prefix tokens/s", "value": L / (ms * 1e-3),
+            "unit": "tokens/s", "n_gpus": 1, "steps": reps, "ms_per_call": ms, "higher_is_better": True,
+            "dtype": "f32 state, bf16 I/O", "data": "synthetic",
+            "config": {"workload": f"cache build over a {L}-token prefix, block {Bs}, d_inner 2048, d_state 16, "
+                                   f"batch 1, bf16; emits {name}",
+                       "batch": 1, "seq_len": L, "block": Bs, "d_inner": D, "d_state": N, "emit_all": emit_all},
+            "hbm": {"achieved": round(gbs, 1), "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
+                    "frac": round(gbs / float(peaks.get("hbm_gbs", 6800.0)), 4),
+                    "alg_bytes_per_call": read_b + extra_b, "peak_kind": peak_kind}}), flush=True)
+    # active blocks from the cached final state (read-only seed)
+    binding.boundary_states(dims, t, None, None, fin, 0, ws[0], stream)
+    blocks = []
+    for j in range(calls):
+        blk = Workload(1, Bs, Bs, D, N, dtype="bf16", seed=5, with_grads=False, parts=("noisy",), part=j + 1)
+        tb = {k: to_device(blk.dev_bits(k), code, "cuda") for k in blk.t32}
+        blocks.append((tb, torch.empty((1, Bs, D), dtype=torch.bfloat16, device="cuda")))
+    bdims = binding.make_dims(1, Bs, Bs, D, N, code)
+    seed = fin[:, 0].contiguous()
+
+    def call(j, s):
+        binding.active_block(bdims, seed, blocks[j][0], blocks[j][1], s)
+
+    for j in range(calls):
+        call(j, stream)
+    torch.cuda.synchronize()
+    per_call = []
+    for j in range(calls):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        call(j, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        per_call.append(1e3 * e0.elapsed_time(e1))
+    graph_us = None
+    try:
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.graph(g, stream=side):
+            for j in range(calls):
+                call(j, side)
+        torch.cuda.synchronize()
+        g.replay()
+        torch.cuda.synchronize()
+        reps = 20
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        graph_us = 1e3 * e0.elapsed_time(e1) / (reps * calls)
+    except Exception as exc:  # report the failure in the line, keep the rest
+        graph_us = f"capture failed: {exc}"
+    blk_bytes = Bs * (D * 2 + 2 * D * 2 + 4 * N * 2 + D * 2) + D * N * 4
+    print(json.dumps({
+        "metric": "active-block call latency (bdscan_active_block)", "value": statistics.median(per_call),
+        "unit": "us per call", "n_gpus": 1, "higher_is_better": False, "dtype": "f32 state, bf16 I/O",
+        "data": "synthetic",
+        "config": {"workload": f"active block of {Bs} tokens from the cached state of a {L}-token prefix, "
+                               "d_inner 2048, d_state 16, batch 1, bf16", "calls": calls},
+        "per_call_us": [round(u, 2) for u in per_call], "graph_replay_us_per_call": graph_us,
+        "bytes_per_call": blk_bytes}), flush=True)
+
+
 def run_e2e(lay, wl, stream, dev, args):
     """Forward + backward through the C ABI with host (pinned) inputs and a
     device-to-host read of every output and gradient, timed per step."""
@@ -392,6 +574,8 @@ def main():
     ap.add_argument("--warmup-seconds", type=float, default=1.0,
                     help="keep warming up for at least this long (clock sampling under load)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (smaller profiling case)")
+    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k"],
+                    help="layer: the step line; others: extra lines on one GPU")
     args = ap.parse_args()
     if args.batch:
         CFG["batch"] = args.batch
@@ -400,6 +584,15 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.workload != "layer":
+        if rank == 0:
+            if args.workload == "sweep":
+                run_sweep(args)
+            elif args.workload == "prefill65k":
+                run_prefill(args, 65536, 32, 1)
+            else:
+                run_prefill(args, 262144, 16, 16)
         return
     if world > 1:
         import torch.distributed as dist
