@@ -77,6 +77,12 @@ def kernel_bytes(Bt, L, D, N, Bs, in_b=2, out_b=2):
     }
 
 
+# DRAM bytes (read + write) per launch of the dominant kernel, from one
+# `ncu --set full` capture at batch 4 (profiles/k_bwd_noisy_87m_layer_batch4.md),
+# scaled by batch / 4: the kernel's traffic is proportional to the batch. Set
+# to None whenever the kernel changes until it is captured again.
+MEASURED_TRAFFIC_BATCH4 = {"bwd_noisy": 330_542_848}
+
 # FP32 work per (token, channel, state) element of each scan kernel, counted
 # from the kernel's arithmetic (FMA = 2 flops; ex2, mul, add, reduction add = 1).
 KERNEL_FLOPS_PER_ELEM = {
@@ -329,7 +335,8 @@ def run_ours(args, rank, world, local_rank):
                 "achieved": round(dom_flops / (avg_us[dom] * 1e-6) / 1e12, 2),
                 "peak": round(fp32_peak_tflops, 1), "unit": "TFLOP/s",
                 "frac": round(dom_flops / (avg_us[dom] * 1e-6) / 1e12 / fp32_peak_tflops, 4),
-                "traffic": None,
+                "traffic": (None if MEASURED_TRAFFIC_BATCH4.get(dname) is None
+                            else int(MEASURED_TRAFFIC_BATCH4[dname] * Bt / 4)),
                 "peak_kind": "derived: 152 SMs x 128 FP32 lanes x 2 flop/FMA x max SM clock",
                 "flops_per_launch": dom_flops}
     hbm = {"bound": "hbm", "achieved": round((fb + bb) / (ms_step * 1e-3) / 1e9, 1),
