@@ -62,20 +62,22 @@ __device__ __forceinline__ void ck_load(float2 (&h)[N / 2], const float* ck, int
 // of the reduction buffer, so that their addresses are immediates.
 constexpr int kBwdTS = 16;
 
-// red[which][i][warp][n] (i < kBwdTS): which 0 = dB (adjoint pass), 1 = dC
-// (recompute pass). `mine` is this thread's slot, red + warp * N + lane; only
-// lanes below N store.
+// red[which][i][warp][lane] (i < kBwdTS): which 0 = dB (adjoint pass), 1 =
+// dC (recompute pass); every lane stores its warp_reduce_swz_part value, a
+// partial for state lane % N. `mine` is this thread's slot, red + warp * 32 + lane.
+constexpr int kRedRow = kWarps * 32;  // floats per (which, token)
 template <int N>
 __device__ __forceinline__ float* red_slot(float* red) {
-  return red + (threadIdx.x >> 5) * N + (threadIdx.x & 31);
+  return red + threadIdx.x;
 }
 template <int N>
 __device__ __forceinline__ void red_put(float* mine, int which, int i, float v) {
-  if ((threadIdx.x & 31) < N) mine[(which * kBwdTS + i) * kWarps * N] = v;
+  mine[(which * kBwdTS + i) * kRedRow] = v;
 }
 
-// Sums the 4 warps' rows and stores the CTA's channel-group partials of two
-// token-by-state gradients for tokens [tstart, tstart+TS).
+// Sums the 4 warps' rows (32/N lane partials each, in a fixed order) and
+// stores the CTA's channel-group partials of two token-by-state gradients for
+// tokens [tstart, tstart+TS).
 template <int N>
 __device__ void red_flush(const BwdParams& p, const float* red, int tensB, int tensC, int64_t b,
                           int64_t tstart, int TS) {
@@ -86,10 +88,12 @@ __device__ void red_flush(const BwdParams& p, const float* red, int tensB, int t
     const int j = j0 + threadIdx.x;
     const int which = j / (kBwdTS * N), i = (j / N) % kBwdTS, n = j % N;
     if (i < TS) {
-      const float* src = red + ((which * kBwdTS + i) * kWarps) * N + n;
-      float s = src[0];
+      const float* src = red + (which * kBwdTS + i) * kRedRow + n;
+      float s = 0.f;
 #pragma unroll
-      for (int w = 1; w < kWarps; ++w) s += src[w * N];
+      for (int w = 0; w < kWarps; ++w)
+#pragma unroll
+        for (int r = 0; r < 32 / N; ++r) s += src[w * 32 + r * N];
       const int tensor = which == 0 ? tensB : tensC;
       p.part_tok[((((int64_t)tensor * g.Bt + b) * g.L + tstart + i) * g.G + blockIdx.x) * N + n] = s;
     }
@@ -154,10 +158,10 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
       w[j] = mul2(dy2, h[j]);
     }
     tmem_st2<N>(tb + (uint32_t)(i * N), pv);
-    red_put<N>(mine, 1, i, warp_reduce_swz<N>(w));
+    red_put<N>(mine, 1, i, warp_reduce_swz_part<N>(w));
   }
   tmem_wait_st();
-#pragma unroll 2
+#pragma unroll 4
   for (int k = 0; k < TS; ++k) {  // adjoint, against scan order
     const int i = FWDDIR ? TS - 1 - k : k;
     float2 pv[N / 2];
@@ -180,7 +184,7 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
       sg[j & 1] = fma2(gb, B[j], sg[j & 1]);
       w[j] = mul2(gb, u2);
     }
-    red_put<N>(mine, 0, i, warp_reduce_swz<N>(w));
+    red_put<N>(mine, 0, i, warp_reduce_swz_part<N>(w));
     const float2 sgs = add2(sg[0], sg[1]), sas = add2(sa[0], sa[1]);
     epi(i, dt, x, dy, __fadd_rn(sgs.x, sgs.y), __fadd_rn(sas.x, sas.y));
   }
@@ -213,7 +217,7 @@ __device__ __forceinline__ void seg_bwd_half(const St& st, int TS, int jx, int j
       h[j] = fma2(u2, B[j], mul2(a, h[j]));
       w[j] = mul2(dy2, h[j]);
     }
-    red_put<N>(mine, 1, i, warp_reduce_swz<N>(w));
+    red_put<N>(mine, 1, i, warp_reduce_swz_part<N>(w));
   }
   tmem_wait_st();
 
@@ -236,7 +240,7 @@ __device__ __forceinline__ void seg_bwd_half(const St& st, int TS, int jx, int j
       sg[j & 1] = fma2(gb, B[j], sg[j & 1]);
       w[j] = mul2(gb, u2);
     }
-    red_put<N>(mine, 0, i, warp_reduce_swz<N>(w));
+    red_put<N>(mine, 0, i, warp_reduce_swz_part<N>(w));
     const float2 sgs = add2(sg[0], sg[1]), sas = add2(sa[0], sa[1]);
     epi(i, dt, x, dy, __fadd_rn(sgs.x, sgs.y), __fadd_rn(sas.x, sas.y));
   };
@@ -291,7 +295,7 @@ struct NoisyBwdSmem {
   // two staging buffers when a block is a single segment (prefetch of the next block)
   static __host__ __device__ size_t dx_off(int TS, int Bs) { return align16(St::buf_bytes(kBwdTS) * (Bs / TS == 1 ? 2 : 1)); }
   static __host__ __device__ size_t red_off(int TS, int Bs) { return dx_off(TS, Bs) + (size_t)Bs * kCta * 4; }
-  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kWarps * N * 4; }
+  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kRedRow * 4; }
   static __host__ __device__ size_t slot_off(int TS, int Bs) {
     const int nseg = Bs / TS;
     return ck_off(TS, Bs) + (size_t)(nseg > 1 ? nseg - 1 : 1) * N * kCta * 4;
@@ -388,7 +392,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
     }
     for (int s = NSEG - 1; s >= 0; --s) {
       if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
-#pragma unroll 2
+#pragma unroll 4
       for (int i = TS - 1; i >= 0; --i) {
         const float dt = st.at(DTC, i), dy = st.at(DYC, i);
         const float2 dt2 = f2(dt), dy2 = f2(dy);
@@ -552,7 +556,7 @@ template <typename T, int N>
 struct CleanBwdSmem {
   using St = Stage<T, N, 3, 2, 2, kBwdTS>;  // x_c, dt_c, dy_c; B_c, C_c
   static __host__ __device__ size_t red_off(int TS, int Bs) { return align16(St::buf_bytes(kBwdTS) * (Bs / TS == 1 ? 2 : 1)); }
-  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kWarps * N * 4; }
+  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kRedRow * 4; }
   static __host__ __device__ size_t slot_off(int TS, int Bs) {
     const int nseg = Bs / TS;
     return ck_off(TS, Bs) + (size_t)(nseg - 1) * N * kCta * 4;

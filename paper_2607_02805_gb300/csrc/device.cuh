@@ -325,6 +325,32 @@ __device__ __forceinline__ float warp_reduce_swz(float2 (&v)[N / 2]) {
   for (int o = N; o < 32; o <<= 1) k += __shfl_xor_sync(0xffffffffu, k, o);
   return k;
 }
+// The same without the final butterfly over lane bits N..16: lane l holds a
+// partial for state l % N, and the 32/N lanes l' with l' % N == l % N hold
+// partials that sum to the warp total.
+template <int N>
+__device__ __forceinline__ float warp_reduce_swz_part(float2 (&v)[N / 2]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = N / 4; o >= 2; o >>= 1) {
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const float2 r = make_float2(__shfl_xor_sync(0xffffffffu, v[i + o].x, 2 * o),
+                                   __shfl_xor_sync(0xffffffffu, v[i + o].y, 2 * o));
+      v[i] = add2(v[i], r);
+    }
+  }
+  const bool up1 = (lane & 2) != 0;
+  float k0 = up1 ? v[1].x : v[0].x, k1 = up1 ? v[1].y : v[0].y;
+  const float s0 = up1 ? v[0].x : v[1].x, s1 = up1 ? v[0].y : v[1].y;
+  k0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+  k1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+  const bool up0 = (lane & 1) != 0;
+  float k = up0 ? k1 : k0;
+  const float s = up0 ? k0 : k1;
+  k += __shfl_xor_sync(0xffffffffu, s, 1);
+  return k;
+}
 
 // ---------------------------------------------------------------------------
 // The selective-scan step (eq. mamba-scan-background with A_t = exp(dt A)):
