@@ -362,7 +362,7 @@ int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan
   p.Dr = params->D_r;
   p.yn = y_n;
   p.seed = seed;
-  cudaError_t e = launched(bds::launch_block_scan(c.dt, c.N, 2, 1, p, (cudaStream_t)stream), (cudaStream_t)stream);
+  cudaError_t e = launched(bds::launch_active_block(c.dt, c.N, p, (cudaStream_t)stream), (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, fn);
   return ok();
 }

@@ -15,6 +15,9 @@
 //                  direction, eq. partial-reverse first line) and run the
 //                  block-local reverse scan from zero (second line), and
 //                  write their sum (third line).
+//   k_active_block each (batch, 32 channels): one noisy block from a cached
+//                  seed (the inference step), forward and reverse scans in
+//                  two warps at once.
 // The state at the end of a chunk's last block is taken from the carry
 // kernel (the same value the next chunk starts from), so every consumer of
 // a boundary state sees one value, and boundary states of a prefix equal
@@ -113,19 +116,20 @@ __global__ void __launch_bounds__(256) k_chunk_carry(const FwdParams p) {
 }
 
 // MODE 0: all-block forward (clean + noisy). MODE 1: clean scan only (cache
-// build). MODE 2: one noisy block from a cached seed (active block).
+// build). The active block has its own kernel (k_active_block).
 template <int MODE>
 struct ScanLayout {
-  static constexpr bool kClean = MODE != 2;
-  static constexpr bool kNoisy = MODE != 1;
-  static constexpr int NTD = MODE == 0 ? 5 : (MODE == 1 ? 2 : 3);
-  static constexpr int NROW = MODE == 0 ? 6 : (MODE == 1 ? 2 : 4);
+  static_assert(MODE == 0 || MODE == 1, "block scan modes");
+  static constexpr bool kClean = true;
+  static constexpr bool kNoisy = MODE == 0;
+  static constexpr int NTD = MODE == 0 ? 5 : 2;
+  static constexpr int NROW = MODE == 0 ? 6 : 2;
   // token-by-channel slots
   static constexpr int XC = 0, DTC = 1;
-  static constexpr int XN = MODE == 0 ? 2 : 0, DTF = XN + 1, DTR = XN + 2;
+  static constexpr int XN = 2, DTF = XN + 1, DTR = XN + 2;
   // token-by-state slots
   static constexpr int BC = 0, CC = 1;
-  static constexpr int BF = MODE == 0 ? 2 : 0, CF = BF + 1, BR = BF + 2, CR = BF + 3;
+  static constexpr int BF = 2, CF = BF + 1, BR = BF + 2, CR = BF + 3;
 };
 
 template <typename T, typename TO, int N, int MODE>
@@ -177,21 +181,11 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
     }
   }
 
-  int k_lo = 0, k_hi = 0;
-  bool full = false;
-  if (MODE != 2) {
-    k_lo = c * g.m;
-    k_hi = min(k_lo + g.m, g.nb) - 1;
-    full = c < g.nc_full;
-  }
+  const int k_lo = c * g.m, k_hi = min(k_lo + g.m, g.nb) - 1;
+  const bool full = c < g.nc_full;
   float2 hc[N / 2];
   vzero2<N>(hc);
-  if (act) {
-    if (MODE == 2)
-      vload2<N>(hc, p.seed + (b * g.D + d) * N, 0);
-    else
-      vload2<N>(hc, p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, 0);
-  }
+  if (act) vload2<N>(hc, p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, 0);
 
   if (dbuf) st.issue(0, b * g.L + (int64_t)k_lo * Bs, Bs, g.D, d0);
   for (int k = k_lo; k <= k_hi; ++k) {
@@ -257,6 +251,116 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
 }
 
 // ---------------------------------------------------------------------------
+// Active block (the inference step): one noisy block per batch row from a
+// read-only cached seed. A CTA covers 32 channels of one row; warp 0 runs the
+// seeded forward scan and warp 1 the block-local reverse scan at the same
+// time, each with the per-channel arithmetic of k_block_scan (scan_step,
+// with_skip, combine_dirs), so the outputs equal those of the all-block
+// forward bit for bit. The step is bound by the latency of the serial scan,
+// so small CTAs spread it over many SMs.
+// ---------------------------------------------------------------------------
+constexpr int kActW = 32;  // channels per active-block CTA
+
+template <typename T, int N>
+struct ActiveLayout {
+  // [3][Bs][32] x, dt_f, dt_r as stored; [4][Bs][N] B_f, C_f, B_r, C_r as
+  // loaded and widened to fp32; [2][Bs][32] forward and reverse outputs
+  static __host__ __device__ size_t td_bytes(int Bs) {
+    return ((size_t)3 * Bs * kActW * sizeof(T) + 15) & ~(size_t)15;
+  }
+  static __host__ __device__ size_t raw_bytes(int Bs) {
+    return is_f32<T>::value ? 0 : (((size_t)4 * Bs * N * sizeof(T) + 15) & ~(size_t)15);
+  }
+  static __host__ __device__ size_t rows_bytes(int Bs) { return (size_t)4 * Bs * N * 4; }
+  static __host__ __device__ size_t bytes(int Bs) {
+    return td_bytes(Bs) + raw_bytes(Bs) + rows_bytes(Bs) + (size_t)2 * Bs * kActW * 4;
+  }
+};
+
+template <typename T, typename TO, int N>
+__global__ void __launch_bounds__(2 * kActW, 1) k_active_block(const FwdParams p) {
+  using Ly = ActiveLayout<T, N>;
+  extern __shared__ __align__(16) unsigned char smem[];
+  const Geo& g = p.g;
+  const int Bs = (int)g.Bs;
+  const int64_t b = blockIdx.y, d0 = (int64_t)blockIdx.x * kActW;
+  const int lane = threadIdx.x & 31, dir = threadIdx.x >> 5;  // dir 0: forward, 1: reverse
+  const int64_t d = d0 + lane;
+  const bool act = d < g.D;
+  T* td = reinterpret_cast<T*>(smem);
+  float* rows = reinterpret_cast<float*>(smem + Ly::td_bytes(Bs) + Ly::raw_bytes(Bs));
+  T* raw = is_f32<T>::value ? reinterpret_cast<T*>(rows) : reinterpret_cast<T*>(smem + Ly::td_bytes(Bs));
+  float* ybuf = rows + (size_t)4 * Bs * N;
+
+  // copies (16-byte chunks; channels past D read as zero)
+  constexpr int E = 16 / (int)sizeof(T);
+  constexpr int CPR = kActW / E;
+  const int64_t row0 = b * g.L;
+  for (int q = threadIdx.x; q < 3 * Bs * CPR; q += 2 * kActW) {
+    const int j = q / (Bs * CPR), r = q - j * (Bs * CPR), t = r / CPR, cc = (r - t * CPR) * E;
+    const T* src = (const T*)(j == 0 ? p.xn : (j == 1 ? p.dtf : p.dtr));
+    const bool ok = d0 + cc < g.D;
+    cp_async16(td + ((size_t)j * Bs + t) * kActW + cc,
+               ok ? (const void*)(src + (row0 + t) * g.D + d0 + cc) : (const void*)src, ok ? 16 : 0);
+  }
+  const int rch = Bs * N / E;
+  for (int q = threadIdx.x; q < 4 * rch; q += 2 * kActW) {
+    const int j = q / rch, r = q - j * rch;
+    const T* src = (const T*)(j == 0 ? p.Bf : (j == 1 ? p.Cf : (j == 2 ? p.Br : p.Cr)));
+    cp_async16(raw + (size_t)j * Bs * N + r * E, src + row0 * N + (int64_t)r * E, 16);
+  }
+  cp_async_commit();
+
+  // parameters and the seed while the copies are in flight
+  float2 A2[N / 2], h[N / 2];
+  vzero2<N>(A2);
+  vzero2<N>(h);
+  float Dd = 0.f;
+  if (act) {
+    vload2<N>(A2, (dir == 0 ? p.Af : p.Ar) + d * N, 0);
+#pragma unroll
+    for (int j = 0; j < N / 2; ++j) A2[j] = mul2(A2[j], f2(kLog2e));
+    Dd = dir == 0 ? p.Df[d] : p.Dr[d];
+    if (dir == 0) vload2<N>(h, p.seed + (b * g.D + d) * N, 0);
+  }
+  cp_async_wait_all();
+  __syncthreads();
+  if (!is_f32<T>::value) {
+    for (int q = threadIdx.x; q < 2 * Bs * N; q += 2 * kActW)
+      reinterpret_cast<float2*>(rows)[q] = make_float2(cvt(raw[2 * q]), cvt(raw[2 * q + 1]));
+    __syncthreads();
+  }
+
+  const T* xs = td;
+  const T* dts = td + (size_t)(1 + dir) * Bs * kActW;
+  const float* Brow = rows + (size_t)(2 * dir) * Bs * N;
+  const float* Crow = Brow + (size_t)Bs * N;
+  float* yb = ybuf + (size_t)dir * Bs * kActW;
+  if (dir == 0) {
+#pragma unroll 4
+    for (int i = 0; i < Bs; ++i) {
+      const float x = cvt(xs[i * kActW + lane]), dt = cvt(dts[i * kActW + lane]);
+      const float y = scan_step<N>(h, A2, dt, x, Brow + i * N, Crow + i * N);
+      yb[i * kActW + lane] = with_skip(y, Dd, x);
+    }
+  } else {
+#pragma unroll 4
+    for (int i = Bs - 1; i >= 0; --i) {
+      const float x = cvt(xs[i * kActW + lane]), dt = cvt(dts[i * kActW + lane]);
+      const float y = scan_step<N>(h, A2, dt, x, Brow + i * N, Crow + i * N);
+      yb[i * kActW + lane] = with_skip(y, Dd, x);
+    }
+  }
+  __syncthreads();
+  for (int q = threadIdx.x; q < Bs * kActW; q += 2 * kActW) {
+    const int i = q / kActW, c = q - i * kActW;
+    if (d0 + c < g.D)
+      reinterpret_cast<TO*>(p.yn)[(row0 + i) * g.D + d0 + c] =
+          to_out<TO>(combine_dirs(ybuf[q], ybuf[(size_t)Bs * kActW + q]));
+  }
+}
+
+// ---------------------------------------------------------------------------
 // launchers
 // ---------------------------------------------------------------------------
 namespace {
@@ -309,7 +413,7 @@ cudaError_t block_scan_mode(int mode, int nchunks, const FwdParams& p, cudaStrea
   switch (mode) {
     case 0: return block_scan_t<T, TO, N, 0>(nchunks, p, s);
     case 1: return block_scan_t<T, TO, N, 1>(nchunks, p, s);
-    default: return block_scan_t<T, TO, N, 2>(nchunks, p, s);
+    default: return cudaErrorInvalidValue;
   }
 }
 
@@ -318,8 +422,20 @@ size_t block_scan_smem_mode(int mode, int64_t Bs) {
   switch (mode) {
     case 0: return block_scan_smem_t<T, TO, N, 0>(Bs);
     case 1: return block_scan_smem_t<T, TO, N, 1>(Bs);
-    default: return block_scan_smem_t<T, TO, N, 2>(Bs);
+    default: return 0;
   }
+}
+
+template <typename T, typename TO, int N>
+cudaError_t active_block_t(const FwdParams& p, cudaStream_t s) {
+  const size_t smem = ActiveLayout<T, N>::bytes((int)p.g.Bs);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_active_block<T, TO, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  dim3 grid((unsigned)((p.g.D + kActW - 1) / kActW), (unsigned)p.g.Bt);
+  k_active_block<T, TO, N><<<grid, 2 * kActW, smem, s>>>(p);
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -352,6 +468,15 @@ cudaError_t launch_block_scan(int dt, int N, int mode, int nchunks, const FwdPar
     case 0: BDS_DISPATCH_N(N, return block_scan_mode<float, float, NN>(mode, nchunks, p, s);)
     case 1: BDS_DISPATCH_N(N, return block_scan_mode<bf16, bf16, NN>(mode, nchunks, p, s);)
     default: BDS_DISPATCH_N(N, return block_scan_mode<bf16, float, NN>(mode, nchunks, p, s);)
+  }
+}
+
+cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t s) {
+  if (p.g.Bt == 0 || p.g.D == 0) return cudaSuccess;
+  switch (dt) {
+    case 0: BDS_DISPATCH_N(N, return active_block_t<float, float, NN>(p, s);)
+    case 1: BDS_DISPATCH_N(N, return active_block_t<bf16, bf16, NN>(p, s);)
+    default: BDS_DISPATCH_N(N, return active_block_t<bf16, float, NN>(p, s);)
   }
 }
 

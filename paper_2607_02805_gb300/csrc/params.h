@@ -61,8 +61,10 @@ struct BwdParams {
 // Launchers (fwd.cu / bwd.cu). dt: 0 = f32 in/out, 1 = bf16 in/out, 2 = bf16 in, f32 out.
 cudaError_t launch_chunk_local(int dt, int N, const FwdParams& p, cudaStream_t s);
 cudaError_t launch_chunk_carry(int N, const FwdParams& p, cudaStream_t s);
-// mode 0: all-block forward, 1: clean scan only, 2: active block
+// mode 0: all-block forward, 1: clean scan only (cache build)
 cudaError_t launch_block_scan(int dt, int N, int mode, int nchunks, const FwdParams& p, cudaStream_t s);
+// One noisy block per batch row from p.seed (len == block).
+cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_noisy(int dt, int N, const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_carry(int N, const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_clean(int dt, int N, const BwdParams& p, cudaStream_t s);
