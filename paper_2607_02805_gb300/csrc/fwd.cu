@@ -30,6 +30,10 @@ namespace bds {
 static_assert(kCta == kCtaHost, "host and device CTA widths differ");
 
 constexpr int kLocalSpan = 32;  // tokens staged per step of the chunk-local scan
+// Tokens the block scan stages at once: longer blocks are staged in segments
+// of this many tokens (shared memory, and so residency, stays that of a
+// 16-token block).
+constexpr int kScanSeg = 16;
 
 template <typename T, int N>
 __global__ void __launch_bounds__(kCta) k_chunk_local(const FwdParams p) {
@@ -142,11 +146,12 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
   const bool act = d < g.D;
   const int Bs = (int)g.Bs;
+  const int SEG = Bs < kScanSeg ? Bs : kScanSeg, NSEG = (Bs + SEG - 1) / SEG;
   Stage<T, N, Ly::NTD, Ly::NROW, 2> st;
-  st.carve(smem, Bs);
-  const bool dbuf = p.stage_bufs == 2;
+  st.carve(smem, SEG);
+  const bool dbuf = p.stage_bufs == 2 && NSEG == 1;
   float* yfbuf =
-      reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(Bs) * (dbuf ? 2 : 1));
+      reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(SEG) * (dbuf ? 2 : 1));
   if (Ly::kClean) {
     st.td_src[Ly::XC] = (const T*)p.xc;
     st.td_src[Ly::DTC] = (const T*)p.dtc;
@@ -194,24 +199,29 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
       __syncthreads();  // the other buffer is no longer read
       if (k < k_hi) st.issue((k - k_lo + 1) & 1, row0 + Bs, Bs, g.D, d0);
       st.complete((k - k_lo) & 1, Bs, k < k_hi ? 1 : 0);
-    } else {
+    } else if (NSEG == 1) {
       st.load(row0, Bs, g.D, d0);
     }
     float2 hs[N / 2];
 #pragma unroll
     for (int j = 0; j < N / 2; ++j) hs[j] = hc[j];  // the block's seed: state before its first token
+    for (int sg = 0; sg < NSEG; ++sg) {  // segments left to right
+      const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
+      if (NSEG > 1) st.load(row0 + i0, ns, g.D, d0);
 #pragma unroll 4
-    for (int i = 0; i < Bs; ++i) {
-      const int64_t o = (row0 + i) * g.D + d;
-      if (Ly::kClean) {
-        const float x = st.at(Ly::XC, i), dt = st.at(Ly::DTC, i);
-        const float y = scan_step<N>(hc, A2f, dt, x, st.row(Ly::BC, i), st.row(Ly::CC, i));
-        if (p.yc != nullptr && act) reinterpret_cast<TO*>(p.yc)[o] = to_out<TO>(with_skip(y, Df, x));
-      }
-      if (Ly::kNoisy) {
-        const float x = st.at(Ly::XN, i), dt = st.at(Ly::DTF, i);
-        const float y = scan_step<N>(hs, A2f, dt, x, st.row(Ly::BF, i), st.row(Ly::CF, i));
-        yfbuf[i * kCta + threadIdx.x] = with_skip(y, Df, x);
+      for (int ii = 0; ii < ns; ++ii) {
+        const int i = i0 + ii;
+        const int64_t o = (row0 + i) * g.D + d;
+        if (Ly::kClean) {
+          const float x = st.at(Ly::XC, ii), dt = st.at(Ly::DTC, ii);
+          const float y = scan_step<N>(hc, A2f, dt, x, st.row(Ly::BC, ii), st.row(Ly::CC, ii));
+          if (p.yc != nullptr && act) reinterpret_cast<TO*>(p.yc)[o] = to_out<TO>(with_skip(y, Df, x));
+        }
+        if (Ly::kNoisy) {
+          const float x = st.at(Ly::XN, ii), dt = st.at(Ly::DTF, ii);
+          const float y = scan_step<N>(hs, A2f, dt, x, st.row(Ly::BF, ii), st.row(Ly::CF, ii));
+          yfbuf[i * kCta + threadIdx.x] = with_skip(y, Df, x);
+        }
       }
     }
     if (Ly::kClean && p.emit_all && act) {
@@ -227,14 +237,19 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
     if (Ly::kNoisy) {
       float2 hr[N / 2];
       vzero2<N>(hr);
+      for (int sg = NSEG - 1; sg >= 0; --sg) {  // segments right to left; the last is still staged
+        const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
+        if (sg < NSEG - 1) st.load(row0 + i0, ns, g.D, d0);
 #pragma unroll 4
-      for (int i = Bs - 1; i >= 0; --i) {
-        const int64_t o = (row0 + i) * g.D + d;
-        const float x = st.at(Ly::XN, i), dt = st.at(Ly::DTR, i);
-        const float y = scan_step<N>(hr, A2r, dt, x, st.row(Ly::BR, i), st.row(Ly::CR, i));
-        if (act)
-          reinterpret_cast<TO*>(p.yn)[o] =
-              to_out<TO>(combine_dirs(yfbuf[i * kCta + threadIdx.x], with_skip(y, Dr, x)));
+        for (int ii = ns - 1; ii >= 0; --ii) {
+          const int i = i0 + ii;
+          const int64_t o = (row0 + i) * g.D + d;
+          const float x = st.at(Ly::XN, ii), dt = st.at(Ly::DTR, ii);
+          const float y = scan_step<N>(hr, A2r, dt, x, st.row(Ly::BR, ii), st.row(Ly::CR, ii));
+          if (act)
+            reinterpret_cast<TO*>(p.yn)[o] =
+                to_out<TO>(combine_dirs(yfbuf[i * kCta + threadIdx.x], with_skip(y, Dr, x)));
+        }
       }
     }
   }
@@ -383,6 +398,7 @@ constexpr size_t kDoubleBufferLimit = 48 * 1024;
 template <typename T, typename TO, int N, int MODE>
 int block_scan_bufs_t(int64_t Bs) {
   using Ly = ScanLayout<MODE>;
+  if (Bs > kScanSeg) return 1;  // segments are staged when needed
   const size_t extra = Ly::kNoisy ? (size_t)Bs * kCta * sizeof(float) : 0;
   return 2 * Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes((int)Bs) + extra <= kDoubleBufferLimit ? 2 : 1;
 }
@@ -390,7 +406,8 @@ int block_scan_bufs_t(int64_t Bs) {
 template <typename T, typename TO, int N, int MODE>
 size_t block_scan_smem_t(int64_t Bs) {
   using Ly = ScanLayout<MODE>;
-  size_t b = Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes((int)Bs) * block_scan_bufs_t<T, TO, N, MODE>(Bs);
+  const int seg = Bs < kScanSeg ? (int)Bs : kScanSeg;
+  size_t b = Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(seg) * block_scan_bufs_t<T, TO, N, MODE>(Bs);
   if (Ly::kNoisy) b += (size_t)Bs * kCta * sizeof(float);
   return b;
 }
