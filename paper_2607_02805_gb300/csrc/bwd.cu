@@ -292,15 +292,16 @@ template <typename T, int N>
 struct NoisyBwdSmem {
   // token-by-channel: x_n, dt_f, dt_r, dy_n, dt_c, dy_c; token-by-state: B_f, C_f, B_r, C_r, C_c
   using St = Stage<T, N, 6, 5, 2, kBwdTS>;
-  // two staging buffers when a block is a single segment (prefetch of the next block)
-  static __host__ __device__ size_t dx_off(int TS, int Bs) { return align16(St::buf_bytes(kBwdTS) * (Bs / TS == 1 ? 2 : 1)); }
-  static __host__ __device__ size_t red_off(int TS, int Bs) { return dx_off(TS, Bs) + (size_t)Bs * kCta * 4; }
-  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kRedRow * 4; }
-  static __host__ __device__ size_t slot_off(int TS, int Bs) {
-    const int nseg = Bs / TS;
-    return ck_off(TS, Bs) + (size_t)(nseg > 1 ? nseg - 1 : 1) * N * kCta * 4;
+  // `bufs` staging buffers: 2 for one-segment blocks (the next block is
+  // copied while the current one is used); for longer blocks one per segment
+  // (the whole block resident) or 1 (each segment copied when needed)
+  static __host__ __device__ size_t dx_off(int bufs) { return align16(St::buf_bytes(kBwdTS) * bufs); }
+  static __host__ __device__ size_t red_off(int bufs, int Bs) { return dx_off(bufs) + (size_t)Bs * kCta * 4; }
+  static __host__ __device__ size_t ck_off(int bufs, int Bs) { return red_off(bufs, Bs) + (size_t)2 * kBwdTS * kRedRow * 4; }
+  static __host__ __device__ size_t slot_off(int bufs, int TS, int Bs) {
+    return ck_off(bufs, Bs) + (size_t)(Bs / TS - 1) * N * kCta * 4;
   }
-  static __host__ __device__ size_t bytes(int TS, int Bs) { return slot_off(TS, Bs) + 16; }
+  static __host__ __device__ size_t bytes(int bufs, int TS, int Bs) { return slot_off(bufs, TS, Bs) + 16; }
 };
 
 template <typename T, typename TO, int N>
@@ -332,11 +333,13 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   st.row_src[BR] = (const T*)p.Br;
   st.row_src[CR] = (const T*)p.Cr;
   st.row_src[CC] = (const T*)p.Cc;
-  float* dxbuf = reinterpret_cast<float*>(smem + L::dx_off(TS, Bs));
-  float* red = reinterpret_cast<float*>(smem + L::red_off(TS, Bs));
+  const bool resident = NSEG > 1 && p.seg_resident;
+  const int bufs = NSEG == 1 ? 2 : (resident ? NSEG : 1);
+  float* dxbuf = reinterpret_cast<float*>(smem + L::dx_off(bufs));
+  float* red = reinterpret_cast<float*>(smem + L::red_off(bufs, Bs));
   float* mine = red_slot<N>(red);
-  float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
+  float* ck = reinterpret_cast<float*>(smem + L::ck_off(bufs, Bs));
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(bufs, TS, Bs));
 
   const uint32_t tcols = full_cols(TS, N);
   if (warp == 0) tmem_alloc(tslot, tcols);
@@ -377,7 +380,18 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
       __syncthreads();  // the other buffer is no longer read
       if (k > k_lo) st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
       st.complete(buf, TS, k > k_lo ? 1 : 0);
+    } else if (resident) {  // every segment of the block, once
+      __syncthreads();  // the previous block is no longer read
+      for (int s = 0; s < NSEG; ++s) st.issue(s, row0 + (int64_t)s * TS, TS, g.D, d0);
+      for (int s = 0; s < NSEG; ++s) st.complete(s, TS, 0);
     }
+    // make segment s current: staged now, or already resident
+    auto stage_seg = [&](int s) {
+      if (resident)
+        st.select(s);
+      else
+        st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+    };
 
     // ---- clean stream: chunk-local adjoint over block k ----
     if (k < k_hi) {
@@ -391,7 +405,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
       }
     }
     for (int s = NSEG - 1; s >= 0; --s) {
-      if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+      if (NSEG > 1) stage_seg(s);
 #pragma unroll 4
       for (int i = TS - 1; i >= 0; --i) {
         const float dt = st.at(DTC, i), dy = st.at(DYC, i);
@@ -410,7 +424,8 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
         float2 h[N / 2];
         vzero2<N>(h);
         for (int s = NSEG - 1; s >= 1; --s) {
-          st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+          stage_seg(s);
+#pragma unroll 4
           for (int i = TS - 1; i >= 0; --i) scan_state_swz<N>(h, A2r, st.at(DTR, i), st.at(XN, i), st.row(BR, i), sw);
           ck_store<N>(ck, s - 1, h);
         }
@@ -418,7 +433,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
       float2 gr[N / 2];  // a_{t-1} gbar_{t-1}, entering token t from the left
       vzero2<N>(gr);
       for (int s = 0; s < NSEG; ++s) {
-        if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+        if (NSEG > 1) stage_seg(s);
         float2 h[N / 2];
         if (s == NSEG - 1)
           vzero2<N>(h);
@@ -446,7 +461,8 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
 #pragma unroll
         for (int j = 0; j < N / 2; ++j) h[j] = seed[j];
         for (int s = 0; s < NSEG - 1; ++s) {
-          st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+          stage_seg(s);
+#pragma unroll 4
           for (int i = 0; i < TS; ++i) scan_state_swz<N>(h, A2f, st.at(DTF, i), st.at(XN, i), st.row(BF, i), sw);
           ck_store<N>(ck, s, h);
         }
@@ -454,7 +470,7 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
       float2 gf[N / 2];  // a_{t+1} gbar_{t+1}, entering token t from the right
       vzero2<N>(gf);
       for (int s = NSEG - 1; s >= 0; --s) {
-        if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+        if (NSEG > 1) stage_seg(s);
         float2 h[N / 2];
         if (s == 0) {
 #pragma unroll
@@ -555,13 +571,13 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
 template <typename T, int N>
 struct CleanBwdSmem {
   using St = Stage<T, N, 3, 2, 2, kBwdTS>;  // x_c, dt_c, dy_c; B_c, C_c
-  static __host__ __device__ size_t red_off(int TS, int Bs) { return align16(St::buf_bytes(kBwdTS) * (Bs / TS == 1 ? 2 : 1)); }
-  static __host__ __device__ size_t ck_off(int TS, int Bs) { return red_off(TS, Bs) + (size_t)2 * kBwdTS * kRedRow * 4; }
-  static __host__ __device__ size_t slot_off(int TS, int Bs) {
-    const int nseg = Bs / TS;
-    return ck_off(TS, Bs) + (size_t)(nseg - 1) * N * kCta * 4;
+  // `bufs` staging buffers, as for the noisy kernel
+  static __host__ __device__ size_t red_off(int bufs) { return align16(St::buf_bytes(kBwdTS) * bufs); }
+  static __host__ __device__ size_t ck_off(int bufs) { return red_off(bufs) + (size_t)2 * kBwdTS * kRedRow * 4; }
+  static __host__ __device__ size_t slot_off(int bufs, int TS, int Bs) {
+    return ck_off(bufs) + (size_t)(Bs / TS - 1) * N * kCta * 4;
   }
-  static __host__ __device__ size_t bytes(int TS, int Bs) { return slot_off(TS, Bs) + 16; }
+  static __host__ __device__ size_t bytes(int bufs, int TS, int Bs) { return slot_off(bufs, TS, Bs) + 16; }
 };
 
 template <typename T, typename TO, int N>
@@ -587,10 +603,12 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   st.td_src[DYC] = (const T*)p.dyc;
   st.row_src[BC] = (const T*)p.Bc;
   st.row_src[CC] = (const T*)p.Cc;
-  float* red = reinterpret_cast<float*>(smem + L::red_off(TS, Bs));
+  const bool resident = NSEG > 1 && p.seg_resident;
+  const int bufs = NSEG == 1 ? 2 : (resident ? NSEG : 1);
+  float* red = reinterpret_cast<float*>(smem + L::red_off(bufs));
   float* mine = red_slot<N>(red);
-  float* ck = reinterpret_cast<float*>(smem + L::ck_off(TS, Bs));
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(TS, Bs));
+  float* ck = reinterpret_cast<float*>(smem + L::ck_off(bufs));
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(bufs, TS, Bs));
 
   const uint32_t tcols = half_cols(TS, N);  // held states of a segment
   if (warp == 0) tmem_alloc(tslot, tcols);
@@ -623,7 +641,18 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
       __syncthreads();  // the other buffer is no longer read
       if (k > k_lo) st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
       st.complete(buf, TS, k > k_lo ? 1 : 0);
+    } else if (resident) {  // every segment of the block, once
+      __syncthreads();  // the previous block is no longer read
+      for (int s = 0; s < NSEG; ++s) st.issue(s, row0 + (int64_t)s * TS, TS, g.D, d0);
+      for (int s = 0; s < NSEG; ++s) st.complete(s, TS, 0);
     }
+    // make segment s current: staged now, or already resident
+    auto stage_seg = [&](int s) {
+      if (resident)
+        st.select(s);
+      else
+        st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+    };
     if (k == k_hi) {
       if (act) vload2<N>(gc, p.Lc + ((b * g.nc + c) * g.D + d) * N, sw);
     } else if (act) {
@@ -645,13 +674,14 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
 #pragma unroll
       for (int j = 0; j < N / 2; ++j) h[j] = seed[j];
       for (int s = 0; s < NSEG - 1; ++s) {
-        st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+        stage_seg(s);
+#pragma unroll 4
         for (int i = 0; i < TS; ++i) scan_state_swz<N>(h, A2, st.at(DTC, i), st.at(XC, i), st.row(BC, i), sw);
         ck_store<N>(ck, s, h);
       }
     }
     for (int s = NSEG - 1; s >= 0; --s) {
-      if (NSEG > 1) st.load(row0 + (int64_t)s * TS, TS, g.D, d0);
+      if (NSEG > 1) stage_seg(s);
       float2 h[N / 2];
       if (s == 0) {
 #pragma unroll
@@ -819,34 +849,65 @@ int resident_ctas(K kernel, size_t smem, uint32_t tcols, int dev) {
   return n;
 }
 
+// Shared memory of a launch, and whether a block of several segments is
+// staged whole (one buffer per segment): only where that costs no resident CTA.
+struct BwdLaunch {
+  size_t smem;
+  int resident;
+};
+template <typename L, typename K>
+BwdLaunch bwd_launch(K kernel, int Bs, uint32_t cols, int dev) {
+  const int TS = Bs < 16 ? Bs : 16, nseg = Bs / TS;
+  if (nseg == 1) return {pad_for_tmem(L::bytes(2, TS, Bs), cols), 0};
+  const size_t one = pad_for_tmem(L::bytes(1, TS, Bs), cols), all = pad_for_tmem(L::bytes(nseg, TS, Bs), cols);
+  const int r1 = resident_ctas(kernel, one, cols, dev), ra = resident_ctas(kernel, all, cols, dev);
+  return ra >= r1 && ra > 0 ? BwdLaunch{all, 1} : BwdLaunch{one, 0};
+}
 template <typename T, typename TO, int N>
-void bwd_per_sm(int Bs, int dev, int& noisy, int& clean) {
+BwdLaunch noisy_launch(int Bs, int dev) {
   const int TS = Bs < 16 ? Bs : 16;
-  noisy = resident_ctas(k_bwd_noisy<T, TO, N>, pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), full_cols(TS, N)),
-                        full_cols(TS, N), dev);
-  clean = resident_ctas(k_bwd_clean<T, TO, N>, pad_for_tmem(CleanBwdSmem<T, N>::bytes(TS, Bs), half_cols(TS, N)),
-                        half_cols(TS, N), dev);
+  return bwd_launch<NoisyBwdSmem<T, N>>(k_bwd_noisy<T, TO, N>, Bs, full_cols(TS, N), dev);
+}
+template <typename T, typename TO, int N>
+BwdLaunch clean_launch(int Bs, int dev) {
+  const int TS = Bs < 16 ? Bs : 16;
+  return bwd_launch<CleanBwdSmem<T, N>>(k_bwd_clean<T, TO, N>, Bs, half_cols(TS, N), dev);
 }
 
 template <typename T, typename TO, int N>
-cudaError_t bwd_noisy_t(const BwdParams& p, cudaStream_t s) {
-  const int Bs = (int)p.g.Bs, TS = Bs < 16 ? Bs : 16;
-  const size_t smem = pad_for_tmem(NoisyBwdSmem<T, N>::bytes(TS, Bs), full_cols(TS, N));
-  cudaError_t e = set_bwd_attrs(k_bwd_noisy<T, TO, N>, smem);
+void bwd_per_sm(int Bs, int dev, int& noisy, int& clean) {
+  const int TS = Bs < 16 ? Bs : 16;
+  noisy = resident_ctas(k_bwd_noisy<T, TO, N>, noisy_launch<T, TO, N>(Bs, dev).smem, full_cols(TS, N), dev);
+  clean = resident_ctas(k_bwd_clean<T, TO, N>, clean_launch<T, TO, N>(Bs, dev).smem, half_cols(TS, N), dev);
+}
+
+template <typename T, typename TO, int N>
+cudaError_t bwd_noisy_t(const BwdParams& p_in, cudaStream_t s) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const BwdLaunch l = noisy_launch<T, TO, N>((int)p_in.g.Bs, dev);
+  BwdParams p = p_in;
+  p.seg_resident = l.resident;
+  e = set_bwd_attrs(k_bwd_noisy<T, TO, N>, l.smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
-  k_bwd_noisy<T, TO, N><<<grid, kCta, smem, s>>>(p);
+  k_bwd_noisy<T, TO, N><<<grid, kCta, l.smem, s>>>(p);
   return cudaGetLastError();
 }
 
 template <typename T, typename TO, int N>
-cudaError_t bwd_clean_t(const BwdParams& p, cudaStream_t s) {
-  const int Bs = (int)p.g.Bs, TS = Bs < 16 ? Bs : 16;
-  const size_t smem = pad_for_tmem(CleanBwdSmem<T, N>::bytes(TS, Bs), half_cols(TS, N));
-  cudaError_t e = set_bwd_attrs(k_bwd_clean<T, TO, N>, smem);
+cudaError_t bwd_clean_t(const BwdParams& p_in, cudaStream_t s) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const BwdLaunch l = clean_launch<T, TO, N>((int)p_in.g.Bs, dev);
+  BwdParams p = p_in;
+  p.seg_resident = l.resident;
+  e = set_bwd_attrs(k_bwd_clean<T, TO, N>, l.smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
-  k_bwd_clean<T, TO, N><<<grid, kCta, smem, s>>>(p);
+  k_bwd_clean<T, TO, N><<<grid, kCta, l.smem, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -934,18 +995,6 @@ int bwd_chunk_count(int dt, int N, const Geo& g) {
     }
   }
   return best;
-}
-
-size_t bwd_noisy_smem(int dt, int N, int64_t Bs) {
-  const int TS = Bs < 16 ? (int)Bs : 16;
-  if (dt == 0) return N == 8 ? NoisyBwdSmem<float, 8>::bytes(TS, (int)Bs) : NoisyBwdSmem<float, 16>::bytes(TS, (int)Bs);
-  return N == 8 ? NoisyBwdSmem<bf16, 8>::bytes(TS, (int)Bs) : NoisyBwdSmem<bf16, 16>::bytes(TS, (int)Bs);
-}
-
-size_t bwd_clean_smem(int dt, int N, int64_t Bs) {
-  const int TS = Bs < 16 ? (int)Bs : 16;
-  if (dt == 0) return N == 8 ? CleanBwdSmem<float, 8>::bytes(TS, (int)Bs) : CleanBwdSmem<float, 16>::bytes(TS, (int)Bs);
-  return N == 8 ? CleanBwdSmem<bf16, 8>::bytes(TS, (int)Bs) : CleanBwdSmem<bf16, 16>::bytes(TS, (int)Bs);
 }
 
 }  // namespace bds

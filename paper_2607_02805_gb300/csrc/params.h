@@ -56,6 +56,7 @@ struct BwdParams {
   float* part_tok;  // [6][Bt][L][G][N] per channel-group sums of dB_c, dC_c, dB_f, dC_f, dB_r, dC_r
   float* part_A;    // [3][Bt*nc][D][N] dA partial sums: noisy fwd, noisy rev, clean
   float* part_D;    // [2][Bt*nc][D]    dD partial sums: noisy, clean
+  int seg_resident;  // set per launch: blocks of several segments staged whole
 };
 
 // Launchers (fwd.cu / bwd.cu). dt: 0 = f32 in/out, 1 = bf16 in/out, 2 = bf16 in, f32 out.
@@ -78,12 +79,10 @@ int api_fail(int code, const char* msg);
 int api_ok();
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn);
 size_t api_fwd_workspace(const Geo& g, int N);
-size_t bwd_noisy_smem(int dt, int N, int64_t Bs);
 int bwd_chunk_count(int dt, int N, const Geo& g);
 // Upper bound of the backward's chunks per batch row (sizes its workspace
 // independently of the device): twice the forward chunking, at most one
 // chunk per block.
 inline int bwd_max_chunks(const Geo& g) { return g.nb < 2 * g.nc ? g.nb : 2 * g.nc; }
-size_t bwd_clean_smem(int dt, int N, int64_t Bs);
 
 }  // namespace bds
