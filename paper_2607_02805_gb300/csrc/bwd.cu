@@ -26,10 +26,13 @@
 //                exact carry, emit the clean-stream gradients.
 //   k_reduce_*   sum the per-channel-group dB, dC and the per-chunk dA, dD
 //                partials in a fixed order (deterministic results).
-// The recompute stores p_t for up to 16 tokens per thread in tensor memory
-// (TMEM): 16 x N fp32 per thread would not fit in registers next to the
-// scan state, and TMEM is otherwise idle in this path. Blocks longer than 16
-// tokens are processed in 16-token segments from checkpointed states.
+// The recompute keeps its values for up to 16 tokens per thread in tensor
+// memory (TMEM): 16 x N fp32 per thread would not fit in registers next to
+// the scan state, and TMEM is otherwise idle in this path. k_bwd_noisy holds
+// p_t of every token; k_bwd_clean holds the state entering every other token
+// and redoes one scan step for the rest (half the columns, three CTAs per SM).
+// Blocks longer than 16 tokens are processed in 16-token segments from
+// checkpointed states.
 //
 // Arithmetic is packed two state indices per FFMA2/FMUL2/FADD2, and per-thread
 // state vectors use the group-swizzled order of device.cuh, which makes the

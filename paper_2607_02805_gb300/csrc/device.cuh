@@ -265,7 +265,7 @@ __device__ __forceinline__ float2 ex2x2(float2 v) { return make_float2(ex2(v.x),
 // kernels the 4-float groups of a vector are stored in a lane-dependent
 // order: slot group j holds state group j ^ sw with sw = (lane >> 2) & (N/4 - 1).
 // This makes the first halving levels of the channel reduction select-free
-// (see warp_reduce_swz). The forward kernels use the natural order (sw = 0).
+// (see warp_reduce_swz_part). The forward kernels use the natural order (sw = 0).
 template <int N>
 __device__ __forceinline__ int swz_of_lane() {
   return (int)((threadIdx.x >> 2) & (N / 4 - 1));
@@ -292,42 +292,13 @@ __device__ __forceinline__ void vzero2(float2 (&v)[N / 2]) {
   for (int j = 0; j < N / 2; ++j) v[j] = make_float2(0.f, 0.f);
 }
 
-// Channel reduction of a group-swizzled vector: v summed over the 32 lanes;
-// afterwards every lane l holds the total for state index l % N. The levels
-// over lane bits 3 and 2 exchange whole slot halves without selects (the
-// partner's matching state sits in the complementary slot); the levels over
-// lane bits 1 and 0 exchange within a 4-group with selects; the remaining
-// lane bits are a butterfly. Fixed order: deterministic.
-template <int N>
-__device__ __forceinline__ float warp_reduce_swz(float2 (&v)[N / 2]) {
-  const int lane = threadIdx.x & 31;
-  // group levels: offsets N/2 ... 4 (in floats), i.e. N/4 ... 2 float2 slots
-#pragma unroll
-  for (int o = N / 4; o >= 2; o >>= 1) {
-#pragma unroll
-    for (int i = 0; i < o; ++i) {
-      const float2 r = make_float2(__shfl_xor_sync(0xffffffffu, v[i + o].x, 2 * o),
-                                   __shfl_xor_sync(0xffffffffu, v[i + o].y, 2 * o));
-      v[i] = add2(v[i], r);
-    }
-  }
-  // v[0], v[1] now hold the four states of group sw; lane bit 1 picks a pair
-  const bool up1 = (lane & 2) != 0;
-  float k0 = up1 ? v[1].x : v[0].x, k1 = up1 ? v[1].y : v[0].y;
-  const float s0 = up1 ? v[0].x : v[1].x, s1 = up1 ? v[0].y : v[1].y;
-  k0 += __shfl_xor_sync(0xffffffffu, s0, 2);
-  k1 += __shfl_xor_sync(0xffffffffu, s1, 2);
-  const bool up0 = (lane & 1) != 0;
-  float k = up0 ? k1 : k0;
-  const float s = up0 ? k0 : k1;
-  k += __shfl_xor_sync(0xffffffffu, s, 1);
-#pragma unroll
-  for (int o = N; o < 32; o <<= 1) k += __shfl_xor_sync(0xffffffffu, k, o);
-  return k;
-}
-// The same without the final butterfly over lane bits N..16: lane l holds a
-// partial for state l % N, and the 32/N lanes l' with l' % N == l % N hold
-// partials that sum to the warp total.
+// Channel reduction of a group-swizzled vector, stopped before the last
+// butterfly: afterwards lane l holds a partial sum for state index l % N,
+// and the 32/N lanes l' with l' % N == l % N hold partials that add up to the
+// total over the 32 lanes. The levels over lane bits 3 and 2 exchange whole
+// slot halves without selects (the partner's matching state sits in the
+// complementary slot); the levels over lane bits 1 and 0 exchange within a
+// 4-group with selects. Fixed order: deterministic.
 template <int N>
 __device__ __forceinline__ float warp_reduce_swz_part(float2 (&v)[N / 2]) {
   const int lane = threadIdx.x & 31;
@@ -432,19 +403,6 @@ template <int N>
 __device__ __forceinline__ void tmem_ld2(uint32_t ta, float2 (&v)[N / 2]) {
   Tmem<N>::ld(ta, *reinterpret_cast<float(*)[N]>(&v[0]));
 }
-// Split form: request a row into raw registers r, do other work, then wait.
-// r must not be read, written or copied between the two calls (the load
-// writes it asynchronously); the wait names r, so no use of it can be
-// scheduled before the wait.
-template <int N>
-__device__ __forceinline__ void tmem_ld_async(uint32_t ta, uint32_t (&r)[N]) {
-  Tmem<N>::ld_nowait(ta, r);
-}
-template <int N>
-__device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[N]) {
-  Tmem<N>::wait(r);
-}
-
 template <>
 struct Tmem<16> {
   static __device__ __forceinline__ void st(uint32_t ta, const float (&v)[16]) {
@@ -475,21 +433,6 @@ struct Tmem<16> {
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
   }
-  static __device__ __forceinline__ void ld_nowait(uint32_t ta, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, "
-        "%13, %14, %15}, [%16];\n"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(ta));
-  }
-  static __device__ __forceinline__ void wait(uint32_t (&r)[16]) {
-    asm volatile("tcgen05.wait::ld.sync.aligned;\n"
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
-                   "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
-                   "+r"(r[14]), "+r"(r[15])
-                 :);
-  }
 };
 
 template <>
@@ -510,16 +453,6 @@ struct Tmem<8> {
                  :);
 #pragma unroll
     for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
-  }
-  static __device__ __forceinline__ void ld_nowait(uint32_t ta, uint32_t (&r)[8]) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];\n"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                 : "r"(ta));
-  }
-  static __device__ __forceinline__ void wait(uint32_t (&r)[8]) {
-    asm volatile("tcgen05.wait::ld.sync.aligned;\n"
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7])
-                 :);
   }
 };
 

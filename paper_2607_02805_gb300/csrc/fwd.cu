@@ -435,15 +435,6 @@ cudaError_t block_scan_mode(int mode, int nchunks, const FwdParams& p, cudaStrea
 }
 
 template <typename T, typename TO, int N>
-size_t block_scan_smem_mode(int mode, int64_t Bs) {
-  switch (mode) {
-    case 0: return block_scan_smem_t<T, TO, N, 0>(Bs);
-    case 1: return block_scan_smem_t<T, TO, N, 1>(Bs);
-    default: return 0;
-  }
-}
-
-template <typename T, typename TO, int N>
 cudaError_t active_block_t(const FwdParams& p, cudaStream_t s) {
   const size_t smem = ActiveLayout<T, N>::bytes((int)p.g.Bs);
   if (smem > 48 * 1024) {
@@ -495,12 +486,6 @@ cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t 
     case 1: BDS_DISPATCH_N(N, return active_block_t<bf16, bf16, NN>(p, s);)
     default: BDS_DISPATCH_N(N, return active_block_t<bf16, float, NN>(p, s);)
   }
-}
-
-size_t block_scan_smem(int dt, int N, int mode, int64_t Bs) {
-  if (N != 8 && N != 16) return 0;
-  if (dt == 0) return N == 8 ? block_scan_smem_mode<float, float, 8>(mode, Bs) : block_scan_smem_mode<float, float, 16>(mode, Bs);
-  return N == 8 ? block_scan_smem_mode<bf16, bf16, 8>(mode, Bs) : block_scan_smem_mode<bf16, bf16, 16>(mode, Bs);
 }
 
 }  // namespace bds

@@ -72,7 +72,6 @@ cudaError_t launch_bwd_clean(int dt, int N, const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_reduce_tok(int dt, int N, const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s);
 
-size_t block_scan_smem(int dt, int N, int mode, int64_t Bs);
 
 // Helpers of api.cu for other translation units of the library.
 int api_fail(int code, const char* msg);
