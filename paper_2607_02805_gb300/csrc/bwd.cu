@@ -106,6 +106,21 @@ __device__ void red_flush(const BwdParams& p, const float* red, int tensB, int t
 
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 
+// Copies states[k-1] of the CTA's 128 channels (the seed of block k) into
+// dst, [kCta][N] fp32, in the caller's cp.async group; zeros for k = 0 and
+// for channels past D. The clean backward stages it with the block's inputs,
+// so the state its recompute starts from arrives with the prefetch.
+template <int N>
+__device__ __forceinline__ void issue_seed(float* dst, const float* states, const Geo& g, int64_t b, int k,
+                                           int64_t d0) {
+  constexpr int CPC = N / 4;  // 16-byte chunks per channel
+  for (int q = threadIdx.x; q < kCta * CPC; q += kCta) {
+    const bool ok = k > 0 && d0 + q / CPC < g.D;
+    const float* src = ok ? states + ((b * g.nb + (k - 1)) * g.D + d0) * N + (int64_t)q * 4 : states;
+    cp_async16(dst + q * 4, src, ok ? 16 : 0);
+  }
+}
+
 // The backward splits each batch row's blocks into g.nc nearly equal chunks
 // (its own partition, chosen per call so the last wave of CTAs is nearly
 // full); chunk c holds blocks [chunk_lo(c), chunk_lo(c+1)).
@@ -580,7 +595,11 @@ struct CleanBwdSmem {
   static __host__ __device__ size_t slot_off(int bufs, int TS, int Bs) {
     return ck_off(bufs) + (size_t)(Bs / TS - 1) * N * kCta * 4;
   }
-  static __host__ __device__ size_t bytes(int bufs, int TS, int Bs) { return slot_off(bufs, TS, Bs) + 16; }
+  // one-segment blocks: the seeds of the current and the next block
+  static __host__ __device__ size_t seed_off(int bufs, int TS, int Bs) { return slot_off(bufs, TS, Bs) + 16; }
+  static __host__ __device__ size_t bytes(int bufs, int TS, int Bs) {
+    return seed_off(bufs, TS, Bs) + (Bs / TS == 1 ? (size_t)2 * kCta * N * 4 : 0);
+  }
 };
 
 template <typename T, typename TO, int N>
@@ -612,6 +631,7 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   float* mine = red_slot<N>(red);
   float* ck = reinterpret_cast<float*>(smem + L::ck_off(bufs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(bufs, TS, Bs));
+  float* seedb = reinterpret_cast<float*>(smem + L::seed_off(bufs, TS, Bs));  // [2][kCta][N]
 
   const uint32_t tcols = half_cols(TS, N);  // held states of a segment
   if (warp == 0) tmem_alloc(tslot, tcols);
@@ -635,14 +655,20 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   vzero2<N>(gc);
 
   // one-segment blocks: block k-1 is copied while block k is processed
-  if (NSEG == 1) st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
+  if (NSEG == 1) {
+    issue_seed<N>(seedb, p.states, g, b, k_hi, d0);  // same cp.async group as the block
+    st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
+  }
   for (int k = k_hi; k >= k_lo; --k) {
     const int64_t t0 = (int64_t)k * Bs;
     const int64_t row0 = b * g.L + t0;
+    const int buf = (k_hi - k) & 1;
     if (NSEG == 1) {
-      const int buf = (k_hi - k) & 1;
       __syncthreads();  // the other buffer is no longer read
-      if (k > k_lo) st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
+      if (k > k_lo) {
+        issue_seed<N>(seedb + (buf ^ 1) * kCta * N, p.states, g, b, k - 1, d0);
+        st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
+      }
       st.complete(buf, TS, k > k_lo ? 1 : 0);
     } else if (resident) {  // every segment of the block, once
       __syncthreads();  // the previous block is no longer read
@@ -671,7 +697,10 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
     }
     float2 seed[N / 2];
     vzero2<N>(seed);
-    if (k > 0 && act) vload2<N>(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N, sw);
+    if (NSEG == 1)
+        vload2<N>(seed, seedb + (buf * kCta + tid) * N, sw);  // staged with the block
+      else if (k > 0 && act)
+        vload2<N>(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N, sw);
     if (NSEG > 1) {
       float2 h[N / 2];
 #pragma unroll
