@@ -136,7 +136,8 @@ struct ScanLayout {
   static constexpr int BF = 2, CF = BF + 1, BR = BF + 2, CR = BF + 3;
 };
 
-template <typename T, typename TO, int N, int MODE>
+// TILED (blocks shorter than kScanSeg): several blocks per staged tile.
+template <typename T, typename TO, int N, int MODE, bool TILED>
 __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   using Ly = ScanLayout<MODE>;
   extern __shared__ __align__(16) unsigned char smem[];
@@ -147,11 +148,14 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   const bool act = d < g.D;
   const int Bs = (int)g.Bs;
   const int SEG = Bs < kScanSeg ? Bs : kScanSeg, NSEG = (Bs + SEG - 1) / SEG;
+  // blocks shorter than kScanSeg are staged TB at a time (one tile of at most
+  // kScanSeg tokens), so the staging and its barriers are paid per tile
+  const int TB = TILED ? kScanSeg / Bs : 1;
   Stage<T, N, Ly::NTD, Ly::NROW, 2> st;
-  st.carve(smem, SEG);
+  st.carve(smem, NSEG == 1 ? TB * Bs : SEG);
   const bool dbuf = p.stage_bufs == 2 && NSEG == 1;
-  float* yfbuf =
-      reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(SEG) * (dbuf ? 2 : 1));
+  float* yfbuf = reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(st.stride()) *
+                                                       (dbuf ? 2 : 1));
   if (Ly::kClean) {
     st.td_src[Ly::XC] = (const T*)p.xc;
     st.td_src[Ly::DTC] = (const T*)p.dtc;
@@ -192,63 +196,71 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   vzero2<N>(hc);
   if (act) vload2<N>(hc, p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, 0);
 
-  if (dbuf) st.issue(0, b * g.L + (int64_t)k_lo * Bs, Bs, g.D, d0);
-  for (int k = k_lo; k <= k_hi; ++k) {
-    const int64_t row0 = b * g.L + (int64_t)k * Bs;
+  auto tile_blocks = [&](int k0) { return k_hi - k0 + 1 < TB ? k_hi - k0 + 1 : TB; };
+  if (dbuf) st.issue(0, b * g.L + (int64_t)k_lo * Bs, tile_blocks(k_lo) * Bs, g.D, d0);
+  for (int k0 = k_lo; k0 <= k_hi; k0 += TB) {
+    const int nbk = tile_blocks(k0), tile = (k0 - k_lo) / TB;
+    const int64_t trow = b * g.L + (int64_t)k0 * Bs;
     if (dbuf) {
       __syncthreads();  // the other buffer is no longer read
-      if (k < k_hi) st.issue((k - k_lo + 1) & 1, row0 + Bs, Bs, g.D, d0);
-      st.complete((k - k_lo) & 1, Bs, k < k_hi ? 1 : 0);
+      const int k1 = k0 + TB;
+      if (k1 <= k_hi) st.issue((tile + 1) & 1, trow + (int64_t)nbk * Bs, tile_blocks(k1) * Bs, g.D, d0);
+      st.complete(tile & 1, nbk * Bs, k1 <= k_hi ? 1 : 0);
     } else if (NSEG == 1) {
-      st.load(row0, Bs, g.D, d0);
+      st.load(trow, nbk * Bs, g.D, d0);
     }
-    float2 hs[N / 2];
+    for (int kk = 0; kk < nbk; ++kk) {
+      const int k = k0 + kk;
+      const int64_t row0 = trow + (int64_t)kk * Bs;
+      const int toff = kk * Bs;  // the block's first token in the staged tile (0 for long blocks)
+      float2 hs[N / 2];
 #pragma unroll
-    for (int j = 0; j < N / 2; ++j) hs[j] = hc[j];  // the block's seed: state before its first token
-    for (int sg = 0; sg < NSEG; ++sg) {  // segments left to right
-      const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
-      if (NSEG > 1) st.load(row0 + i0, ns, g.D, d0);
-#pragma unroll 4
-      for (int ii = 0; ii < ns; ++ii) {
-        const int i = i0 + ii;
-        const int64_t o = (row0 + i) * g.D + d;
-        if (Ly::kClean) {
-          const float x = st.at(Ly::XC, ii), dt = st.at(Ly::DTC, ii);
-          const float y = scan_step<N>(hc, A2f, dt, x, st.row(Ly::BC, ii), st.row(Ly::CC, ii));
-          if (p.yc != nullptr && act) reinterpret_cast<TO*>(p.yc)[o] = to_out<TO>(with_skip(y, Df, x));
-        }
-        if (Ly::kNoisy) {
-          const float x = st.at(Ly::XN, ii), dt = st.at(Ly::DTF, ii);
-          const float y = scan_step<N>(hs, A2f, dt, x, st.row(Ly::BF, ii), st.row(Ly::CF, ii));
-          yfbuf[i * kCta + threadIdx.x] = with_skip(y, Df, x);
-        }
-      }
-    }
-    if (Ly::kClean && p.emit_all && act) {
-      float* dst = p.states + ((b * g.nb + k) * g.D + d) * N;
-      if (k == k_hi && full) {
-        float2 e[N / 2];
-        vload2<N>(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N, 0);
-        vstore2<N>(dst, e, 0);
-      } else {
-        vstore2<N>(dst, hc, 0);
-      }
-    }
-    if (Ly::kNoisy) {
-      float2 hr[N / 2];
-      vzero2<N>(hr);
-      for (int sg = NSEG - 1; sg >= 0; --sg) {  // segments right to left; the last is still staged
+      for (int j = 0; j < N / 2; ++j) hs[j] = hc[j];  // the block's seed: state before its first token
+      for (int sg = 0; sg < NSEG; ++sg) {  // segments left to right
         const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
-        if (sg < NSEG - 1) st.load(row0 + i0, ns, g.D, d0);
+        if (NSEG > 1) st.load(row0 + i0, ns, g.D, d0);
 #pragma unroll 4
-        for (int ii = ns - 1; ii >= 0; --ii) {
+        for (int ii = 0; ii < ns; ++ii) {
           const int i = i0 + ii;
           const int64_t o = (row0 + i) * g.D + d;
-          const float x = st.at(Ly::XN, ii), dt = st.at(Ly::DTR, ii);
-          const float y = scan_step<N>(hr, A2r, dt, x, st.row(Ly::BR, ii), st.row(Ly::CR, ii));
-          if (act)
-            reinterpret_cast<TO*>(p.yn)[o] =
-                to_out<TO>(combine_dirs(yfbuf[i * kCta + threadIdx.x], with_skip(y, Dr, x)));
+          if (Ly::kClean) {
+            const float x = st.at(Ly::XC, toff + ii), dt = st.at(Ly::DTC, toff + ii);
+            const float y = scan_step<N>(hc, A2f, dt, x, st.row(Ly::BC, toff + ii), st.row(Ly::CC, toff + ii));
+            if (p.yc != nullptr && act) reinterpret_cast<TO*>(p.yc)[o] = to_out<TO>(with_skip(y, Df, x));
+          }
+          if (Ly::kNoisy) {
+            const float x = st.at(Ly::XN, toff + ii), dt = st.at(Ly::DTF, toff + ii);
+            const float y = scan_step<N>(hs, A2f, dt, x, st.row(Ly::BF, toff + ii), st.row(Ly::CF, toff + ii));
+            yfbuf[i * kCta + threadIdx.x] = with_skip(y, Df, x);
+          }
+        }
+      }
+      if (Ly::kClean && p.emit_all && act) {
+        float* dst = p.states + ((b * g.nb + k) * g.D + d) * N;
+        if (k == k_hi && full) {
+          float2 e[N / 2];
+          vload2<N>(e, p.hst + ((b * (g.nc + 1) + c + 1) * g.D + d) * N, 0);
+          vstore2<N>(dst, e, 0);
+        } else {
+          vstore2<N>(dst, hc, 0);
+        }
+      }
+      if (Ly::kNoisy) {
+        float2 hr[N / 2];
+        vzero2<N>(hr);
+        for (int sg = NSEG - 1; sg >= 0; --sg) {  // segments right to left; the last is still staged
+          const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
+          if (sg < NSEG - 1) st.load(row0 + i0, ns, g.D, d0);
+#pragma unroll 4
+          for (int ii = ns - 1; ii >= 0; --ii) {
+            const int i = i0 + ii;
+            const int64_t o = (row0 + i) * g.D + d;
+            const float x = st.at(Ly::XN, toff + ii), dt = st.at(Ly::DTR, toff + ii);
+            const float y = scan_step<N>(hr, A2r, dt, x, st.row(Ly::BR, toff + ii), st.row(Ly::CR, toff + ii));
+            if (act)
+              reinterpret_cast<TO*>(p.yn)[o] =
+                  to_out<TO>(combine_dirs(yfbuf[i * kCta + threadIdx.x], with_skip(y, Dr, x)));
+          }
         }
       }
     }
@@ -399,14 +411,15 @@ template <typename T, typename TO, int N, int MODE>
 int block_scan_bufs_t(int64_t Bs) {
   using Ly = ScanLayout<MODE>;
   if (Bs > kScanSeg) return 1;  // segments are staged when needed
+  const int tile = (int)(kScanSeg / Bs * Bs);
   const size_t extra = Ly::kNoisy ? (size_t)Bs * kCta * sizeof(float) : 0;
-  return 2 * Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes((int)Bs) + extra <= kDoubleBufferLimit ? 2 : 1;
+  return 2 * Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(tile) + extra <= kDoubleBufferLimit ? 2 : 1;
 }
 
 template <typename T, typename TO, int N, int MODE>
 size_t block_scan_smem_t(int64_t Bs) {
   using Ly = ScanLayout<MODE>;
-  const int seg = Bs < kScanSeg ? (int)Bs : kScanSeg;
+  const int seg = Bs < kScanSeg ? (int)(kScanSeg / Bs * Bs) : kScanSeg;  // staged tokens
   size_t b = Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(seg) * block_scan_bufs_t<T, TO, N, MODE>(Bs);
   if (Ly::kNoisy) b += (size_t)Bs * kCta * sizeof(float);
   return b;
@@ -417,11 +430,18 @@ cudaError_t block_scan_t(int nchunks, const FwdParams& p_in, cudaStream_t s) {
   FwdParams p = p_in;
   p.stage_bufs = block_scan_bufs_t<T, TO, N, MODE>(p.g.Bs);
   const size_t smem = block_scan_smem_t<T, TO, N, MODE>(p.g.Bs);
-  cudaError_t e = cudaFuncSetAttribute(k_block_scan<T, TO, N, MODE>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)nchunks, (unsigned)p.g.Bt);
-  k_block_scan<T, TO, N, MODE><<<grid, kCta, smem, s>>>(p);
+  if (p.g.Bs < kScanSeg) {
+    cudaError_t e = cudaFuncSetAttribute(k_block_scan<T, TO, N, MODE, true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_block_scan<T, TO, N, MODE, true><<<grid, kCta, smem, s>>>(p);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(k_block_scan<T, TO, N, MODE, false>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_block_scan<T, TO, N, MODE, false><<<grid, kCta, smem, s>>>(p);
+  }
   return cudaGetLastError();
 }
 
