@@ -65,9 +65,10 @@ __device__ __forceinline__ void ck_load(float2 (&h)[N / 2], const float* ck, int
 // of the reduction buffer, so that their addresses are immediates.
 constexpr int kBwdTS = 16;
 
-// red[which][i][warp][lane] (i < kBwdTS): which 0 = dB (adjoint pass), 1 =
-// dC (recompute pass); every lane stores its warp_reduce_swz_part value, a
-// partial for state lane % N. `mine` is this thread's slot, red + warp * 32 + lane.
+// red[slot][i][warp][lane] (i < kBwdTS): per direction a dB slot (adjoint
+// pass) and the next one for dC (recompute pass); every lane stores its
+// warp_reduce_swz_part value, a partial for state lane % N. `mine` is this
+// thread's place, red + warp * 32 + lane.
 constexpr int kRedRow = kWarps * 32;  // floats per (which, token)
 template <int N>
 __device__ __forceinline__ float* red_slot(float* red) {
@@ -78,11 +79,11 @@ __device__ __forceinline__ void red_put(float* mine, int which, int i, float v) 
   mine[(which * kBwdTS + i) * kRedRow] = v;
 }
 
-// Sums the 4 warps' rows (32/N lane partials each, in a fixed order) and
-// stores the CTA's channel-group partials of two token-by-state gradients for
-// tokens [tstart, tstart+TS).
+// Sums the 4 warps' rows (32/N lane partials each, in a fixed order) of the
+// slots sB (a dB) and sC (a dC) and stores the CTA's channel-group partials
+// of the two token-by-state gradients for tokens [tstart, tstart+TS).
 template <int N>
-__device__ void red_flush(const BwdParams& p, const float* red, int tensB, int tensC, int64_t b,
+__device__ void red_flush(const BwdParams& p, const float* red, int sB, int sC, int tensB, int tensC, int64_t b,
                           int64_t tstart, int TS) {
   __syncthreads();
   const Geo& g = p.g;
@@ -91,7 +92,7 @@ __device__ void red_flush(const BwdParams& p, const float* red, int tensB, int t
     const int j = j0 + threadIdx.x;
     const int which = j / (kBwdTS * N), i = (j / N) % kBwdTS, n = j % N;
     if (i < TS) {
-      const float* src = red + (which * kBwdTS + i) * kRedRow + n;
+      const float* src = red + ((which == 0 ? sB : sC) * kBwdTS + i) * kRedRow + n;
       float s = 0.f;
 #pragma unroll
       for (int w = 0; w < kWarps; ++w)
@@ -154,20 +155,21 @@ __device__ __forceinline__ void scan_state_swz(float2 (&h)[N / 2], const float2 
 //   g   a_next gbar_next entering the segment's last scanned token (in/out)
 //   dA  accumulated sum of dt * gbar * p (in/out)
 //   epi(i, dt, x, dy, sum_n gbar B, sum_n A2 gbar p) writes the per-token results.
-// Channel sums of dy*h (dC) and gbar*dt*x (dB) go to red[1] and red[0]
-// through this thread's slot `mine`.
+//   off  the segment's first token in the staged tile
+// Channel sums of dy*h (dC) and gbar*dt*x (dB) go to red slots rb + 1 and rb
+// through this thread's place `mine`.
 template <int N, bool FWDDIR, typename St, typename Epi>
 __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, int jdy, int rB, int rC,
                                         const float2 (&A2)[N / 2], int sw, float2 (&h)[N / 2],
-                                        float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* mine,
+                                        float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* mine, int off, int rb,
                                         Epi epi) {
 #pragma unroll 2
   for (int k = 0; k < TS; ++k) {  // recompute, in scan order
     const int i = FWDDIR ? k : TS - 1 - k;
-    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float dt = st.at(jdt, off + i), x = st.at(jx, off + i), dy = st.at(jdy, off + i);
     const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
     float2 B[N / 2], pv[N / 2], w[N / 2];
-    vload2<N>(B, st.row(rB, i), sw);
+    vload2<N>(B, st.row(rB, off + i), sw);
 #pragma unroll
     for (int j = 0; j < N / 2; ++j) {
       const float2 a = ex2x2(mul2(dt2, A2[j]));
@@ -176,7 +178,7 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
       w[j] = mul2(dy2, h[j]);
     }
     tmem_st2<N>(tb + (uint32_t)(i * N), pv);
-    red_put<N>(mine, 1, i, warp_reduce_swz_part<N>(w));
+    red_put<N>(mine, rb + 1, off + i, warp_reduce_swz_part<N>(w));
   }
   tmem_wait_st();
 #pragma unroll 4
@@ -184,11 +186,11 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
     const int i = FWDDIR ? TS - 1 - k : k;
     float2 pv[N / 2];
     tmem_ld2<N>(tb + (uint32_t)(i * N), pv);
-    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float dt = st.at(jdt, off + i), x = st.at(jx, off + i), dy = st.at(jdy, off + i);
     const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
     float2 B[N / 2], C[N / 2], w[N / 2];
-    vload2<N>(B, st.row(rB, i), sw);
-    vload2<N>(C, st.row(rC, i), sw);
+    vload2<N>(B, st.row(rB, off + i), sw);
+    vload2<N>(C, st.row(rC, off + i), sw);
     float2 sg[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
     float2 sa[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
@@ -202,7 +204,7 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
       sg[j & 1] = fma2(gb, B[j], sg[j & 1]);
       w[j] = mul2(gb, u2);
     }
-    red_put<N>(mine, 0, i, warp_reduce_swz_part<N>(w));
+    red_put<N>(mine, rb, off + i, warp_reduce_swz_part<N>(w));
     const float2 sgs = add2(sg[0], sg[1]), sas = add2(sa[0], sa[1]);
     epi(i, dt, x, dy, __fadd_rn(sgs.x, sgs.y), __fadd_rn(sas.x, sas.y));
   }
@@ -219,33 +221,33 @@ __device__ __forceinline__ void seg_bwd(const St& st, int TS, int jx, int jdt, i
 template <int N, bool FWDDIR, typename St, typename Epi>
 __device__ __forceinline__ void seg_bwd_half(const St& st, int TS, int jx, int jdt, int jdy, int rB, int rC,
                                              const float2 (&A2)[N / 2], int sw, float2 (&h)[N / 2],
-                                             float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* mine,
+                                             float2 (&g)[N / 2], float2 (&dA)[N / 2], uint32_t tb, float* mine, int off, int rb,
                                              Epi epi) {
 #pragma unroll 2
   for (int k = 0; k < TS; ++k) {  // recompute, in scan order
     const int i = FWDDIR ? k : TS - 1 - k;
     if ((k & 1) == 0) tmem_st2<N>(tb + (uint32_t)((k >> 1) * N), h);
-    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float dt = st.at(jdt, off + i), x = st.at(jx, off + i), dy = st.at(jdy, off + i);
     const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
     float2 B[N / 2], w[N / 2];
-    vload2<N>(B, st.row(rB, i), sw);
+    vload2<N>(B, st.row(rB, off + i), sw);
 #pragma unroll
     for (int j = 0; j < N / 2; ++j) {
       const float2 a = ex2x2(mul2(dt2, A2[j]));
       h[j] = fma2(u2, B[j], mul2(a, h[j]));
       w[j] = mul2(dy2, h[j]);
     }
-    red_put<N>(mine, 1, i, warp_reduce_swz_part<N>(w));
+    red_put<N>(mine, rb + 1, off + i, warp_reduce_swz_part<N>(w));
   }
   tmem_wait_st();
 
   // one adjoint step at token i, given a = a_i and pv = a_i * (state entering i)
   auto step = [&](int i, const float2 (&a)[N / 2], const float2 (&pv)[N / 2]) {
-    const float dt = st.at(jdt, i), x = st.at(jx, i), dy = st.at(jdy, i);
+    const float dt = st.at(jdt, off + i), x = st.at(jx, off + i), dy = st.at(jdy, off + i);
     const float2 dt2 = f2(dt), u2 = f2(__fmul_rn(dt, x)), dy2 = f2(dy);
     float2 B[N / 2], C[N / 2], w[N / 2];
-    vload2<N>(B, st.row(rB, i), sw);
-    vload2<N>(C, st.row(rC, i), sw);
+    vload2<N>(B, st.row(rB, off + i), sw);
+    vload2<N>(C, st.row(rC, off + i), sw);
     float2 sg[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
     float2 sa[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
@@ -258,7 +260,7 @@ __device__ __forceinline__ void seg_bwd_half(const St& st, int TS, int jx, int j
       sg[j & 1] = fma2(gb, B[j], sg[j & 1]);
       w[j] = mul2(gb, u2);
     }
-    red_put<N>(mine, 0, i, warp_reduce_swz_part<N>(w));
+    red_put<N>(mine, rb, off + i, warp_reduce_swz_part<N>(w));
     const float2 sgs = add2(sg[0], sg[1]), sas = add2(sa[0], sa[1]);
     epi(i, dt, x, dy, __fadd_rn(sgs.x, sgs.y), __fadd_rn(sas.x, sas.y));
   };
@@ -268,7 +270,7 @@ __device__ __forceinline__ void seg_bwd_half(const St& st, int TS, int jx, int j
     const int i = FWDDIR ? k : TS - 1 - k;
     float2 S[N / 2], a[N / 2], pv[N / 2];
     tmem_ld2<N>(tb + (uint32_t)((k >> 1) * N), S);
-    const float2 dt2 = f2(st.at(jdt, i));
+    const float2 dt2 = f2(st.at(jdt, off + i));
 #pragma unroll
     for (int j = 0; j < N / 2; ++j) {
       a[j] = ex2x2(mul2(dt2, A2[j]));
@@ -283,10 +285,10 @@ __device__ __forceinline__ void seg_bwd_half(const St& st, int TS, int jx, int j
     float2 S[N / 2], a0[N / 2], pv0[N / 2], a1[N / 2], pv1[N / 2];
     tmem_ld2<N>(tb + (uint32_t)(((k - 1) >> 1) * N), S);  // state entering step k-1
     {
-      const float dt1 = st.at(jdt, i1), x1 = st.at(jx, i1);
-      const float2 dt12 = f2(dt1), u12 = f2(__fmul_rn(dt1, x1)), dt02 = f2(st.at(jdt, i0));
+      const float dt1 = st.at(jdt, off + i1), x1 = st.at(jx, off + i1);
+      const float2 dt12 = f2(dt1), u12 = f2(__fmul_rn(dt1, x1)), dt02 = f2(st.at(jdt, off + i0));
       float2 B1[N / 2];
-      vload2<N>(B1, st.row(rB, i1), sw);
+      vload2<N>(B1, st.row(rB, off + i1), sw);
 #pragma unroll
       for (int j = 0; j < N / 2; ++j) {
         a1[j] = ex2x2(mul2(dt12, A2[j]));
@@ -314,15 +316,20 @@ struct NoisyBwdSmem {
   // copied while the current one is used); for longer blocks one per segment
   // (the whole block resident) or 1 (each segment copied when needed)
   static __host__ __device__ size_t dx_off(int bufs) { return align16(St::buf_bytes(kBwdTS) * bufs); }
-  static __host__ __device__ size_t red_off(int bufs, int Bs) { return dx_off(bufs) + (size_t)Bs * kCta * 4; }
-  static __host__ __device__ size_t ck_off(int bufs, int Bs) { return red_off(bufs, Bs) + (size_t)2 * kBwdTS * kRedRow * 4; }
+  // dx partials of a tile (several short blocks) or of one long block
+  static __host__ __device__ size_t red_off(int bufs, int Bs) { return dx_off(bufs) + (size_t)(Bs < kBwdTS ? kBwdTS : Bs) * kCta * 4; }
+  // red slots: both directions of a tile at once for short blocks, one
+  // direction's segment at a time otherwise
+  static __host__ __device__ int red_slots(int Bs) { return Bs < kBwdTS ? 4 : 2; }
+  static __host__ __device__ size_t ck_off(int bufs, int Bs) { return red_off(bufs, Bs) + (size_t)red_slots(Bs) * kBwdTS * kRedRow * 4; }
   static __host__ __device__ size_t slot_off(int bufs, int TS, int Bs) {
     return ck_off(bufs, Bs) + (size_t)(Bs / TS - 1) * N * kCta * 4;
   }
   static __host__ __device__ size_t bytes(int bufs, int TS, int Bs) { return slot_off(bufs, TS, Bs) + 16; }
 };
 
-template <typename T, typename TO, int N>
+// TILED (blocks shorter than kBwdTS tokens): several blocks per staged tile.
+template <typename T, typename TO, int N, bool TILED>
 __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   extern __shared__ __align__(16) unsigned char smem[];
   using L = NoisyBwdSmem<T, N>;
@@ -388,21 +395,10 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   float2 dSn[N / 2];  // seed gradient of the block to the right of the current one
   vzero2<N>(dSn);
 
-  // one-segment blocks: block k-1 is copied while block k is processed
-  if (NSEG == 1) st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
-  for (int k = k_hi; k >= k_lo; --k) {
+  // everything for block k, whose tokens start at `off` in the staged tile
+  auto block = [&](int k, int off) {
     const int64_t t0 = (int64_t)k * Bs;
     const int64_t row0 = b * g.L + t0;
-    if (NSEG == 1) {
-      const int buf = (k_hi - k) & 1;
-      __syncthreads();  // the other buffer is no longer read
-      if (k > k_lo) st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
-      st.complete(buf, TS, k > k_lo ? 1 : 0);
-    } else if (resident) {  // every segment of the block, once
-      __syncthreads();  // the previous block is no longer read
-      for (int s = 0; s < NSEG; ++s) st.issue(s, row0 + (int64_t)s * TS, TS, g.D, d0);
-      for (int s = 0; s < NSEG; ++s) st.complete(s, TS, 0);
-    }
     // make segment s current: staged now, or already resident
     auto stage_seg = [&](int s) {
       if (resident)
@@ -426,10 +422,10 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
       if (NSEG > 1) stage_seg(s);
 #pragma unroll 4
       for (int i = TS - 1; i >= 0; --i) {
-        const float dt = st.at(DTC, i), dy = st.at(DYC, i);
+        const float dt = st.at(DTC, off + i), dy = st.at(DYC, off + i);
         const float2 dt2 = f2(dt), dy2 = f2(dy);
         float2 C[N / 2];
-        vload2<N>(C, st.row(CC, i), sw);
+        vload2<N>(C, st.row(CC, off + i), sw);
 #pragma unroll
         for (int j = 0; j < N / 2; ++j) carry[j] = mul2(ex2x2(mul2(dt2, A2f[j])), fma2(C[j], dy2, carry[j]));
         sdt = __fadd_rn(sdt, dt);
@@ -457,15 +453,15 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
           vzero2<N>(h);
         else
           ck_load<N>(h, ck, s);
-        seg_bwd<N, false>(st, TS, XN, DTR, DYN, BR, CR, A2r, sw, h, gr, dAr, tb, mine,
+        seg_bwd<N, false>(st, TS, XN, DTR, DYN, BR, CR, A2r, sw, h, gr, dAr, tb, mine, off, 0,
                           [&](int i, float dt, float x, float dy, float sgB, float sAq) {
                             const int ib = s * TS + i;
                             if (act)
                               reinterpret_cast<TO*>(p.ddtr)[(row0 + ib) * g.D + d] =
                                   to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
-                            dxbuf[ib * kCta + tid] = __fmul_rn(dt, sgB);
+                            dxbuf[(off + ib) * kCta + tid] = __fmul_rn(dt, sgB);
                           });
-        red_flush<N>(p, red, 4, 5, b, t0 + (int64_t)s * TS, TS);
+        if (!TILED) red_flush<N>(p, red, 0, 1, 4, 5, b, t0 + (int64_t)s * TS, TS);
       }
     }
 
@@ -496,24 +492,66 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
         } else {
           ck_load<N>(h, ck, s - 1);
         }
-        seg_bwd<N, true>(st, TS, XN, DTF, DYN, BF, CF, A2f, sw, h, gf, dAf, tb, mine,
+        seg_bwd<N, true>(st, TS, XN, DTF, DYN, BF, CF, A2f, sw, h, gf, dAf, tb, mine, off, TILED ? 2 : 0,
                          [&](int i, float dt, float x, float dy, float sgB, float sAq) {
                            const int ib = s * TS + i;
                            const int64_t o = (row0 + ib) * g.D + d;
                            if (act) {
                              reinterpret_cast<TO*>(p.ddtf)[o] = to_out<TO>(__fmaf_rn(x, sgB, __fmul_rn(kLn2, sAq)));
                              const float dxv =
-                                 __fmaf_rn(Dsum, dy, __fadd_rn(dxbuf[ib * kCta + tid], __fmul_rn(dt, sgB)));
+                                 __fmaf_rn(Dsum, dy, __fadd_rn(dxbuf[(off + ib) * kCta + tid], __fmul_rn(dt, sgB)));
                              reinterpret_cast<TO*>(p.dxn)[o] = to_out<TO>(dxv);
                            }
                            dDn = __fmaf_rn(dy, x, dDn);
                          });
-        red_flush<N>(p, red, 2, 3, b, t0 + (int64_t)s * TS, TS);
+        if (!TILED) red_flush<N>(p, red, 0, 1, 2, 3, b, t0 + (int64_t)s * TS, TS);
       }
       // gradient of this block's seed, states[k-1]: a_{t0} gbar_{t0}
 #pragma unroll
       for (int j = 0; j < N / 2; ++j) dSn[j] = gf[j];
       if (k > 0 && act) vstore2<N>(p.dS + ((b * g.nb + (k - 1)) * g.D + d) * N, gf, sw);
+    }
+  };
+
+  if (TILED) {
+    // Short blocks are staged in tiles of TB blocks (at most kBwdTS tokens),
+    // the next tile copied while the current one is used, and the dB/dC
+    // partials of a tile are flushed once for both directions.
+    const int TB = kBwdTS / Bs;
+    auto tile_lo = [&](int hi) { return hi - TB + 1 > k_lo ? hi - TB + 1 : k_lo; };
+    st.issue(0, b * g.L + (int64_t)tile_lo(k_hi) * Bs, (k_hi - tile_lo(k_hi) + 1) * Bs, g.D, d0);
+    int tile = 0;
+    for (int kt_hi = k_hi; kt_hi >= k_lo; ++tile) {
+      const int kt_lo = tile_lo(kt_hi), nbk = kt_hi - kt_lo + 1;
+      const int buf = tile & 1;
+      __syncthreads();  // the other buffer is no longer read
+      if (kt_lo > k_lo) {
+        const int nhi = kt_lo - 1, nlo = tile_lo(nhi);
+        st.issue(buf ^ 1, b * g.L + (int64_t)nlo * Bs, (nhi - nlo + 1) * Bs, g.D, d0);
+      }
+      st.complete(buf, nbk * Bs, kt_lo > k_lo ? 1 : 0);
+      for (int k = kt_hi; k >= kt_lo; --k) block(k, (k - kt_lo) * Bs);
+      const int64_t ts0 = (int64_t)kt_lo * Bs;  // the tile's dB/dC partials, both directions
+      red_flush<N>(p, red, 0, 1, 4, 5, b, ts0, nbk * Bs);
+      red_flush<N>(p, red, 2, 3, 2, 3, b, ts0, nbk * Bs);
+      kt_hi = kt_lo - 1;
+    }
+  } else {
+    // one-segment blocks: block k-1 is copied while block k is processed
+    if (NSEG == 1) st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
+    for (int k = k_hi; k >= k_lo; --k) {
+      const int64_t row0 = b * g.L + (int64_t)k * Bs;
+      if (NSEG == 1) {
+        const int buf = (k_hi - k) & 1;
+        __syncthreads();  // the other buffer is no longer read
+        if (k > k_lo) st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
+        st.complete(buf, TS, k > k_lo ? 1 : 0);
+      } else if (resident) {  // every segment of the block, once
+        __syncthreads();  // the previous block is no longer read
+        for (int s = 0; s < NSEG; ++s) st.issue(s, row0 + (int64_t)s * TS, TS, g.D, d0);
+        for (int s = 0; s < NSEG; ++s) st.complete(s, TS, 0);
+      }
+      block(k, 0);
     }
   }
 
@@ -602,7 +640,7 @@ struct CleanBwdSmem {
   }
 };
 
-template <typename T, typename TO, int N>
+template <typename T, typename TO, int N, bool TILED>
 __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   extern __shared__ __align__(16) unsigned char smem[];
   using L = CleanBwdSmem<T, N>;
@@ -654,27 +692,11 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   float2 gc[N / 2];  // a_{t+1} gbar_{t+1} (+ injections) entering token t from the right
   vzero2<N>(gc);
 
-  // one-segment blocks: block k-1 is copied while block k is processed
-  if (NSEG == 1) {
-    issue_seed<N>(seedb, p.states, g, b, k_hi, d0);  // same cp.async group as the block
-    st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
-  }
-  for (int k = k_hi; k >= k_lo; --k) {
+  // everything for block k, whose tokens start at `off` in the staged tile;
+  // seed_staged: its seed is in seedb[buf]
+  auto block = [&](int k, int off, int buf, bool seed_staged) {
     const int64_t t0 = (int64_t)k * Bs;
     const int64_t row0 = b * g.L + t0;
-    const int buf = (k_hi - k) & 1;
-    if (NSEG == 1) {
-      __syncthreads();  // the other buffer is no longer read
-      if (k > k_lo) {
-        issue_seed<N>(seedb + (buf ^ 1) * kCta * N, p.states, g, b, k - 1, d0);
-        st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
-      }
-      st.complete(buf, TS, k > k_lo ? 1 : 0);
-    } else if (resident) {  // every segment of the block, once
-      __syncthreads();  // the previous block is no longer read
-      for (int s = 0; s < NSEG; ++s) st.issue(s, row0 + (int64_t)s * TS, TS, g.D, d0);
-      for (int s = 0; s < NSEG; ++s) st.complete(s, TS, 0);
-    }
     // make segment s current: staged now, or already resident
     auto stage_seg = [&](int s) {
       if (resident)
@@ -697,8 +719,10 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
     }
     float2 seed[N / 2];
     vzero2<N>(seed);
-    if (NSEG == 1)
-        vload2<N>(seed, seedb + (buf * kCta + tid) * N, sw);  // staged with the block
+    if (seed_staged)
+        vload2<N>(seed, seedb + (buf * kCta + tid) * N, sw);  // staged with the tile
+      else if (NSEG == 1 && k > 0 && act)
+        vload2<N>(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N, sw);
       else if (k > 0 && act)
         vload2<N>(seed, p.states + ((b * g.nb + (k - 1)) * g.D + d) * N, sw);
     if (NSEG > 1) {
@@ -721,7 +745,7 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
       } else {
         ck_load<N>(h, ck, s - 1);
       }
-      seg_bwd_half<N, true>(st, TS, XC, DTC, DYC, BC, CC, A2, sw, h, gc, dA, tb, mine,
+      seg_bwd_half<N, true>(st, TS, XC, DTC, DYC, BC, CC, A2, sw, h, gc, dA, tb, mine, off, 0,
                        [&](int i, float dt, float x, float dy, float sgB, float sAq) {
                          const int64_t o = (row0 + s * TS + i) * g.D + d;
                          if (act) {
@@ -730,7 +754,56 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
                          }
                          dDc = __fmaf_rn(dy, x, dDc);
                        });
-      red_flush<N>(p, red, 0, 1, b, t0 + (int64_t)s * TS, TS);
+      if (!TILED) red_flush<N>(p, red, 0, 1, 0, 1, b, t0 + (int64_t)s * TS, TS);
+    }
+  };
+
+  if (TILED) {
+    // Short blocks are staged in tiles of TB blocks (at most kBwdTS tokens)
+    // together with the seed of the tile's last block, the next tile copied
+    // while the current one is used, and the dB/dC partials of a tile are
+    // flushed once.
+    const int TB = kBwdTS / Bs;
+    auto tile_lo = [&](int hi) { return hi - TB + 1 > k_lo ? hi - TB + 1 : k_lo; };
+    issue_seed<N>(seedb, p.states, g, b, k_hi, d0);  // same cp.async group as the tile
+    st.issue(0, b * g.L + (int64_t)tile_lo(k_hi) * Bs, (k_hi - tile_lo(k_hi) + 1) * Bs, g.D, d0);
+    int tile = 0;
+    for (int kt_hi = k_hi; kt_hi >= k_lo; ++tile) {
+      const int kt_lo = tile_lo(kt_hi), nbk = kt_hi - kt_lo + 1;
+      const int buf = tile & 1;
+      __syncthreads();  // the other buffer is no longer read
+      if (kt_lo > k_lo) {
+        const int nhi = kt_lo - 1, nlo = tile_lo(nhi);
+        issue_seed<N>(seedb + (buf ^ 1) * kCta * N, p.states, g, b, nhi, d0);
+        st.issue(buf ^ 1, b * g.L + (int64_t)nlo * Bs, (nhi - nlo + 1) * Bs, g.D, d0);
+      }
+      st.complete(buf, nbk * Bs, kt_lo > k_lo ? 1 : 0);
+      for (int k = kt_hi; k >= kt_lo; --k) block(k, (k - kt_lo) * Bs, buf, k == kt_hi);
+      red_flush<N>(p, red, 0, 1, 0, 1, b, (int64_t)kt_lo * Bs, nbk * Bs);  // the tile's dB/dC
+      kt_hi = kt_lo - 1;
+    }
+  } else {
+    // one-segment blocks: block k-1 (and its seed) is copied while block k is processed
+    if (NSEG == 1) {
+      issue_seed<N>(seedb, p.states, g, b, k_hi, d0);  // same cp.async group as the block
+      st.issue(0, b * g.L + (int64_t)k_hi * Bs, TS, g.D, d0);
+    }
+    for (int k = k_hi; k >= k_lo; --k) {
+      const int64_t row0 = b * g.L + (int64_t)k * Bs;
+      const int buf = (k_hi - k) & 1;
+      if (NSEG == 1) {
+        __syncthreads();  // the other buffer is no longer read
+        if (k > k_lo) {
+          issue_seed<N>(seedb + (buf ^ 1) * kCta * N, p.states, g, b, k - 1, d0);
+          st.issue(buf ^ 1, row0 - Bs, TS, g.D, d0);
+        }
+        st.complete(buf, TS, k > k_lo ? 1 : 0);
+      } else if (resident) {  // every segment of the block, once
+        __syncthreads();  // the previous block is no longer read
+        for (int s = 0; s < NSEG; ++s) st.issue(s, row0 + (int64_t)s * TS, TS, g.D, d0);
+        for (int s = 0; s < NSEG; ++s) st.complete(s, TS, 0);
+      }
+      block(k, 0, buf, NSEG == 1);
     }
   }
   if (act) {
@@ -895,52 +968,69 @@ BwdLaunch bwd_launch(K kernel, int Bs, uint32_t cols, int dev) {
   const int r1 = resident_ctas(kernel, one, cols, dev), ra = resident_ctas(kernel, all, cols, dev);
   return ra >= r1 && ra > 0 ? BwdLaunch{all, 1} : BwdLaunch{one, 0};
 }
-template <typename T, typename TO, int N>
+template <typename T, typename TO, int N, bool TILED>
 BwdLaunch noisy_launch(int Bs, int dev) {
   const int TS = Bs < 16 ? Bs : 16;
-  return bwd_launch<NoisyBwdSmem<T, N>>(k_bwd_noisy<T, TO, N>, Bs, full_cols(TS, N), dev);
+  return bwd_launch<NoisyBwdSmem<T, N>>(k_bwd_noisy<T, TO, N, TILED>, Bs, full_cols(TS, N), dev);
 }
-template <typename T, typename TO, int N>
+template <typename T, typename TO, int N, bool TILED>
 BwdLaunch clean_launch(int Bs, int dev) {
   const int TS = Bs < 16 ? Bs : 16;
-  return bwd_launch<CleanBwdSmem<T, N>>(k_bwd_clean<T, TO, N>, Bs, half_cols(TS, N), dev);
+  return bwd_launch<CleanBwdSmem<T, N>>(k_bwd_clean<T, TO, N, TILED>, Bs, half_cols(TS, N), dev);
 }
 
+template <typename T, typename TO, int N, bool TILED>
+void bwd_per_sm_t(int Bs, int dev, int& noisy, int& clean) {
+  const int TS = Bs < 16 ? Bs : 16;
+  noisy = resident_ctas(k_bwd_noisy<T, TO, N, TILED>, noisy_launch<T, TO, N, TILED>(Bs, dev).smem,
+                        full_cols(TS, N), dev);
+  clean = resident_ctas(k_bwd_clean<T, TO, N, TILED>, clean_launch<T, TO, N, TILED>(Bs, dev).smem,
+                        half_cols(TS, N), dev);
+}
 template <typename T, typename TO, int N>
 void bwd_per_sm(int Bs, int dev, int& noisy, int& clean) {
-  const int TS = Bs < 16 ? Bs : 16;
-  noisy = resident_ctas(k_bwd_noisy<T, TO, N>, noisy_launch<T, TO, N>(Bs, dev).smem, full_cols(TS, N), dev);
-  clean = resident_ctas(k_bwd_clean<T, TO, N>, clean_launch<T, TO, N>(Bs, dev).smem, half_cols(TS, N), dev);
+  if (Bs < kBwdTS)
+    bwd_per_sm_t<T, TO, N, true>(Bs, dev, noisy, clean);
+  else
+    bwd_per_sm_t<T, TO, N, false>(Bs, dev, noisy, clean);
 }
 
-template <typename T, typename TO, int N>
-cudaError_t bwd_noisy_t(const BwdParams& p_in, cudaStream_t s) {
+template <typename T, typename TO, int N, bool TILED>
+cudaError_t bwd_noisy_tt(const BwdParams& p_in, cudaStream_t s) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  const BwdLaunch l = noisy_launch<T, TO, N>((int)p_in.g.Bs, dev);
+  const BwdLaunch l = noisy_launch<T, TO, N, TILED>((int)p_in.g.Bs, dev);
   BwdParams p = p_in;
   p.seg_resident = l.resident;
-  e = set_bwd_attrs(k_bwd_noisy<T, TO, N>, l.smem);
+  e = set_bwd_attrs(k_bwd_noisy<T, TO, N, TILED>, l.smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
-  k_bwd_noisy<T, TO, N><<<grid, kCta, l.smem, s>>>(p);
+  k_bwd_noisy<T, TO, N, TILED><<<grid, kCta, l.smem, s>>>(p);
   return cudaGetLastError();
 }
-
 template <typename T, typename TO, int N>
-cudaError_t bwd_clean_t(const BwdParams& p_in, cudaStream_t s) {
+cudaError_t bwd_noisy_t(const BwdParams& p, cudaStream_t s) {
+  return p.g.Bs < kBwdTS ? bwd_noisy_tt<T, TO, N, true>(p, s) : bwd_noisy_tt<T, TO, N, false>(p, s);
+}
+
+template <typename T, typename TO, int N, bool TILED>
+cudaError_t bwd_clean_tt(const BwdParams& p_in, cudaStream_t s) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  const BwdLaunch l = clean_launch<T, TO, N>((int)p_in.g.Bs, dev);
+  const BwdLaunch l = clean_launch<T, TO, N, TILED>((int)p_in.g.Bs, dev);
   BwdParams p = p_in;
   p.seg_resident = l.resident;
-  e = set_bwd_attrs(k_bwd_clean<T, TO, N>, l.smem);
+  e = set_bwd_attrs(k_bwd_clean<T, TO, N, TILED>, l.smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc, (unsigned)p.g.Bt);
-  k_bwd_clean<T, TO, N><<<grid, kCta, l.smem, s>>>(p);
+  k_bwd_clean<T, TO, N, TILED><<<grid, kCta, l.smem, s>>>(p);
   return cudaGetLastError();
+}
+template <typename T, typename TO, int N>
+cudaError_t bwd_clean_t(const BwdParams& p, cudaStream_t s) {
+  return p.g.Bs < kBwdTS ? bwd_clean_tt<T, TO, N, true>(p, s) : bwd_clean_tt<T, TO, N, false>(p, s);
 }
 
 }  // namespace
