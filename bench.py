@@ -14,7 +14,8 @@ step line: the block-size sweep at d_inner 2048 (forward+backward for block
 4, 8, 16, 32, 64), and the inference cache path: boundary_states over a
 65,536-token prefix (block 32) or a 262,144-token prefix (block 16), then
 active-block calls from the cached state, each call timed on its own and all
-calls replayed as one CUDA graph.
+calls replayed as one CUDA graph, and the cost of the same layer step without
+the cache (full-sequence bidirectional scan).
 
 Under torchrun each rank runs an independent replica on its own GPU (the
 scan needs no exchange between replicas); the elapsed time is the maximum
@@ -445,7 +446,10 @@ def run_prefill(args, L, Bs, calls):
     """Inference cache path at d_inner 2048, d_state 16, batch 1: the cache
     build over an L-token clean prefix (final state only, and every block-end
     state plus the clean outputs), then `calls` active-block calls from the
-    cached state, each timed on its own and all replayed as one CUDA graph."""
+    cached state, each timed on its own and all replayed as one CUDA graph,
+    against the same layer step without a cache (a full-sequence
+    bidirectional scan over the L tokens, as a DiffuMamba sampler must run
+    at every denoising step)."""
     import torch
     from paper_2607_02805_gb300 import binding
     from paper_2607_02805_gb300.inputs import Workload
@@ -538,7 +542,36 @@ def run_prefill(args, L, Bs, calls):
         graph_us = 1e3 * e0.elapsed_time(e1) / (reps * calls)
     except Exception as exc:  # report the failure in the line, keep the rest
         graph_us = f"capture failed: {exc}"
+    # the same layer step without the cache: a full-sequence bidirectional
+    # layer (DiffuMamba) rescans the whole sequence in both directions at every
+    # denoising step, because its reverse states depend on the active block
+    tf = {"x_n": t["x_c"], "dt_f": t["dt_c"], "B_f": t["B_c"], "C_f": t["C_c"], "dt_r": t["dt_c"],
+          "B_r": t["B_c"], "C_r": t["C_c"], "A_f": t["A_f"], "D_f": t["D_f"], "A_r": t["A_f"], "D_r": t["D_f"]}
+    y_full = torch.empty((1, L, D), dtype=torch.bfloat16, device="cuda")
+    fbytes = binding.bdscan_full_bidir_workspace_size(dims)
+    ws_full = torch.empty(max(1, (fbytes + 3) // 4), dtype=torch.float32, device="cuda")
+    for _ in range(2):
+        binding.full_bidir_forward(dims, tf, y_full, ws_full, stream)
+    reps = 5
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        binding.full_bidir_forward(dims, tf, y_full, ws_full, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    full_ms = e0.elapsed_time(e1) / reps
+    del ws_full, y_full
     blk_bytes = Bs * (D * 2 + 2 * D * 2 + 4 * N * 2 + D * 2) + D * N * 4
+    graph_us_num = graph_us if isinstance(graph_us, float) else statistics.median(per_call)
+    print(json.dumps({
+        "metric": "layer step per denoising step: full-sequence bidirectional (no cache) over cached active block",
+        "value": full_ms * 1e3 / graph_us_num, "unit": "x", "n_gpus": 1, "higher_is_better": True,
+        "dtype": "f32 state, bf16 I/O", "data": "synthetic",
+        "config": {"workload": f"one layer at a {L}-token context, block {Bs}, d_inner 2048, d_state 16, batch 1: "
+                               "bdscan_full_bidir_forward over the whole sequence vs bdscan_active_block from "
+                               "the cached state (in a CUDA graph)", "context": L, "block": Bs},
+        "full_bidir_ms": round(full_ms, 4), "active_block_us": round(graph_us_num, 3)}), flush=True)
     print(json.dumps({
         "metric": "active-block call latency (bdscan_active_block)", "value": statistics.median(per_call),
         "unit": "us per call", "n_gpus": 1, "higher_is_better": False, "dtype": "f32 state, bf16 I/O",

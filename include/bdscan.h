@@ -213,11 +213,30 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
 /* ---------------------------------------------------------------------- */
 /* seed [Bt][D][N] fp32 is read only (reused across denoising steps). The
  * noisy tensors hold one block: x, dt_* [Bt][Bs][D], B_*, C_* [Bt][Bs][N].
- * Writes y_n [Bt][Bs][D]. The block computation is the same device code as
- * the noisy blocks of bdscan_forward, so outputs are bit-identical to the
- * forward's outputs for the same block and the same seed. */
+ * Writes y_n [Bt][Bs][D]. Each channel goes through the same arithmetic, in
+ * the same order, as the noisy blocks of bdscan_forward, so outputs are
+ * bit-identical to the forward's outputs for the same block and seed. */
 int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan_noisy* noisy,
                         const bdscan_params* params, void* y_n, void* stream);
+
+/* ---------------------------------------------------------------------- */
+/* Full-sequence bidirectional layer (Sec. 4: the fully bidirectional Mamba */
+/* denoiser of DiffuMamba, a forward scan and a reverse scan over the whole */
+/* sequence, which the block partial-reverse design replaces). A comparator */
+/* for the cache: its reverse states depend on every later token, so a     */
+/* sampler must rerun it over the whole sequence at every denoising step.   */
+/* ---------------------------------------------------------------------- */
+size_t bdscan_full_bidir_workspace_size(const bdscan_dims* dims);
+
+/* y [Bt][L][D] (out_dtype) = forward scan of (x, dt_f, B_f, C_f; A_f, D_f)
+ * from a zero state at token 0 plus reverse scan of (x, dt_r, B_r, C_r;
+ * A_r, D_r) from a zero state at token L-1, each with its own D x term;
+ * noisy.x is the input of both directions. dims.block only sets the time
+ * chunking of the scans (no block restriction applies); the usual block
+ * limits hold. Each direction's output is kept in fp32 in the workspace
+ * before the sum is rounded. */
+int bdscan_full_bidir_forward(const bdscan_dims* dims, const bdscan_noisy* noisy, const bdscan_params* params,
+                              void* y, void* workspace, size_t workspace_bytes, void* stream);
 
 /* ---------------------------------------------------------------------- */
 /* Cache build for callers that cannot allocate device memory. The paper    */

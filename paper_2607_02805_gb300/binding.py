@@ -84,6 +84,9 @@ SIGNATURES = [
      [_P(bdscan_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
     ("bdscan_boundary_states_noalloc", ctypes.c_int,
      [_P(bdscan_dims), _P(bdscan_clean), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, ctypes.c_int, c_void_p]),
+    ("bdscan_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_full_bidir_forward", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
 ]
 
 BDSCAN_NOALLOC_SCRATCH_BYTES = 32 << 20
@@ -191,6 +194,15 @@ def bdscan_boundary_states_noalloc(dims, clean, A_f, D_f, init_state, y_c, state
                                                  int(emit_all), stream)
 
 
+def bdscan_full_bidir_workspace_size(dims) -> int:
+    return load().bdscan_full_bidir_workspace_size(_ref(dims))
+
+
+def bdscan_full_bidir_forward(dims, noisy, params, y, workspace, workspace_bytes, stream):
+    return load().bdscan_full_bidir_forward(_ref(dims), _ref(noisy), _ref(params), y, workspace,
+                                            workspace_bytes, stream)
+
+
 # ---------------------------------------------------------------------------
 # torch-tensor helpers (marshalling only)
 # ---------------------------------------------------------------------------
@@ -263,3 +275,11 @@ def boundary_states(dims, t, init_state, y_c, states, emit_all, workspace, strea
 def active_block(dims, seed, t, y_n, stream=None):
     _call("bdscan_active_block", ctypes.byref(dims), _ptr(seed), ctypes.byref(make_noisy(t)),
           ctypes.byref(make_params(t)), _ptr(y_n), _stream(stream))
+
+
+def full_bidir_forward(dims, t, y, workspace, stream=None):
+    """Full-sequence bidirectional layer (no block restriction) of the noisy
+    tensors in t; y [Bt][L][D]."""
+    _call("bdscan_full_bidir_forward", ctypes.byref(dims), ctypes.byref(make_noisy(t)), ctypes.byref(make_params(t)),
+          _ptr(y), _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
+          _stream(stream))

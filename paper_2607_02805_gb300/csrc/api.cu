@@ -367,6 +367,54 @@ int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan
   return ok();
 }
 
+size_t bdscan_full_bidir_workspace_size(const bdscan_dims* dims) {
+  Call c;
+  if (check_dims(dims, &c, "bdscan_full_bidir_workspace_size") != BDSCAN_OK) return 0;
+  const size_t y32 = al256((size_t)c.g.Bt * c.g.L * c.g.D * 4);
+  return fwd_ws(c.g, c.N) + 2 * y32;
+}
+
+int bdscan_full_bidir_forward(const bdscan_dims* dims, const bdscan_noisy* noisy, const bdscan_params* params,
+                              void* y, void* workspace, size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_full_bidir_forward";
+  Call c;
+  int rc = check_dims(dims, &c, fn);
+  if (rc) return rc;
+  if ((rc = check_block_limits(c, false, fn))) return rc;
+  if (c.g.Bt == 0 || c.g.L == 0) return ok();
+  if ((rc = check_noisy(noisy, fn)) || (rc = check_params(params, fn))) return rc;
+  REQ(y, fn, "y");
+  const size_t y32 = al256((size_t)c.g.Bt * c.g.L * c.g.D * 4), fws = fwd_ws(c.g, c.N);
+  REQ(workspace, fn, "workspace");
+  if (workspace_bytes < fws + 2 * y32)
+    return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, fws + 2 * y32);
+  cudaStream_t s = (cudaStream_t)stream;
+  float* yf = (float*)((char*)workspace + fws);
+  float* yr = (float*)((char*)workspace + fws + y32);
+  const int dt_scan = c.dt == 0 ? 0 : 2;  // fp32 outputs of each direction
+  for (int dir = 0; dir < 2; ++dir) {
+    bds::FwdParams p;
+    memset(&p, 0, sizeof(p));
+    p.g = c.g;
+    p.xc = noisy->x;
+    p.dtc = dir == 0 ? noisy->dt_f : noisy->dt_r;
+    p.Bc = dir == 0 ? noisy->B_f : noisy->B_r;
+    p.Cc = dir == 0 ? noisy->C_f : noisy->C_r;
+    p.Af = dir == 0 ? params->A_f : params->A_r;
+    p.Df = dir == 0 ? params->D_f : params->D_r;
+    p.yc = dir == 0 ? yf : yr;
+    p.rev = dir;
+    p.hst = (float*)workspace;  // the chunk states of one direction, then of the other
+    p.sdt = (float*)((char*)workspace + al256((size_t)c.g.Bt * (c.g.nc + 1) * c.g.D * c.N * 4));
+    if ((rc = run_chunk_states(c, p, s, fn))) return rc;
+    cudaError_t e = launched(bds::launch_block_scan(dt_scan, c.N, dir == 0 ? 1 : 2, c.g.nc, p, s), s);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+  }
+  cudaError_t e = launched(bds::launch_combine(c.dt != 1, yf, yr, y, c.g.Bt * c.g.L * c.g.D, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
 int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
                     const bdscan_params* params, const float* states, const void* dy_c, const void* dy_n,
                     const float* dstates, const bdscan_clean_grads* gclean, const bdscan_noisy_grads* gnoisy,

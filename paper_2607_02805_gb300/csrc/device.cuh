@@ -58,10 +58,11 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
 // Copies `nsteps` token rows of a token-by-channel tensor g [.., D] for the
-// channels [d0, d0+128) into tile[step][128]. Channels >= D read as zero; a
-// null tensor stages zeros. Row starts are 16-byte aligned because D is a
-// multiple of 16/sizeof(T) (checked on the host).
-template <typename T>
+// channels [d0, d0+128) into tile[step][128]: step r is row row0 + r, or
+// row0 - r with REV (a span staged in reversed time). Channels >= D read as
+// zero; a null tensor stages zeros. Row starts are 16-byte aligned because D
+// is a multiple of 16/sizeof(T) (checked on the host).
+template <typename T, bool REV = false>
 __device__ __forceinline__ void issue_td(T* tile, const T* g, int64_t row0, int nsteps, int64_t D,
                                          int64_t d0) {
   constexpr int E = 16 / (int)sizeof(T);
@@ -75,22 +76,28 @@ __device__ __forceinline__ void issue_td(T* tile, const T* g, int64_t row0, int 
       *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
     } else {
       const bool ok = d < D;
-      cp_async16(dst, ok ? (const void*)(g + (row0 + r) * D + d) : (const void*)g, ok ? 16 : 0);
+      cp_async16(dst, ok ? (const void*)(g + (REV ? row0 - r : row0 + r) * D + d) : (const void*)g, ok ? 16 : 0);
     }
   }
 }
 
-// Copies nsteps*N contiguous elements (token-by-state rows) starting at row0.
-template <typename T, int N>
+// Copies nsteps token-by-state rows [N] into dst[step][N]: step r is row
+// row0 + r, or row0 - r with REV.
+template <typename T, int N, bool REV = false>
 __device__ __forceinline__ void issue_rows(T* dst, const T* g, int64_t row0, int nsteps) {
   constexpr int E = 16 / (int)sizeof(T);
   static_assert((N * sizeof(T)) % 16 == 0, "state rows must be whole 16-byte chunks");
-  const int total = nsteps * N / E;
+  constexpr int RPC = N / E;  // 16-byte chunks per row
+  const int total = nsteps * RPC;
   for (int i = threadIdx.x; i < total; i += kCta) {
-    if (g == nullptr)
+    if (g == nullptr) {
       *reinterpret_cast<uint4*>(dst + i * E) = make_uint4(0u, 0u, 0u, 0u);
-    else
+    } else if (REV) {
+      const int r = i / RPC, q = i - r * RPC;
+      cp_async16(dst + i * E, g + (row0 - r) * N + q * E, 16);
+    } else {
       cp_async16(dst + i * E, g + row0 * N + (int64_t)i * E, 16);
+    }
   }
 }
 
@@ -100,8 +107,10 @@ __device__ __forceinline__ void cp_async_wait_one() { asm volatile("cp.async.wai
 // shared-memory buffers. With two buffers the next span is copied while the
 // current one is processed: issue(next) ... complete(current, pending = 1).
 // TSMAX > 0 fixes the span stride at compile time (every staged address is
-// then a base plus an immediate); 0 takes it from carve().
-template <typename T, int N, int NTD, int NROW, int NBUF = 1, int TSMAX = 0>
+// then a base plus an immediate); 0 takes it from carve(). REV stages spans in
+// reversed time: issue's row0 is the row of the span's first step and the
+// following steps are the rows below it.
+template <typename T, int N, int NTD, int NROW, int NBUF = 1, int TSMAX = 0, bool REV = false>
 struct Stage {
   unsigned char* base;
   int tsmax;
@@ -142,9 +151,9 @@ struct Stage {
     T* t = td(buf);
     T* r = raw(buf);
 #pragma unroll
-    for (int j = 0; j < NTD; ++j) issue_td<T>(t + (size_t)j * stride() * kCta, td_src[j], row0, nsteps, D, d0);
+    for (int j = 0; j < NTD; ++j) issue_td<T, REV>(t + (size_t)j * stride() * kCta, td_src[j], row0, nsteps, D, d0);
 #pragma unroll
-    for (int j = 0; j < NROW; ++j) issue_rows<T, N>(r + (size_t)j * stride() * N, row_src[j], row0, nsteps);
+    for (int j = 0; j < NROW; ++j) issue_rows<T, N, REV>(r + (size_t)j * stride() * N, row_src[j], row0, nsteps);
     cp_async_commit();
   }
   // Waits for the copies of buffer `buf` (with `pending` newer groups still in

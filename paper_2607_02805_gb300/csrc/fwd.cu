@@ -35,7 +35,8 @@ constexpr int kLocalSpan = 32;  // tokens staged per step of the chunk-local sca
 // 16-token block).
 constexpr int kScanSeg = 16;
 
-template <typename T, int N>
+// REV: the scan runs right to left in time (logical token t is row L-1-t).
+template <typename T, int N, bool REV>
 __global__ void __launch_bounds__(kCta) k_chunk_local(const FwdParams p) {
   extern __shared__ __align__(16) unsigned char smem[];
   const Geo& g = p.g;
@@ -43,8 +44,9 @@ __global__ void __launch_bounds__(kCta) k_chunk_local(const FwdParams p) {
   const int c = blockIdx.y;
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
   const bool act = d < g.D;
-  Stage<T, N, 2, 1, 2> st;
+  Stage<T, N, 2, 1, 2, 0, REV> st;
   st.carve(smem, kLocalSpan);
+  auto prow = [&](int64_t t) { return b * g.L + (REV ? g.L - 1 - t : t); };  // row of logical token t
   st.td_src[0] = (const T*)p.xc;
   st.td_src[1] = (const T*)p.dtc;
   st.row_src[0] = (const T*)p.Bc;
@@ -61,14 +63,14 @@ __global__ void __launch_bounds__(kCta) k_chunk_local(const FwdParams p) {
   const int64_t tc = (int64_t)g.m * g.Bs;
   const int64_t tbeg = (int64_t)c * tc;
   const int nspan = (int)((tc + kLocalSpan - 1) / kLocalSpan);
-  st.issue(0, b * g.L + tbeg, (int)(tc < kLocalSpan ? tc : kLocalSpan), g.D, d0);
+  st.issue(0, prow(tbeg), (int)(tc < kLocalSpan ? tc : kLocalSpan), g.D, d0);
   for (int sp = 0; sp < nspan; ++sp) {
     const int64_t t = (int64_t)sp * kLocalSpan;
     const int ns = (int)((tc - t) < kLocalSpan ? (tc - t) : kLocalSpan);
     __syncthreads();  // the other buffer is no longer read
     if (sp + 1 < nspan) {
       const int64_t tn = t + kLocalSpan;
-      st.issue((sp + 1) & 1, b * g.L + tbeg + tn, (int)((tc - tn) < kLocalSpan ? (tc - tn) : kLocalSpan), g.D, d0);
+      st.issue((sp + 1) & 1, prow(tbeg + tn), (int)((tc - tn) < kLocalSpan ? (tc - tn) : kLocalSpan), g.D, d0);
     }
     st.complete(sp & 1, ns, sp + 1 < nspan ? 1 : 0);
 #pragma unroll 4
@@ -120,10 +122,12 @@ __global__ void __launch_bounds__(256) k_chunk_carry(const FwdParams p) {
 }
 
 // MODE 0: all-block forward (clean + noisy). MODE 1: clean scan only (cache
-// build). The active block has its own kernel (k_active_block).
+// build). MODE 2: clean scan only, right to left in time (logical token t is
+// row L-1-t; the reverse direction of a full-sequence bidirectional layer).
+// The active block has its own kernel (k_active_block).
 template <int MODE>
 struct ScanLayout {
-  static_assert(MODE == 0 || MODE == 1, "block scan modes");
+  static_assert(MODE >= 0 && MODE <= 2, "block scan modes");
   static constexpr bool kClean = true;
   static constexpr bool kNoisy = MODE == 0;
   static constexpr int NTD = MODE == 0 ? 5 : 2;
@@ -151,10 +155,13 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   // blocks shorter than kScanSeg are staged TB at a time (one tile of at most
   // kScanSeg tokens), so the staging and its barriers are paid per tile
   const int TB = TILED ? kScanSeg / Bs : 1;
-  Stage<T, N, Ly::NTD, Ly::NROW, 2> st;
+  constexpr bool kRev = MODE == 2;
+  Stage<T, N, Ly::NTD, Ly::NROW, 2, 0, kRev> st;
   st.carve(smem, NSEG == 1 ? TB * Bs : SEG);
+  // the row holding logical row x = b L + t (t reversed in time for MODE 2)
+  auto prow = [&](int64_t x) { return kRev ? 2 * b * g.L + g.L - 1 - x : x; };
   const bool dbuf = p.stage_bufs == 2 && NSEG == 1;
-  float* yfbuf = reinterpret_cast<float*>(smem + Stage<T, N, Ly::NTD, Ly::NROW, 2>::buf_bytes(st.stride()) *
+  float* yfbuf = reinterpret_cast<float*>(smem + decltype(st)::buf_bytes(st.stride()) *
                                                        (dbuf ? 2 : 1));
   if (Ly::kClean) {
     st.td_src[Ly::XC] = (const T*)p.xc;
@@ -197,17 +204,17 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   if (act) vload2<N>(hc, p.hst + ((b * (g.nc + 1) + c) * g.D + d) * N, 0);
 
   auto tile_blocks = [&](int k0) { return k_hi - k0 + 1 < TB ? k_hi - k0 + 1 : TB; };
-  if (dbuf) st.issue(0, b * g.L + (int64_t)k_lo * Bs, tile_blocks(k_lo) * Bs, g.D, d0);
+  if (dbuf) st.issue(0, prow(b * g.L + (int64_t)k_lo * Bs), tile_blocks(k_lo) * Bs, g.D, d0);
   for (int k0 = k_lo; k0 <= k_hi; k0 += TB) {
     const int nbk = tile_blocks(k0), tile = (k0 - k_lo) / TB;
     const int64_t trow = b * g.L + (int64_t)k0 * Bs;
     if (dbuf) {
       __syncthreads();  // the other buffer is no longer read
       const int k1 = k0 + TB;
-      if (k1 <= k_hi) st.issue((tile + 1) & 1, trow + (int64_t)nbk * Bs, tile_blocks(k1) * Bs, g.D, d0);
+      if (k1 <= k_hi) st.issue((tile + 1) & 1, prow(trow + (int64_t)nbk * Bs), tile_blocks(k1) * Bs, g.D, d0);
       st.complete(tile & 1, nbk * Bs, k1 <= k_hi ? 1 : 0);
     } else if (NSEG == 1) {
-      st.load(trow, nbk * Bs, g.D, d0);
+      st.load(prow(trow), nbk * Bs, g.D, d0);
     }
     for (int kk = 0; kk < nbk; ++kk) {
       const int k = k0 + kk;
@@ -218,11 +225,11 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
       for (int j = 0; j < N / 2; ++j) hs[j] = hc[j];  // the block's seed: state before its first token
       for (int sg = 0; sg < NSEG; ++sg) {  // segments left to right
         const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
-        if (NSEG > 1) st.load(row0 + i0, ns, g.D, d0);
+        if (NSEG > 1) st.load(prow(row0 + i0), ns, g.D, d0);
 #pragma unroll 4
         for (int ii = 0; ii < ns; ++ii) {
           const int i = i0 + ii;
-          const int64_t o = (row0 + i) * g.D + d;
+          const int64_t o = prow(row0 + i) * g.D + d;
           if (Ly::kClean) {
             const float x = st.at(Ly::XC, toff + ii), dt = st.at(Ly::DTC, toff + ii);
             const float y = scan_step<N>(hc, A2f, dt, x, st.row(Ly::BC, toff + ii), st.row(Ly::CC, toff + ii));
@@ -250,11 +257,11 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
         vzero2<N>(hr);
         for (int sg = NSEG - 1; sg >= 0; --sg) {  // segments right to left; the last is still staged
           const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
-          if (sg < NSEG - 1) st.load(row0 + i0, ns, g.D, d0);
+          if (sg < NSEG - 1) st.load(prow(row0 + i0), ns, g.D, d0);
 #pragma unroll 4
           for (int ii = ns - 1; ii >= 0; --ii) {
             const int i = i0 + ii;
-            const int64_t o = (row0 + i) * g.D + d;
+            const int64_t o = prow(row0 + i) * g.D + d;
             const float x = st.at(Ly::XN, toff + ii), dt = st.at(Ly::DTR, toff + ii);
             const float y = scan_step<N>(hr, A2r, dt, x, st.row(Ly::BR, toff + ii), st.row(Ly::CR, toff + ii));
             if (act)
@@ -388,18 +395,39 @@ __global__ void __launch_bounds__(2 * kActW, 1) k_active_block(const FwdParams p
 }
 
 // ---------------------------------------------------------------------------
+// Sum of the two directions of a full-sequence bidirectional layer: each fp32
+// input already holds its direction's output with its own skip term.
+// ---------------------------------------------------------------------------
+template <typename TO>
+__global__ void __launch_bounds__(256) k_combine(const float* yf, const float* yr, TO* y, int64_t n4) {
+  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;  // four elements each
+  if (i >= n4) return;
+  const float4 a = reinterpret_cast<const float4*>(yf)[i], r = reinterpret_cast<const float4*>(yr)[i];
+  TO* o = y + 4 * i;
+  o[0] = to_out<TO>(combine_dirs(a.x, r.x));
+  o[1] = to_out<TO>(combine_dirs(a.y, r.y));
+  o[2] = to_out<TO>(combine_dirs(a.z, r.z));
+  o[3] = to_out<TO>(combine_dirs(a.w, r.w));
+}
+
+// ---------------------------------------------------------------------------
 // launchers
 // ---------------------------------------------------------------------------
 namespace {
 
-template <typename T, int N>
-cudaError_t chunk_local_t(const FwdParams& p, cudaStream_t s) {
+template <typename T, int N, bool REV>
+cudaError_t chunk_local_rt(const FwdParams& p, cudaStream_t s) {
   const size_t smem = Stage<T, N, 2, 1, 2>::bytes(kLocalSpan);
-  cudaError_t e = cudaFuncSetAttribute(k_chunk_local<T, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e =
+      cudaFuncSetAttribute(k_chunk_local<T, N, REV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)p.g.G, (unsigned)p.g.nc_full, (unsigned)p.g.Bt);
-  k_chunk_local<T, N><<<grid, kCta, smem, s>>>(p);
+  k_chunk_local<T, N, REV><<<grid, kCta, smem, s>>>(p);
   return cudaGetLastError();
+}
+template <typename T, int N>
+cudaError_t chunk_local_t(const FwdParams& p, cudaStream_t s) {
+  return p.rev ? chunk_local_rt<T, N, true>(p, s) : chunk_local_rt<T, N, false>(p, s);
 }
 
 // Above this much shared memory per CTA the block scan stages synchronously:
@@ -450,6 +478,7 @@ cudaError_t block_scan_mode(int mode, int nchunks, const FwdParams& p, cudaStrea
   switch (mode) {
     case 0: return block_scan_t<T, TO, N, 0>(nchunks, p, s);
     case 1: return block_scan_t<T, TO, N, 1>(nchunks, p, s);
+    case 2: return block_scan_t<T, TO, N, 2>(nchunks, p, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -506,6 +535,17 @@ cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t 
     case 1: BDS_DISPATCH_N(N, return active_block_t<bf16, bf16, NN>(p, s);)
     default: BDS_DISPATCH_N(N, return active_block_t<bf16, float, NN>(p, s);)
   }
+}
+
+cudaError_t launch_combine(int out_f32, const float* yf, const float* yr, void* y, int64_t n, cudaStream_t s) {
+  const int64_t n4 = n / 4;  // D is a multiple of 4
+  if (n4 == 0) return cudaSuccess;
+  const unsigned blocks = (unsigned)((n4 + 255) / 256);
+  if (out_f32)
+    k_combine<float><<<blocks, 256, 0, s>>>(yf, yr, reinterpret_cast<float*>(y), n4);
+  else
+    k_combine<bf16><<<blocks, 256, 0, s>>>(yf, yr, reinterpret_cast<bf16*>(y), n4);
+  return cudaGetLastError();
 }
 
 }  // namespace bds

@@ -35,6 +35,7 @@ struct FwdParams {
   const float* seed;   // active block: [Bt][D][N]
   int c_begin;         // first chunk handled by a block-scan launch
   int stage_bufs;      // block scan: 2 = copy the next block while computing, 1 = synchronous
+  int rev;             // chunk-local scan: right to left in time (with block-scan mode 2)
 };
 
 // Backward-side kernels.
@@ -62,10 +63,12 @@ struct BwdParams {
 // Launchers (fwd.cu / bwd.cu). dt: 0 = f32 in/out, 1 = bf16 in/out, 2 = bf16 in, f32 out.
 cudaError_t launch_chunk_local(int dt, int N, const FwdParams& p, cudaStream_t s);
 cudaError_t launch_chunk_carry(int N, const FwdParams& p, cudaStream_t s);
-// mode 0: all-block forward, 1: clean scan only (cache build)
+// mode 0: all-block forward, 1: clean scan only (cache build), 2: clean scan right to left
 cudaError_t launch_block_scan(int dt, int N, int mode, int nchunks, const FwdParams& p, cudaStream_t s);
 // One noisy block per batch row from p.seed (len == block).
 cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t s);
+// y = yf + yr elementwise (n elements, a multiple of 4), rounded to f32 or bf16.
+cudaError_t launch_combine(int out_f32, const float* yf, const float* yr, void* y, int64_t n, cudaStream_t s);
 cudaError_t launch_bwd_noisy(int dt, int N, const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_carry(int N, const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_clean(int dt, int N, const BwdParams& p, cudaStream_t s);

@@ -136,6 +136,23 @@ def test_boundary_states_checks():
     assert rc == binding.BDSCAN_ERR_ARG and "A_f is NULL" in binding.bdscan_last_error()
 
 
+def test_full_bidir_checks_and_workspace():
+    d = _dims(batch=2, length=64, block=16, d_inner=32, d_state=16)
+    al = lambda x: (x + 255) // 256 * 256
+    # the chunk states of one direction at a time, and each direction's fp32 output
+    assert binding.bdscan_full_bidir_workspace_size(d) == (binding.bdscan_forward_workspace_size(d)
+                                                           + 2 * al(2 * 64 * 32 * 4))
+    _, n, p = _structs()
+    n.dt_r = None
+    rc = binding.bdscan_full_bidir_forward(d, n, p, FAKE, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "noisy.dt_r is NULL" in binding.bdscan_last_error()
+    _, n, p = _structs()
+    rc = binding.bdscan_full_bidir_forward(d, n, p, FAKE, FAKE, 64, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "workspace" in binding.bdscan_last_error()
+    rc = binding.bdscan_full_bidir_forward(_dims(length=60), n, p, FAKE, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG
+
+
 def test_fails_loudly_without_a_gpu():
     torch = pytest.importorskip("torch")
     if torch.cuda.is_available():

@@ -193,6 +193,38 @@ def test_zero_size_calls_are_noops():
 
 
 # ---------------------------------------------------------------------------
+# full-sequence bidirectional layer (the DiffuMamba comparator)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("Bt,L,Bs,D,N,dt,od,seed", [
+    (2, 512, 16, 136, 16, "bf16", None, 31),               # ragged channel group
+    (1, 400, 16, 64, 8, "f32", None, 32),                  # ragged last chunk, N = 8
+    (2, 384, 32, 128, 16, "bf16", binding.BDSCAN_F32, 33),  # 32-token chunking blocks, fp32 output
+    (1, 256, 4, 64, 16, "bf16", None, 34),                 # tiled 4-token chunking blocks
+])
+def test_full_bidir_matches_oracle(Bt, L, Bs, D, N, dt, od, seed):
+    """Forward and reverse scans over the whole sequence: the oracle's
+    all-block forward with one block spanning the sequence (its noisy output
+    is exactly that layer; the block size of the call only sets the chunking)."""
+    import oracle
+    wl = Workload(Bt, L, Bs, D, N, dtype=dt, seed=seed, with_grads=False, parts=("noisy",))
+    code = binding.BDSCAN_F32 if dt == "f32" else binding.BDSCAN_BF16
+    dims = binding.make_dims(Bt, L, Bs, D, N, code, od)
+    t = {k: to_device(wl.dev_bits(k), code, "cuda") for k in wl.t32}
+    out_t = torch.float32 if (dt == "f32" or od == binding.BDSCAN_F32) else torch.bfloat16
+    y = torch.full((Bt, L, D), float("nan"), dtype=out_t, device="cuda")
+    nbytes = binding.bdscan_full_bidir_workspace_size(dims)
+    ws = torch.empty((nbytes + 3) // 4, dtype=torch.float32, device="cuda")
+    binding.full_bidir_forward(dims, t, y, ws)
+    torch.cuda.synchronize()
+    d = P.slice_channels(wl, None)
+    zeros = np.zeros_like(d["x_n"])
+    zrow = np.zeros_like(d["B_f"])
+    _, y_n, _ = oracle.forward(L, zeros, zeros, zrow, zrow, d["x_n"], d["dt_f"], d["B_f"], d["C_f"], d["dt_r"],
+                               d["B_r"], d["C_r"], d["A_f"], d["D_f"], d["A_r"], d["D_r"])
+    P.assert_close("y", to_numpy(y), y_n, P.FWD_TOL, P.BF16_U if out_t == torch.bfloat16 else 0.0)
+
+
+# ---------------------------------------------------------------------------
 # full-size configurations, in the launch configuration the benchmark times
 # ---------------------------------------------------------------------------
 def _batch_row(wl, b):
