@@ -583,34 +583,61 @@ def run_prefill(args, L, Bs, calls):
 
 
 def run_e2e(lay, wl, stream, dev, args):
-    """Forward + backward through the C ABI with host (pinned) inputs and a
-    device-to-host read of every output and gradient, timed per step."""
+    """Forward + backward through the C ABI end to end: every step copies its
+    inputs from pinned host memory to the device and reads every output and
+    gradient back, as a training loop streaming its batches would. Copies run
+    on their own streams and two device buffer sets alternate, so that step
+    i+1's inputs go up and step i-1's results come down while step i computes.
+    The timed region covers all copies of every step."""
     import torch
+    from paper_2607_02805_gb300.layer import Layer
+    lays = [lay, Layer(wl, device=dev)]
+    lays[1].alloc_backward()
     ins = [k for k in wl.t32]
     host_in = {k: lay.t[k].detach().to("cpu").pin_memory() for k in ins}
-    outs = [lay.y_c, lay.y_n] + [lay.g[k] for k in lay.g]
-    host_out = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    outs = [[la.y_c, la.y_n] + [la.g[k] for k in la.g] for la in lays]
+    host_out = [[torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs[0]] for _ in range(2)]
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
-    d2h = sum(t.numel() * t.element_size() for t in host_out)
-    steps = max(3, min(args.steps, 20))
+    d2h = sum(t.numel() * t.element_size() for t in host_out[0])
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    steps = max(4, min(args.steps, 20))
 
-    def one():
-        for k in ins:
-            lay.t[k].copy_(host_in[k], non_blocking=True)
-        lay.forward(stream)
-        lay.backward(stream, use_dstates=False)
-        for o, h in zip(outs, host_out):
-            h.copy_(o, non_blocking=True)
+    def run(n):
+        ev_in = [torch.cuda.Event() for _ in range(n)]
+        ev_comp = [torch.cuda.Event() for _ in range(n)]
+        ev_out = [torch.cuda.Event() for _ in range(n)]
+        for i in range(n):
+            j = i % 2
+            la = lays[j]
+            if i >= 2:
+                s_in.wait_event(ev_comp[i - 2])  # this buffer set's inputs are no longer read
+            with torch.cuda.stream(s_in):
+                for k in ins:
+                    la.t[k].copy_(host_in[k], non_blocking=True)
+            ev_in[i].record(s_in)
+            stream.wait_event(ev_in[i])
+            if i >= 2:
+                stream.wait_event(ev_out[i - 2])  # its outputs have been read back
+            la.forward(stream)
+            la.backward(stream, use_dstates=False)
+            ev_comp[i].record(stream)
+            s_out.wait_event(ev_comp[i])
+            with torch.cuda.stream(s_out):
+                for o, h in zip(outs[j], host_out[j]):
+                    h.copy_(o, non_blocking=True)
+            ev_out[i].record(s_out)
+        stream.wait_event(ev_out[n - 1])
 
-    for _ in range(3):
-        one()
+    run(3)
     torch.cuda.synchronize(dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(steps):
-        one()
+    s_in.wait_event(e0)
+    s_out.wait_event(e0)
+    run(steps)
     e1.record(stream)
     torch.cuda.synchronize(dev)
+    del lays[1]
     return {"ms": e0.elapsed_time(e1) / steps, "h2d": h2d, "d2h": d2h}
 
 
