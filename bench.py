@@ -82,7 +82,7 @@ def kernel_bytes(Bt, L, D, N, Bs, in_b=2, out_b=2):
 # `ncu --set full` capture at batch 4 (profiles/k_bwd_noisy_87m_layer_batch4.md),
 # scaled by batch / 4: the kernel's traffic is proportional to the batch. Set
 # to None whenever the kernel changes until it is captured again.
-MEASURED_TRAFFIC_BATCH4 = {"bwd_noisy": 331_150_336}
+MEASURED_TRAFFIC_BATCH4 = {"bwd_noisy": 330_220_544}
 
 # FP32 work per (token, channel, state) element of each scan kernel, counted
 # from the kernel's arithmetic (FMA = 2 flops; ex2, mul, add, reduction add = 1).

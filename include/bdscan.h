@@ -5,7 +5,7 @@
  *
  * The layer (Sec. 4 of the paper):
  *   - a causal forward selective scan over the clean token stream
- *     (Sec. 2, eq. mamba-scan-background, with A_t = exp(dt_t * A) for a
+ *     (Sec. 3, eq. mamba-scan-background, with A_t = exp(dt_t * A) for a
  *     diagonal A holding one decay per channel d and state index n), whose
  *     state at every block end is the exact prefix cache
  *     s_k = F_fwd(c^(k))                          (eq. boundary-state);
@@ -192,7 +192,7 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
                     void* workspace, size_t workspace_bytes, void* stream);
 
 /* ---------------------------------------------------------------------- */
-/* Cache build / append (Sec. 2 cache interface: a clean forward pass over  */
+/* Cache build / append (Sec. 3 cache interface: a clean forward pass over  */
 /* finalised blocks; eq. boundary-state).                                  */
 /* ---------------------------------------------------------------------- */
 size_t bdscan_boundary_states_workspace_size(const bdscan_dims* dims, int emit_all);
@@ -207,7 +207,7 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
                            int emit_all, void* workspace, size_t workspace_bytes, void* stream);
 
 /* ---------------------------------------------------------------------- */
-/* Cached active-block denoising step (Sec. 2: denoise the current block    */
+/* Cached active-block denoising step (Sec. 3: denoise the current block    */
 /* while reading the prefix cache; Sec. 4: the cache stays valid because the */
 /* reverse scan is local). dims.len must equal dims.block.                  */
 /* ---------------------------------------------------------------------- */

@@ -10,7 +10,7 @@
  *
  * What it computes, in the paper's terms:
  *
- *  - The selective update of Sec. 2 (eq. mamba-scan-background),
+ *  - The selective update of Sec. 3 (eq. mamba-scan-background),
  *        s_t = A_t s_{t-1} + B_t x_t,   y_t = C_t s_t + D x_t,
  *    with the Mamba-1 discretisation A_t = exp(dt_t * A) for a diagonal A
  *    holding one decay per (channel d, state n), and B_t x_t read as

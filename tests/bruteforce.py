@@ -6,7 +6,7 @@ positions between s and t) times the input at s, with the sums of dt formed
 explicitly for each (t, s) pair. Nothing here runs a recurrence, so an error
 in the oracle's step order, indexing or seeding shows up as a mismatch.
 
-For the selective update of Sec. 2 with a_t = exp(dt_t A):
+For the selective update of Sec. 3 with a_t = exp(dt_t A):
   forward scan:  h_t = sum_{s<=t} exp(A sum_{r=s+1..t} dt_r) dt_s B_s x_s
   reverse scan:  h_t = sum_{s>=t} exp(A sum_{r=t..s-1} dt_r) dt_s B_s x_s
   seeded block:  h_t += exp(A sum_{r=t0..t} dt_r) seed

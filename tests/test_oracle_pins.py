@@ -169,7 +169,7 @@ def test_caching_is_exact(oracle_mod, L, Bs):
 
 def test_cache_append_is_exact(oracle_mod):
     """Appending a finalised block to the cache (a clean pass continued from
-    the cached state, Sec. 2 cache interface) equals scanning the longer
+    the cached state, Sec. 3 cache interface) equals scanning the longer
     prefix from scratch."""
     Bt, L, Bs, D, N = 1, 24, 4, 3, 4
     w = Workload(Bt, L, Bs, D, N, dtype="f32", seed=41, with_grads=False)
