@@ -1,0 +1,118 @@
+/*
+ * bdscan_ssd.h -- C ABI of the Mamba-2 (SSD) form of the block-restricted
+ * bidirectional scan in libbdscan (arXiv 2607.02805, sm_103a).
+ *
+ * The paper's trained BDLM Mamba-H layers are Mamba-2 mixers (Appendix C:
+ * head dimension 64, state 64 or 128, chunk 128; block 256 in Appendix C's
+ * hyperparameter table). In that form the decay is one scalar per head and
+ * B_t, C_t are shared by every channel (one group): for channel p of head h,
+ *   h_t[p, :] = exp(dt_t[h] A[h]) h_{t-1}[p, :] + dt_t[h] x_t[h, p] B_t
+ *   y_t[h, p] = C_t . h_t[p, :] + D[h] x_t[h, p]
+ * (Sec. 3, eq. mamba-scan-background with tied parameters). The block
+ * restriction is the one of bdscan.h (Sec. 4, eqs. boundary-state and
+ * partial-reverse): a clean forward scan whose block-end states are the
+ * prefix cache; every noisy block scanned forward from the clean state at its
+ * start plus a reverse scan confined to the block and started from zero,
+ * outputs summed, each direction with its own dt, B, C, A, D.
+ *
+ * Because the decay is scalar per head, one block's output is a product of
+ * small matrices (the SSD form): y = (L_f o C_f B_f^T + U_r o C_r B_r^T) diag(dt) x
+ * + diag(decay) C_f seed^T + D x, with lower/upper-triangular decay masks
+ * L_f, U_r inside the block. The kernels evaluate these products on the
+ * tcgen05 tensor cores (bf16 operands, fp32 accumulation in TMEM).
+ *
+ * Notation: Bt batch, L tokens per stream, Bs block size, nb = L / Bs,
+ * H heads, P = 64 channels per head, N state size.
+ *
+ * Layouts (row-major, contiguous, no padding):
+ *   x, y             [Bt][L][H][P] bf16
+ *   dt               [Bt][L][H]    bf16 (after softplus)
+ *   B, C             [Bt][L][N]    bf16
+ *   A, D             [H] fp32 (A < 0)
+ *   states           [Bt][nS][H][P][N] fp32; states[b][k] is the clean state
+ *                    after token (k+1)*Bs-1; noisy block k is seeded with
+ *                    states[b][k-1], block 0 with zero.
+ *   seed, init state [Bt][H][P][N] fp32
+ * The structs bdscan_clean, bdscan_noisy and bdscan_params of bdscan.h carry
+ * the pointers, with these layouts.
+ *
+ * Supported shapes: dtype bf16 (inputs and outputs), P = 64, N = 64 or 128,
+ * Bs = 128 or 256, L a multiple of Bs.
+ *
+ * Conventions are those of bdscan.h: device pointers, 16-byte aligned,
+ * caller-owned memory, asynchronous on the given stream, return codes
+ * BDSCAN_OK / BDSCAN_ERR_ARG / BDSCAN_ERR_UNSUPPORTED / BDSCAN_ERR_CUDA with
+ * a thread-local message (bdscan_last_error). The kernels wait on their own
+ * tensor-core work with a bounded number of polls; a wait that gives up sets
+ * a device flag (bdscan_ssd_wait_flag) instead of hanging.
+ */
+#ifndef BDSCAN_SSD_H
+#define BDSCAN_SSD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include "bdscan.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct {
+  int64_t batch;     /* Bt */
+  int64_t len;       /* L, tokens per stream */
+  int64_t block;     /* Bs: 128 or 256 */
+  int64_t heads;     /* H */
+  int64_t head_dim;  /* P: 64 */
+  int64_t d_state;   /* N: 64 or 128 */
+  int32_t dtype;     /* BDSCAN_BF16 */
+} bdscan_ssd_dims;
+
+/* Workspace bytes of bdscan_ssd_forward: the per-block sums of dt of the
+ * clean stream, [Bt][nb][H] fp32. 0 for invalid dims. */
+size_t bdscan_ssd_forward_workspace_size(const bdscan_ssd_dims* dims);
+
+/* All-block forward (Sec. 4.1): clean output y_c, noisy output y_n and every
+ * block-end state of the clean stream.
+ *   clean  x [Bt][L][H][P], dt [Bt][L][H], B, C [Bt][L][N] (bf16);
+ *   noisy  x, dt_f, B_f, C_f, dt_r, B_r, C_r, same layouts;
+ *   params A_f, D_f, A_r, D_r [H] fp32;
+ *   y_c, y_n [Bt][L][H][P] bf16 (written); states [Bt][nb][H][P][N] fp32
+ *   (written); workspace of at least bdscan_ssd_forward_workspace_size. */
+int bdscan_ssd_forward(const bdscan_ssd_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
+                       const bdscan_params* params, void* y_c, void* y_n, float* states, void* workspace,
+                       size_t workspace_bytes, void* stream);
+
+/* Workspace bytes of bdscan_ssd_boundary_states: the dt sums [Bt][nb][H]
+ * fp32, plus the block-local states [Bt][nb][H][P][N] fp32 when only the
+ * final state is emitted. 0 for invalid dims. */
+size_t bdscan_ssd_boundary_states_workspace_size(const bdscan_ssd_dims* dims, int emit_all);
+
+/* Cache build / append (Sec. 3 block-cached decoding; Sec. 4
+ * eq. boundary-state): the clean forward scan from init_state (nullable,
+ * [Bt][H][P][N] fp32; zero if NULL). emit_all != 0 writes every block-end
+ * state, states [Bt][nb][H][P][N]; emit_all == 0 writes the final state only,
+ * states [Bt][1][H][P][N]. y_c (nullable) receives the clean output. The same
+ * kernels as bdscan_ssd_forward, so the states are the same bits. */
+int bdscan_ssd_boundary_states(const bdscan_ssd_dims* dims, const bdscan_clean* clean, const float* A_f,
+                               const float* D_f, const float* init_state, void* y_c, float* states,
+                               int emit_all, void* workspace, size_t workspace_bytes, void* stream);
+
+/* Cached active-block step (Sec. 3: denoise the current block against the
+ * cache; Sec. 4 eq. prefix-cache): one noisy block, len == block, seeded with
+ * the read-only cached state seed [Bt][H][P][N] fp32 (NULL = zero). Writes
+ * y_n [Bt][Bs][H][P] bf16. Same kernel as the noisy blocks of
+ * bdscan_ssd_forward: the outputs equal that call's block bit for bit. */
+int bdscan_ssd_active_block(const bdscan_ssd_dims* dims, const float* seed, const bdscan_noisy* noisy,
+                            const bdscan_params* params, void* y_n, void* stream);
+
+/* The device flag set by a kernel whose bounded wait on its tensor-core work
+ * gave up (0 = never). Synchronises the current device; reset != 0 clears it.
+ * Returns -1 if the flag cannot be read. */
+int bdscan_ssd_wait_flag(int reset);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BDSCAN_SSD_H */

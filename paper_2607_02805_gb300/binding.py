@@ -33,6 +33,12 @@ class bdscan_dims(ctypes.Structure):
                 ("out_dtype", ctypes.c_int32)]
 
 
+class bdscan_ssd_dims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int64), ("len", ctypes.c_int64), ("block", ctypes.c_int64),
+                ("heads", ctypes.c_int64), ("head_dim", ctypes.c_int64), ("d_state", ctypes.c_int64),
+                ("dtype", ctypes.c_int32)]
+
+
 class bdscan_clean(ctypes.Structure):
     _fields_ = [("x", c_void_p), ("dt", c_void_p), ("B", c_void_p), ("C", c_void_p)]
 
@@ -87,6 +93,17 @@ SIGNATURES = [
     ("bdscan_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
     ("bdscan_full_bidir_forward", ctypes.c_int,
      [_P(bdscan_dims), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_ssd_forward_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
+    ("bdscan_ssd_forward", ctypes.c_int,
+     [_P(bdscan_ssd_dims), _P(bdscan_clean), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, c_void_p,
+      c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_ssd_boundary_states_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims), ctypes.c_int]),
+    ("bdscan_ssd_boundary_states", ctypes.c_int,
+     [_P(bdscan_ssd_dims), _P(bdscan_clean), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, ctypes.c_int,
+      c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_ssd_active_block", ctypes.c_int,
+     [_P(bdscan_ssd_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
+    ("bdscan_ssd_wait_flag", ctypes.c_int, [ctypes.c_int]),
 ]
 
 BDSCAN_NOALLOC_SCRATCH_BYTES = 32 << 20
@@ -203,6 +220,32 @@ def bdscan_full_bidir_forward(dims, noisy, params, y, workspace, workspace_bytes
                                             workspace_bytes, stream)
 
 
+def bdscan_ssd_forward_workspace_size(dims) -> int:
+    return load().bdscan_ssd_forward_workspace_size(_ref(dims))
+
+
+def bdscan_ssd_forward(dims, clean, noisy, params, y_c, y_n, states, workspace, workspace_bytes, stream):
+    return load().bdscan_ssd_forward(_ref(dims), _ref(clean), _ref(noisy), _ref(params), y_c, y_n, states,
+                                     workspace, workspace_bytes, stream)
+
+
+def bdscan_ssd_boundary_states_workspace_size(dims, emit_all) -> int:
+    return load().bdscan_ssd_boundary_states_workspace_size(_ref(dims), int(emit_all))
+
+
+def bdscan_ssd_boundary_states(dims, clean, A_f, D_f, init_state, y_c, states, emit_all, workspace,
+                               workspace_bytes, stream):
+    return load().bdscan_ssd_boundary_states(_ref(dims), _ref(clean), A_f, D_f, init_state, y_c, states,
+                                             int(emit_all), workspace, workspace_bytes, stream)
+
+
+def bdscan_ssd_active_block(dims, seed, noisy, params, y_n, stream):
+    return load().bdscan_ssd_active_block(_ref(dims), seed, _ref(noisy), _ref(params), y_n, stream)
+
+
+def bdscan_ssd_wait_flag(reset) -> int:
+    return load().bdscan_ssd_wait_flag(int(reset))
+
 # ---------------------------------------------------------------------------
 # torch-tensor helpers (marshalling only)
 # ---------------------------------------------------------------------------
@@ -283,3 +326,31 @@ def full_bidir_forward(dims, t, y, workspace, stream=None):
     _call("bdscan_full_bidir_forward", ctypes.byref(dims), ctypes.byref(make_noisy(t)), ctypes.byref(make_params(t)),
           _ptr(y), _ptr(workspace), 0 if workspace is None else workspace.numel() * workspace.element_size(),
           _stream(stream))
+
+
+def make_ssd_dims(batch, length, block, heads, d_state, head_dim=64):
+    return bdscan_ssd_dims(int(batch), int(length), int(block), int(heads), int(head_dim), int(d_state),
+                           BDSCAN_BF16)
+
+
+def _nbytes(t):
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def ssd_forward(dims, t, y_c, y_n, states, workspace, stream=None):
+    """SSD-form all-block forward; t holds the tensors in the layouts of
+    include/bdscan_ssd.h, keyed like the diagonal layer's (x_c, ..., D_r)."""
+    _call("bdscan_ssd_forward", ctypes.byref(dims), ctypes.byref(make_clean(t)), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), _ptr(y_c), _ptr(y_n), _ptr(states), _ptr(workspace), _nbytes(workspace),
+          _stream(stream))
+
+
+def ssd_boundary_states(dims, t, init_state, y_c, states, emit_all, workspace, stream=None):
+    _call("bdscan_ssd_boundary_states", ctypes.byref(dims), ctypes.byref(make_clean(t)), _ptr(t["A_f"]),
+          _ptr(t["D_f"]), _ptr(init_state), _ptr(y_c), _ptr(states), int(emit_all), _ptr(workspace),
+          _nbytes(workspace), _stream(stream))
+
+
+def ssd_active_block(dims, seed, t, y_n, stream=None):
+    _call("bdscan_ssd_active_block", ctypes.byref(dims), _ptr(seed), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), _ptr(y_n), _stream(stream))

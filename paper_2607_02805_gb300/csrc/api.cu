@@ -528,6 +528,12 @@ int api_fail(int code, const char* msg) { return fail(code, "%s", msg); }
 
 int api_ok() { return ok(); }
 
+// Kernel-launch bookkeeping for entry points defined in other files: reset at
+// the start of a call, then every launch goes through api_launched.
+void api_begin() { g_launches = 0; }
+
+cudaError_t api_launched(cudaError_t e, cudaStream_t s) { return launched(e, s); }
+
 // Validation shared with other entry points that take forward-side dims.
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn) {
   Call c;

@@ -79,6 +79,8 @@ cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s);
 // Helpers of api.cu for other translation units of the library.
 int api_fail(int code, const char* msg);
 int api_ok();
+void api_begin();
+cudaError_t api_launched(cudaError_t e, cudaStream_t s);
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn);
 size_t api_fwd_workspace(const Geo& g, int N);
 int bwd_chunk_count(int dt, int N, const Geo& g);

@@ -1,0 +1,598 @@
+// ssd.cu -- kernels of the SSD form (Mamba-2: one scalar decay per head,
+// B and C shared by all channels) of the block-restricted bidirectional scan,
+// on the tcgen05 tensor cores of sm_103a.
+//
+// Per block of Bs tokens (Bs = 128 m) and head h, with a_t = exp(dt_t A[h]):
+//   * block-local end state (k_ssd_block_state):
+//       T = sum_s w_s x_s B_s^T, w_s = exp(A sum_{r>s} dt_r) dt_s,
+//     one MMA chain (M = 128 state rows, N = 64 channels, K = Bs tokens) per
+//     head, with A = (w o B)^T split into bf16 high and low parts;
+//   * the exact state at each block end (k_ssd_state_pass):
+//       S_k = exp(A sum_block dt) S_{k-1} + T_k, in fp32, sequential in k;
+//   * the block's output (k_ssd_block_scan), for a 128-token tile t of the block:
+//       y_t = sum_s M[t, s] x_s + exp(A sum_{r<=t} dt_r) C_t . seed + D x_t,
+//       M[t, s] = (C^f_t . B^f_s) exp(A_f sum_{s<r<=t} dt^f_r) dt^f_s  for s <= t
+//               + (C^r_t . B^r_s) exp(A_r sum_{t<=r<s} dt^r_r) dt^r_s  for s >= t
+//     (the reverse term only for noisy blocks). The Gram products C B^T are
+//     shared by all heads and stay in TMEM; each head's decay-weighted M tile
+//     is written to shared memory in bf16 and multiplied with x on the tensor
+//     core; the seed term is a second MMA (seed split into bf16 high and low
+//     parts); the epilogue adds the decayed seed term and D x.
+#include <cstdio>
+
+#include "device.cuh"
+#include "ssd.cuh"
+#include "umma.cuh"
+
+namespace bds {
+namespace {
+
+using umma::sw128;
+
+__device__ int g_ssd_wait_flag;
+
+constexpr uint32_t kTile16 = 16384;  // one atom column of a 128-row operand tile
+
+// Bounded wait shared by all threads of the CTA; a give-up sets the flag and
+// makes every thread see the failure.
+__device__ __forceinline__ bool cta_wait(uint64_t* bar, uint32_t parity, int* flag) {
+  const bool ok = umma::bar_wait(bar, parity);
+  const int bad = __syncthreads_or(ok ? 0 : 1);
+  if (bad && threadIdx.x == 0) atomicExch(flag, 1);
+  return bad == 0;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// Inclusive scan of dt over `n` tokens by one warp (n a multiple of 32):
+// lane l sums tokens [l*n/32, (l+1)*n/32) in order, then the lane totals are
+// scanned. REV = true scans from the last token (suffix sums).
+template <bool REV>
+__device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t stride, int n, float* out) {
+  const int lane = threadIdx.x & 31, per = n / 32;
+  float loc[8];
+  float s = 0.f;
+  for (int q = 0; q < per; ++q) {
+    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
+    s = __fadd_rn(s, __bfloat162float(dt[pos * stride]));
+    loc[q] = s;
+  }
+  float inc = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float v = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc = __fadd_rn(inc, v);
+  }
+  float base = __shfl_up_sync(0xffffffffu, inc, 1);
+  if (lane == 0) base = 0.f;
+  for (int q = 0; q < per; ++q) {
+    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
+    out[pos] = __fadd_rn(base, loc[q]);
+  }
+  return __shfl_sync(0xffffffffu, inc, 31);  // total
+}
+
+
+__device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
+  return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~(uintptr_t)1023);
+}
+
+// Waits for every MMA batch still pending on the two buffer barriers.
+__device__ __forceinline__ bool drain(uint64_t* bar, bool (&pend)[2], uint32_t (&ph)[2], int* flag) {
+  bool ok = true;
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    if (pend[q]) {
+      ok = ok && cta_wait(&bar[q], ph[q], flag);
+      ph[q] ^= 1u;
+      pend[q] = false;
+    }
+  }
+  return ok;
+}
+
+// Shared memory of k_ssd_block_state (offsets from a 1024-aligned base).
+struct StateSmem {
+  static constexpr uint32_t kA = 0;        // [2 buffers][hi, lo][128 rows x 64 tokens] bf16, swizzled
+  static constexpr uint32_t kX = 65536;    // [Bs][64] bf16, MN-major swizzled
+  static constexpr uint32_t kB = 98304;    // [Bs][N] bf16, plain row-major
+  static __host__ __device__ uint32_t w(int N) { return kB + 256u * (uint32_t)N * 2u; }  // w[256], suf[256]
+  static __host__ __device__ uint32_t bytes(int N) { return w(N) + 2048u + 1024u; }
+};
+
+// One CTA per (batch row, block) and group of heads; thread n owns state row n.
+template <int N>
+__global__ void __launch_bounds__(128, 1) k_ssd_block_state(const SsdStateParams p) {
+  extern __shared__ unsigned char smraw[];
+  unsigned char* sm = align1024(smraw);
+  __shared__ uint64_t bar[2];
+  __shared__ uint32_t tslot;
+  const SsdGeo& g = p.g;
+  const int Bs = (int)g.Bs, H = g.H, t = threadIdx.x;
+  const int64_t bk = blockIdx.x, b = bk / g.nb;
+  const int k = (int)(bk % g.nb);
+  const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg);
+  unsigned char* sA = sm + StateSmem::kA;
+  unsigned char* sX = sm + StateSmem::kX;
+  const __nv_bfloat16* sB = reinterpret_cast<const __nv_bfloat16*>(sm + StateSmem::kB);
+  float* sw = reinterpret_cast<float*>(sm + StateSmem::w(N));
+  float* ssuf = sw + 256;
+  const int64_t tok0 = b * g.L + (int64_t)k * Bs;
+  {  // the block's B rows are contiguous in memory
+    const char* src = reinterpret_cast<const char*>(p.B + tok0 * N);
+    for (int c = t; c < Bs * N / 8; c += 128) cp_async16(sm + StateSmem::kB + c * 16, src + c * 16, 16);
+    cp_async_commit();
+  }
+  if (N < 128 && t >= N) {  // state rows beyond N stay zero in both buffers
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(sA + q * kTile16 + sw128(t, c)) = make_uint4(0, 0, 0, 0);
+  }
+  if (t == 0) {
+    umma::bar_init(&bar[0], 1);
+    umma::bar_init(&bar[1], 1);
+  }
+  if (t < 32) tmem_alloc(&tslot, 64);
+  umma::fence_before_sync();
+  __syncthreads();
+  umma::fence_after_sync();
+  const uint32_t tm = tslot;
+  bool pend[2] = {false, false};
+  uint32_t ph[2] = {0u, 0u};
+  int qg = 0;
+  bool alive = true;
+  for (int h = h0; h < h1 && alive; ++h) {
+    for (int c = t; c < Bs * 8; c += 128) {
+      const int s = c >> 3, ch = c & 7;
+      cp_async16(sX + sw128(s, ch), p.x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+    }
+    cp_async_commit();
+    if (t < 32) {
+      const __nv_bfloat16* dth = p.dt + tok0 * H + h;
+      const float tot = warp_scan_dt<true>(dth, H, Bs, ssuf);  // inclusive suffix sums
+      __syncwarp();
+      const float A2 = __fmul_rn(p.A[h], kLog2e);
+      for (int s = t; s < Bs; s += 32) {
+        const float after = s + 1 < Bs ? ssuf[s + 1] : 0.f;  // sum of dt over tokens after s
+        sw[s] = __fmul_rn(ex2(__fmul_rn(A2, after)), __bfloat162float(dth[(int64_t)s * H]));
+      }
+      if (t == 0) p.sumdt[bk * H + h] = tot;
+    }
+    cp_async_wait_all();
+    umma::fence_async_smem();
+    __syncthreads();
+    for (int q = 0; q < Bs / 64; ++q, ++qg) {
+      const int bb = qg & 1;
+      if (pend[bb]) {
+        if (!cta_wait(&bar[bb], ph[bb], p.flag)) {
+          alive = false;
+          break;
+        }
+        ph[bb] ^= 1u;
+        pend[bb] = false;
+      }
+      unsigned char* hi = sA + bb * 2 * kTile16;
+      unsigned char* lo = hi + kTile16;
+      if (t < N) {
+#pragma unroll 2
+        for (int c = 0; c < 8; ++c) {
+          uint32_t wh[4], wl[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int s0 = q * 64 + c * 8 + 2 * e;
+            const float v0 = __fmul_rn(sw[s0], __bfloat162float(sB[s0 * N + t]));
+            const float v1 = __fmul_rn(sw[s0 + 1], __bfloat162float(sB[(s0 + 1) * N + t]));
+            const __nv_bfloat162 hv = __floats2bfloat162_rn(v0, v1);
+            wh[e] = *reinterpret_cast<const uint32_t*>(&hv);
+            wl[e] = pack_bf16(__fsub_rn(v0, __low2float(hv)), __fsub_rn(v1, __high2float(hv)));
+          }
+          *reinterpret_cast<uint4*>(hi + sw128(t, c)) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+          *reinterpret_cast<uint4*>(lo + sw128(t, c)) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+        }
+      }
+      umma::fence_async_smem();
+      __syncthreads();
+      if (t == 0) {
+        umma::fence_after_sync();
+        const uint32_t ah = umma::smem_u32(hi), al = umma::smem_u32(lo);
+        const uint32_t xb = umma::smem_u32(sX) + (uint32_t)q * 64u * 128u;
+        constexpr uint32_t id = umma::idesc_bf16(128, 64, false, true);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t bd = umma::sdesc(xb + kk * 2048u, 1024, 1024);
+          umma::mma_bf16(tm, umma::sdesc(ah + kk * 32u, 16, 1024), bd, id, q > 0 || kk > 0);
+          umma::mma_bf16(tm, umma::sdesc(al + kk * 32u, 16, 1024), bd, id, true);
+        }
+        umma::mma_commit(&bar[bb]);
+      }
+      pend[bb] = true;
+    }
+    if (!alive || !drain(bar, pend, ph, p.flag)) {
+      alive = false;
+      break;
+    }
+    umma::fence_after_sync();
+    if (t < N) {  // whole warps: N is a multiple of 32
+      float v[32];
+      float* dst = p.T + ((bk * H + h) * kSsdP) * N + t;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        umma::tmem_ld32(tm + ((uint32_t)(t & ~31) << 16) + j * 32, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) dst[(int64_t)(j * 32 + i) * N] = v[i];
+      }
+    }
+    umma::fence_before_sync();
+    __syncthreads();
+    umma::fence_after_sync();
+  }
+  cp_async_wait_all();
+  umma::fence_before_sync();
+  __syncthreads();
+  if (t < 32) tmem_dealloc(tm, 64);
+}
+
+// One thread per (batch row, head, channel, state index), sequential in k.
+__global__ void __launch_bounds__(256) k_ssd_state_pass(const SsdPassParams p) {
+  const SsdGeo& g = p.g;
+  const int64_t per_b = (int64_t)g.H * kSsdP * g.N;
+  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (idx >= g.Bt * per_b) return;
+  const int64_t b = idx / per_b, r = idx - b * per_b;
+  const int h = (int)(r / ((int64_t)kSsdP * g.N));
+  const float A2 = __fmul_rn(p.A[h], kLog2e);
+  float S = p.init != nullptr ? p.init[idx] : 0.f;
+  const float* T = p.T + b * g.nb * per_b + r;
+  const float* sd = p.sumdt + b * g.nb * g.H + h;
+  for (int k = 0; k < g.nb; ++k) {
+    S = __fmaf_rn(ex2(__fmul_rn(A2, sd[(int64_t)k * g.H])), S, T[(int64_t)k * per_b]);
+    if (p.emit_all) p.states[(b * g.nb + k) * per_b + r] = S;
+  }
+  if (!p.emit_all) p.states[b * per_b + r] = S;
+  if (p.final_state != nullptr) p.final_state[b * per_b + r] = S;
+}
+
+// Shared memory of k_ssd_block_scan (offsets from a 1024-aligned base):
+//   Cf   the tile's C^f rows, K-major (N / 64 atom columns)
+//   M0   decay-weighted mixing tile, buffer 0 (128 x 128 bf16, K-major)
+//   M1   buffer 1; holds the tile's C^r rows until the Gram products are done
+//   R    the B tiles of the Gram products; afterwards the head's x tiles
+//        (MN-major, 16 KB each) followed by the seed's high and low parts
+//        (64 rows x N, K-major)
+//   cum  per token: A2 * cumulative dt and dt, for both directions
+struct ScanSmem {
+  uint32_t cf, m0, m1, r, x, seed, cum, total;
+  __host__ __device__ ScanSmem(int N, int m) {
+    const uint32_t tileC = 128u * (uint32_t)N * 2u;
+    const uint32_t tileM = 32768u;
+    cf = 0;
+    m0 = cf + tileC;
+    m1 = m0 + tileM;
+    const uint32_t m1sz = tileC > tileM ? tileC : tileM;
+    r = m1 + m1sz;
+    const uint32_t gram = (uint32_t)(m + 1) * tileC;
+    const uint32_t xs = (uint32_t)m * 16384u + 2u * 64u * (uint32_t)N * 2u;
+    x = r;
+    seed = r + (uint32_t)m * 16384u;
+    cum = r + (gram > xs ? gram : xs);
+    total = cum + 4u * 256u * 4u + 1024u;  // + alignment slack of the dynamic base
+  }
+};
+
+// Copies one 128-token tile of a [tokens][N] bf16 tensor into K-major
+// swizzled shared memory (N / 64 atom columns).
+template <int N>
+__device__ __forceinline__ void stage_rows(unsigned char* dst, const __nv_bfloat16* src) {
+  for (int c = threadIdx.x; c < 128 * N / 8; c += 128) {
+    const int r = c / (N / 8), ch = c % (N / 8);
+    cp_async16(dst + (ch >> 3) * kTile16 + sw128(r, ch & 7), src + (int64_t)r * N + ch * 8, 16);
+  }
+}
+
+// Gram product D[128 x 128] = A_rows . B_rows^T over K = N (both K-major).
+template <int N>
+__device__ __forceinline__ void mma_gram(uint32_t d, uint32_t a, uint32_t b) {
+  constexpr uint32_t id = umma::idesc_bf16(128, 128, false, false);
+#pragma unroll
+  for (int kk = 0; kk < N / 16; ++kk) {
+    const uint32_t off = (kk >> 2) * kTile16 + (kk & 3) * 32u;
+    umma::mma_bf16(d, umma::sdesc(a + off, 16, 1024), umma::sdesc(b + off, 16, 1024), id, kk > 0);
+  }
+}
+
+// One CTA per (batch row, block, 128-token tile i of the block) and group of
+// heads. Thread t owns token row t of the tile (TMEM lane t).
+// TMEM columns: Gram products at 128 q (forward products of s-tiles 0..i,
+// then, for noisy blocks, reverse products of s-tiles i..m-1), the output
+// accumulator at 384 and the seed term at 448.
+template <int N, bool NOISY>
+__global__ void __launch_bounds__(128, 1) k_ssd_block_scan(const SsdScanParams p) {
+  extern __shared__ unsigned char smraw[];
+  unsigned char* sm = align1024(smraw);
+  __shared__ uint64_t bar[3];
+  __shared__ uint32_t tslot;
+  const SsdGeo& g = p.g;
+  const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x;
+  const ScanSmem L(N, m);
+  const int64_t idx = blockIdx.x;
+  const int i = (int)(idx % m);
+  const int64_t bk = idx / m, b = bk / g.nb;
+  const int k = (int)(bk % g.nb);
+  const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg);
+  const int64_t tok0 = b * g.L + (int64_t)k * Bs;
+  const int tt = i * kSsdT + t;  // this thread's token inside the block
+  float* s_af = reinterpret_cast<float*>(sm + L.cum);  // A2_f * inclusive prefix sums of dt_f
+  float* s_wf = s_af + 256;                            // dt_f
+  float* s_ar = s_wf + 256;                            // A2_r * inclusive suffix sums of dt_r
+  float* s_wr = s_ar + 256;                            // dt_r
+  const int nf = i + 1, nr = NOISY ? m - i : 0;        // Gram products per direction
+  // --- Gram products C B^T of this tile against the block's s-tiles
+  stage_rows<N>(sm + L.cf, p.Cf + (tok0 + i * kSsdT) * N);
+  for (int j = 0; j < nf; ++j) stage_rows<N>(sm + L.r + j * 128u * N * 2u, p.Bf + (tok0 + j * kSsdT) * N);
+  if (NOISY) {
+    stage_rows<N>(sm + L.m1, p.Cr + (tok0 + i * kSsdT) * N);
+    for (int j = i; j < m; ++j)
+      stage_rows<N>(sm + L.r + (nf + j - i) * 128u * N * 2u, p.Br + (tok0 + j * kSsdT) * N);
+  }
+  cp_async_commit();
+  if (t == 0) {
+    umma::bar_init(&bar[0], 1);
+    umma::bar_init(&bar[1], 1);
+    umma::bar_init(&bar[2], 1);
+  }
+  if (t < 32) tmem_alloc(&tslot, 512);
+  cp_async_wait_all();
+  umma::fence_async_smem();
+  umma::fence_before_sync();
+  __syncthreads();
+  umma::fence_after_sync();
+  const uint32_t tm = tslot;
+  const uint32_t lane = tm + ((uint32_t)(t & ~31) << 16);
+  if (t == 0) {
+    const uint32_t base = umma::smem_u32(sm);
+    for (int q = 0; q < nf + nr; ++q)
+      mma_gram<N>(tm + 128u * q, base + (q < nf ? L.cf : L.m1), base + L.r + q * 128u * N * 2u);
+    umma::mma_commit(&bar[2]);
+  }
+  bool alive = cta_wait(&bar[2], 0, p.flag);
+  umma::fence_after_sync();
+  bool pend[2] = {false, false};
+  uint32_t ph[2] = {0u, 0u};
+  int gt = 0;  // M tiles issued so far (selects the buffer)
+  // this block's seed: slot k - 1 (or k) of p.seed; block 0 of a shifted
+  // layout starts from init_seed
+  const float* seed_src = nullptr;
+  if (p.seed_shift && k == 0) {
+    if (p.init_seed != nullptr) seed_src = p.init_seed + b * (int64_t)H * kSsdP * N;
+  } else if (p.seed != nullptr) {
+    seed_src = p.seed + b * p.seed_bstride + (int64_t)(p.seed_shift ? k - 1 : k) * H * kSsdP * N;
+  }
+  const bool has_seed = seed_src != nullptr;
+  const int ntile = NOISY ? m : i + 1;  // s-tiles whose x the head needs
+  for (int h = h0; h < h1 && alive; ++h) {
+    // --- the head's x tiles (MN-major) and its seed (bf16 high + low, K-major)
+    for (int c = t; c < ntile * kSsdT * 8; c += 128) {
+      const int s = c >> 3, ch = c & 7;  // token s of the block (tile s / 128)
+      cp_async16(sm + L.x + (s >> 7) * 16384u + sw128(s & 127, ch), p.x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+    }
+    cp_async_commit();
+    if (has_seed) {
+      const float* src = seed_src + (int64_t)h * kSsdP * N;
+      for (int c = t; c < kSsdP * N / 8; c += 128) {
+        const int pr = c / (N / 8), ch = c % (N / 8);
+        const float4 u0 = *reinterpret_cast<const float4*>(src + (int64_t)pr * N + ch * 8);
+        const float4 u1 = *reinterpret_cast<const float4*>(src + (int64_t)pr * N + ch * 8 + 4);
+        const float v[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+        uint32_t wh[4], wl[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+          wh[e] = *reinterpret_cast<const uint32_t*>(&hv);
+          wl[e] = pack_bf16(__fsub_rn(v[2 * e], __low2float(hv)), __fsub_rn(v[2 * e + 1], __high2float(hv)));
+        }
+        const uint32_t off = (ch >> 3) * 8192u + sw128(pr, ch & 7);
+        *reinterpret_cast<uint4*>(sm + L.seed + off) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+        *reinterpret_cast<uint4*>(sm + L.seed + 128u * N + off) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+      }
+    }
+    // --- decay exponents of the head: A2 * cumulative dt (fp32, fixed order)
+    if (t < 32) {
+      const __nv_bfloat16* d = p.dtf + tok0 * H + h;
+      warp_scan_dt<false>(d, H, Bs, s_af);
+      __syncwarp();
+      const float A2 = __fmul_rn(p.Af[h], kLog2e);
+      for (int s = t; s < Bs; s += 32) {
+        s_af[s] = __fmul_rn(A2, s_af[s]);
+        s_wf[s] = __bfloat162float(d[(int64_t)s * H]);
+      }
+    } else if (NOISY && t < 64) {
+      const __nv_bfloat16* d = p.dtr + tok0 * H + h;
+      warp_scan_dt<true>(d, H, Bs, s_ar);
+      __syncwarp();
+      const float A2 = __fmul_rn(p.Ar[h], kLog2e);
+      for (int s = t - 32; s < Bs; s += 32) {
+        s_ar[s] = __fmul_rn(A2, s_ar[s]);
+        s_wr[s] = __bfloat162float(d[(int64_t)s * H]);
+      }
+    }
+    cp_async_wait_all();
+    umma::fence_async_smem();
+    __syncthreads();
+    if (t == 0 && has_seed) {  // seed term C^f . seed^T into columns 448..511
+      umma::fence_after_sync();
+      const uint32_t base = umma::smem_u32(sm);
+      constexpr uint32_t id = umma::idesc_bf16(128, 64, false, false);
+#pragma unroll
+      for (int kk = 0; kk < N / 16; ++kk) {
+        const uint32_t offc = (kk >> 2) * kTile16 + (kk & 3) * 32u;
+        const uint32_t offs = (kk >> 2) * 8192u + (kk & 3) * 32u;
+        const uint64_t a = umma::sdesc(base + L.cf + offc, 16, 1024);
+        umma::mma_bf16(tm + 448, a, umma::sdesc(base + L.seed + offs, 16, 1024), id, kk > 0);
+        umma::mma_bf16(tm + 448, a, umma::sdesc(base + L.seed + 128u * N + offs, 16, 1024), id, true);
+      }
+    }
+    // --- decay-weighted mixing tiles, one per s-tile, each multiplied with x
+    const float af_t = s_af[tt];
+    const float ar_t = NOISY ? s_ar[tt] : 0.f;
+    for (int j = 0; j < ntile; ++j, ++gt) {
+      const int bb = gt & 1;
+      if (pend[bb]) {
+        if (!cta_wait(&bar[bb], ph[bb], p.flag)) {
+          alive = false;
+          break;
+        }
+        ph[bb] ^= 1u;
+        pend[bb] = false;
+      }
+      unsigned char* mt = sm + (bb ? L.m1 : L.m0);
+      const bool use_f = j <= i, use_r = NOISY && j >= i;  // uniform over the CTA
+      const uint32_t colf = 128u * j, colr = 128u * (nf + j - i);
+#pragma unroll 1
+      for (int c32 = 0; c32 < 4; ++c32) {
+        float gf[32], gr[32], v[32];
+        if (use_f) umma::tmem_ld32(lane + colf + 32u * c32, gf);
+        if (use_r) umma::tmem_ld32(lane + colr + 32u * c32, gr);
+#pragma unroll
+        for (int q = 0; q < 32; ++q) {
+          const int ss = j * kSsdT + c32 * 32 + q;
+          float val = 0.f;
+          if (use_f) {
+            const float e = __fmul_rn(ex2(__fsub_rn(af_t, s_af[ss])), s_wf[ss]);
+            val = ss <= tt ? __fmul_rn(gf[q], e) : 0.f;
+          }
+          if (use_r) {
+            const float e = __fmul_rn(ex2(__fsub_rn(ar_t, s_ar[ss])), s_wr[ss]);
+            val = __fadd_rn(val, ss >= tt ? __fmul_rn(gr[q], e) : 0.f);
+          }
+          v[q] = val;
+        }
+#pragma unroll
+        for (int ch = 0; ch < 4; ++ch) {
+          const int col = c32 * 32 + ch * 8;  // s inside the tile
+          *reinterpret_cast<uint4*>(mt + (col >> 6) * kTile16 + sw128(t, (col & 63) >> 3)) =
+              make_uint4(pack_bf16(v[ch * 8], v[ch * 8 + 1]), pack_bf16(v[ch * 8 + 2], v[ch * 8 + 3]),
+                         pack_bf16(v[ch * 8 + 4], v[ch * 8 + 5]), pack_bf16(v[ch * 8 + 6], v[ch * 8 + 7]));
+        }
+      }
+      umma::fence_async_smem();
+      umma::fence_before_sync();
+      __syncthreads();
+      if (t == 0) {
+        umma::fence_after_sync();
+        const uint32_t ma = umma::smem_u32(mt), xb = umma::smem_u32(sm + L.x) + (uint32_t)j * 16384u;
+        constexpr uint32_t id = umma::idesc_bf16(128, 64, false, true);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          umma::mma_bf16(tm + 384, umma::sdesc(ma + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
+                         umma::sdesc(xb + kk * 2048u, 1024, 1024), id, j > 0 || kk > 0);
+        umma::mma_commit(&bar[bb]);
+      }
+      pend[bb] = true;
+    }
+    if (!alive || !drain(bar, pend, ph, p.flag)) {
+      alive = false;
+      break;
+    }
+    umma::fence_after_sync();
+    // --- epilogue: y = mixing term + decayed seed term + D x, bf16 out
+    {
+      float ya[64], yo[64];
+      umma::tmem_ld32(lane + 384, *reinterpret_cast<float(*)[32]>(&ya[0]));
+      umma::tmem_ld32(lane + 416, *reinterpret_cast<float(*)[32]>(&ya[32]));
+      if (has_seed) {
+        umma::tmem_ld32(lane + 448, *reinterpret_cast<float(*)[32]>(&yo[0]));
+        umma::tmem_ld32(lane + 480, *reinterpret_cast<float(*)[32]>(&yo[32]));
+      }
+      const float dec = has_seed ? ex2(af_t) : 0.f;
+      const float Dd = NOISY ? __fadd_rn(p.Df[h], p.Dr[h]) : p.Df[h];
+      const unsigned char* xr = sm + L.x + (uint32_t)i * 16384u;
+      __nv_bfloat16* dst = p.y + ((tok0 + tt) * H + h) * kSsdP;
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {
+        const uint4 xv = *reinterpret_cast<const uint4*>(xr + sw128(t, ch));
+        const __nv_bfloat16* xe = reinterpret_cast<const __nv_bfloat16*>(&xv);
+        float o[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const int q = ch * 8 + e;
+          float acc = ya[q];
+          if (has_seed) acc = __fmaf_rn(dec, yo[q], acc);
+          o[e] = __fmaf_rn(Dd, __bfloat162float(xe[e]), acc);
+        }
+        *reinterpret_cast<uint4*>(dst + ch * 8) =
+            make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]), pack_bf16(o[6], o[7]));
+      }
+    }
+    umma::fence_before_sync();
+    __syncthreads();
+    umma::fence_after_sync();
+  }
+  cp_async_wait_all();
+  umma::fence_before_sync();
+  __syncthreads();
+  if (t < 32) tmem_dealloc(tm, 512);
+}
+
+}  // namespace
+
+int* ssd_wait_flag_ptr() {
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_ssd_wait_flag) != cudaSuccess) return nullptr;
+  return static_cast<int*>(p);
+}
+
+namespace {
+
+template <typename K>
+cudaError_t set_smem(K kernel, uint32_t bytes) {
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+}
+
+}  // namespace
+
+cudaError_t launch_ssd_block_state(const SsdStateParams& p, cudaStream_t s) {
+  const int64_t rows = p.g.Bt * p.g.nb;
+  if (rows == 0 || p.g.H == 0) return cudaSuccess;
+  const dim3 grid((unsigned)rows, (unsigned)((p.g.H + p.hg - 1) / p.hg));
+  const uint32_t bytes = StateSmem::bytes(p.g.N);
+  cudaError_t e;
+  if (p.g.N == 64) {
+    if ((e = set_smem(k_ssd_block_state<64>, bytes)) != cudaSuccess) return e;
+    k_ssd_block_state<64><<<grid, 128, bytes, s>>>(p);
+  } else {
+    if ((e = set_smem(k_ssd_block_state<128>, bytes)) != cudaSuccess) return e;
+    k_ssd_block_state<128><<<grid, 128, bytes, s>>>(p);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ssd_state_pass(const SsdPassParams& p, cudaStream_t s) {
+  const int64_t n = p.g.Bt * p.g.H * kSsdP * p.g.N;
+  if (n == 0) return cudaSuccess;
+  k_ssd_state_pass<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <int N, bool NOISY>
+cudaError_t scan_t(const SsdScanParams& p, cudaStream_t s) {
+  const int64_t tiles = p.g.Bt * p.g.nb * p.g.m;
+  if (tiles == 0 || p.g.H == 0) return cudaSuccess;
+  const ScanSmem L(N, p.g.m);
+  cudaError_t e = set_smem(k_ssd_block_scan<N, NOISY>, L.total);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((unsigned)tiles, (unsigned)((p.g.H + p.hg - 1) / p.hg));
+  k_ssd_block_scan<N, NOISY><<<grid, 128, L.total, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ssd_block_scan(bool noisy, const SsdScanParams& p, cudaStream_t s) {
+  if (p.g.N == 64) return noisy ? scan_t<64, true>(p, s) : scan_t<64, false>(p, s);
+  return noisy ? scan_t<128, true>(p, s) : scan_t<128, false>(p, s);
+}
+
+}  // namespace bds

@@ -1,0 +1,288 @@
+// ssd_api.cu -- the C ABI of the SSD-form scan (include/bdscan_ssd.h):
+// argument validation, workspace layout and the launch sequence.
+#include <cstdio>
+
+#include "bdscan_ssd.h"
+#include "params.h"
+#include "ssd.cuh"
+
+namespace {
+
+int failf(int code, const char* fmt, const char* fn, const char* what = "") {
+  char msg[384];
+  snprintf(msg, sizeof(msg), fmt, fn, what);
+  return bds::api_fail(code, msg);
+}
+
+int cuda_fail(cudaError_t e, const char* fn) {
+  char msg[384];
+  snprintf(msg, sizeof(msg), "%s: %s", fn, cudaGetErrorString(e));
+  return bds::api_fail(BDSCAN_ERR_CUDA, msg);
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+#define SSD_REQ(ptr, fn, name)                                                              \
+  do {                                                                                      \
+    if ((ptr) == nullptr) return failf(BDSCAN_ERR_ARG, "%s: %s is NULL", fn, name);         \
+    if (!aligned16(ptr)) return failf(BDSCAN_ERR_ARG, "%s: %s is not 16-byte aligned", fn, name); \
+  } while (0)
+#define SSD_OPT(ptr, fn, name)                                                              \
+  do {                                                                                      \
+    if ((ptr) != nullptr && !aligned16(ptr))                                                \
+      return failf(BDSCAN_ERR_ARG, "%s: %s is not 16-byte aligned", fn, name);              \
+  } while (0)
+
+// Validates the dimensions and fills the geometry.
+int check(const bdscan_ssd_dims* d, bds::SsdGeo* g, const char* fn) {
+  bds::api_begin();
+  if (d == nullptr) return failf(BDSCAN_ERR_ARG, "%s: dims is NULL", fn);
+  if (d->batch < 0 || d->len < 0 || d->heads < 0) return failf(BDSCAN_ERR_ARG, "%s: negative batch, len or heads", fn);
+  if (d->block <= 0) return failf(BDSCAN_ERR_ARG, "%s: block must be positive", fn);
+  if (d->len % d->block != 0) return failf(BDSCAN_ERR_ARG, "%s: len is not a multiple of block", fn);
+  if (d->dtype != BDSCAN_BF16) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: dtype must be bf16", fn);
+  if (d->head_dim != 64) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: head_dim must be 64", fn);
+  if (d->d_state != 64 && d->d_state != 128) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: d_state must be 64 or 128", fn);
+  if (d->block != 128 && d->block != 256) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: block must be 128 or 256", fn);
+  if (d->heads > 65535 * 8) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: too many heads", fn);
+  const int64_t nb = d->len / d->block;
+  if (d->batch * nb * (d->block / 128) > 0x7fffffffLL) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: too many blocks", fn);
+  g->Bt = d->batch;
+  g->L = d->len;
+  g->Bs = d->block;
+  g->H = (int)d->heads;
+  g->N = (int)d->d_state;
+  g->nb = (int)nb;
+  g->m = (int)(d->block / 128);
+  return BDSCAN_OK;
+}
+
+// Heads per CTA: groups of at most 8 heads, as even as possible. The Gram
+// products of a tile are computed once per CTA and shared by its heads.
+int heads_per_cta(int H) {
+  if (H <= 0) return 1;
+  const int groups = (H + 7) / 8;
+  return (H + groups - 1) / groups;
+}
+
+size_t sumdt_bytes(const bds::SsdGeo& g) { return al256((size_t)g.Bt * g.nb * g.H * 4); }
+size_t states_bytes(const bds::SsdGeo& g) { return al256((size_t)g.Bt * g.nb * g.H * 64 * g.N * 4); }
+
+int check_clean(const bdscan_clean* c, const char* fn) {
+  if (c == nullptr) return failf(BDSCAN_ERR_ARG, "%s: clean is NULL", fn);
+  SSD_REQ(c->x, fn, "clean.x");
+  SSD_REQ(c->dt, fn, "clean.dt");
+  SSD_REQ(c->B, fn, "clean.B");
+  SSD_REQ(c->C, fn, "clean.C");
+  return BDSCAN_OK;
+}
+
+int check_noisy(const bdscan_noisy* n, const bdscan_params* pr, const char* fn) {
+  if (n == nullptr) return failf(BDSCAN_ERR_ARG, "%s: noisy is NULL", fn);
+  if (pr == nullptr) return failf(BDSCAN_ERR_ARG, "%s: params is NULL", fn);
+  SSD_REQ(n->x, fn, "noisy.x");
+  SSD_REQ(n->dt_f, fn, "noisy.dt_f");
+  SSD_REQ(n->B_f, fn, "noisy.B_f");
+  SSD_REQ(n->C_f, fn, "noisy.C_f");
+  SSD_REQ(n->dt_r, fn, "noisy.dt_r");
+  SSD_REQ(n->B_r, fn, "noisy.B_r");
+  SSD_REQ(n->C_r, fn, "noisy.C_r");
+  SSD_REQ(pr->A_f, fn, "params.A_f");
+  SSD_REQ(pr->D_f, fn, "params.D_f");
+  SSD_REQ(pr->A_r, fn, "params.A_r");
+  SSD_REQ(pr->D_r, fn, "params.D_r");
+  return BDSCAN_OK;
+}
+
+using bf = __nv_bfloat16;
+
+}  // namespace
+
+namespace {
+
+bds::SsdScanParams clean_scan(const bds::SsdGeo& g, const bdscan_clean* c, const float* A_f, const float* D_f,
+                              const float* seeds, const float* init, void* y, int* flag) {
+  bds::SsdScanParams p{};
+  p.g = g;
+  p.x = (const bf*)c->x;
+  p.dtf = (const bf*)c->dt;
+  p.Bf = (const bf*)c->B;
+  p.Cf = (const bf*)c->C;
+  p.Af = A_f;
+  p.Df = D_f;
+  p.seed = seeds;
+  p.seed_bstride = (int64_t)g.nb * g.H * 64 * g.N;
+  p.seed_shift = 1;
+  p.init_seed = init;
+  p.y = (bf*)y;
+  p.hg = heads_per_cta(g.H);
+  p.flag = flag;
+  return p;
+}
+
+bds::SsdScanParams noisy_scan(const bds::SsdGeo& g, const bdscan_noisy* n, const bdscan_params* pr, void* y,
+                              int* flag) {
+  bds::SsdScanParams p{};
+  p.g = g;
+  p.x = (const bf*)n->x;
+  p.dtf = (const bf*)n->dt_f;
+  p.Bf = (const bf*)n->B_f;
+  p.Cf = (const bf*)n->C_f;
+  p.dtr = (const bf*)n->dt_r;
+  p.Br = (const bf*)n->B_r;
+  p.Cr = (const bf*)n->C_r;
+  p.Af = pr->A_f;
+  p.Df = pr->D_f;
+  p.Ar = pr->A_r;
+  p.Dr = pr->D_r;
+  p.y = (bf*)y;
+  p.hg = heads_per_cta(g.H);
+  p.flag = flag;
+  return p;
+}
+
+// Block-local states into T, then the exact states (in place when T is the
+// emitted states array).
+cudaError_t build_states(const bds::SsdGeo& g, const bdscan_clean* c, const float* A_f, const float* init,
+                         float* T, float* sumdt, float* final_state, int* flag, cudaStream_t s) {
+  bds::SsdStateParams sp{};
+  sp.g = g;
+  sp.x = (const bf*)c->x;
+  sp.dt = (const bf*)c->dt;
+  sp.B = (const bf*)c->B;
+  sp.A = A_f;
+  sp.T = T;
+  sp.sumdt = sumdt;
+  sp.hg = heads_per_cta(g.H);
+  sp.flag = flag;
+  cudaError_t e = bds::api_launched(bds::launch_ssd_block_state(sp, s), s);
+  if (e != cudaSuccess) return e;
+  bds::SsdPassParams pp{};
+  pp.g = g;
+  pp.T = T;
+  pp.sumdt = sumdt;
+  pp.A = A_f;
+  pp.init = init;
+  pp.states = T;
+  pp.emit_all = 1;
+  pp.final_state = final_state;
+  return bds::api_launched(bds::launch_ssd_state_pass(pp, s), s);
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t bdscan_ssd_forward_workspace_size(const bdscan_ssd_dims* dims) {
+  bds::SsdGeo g;
+  if (check(dims, &g, "bdscan_ssd_forward_workspace_size") != BDSCAN_OK) return 0;
+  return sumdt_bytes(g);
+}
+
+int bdscan_ssd_forward(const bdscan_ssd_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
+                       const bdscan_params* params, void* y_c, void* y_n, float* states, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_ssd_forward";
+  bds::SsdGeo g;
+  int rc = check(dims, &g, fn);
+  if (rc) return rc;
+  if (g.Bt == 0 || g.nb == 0 || g.H == 0) return bds::api_ok();
+  if ((rc = check_clean(clean, fn)) || (rc = check_noisy(noisy, params, fn))) return rc;
+  SSD_REQ(y_c, fn, "y_c");
+  SSD_REQ(y_n, fn, "y_n");
+  SSD_REQ(states, fn, "states");
+  SSD_REQ(workspace, fn, "workspace");
+  if (workspace_bytes < sumdt_bytes(g)) return failf(BDSCAN_ERR_ARG, "%s: workspace too small%s", fn);
+  int* flag = bds::ssd_wait_flag_ptr();
+  if (flag == nullptr) return cuda_fail(cudaGetLastError(), fn);
+  cudaStream_t s = (cudaStream_t)stream;
+  float* sumdt = (float*)workspace;
+  cudaError_t e = build_states(g, clean, params->A_f, nullptr, states, sumdt, nullptr, flag, s);
+  if (e == cudaSuccess) {
+    const bds::SsdScanParams cp = clean_scan(g, clean, params->A_f, params->D_f, states, nullptr, y_c, flag);
+    e = bds::api_launched(bds::launch_ssd_block_scan(false, cp, s), s);
+  }
+  if (e == cudaSuccess) {
+    bds::SsdScanParams np = noisy_scan(g, noisy, params, y_n, flag);
+    np.seed = states;
+    np.seed_bstride = (int64_t)g.nb * g.H * 64 * g.N;
+    np.seed_shift = 1;
+    e = bds::api_launched(bds::launch_ssd_block_scan(true, np, s), s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return bds::api_ok();
+}
+
+size_t bdscan_ssd_boundary_states_workspace_size(const bdscan_ssd_dims* dims, int emit_all) {
+  bds::SsdGeo g;
+  if (check(dims, &g, "bdscan_ssd_boundary_states_workspace_size") != BDSCAN_OK) return 0;
+  return sumdt_bytes(g) + (emit_all ? 0 : states_bytes(g));
+}
+
+int bdscan_ssd_boundary_states(const bdscan_ssd_dims* dims, const bdscan_clean* clean, const float* A_f,
+                               const float* D_f, const float* init_state, void* y_c, float* states,
+                               int emit_all, void* workspace, size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_ssd_boundary_states";
+  bds::SsdGeo g;
+  int rc = check(dims, &g, fn);
+  if (rc) return rc;
+  if (g.Bt == 0 || g.nb == 0 || g.H == 0) return bds::api_ok();
+  if ((rc = check_clean(clean, fn))) return rc;
+  SSD_REQ(A_f, fn, "A_f");
+  SSD_REQ(states, fn, "states");
+  SSD_REQ(workspace, fn, "workspace");
+  SSD_OPT(init_state, fn, "init_state");
+  SSD_OPT(y_c, fn, "y_c");
+  if (y_c != nullptr) SSD_REQ(D_f, fn, "D_f");
+  if (workspace_bytes < sumdt_bytes(g) + (emit_all ? 0 : states_bytes(g)))
+    return failf(BDSCAN_ERR_ARG, "%s: workspace too small%s", fn);
+  int* flag = bds::ssd_wait_flag_ptr();
+  if (flag == nullptr) return cuda_fail(cudaGetLastError(), fn);
+  cudaStream_t s = (cudaStream_t)stream;
+  float* sumdt = (float*)workspace;
+  // every block-end state goes to `states` (emit_all) or to the workspace,
+  // with the final one copied out
+  float* all = emit_all ? states : (float*)((char*)workspace + sumdt_bytes(g));
+  cudaError_t e = build_states(g, clean, A_f, init_state, all, sumdt, emit_all ? nullptr : states, flag, s);
+  if (e == cudaSuccess && y_c != nullptr) {
+    const bds::SsdScanParams cp = clean_scan(g, clean, A_f, D_f, all, init_state, y_c, flag);
+    e = bds::api_launched(bds::launch_ssd_block_scan(false, cp, s), s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return bds::api_ok();
+}
+
+int bdscan_ssd_active_block(const bdscan_ssd_dims* dims, const float* seed, const bdscan_noisy* noisy,
+                            const bdscan_params* params, void* y_n, void* stream) {
+  const char* fn = "bdscan_ssd_active_block";
+  bds::SsdGeo g;
+  int rc = check(dims, &g, fn);
+  if (rc) return rc;
+  if (dims->len != dims->block) return failf(BDSCAN_ERR_ARG, "%s: len must equal block%s", fn);
+  if (g.Bt == 0 || g.H == 0) return bds::api_ok();
+  if ((rc = check_noisy(noisy, params, fn))) return rc;
+  SSD_OPT(seed, fn, "seed");
+  SSD_REQ(y_n, fn, "y_n");
+  int* flag = bds::ssd_wait_flag_ptr();
+  if (flag == nullptr) return cuda_fail(cudaGetLastError(), fn);
+  cudaStream_t s = (cudaStream_t)stream;
+  bds::SsdScanParams np = noisy_scan(g, noisy, params, y_n, flag);
+  np.seed = seed;
+  np.seed_bstride = (int64_t)g.H * 64 * g.N;
+  np.seed_shift = 0;
+  const cudaError_t e = bds::api_launched(bds::launch_ssd_block_scan(true, np, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return bds::api_ok();
+}
+
+int bdscan_ssd_wait_flag(int reset) {
+  int* flag = bds::ssd_wait_flag_ptr();
+  if (flag == nullptr) return -1;
+  int v = 0;
+  if (cudaMemcpy(&v, flag, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+  if (reset && cudaMemset(flag, 0, sizeof(int)) != cudaSuccess) return -1;
+  return v;
+}
+
+}  // extern "C"

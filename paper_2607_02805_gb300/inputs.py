@@ -143,3 +143,28 @@ class Workload:
         if self.dtype == "bf16" and name not in PARAMS and name not in ("dstates", "init_state"):
             a = bf16_bits_to_f32(f32_to_bf16_bits(a)).reshape(a.shape)
         self.t32[name] = np.ascontiguousarray(a)
+
+
+class SsdWorkload(Workload):
+    """A seeded problem instance of the SSD (Mamba-2) form: x [Bt, L, H, 64],
+    dt [Bt, L, H], B, C [Bt, L, N], A and D per head [H]; init_state and seeds
+    [Bt, H, 64, N]. Same draws as the diagonal layer (same stream ids and value
+    recipe), with these shapes; the forward-side tensors only."""
+
+    def __init__(self, batch, length, block, heads, d_state, seed=0, with_init=False, head_dim=64, part=0):
+        self.batch, self.len, self.block = int(batch), int(length), int(block)
+        self.heads, self.head_dim, self.d_state = int(heads), int(head_dim), int(d_state)
+        self.d_inner, self.dtype, self.seed = self.heads * self.head_dim, "bf16", int(seed)
+        Bt, L, H, P, N = self.batch, self.len, self.heads, self.head_dim, self.d_state
+        shapes = {"x_c": (Bt, L, H, P), "dt_c": (Bt, L, H), "B_c": (Bt, L, N), "C_c": (Bt, L, N),
+                  "x_n": (Bt, L, H, P), "dt_f": (Bt, L, H), "B_f": (Bt, L, N), "C_f": (Bt, L, N),
+                  "dt_r": (Bt, L, H), "B_r": (Bt, L, N), "C_r": (Bt, L, N),
+                  "A_f": (H,), "A_r": (H,), "D_f": (H,), "D_r": (H,)}
+        if with_init:
+            shapes["init_state"] = (Bt, H, P, N)
+        self.t32 = {}
+        for k, shp in shapes.items():
+            a = draw(k, shp, self.seed, 0 if k in PARAMS else part)
+            if k not in PARAMS and k != "init_state":
+                a = bf16_bits_to_f32(f32_to_bf16_bits(a)).reshape(shp)
+            self.t32[k] = a

@@ -8,13 +8,16 @@ import pytest
 
 from paper_2607_02805_gb300 import binding
 
-HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "bdscan.h")
+INCLUDE = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+HEADERS = [os.path.join(INCLUDE, h) for h in ("bdscan.h", "bdscan_ssd.h")]
 
 
 def header_functions():
-    text = open(HEADER).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(bdscan_\w+)\s*\(", text)))
+    names = set()
+    for h in HEADERS:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names.update(re.findall(r"\b(bdscan_\w+)\s*\(", text))
+    return sorted(names)
 
 
 def test_library_exports_every_declared_function():
@@ -161,3 +164,53 @@ def test_fails_loudly_without_a_gpu():
     rc = _fwd(d)
     assert rc == binding.BDSCAN_ERR_CUDA
     assert "bdscan_forward" in binding.bdscan_last_error()
+
+
+def _ssd_dims(**kw):
+    base = dict(batch=2, length=512, block=256, heads=4, d_state=128)
+    base.update(kw)
+    return binding.make_ssd_dims(base["batch"], base["length"], base["block"], base["heads"], base["d_state"],
+                                 base.get("head_dim", 64))
+
+
+def test_ssd_workspace_sizes():
+    al = lambda x: (x + 255) // 256 * 256
+    d = _ssd_dims(batch=8, length=8192, block=256, heads=26, d_state=128)
+    nb = 8192 // 256
+    assert binding.bdscan_ssd_forward_workspace_size(d) == al(8 * nb * 26 * 4)
+    assert binding.bdscan_ssd_boundary_states_workspace_size(d, 1) == al(8 * nb * 26 * 4)
+    assert binding.bdscan_ssd_boundary_states_workspace_size(d, 0) == al(8 * nb * 26 * 4) + al(8 * nb * 26 * 64 * 128 * 4)
+
+
+@pytest.mark.parametrize("kw,code,msg", [
+    (dict(length=500), binding.BDSCAN_ERR_ARG, "not a multiple of block"),
+    (dict(block=64, length=512), binding.BDSCAN_ERR_UNSUPPORTED, "128 or 256"),
+    (dict(head_dim=32), binding.BDSCAN_ERR_UNSUPPORTED, "head_dim"),
+    (dict(d_state=16), binding.BDSCAN_ERR_UNSUPPORTED, "d_state"),
+    (dict(batch=-1), binding.BDSCAN_ERR_ARG, "negative"),
+])
+def test_ssd_rejects_bad_dims(kw, code, msg):
+    c, n, p = _structs()
+    rc = binding.bdscan_ssd_forward(_ssd_dims(**kw), c, n, p, FAKE, FAKE, FAKE, FAKE, 1 << 40, None)
+    assert rc == code and msg in binding.bdscan_last_error()
+    assert binding.bdscan_ssd_forward_workspace_size(_ssd_dims(**kw)) == 0
+
+
+def test_ssd_rejects_bad_pointers():
+    d = _ssd_dims()
+    c, n, p = _structs()
+    n.B_r = None
+    rc = binding.bdscan_ssd_forward(d, c, n, p, FAKE, FAKE, FAKE, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "noisy.B_r is NULL" in binding.bdscan_last_error()
+    c, n, p = _structs()
+    rc = binding.bdscan_ssd_forward(d, c, n, p, FAKE, FAKE, FAKE + 8, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "states is not 16-byte aligned" in binding.bdscan_last_error()
+    rc = binding.bdscan_ssd_forward(d, c, n, p, FAKE, FAKE, FAKE, FAKE, 16, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "workspace too small" in binding.bdscan_last_error()
+    rc = binding.bdscan_ssd_boundary_states(d, c, FAKE, FAKE, FAKE + 4, None, FAKE, 1, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "init_state" in binding.bdscan_last_error()
+    rc = binding.bdscan_ssd_active_block(d, FAKE, n, p, FAKE, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "must equal block" in binding.bdscan_last_error()
+    # an empty batch needs no pointers
+    c0, n0, p0 = _structs(None)
+    assert binding.bdscan_ssd_forward(_ssd_dims(batch=0), c0, n0, p0, None, None, None, None, 0, None) == 0
