@@ -442,6 +442,118 @@ def run_sweep(args):
         torch.cuda.empty_cache()
 
 
+SSD_KERNELS = ("ssd_block_state", "ssd_state_pass", "ssd_scan_clean", "ssd_scan_noisy")
+
+
+def ssd_costs(Bt, L, Bs, H, N, hg):
+    """Algorithmic HBM bytes and tensor-core flops of each SSD forward kernel.
+    Bytes: every tensor a kernel must touch, once (x, dt, B, C of its streams,
+    the states it writes or reads as seeds, its outputs). Flops: the MMAs the
+    kernels issue, counting the high and low bf16 parts of split operands."""
+    P, nb, m = 64, L // Bs, Bs // 128
+    tok = Bt * L
+    x, dt, bc = tok * H * P * 2, tok * H * 2, tok * N * 2
+    st = Bt * nb * H * P * N * 4
+    sd = Bt * nb * H * 4
+    groups = -(-H // hg)
+    b = {"ssd_block_state": x + dt + bc + st + sd,
+         "ssd_state_pass": 2 * st + sd,
+         "ssd_scan_clean": x + dt + 2 * bc + st + x,
+         "ssd_scan_noisy": x + 2 * dt + 4 * bc + st + x}
+    tiles = Bt * nb * m
+    gram_c = sum(i + 1 for i in range(m))       # Gram products per block, clean
+    gram_n = m * (m + 1)                        # forward + reverse per block
+    mix_c = gram_c                              # mixing tiles per head and block
+    mix_n = m * m
+    f = {"ssd_block_state": Bt * nb * H * 2 * (2.0 * 128 * P * Bs),
+         "ssd_state_pass": 0.0,
+         "ssd_scan_clean": Bt * nb * (groups * gram_c * 2.0 * 128 * 128 * N + H * (mix_c * 2.0 * 128 * 128 * P)
+                                      + H * m * 2 * 2.0 * 128 * P * N),
+         "ssd_scan_noisy": Bt * nb * (groups * gram_n * 2.0 * 128 * 128 * N + H * (mix_n * 2.0 * 128 * 128 * P)
+                                      + H * m * 2 * 2.0 * 128 * P * N)}
+    del tiles
+    return b, f
+
+
+def run_ssd(args):
+    """Forward of the SSD (Mamba-2) form at the paper's two model sizes, one
+    line each: clean scan with every block-end state, noisy blocks (seeded
+    forward + block-local reverse), through bdscan_ssd_forward."""
+    import torch
+    from paper_2607_02805_gb300 import binding
+    from paper_2607_02805_gb300.inputs import SsdWorkload
+    from paper_2607_02805_gb300.layer import to_device
+    peaks, peak_kind = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    tc_peak = float(peaks.get("bf16_tflops", 1900.0))
+    for name, (Bt, L, Bs, H, N) in (("350M-class Mamba-2 layer: 26 heads of 64, state 128", (8, 8192, 256, 26, 128)),
+                                   ("87M-class Mamba-2 layer: 14 heads of 64, state 64", (8, 8192, 256, 14, 64))):
+        if args.batch:
+            Bt = args.batch
+        wl = SsdWorkload(Bt, L, Bs, H, N, seed=0)
+        t = {k: to_device(wl.dev_bits(k), binding.BDSCAN_F32 if k in ("A_f", "A_r", "D_f", "D_r")
+                          else binding.BDSCAN_BF16, "cuda") for k in wl.t32}
+        d = binding.make_ssd_dims(Bt, L, Bs, H, N)
+        y_c = torch.empty((Bt, L, H, 64), dtype=torch.bfloat16, device="cuda")
+        y_n = torch.empty_like(y_c)
+        st = torch.empty((Bt, L // Bs, H, 64, N), dtype=torch.float32, device="cuda")
+        ws = torch.empty(binding.bdscan_ssd_forward_workspace_size(d), dtype=torch.uint8, device="cuda")
+        stream = torch.cuda.current_stream()
+        for _ in range(max(3, args.warmup)):
+            binding.ssd_forward(d, t, y_c, y_n, st, ws)
+        nk = len(SSD_KERNELS)
+        steps = max(1, args.steps)
+        ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        ev_k = [[torch.cuda.Event(enable_timing=True) for _ in range(nk)] for _ in range(steps)]
+        for evs in ev_k:
+            for e in evs:
+                e.record(stream)
+        torch.cuda.synchronize()
+        arr = [(ctypes.c_void_p * nk)(*[e.cuda_event for e in evs]) for evs in ev_k]
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(steps):
+            ev_s[i].record(stream)
+            binding.bdscan_profile_events(arr[i], nk)
+            binding.ssd_forward(d, t, y_c, y_n, st, ws)
+            binding.bdscan_profile_events(None, 0)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        flag = binding.bdscan_ssd_wait_flag(1)
+        ms = e0.elapsed_time(e1) / steps
+        per = {k: [] for k in SSD_KERNELS}
+        for i in range(steps):
+            prev = ev_s[i]
+            for j, k in enumerate(SSD_KERNELS):
+                per[k].append(prev.elapsed_time(ev_k[i][j]))
+                prev = ev_k[i][j]
+        hg = -(-H // -(-H // 8))
+        bts, fls = ssd_costs(Bt, L, Bs, H, N, hg)
+        kern = []
+        for k in SSD_KERNELS:
+            us = 1e3 * statistics.mean(per[k])
+            kern.append({"name": k, "avg_us": round(us, 2), "alg_bytes": bts[k],
+                         "alg_gbs": round(bts[k] / (us * 1e-6) / 1e9, 1),
+                         "tflops": round(fls[k] / (us * 1e-6) / 1e12, 1)})
+        tot_b = sum(bts.values())
+        dom = max(kern, key=lambda r: r["avg_us"])
+        print(json.dumps({
+            "metric": "SSD-form block-bidirectional forward tokens/s (clean + noisy stream pair counts once)",
+            "value": Bt * L / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": steps, "ms_per_step": ms,
+            "higher_is_better": True, "dtype": "bf16 operands, fp32 accumulate and state", "data": "synthetic",
+            "config": {"workload": f"{name}; batch {Bt}, {L} tokens per stream, block {Bs}; forward with every "
+                                   "block-end state", "batch": Bt, "seq_len": L, "block": Bs, "heads": H,
+                       "head_dim": 64, "d_state": N},
+            "hbm": {"achieved": round(tot_b / (ms * 1e-3) / 1e9, 1), "peak": hbm_peak, "unit": "GB/s",
+                    "frac": round(tot_b / (ms * 1e-3) / 1e9 / hbm_peak, 4), "alg_bytes_per_step": tot_b,
+                    "peak_kind": peak_kind},
+            "dominant": {"name": dom["name"], "hbm_frac": round(dom["alg_gbs"] / hbm_peak, 4),
+                         "tensor_frac": round(dom["tflops"] / tc_peak, 4)},
+            "wait_flag": flag, "kernels": kern}), flush=True)
+        del t, y_c, y_n, st, ws
+        torch.cuda.empty_cache()
+
+
 def run_prefill(args, L, Bs, calls):
     """Inference cache path at d_inner 2048, d_state 16, batch 1: the cache
     build over an L-token clean prefix (final state only, and every block-end
@@ -651,7 +763,7 @@ def main():
     ap.add_argument("--warmup-seconds", type=float, default=1.0,
                     help="keep warming up for at least this long (clock sampling under load)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (smaller profiling case)")
-    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k"],
+    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k", "ssd"],
                     help="layer: the step line; others: extra lines on one GPU")
     args = ap.parse_args()
     if args.batch:
@@ -666,6 +778,8 @@ def main():
         if rank == 0:
             if args.workload == "sweep":
                 run_sweep(args)
+            elif args.workload == "ssd":
+                run_ssd(args)
             elif args.workload == "prefill65k":
                 run_prefill(args, 65536, 32, 1)
             else:
