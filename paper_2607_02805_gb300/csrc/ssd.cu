@@ -247,46 +247,31 @@ __global__ void __launch_bounds__(256) k_ssd_state_pass(const SsdPassParams p) {
   float S = p.init != nullptr ? p.init[idx] : 0.f;
   const float* T = p.T + b * g.nb * per_b + r;
   const float* sd = p.sumdt + b * g.nb * g.H + h;
-  for (int k = 0; k < g.nb; ++k) {
-    S = __fmaf_rn(ex2(__fmul_rn(A2, sd[(int64_t)k * g.H])), S, T[(int64_t)k * per_b]);
-    if (p.emit_all) p.states[(b * g.nb + k) * per_b + r] = S;
+  constexpr int U = 8;  // loads of U blocks first: they do not depend on the state
+  for (int k0 = 0; k0 < g.nb; k0 += U) {
+    float tv[U], dv[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int k = min(k0 + u, g.nb - 1);
+      tv[u] = T[(int64_t)k * per_b];
+      dv[u] = sd[(int64_t)k * g.H];
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (k0 + u >= g.nb) break;
+      S = __fmaf_rn(ex2(__fmul_rn(A2, dv[u])), S, tv[u]);
+      if (p.emit_all) p.states[(b * g.nb + k0 + u) * per_b + r] = S;
+    }
   }
   if (!p.emit_all) p.states[b * per_b + r] = S;
   if (p.final_state != nullptr) p.final_state[b * per_b + r] = S;
 }
 
-// Shared memory of k_ssd_block_scan (offsets from a 1024-aligned base):
-//   Cf   the tile's C^f rows, K-major (N / 64 atom columns)
-//   M0   decay-weighted mixing tile, buffer 0 (128 x 128 bf16, K-major)
-//   M1   buffer 1; holds the tile's C^r rows until the Gram products are done
-//   R    the B tiles of the Gram products; afterwards the head's x tiles
-//        (MN-major, 16 KB each) followed by the seed's high and low parts
-//        (64 rows x N, K-major)
-//   cum  per token: A2 * cumulative dt and dt, for both directions
-struct ScanSmem {
-  uint32_t cf, m0, m1, r, x, seed, cum, total;
-  __host__ __device__ ScanSmem(int N, int m) {
-    const uint32_t tileC = 128u * (uint32_t)N * 2u;
-    const uint32_t tileM = 32768u;
-    cf = 0;
-    m0 = cf + tileC;
-    m1 = m0 + tileM;
-    const uint32_t m1sz = tileC > tileM ? tileC : tileM;
-    r = m1 + m1sz;
-    const uint32_t gram = (uint32_t)(m + 1) * tileC;
-    const uint32_t xs = (uint32_t)m * 16384u + 2u * 64u * (uint32_t)N * 2u;
-    x = r;
-    seed = r + (uint32_t)m * 16384u;
-    cum = r + (gram > xs ? gram : xs);
-    total = cum + 4u * 256u * 4u + 1024u;  // + alignment slack of the dynamic base
-  }
-};
-
 // Copies one 128-token tile of a [tokens][N] bf16 tensor into K-major
 // swizzled shared memory (N / 64 atom columns).
 template <int N>
 __device__ __forceinline__ void stage_rows(unsigned char* dst, const __nv_bfloat16* src) {
-  for (int c = threadIdx.x; c < 128 * N / 8; c += 128) {
+  for (int c = threadIdx.x; c < 128 * N / 8; c += blockDim.x) {
     const int r = c / (N / 8), ch = c % (N / 8);
     cp_async16(dst + (ch >> 3) * kTile16 + sw128(r, ch & 7), src + (int64_t)r * N + ch * 8, 16);
   }
@@ -303,32 +288,128 @@ __device__ __forceinline__ void mma_gram(uint32_t d, uint32_t a, uint32_t b) {
   }
 }
 
-// One CTA per (batch row, block, 128-token tile i of the block) and group of
-// heads. Thread t owns token row t of the tile (TMEM lane t).
+// Shared memory of k_ssd_block_scan (offsets from a 1024-aligned base):
+//   cf    the tile's C^f rows, K-major (N / 64 atom columns)
+//   m0    decay-weighted mixing tile, buffer 0 (128 x 128 bf16, K-major)
+//   m1    buffer 1; holds the tile's C^r rows until the Gram products are done
+//   r     the B tiles of the Gram products; afterwards the head's x tiles
+//         (MN-major, 16 KB each), the seed's bf16 high and low parts (64 rows
+//         x N, K-major) and the next head's seed as loaded (fp32)
+//   dt    dt of every head of the CTA, per token, both directions (fp32)
+//   vec   per token of the block, for the current head: A2 * cumulative dt,
+//         dt and the column factors of both directions
+struct ScanSmem {
+  uint32_t cf, m0, m1, r, x, seed, raw, dt, vec, total;
+  __host__ __device__ ScanSmem(int N, int m) {
+    const uint32_t tileC = 128u * (uint32_t)N * 2u;
+    const uint32_t tileM = 32768u;
+    cf = 0;
+    m0 = cf + tileC;
+    m1 = m0 + tileM;
+    r = m1 + (tileC > tileM ? tileC : tileM);
+    const uint32_t gram = (uint32_t)(m + 1) * tileC;
+    x = r;
+    seed = x + (uint32_t)m * 16384u;
+    raw = seed + 256u * (uint32_t)N;
+    const uint32_t xs = raw + 256u * (uint32_t)N - r;
+    dt = r + (gram > xs ? gram : xs);
+    vec = dt + 2u * 256u * 8u * 4u;
+    total = vec + 6u * 256u * 4u + 1024u;  // + alignment slack of the dynamic base
+  }
+};
+
+constexpr int kScanThreads = 256;
+constexpr int kMaxHeadsPerCta = 8;
+
+// Issues the cp.async copies of one head's x tiles (MN-major) and its seed
+// (fp32, as stored) for a CTA of kScanThreads threads.
+template <int N>
+__device__ __forceinline__ void issue_head_loads(unsigned char* sm, const ScanSmem& L, const __nv_bfloat16* x,
+                                                 int64_t tok0, int H, int h, int ntile, const float* seed_h) {
+  for (int c = threadIdx.x; c < ntile * kSsdT * 8; c += kScanThreads) {
+    const int s = c >> 3, ch = c & 7;
+    cp_async16(sm + L.x + (s >> 7) * 16384u + sw128(s & 127, ch), x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+  }
+  if (seed_h != nullptr)
+    for (int c = threadIdx.x; c < kSsdP * N / 4; c += kScanThreads) cp_async16(sm + L.raw + c * 16, seed_h + c * 4, 16);
+  cp_async_commit();
+}
+
+// Inclusive scan over the block of one head's dt held in shared memory
+// (stride `hs` floats between tokens), by one warp; REV scans from the end.
+template <bool REV>
+__device__ __forceinline__ void warp_scan_smem(const float* dt, int hs, int n, float* out) {
+  const int lane = threadIdx.x & 31, per = n / 32;
+  float loc[8];
+  float s = 0.f;
+  for (int q = 0; q < per; ++q) {
+    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
+    s = __fadd_rn(s, dt[pos * hs]);
+    loc[q] = s;
+  }
+  float inc = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float v = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc = __fadd_rn(inc, v);
+  }
+  float base = __shfl_up_sync(0xffffffffu, inc, 1);
+  if (lane == 0) base = 0.f;
+  for (int q = 0; q < per; ++q) {
+    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
+    out[pos] = __fadd_rn(base, loc[q]);
+  }
+}
+
+// One CTA of 8 warps per (batch row, block, 128-token tile i of the block)
+// and group of at most 8 heads. Warp w serves token rows 32 (w % 4) .. +31 of
+// the tile (TMEM lanes of its quarter) and column half w / 4 of each mixing
+// tile and of the output.
 // TMEM columns: Gram products at 128 q (forward products of s-tiles 0..i,
 // then, for noisy blocks, reverse products of s-tiles i..m-1), the output
 // accumulator at 384 and the seed term at 448.
+// Decays: inside the block, exp(A sum dt) between rows and columns that are
+// 32-token groups apart factors exactly into a row factor times a column
+// factor, both at most 1 (referenced to the column group's last token for
+// the forward direction and its first token for the reverse one); only the
+// 32 x 32 blocks on the diagonal take one exp per element.
 template <int N, bool NOISY>
-__global__ void __launch_bounds__(128, 1) k_ssd_block_scan(const SsdScanParams p) {
+__global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdScanParams p) {
   extern __shared__ unsigned char smraw[];
   unsigned char* sm = align1024(smraw);
   __shared__ uint64_t bar[3];
   __shared__ uint32_t tslot;
   const SsdGeo& g = p.g;
   const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x;
+  const int w = t >> 5, lane = t & 31, q4 = w & 3, hf = w >> 2;
   const ScanSmem L(N, m);
   const int64_t idx = blockIdx.x;
   const int i = (int)(idx % m);
   const int64_t bk = idx / m, b = bk / g.nb;
   const int k = (int)(bk % g.nb);
-  const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg);
+  const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
   const int64_t tok0 = b * g.L + (int64_t)k * Bs;
-  const int tt = i * kSsdT + t;  // this thread's token inside the block
-  float* s_af = reinterpret_cast<float*>(sm + L.cum);  // A2_f * inclusive prefix sums of dt_f
-  float* s_wf = s_af + 256;                            // dt_f
-  float* s_ar = s_wf + 256;                            // A2_r * inclusive suffix sums of dt_r
-  float* s_wr = s_ar + 256;                            // dt_r
-  const int nf = i + 1, nr = NOISY ? m - i : 0;        // Gram products per direction
+  const int row = 32 * q4 + lane, tt = i * kSsdT + row;  // token row in the tile / in the block
+  const int rg = 4 * i + q4;                              // 32-token row group in the block
+  float* s_dtf = reinterpret_cast<float*>(sm + L.dt);     // [Bs][hg]
+  float* s_dtr = s_dtf + 256 * kMaxHeadsPerCta;
+  float* s_af = reinterpret_cast<float*>(sm + L.vec);     // A2_f * inclusive prefix sums of dt_f
+  float* s_wf = s_af + 256;                               // dt_f
+  float* s_cf = s_wf + 256;                               // forward column factors
+  float* s_ar = s_cf + 256;                               // A2_r * inclusive suffix sums of dt_r
+  float* s_wr = s_ar + 256;                               // dt_r
+  float* s_cr = s_wr + 256;                               // reverse column factors
+  const int nf = i + 1, nr = NOISY ? m - i : 0;           // Gram products per direction
+  const int ntile = NOISY ? m : i + 1;                    // s-tiles whose x a head needs
+  // this block's seed: slot k - 1 (or k) of p.seed; block 0 of a shifted
+  // layout starts from init_seed
+  const float* seed_src = nullptr;
+  if (p.seed_shift && k == 0) {
+    if (p.init_seed != nullptr) seed_src = p.init_seed + b * (int64_t)H * kSsdP * N;
+  } else if (p.seed != nullptr) {
+    seed_src = p.seed + b * p.seed_bstride + (int64_t)(p.seed_shift ? k - 1 : k) * H * kSsdP * N;
+  }
+  const bool has_seed = seed_src != nullptr;
   // --- Gram products C B^T of this tile against the block's s-tiles
   stage_rows<N>(sm + L.cf, p.Cf + (tok0 + i * kSsdT) * N);
   for (int j = 0; j < nf; ++j) stage_rows<N>(sm + L.r + j * 128u * N * 2u, p.Bf + (tok0 + j * kSsdT) * N);
@@ -338,6 +419,11 @@ __global__ void __launch_bounds__(128, 1) k_ssd_block_scan(const SsdScanParams p
       stage_rows<N>(sm + L.r + (nf + j - i) * 128u * N * 2u, p.Br + (tok0 + j * kSsdT) * N);
   }
   cp_async_commit();
+  for (int e = t; e < Bs * hg; e += kScanThreads) {  // dt of the CTA's heads, fp32
+    const int s = e / hg, hh = e - s * hg;
+    s_dtf[s * hg + hh] = __bfloat162float(p.dtf[(tok0 + s) * H + h0 + hh]);
+    if (NOISY) s_dtr[s * hg + hh] = __bfloat162float(p.dtr[(tok0 + s) * H + h0 + hh]);
+  }
   if (t == 0) {
     umma::bar_init(&bar[0], 1);
     umma::bar_init(&bar[1], 1);
@@ -350,41 +436,54 @@ __global__ void __launch_bounds__(128, 1) k_ssd_block_scan(const SsdScanParams p
   __syncthreads();
   umma::fence_after_sync();
   const uint32_t tm = tslot;
-  const uint32_t lane = tm + ((uint32_t)(t & ~31) << 16);
+  const uint32_t lane_base = tm + ((uint32_t)(32 * q4) << 16);
   if (t == 0) {
     const uint32_t base = umma::smem_u32(sm);
-    for (int q = 0; q < nf + nr; ++q)
-      mma_gram<N>(tm + 128u * q, base + (q < nf ? L.cf : L.m1), base + L.r + q * 128u * N * 2u);
+    for (int qq = 0; qq < nf + nr; ++qq)
+      mma_gram<N>(tm + 128u * qq, base + (qq < nf ? L.cf : L.m1), base + L.r + qq * 128u * N * 2u);
     umma::mma_commit(&bar[2]);
   }
   bool alive = cta_wait(&bar[2], 0, p.flag);
   umma::fence_after_sync();
-  bool pend[2] = {false, false};
-  uint32_t ph[2] = {0u, 0u};
-  int gt = 0;  // M tiles issued so far (selects the buffer)
-  // this block's seed: slot k - 1 (or k) of p.seed; block 0 of a shifted
-  // layout starts from init_seed
-  const float* seed_src = nullptr;
-  if (p.seed_shift && k == 0) {
-    if (p.init_seed != nullptr) seed_src = p.init_seed + b * (int64_t)H * kSsdP * N;
-  } else if (p.seed != nullptr) {
-    seed_src = p.seed + b * p.seed_bstride + (int64_t)(p.seed_shift ? k - 1 : k) * H * kSsdP * N;
-  }
-  const bool has_seed = seed_src != nullptr;
-  const int ntile = NOISY ? m : i + 1;  // s-tiles whose x the head needs
+  // the first head's x and seed (the B tiles are no longer read)
+  if (alive && h0 < h1)
+    issue_head_loads<N>(sm, L, p.x, tok0, H, h0, ntile, has_seed ? seed_src + (int64_t)h0 * kSsdP * N : nullptr);
+  uint32_t pend = 0u, ph = 0u;  // per mixing buffer: a commit not yet waited for; its phase parity
+  int gt = 0;                    // mixing tiles issued so far (selects the buffer)
+  auto wait_buf = [&](int bb) -> bool {
+    if (!((pend >> bb) & 1u)) return true;
+    if (!cta_wait(&bar[bb], (ph >> bb) & 1u, p.flag)) return false;
+    ph ^= 1u << bb;
+    pend &= ~(1u << bb);
+    return true;
+  };
   for (int h = h0; h < h1 && alive; ++h) {
-    // --- the head's x tiles (MN-major) and its seed (bf16 high + low, K-major)
-    for (int c = t; c < ntile * kSsdT * 8; c += 128) {
-      const int s = c >> 3, ch = c & 7;  // token s of the block (tile s / 128)
-      cp_async16(sm + L.x + (s >> 7) * 16384u + sw128(s & 127, ch), p.x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+    const int hh = h - h0;
+    cp_async_wait_all();
+    __syncthreads();
+    // --- the head's decay exponents (fp32, fixed order) and its seed in bf16 high + low parts
+    if (w == 0) {
+      warp_scan_smem<false>(s_dtf + hh, hg, Bs, s_af);
+      __syncwarp();
+      const float A2 = __fmul_rn(p.Af[h], kLog2e);
+      for (int s = lane; s < Bs; s += 32) {
+        s_af[s] = __fmul_rn(A2, s_af[s]);
+        s_wf[s] = s_dtf[s * hg + hh];
+      }
+    } else if (NOISY && w == 1) {
+      warp_scan_smem<true>(s_dtr + hh, hg, Bs, s_ar);
+      __syncwarp();
+      const float A2 = __fmul_rn(p.Ar[h], kLog2e);
+      for (int s = lane; s < Bs; s += 32) {
+        s_ar[s] = __fmul_rn(A2, s_ar[s]);
+        s_wr[s] = s_dtr[s * hg + hh];
+      }
     }
-    cp_async_commit();
     if (has_seed) {
-      const float* src = seed_src + (int64_t)h * kSsdP * N;
-      for (int c = t; c < kSsdP * N / 8; c += 128) {
+      for (int c = t; c < kSsdP * N / 8; c += kScanThreads) {
         const int pr = c / (N / 8), ch = c % (N / 8);
-        const float4 u0 = *reinterpret_cast<const float4*>(src + (int64_t)pr * N + ch * 8);
-        const float4 u1 = *reinterpret_cast<const float4*>(src + (int64_t)pr * N + ch * 8 + 4);
+        const float4 u0 = *reinterpret_cast<const float4*>(sm + L.raw + (pr * N + ch * 8) * 4);
+        const float4 u1 = *reinterpret_cast<const float4*>(sm + L.raw + (pr * N + ch * 8 + 4) * 4);
         const float v[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
         uint32_t wh[4], wl[4];
 #pragma unroll
@@ -398,29 +497,15 @@ __global__ void __launch_bounds__(128, 1) k_ssd_block_scan(const SsdScanParams p
         *reinterpret_cast<uint4*>(sm + L.seed + 128u * N + off) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
       }
     }
-    // --- decay exponents of the head: A2 * cumulative dt (fp32, fixed order)
-    if (t < 32) {
-      const __nv_bfloat16* d = p.dtf + tok0 * H + h;
-      warp_scan_dt<false>(d, H, Bs, s_af);
-      __syncwarp();
-      const float A2 = __fmul_rn(p.Af[h], kLog2e);
-      for (int s = t; s < Bs; s += 32) {
-        s_af[s] = __fmul_rn(A2, s_af[s]);
-        s_wf[s] = __bfloat162float(d[(int64_t)s * H]);
-      }
-    } else if (NOISY && t < 64) {
-      const __nv_bfloat16* d = p.dtr + tok0 * H + h;
-      warp_scan_dt<true>(d, H, Bs, s_ar);
-      __syncwarp();
-      const float A2 = __fmul_rn(p.Ar[h], kLog2e);
-      for (int s = t - 32; s < Bs; s += 32) {
-        s_ar[s] = __fmul_rn(A2, s_ar[s]);
-        s_wr[s] = __bfloat162float(d[(int64_t)s * H]);
-      }
-    }
-    cp_async_wait_all();
     umma::fence_async_smem();
     __syncthreads();
+    // column factors: forward referenced to the column group's last token,
+    // reverse to its first
+    for (int s = t; s < Bs; s += kScanThreads) {
+      const int g0 = s & ~31;
+      s_cf[s] = __fmul_rn(ex2(__fsub_rn(s_af[g0 + 31], s_af[s])), s_wf[s]);
+      if (NOISY) s_cr[s] = __fmul_rn(ex2(__fsub_rn(s_ar[g0], s_ar[s])), s_wr[s]);
+    }
     if (t == 0 && has_seed) {  // seed term C^f . seed^T into columns 448..511
       umma::fence_after_sync();
       const uint32_t base = umma::smem_u32(sm);
@@ -434,45 +519,61 @@ __global__ void __launch_bounds__(128, 1) k_ssd_block_scan(const SsdScanParams p
         umma::mma_bf16(tm + 448, a, umma::sdesc(base + L.seed + 128u * N + offs, 16, 1024), id, true);
       }
     }
+    __syncthreads();
     // --- decay-weighted mixing tiles, one per s-tile, each multiplied with x
     const float af_t = s_af[tt];
     const float ar_t = NOISY ? s_ar[tt] : 0.f;
     for (int j = 0; j < ntile; ++j, ++gt) {
       const int bb = gt & 1;
-      if (pend[bb]) {
-        if (!cta_wait(&bar[bb], ph[bb], p.flag)) {
-          alive = false;
-          break;
-        }
-        ph[bb] ^= 1u;
-        pend[bb] = false;
+      if (!wait_buf(bb)) {
+        alive = false;
+        break;
       }
       unsigned char* mt = sm + (bb ? L.m1 : L.m0);
-      const bool use_f = j <= i, use_r = NOISY && j >= i;  // uniform over the CTA
       const uint32_t colf = 128u * j, colr = 128u * (nf + j - i);
 #pragma unroll 1
-      for (int c32 = 0; c32 < 4; ++c32) {
-        float gf[32], gr[32], v[32];
-        if (use_f) umma::tmem_ld32(lane + colf + 32u * c32, gf);
-        if (use_r) umma::tmem_ld32(lane + colr + 32u * c32, gr);
+      for (int c = 0; c < 2; ++c) {
+        const int cg = 2 * hf + c, sg = 4 * j + cg, s0 = 32 * sg;  // column group of the tile / block
+        // 0: no term, 1: factored decay, 2: diagonal block (one exp per element); uniform per warp
+        const int fm = j > i ? 0 : (sg < rg ? 1 : (sg == rg ? 2 : 0));
+        const int rm = !NOISY || j < i ? 0 : (sg > rg ? 1 : (sg == rg ? 2 : 0));
+        float v[32];
 #pragma unroll
-        for (int q = 0; q < 32; ++q) {
-          const int ss = j * kSsdT + c32 * 32 + q;
-          float val = 0.f;
-          if (use_f) {
-            const float e = __fmul_rn(ex2(__fsub_rn(af_t, s_af[ss])), s_wf[ss]);
-            val = ss <= tt ? __fmul_rn(gf[q], e) : 0.f;
+        for (int e = 0; e < 32; ++e) v[e] = 0.f;
+        if (fm != 0) {
+          float gv[32];
+          umma::tmem_ld32(lane_base + colf + 32u * cg, gv);
+          if (fm == 1) {
+            const float rf = ex2(__fsub_rn(af_t, s_af[s0 + 31]));
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] = __fmul_rn(__fmul_rn(gv[e], s_cf[s0 + e]), rf);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const float d = __fmul_rn(ex2(__fsub_rn(af_t, s_af[s0 + e])), s_wf[s0 + e]);
+              v[e] = s0 + e <= tt ? __fmul_rn(gv[e], d) : 0.f;
+            }
           }
-          if (use_r) {
-            const float e = __fmul_rn(ex2(__fsub_rn(ar_t, s_ar[ss])), s_wr[ss]);
-            val = __fadd_rn(val, ss >= tt ? __fmul_rn(gr[q], e) : 0.f);
+        }
+        if (rm != 0) {
+          float gv[32];
+          umma::tmem_ld32(lane_base + colr + 32u * cg, gv);
+          if (rm == 1) {
+            const float rf = ex2(__fsub_rn(ar_t, s_ar[s0]));
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] = __fadd_rn(v[e], __fmul_rn(__fmul_rn(gv[e], s_cr[s0 + e]), rf));
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const float d = __fmul_rn(ex2(__fsub_rn(ar_t, s_ar[s0 + e])), s_wr[s0 + e]);
+              v[e] = __fadd_rn(v[e], s0 + e >= tt ? __fmul_rn(gv[e], d) : 0.f);
+            }
           }
-          v[q] = val;
         }
 #pragma unroll
         for (int ch = 0; ch < 4; ++ch) {
-          const int col = c32 * 32 + ch * 8;  // s inside the tile
-          *reinterpret_cast<uint4*>(mt + (col >> 6) * kTile16 + sw128(t, (col & 63) >> 3)) =
+          const int col = 32 * cg + 8 * ch;  // s inside the tile
+          *reinterpret_cast<uint4*>(mt + (col >> 6) * kTile16 + sw128(row, (col & 63) >> 3)) =
               make_uint4(pack_bf16(v[ch * 8], v[ch * 8 + 1]), pack_bf16(v[ch * 8 + 2], v[ch * 8 + 3]),
                          pack_bf16(v[ch * 8 + 4], v[ch * 8 + 5]), pack_bf16(v[ch * 8 + 6], v[ch * 8 + 7]));
         }
@@ -490,40 +591,39 @@ __global__ void __launch_bounds__(128, 1) k_ssd_block_scan(const SsdScanParams p
                          umma::sdesc(xb + kk * 2048u, 1024, 1024), id, j > 0 || kk > 0);
         umma::mma_commit(&bar[bb]);
       }
-      pend[bb] = true;
+      pend |= 1u << bb;
     }
-    if (!alive || !drain(bar, pend, ph, p.flag)) {
+    if (!alive || !wait_buf(0) || !wait_buf(1)) {
       alive = false;
       break;
     }
     umma::fence_after_sync();
-    // --- epilogue: y = mixing term + decayed seed term + D x, bf16 out
+    // the next head's loads run under this head's epilogue
+    if (h + 1 < h1)
+      issue_head_loads<N>(sm, L, p.x, tok0, H, h + 1, ntile, has_seed ? seed_src + (int64_t)(h + 1) * kSsdP * N : nullptr);
+    // --- epilogue: y = mixing term + decayed seed term + D x, bf16 out;
+    // this warp's 32 channels of its token row
     {
-      float ya[64], yo[64];
-      umma::tmem_ld32(lane + 384, *reinterpret_cast<float(*)[32]>(&ya[0]));
-      umma::tmem_ld32(lane + 416, *reinterpret_cast<float(*)[32]>(&ya[32]));
-      if (has_seed) {
-        umma::tmem_ld32(lane + 448, *reinterpret_cast<float(*)[32]>(&yo[0]));
-        umma::tmem_ld32(lane + 480, *reinterpret_cast<float(*)[32]>(&yo[32]));
-      }
+      float ya[32], yo[32];
+      umma::tmem_ld32(lane_base + 384u + 32u * hf, ya);
+      if (has_seed) umma::tmem_ld32(lane_base + 448u + 32u * hf, yo);
       const float dec = has_seed ? ex2(af_t) : 0.f;
       const float Dd = NOISY ? __fadd_rn(p.Df[h], p.Dr[h]) : p.Df[h];
-      const unsigned char* xr = sm + L.x + (uint32_t)i * 16384u;
-      __nv_bfloat16* dst = p.y + ((tok0 + tt) * H + h) * kSsdP;
+      const int64_t off = ((tok0 + tt) * H + h) * kSsdP + 32 * hf;
+      const uint4* xg = reinterpret_cast<const uint4*>(p.x + off);
+      uint4* yg = reinterpret_cast<uint4*>(p.y + off);
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) {
-        const uint4 xv = *reinterpret_cast<const uint4*>(xr + sw128(t, ch));
+      for (int ch = 0; ch < 4; ++ch) {
+        const uint4 xv = xg[ch];
         const __nv_bfloat16* xe = reinterpret_cast<const __nv_bfloat16*>(&xv);
         float o[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const int q = ch * 8 + e;
-          float acc = ya[q];
-          if (has_seed) acc = __fmaf_rn(dec, yo[q], acc);
+          float acc = ya[ch * 8 + e];
+          if (has_seed) acc = __fmaf_rn(dec, yo[ch * 8 + e], acc);
           o[e] = __fmaf_rn(Dd, __bfloat162float(xe[e]), acc);
         }
-        *reinterpret_cast<uint4*>(dst + ch * 8) =
-            make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]), pack_bf16(o[6], o[7]));
+        yg[ch] = make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]), pack_bf16(o[6], o[7]));
       }
     }
     umma::fence_before_sync();
@@ -582,11 +682,12 @@ template <int N, bool NOISY>
 cudaError_t scan_t(const SsdScanParams& p, cudaStream_t s) {
   const int64_t tiles = p.g.Bt * p.g.nb * p.g.m;
   if (tiles == 0 || p.g.H == 0) return cudaSuccess;
+  if (p.hg < 1 || p.hg > kMaxHeadsPerCta) return cudaErrorInvalidValue;
   const ScanSmem L(N, p.g.m);
   cudaError_t e = set_smem(k_ssd_block_scan<N, NOISY>, L.total);
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)tiles, (unsigned)((p.g.H + p.hg - 1) / p.hg));
-  k_ssd_block_scan<N, NOISY><<<grid, 128, L.total, s>>>(p);
+  k_ssd_block_scan<N, NOISY><<<grid, kScanThreads, L.total, s>>>(p);
   return cudaGetLastError();
 }
 
