@@ -292,14 +292,16 @@ __device__ __forceinline__ void mma_gram(uint32_t d, uint32_t a, uint32_t b) {
 //   cf    the tile's C^f rows, K-major (N / 64 atom columns)
 //   m0    decay-weighted mixing tile, buffer 0 (128 x 128 bf16, K-major)
 //   m1    buffer 1; holds the tile's C^r rows until the Gram products are done
-//   r     the B tiles of the Gram products; afterwards the head's x tiles
-//         (MN-major, 16 KB each), the seed's bf16 high and low parts (64 rows
-//         x N, K-major) and the next head's seed as loaded (fp32)
+//   r     the B tiles of the Gram products; afterwards two buffers of a
+//         head's x tiles (MN-major, 16 KB each; the current head and the next)
+//         and the seed's bf16 high and low parts (64 rows x N, K-major).
+//         The next head's seed, as loaded (fp32), waits in m1 (free between
+//         a head's last mixing tile and the next head's second one).
 //   dt    dt of every head of the CTA, per token, both directions (fp32)
 //   vec   per token of the block, for the current head: A2 * cumulative dt,
 //         dt and the column factors of both directions
 struct ScanSmem {
-  uint32_t cf, m0, m1, r, x, seed, raw, dt, vec, total;
+  uint32_t cf, m0, m1, r, x, xsz, seed, raw, dt, vec, prm, total;
   __host__ __device__ ScanSmem(int N, int m) {
     const uint32_t tileC = 128u * (uint32_t)N * 2u;
     const uint32_t tileM = 32768u;
@@ -309,12 +311,14 @@ struct ScanSmem {
     r = m1 + (tileC > tileM ? tileC : tileM);
     const uint32_t gram = (uint32_t)(m + 1) * tileC;
     x = r;
-    seed = x + (uint32_t)m * 16384u;
-    raw = seed + 256u * (uint32_t)N;
-    const uint32_t xs = raw + 256u * (uint32_t)N - r;
+    xsz = (uint32_t)m * 16384u;
+    seed = x + 2u * xsz;
+    raw = m1;
+    const uint32_t xs = 2u * xsz + 256u * (uint32_t)N;
     dt = r + (gram > xs ? gram : xs);
     vec = dt + 2u * 256u * 8u * 4u;
-    total = vec + 6u * 256u * 4u + 1024u;  // + alignment slack of the dynamic base
+    prm = vec + 6u * 256u * 4u;
+    total = prm + 4u * 8u * 4u + 1024u;  // + alignment slack of the dynamic base
   }
 };
 
@@ -325,10 +329,11 @@ constexpr int kMaxHeadsPerCta = 8;
 // (fp32, as stored) for a CTA of kScanThreads threads.
 template <int N>
 __device__ __forceinline__ void issue_head_loads(unsigned char* sm, const ScanSmem& L, const __nv_bfloat16* x,
-                                                 int64_t tok0, int H, int h, int ntile, const float* seed_h) {
+                                                 int64_t tok0, int H, int h, int ntile, const float* seed_h,
+                                                 uint32_t xbuf) {
   for (int c = threadIdx.x; c < ntile * kSsdT * 8; c += kScanThreads) {
     const int s = c >> 3, ch = c & 7;
-    cp_async16(sm + L.x + (s >> 7) * 16384u + sw128(s & 127, ch), x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+    cp_async16(sm + xbuf + (s >> 7) * 16384u + sw128(s & 127, ch), x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
   }
   if (seed_h != nullptr)
     for (int c = threadIdx.x; c < kSsdP * N / 4; c += kScanThreads) cp_async16(sm + L.raw + c * 16, seed_h + c * 4, 16);
@@ -419,6 +424,15 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       stage_rows<N>(sm + L.r + (nf + j - i) * 128u * N * 2u, p.Br + (tok0 + j * kSsdT) * N);
   }
   cp_async_commit();
+  float* s_prm = reinterpret_cast<float*>(sm + L.prm);  // [4][8]: A_f, D_f, A_r, D_r of the CTA's heads
+  if (t < hg) {
+    s_prm[t] = p.Af[h0 + t];
+    s_prm[8 + t] = p.Df[h0 + t];
+    if (NOISY) {
+      s_prm[16 + t] = p.Ar[h0 + t];
+      s_prm[24 + t] = p.Dr[h0 + t];
+    }
+  }
   for (int e = t; e < Bs * hg; e += kScanThreads) {  // dt of the CTA's heads, fp32
     const int s = e / hg, hh = e - s * hg;
     s_dtf[s * hg + hh] = __bfloat162float(p.dtf[(tok0 + s) * H + h0 + hh]);
@@ -447,9 +461,8 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   umma::fence_after_sync();
   // the first head's x and seed (the B tiles are no longer read)
   if (alive && h0 < h1)
-    issue_head_loads<N>(sm, L, p.x, tok0, H, h0, ntile, has_seed ? seed_src + (int64_t)h0 * kSsdP * N : nullptr);
+    issue_head_loads<N>(sm, L, p.x, tok0, H, h0, ntile, has_seed ? seed_src + (int64_t)h0 * kSsdP * N : nullptr, L.x);
   uint32_t pend = 0u, ph = 0u;  // per mixing buffer: a commit not yet waited for; its phase parity
-  int gt = 0;                    // mixing tiles issued so far (selects the buffer)
   auto wait_buf = [&](int bb) -> bool {
     if (!((pend >> bb) & 1u)) return true;
     if (!cta_wait(&bar[bb], (ph >> bb) & 1u, p.flag)) return false;
@@ -459,13 +472,14 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   };
   for (int h = h0; h < h1 && alive; ++h) {
     const int hh = h - h0;
+    const uint32_t xcur = L.x + (hh & 1) * L.xsz;  // this head's x tiles
     cp_async_wait_all();
     __syncthreads();
     // --- the head's decay exponents (fp32, fixed order) and its seed in bf16 high + low parts
     if (w == 0) {
       warp_scan_smem<false>(s_dtf + hh, hg, Bs, s_af);
       __syncwarp();
-      const float A2 = __fmul_rn(p.Af[h], kLog2e);
+      const float A2 = __fmul_rn(s_prm[hh], kLog2e);
       for (int s = lane; s < Bs; s += 32) {
         s_af[s] = __fmul_rn(A2, s_af[s]);
         s_wf[s] = s_dtf[s * hg + hh];
@@ -473,7 +487,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     } else if (NOISY && w == 1) {
       warp_scan_smem<true>(s_dtr + hh, hg, Bs, s_ar);
       __syncwarp();
-      const float A2 = __fmul_rn(p.Ar[h], kLog2e);
+      const float A2 = __fmul_rn(s_prm[16 + hh], kLog2e);
       for (int s = lane; s < Bs; s += 32) {
         s_ar[s] = __fmul_rn(A2, s_ar[s]);
         s_wr[s] = s_dtr[s * hg + hh];
@@ -523,8 +537,8 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     // --- decay-weighted mixing tiles, one per s-tile, each multiplied with x
     const float af_t = s_af[tt];
     const float ar_t = NOISY ? s_ar[tt] : 0.f;
-    for (int j = 0; j < ntile; ++j, ++gt) {
-      const int bb = gt & 1;
+    for (int j = 0; j < ntile; ++j) {
+      const int bb = j & 1;  // tile 0 -> m0, tile 1 -> m1 (m1 also holds the next seed in between)
       if (!wait_buf(bb)) {
         alive = false;
         break;
@@ -583,7 +597,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       __syncthreads();
       if (t == 0) {
         umma::fence_after_sync();
-        const uint32_t ma = umma::smem_u32(mt), xb = umma::smem_u32(sm + L.x) + (uint32_t)j * 16384u;
+        const uint32_t ma = umma::smem_u32(mt), xb = umma::smem_u32(sm + xcur) + (uint32_t)j * 16384u;
         constexpr uint32_t id = umma::idesc_bf16(128, 64, false, true);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
@@ -600,7 +614,8 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     umma::fence_after_sync();
     // the next head's loads run under this head's epilogue
     if (h + 1 < h1)
-      issue_head_loads<N>(sm, L, p.x, tok0, H, h + 1, ntile, has_seed ? seed_src + (int64_t)(h + 1) * kSsdP * N : nullptr);
+      issue_head_loads<N>(sm, L, p.x, tok0, H, h + 1, ntile, has_seed ? seed_src + (int64_t)(h + 1) * kSsdP * N : nullptr,
+                          L.x + ((hh + 1) & 1) * L.xsz);
     // --- epilogue: y = mixing term + decayed seed term + D x, bf16 out;
     // this warp's 32 channels of its token row
     {
@@ -608,13 +623,13 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       umma::tmem_ld32(lane_base + 384u + 32u * hf, ya);
       if (has_seed) umma::tmem_ld32(lane_base + 448u + 32u * hf, yo);
       const float dec = has_seed ? ex2(af_t) : 0.f;
-      const float Dd = NOISY ? __fadd_rn(p.Df[h], p.Dr[h]) : p.Df[h];
+      const float Dd = NOISY ? __fadd_rn(s_prm[8 + hh], s_prm[24 + hh]) : s_prm[8 + hh];
       const int64_t off = ((tok0 + tt) * H + h) * kSsdP + 32 * hf;
-      const uint4* xg = reinterpret_cast<const uint4*>(p.x + off);
+      const unsigned char* xr = sm + xcur + (uint32_t)i * 16384u;
       uint4* yg = reinterpret_cast<uint4*>(p.y + off);
 #pragma unroll
       for (int ch = 0; ch < 4; ++ch) {
-        const uint4 xv = xg[ch];
+        const uint4 xv = *reinterpret_cast<const uint4*>(xr + sw128(row, 4 * hf + ch));
         const __nv_bfloat16* xe = reinterpret_cast<const __nv_bfloat16*>(&xv);
         float o[8];
 #pragma unroll
