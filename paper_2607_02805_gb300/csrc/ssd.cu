@@ -94,146 +94,165 @@ __device__ __forceinline__ bool drain(uint64_t* bar, bool (&pend)[2], uint32_t (
   return ok;
 }
 
-// Shared memory of k_ssd_block_state (offsets from a 1024-aligned base).
+// Shared memory of k_ssd_block_state (offsets from a 1024-aligned base):
+//   b     the block's B rows as the MN-major A operand: two 64-wide halves of
+//         [Bs][64] bf16 (state rows 64..127 are zero when N = 64)
+//   xr    two buffers of a head's x rows as loaded ([Bs][64] bf16, swizzled)
+//   xs    the weighted x of the current head, bf16 high and low parts, each
+//         [Bs][64] MN-major (the B operand)
+//   w     per head of the CTA and token: exp(A sum_{r>s} dt_r) dt_s
 struct StateSmem {
-  static constexpr uint32_t kA = 0;        // [2 buffers][hi, lo][128 rows x 64 tokens] bf16, swizzled
-  static constexpr uint32_t kX = 65536;    // [Bs][64] bf16, MN-major swizzled
-  static constexpr uint32_t kB = 98304;    // [Bs][N] bf16, plain row-major
-  static __host__ __device__ uint32_t w(int N) { return kB + 256u * (uint32_t)N * 2u; }  // w[256], suf[256]
-  static __host__ __device__ uint32_t bytes(int N) { return w(N) + 2048u + 1024u; }
+  uint32_t b, xr, xs, w, total;
+  __host__ __device__ StateSmem(int Bs) {
+    const uint32_t half = (uint32_t)Bs * 128u;
+    b = 0;
+    xr = b + 2u * half;
+    xs = xr + 2u * half;
+    w = xs + 2u * half;
+    total = w + 8u * 256u * 4u + 1024u;
+  }
 };
 
-// One CTA per (batch row, block) and group of heads; thread n owns state row n.
+constexpr int kStateThreads = 256;
+
+// One CTA of 8 warps per (batch row, block) and group of at most 8 heads.
+// T^T[n][p] = sum_s B_s[n] (w_s x_s[p]): M = 128 state rows, N = 64
+// channels, K = Bs tokens; warps w and w + 4 read TMEM lanes 32 (w % 4) and
+// split the 64 channels. Head h's MMAs run while head h-1's accumulator is
+// written out (two accumulators, TMEM columns 0..63 and 64..127).
 template <int N>
-__global__ void __launch_bounds__(128, 1) k_ssd_block_state(const SsdStateParams p) {
+__global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdStateParams p) {
   extern __shared__ unsigned char smraw[];
   unsigned char* sm = align1024(smraw);
   __shared__ uint64_t bar[2];
   __shared__ uint32_t tslot;
   const SsdGeo& g = p.g;
-  const int Bs = (int)g.Bs, H = g.H, t = threadIdx.x;
+  const int Bs = (int)g.Bs, H = g.H, t = threadIdx.x, w = t >> 5, lane = t & 31;
+  const StateSmem S(Bs);
+  const uint32_t half = (uint32_t)Bs * 128u;
   const int64_t bk = blockIdx.x, b = bk / g.nb;
   const int k = (int)(bk % g.nb);
-  const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg);
-  unsigned char* sA = sm + StateSmem::kA;
-  unsigned char* sX = sm + StateSmem::kX;
-  const __nv_bfloat16* sB = reinterpret_cast<const __nv_bfloat16*>(sm + StateSmem::kB);
-  float* sw = reinterpret_cast<float*>(sm + StateSmem::w(N));
-  float* ssuf = sw + 256;
+  const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
   const int64_t tok0 = b * g.L + (int64_t)k * Bs;
-  {  // the block's B rows are contiguous in memory
-    const char* src = reinterpret_cast<const char*>(p.B + tok0 * N);
-    for (int c = t; c < Bs * N / 8; c += 128) cp_async16(sm + StateSmem::kB + c * 16, src + c * 16, 16);
-    cp_async_commit();
+  float* s_w = reinterpret_cast<float*>(sm + S.w);  // [hg][256]
+  // B rows: chunk c of 8 state indices of token s goes to half c / 8
+  for (int c = t; c < Bs * N / 8; c += kStateThreads) {
+    const int s = c / (N / 8), ch = c % (N / 8);
+    cp_async16(sm + S.b + (ch >> 3) * half + sw128(s, ch & 7), p.B + (tok0 + s) * N + ch * 8, 16);
   }
-  if (N < 128 && t >= N) {  // state rows beyond N stay zero in both buffers
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(sA + q * kTile16 + sw128(t, c)) = make_uint4(0, 0, 0, 0);
+  if (N == 64)
+    for (int c = t; c < Bs * 8; c += kStateThreads)
+      *reinterpret_cast<uint4*>(sm + S.b + half + c * 16) = make_uint4(0, 0, 0, 0);
+  auto load_x = [&](int h, int buf) {
+    for (int c = t; c < Bs * 8; c += kStateThreads) {
+      const int s = c >> 3, ch = c & 7;
+      cp_async16(sm + S.xr + buf * half + sw128(s, ch), p.x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+    }
+    cp_async_commit();
+  };
+  if (h0 < h1) load_x(h0, 0);
+  // weights of every head of the CTA: warp hh scans head hh (suffix sums)
+  if (w < hg) {
+    const int h = h0 + w;
+    const __nv_bfloat16* dth = p.dt + tok0 * H + h;
+    float* suf = s_w + w * 256;
+    const float tot = warp_scan_dt<true>(dth, H, Bs, suf);  // inclusive suffix sums
+    __syncwarp();
+    const float A2 = __fmul_rn(p.A[h], kLog2e);
+    float wv[8];
+    for (int q = 0, s = lane; s < Bs; s += 32, ++q) {
+      const float after = s + 1 < Bs ? suf[s + 1] : 0.f;  // sum of dt over tokens after s
+      wv[q] = __fmul_rn(ex2(__fmul_rn(A2, after)), __bfloat162float(dth[(int64_t)s * H]));
+    }
+    __syncwarp();
+    for (int q = 0, s = lane; s < Bs; s += 32, ++q) suf[s] = wv[q];
+    if (lane == 0) p.sumdt[bk * H + h] = tot;
   }
   if (t == 0) {
     umma::bar_init(&bar[0], 1);
     umma::bar_init(&bar[1], 1);
   }
-  if (t < 32) tmem_alloc(&tslot, 64);
+  if (t < 32) tmem_alloc(&tslot, 128);
   umma::fence_before_sync();
   __syncthreads();
   umma::fence_after_sync();
   const uint32_t tm = tslot;
-  bool pend[2] = {false, false};
-  uint32_t ph[2] = {0u, 0u};
-  int qg = 0;
+  const uint32_t lane_base = tm + ((uint32_t)(32 * (w & 3)) << 16);
+  uint32_t ph = 0u;  // phase parity per accumulator barrier
   bool alive = true;
-  for (int h = h0; h < h1 && alive; ++h) {
-    for (int c = t; c < Bs * 8; c += 128) {
-      const int s = c >> 3, ch = c & 7;
-      cp_async16(sX + sw128(s, ch), p.x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
-    }
-    cp_async_commit();
-    if (t < 32) {
-      const __nv_bfloat16* dth = p.dt + tok0 * H + h;
-      const float tot = warp_scan_dt<true>(dth, H, Bs, ssuf);  // inclusive suffix sums
-      __syncwarp();
-      const float A2 = __fmul_rn(p.A[h], kLog2e);
-      for (int s = t; s < Bs; s += 32) {
-        const float after = s + 1 < Bs ? ssuf[s + 1] : 0.f;  // sum of dt over tokens after s
-        sw[s] = __fmul_rn(ex2(__fmul_rn(A2, after)), __bfloat162float(dth[(int64_t)s * H]));
-      }
-      if (t == 0) p.sumdt[bk * H + h] = tot;
-    }
-    cp_async_wait_all();
-    umma::fence_async_smem();
-    __syncthreads();
-    for (int q = 0; q < Bs / 64; ++q, ++qg) {
-      const int bb = qg & 1;
-      if (pend[bb]) {
-        if (!cta_wait(&bar[bb], ph[bb], p.flag)) {
-          alive = false;
-          break;
-        }
-        ph[bb] ^= 1u;
-        pend[bb] = false;
-      }
-      unsigned char* hi = sA + bb * 2 * kTile16;
-      unsigned char* lo = hi + kTile16;
-      if (t < N) {
-#pragma unroll 2
-        for (int c = 0; c < 8; ++c) {
-          uint32_t wh[4], wl[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int s0 = q * 64 + c * 8 + 2 * e;
-            const float v0 = __fmul_rn(sw[s0], __bfloat162float(sB[s0 * N + t]));
-            const float v1 = __fmul_rn(sw[s0 + 1], __bfloat162float(sB[(s0 + 1) * N + t]));
-            const __nv_bfloat162 hv = __floats2bfloat162_rn(v0, v1);
-            wh[e] = *reinterpret_cast<const uint32_t*>(&hv);
-            wl[e] = pack_bf16(__fsub_rn(v0, __low2float(hv)), __fsub_rn(v1, __high2float(hv)));
-          }
-          *reinterpret_cast<uint4*>(hi + sw128(t, c)) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
-          *reinterpret_cast<uint4*>(lo + sw128(t, c)) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
-        }
-      }
-      umma::fence_async_smem();
-      __syncthreads();
-      if (t == 0) {
-        umma::fence_after_sync();
-        const uint32_t ah = umma::smem_u32(hi), al = umma::smem_u32(lo);
-        const uint32_t xb = umma::smem_u32(sX) + (uint32_t)q * 64u * 128u;
-        constexpr uint32_t id = umma::idesc_bf16(128, 64, false, true);
-#pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          const uint64_t bd = umma::sdesc(xb + kk * 2048u, 1024, 1024);
-          umma::mma_bf16(tm, umma::sdesc(ah + kk * 32u, 16, 1024), bd, id, q > 0 || kk > 0);
-          umma::mma_bf16(tm, umma::sdesc(al + kk * 32u, 16, 1024), bd, id, true);
-        }
-        umma::mma_commit(&bar[bb]);
-      }
-      pend[bb] = true;
-    }
-    if (!alive || !drain(bar, pend, ph, p.flag)) {
-      alive = false;
-      break;
-    }
-    umma::fence_after_sync();
-    if (t < N) {  // whole warps: N is a multiple of 32
+  // writes head (h0 + j)'s T from accumulator j & 1: lane n = state row n,
+  // this warp's 32 of the 64 channels
+  auto write_out = [&](int j) {
+    const int n = 32 * (w & 3) + lane, pc = 32 * (w >> 2);
+    if (32 * (w & 3) < N) {  // whole warps
       float v[32];
-      float* dst = p.T + ((bk * H + h) * kSsdP) * N + t;
+      umma::tmem_ld32(lane_base + 64u * (uint32_t)(j & 1) + (uint32_t)pc, v);
+      float* dst = p.T + ((bk * H + h0 + j) * kSsdP + pc) * N + n;
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        umma::tmem_ld32(tm + ((uint32_t)(t & ~31) << 16) + j * 32, v);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) dst[(int64_t)(j * 32 + i) * N] = v[i];
-      }
+      for (int e = 0; e < 32; ++e) dst[(int64_t)e * N] = v[e];
     }
+  };
+  for (int hh = 0; hh < hg && alive; ++hh) {
+    const int h = h0 + hh;
+    cp_async_wait_all();
+    __syncthreads();  // head hh's x rows are in shared memory
+    if (hh + 1 < hg) load_x(h + 1, (hh + 1) & 1);
+    if (hh > 0) {  // head hh-1's MMAs are done reading the weighted x
+      if (!cta_wait(&bar[(hh - 1) & 1], ((hh - 1) >> 1) & 1, p.flag)) {
+        alive = false;
+        break;
+      }
+      umma::fence_after_sync();
+    }
+    const unsigned char* xr = sm + S.xr + (hh & 1) * half;
+    const float* wv = s_w + hh * 256;
+    for (int c = t; c < Bs * 8; c += kStateThreads) {
+      const int s = c >> 3, ch = c & 7;
+      const uint32_t off = sw128(s, ch);
+      const uint4 u = *reinterpret_cast<const uint4*>(xr + off);
+      const __nv_bfloat162* xv = reinterpret_cast<const __nv_bfloat162*>(&u);
+      const float ws = wv[s];
+      uint32_t wh[4], wl[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __bfloat1622float2(xv[e]);
+        const float v0 = __fmul_rn(ws, f.x), v1 = __fmul_rn(ws, f.y);
+        const __nv_bfloat162 hv = __floats2bfloat162_rn(v0, v1);
+        wh[e] = *reinterpret_cast<const uint32_t*>(&hv);
+        wl[e] = pack_bf16(__fsub_rn(v0, __low2float(hv)), __fsub_rn(v1, __high2float(hv)));
+      }
+      *reinterpret_cast<uint4*>(sm + S.xs + off) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+      *reinterpret_cast<uint4*>(sm + S.xs + half + off) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+    }
+    umma::fence_async_smem();
     umma::fence_before_sync();
     __syncthreads();
-    umma::fence_after_sync();
+    if (t == 0) {
+      umma::fence_after_sync();
+      const uint32_t a0 = umma::smem_u32(sm + S.b), x0 = umma::smem_u32(sm + S.xs);
+      constexpr uint32_t id = umma::idesc_bf16(128, 64, true, true);
+      const uint32_t d = tm + 64u * (uint32_t)(hh & 1);
+      for (int kk = 0; kk < Bs / 16; ++kk) {
+        const uint64_t a = umma::sdesc(a0 + kk * 2048u, half, 1024);
+        umma::mma_bf16(d, a, umma::sdesc(x0 + kk * 2048u, 1024, 1024), id, kk > 0);
+        umma::mma_bf16(d, a, umma::sdesc(x0 + half + kk * 2048u, 1024, 1024), id, true);
+      }
+      umma::mma_commit(&bar[hh & 1]);
+    }
+    if (hh > 0) write_out(hh - 1);  // under head hh's MMAs
+  }
+  if (alive && hg > 0) {
+    if (cta_wait(&bar[(hg - 1) & 1], ((hg - 1) >> 1) & 1, p.flag)) {
+      umma::fence_after_sync();
+      write_out(hg - 1);
+    }
   }
   cp_async_wait_all();
   umma::fence_before_sync();
   __syncthreads();
-  if (t < 32) tmem_dealloc(tm, 64);
+  if (t < 32) tmem_dealloc(tm, 128);
 }
+
 
 // One thread per (batch row, head, channel, state index), sequential in k.
 __global__ void __launch_bounds__(256) k_ssd_state_pass(const SsdPassParams p) {
@@ -674,14 +693,15 @@ cudaError_t launch_ssd_block_state(const SsdStateParams& p, cudaStream_t s) {
   const int64_t rows = p.g.Bt * p.g.nb;
   if (rows == 0 || p.g.H == 0) return cudaSuccess;
   const dim3 grid((unsigned)rows, (unsigned)((p.g.H + p.hg - 1) / p.hg));
-  const uint32_t bytes = StateSmem::bytes(p.g.N);
+  if (p.hg < 1 || p.hg > 8) return cudaErrorInvalidValue;
+  const uint32_t bytes = StateSmem((int)p.g.Bs).total;
   cudaError_t e;
   if (p.g.N == 64) {
     if ((e = set_smem(k_ssd_block_state<64>, bytes)) != cudaSuccess) return e;
-    k_ssd_block_state<64><<<grid, 128, bytes, s>>>(p);
+    k_ssd_block_state<64><<<grid, kStateThreads, bytes, s>>>(p);
   } else {
     if ((e = set_smem(k_ssd_block_state<128>, bytes)) != cudaSuccess) return e;
-    k_ssd_block_state<128><<<grid, 128, bytes, s>>>(p);
+    k_ssd_block_state<128><<<grid, kStateThreads, bytes, s>>>(p);
   }
   return cudaGetLastError();
 }
