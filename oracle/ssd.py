@@ -19,18 +19,26 @@ partial-reverse of Sec. 4). Nothing is blocked, chunked or reordered here.
 Layouts: x [Bt, L, H, P]; dt [Bt, L, H] (after softplus); B, C [Bt, L, N];
 A, D [H]; states [Bt, nS, H, P, N] (states[k] follows token (k+1)Bs - 1).
 
+The backward is the diagonal layer's backward with the same tie: a tied
+parameter's gradient is the sum of the gradients of the entries it stands for
+(dt[h] over the head's channels, A[h] over its channels and state indices,
+D[h] over its channels).
+
 Parity status: pinned in ``tests/test_ssd_oracle_pins.py`` by the per-head
 semiseparable-matrix form of the block restriction (y = M x with the scalar
 decay written as exp of a sum, built independently of any recurrence), the
-closed form of the state at a block end, the single-block invariant and
-bit-exact caching.
+closed form of the state at a block end, the single-block invariant,
+bit-exact caching, and (backward) central finite differences of the pinned
+forward for every input, including the tied A, D and dt.
 """
 
 from __future__ import annotations
 
 import numpy as np
 
+from . import GRAD_NAMES
 from . import active_block as _active_block
+from . import backward as _backward
 from . import boundary_states as _boundary_states
 from . import forward as _forward
 
@@ -85,3 +93,36 @@ def active_block(seed, x_n, dt_f, B_f, C_f, dt_r, B_r, C_r, A_f, D_f, A_r, D_r):
     sd = np.asarray(seed, np.float64).reshape(xn.shape[0], H * P, N)
     y = _active_block(sd, xn, dtf, B_f, C_f, dtr, B_r, C_r, Afd, Dfd, Ard, Drd)
     return _heads(y, H, P)
+
+
+def backward(block, x_c, dt_c, B_c, C_c, x_n, dt_f, B_f, C_f, dt_r, B_r, C_r, A_f, D_f, A_r, D_r,
+             states, dy_c, dy_n, dstates=None):
+    """Gradients of <dy_c,y_c> + <dy_n,y_n> + <dstates,states> for the SSD
+    layer (states as returned by ``forward``). Returns a dict keyed like the
+    inputs, in the SSD layouts; dy_c and dstates may be None."""
+    H, P = np.asarray(x_c).shape[2:]
+    N = np.asarray(B_c).shape[2]
+    xc, dtc, Afd, Dfd = _tie(x_c, dt_c, A_f, D_f, N)
+    xn, dtf, _, _ = _tie(x_n, dt_f)
+    _, dtr, Ard, Drd = _tie(x_n, dt_r, A_r, D_r, N)
+    Bt, L = xc.shape[:2]
+    st = np.asarray(states, np.float64).reshape(Bt, -1, H * P, N)
+    dyc = None if dy_c is None else np.asarray(dy_c, np.float64).reshape(Bt, L, H * P)
+    dyn = np.asarray(dy_n, np.float64).reshape(Bt, L, H * P)
+    dst = None if dstates is None else np.asarray(dstates, np.float64).reshape(Bt, -1, H * P, N)
+    g = _backward(block, xc, dtc, B_c, C_c, xn, dtf, B_f, C_f, dtr, B_r, C_r, Afd, Dfd, Ard, Drd,
+                  st, dyc, dyn, dst)
+    out = {}
+    for k in GRAD_NAMES:
+        a = g[k]
+        if k in ("x_c", "x_n"):
+            out[k] = a.reshape(Bt, L, H, P)
+        elif k in ("dt_c", "dt_f", "dt_r"):
+            out[k] = a.reshape(Bt, L, H, P).sum(axis=3)
+        elif k in ("A_f", "A_r"):
+            out[k] = a.reshape(H, P, N).sum(axis=(1, 2))
+        elif k in ("D_f", "D_r"):
+            out[k] = a.reshape(H, P).sum(axis=1)
+        else:
+            out[k] = a
+    return out

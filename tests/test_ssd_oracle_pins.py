@@ -125,3 +125,28 @@ def test_ssd_planted_head_map_fails(monkeypatch):
     monkeypatch.setattr(ssd, "_tie", bad_tie)
     y_c, y_n, _ = ssd.forward(Bs, *[d[k] for k in NAMES])
     assert np.max(np.abs(y_c - m_c)) > 1e-3 and np.max(np.abs(y_n - m_n)) > 1e-3
+
+
+@pytest.mark.parametrize("seed,Bs", [(0, 4), (6, 3)])
+def test_ssd_backward_matches_finite_differences(seed, Bs):
+    """Central differences of the pinned SSD forward, along a random direction
+    per input, against the oracle's gradients of <dy_c,y_c>+<dy_n,y_n>+<dS,S>
+    (tied A, D and dt included)."""
+    _, d = _inputs(seed, Bs=Bs)
+    y_c, y_n, st = ssd.forward(Bs, *[d[k] for k in NAMES])
+    rng = np.random.default_rng(100 + seed)
+    dyc, dyn, dst = rng.standard_normal(y_c.shape), rng.standard_normal(y_n.shape), rng.standard_normal(st.shape)
+    g = ssd.backward(Bs, *[d[k] for k in NAMES], st, dyc, dyn, dst)
+
+    def loss(dd):
+        a, b, c = ssd.forward(Bs, *[dd[k] for k in NAMES])
+        return float((a * dyc).sum() + (b * dyn).sum() + (c * dst).sum())
+
+    for k in NAMES:
+        v = rng.standard_normal(d[k].shape)
+        eps = 1e-6
+        dp, dm = dict(d), dict(d)
+        dp[k], dm[k] = d[k] + eps * v, d[k] - eps * v
+        fd = (loss(dp) - loss(dm)) / (2 * eps)
+        an = float((g[k] * v).sum())
+        assert abs(fd - an) <= 1e-6 * max(1.0, abs(an)), (k, an, fd)
