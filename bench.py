@@ -527,7 +527,7 @@ def run_ssd(args):
             for j, k in enumerate(SSD_KERNELS):
                 per[k].append(prev.elapsed_time(ev_k[i][j]))
                 prev = ev_k[i][j]
-        hg = -(-H // -(-H // 8))
+        hg = -(-H // -(-H // 8))  # the launch's head groups at these sizes (grids above the SM count)
         bts, fls = ssd_costs(Bt, L, Bs, H, N, hg)
         kern = []
         for k in SSD_KERNELS:
@@ -552,6 +552,108 @@ def run_ssd(args):
             "wait_flag": flag, "kernels": kern}), flush=True)
         del t, y_c, y_n, st, ws
         torch.cuda.empty_cache()
+
+
+def run_ssd_cache(args, L=65536, Bs=256, calls=16):
+    """Inference cache path of the SSD form (350M-class Mamba-2 layer, 26 heads
+    of 64, state 128, batch 1): cache build over an L-token prefix (final state
+    only; every block-end state and the clean outputs), then `calls`
+    active-block calls from the cached state, each timed on its own and all
+    replayed as one CUDA graph."""
+    import torch
+    from paper_2607_02805_gb300 import binding
+    from paper_2607_02805_gb300.inputs import SsdWorkload
+    from paper_2607_02805_gb300.layer import to_device
+    peaks, peak_kind = measured_peaks()
+    H, N = 26, 128
+    wl = SsdWorkload(1, L, Bs, H, N, seed=7)
+    t = {k: to_device(wl.dev_bits(k), binding.BDSCAN_F32 if k in ("A_f", "A_r", "D_f", "D_r")
+                      else binding.BDSCAN_BF16, "cuda") for k in wl.t32}
+    d = binding.make_ssd_dims(1, L, Bs, H, N)
+    stream = torch.cuda.current_stream()
+    nb = L // Bs
+    fin = torch.empty((1, 1, H, 64, N), dtype=torch.float32, device="cuda")
+    allst = torch.empty((1, nb, H, 64, N), dtype=torch.float32, device="cuda")
+    y_c = torch.empty((1, L, H, 64), dtype=torch.bfloat16, device="cuda")
+    ws = {e: torch.empty(binding.bdscan_ssd_boundary_states_workspace_size(d, e), dtype=torch.uint8, device="cuda")
+          for e in (0, 1)}
+    read_b = L * (H * 64 * 2 + H * 2 + N * 2)  # x, dt, B
+    st_b = nb * H * 64 * N * 4
+    for name, emit_all, y, st, alg in (("final state only", 0, None, fin, read_b + 2 * st_b),
+                                       ("every block-end state and the clean outputs", 1, y_c, allst,
+                                        read_b + L * N * 2 + 3 * st_b + L * H * 64 * 4)):
+        def one():
+            binding.ssd_boundary_states(d, t, None, y, st, emit_all, ws[emit_all], stream)
+        for _ in range(max(3, args.warmup)):
+            one()
+        reps = max(3, min(args.steps, 20))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            one()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        gbs = alg / (ms * 1e-3) / 1e9
+        print(json.dumps({
+            "metric": "SSD-form cache build (bdscan_ssd_boundary_states) prefix tokens/s", "value": L / (ms * 1e-3),
+            "unit": "tokens/s", "n_gpus": 1, "steps": reps, "ms_per_call": ms, "higher_is_better": True,
+            "dtype": "bf16 operands, fp32 accumulate and state", "data": "synthetic",
+            "config": {"workload": f"SSD cache build over a {L}-token prefix, block {Bs}, 26 heads of 64, state 128, "
+                                   f"batch 1; {name}", "seq_len": L, "block": Bs, "emit_all": emit_all},
+            "hbm": {"achieved": round(gbs, 1), "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
+                    "frac": round(gbs / float(peaks.get("hbm_gbs", 6800.0)), 4), "alg_bytes_per_call": alg,
+                    "peak_kind": peak_kind}}), flush=True)
+    # active blocks: fresh noisy draws per call, seeded from the cached final state
+    da = binding.make_ssd_dims(1, Bs, Bs, H, N)
+    blocks = []
+    for c in range(calls):
+        nw = SsdWorkload(1, Bs, Bs, H, N, seed=7, part=c + 1)
+        blocks.append({k: to_device(nw.dev_bits(k), binding.BDSCAN_F32 if k in ("A_f", "A_r", "D_f", "D_r")
+                                    else binding.BDSCAN_BF16, "cuda") for k in nw.t32})
+    ya = torch.empty((1, Bs, H, 64), dtype=torch.bfloat16, device="cuda")
+    seed = fin[:, 0].contiguous()
+    for _ in range(max(3, args.warmup)):
+        binding.ssd_active_block(da, seed, blocks[0], ya, stream)
+    per = []
+    for c in range(calls):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        binding.ssd_active_block(da, seed, blocks[c], ya, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        per.append(e0.elapsed_time(e1) * 1e3)
+    gs = torch.cuda.Stream()
+    gs.wait_stream(stream)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(gs):
+        binding.ssd_active_block(da, seed, blocks[0], ya, gs)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph, stream=gs):
+            for c in range(calls):
+                binding.ssd_active_block(da, seed, blocks[c], ya, gs)
+    torch.cuda.synchronize()
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 20
+    e0.record(stream)
+    for _ in range(reps):
+        graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    flag = binding.bdscan_ssd_wait_flag(1)
+    print(json.dumps({
+        "metric": "SSD-form active-block call latency (bdscan_ssd_active_block)", "value": statistics.median(per),
+        "unit": "us per call", "n_gpus": 1, "higher_is_better": False,
+        "dtype": "bf16 operands, fp32 accumulate and state", "data": "synthetic",
+        "config": {"workload": f"active block of {Bs} tokens from the cached state of a {L}-token prefix, 26 heads of "
+                               "64, state 128, batch 1", "calls": calls},
+        "per_call_us": [round(v, 2) for v in per],
+        "graph_replay_us_per_call": e0.elapsed_time(e1) * 1e3 / (reps * calls), "wait_flag": flag}), flush=True)
 
 
 def run_prefill(args, L, Bs, calls):
@@ -763,7 +865,7 @@ def main():
     ap.add_argument("--warmup-seconds", type=float, default=1.0,
                     help="keep warming up for at least this long (clock sampling under load)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (smaller profiling case)")
-    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k", "ssd"],
+    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k", "ssd", "ssd_cache"],
                     help="layer: the step line; others: extra lines on one GPU")
     args = ap.parse_args()
     if args.batch:
@@ -780,6 +882,8 @@ def main():
                 run_sweep(args)
             elif args.workload == "ssd":
                 run_ssd(args)
+            elif args.workload == "ssd_cache":
+                run_ssd_cache(args)
             elif args.workload == "prefill65k":
                 run_prefill(args, 65536, 32, 1)
             else:

@@ -58,11 +58,22 @@ int check(const bdscan_ssd_dims* d, bds::SsdGeo* g, const char* fn) {
   return BDSCAN_OK;
 }
 
-// Heads per CTA: groups of at most 8 heads, as even as possible. The Gram
-// products of a tile are computed once per CTA and shared by its heads.
-int heads_per_cta(int H) {
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 1;
+  return n > 0 ? n : 1;
+}
+
+// Heads per CTA: groups of at most 8 heads, as even as possible (the Gram
+// products of a tile are computed once per CTA and shared by its heads).
+// When `units` CTAs per head group would not fill the GPU (an active block,
+// a short prefix), the groups are split further, down to one head per CTA.
+int heads_per_cta(int H, int64_t units) {
   if (H <= 0) return 1;
-  const int groups = (H + 7) / 8;
+  int groups = (H + 7) / 8;
+  const int64_t sms = sm_count();
+  while (groups < H && units * groups < sms) groups = groups * 2 < H ? groups * 2 : H;
   return (H + groups - 1) / groups;
 }
 
@@ -116,7 +127,7 @@ bds::SsdScanParams clean_scan(const bds::SsdGeo& g, const bdscan_clean* c, const
   p.seed_shift = 1;
   p.init_seed = init;
   p.y = (bf*)y;
-  p.hg = heads_per_cta(g.H);
+  p.hg = heads_per_cta(g.H, g.Bt * g.nb * g.m);
   p.flag = flag;
   return p;
 }
@@ -137,7 +148,7 @@ bds::SsdScanParams noisy_scan(const bds::SsdGeo& g, const bdscan_noisy* n, const
   p.Ar = pr->A_r;
   p.Dr = pr->D_r;
   p.y = (bf*)y;
-  p.hg = heads_per_cta(g.H);
+  p.hg = heads_per_cta(g.H, g.Bt * g.nb * g.m);
   p.flag = flag;
   return p;
 }
@@ -154,7 +165,7 @@ cudaError_t build_states(const bds::SsdGeo& g, const bdscan_clean* c, const floa
   sp.A = A_f;
   sp.T = T;
   sp.sumdt = sumdt;
-  sp.hg = heads_per_cta(g.H);
+  sp.hg = heads_per_cta(g.H, g.Bt * g.nb);
   sp.flag = flag;
   cudaError_t e = bds::api_launched(bds::launch_ssd_block_state(sp, s), s);
   if (e != cudaSuccess) return e;
