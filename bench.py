@@ -527,7 +527,7 @@ def run_ssd(args):
             for j, k in enumerate(SSD_KERNELS):
                 per[k].append(prev.elapsed_time(ev_k[i][j]))
                 prev = ev_k[i][j]
-        hg = -(-H // -(-H // 8))  # the launch's head groups at these sizes (grids above the SM count)
+        hg = -(-H // -(-H // 16))  # heads per block-scan CTA at these sizes (grids above the SM count)
         bts, fls = ssd_costs(Bt, L, Bs, H, N, hg)
         kern = []
         for k in SSD_KERNELS:

@@ -80,20 +80,6 @@ __device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
   return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~(uintptr_t)1023);
 }
 
-// Waits for every MMA batch still pending on the two buffer barriers.
-__device__ __forceinline__ bool drain(uint64_t* bar, bool (&pend)[2], uint32_t (&ph)[2], int* flag) {
-  bool ok = true;
-#pragma unroll
-  for (int q = 0; q < 2; ++q) {
-    if (pend[q]) {
-      ok = ok && cta_wait(&bar[q], ph[q], flag);
-      ph[q] ^= 1u;
-      pend[q] = false;
-    }
-  }
-  return ok;
-}
-
 // Shared memory of k_ssd_block_state (offsets from a 1024-aligned base):
 //   b     the block's B rows as the MN-major A operand: two 64-wide halves of
 //         [Bs][64] bf16 (state rows 64..127 are zero when N = 64)
@@ -178,7 +164,6 @@ __global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdS
   umma::fence_after_sync();
   const uint32_t tm = tslot;
   const uint32_t lane_base = tm + ((uint32_t)(32 * (w & 3)) << 16);
-  uint32_t ph = 0u;  // phase parity per accumulator barrier
   bool alive = true;
   // writes head (h0 + j)'s T from accumulator j & 1: lane n = state row n,
   // this warp's 32 of the 64 channels
@@ -316,7 +301,7 @@ __device__ __forceinline__ void mma_gram(uint32_t d, uint32_t a, uint32_t b) {
 //         and the seed's bf16 high and low parts (64 rows x N, K-major).
 //         The next head's seed, as loaded (fp32), waits in m1 (free between
 //         a head's last mixing tile and the next head's second one).
-//   dt    dt of every head of the CTA, per token, both directions (fp32)
+//   dt    dt of every head of the CTA, per token, both directions (bf16)
 //   vec   per token of the block, for the current head: A2 * cumulative dt,
 //         dt and the column factors of both directions
 struct ScanSmem {
@@ -335,14 +320,14 @@ struct ScanSmem {
     raw = m1;
     const uint32_t xs = 2u * xsz + 256u * (uint32_t)N;
     dt = r + (gram > xs ? gram : xs);
-    vec = dt + 2u * 256u * 8u * 4u;
-    prm = vec + 6u * 256u * 4u;
-    total = prm + 4u * 8u * 4u + 1024u;  // + alignment slack of the dynamic base
+    vec = dt + 2u * 256u * 16u * 2u;
+    prm = vec + 2u * 6u * 256u * 4u;
+    total = prm + 4u * 16u * 4u + 1024u;  // + alignment slack of the dynamic base
   }
 };
 
 constexpr int kScanThreads = 256;
-constexpr int kMaxHeadsPerCta = 8;
+constexpr int kMaxHeadsPerCta = 16;
 
 // Issues the cp.async copies of one head's x tiles (MN-major) and its seed
 // (fp32, as stored) for a CTA of kScanThreads threads.
@@ -361,14 +346,14 @@ __device__ __forceinline__ void issue_head_loads(unsigned char* sm, const ScanSm
 
 // Inclusive scan over the block of one head's dt held in shared memory
 // (stride `hs` floats between tokens), by one warp; REV scans from the end.
-template <bool REV>
-__device__ __forceinline__ void warp_scan_smem(const float* dt, int hs, int n, float* out) {
+template <bool REV, typename T>
+__device__ __forceinline__ void warp_scan_smem(const T* dt, int hs, int n, float* out) {
   const int lane = threadIdx.x & 31, per = n / 32;
   float loc[8];
   float s = 0.f;
   for (int q = 0; q < per; ++q) {
     const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
-    s = __fadd_rn(s, dt[pos * hs]);
+    s = __fadd_rn(s, cvt(dt[pos * hs]));
     loc[q] = s;
   }
   float inc = s;
@@ -386,7 +371,7 @@ __device__ __forceinline__ void warp_scan_smem(const float* dt, int hs, int n, f
 }
 
 // One CTA of 8 warps per (batch row, block, 128-token tile i of the block)
-// and group of at most 8 heads. Warp w serves token rows 32 (w % 4) .. +31 of
+// and group of at most 16 heads. Warp w serves token rows 32 (w % 4) .. +31 of
 // the tile (TMEM lanes of its quarter) and column half w / 4 of each mixing
 // tile and of the output.
 // TMEM columns: Gram products at 128 q (forward products of s-tiles 0..i,
@@ -415,14 +400,13 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   const int64_t tok0 = b * g.L + (int64_t)k * Bs;
   const int row = 32 * q4 + lane, tt = i * kSsdT + row;  // token row in the tile / in the block
   const int rg = 4 * i + q4;                              // 32-token row group in the block
-  float* s_dtf = reinterpret_cast<float*>(sm + L.dt);     // [Bs][hg]
-  float* s_dtr = s_dtf + 256 * kMaxHeadsPerCta;
-  float* s_af = reinterpret_cast<float*>(sm + L.vec);     // A2_f * inclusive prefix sums of dt_f
-  float* s_wf = s_af + 256;                               // dt_f
-  float* s_cf = s_wf + 256;                               // forward column factors
-  float* s_ar = s_cf + 256;                               // A2_r * inclusive suffix sums of dt_r
-  float* s_wr = s_ar + 256;                               // dt_r
-  float* s_cr = s_wr + 256;                               // reverse column factors
+  __nv_bfloat16* s_dtf = reinterpret_cast<__nv_bfloat16*>(sm + L.dt);  // [Bs][hg], as stored
+  __nv_bfloat16* s_dtr = s_dtf + 256 * kMaxHeadsPerCta;
+  // per-head decay vectors, two buffers (the next head's are prepared while
+  // the current head's MMAs run): A2_f * inclusive prefix sums of dt_f, dt_f,
+  // forward column factors, A2_r * inclusive suffix sums of dt_r, dt_r,
+  // reverse column factors; 256 floats each
+  float* const vec0 = reinterpret_cast<float*>(sm + L.vec);
   const int nf = i + 1, nr = NOISY ? m - i : 0;           // Gram products per direction
   const int ntile = NOISY ? m : i + 1;                    // s-tiles whose x a head needs
   // this block's seed: slot k - 1 (or k) of p.seed; block 0 of a shifted
@@ -443,19 +427,19 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       stage_rows<N>(sm + L.r + (nf + j - i) * 128u * N * 2u, p.Br + (tok0 + j * kSsdT) * N);
   }
   cp_async_commit();
-  float* s_prm = reinterpret_cast<float*>(sm + L.prm);  // [4][8]: A_f, D_f, A_r, D_r of the CTA's heads
+  float* s_prm = reinterpret_cast<float*>(sm + L.prm);  // [4][16]: A_f, D_f, A_r, D_r of the CTA's heads
   if (t < hg) {
     s_prm[t] = p.Af[h0 + t];
-    s_prm[8 + t] = p.Df[h0 + t];
+    s_prm[16 + t] = p.Df[h0 + t];
     if (NOISY) {
-      s_prm[16 + t] = p.Ar[h0 + t];
-      s_prm[24 + t] = p.Dr[h0 + t];
+      s_prm[32 + t] = p.Ar[h0 + t];
+      s_prm[48 + t] = p.Dr[h0 + t];
     }
   }
   for (int e = t; e < Bs * hg; e += kScanThreads) {  // dt of the CTA's heads, fp32
     const int s = e / hg, hh = e - s * hg;
-    s_dtf[s * hg + hh] = __bfloat162float(p.dtf[(tok0 + s) * H + h0 + hh]);
-    if (NOISY) s_dtr[s * hg + hh] = __bfloat162float(p.dtr[(tok0 + s) * H + h0 + hh]);
+    s_dtf[s * hg + hh] = p.dtf[(tok0 + s) * H + h0 + hh];
+    if (NOISY) s_dtr[s * hg + hh] = p.dtr[(tok0 + s) * H + h0 + hh];
   }
   if (t == 0) {
     umma::bar_init(&bar[0], 1);
@@ -481,67 +465,123 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   // the first head's x and seed (the B tiles are no longer read)
   if (alive && h0 < h1)
     issue_head_loads<N>(sm, L, p.x, tok0, H, h0, ntile, has_seed ? seed_src + (int64_t)h0 * kSsdP * N : nullptr, L.x);
-  uint32_t pend = 0u, ph = 0u;  // per mixing buffer: a commit not yet waited for; its phase parity
-  auto wait_buf = [&](int bb) -> bool {
-    if (!((pend >> bb) & 1u)) return true;
-    if (!cta_wait(&bar[bb], (ph >> bb) & 1u, p.flag)) return false;
-    ph ^= 1u << bb;
-    pend &= ~(1u << bb);
-    return true;
-  };
-  for (int h = h0; h < h1 && alive; ++h) {
-    const int hh = h - h0;
-    const uint32_t xcur = L.x + (hh & 1) * L.xsz;  // this head's x tiles
-    cp_async_wait_all();
-    __syncthreads();
-    // --- the head's decay exponents (fp32, fixed order) and its seed in bf16 high + low parts
+  // decay vectors of head hh into buffer `buf`: warp 0 the forward direction,
+  // warp 1 the reverse one (each scans, then fills its column factors;
+  // forward referenced to the column group's last token, reverse to its first)
+  auto setup = [&](int hh, int buf) {
+    float* v = vec0 + buf * 1536;
     if (w == 0) {
-      warp_scan_smem<false>(s_dtf + hh, hg, Bs, s_af);
+      warp_scan_smem<false>(s_dtf + hh, hg, Bs, v);
       __syncwarp();
       const float A2 = __fmul_rn(s_prm[hh], kLog2e);
       for (int s = lane; s < Bs; s += 32) {
-        s_af[s] = __fmul_rn(A2, s_af[s]);
-        s_wf[s] = s_dtf[s * hg + hh];
+        v[s] = __fmul_rn(A2, v[s]);
+        v[256 + s] = __bfloat162float(s_dtf[s * hg + hh]);
       }
-    } else if (NOISY && w == 1) {
-      warp_scan_smem<true>(s_dtr + hh, hg, Bs, s_ar);
       __syncwarp();
-      const float A2 = __fmul_rn(s_prm[16 + hh], kLog2e);
+      for (int s = lane; s < Bs; s += 32) v[512 + s] = __fmul_rn(ex2(__fsub_rn(v[(s & ~31) + 31], v[s])), v[256 + s]);
+    } else if (NOISY && w == 1) {
+      warp_scan_smem<true>(s_dtr + hh, hg, Bs, v + 768);
+      __syncwarp();
+      const float A2 = __fmul_rn(s_prm[32 + hh], kLog2e);
       for (int s = lane; s < Bs; s += 32) {
-        s_ar[s] = __fmul_rn(A2, s_ar[s]);
-        s_wr[s] = s_dtr[s * hg + hh];
+        v[768 + s] = __fmul_rn(A2, v[768 + s]);
+        v[1024 + s] = __bfloat162float(s_dtr[s * hg + hh]);
       }
+      __syncwarp();
+      for (int s = lane; s < Bs; s += 32)
+        v[1280 + s] = __fmul_rn(ex2(__fsub_rn(v[768 + (s & ~31)], v[768 + s])), v[1024 + s]);
     }
-    if (has_seed) {
-      for (int c = t; c < kSsdP * N / 8; c += kScanThreads) {
-        const int pr = c / (N / 8), ch = c % (N / 8);
-        const float4 u0 = *reinterpret_cast<const float4*>(sm + L.raw + (pr * N + ch * 8) * 4);
-        const float4 u1 = *reinterpret_cast<const float4*>(sm + L.raw + (pr * N + ch * 8 + 4) * 4);
-        const float v[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-        uint32_t wh[4], wl[4];
+  };
+  if (alive && h0 < h1) setup(0, 0);
+  // mixing tile j of head hh into shared buffer mt: this warp's two 32-column
+  // groups (0: no term, 1: factored decay, 2: diagonal block; uniform per warp)
+  auto build = [&](int j, const float* v, unsigned char* mt) {
+    const float af_t = v[tt];
+    const float ar_t = NOISY ? v[768 + tt] : 0.f;
+    const uint32_t colf = 128u * j, colr = 128u * (nf + j - i);
+#pragma unroll 1
+    for (int c = 0; c < 2; ++c) {
+      const int cg = 2 * hf + c, sg = 4 * j + cg, s0 = 32 * sg;  // column group of the tile / block
+      const int fm = j > i ? 0 : (sg < rg ? 1 : (sg == rg ? 2 : 0));
+      const int rm = !NOISY || j < i ? 0 : (sg > rg ? 1 : (sg == rg ? 2 : 0));
+      // pairs of columns in packed fp32 (FMUL2 / FFMA2); decay vectors read 4 at a time
+      float2 o[16];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-          wh[e] = *reinterpret_cast<const uint32_t*>(&hv);
-          wl[e] = pack_bf16(__fsub_rn(v[2 * e], __low2float(hv)), __fsub_rn(v[2 * e + 1], __high2float(hv)));
+      for (int e = 0; e < 16; ++e) o[e] = make_float2(0.f, 0.f);
+      const float4* va = reinterpret_cast<const float4*>(v + s0);           // A2 * cumulative dt (forward)
+      const float4* vw = reinterpret_cast<const float4*>(v + 256 + s0);     // dt (forward)
+      const float4* vc = reinterpret_cast<const float4*>(v + 512 + s0);     // column factors (forward)
+      if (fm != 0) {
+        float gv[32];
+        umma::tmem_ld32(lane_base + colf + 32u * cg, gv);
+        if (fm == 1) {
+          const float2 rf = f2(ex2(__fsub_rn(af_t, v[s0 + 31])));
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float4 c4 = vc[e];
+            o[2 * e] = mul2(mul2(make_float2(gv[4 * e], gv[4 * e + 1]), make_float2(c4.x, c4.y)), rf);
+            o[2 * e + 1] = mul2(mul2(make_float2(gv[4 * e + 2], gv[4 * e + 3]), make_float2(c4.z, c4.w)), rf);
+          }
+        } else {
+          const float2 at = f2(af_t), neg = f2(-1.f);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float4 a4 = va[e], w4 = vw[e];
+            const float2 d0 = mul2(ex2x2(fma2(make_float2(a4.x, a4.y), neg, at)), make_float2(w4.x, w4.y));
+            const float2 d1 = mul2(ex2x2(fma2(make_float2(a4.z, a4.w), neg, at)), make_float2(w4.z, w4.w));
+            const float2 p0 = mul2(make_float2(gv[4 * e], gv[4 * e + 1]), d0);
+            const float2 p1 = mul2(make_float2(gv[4 * e + 2], gv[4 * e + 3]), d1);
+            const int sc = s0 + 4 * e;  // columns sc..sc+3
+            o[2 * e] = make_float2(sc <= tt ? p0.x : 0.f, sc + 1 <= tt ? p0.y : 0.f);
+            o[2 * e + 1] = make_float2(sc + 2 <= tt ? p1.x : 0.f, sc + 3 <= tt ? p1.y : 0.f);
+          }
         }
-        const uint32_t off = (ch >> 3) * 8192u + sw128(pr, ch & 7);
-        *reinterpret_cast<uint4*>(sm + L.seed + off) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
-        *reinterpret_cast<uint4*>(sm + L.seed + 128u * N + off) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+      }
+      if (rm != 0) {
+        float gv[32];
+        umma::tmem_ld32(lane_base + colr + 32u * cg, gv);
+        const float4* ra = reinterpret_cast<const float4*>(v + 768 + s0);   // A2 * cumulative dt (reverse)
+        const float4* rw = reinterpret_cast<const float4*>(v + 1024 + s0);  // dt (reverse)
+        const float4* rc = reinterpret_cast<const float4*>(v + 1280 + s0);  // column factors (reverse)
+        if (rm == 1) {
+          const float2 rf = f2(ex2(__fsub_rn(ar_t, v[768 + s0])));
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float4 c4 = rc[e];
+            o[2 * e] = fma2(mul2(make_float2(gv[4 * e], gv[4 * e + 1]), make_float2(c4.x, c4.y)), rf, o[2 * e]);
+            o[2 * e + 1] = fma2(mul2(make_float2(gv[4 * e + 2], gv[4 * e + 3]), make_float2(c4.z, c4.w)), rf,
+                                o[2 * e + 1]);
+          }
+        } else {
+          const float2 at = f2(ar_t), neg = f2(-1.f);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float4 a4 = ra[e], w4 = rw[e];
+            const float2 d0 = mul2(ex2x2(fma2(make_float2(a4.x, a4.y), neg, at)), make_float2(w4.x, w4.y));
+            const float2 d1 = mul2(ex2x2(fma2(make_float2(a4.z, a4.w), neg, at)), make_float2(w4.z, w4.w));
+            const float2 p0 = mul2(make_float2(gv[4 * e], gv[4 * e + 1]), d0);
+            const float2 p1 = mul2(make_float2(gv[4 * e + 2], gv[4 * e + 3]), d1);
+            const int sc = s0 + 4 * e;
+            o[2 * e] = add2(o[2 * e], make_float2(sc >= tt ? p0.x : 0.f, sc + 1 >= tt ? p0.y : 0.f));
+            o[2 * e + 1] = add2(o[2 * e + 1], make_float2(sc + 2 >= tt ? p1.x : 0.f, sc + 3 >= tt ? p1.y : 0.f));
+          }
+        }
+      }
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch) {
+        const int col = 32 * cg + 8 * ch;  // s inside the tile
+        *reinterpret_cast<uint4*>(mt + (col >> 6) * kTile16 + sw128(row, (col & 63) >> 3)) =
+            make_uint4(pack_bf16(o[ch * 4].x, o[ch * 4].y), pack_bf16(o[ch * 4 + 1].x, o[ch * 4 + 1].y),
+                       pack_bf16(o[ch * 4 + 2].x, o[ch * 4 + 2].y), pack_bf16(o[ch * 4 + 3].x, o[ch * 4 + 3].y));
       }
     }
-    umma::fence_async_smem();
-    __syncthreads();
-    // column factors: forward referenced to the column group's last token,
-    // reverse to its first
-    for (int s = t; s < Bs; s += kScanThreads) {
-      const int g0 = s & ~31;
-      s_cf[s] = __fmul_rn(ex2(__fsub_rn(s_af[g0 + 31], s_af[s])), s_wf[s]);
-      if (NOISY) s_cr[s] = __fmul_rn(ex2(__fsub_rn(s_ar[g0], s_ar[s])), s_wr[s]);
-    }
-    if (t == 0 && has_seed) {  // seed term C^f . seed^T into columns 448..511
-      umma::fence_after_sync();
-      const uint32_t base = umma::smem_u32(sm);
+  };
+  // MMAs of mixing tile j (and, first, the seed term) by thread 0
+  auto issue = [&](int j, uint32_t xcur, bool seed_term) {
+    umma::fence_after_sync();
+    const uint32_t base = umma::smem_u32(sm);
+    if (seed_term) {  // C^f . seed^T into columns 448..511
       constexpr uint32_t id = umma::idesc_bf16(128, 64, false, false);
 #pragma unroll
       for (int kk = 0; kk < N / 16; ++kk) {
@@ -552,87 +592,63 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
         umma::mma_bf16(tm + 448, a, umma::sdesc(base + L.seed + 128u * N + offs, 16, 1024), id, true);
       }
     }
+    const uint32_t ma = base + (j ? L.m1 : L.m0), xb = base + xcur + (uint32_t)j * 16384u;
+    constexpr uint32_t id = umma::idesc_bf16(128, 64, false, true);
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk)
+      umma::mma_bf16(tm + 384, umma::sdesc(ma + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
+                     umma::sdesc(xb + kk * 2048u, 1024, 1024), id, j > 0 || kk > 0);
+  };
+  for (int hh = 0; hh < hg && alive; ++hh) {
+    const int h = h0 + hh;
+    const uint32_t xcur = L.x + (hh & 1) * L.xsz;  // this head's x tiles
+    const float* v = vec0 + (hh & 1) * 1536;       // this head's decay vectors
+    cp_async_wait_all();
+    __syncthreads();  // the head's x and raw seed have landed, its decay vectors are ready
+    if (has_seed) {   // seed (fp32, staged in m1) -> bf16 high + low parts, K-major
+      for (int c = t; c < kSsdP * N / 8; c += kScanThreads) {
+        const int pr = c / (N / 8), ch = c % (N / 8);
+        const float4 u0 = *reinterpret_cast<const float4*>(sm + L.raw + (pr * N + ch * 8) * 4);
+        const float4 u1 = *reinterpret_cast<const float4*>(sm + L.raw + (pr * N + ch * 8 + 4) * 4);
+        const float vv[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+        uint32_t wh[4], wl[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat162 hv = __floats2bfloat162_rn(vv[2 * e], vv[2 * e + 1]);
+          wh[e] = *reinterpret_cast<const uint32_t*>(&hv);
+          wl[e] = pack_bf16(__fsub_rn(vv[2 * e], __low2float(hv)), __fsub_rn(vv[2 * e + 1], __high2float(hv)));
+        }
+        const uint32_t off = (ch >> 3) * 8192u + sw128(pr, ch & 7);
+        *reinterpret_cast<uint4*>(sm + L.seed + off) = make_uint4(wh[0], wh[1], wh[2], wh[3]);
+        *reinterpret_cast<uint4*>(sm + L.seed + 128u * N + off) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+      }
+    }
+    build(0, v, sm + L.m0);
+    umma::fence_async_smem();
+    umma::fence_before_sync();
     __syncthreads();
-    // --- decay-weighted mixing tiles, one per s-tile, each multiplied with x
-    const float af_t = s_af[tt];
-    const float ar_t = NOISY ? s_ar[tt] : 0.f;
-    for (int j = 0; j < ntile; ++j) {
-      const int bb = j & 1;  // tile 0 -> m0, tile 1 -> m1 (m1 also holds the next seed in between)
-      if (!wait_buf(bb)) {
-        alive = false;
-        break;
-      }
-      unsigned char* mt = sm + (bb ? L.m1 : L.m0);
-      const uint32_t colf = 128u * j, colr = 128u * (nf + j - i);
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
-        const int cg = 2 * hf + c, sg = 4 * j + cg, s0 = 32 * sg;  // column group of the tile / block
-        // 0: no term, 1: factored decay, 2: diagonal block (one exp per element); uniform per warp
-        const int fm = j > i ? 0 : (sg < rg ? 1 : (sg == rg ? 2 : 0));
-        const int rm = !NOISY || j < i ? 0 : (sg > rg ? 1 : (sg == rg ? 2 : 0));
-        float v[32];
-#pragma unroll
-        for (int e = 0; e < 32; ++e) v[e] = 0.f;
-        if (fm != 0) {
-          float gv[32];
-          umma::tmem_ld32(lane_base + colf + 32u * cg, gv);
-          if (fm == 1) {
-            const float rf = ex2(__fsub_rn(af_t, s_af[s0 + 31]));
-#pragma unroll
-            for (int e = 0; e < 32; ++e) v[e] = __fmul_rn(__fmul_rn(gv[e], s_cf[s0 + e]), rf);
-          } else {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const float d = __fmul_rn(ex2(__fsub_rn(af_t, s_af[s0 + e])), s_wf[s0 + e]);
-              v[e] = s0 + e <= tt ? __fmul_rn(gv[e], d) : 0.f;
-            }
-          }
-        }
-        if (rm != 0) {
-          float gv[32];
-          umma::tmem_ld32(lane_base + colr + 32u * cg, gv);
-          if (rm == 1) {
-            const float rf = ex2(__fsub_rn(ar_t, s_ar[s0]));
-#pragma unroll
-            for (int e = 0; e < 32; ++e) v[e] = __fadd_rn(v[e], __fmul_rn(__fmul_rn(gv[e], s_cr[s0 + e]), rf));
-          } else {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const float d = __fmul_rn(ex2(__fsub_rn(ar_t, s_ar[s0 + e])), s_wr[s0 + e]);
-              v[e] = __fadd_rn(v[e], s0 + e >= tt ? __fmul_rn(gv[e], d) : 0.f);
-            }
-          }
-        }
-#pragma unroll
-        for (int ch = 0; ch < 4; ++ch) {
-          const int col = 32 * cg + 8 * ch;  // s inside the tile
-          *reinterpret_cast<uint4*>(mt + (col >> 6) * kTile16 + sw128(row, (col & 63) >> 3)) =
-              make_uint4(pack_bf16(v[ch * 8], v[ch * 8 + 1]), pack_bf16(v[ch * 8 + 2], v[ch * 8 + 3]),
-                         pack_bf16(v[ch * 8 + 4], v[ch * 8 + 5]), pack_bf16(v[ch * 8 + 6], v[ch * 8 + 7]));
-        }
-      }
+    if (t == 0) {
+      issue(0, xcur, has_seed);
+      if (ntile == 1) umma::mma_commit(&bar[0]);
+    }
+    if (ntile > 1) {  // the second tile is built while the first one's MMAs run
+      build(1, v, sm + L.m1);
       umma::fence_async_smem();
       umma::fence_before_sync();
       __syncthreads();
       if (t == 0) {
-        umma::fence_after_sync();
-        const uint32_t ma = umma::smem_u32(mt), xb = umma::smem_u32(sm + xcur) + (uint32_t)j * 16384u;
-        constexpr uint32_t id = umma::idesc_bf16(128, 64, false, true);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          umma::mma_bf16(tm + 384, umma::sdesc(ma + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
-                         umma::sdesc(xb + kk * 2048u, 1024, 1024), id, j > 0 || kk > 0);
-        umma::mma_commit(&bar[bb]);
+        issue(1, xcur, false);
+        umma::mma_commit(&bar[0]);
       }
-      pend |= 1u << bb;
     }
-    if (!alive || !wait_buf(0) || !wait_buf(1)) {
+    if (hh + 1 < hg) setup(hh + 1, (hh + 1) & 1);  // under this head's MMAs
+    if (!cta_wait(&bar[0], hh & 1, p.flag)) {
       alive = false;
       break;
     }
     umma::fence_after_sync();
     // the next head's loads run under this head's epilogue
-    if (h + 1 < h1)
+    if (hh + 1 < hg)
       issue_head_loads<N>(sm, L, p.x, tok0, H, h + 1, ntile, has_seed ? seed_src + (int64_t)(h + 1) * kSsdP * N : nullptr,
                           L.x + ((hh + 1) & 1) * L.xsz);
     // --- epilogue: y = mixing term + decayed seed term + D x, bf16 out;
@@ -641,8 +657,8 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       float ya[32], yo[32];
       umma::tmem_ld32(lane_base + 384u + 32u * hf, ya);
       if (has_seed) umma::tmem_ld32(lane_base + 448u + 32u * hf, yo);
-      const float dec = has_seed ? ex2(af_t) : 0.f;
-      const float Dd = NOISY ? __fadd_rn(s_prm[8 + hh], s_prm[24 + hh]) : s_prm[8 + hh];
+      const float dec = has_seed ? ex2(v[tt]) : 0.f;
+      const float Dd = NOISY ? __fadd_rn(s_prm[16 + hh], s_prm[48 + hh]) : s_prm[16 + hh];
       const int64_t off = ((tok0 + tt) * H + h) * kSsdP + 32 * hf;
       const unsigned char* xr = sm + xcur + (uint32_t)i * 16384u;
       uint4* yg = reinterpret_cast<uint4*>(p.y + off);

@@ -65,16 +65,28 @@ int sm_count() {
   return n > 0 ? n : 1;
 }
 
-// Heads per CTA: groups of at most 8 heads, as even as possible (the Gram
-// products of a tile are computed once per CTA and shared by its heads).
-// When `units` CTAs per head group would not fill the GPU (an active block,
-// a short prefix), the groups are split further, down to one head per CTA.
-int heads_per_cta(int H, int64_t units) {
-  if (H <= 0) return 1;
-  int groups = (H + 7) / 8;
+// Heads per CTA. A CTA pays a fixed set-up (the block's B/C rows; in the
+// block scan the Gram products, shared by all its heads) and then about the
+// same time per head. Over the group counts g from ceil(H / maxg) to H, the
+// model (waves of g * units CTAs over the SMs) x (1 set-up + ceil(H / g)
+// heads) is minimised; ties keep the smaller g. With few `units` (an active
+// block) this reaches one head per CTA; with many it keeps large groups.
+int heads_per_cta(int H, int64_t units, int maxg) {
+  if (H <= 0 || units <= 0) return 1;
   const int64_t sms = sm_count();
-  while (groups < H && units * groups < sms) groups = groups * 2 < H ? groups * 2 : H;
-  return (H + groups - 1) / groups;
+  int best = (H + maxg - 1) / maxg;
+  int64_t best_cost = -1;
+  for (int g = (H + maxg - 1) / maxg; g <= H; ++g) {
+    const int hg = (H + g - 1) / g;
+    if (g > (H + maxg - 1) / maxg && (H + g - 2) / (g - 1) == hg) continue;  // same heads per CTA, more CTAs
+    const int64_t waves = (units * g + sms - 1) / sms;
+    const int64_t cost = waves * (1 + hg);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = g;
+    }
+  }
+  return (H + best - 1) / best;
 }
 
 size_t sumdt_bytes(const bds::SsdGeo& g) { return al256((size_t)g.Bt * g.nb * g.H * 4); }
@@ -127,7 +139,7 @@ bds::SsdScanParams clean_scan(const bds::SsdGeo& g, const bdscan_clean* c, const
   p.seed_shift = 1;
   p.init_seed = init;
   p.y = (bf*)y;
-  p.hg = heads_per_cta(g.H, g.Bt * g.nb * g.m);
+  p.hg = heads_per_cta(g.H, g.Bt * g.nb * g.m, 16);
   p.flag = flag;
   return p;
 }
@@ -148,7 +160,7 @@ bds::SsdScanParams noisy_scan(const bds::SsdGeo& g, const bdscan_noisy* n, const
   p.Ar = pr->A_r;
   p.Dr = pr->D_r;
   p.y = (bf*)y;
-  p.hg = heads_per_cta(g.H, g.Bt * g.nb * g.m);
+  p.hg = heads_per_cta(g.H, g.Bt * g.nb * g.m, 16);
   p.flag = flag;
   return p;
 }
@@ -165,7 +177,7 @@ cudaError_t build_states(const bds::SsdGeo& g, const bdscan_clean* c, const floa
   sp.A = A_f;
   sp.T = T;
   sp.sumdt = sumdt;
-  sp.hg = heads_per_cta(g.H, g.Bt * g.nb);
+  sp.hg = heads_per_cta(g.H, g.Bt * g.nb, 8);
   sp.flag = flag;
   cudaError_t e = bds::api_launched(bds::launch_ssd_block_state(sp, s), s);
   if (e != cudaSuccess) return e;
