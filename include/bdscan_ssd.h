@@ -111,6 +111,13 @@ int bdscan_ssd_active_block(const bdscan_ssd_dims* dims, const float* seed, cons
  * Returns -1 if the flag cannot be read. */
 int bdscan_ssd_wait_flag(int reset);
 
+/* Failure-detection check of the bounded waits (no GPU fault, no hang): runs
+ * one CTA that waits, through the kernels' own wait path, on an mbarrier that
+ * nothing completes, giving up after `polls` polls (1..2^20). Synchronises
+ * the current device. Returns the wait flag the probe left (1 = the wait gave
+ * up and was reported) after clearing it, or a negative BDSCAN_ERR_* code. */
+int bdscan_ssd_wait_selftest(uint32_t polls);
+
 #ifdef __cplusplus
 }
 #endif

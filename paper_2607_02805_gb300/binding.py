@@ -104,6 +104,7 @@ SIGNATURES = [
     ("bdscan_ssd_active_block", ctypes.c_int,
      [_P(bdscan_ssd_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
     ("bdscan_ssd_wait_flag", ctypes.c_int, [ctypes.c_int]),
+    ("bdscan_ssd_wait_selftest", ctypes.c_int, [ctypes.c_uint32]),
 ]
 
 BDSCAN_NOALLOC_SCRATCH_BYTES = 32 << 20
@@ -245,6 +246,10 @@ def bdscan_ssd_active_block(dims, seed, noisy, params, y_n, stream):
 
 def bdscan_ssd_wait_flag(reset) -> int:
     return load().bdscan_ssd_wait_flag(int(reset))
+
+
+def bdscan_ssd_wait_selftest(polls) -> int:
+    return load().bdscan_ssd_wait_selftest(int(polls))
 
 # ---------------------------------------------------------------------------
 # torch-tensor helpers (marshalling only)

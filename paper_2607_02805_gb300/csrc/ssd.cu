@@ -688,6 +688,29 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
 
 }  // namespace
 
+namespace {
+
+// Failure-detection check of the bounded waits: thread 0 initialises an
+// mbarrier that nothing ever completes; every thread waits on it through the
+// same path as the tensor-core kernels, with `polls` polls, so the wait gives
+// up, sets the flag and the kernel returns normally.
+__global__ void __launch_bounds__(128) k_ssd_wait_probe(int* flag, uint32_t polls) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) umma::bar_init(&bar, 1);
+  __syncthreads();
+  const bool ok = umma::bar_wait(&bar, 0, polls);
+  if (__syncthreads_or(ok ? 0 : 1) && threadIdx.x == 0) atomicExch(flag, 1);
+}
+
+}  // namespace
+
+cudaError_t launch_ssd_wait_probe(uint32_t polls, cudaStream_t s) {
+  int* flag = ssd_wait_flag_ptr();
+  if (flag == nullptr) return cudaErrorInvalidSymbol;
+  k_ssd_wait_probe<<<1, 128, 0, s>>>(flag, polls);
+  return cudaGetLastError();
+}
+
 int* ssd_wait_flag_ptr() {
   void* p = nullptr;
   if (cudaGetSymbolAddress(&p, g_ssd_wait_flag) != cudaSuccess) return nullptr;

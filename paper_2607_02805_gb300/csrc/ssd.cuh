@@ -62,5 +62,6 @@ cudaError_t launch_ssd_block_state(const SsdStateParams& p, cudaStream_t s);
 cudaError_t launch_ssd_state_pass(const SsdPassParams& p, cudaStream_t s);
 cudaError_t launch_ssd_block_scan(bool noisy, const SsdScanParams& p, cudaStream_t s);
 int* ssd_wait_flag_ptr();  // device address of the wait flag (current device), or null
+cudaError_t launch_ssd_wait_probe(uint32_t polls, cudaStream_t s);
 
 }  // namespace bds

@@ -308,4 +308,18 @@ int bdscan_ssd_wait_flag(int reset) {
   return v;
 }
 
+int bdscan_ssd_wait_selftest(uint32_t polls) {
+  const char* fn = "bdscan_ssd_wait_selftest";
+  bds::api_begin();
+  if (polls == 0 || polls > (1u << 20)) return failf(BDSCAN_ERR_ARG, "%s: polls must be in 1..2^20%s", fn);
+  if (bdscan_ssd_wait_flag(1) < 0) return cuda_fail(cudaGetLastError(), fn);
+  cudaError_t e = bds::api_launched(bds::launch_ssd_wait_probe(polls, nullptr), nullptr);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  const int v = bdscan_ssd_wait_flag(1);
+  if (v < 0) return cuda_fail(cudaGetLastError(), fn);
+  bds::api_ok();
+  return v;
+}
+
 }  // extern "C"

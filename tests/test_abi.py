@@ -214,3 +214,8 @@ def test_ssd_rejects_bad_pointers():
     # an empty batch needs no pointers
     c0, n0, p0 = _structs(None)
     assert binding.bdscan_ssd_forward(_ssd_dims(batch=0), c0, n0, p0, None, None, None, None, 0, None) == 0
+
+
+def test_ssd_wait_selftest_checks_polls():
+    assert binding.bdscan_ssd_wait_selftest(0) == binding.BDSCAN_ERR_ARG
+    assert "polls" in binding.bdscan_last_error()

@@ -147,3 +147,13 @@ def test_ssd_deterministic():
     t, y_c, y_n, st = _forward(wl)
     _, y_c2, y_n2, st2 = _forward(wl, t)
     assert torch.equal(y_c, y_c2) and torch.equal(y_n, y_n2) and torch.equal(st, st2)
+
+
+def test_ssd_bounded_wait_reports_instead_of_hanging():
+    """A wait that nothing completes gives up after its poll limit, sets the
+    device flag and returns; the context stays usable for the next call."""
+    assert binding.bdscan_ssd_wait_selftest(256) == 1
+    assert binding.bdscan_ssd_wait_flag(0) == 0
+    wl = SsdWorkload(1, 256, 128, 2, 64, seed=4)
+    _, y_c, y_n, st = _forward(wl)
+    _check(y_c, y_n, st, _oracle(wl))
