@@ -645,7 +645,31 @@ def run_ssd_cache(args, L=65536, Bs=256, calls=16):
         graph.replay()
     e1.record(stream)
     torch.cuda.synchronize()
+    graph_us = e0.elapsed_time(e1) * 1e3 / (reps * calls)
+    # the same denoising step without a cache: a full-sequence bidirectional
+    # layer over the whole context (both directions rescan all L tokens)
+    yf = torch.empty((1, L, H, 64), dtype=torch.bfloat16, device="cuda")
+    wsf = torch.empty(binding.bdscan_ssd_full_bidir_workspace_size(d), dtype=torch.uint8, device="cuda")
+    for _ in range(max(3, args.warmup)):
+        binding.ssd_full_bidir_forward(d, t, yf, wsf, stream)
+    reps_f = max(3, min(args.steps, 10))
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    f0.record(stream)
+    for _ in range(reps_f):
+        binding.ssd_full_bidir_forward(d, t, yf, wsf, stream)
+    f1.record(stream)
+    torch.cuda.synchronize()
+    full_ms = f0.elapsed_time(f1) / reps_f
     flag = binding.bdscan_ssd_wait_flag(1)
+    print(json.dumps({
+        "metric": "SSD-form layer step per denoising step: full-sequence bidirectional (no cache) over cached "
+                  "active block", "value": full_ms * 1e3 / graph_us, "unit": "x", "n_gpus": 1,
+        "higher_is_better": True, "dtype": "bf16 operands, fp32 accumulate and state", "data": "synthetic",
+        "config": {"workload": f"one 350M-class Mamba-2 layer at a {L}-token context, block {Bs}, batch 1: "
+                               "bdscan_ssd_full_bidir_forward over the whole sequence vs bdscan_ssd_active_block "
+                               "from the cached state (in a CUDA graph)", "context": L, "block": Bs},
+        "full_bidir_ms": round(full_ms, 4), "active_block_us": round(graph_us, 3), "wait_flag": flag}), flush=True)
     print(json.dumps({
         "metric": "SSD-form active-block call latency (bdscan_ssd_active_block)", "value": statistics.median(per),
         "unit": "us per call", "n_gpus": 1, "higher_is_better": False,
@@ -653,7 +677,7 @@ def run_ssd_cache(args, L=65536, Bs=256, calls=16):
         "config": {"workload": f"active block of {Bs} tokens from the cached state of a {L}-token prefix, 26 heads of "
                                "64, state 128, batch 1", "calls": calls},
         "per_call_us": [round(v, 2) for v in per],
-        "graph_replay_us_per_call": e0.elapsed_time(e1) * 1e3 / (reps * calls), "wait_flag": flag}), flush=True)
+        "graph_replay_us_per_call": graph_us, "wait_flag": flag}), flush=True)
 
 
 def run_prefill(args, L, Bs, calls):

@@ -106,6 +106,22 @@ int bdscan_ssd_boundary_states(const bdscan_ssd_dims* dims, const bdscan_clean* 
 int bdscan_ssd_active_block(const bdscan_ssd_dims* dims, const float* seed, const bdscan_noisy* noisy,
                             const bdscan_params* params, void* y_n, void* stream);
 
+/* Workspace bytes of bdscan_ssd_full_bidir_forward: dt sums, one direction's
+ * block states and one direction's fp32 output. 0 for invalid dims. */
+size_t bdscan_ssd_full_bidir_workspace_size(const bdscan_ssd_dims* dims);
+
+/* Full-sequence bidirectional layer (no block restriction): the fully
+ * bidirectional Mamba of DiffuMamba that the block partial-reverse design
+ * replaces (Sec. 4). y = F_fwd(x) + rev(F_rev(rev(x))) over the whole sequence
+ * of the noisy tensors: the forward direction uses dt_f, B_f, C_f, A_f, D_f
+ * from the start of the sequence, the reverse direction dt_r, B_r, C_r, A_r,
+ * D_r from its end, both from zero states; y [Bt][L][H][P] bf16 (written).
+ * A comparator for the cache: without one, a denoising step of such a layer
+ * rescans the whole context. Same kernels as the clean scan (the reverse
+ * direction reads tokens right to left); dims.block sets the internal blocking. */
+int bdscan_ssd_full_bidir_forward(const bdscan_ssd_dims* dims, const bdscan_noisy* noisy, const bdscan_params* params,
+                                  void* y, void* workspace, size_t workspace_bytes, void* stream);
+
 /* The device flag set by a kernel whose bounded wait on its tensor-core work
  * gave up (0 = never). Synchronises the current device; reset != 0 clears it.
  * Returns -1 if the flag cannot be read. */

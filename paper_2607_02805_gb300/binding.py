@@ -105,6 +105,9 @@ SIGNATURES = [
      [_P(bdscan_ssd_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
     ("bdscan_ssd_wait_flag", ctypes.c_int, [ctypes.c_int]),
     ("bdscan_ssd_wait_selftest", ctypes.c_int, [ctypes.c_uint32]),
+    ("bdscan_ssd_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
+    ("bdscan_ssd_full_bidir_forward", ctypes.c_int,
+     [_P(bdscan_ssd_dims), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
 ]
 
 BDSCAN_NOALLOC_SCRATCH_BYTES = 32 << 20
@@ -251,6 +254,15 @@ def bdscan_ssd_wait_flag(reset) -> int:
 def bdscan_ssd_wait_selftest(polls) -> int:
     return load().bdscan_ssd_wait_selftest(int(polls))
 
+
+def bdscan_ssd_full_bidir_workspace_size(dims) -> int:
+    return load().bdscan_ssd_full_bidir_workspace_size(_ref(dims))
+
+
+def bdscan_ssd_full_bidir_forward(dims, noisy, params, y, workspace, workspace_bytes, stream):
+    return load().bdscan_ssd_full_bidir_forward(_ref(dims), _ref(noisy), _ref(params), y, workspace,
+                                                workspace_bytes, stream)
+
 # ---------------------------------------------------------------------------
 # torch-tensor helpers (marshalling only)
 # ---------------------------------------------------------------------------
@@ -359,3 +371,10 @@ def ssd_boundary_states(dims, t, init_state, y_c, states, emit_all, workspace, s
 def ssd_active_block(dims, seed, t, y_n, stream=None):
     _call("bdscan_ssd_active_block", ctypes.byref(dims), _ptr(seed), ctypes.byref(make_noisy(t)),
           ctypes.byref(make_params(t)), _ptr(y_n), _stream(stream))
+
+
+def ssd_full_bidir_forward(dims, t, y, workspace, stream=None):
+    """Full-sequence bidirectional SSD layer (no block restriction) of the noisy
+    tensors in t; y [Bt][L][H][64]."""
+    _call("bdscan_ssd_full_bidir_forward", ctypes.byref(dims), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), _ptr(y), _ptr(workspace), _nbytes(workspace), _stream(stream))

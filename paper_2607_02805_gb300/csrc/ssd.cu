@@ -76,6 +76,15 @@ __device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t s
 }
 
 
+// Token index of position s of block k in batch row b: left to right, or
+// right to left (position t of the reversed stream is token L-1-t).
+struct RowMap {
+  int64_t base, step;
+  __device__ __forceinline__ RowMap(int64_t b, int64_t L, int64_t k0, bool rev)
+      : base(rev ? b * L + L - 1 - k0 : b * L + k0), step(rev ? -1 : 1) {}
+  __device__ __forceinline__ int64_t operator()(int64_t s) const { return base + step * s; }
+};
+
 __device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
   return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~(uintptr_t)1023);
 }
@@ -119,12 +128,12 @@ __global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdS
   const int64_t bk = blockIdx.x, b = bk / g.nb;
   const int k = (int)(bk % g.nb);
   const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
-  const int64_t tok0 = b * g.L + (int64_t)k * Bs;
+  const RowMap tok(b, g.L, (int64_t)k * Bs, p.rev != 0);
   float* s_w = reinterpret_cast<float*>(sm + S.w);  // [hg][256]
   // B rows: chunk c of 8 state indices of token s goes to half c / 8
   for (int c = t; c < Bs * N / 8; c += kStateThreads) {
     const int s = c / (N / 8), ch = c % (N / 8);
-    cp_async16(sm + S.b + (ch >> 3) * half + sw128(s, ch & 7), p.B + (tok0 + s) * N + ch * 8, 16);
+    cp_async16(sm + S.b + (ch >> 3) * half + sw128(s, ch & 7), p.B + tok(s) * N + ch * 8, 16);
   }
   if (N == 64)
     for (int c = t; c < Bs * 8; c += kStateThreads)
@@ -132,7 +141,7 @@ __global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdS
   auto load_x = [&](int h, int buf) {
     for (int c = t; c < Bs * 8; c += kStateThreads) {
       const int s = c >> 3, ch = c & 7;
-      cp_async16(sm + S.xr + buf * half + sw128(s, ch), p.x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+      cp_async16(sm + S.xr + buf * half + sw128(s, ch), p.x + (tok(s) * H + h) * kSsdP + ch * 8, 16);
     }
     cp_async_commit();
   };
@@ -140,15 +149,16 @@ __global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdS
   // weights of every head of the CTA: warp hh scans head hh (suffix sums)
   if (w < hg) {
     const int h = h0 + w;
-    const __nv_bfloat16* dth = p.dt + tok0 * H + h;
+    const __nv_bfloat16* dth = p.dt + tok.base * H + h;  // position s at dth[s * dstep]
+    const int64_t dstep = tok.step * H;
     float* suf = s_w + w * 256;
-    const float tot = warp_scan_dt<true>(dth, H, Bs, suf);  // inclusive suffix sums
+    const float tot = warp_scan_dt<true>(dth, dstep, Bs, suf);  // inclusive suffix sums
     __syncwarp();
     const float A2 = __fmul_rn(p.A[h], kLog2e);
     float wv[8];
     for (int q = 0, s = lane; s < Bs; s += 32, ++q) {
       const float after = s + 1 < Bs ? suf[s + 1] : 0.f;  // sum of dt over tokens after s
-      wv[q] = __fmul_rn(ex2(__fmul_rn(A2, after)), __bfloat162float(dth[(int64_t)s * H]));
+      wv[q] = __fmul_rn(ex2(__fmul_rn(A2, after)), __bfloat162float(dth[(int64_t)s * dstep]));
     }
     __syncwarp();
     for (int q = 0, s = lane; s < Bs; s += 32, ++q) suf[s] = wv[q];
@@ -274,10 +284,10 @@ __global__ void __launch_bounds__(256) k_ssd_state_pass(const SsdPassParams p) {
 // Copies one 128-token tile of a [tokens][N] bf16 tensor into K-major
 // swizzled shared memory (N / 64 atom columns).
 template <int N>
-__device__ __forceinline__ void stage_rows(unsigned char* dst, const __nv_bfloat16* src) {
+__device__ __forceinline__ void stage_rows(unsigned char* dst, const __nv_bfloat16* src, const RowMap& tok, int row0) {
   for (int c = threadIdx.x; c < 128 * N / 8; c += blockDim.x) {
     const int r = c / (N / 8), ch = c % (N / 8);
-    cp_async16(dst + (ch >> 3) * kTile16 + sw128(r, ch & 7), src + (int64_t)r * N + ch * 8, 16);
+    cp_async16(dst + (ch >> 3) * kTile16 + sw128(r, ch & 7), src + tok(row0 + r) * N + ch * 8, 16);
   }
 }
 
@@ -333,11 +343,11 @@ constexpr int kMaxHeadsPerCta = 16;
 // (fp32, as stored) for a CTA of kScanThreads threads.
 template <int N>
 __device__ __forceinline__ void issue_head_loads(unsigned char* sm, const ScanSmem& L, const __nv_bfloat16* x,
-                                                 int64_t tok0, int H, int h, int ntile, const float* seed_h,
+                                                 const RowMap& tok, int H, int h, int ntile, const float* seed_h,
                                                  uint32_t xbuf) {
   for (int c = threadIdx.x; c < ntile * kSsdT * 8; c += kScanThreads) {
     const int s = c >> 3, ch = c & 7;
-    cp_async16(sm + xbuf + (s >> 7) * 16384u + sw128(s & 127, ch), x + ((tok0 + s) * H + h) * kSsdP + ch * 8, 16);
+    cp_async16(sm + xbuf + (s >> 7) * 16384u + sw128(s & 127, ch), x + (tok(s) * H + h) * kSsdP + ch * 8, 16);
   }
   if (seed_h != nullptr)
     for (int c = threadIdx.x; c < kSsdP * N / 4; c += kScanThreads) cp_async16(sm + L.raw + c * 16, seed_h + c * 4, 16);
@@ -397,7 +407,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   const int64_t bk = idx / m, b = bk / g.nb;
   const int k = (int)(bk % g.nb);
   const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
-  const int64_t tok0 = b * g.L + (int64_t)k * Bs;
+  const RowMap tok(b, g.L, (int64_t)k * Bs, p.rev != 0);
   const int row = 32 * q4 + lane, tt = i * kSsdT + row;  // token row in the tile / in the block
   const int rg = 4 * i + q4;                              // 32-token row group in the block
   __nv_bfloat16* s_dtf = reinterpret_cast<__nv_bfloat16*>(sm + L.dt);  // [Bs][hg], as stored
@@ -419,12 +429,12 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   }
   const bool has_seed = seed_src != nullptr;
   // --- Gram products C B^T of this tile against the block's s-tiles
-  stage_rows<N>(sm + L.cf, p.Cf + (tok0 + i * kSsdT) * N);
-  for (int j = 0; j < nf; ++j) stage_rows<N>(sm + L.r + j * 128u * N * 2u, p.Bf + (tok0 + j * kSsdT) * N);
+  stage_rows<N>(sm + L.cf, p.Cf, tok, i * kSsdT);
+  for (int j = 0; j < nf; ++j) stage_rows<N>(sm + L.r + j * 128u * N * 2u, p.Bf, tok, j * kSsdT);
   if (NOISY) {
-    stage_rows<N>(sm + L.m1, p.Cr + (tok0 + i * kSsdT) * N);
+    stage_rows<N>(sm + L.m1, p.Cr, tok, i * kSsdT);
     for (int j = i; j < m; ++j)
-      stage_rows<N>(sm + L.r + (nf + j - i) * 128u * N * 2u, p.Br + (tok0 + j * kSsdT) * N);
+      stage_rows<N>(sm + L.r + (nf + j - i) * 128u * N * 2u, p.Br, tok, j * kSsdT);
   }
   cp_async_commit();
   float* s_prm = reinterpret_cast<float*>(sm + L.prm);  // [4][16]: A_f, D_f, A_r, D_r of the CTA's heads
@@ -438,8 +448,8 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   }
   for (int e = t; e < Bs * hg; e += kScanThreads) {  // dt of the CTA's heads, fp32
     const int s = e / hg, hh = e - s * hg;
-    s_dtf[s * hg + hh] = p.dtf[(tok0 + s) * H + h0 + hh];
-    if (NOISY) s_dtr[s * hg + hh] = p.dtr[(tok0 + s) * H + h0 + hh];
+    s_dtf[s * hg + hh] = p.dtf[tok(s) * H + h0 + hh];
+    if (NOISY) s_dtr[s * hg + hh] = p.dtr[tok(s) * H + h0 + hh];
   }
   if (t == 0) {
     umma::bar_init(&bar[0], 1);
@@ -464,7 +474,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   umma::fence_after_sync();
   // the first head's x and seed (the B tiles are no longer read)
   if (alive && h0 < h1)
-    issue_head_loads<N>(sm, L, p.x, tok0, H, h0, ntile, has_seed ? seed_src + (int64_t)h0 * kSsdP * N : nullptr, L.x);
+    issue_head_loads<N>(sm, L, p.x, tok, H, h0, ntile, has_seed ? seed_src + (int64_t)h0 * kSsdP * N : nullptr, L.x);
   // decay vectors of head hh into buffer `buf`: warp 0 the forward direction,
   // warp 1 the reverse one (each scans, then fills its column factors;
   // forward referenced to the column group's last token, reverse to its first)
@@ -649,7 +659,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     umma::fence_after_sync();
     // the next head's loads run under this head's epilogue
     if (hh + 1 < hg)
-      issue_head_loads<N>(sm, L, p.x, tok0, H, h + 1, ntile, has_seed ? seed_src + (int64_t)(h + 1) * kSsdP * N : nullptr,
+      issue_head_loads<N>(sm, L, p.x, tok, H, h + 1, ntile, has_seed ? seed_src + (int64_t)(h + 1) * kSsdP * N : nullptr,
                           L.x + ((hh + 1) & 1) * L.xsz);
     // --- epilogue: y = mixing term + decayed seed term + D x, bf16 out;
     // this warp's 32 channels of its token row
@@ -659,7 +669,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       if (has_seed) umma::tmem_ld32(lane_base + 448u + 32u * hf, yo);
       const float dec = has_seed ? ex2(v[tt]) : 0.f;
       const float Dd = NOISY ? __fadd_rn(s_prm[16 + hh], s_prm[48 + hh]) : s_prm[16 + hh];
-      const int64_t off = ((tok0 + tt) * H + h) * kSsdP + 32 * hf;
+      const int64_t off = (tok(tt) * H + h) * kSsdP + 32 * hf;
       const unsigned char* xr = sm + xcur + (uint32_t)i * 16384u;
       uint4* yg = reinterpret_cast<uint4*>(p.y + off);
 #pragma unroll
@@ -672,6 +682,19 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
           float acc = ya[ch * 8 + e];
           if (has_seed) acc = __fmaf_rn(dec, yo[ch * 8 + e], acc);
           o[e] = __fmaf_rn(Dd, __bfloat162float(xe[e]), acc);
+        }
+        if (p.y32 != nullptr) {  // fp32 output (one direction of a two-pass layer)
+          float4* d4 = reinterpret_cast<float4*>(p.y32 + off + ch * 8);
+          d4[0] = make_float4(o[0], o[1], o[2], o[3]);
+          d4[1] = make_float4(o[4], o[5], o[6], o[7]);
+          continue;
+        }
+        if (p.y32_add != nullptr) {  // the other direction's fp32 output, added before rounding
+          const float4* a4 = reinterpret_cast<const float4*>(p.y32_add + off + ch * 8);
+          const float4 u0 = a4[0], u1 = a4[1];
+          o[0] = __fadd_rn(u0.x, o[0]); o[1] = __fadd_rn(u0.y, o[1]); o[2] = __fadd_rn(u0.z, o[2]);
+          o[3] = __fadd_rn(u0.w, o[3]); o[4] = __fadd_rn(u1.x, o[4]); o[5] = __fadd_rn(u1.y, o[5]);
+          o[6] = __fadd_rn(u1.z, o[6]); o[7] = __fadd_rn(u1.w, o[7]);
         }
         yg[ch] = make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]), pack_bf16(o[6], o[7]));
       }

@@ -29,6 +29,7 @@ struct SsdStateParams {
   float* sumdt;  // [Bt][nb][H]
   int hg;        // heads per CTA
   int* flag;     // wait flag
+  int rev;       // 1: the stream is read right to left (token L-1-t of each batch row at position t)
 };
 
 // Sequential pass over blocks: S_k = exp(A sumdt_k) S_{k-1} + T_k.
@@ -56,6 +57,9 @@ struct SsdScanParams {
   __nv_bfloat16* y;   // [Bt][L][H][P]
   int hg;
   int* flag;
+  int rev;            // 1: the stream is read right to left (as in SsdStateParams)
+  float* y32;         // non-null: write the output in fp32 here instead of y
+  const float* y32_add;  // non-null: add this fp32 array to the output before rounding to y
 };
 
 cudaError_t launch_ssd_block_state(const SsdStateParams& p, cudaStream_t s);

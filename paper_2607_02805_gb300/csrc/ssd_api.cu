@@ -168,7 +168,7 @@ bds::SsdScanParams noisy_scan(const bds::SsdGeo& g, const bdscan_noisy* n, const
 // Block-local states into T, then the exact states (in place when T is the
 // emitted states array).
 cudaError_t build_states(const bds::SsdGeo& g, const bdscan_clean* c, const float* A_f, const float* init,
-                         float* T, float* sumdt, float* final_state, int* flag, cudaStream_t s) {
+                         float* T, float* sumdt, float* final_state, int* flag, cudaStream_t s, int rev = 0) {
   bds::SsdStateParams sp{};
   sp.g = g;
   sp.x = (const bf*)c->x;
@@ -179,6 +179,7 @@ cudaError_t build_states(const bds::SsdGeo& g, const bdscan_clean* c, const floa
   sp.sumdt = sumdt;
   sp.hg = heads_per_cta(g.H, g.Bt * g.nb, 8);
   sp.flag = flag;
+  sp.rev = rev;
   cudaError_t e = bds::api_launched(bds::launch_ssd_block_state(sp, s), s);
   if (e != cudaSuccess) return e;
   bds::SsdPassParams pp{};
@@ -320,6 +321,51 @@ int bdscan_ssd_wait_selftest(uint32_t polls) {
   if (v < 0) return cuda_fail(cudaGetLastError(), fn);
   bds::api_ok();
   return v;
+}
+
+size_t bdscan_ssd_full_bidir_workspace_size(const bdscan_ssd_dims* dims) {
+  bds::SsdGeo g;
+  if (check(dims, &g, "bdscan_ssd_full_bidir_workspace_size") != BDSCAN_OK) return 0;
+  return sumdt_bytes(g) + states_bytes(g) + al256((size_t)g.Bt * g.L * g.H * 64 * 4);
+}
+
+int bdscan_ssd_full_bidir_forward(const bdscan_ssd_dims* dims, const bdscan_noisy* noisy, const bdscan_params* params,
+                                  void* y, void* workspace, size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_ssd_full_bidir_forward";
+  bds::SsdGeo g;
+  int rc = check(dims, &g, fn);
+  if (rc) return rc;
+  if (g.Bt == 0 || g.nb == 0 || g.H == 0) return bds::api_ok();
+  if ((rc = check_noisy(noisy, params, fn))) return rc;
+  SSD_REQ(y, fn, "y");
+  SSD_REQ(workspace, fn, "workspace");
+  const size_t need = sumdt_bytes(g) + states_bytes(g) + al256((size_t)g.Bt * g.L * g.H * 64 * 4);
+  if (workspace_bytes < need) return failf(BDSCAN_ERR_ARG, "%s: workspace too small%s", fn);
+  int* flag = bds::ssd_wait_flag_ptr();
+  if (flag == nullptr) return cuda_fail(cudaGetLastError(), fn);
+  cudaStream_t s = (cudaStream_t)stream;
+  float* sumdt = (float*)workspace;
+  float* st = (float*)((char*)workspace + sumdt_bytes(g));
+  float* y32 = (float*)((char*)st + states_bytes(g));
+  // each direction is the clean-stream scan over the whole sequence: left to
+  // right with the forward parameters, then right to left with the reverse
+  // ones; the first writes fp32, the second adds it and rounds once
+  cudaError_t e = cudaSuccess;
+  for (int dir = 0; dir < 2 && e == cudaSuccess; ++dir) {
+    const bdscan_clean c{noisy->x, dir ? noisy->dt_r : noisy->dt_f, dir ? noisy->B_r : noisy->B_f,
+                         dir ? noisy->C_r : noisy->C_f};
+    const float* A = dir ? params->A_r : params->A_f;
+    const float* D = dir ? params->D_r : params->D_f;
+    e = build_states(g, &c, A, nullptr, st, sumdt, nullptr, flag, s, dir);
+    if (e != cudaSuccess) break;
+    bds::SsdScanParams cp = clean_scan(g, &c, A, D, st, nullptr, y, flag);
+    cp.rev = dir;
+    if (dir == 0) cp.y32 = y32;
+    else cp.y32_add = y32;
+    e = bds::api_launched(bds::launch_ssd_block_scan(false, cp, s), s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return bds::api_ok();
 }
 
 }  // extern "C"

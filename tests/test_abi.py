@@ -219,3 +219,17 @@ def test_ssd_rejects_bad_pointers():
 def test_ssd_wait_selftest_checks_polls():
     assert binding.bdscan_ssd_wait_selftest(0) == binding.BDSCAN_ERR_ARG
     assert "polls" in binding.bdscan_last_error()
+
+
+def test_ssd_full_bidir_checks_and_workspace():
+    al = lambda x: (x + 255) // 256 * 256
+    d = _ssd_dims(batch=2, length=512, block=256, heads=4, d_state=128)
+    nb = 2
+    assert binding.bdscan_ssd_full_bidir_workspace_size(d) == (al(2 * nb * 4 * 4) + al(2 * nb * 4 * 64 * 128 * 4)
+                                                              + al(2 * 512 * 4 * 64 * 4))
+    _, n, p = _structs()
+    rc = binding.bdscan_ssd_full_bidir_forward(d, n, p, FAKE, FAKE, 64, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "workspace too small" in binding.bdscan_last_error()
+    n.C_f = None
+    rc = binding.bdscan_ssd_full_bidir_forward(d, n, p, FAKE, FAKE, 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "noisy.C_f is NULL" in binding.bdscan_last_error()

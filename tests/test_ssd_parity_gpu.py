@@ -157,3 +157,22 @@ def test_ssd_bounded_wait_reports_instead_of_hanging():
     wl = SsdWorkload(1, 256, 128, 2, 64, seed=4)
     _, y_c, y_n, st = _forward(wl)
     _check(y_c, y_n, st, _oracle(wl))
+
+
+@pytest.mark.parametrize("cfg", [(1, 512, 256, 3, 128), (2, 384, 128, 5, 64)])
+def test_ssd_full_bidir_matches_oracle(cfg):
+    """Full-sequence bidirectional SSD layer against the oracle: one noisy block
+    spanning the whole sequence (seed 0) is exactly that layer."""
+    from oracle import ssd
+    wl = SsdWorkload(*cfg, seed=6)
+    t = _dev(wl)
+    d = _dims(wl)
+    y = torch.empty((wl.batch, wl.len, wl.heads, 64), dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(binding.bdscan_ssd_full_bidir_workspace_size(d), dtype=torch.uint8, device="cuda")
+    binding.ssd_full_bidir_forward(d, t, y, ws)
+    torch.cuda.synchronize()
+    assert binding.bdscan_ssd_wait_flag(1) == 0
+    z = {k: np.zeros_like(wl.f64(k)) for k in ("x_c", "dt_c", "B_c", "C_c")}
+    args = [z[k] if k in z else wl.f64(k) for k in NAMES]
+    _, y_ref, _ = ssd.forward(wl.len, *args)
+    P.assert_close("y (full bidirectional)", to_numpy(y), y_ref, P.FWD_TOL, P.BF16_U)
