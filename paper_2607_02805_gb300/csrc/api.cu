@@ -4,6 +4,8 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <atomic>
+#include <mutex>
 
 #include "bdscan.h"
 #include "params.h"
@@ -533,6 +535,51 @@ int api_ok() { return ok(); }
 void api_begin() { g_launches = 0; }
 
 cudaError_t api_launched(cudaError_t e, cudaStream_t s) { return launched(e, s); }
+
+// Kernel attributes are set once per (kernel, device, size): repeated calls
+// (an active-block loop) then skip the runtime calls on their host path.
+cudaError_t set_smem_cached(const void* fn, int bytes, int carveout) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  struct Entry {
+    const void* fn;
+    int dev, bytes, carveout;
+  };
+  static std::mutex mu;
+  static Entry tab[256];
+  static int n = 0;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    for (int i = 0; i < n; ++i)
+      if (tab[i].fn == fn && tab[i].dev == dev && tab[i].bytes >= bytes && tab[i].carveout == carveout)
+        return cudaSuccess;
+  }
+  if ((e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes)) != cudaSuccess) return e;
+  if (carveout >= 0 && (e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, carveout)) !=
+                           cudaSuccess)
+    return e;
+  std::lock_guard<std::mutex> lk(mu);
+  for (int i = 0; i < n; ++i)
+    if (tab[i].fn == fn && tab[i].dev == dev && tab[i].carveout == carveout) {
+      if (bytes > tab[i].bytes) tab[i].bytes = bytes;
+      return cudaSuccess;
+    }
+  if (n < 256) tab[n++] = Entry{fn, dev, bytes, carveout};
+  return cudaSuccess;
+}
+
+// Multiprocessor count of the current device, looked up once per device.
+int sm_count_cached() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return 0;
+  static std::atomic<int> counts[256];
+  int v = counts[dev].load(std::memory_order_relaxed);
+  if (v > 0) return v;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) return 0;
+  counts[dev].store(v, std::memory_order_relaxed);
+  return v;
+}
 
 // Validation shared with other entry points that take forward-side dims.
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn) {

@@ -81,6 +81,8 @@ int api_fail(int code, const char* msg);
 int api_ok();
 void api_begin();
 cudaError_t api_launched(cudaError_t e, cudaStream_t s);
+cudaError_t set_smem_cached(const void* fn, int bytes, int carveout);  // carveout < 0: leave it
+int sm_count_cached();  // 0 if unknown
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn);
 size_t api_fwd_workspace(const Geo& g, int N);
 int bwd_chunk_count(int dt, int N, const Geo& g);

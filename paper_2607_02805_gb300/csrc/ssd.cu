@@ -18,9 +18,11 @@
 //     is written to shared memory in bf16 and multiplied with x on the tensor
 //     core; the seed term is a second MMA (seed split into bf16 high and low
 //     parts); the epilogue adds the decayed seed term and D x.
+#include <atomic>
 #include <cstdio>
 
 #include "device.cuh"
+#include "params.h"
 #include "ssd.cuh"
 #include "umma.cuh"
 
@@ -735,8 +737,16 @@ cudaError_t launch_ssd_wait_probe(uint32_t polls, cudaStream_t s) {
 }
 
 int* ssd_wait_flag_ptr() {
+  // device address of the flag, looked up once per device (the symbol names
+  // a different address on each device)
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return nullptr;
+  static std::atomic<int*> addr[256];
+  int* a = addr[dev].load(std::memory_order_acquire);
+  if (a != nullptr) return a;
   void* p = nullptr;
   if (cudaGetSymbolAddress(&p, g_ssd_wait_flag) != cudaSuccess) return nullptr;
+  addr[dev].store(static_cast<int*>(p), std::memory_order_release);
   return static_cast<int*>(p);
 }
 
@@ -744,9 +754,7 @@ namespace {
 
 template <typename K>
 cudaError_t set_smem(K kernel, uint32_t bytes) {
-  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  return set_smem_cached(reinterpret_cast<const void*>(kernel), (int)bytes, 100);
 }
 
 }  // namespace

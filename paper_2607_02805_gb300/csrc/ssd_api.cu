@@ -59,9 +59,7 @@ int check(const bdscan_ssd_dims* d, bds::SsdGeo* g, const char* fn) {
 }
 
 int sm_count() {
-  int dev = 0, n = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    return 1;
+  const int n = bds::sm_count_cached();
   return n > 0 ? n : 1;
 }
 
