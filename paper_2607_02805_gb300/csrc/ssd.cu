@@ -5,8 +5,9 @@
 // Per block of Bs tokens (Bs = 128 m) and head h, with a_t = exp(dt_t A[h]):
 //   * block-local end state (k_ssd_block_state):
 //       T = sum_s w_s x_s B_s^T, w_s = exp(A sum_{r>s} dt_r) dt_s,
-//     one MMA chain (M = 128 state rows, N = 64 channels, K = Bs tokens) per
-//     head, with A = (w o B)^T split into bf16 high and low parts;
+//     one MMA chain per head (M = 128 state rows, N = 64 channels, K = Bs
+//     tokens): the block's B rows as stored are the MN-major A operand, the
+//     weighted x (w o x, split into bf16 high and low parts) the B operand;
 //   * the exact state at each block end (k_ssd_state_pass):
 //       S_k = exp(A sum_block dt) S_{k-1} + T_k, in fp32, sequential in k;
 //   * the block's output (k_ssd_block_scan), for a 128-token tile t of the block:
@@ -398,7 +399,7 @@ template <int N, bool NOISY>
 __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdScanParams p) {
   extern __shared__ unsigned char smraw[];
   unsigned char* sm = align1024(smraw);
-  __shared__ uint64_t bar[3];
+  __shared__ uint64_t bar[2];  // [0]: a head's MMAs, [1]: the Gram products
   __shared__ uint32_t tslot;
   const SsdGeo& g = p.g;
   const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x;
@@ -448,7 +449,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       s_prm[48 + t] = p.Dr[h0 + t];
     }
   }
-  for (int e = t; e < Bs * hg; e += kScanThreads) {  // dt of the CTA's heads, fp32
+  for (int e = t; e < Bs * hg; e += kScanThreads) {  // dt of the CTA's heads, bf16 as stored
     const int s = e / hg, hh = e - s * hg;
     s_dtf[s * hg + hh] = p.dtf[tok(s) * H + h0 + hh];
     if (NOISY) s_dtr[s * hg + hh] = p.dtr[tok(s) * H + h0 + hh];
@@ -456,7 +457,6 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   if (t == 0) {
     umma::bar_init(&bar[0], 1);
     umma::bar_init(&bar[1], 1);
-    umma::bar_init(&bar[2], 1);
   }
   if (t < 32) tmem_alloc(&tslot, 512);
   cp_async_wait_all();
@@ -470,9 +470,9 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     const uint32_t base = umma::smem_u32(sm);
     for (int qq = 0; qq < nf + nr; ++qq)
       mma_gram<N>(tm + 128u * qq, base + (qq < nf ? L.cf : L.m1), base + L.r + qq * 128u * N * 2u);
-    umma::mma_commit(&bar[2]);
+    umma::mma_commit(&bar[1]);
   }
-  bool alive = cta_wait(&bar[2], 0, p.flag);
+  bool alive = cta_wait(&bar[1], 0, p.flag);
   umma::fence_after_sync();
   // the first head's x and seed (the B tiles are no longer read)
   if (alive && h0 < h1)
