@@ -88,14 +88,16 @@ def test_ssd_forward_matches_oracle(cfg):
     _check(y_c, y_n, st, _oracle(wl))
 
 
-def test_ssd_full_size_sampled():
-    """The 350M-class Mamba-2 layer at training size (batch 8, 8192 tokens per
-    stream, block 256, 26 heads of 64, state 128), in the bench's launch
-    configuration; the oracle runs two heads of one batch row (heads and batch
-    rows are independent given the shared B, C)."""
-    wl = SsdWorkload(8, 8192, 256, 26, 128, seed=0)
+@pytest.mark.parametrize("cfg,heads,rows", [((8, 8192, 256, 26, 128), [0, 25], [5]),
+                                            ((8, 8192, 256, 14, 64), [3, 13], [0])])
+def test_ssd_full_size_sampled(cfg, heads, rows):
+    """The 350M-class (26 heads of 64, state 128) and 87M-class (14 heads,
+    state 64) Mamba-2 layers at training size (batch 8, 8192 tokens per
+    stream, block 256), in the bench's launch configuration; the oracle runs
+    two heads of one batch row (heads and batch rows are independent given
+    the shared B, C)."""
+    wl = SsdWorkload(*cfg, seed=0)
     _, y_c, y_n, st = _forward(wl)
-    heads, rows = [0, 25], [5]
     _check(y_c, y_n, st, _oracle(wl, heads=heads, rows=rows), heads=heads, rows=rows)
 
 
