@@ -63,30 +63,44 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
 // ---------------------------------------------------------------------------
 // Deterministic reductions
 // ---------------------------------------------------------------------------
+// One thread per 4 consecutive state indices of one row of one tensor: the
+// channel-group partials are summed in group order (16-byte loads).
 template <typename TO, int N>
 __global__ void __launch_bounds__(256) k_reduce_tok(const BwdParams p) {
   const Geo& g = p.g;
   const int64_t rows = g.Bt * g.L;
   const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (idx >= 6 * rows * N) return;
-  const int n = (int)(idx % N);
-  const int64_t row = idx / N;
+  if (idx >= 6 * rows * (N / 4)) return;
+  const int n = (int)(idx % (N / 4)) * 4;
+  const int64_t row = idx / (N / 4);
   const int tensor = (int)(row / rows);
   const int64_t bt = row - (int64_t)tensor * rows;
   const float* src = p.part_tok + row * g.G * N + n;
-  float s = 0.f;
-  for (int gi = 0; gi < g.G; ++gi) s += src[(int64_t)gi * N];
+  float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int gi = 0; gi < g.G; ++gi) {
+    const float4 v = *reinterpret_cast<const float4*>(src + (int64_t)gi * N);
+    s.x += v.x;
+    s.y += v.y;
+    s.z += v.z;
+    s.w += v.w;
+  }
   void* dst = tensor == 0 ? p.dBc : tensor == 1 ? p.dCc : tensor == 2 ? p.dBf : tensor == 3 ? p.dCf
             : tensor == 4 ? p.dBr : p.dCr;
-  reinterpret_cast<TO*>(dst)[bt * N + n] = to_out<TO>(s);
+  TO* d = reinterpret_cast<TO*>(dst) + bt * N + n;
+  d[0] = to_out<TO>(s.x);
+  d[1] = to_out<TO>(s.y);
+  d[2] = to_out<TO>(s.z);
+  d[3] = to_out<TO>(s.w);
 }
 
-// One CTA sums 32 columns of the per-chunk partials: 8 slices of threads
-// each add every 8th chunk (in order), then the slices are added in order.
+// One CTA sums 128 columns (32 lanes x 4) of the per-chunk partials: 16
+// slices of threads each add every 16th chunk (in order), then the slices
+// are added in order.
+constexpr int kParSlices = 16;
 template <int N>
-__global__ void __launch_bounds__(256) k_reduce_par(const BwdParams p) {
-  // 8 slices (warps) of the chunk partials; each lane sums 4 adjacent columns
-  __shared__ float4 part[3][8][32];
+__global__ void __launch_bounds__(32 * kParSlices) k_reduce_par(const BwdParams p) {
+  // kParSlices slices (warps) of the chunk partials; each lane sums 4 adjacent columns
+  __shared__ float4 part[3][kParSlices][32];
   const Geo& g = p.g;
   const int64_t U = g.Bt * g.nc;
   const int64_t DN = g.D * N;
@@ -105,7 +119,7 @@ __global__ void __launch_bounds__(256) k_reduce_par(const BwdParams p) {
     const float* a1 = p.part_A + U * DN + col;
     const float* a2 = p.part_A + 2 * U * DN + col;
 #pragma unroll 4
-    for (int64_t u = slice; u < U; u += 8) {
+    for (int64_t u = slice; u < U; u += kParSlices) {
       acc(s0, a0 + u * DN);
       acc(s1, a1 + u * DN);
       acc(s2, a2 + u * DN);
@@ -113,7 +127,7 @@ __global__ void __launch_bounds__(256) k_reduce_par(const BwdParams p) {
   } else if (col < DN + g.D) {
     const int64_t d = col - DN;
 #pragma unroll 4
-    for (int64_t u = slice; u < U; u += 8) {
+    for (int64_t u = slice; u < U; u += kParSlices) {
       acc(s0, p.part_D + u * g.D + d);
       acc(s1, p.part_D + (U + u) * g.D + d);
     }
@@ -125,7 +139,7 @@ __global__ void __launch_bounds__(256) k_reduce_par(const BwdParams p) {
   if (slice == 0) {
     float4 t0 = part[0][0][lane], t1 = part[1][0][lane], t2 = part[2][0][lane];
 #pragma unroll
-    for (int k = 1; k < 8; ++k) {
+    for (int k = 1; k < kParSlices; ++k) {
       const float4 v0 = part[0][k][lane], v1 = part[1][k][lane], v2 = part[2][k][lane];
       t0 = make_float4(t0.x + v0.x, t0.y + v0.y, t0.z + v0.z, t0.w + v0.w);
       t1 = make_float4(t1.x + v1.x, t1.y + v1.y, t1.z + v1.z, t1.w + v1.w);
@@ -150,7 +164,7 @@ cudaError_t launch_bwd_carry(int N, const BwdParams& p, cudaStream_t s) {
 }
 
 cudaError_t launch_bwd_reduce_tok(int dt, int N, const BwdParams& p, cudaStream_t s) {
-  const int64_t ntok = 6 * p.g.Bt * p.g.L * N;
+  const int64_t ntok = 6 * p.g.Bt * p.g.L * (N / 4);
   if (ntok == 0) return cudaSuccess;
   const unsigned blocks = (unsigned)((ntok + 255) / 256);
   if (dt == 1) {
@@ -161,7 +175,8 @@ cudaError_t launch_bwd_reduce_tok(int dt, int N, const BwdParams& p, cudaStream_
 
 cudaError_t launch_bwd_reduce_par(int N, const BwdParams& p, cudaStream_t s) {
   const int64_t npar4 = (p.g.D * N + p.g.D) / 4;  // float4 columns
-  BDS_DISPATCH_N(N, k_reduce_par<NN><<<(unsigned)((npar4 + 31) / 32), 256, 0, s>>>(p); return cudaGetLastError();)
+  BDS_DISPATCH_N(N, k_reduce_par<NN><<<(unsigned)((npar4 + 31) / 32), 32 * kParSlices, 0, s>>>(p);
+                 return cudaGetLastError();)
 }
 
 // Backward chunks per batch row, between 1 and bwd_max_chunks(); both
