@@ -29,7 +29,9 @@ semiseparable-matrix form of the block restriction (y = M x with the scalar
 decay written as exp of a sum, built independently of any recurrence), the
 closed form of the state at a block end, the single-block invariant,
 bit-exact caching, and (backward) central finite differences of the pinned
-forward for every input, including the tied A, D and dt.
+forward for every input, including the tied A, D and dt, plus an exact
+matrix-form check of the linear gradients (dx, dB, dC of every stream,
+including the clean x and B through the cached states).
 """
 
 from __future__ import annotations

@@ -150,3 +150,74 @@ def test_ssd_backward_matches_finite_differences(seed, Bs):
         fd = (loss(dp) - loss(dm)) / (2 * eps)
         an = float((g[k] * v).sum())
         assert abs(fd - an) <= 1e-6 * max(1.0, abs(an)), (k, an, fd)
+
+
+def _kernel(dt, A, lo, hi, t, s):
+    """decay * dt_s of the forward (s <= t) direction inside [lo, hi]."""
+    return np.exp(A * _dsum(dt, s + 1, t)) * dt[s]
+
+
+def test_ssd_backward_linear_gradients_matrix_form():
+    """dx, dB and dC of the oracle's SSD backward against the same gradients
+    written out from the semiseparable matrix form (explicit sums; the clean
+    x and B also receive the gradient through the cached block-end states, as
+    the seed of every next noisy block and through dstates)."""
+    Bs, d = _inputs(7, Bt=1, L=8, Bs=4, H=2, P=2, N=3)
+    Bt, L, H, P = d["x_c"].shape
+    N = d["B_c"].shape[2]
+    nb = L // Bs
+    y_c, y_n, st = ssd.forward(Bs, *[d[k] for k in NAMES])
+    rng = np.random.default_rng(11)
+    dyc, dyn, dst = rng.standard_normal(y_c.shape), rng.standard_normal(y_n.shape), rng.standard_normal(st.shape)
+    g = ssd.backward(Bs, *[d[k] for k in NAMES], st, dyc, dyn, dst)
+    b = 0
+    want = {k: np.zeros_like(d[k]) for k in ("x_c", "x_n", "B_c", "C_c", "B_f", "C_f", "B_r", "C_r")}
+    for h in range(H):
+        dc, df, dr = d["dt_c"][b, :, h], d["dt_f"][b, :, h], d["dt_r"][b, :, h]
+        Af, Ar, Df, Dr = d["A_f"][h], d["A_r"][h], d["D_f"][h], d["D_r"][h]
+        xc, xn = d["x_c"][b, :, h], d["x_n"][b, :, h]
+        Bc, Cc, Bf, Cf, Br, Cr = (d[k][b] for k in ("B_c", "C_c", "B_f", "C_f", "B_r", "C_r"))
+        # total gradient of each block-end state: dstates + the seed term of the next noisy block
+        Gk = np.array(dst[b, :, h], dtype=float)
+        for k in range(nb - 1):
+            lo, hi = (k + 1) * Bs, (k + 2) * Bs - 1
+            for t in range(lo, hi + 1):
+                Gk[k] += np.exp(Af * _dsum(df, lo, t)) * np.outer(dyn[b, t, h], Cf[t])
+        # clean stream: y_c = sum_s (C_t . B_s) K_ts x_s + D_f x_t over the whole stream
+        for t in range(L):
+            want["x_c"][b, t, h] += Df * dyc[b, t, h]
+            for s in range(t + 1):
+                K = _kernel(dc, Af, 0, L - 1, t, s)
+                gts = Cc[t] @ Bc[s]
+                want["x_c"][b, s, h] += gts * K * dyc[b, t, h]
+                q = dyc[b, t, h] @ xc[s]
+                want["C_c"][b, t] += q * K * Bc[s]
+                want["B_c"][b, s] += q * K * Cc[t]
+        # clean x and B through the states: S_k = sum_{s <= e_k} exp(A sum_{s<r<=e_k} dt) dt_s x_s B_s^T
+        for k in range(nb):
+            e = (k + 1) * Bs - 1
+            for s in range(e + 1):
+                w = _kernel(dc, Af, 0, e, e, s)
+                want["x_c"][b, s, h] += w * (Gk[k] @ Bc[s])
+                want["B_c"][b, s] += w * (xc[s] @ Gk[k])
+        # noisy blocks: forward (lower, with seed), reverse (upper), D terms
+        for k in range(nb):
+            lo, hi = k * Bs, (k + 1) * Bs - 1
+            seed = st[b, k - 1, h] if k > 0 else np.zeros((P, N))
+            for t in range(lo, hi + 1):
+                want["x_n"][b, t, h] += (Df + Dr) * dyn[b, t, h]
+                want["C_f"][b, t] += np.exp(Af * _dsum(df, lo, t)) * (dyn[b, t, h] @ seed)
+                for s in range(lo, t + 1):
+                    K = _kernel(df, Af, lo, hi, t, s)
+                    q = dyn[b, t, h] @ xn[s]
+                    want["x_n"][b, s, h] += (Cf[t] @ Bf[s]) * K * dyn[b, t, h]
+                    want["C_f"][b, t] += q * K * Bf[s]
+                    want["B_f"][b, s] += q * K * Cf[t]
+                for s in range(t, hi + 1):
+                    K = np.exp(Ar * _dsum(dr, t, s - 1)) * dr[s]
+                    q = dyn[b, t, h] @ xn[s]
+                    want["x_n"][b, s, h] += (Cr[t] @ Br[s]) * K * dyn[b, t, h]
+                    want["C_r"][b, t] += q * K * Br[s]
+                    want["B_r"][b, s] += q * K * Cr[t]
+    for k, v in want.items():
+        assert np.max(np.abs(g[k] - v)) <= 1e-11 * max(1.0, np.max(np.abs(v))), k
