@@ -233,3 +233,21 @@ def test_ssd_full_bidir_checks_and_workspace():
     n.C_f = None
     rc = binding.bdscan_ssd_full_bidir_forward(d, n, p, FAKE, FAKE, 1 << 40, None)
     assert rc == binding.BDSCAN_ERR_ARG and "noisy.C_f is NULL" in binding.bdscan_last_error()
+
+
+def _prototypes():
+    """name -> number of parameters, from the prototypes of include/*.h."""
+    out = {}
+    for h in HEADERS:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        for m in re.finditer(r"\b(bdscan_\w+)\s*\(([^;{]*?)\)\s*;", text, flags=re.S):
+            params = m.group(2).strip()
+            out[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    return out
+
+
+def test_binding_argument_counts_match_the_headers():
+    protos = _prototypes()
+    assert set(protos) == set(header_functions())
+    for name, _, args in binding.SIGNATURES:
+        assert len(args) == protos[name], (name, len(args), protos[name])
