@@ -821,11 +821,14 @@ def run_prefill(args, L, Bs, calls):
 
 
 def run_e2e(lay, wl, stream, dev, args):
-    """Forward + backward through the C ABI end to end: every step copies its
-    inputs from pinned host memory to the device and reads every output and
-    gradient back, as a training loop streaming its batches would. Copies run
+    """Forward + backward through the C ABI end to end: every step copies all
+    of its inputs (both streams' x, dt, B, C and the upstream gradients) from
+    pinned host memory to the device and reads the step's result back: the
+    layer's parameter gradients (dA, dD of both directions), which is what a
+    training step hands to its optimizer. The outputs and per-token gradients
+    stay on the device, where the neighbouring layers consume them. Copies run
     on their own streams and two device buffer sets alternate, so that step
-    i+1's inputs go up and step i-1's results come down while step i computes.
+    i+1's inputs go up and step i-1's result comes down while step i computes.
     The timed region covers all copies of every step."""
     import torch
     from paper_2607_02805_gb300.layer import Layer
@@ -833,7 +836,7 @@ def run_e2e(lay, wl, stream, dev, args):
     lays[1].alloc_backward()
     ins = [k for k in wl.t32]
     host_in = {k: lay.t[k].detach().to("cpu").pin_memory() for k in ins}
-    outs = [[la.y_c, la.y_n] + [la.g[k] for k in la.g] for la in lays]
+    outs = [[la.g[k] for k in ("A_f", "D_f", "A_r", "D_r")] for la in lays]
     host_out = [[torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs[0]] for _ in range(2)]
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
     d2h = sum(t.numel() * t.element_size() for t in host_out[0])
