@@ -8,9 +8,17 @@
 
 namespace {
 
-int failf(int code, const char* fmt, const char* fn, const char* what = "") {
+// "<function>: <message>" as the thread's last error; returns `code`.
+int fail_msg(int code, const char* fn, const char* what) {
   char msg[384];
-  snprintf(msg, sizeof(msg), fmt, fn, what);
+  snprintf(msg, sizeof(msg), "%s: %s", fn, what);
+  return bds::api_fail(code, msg);
+}
+
+// "<function>: <argument> <problem>" as the thread's last error; returns `code`.
+int fail_arg(int code, const char* fn, const char* name, const char* problem) {
+  char msg[384];
+  snprintf(msg, sizeof(msg), "%s: %s %s", fn, name, problem);
   return bds::api_fail(code, msg);
 }
 
@@ -25,29 +33,29 @@ size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 #define SSD_REQ(ptr, fn, name)                                                              \
   do {                                                                                      \
-    if ((ptr) == nullptr) return failf(BDSCAN_ERR_ARG, "%s: %s is NULL", fn, name);         \
-    if (!aligned16(ptr)) return failf(BDSCAN_ERR_ARG, "%s: %s is not 16-byte aligned", fn, name); \
+    if ((ptr) == nullptr) return fail_arg(BDSCAN_ERR_ARG, fn, name, "is NULL");         \
+    if (!aligned16(ptr)) return fail_arg(BDSCAN_ERR_ARG, fn, name, "is not 16-byte aligned"); \
   } while (0)
 #define SSD_OPT(ptr, fn, name)                                                              \
   do {                                                                                      \
     if ((ptr) != nullptr && !aligned16(ptr))                                                \
-      return failf(BDSCAN_ERR_ARG, "%s: %s is not 16-byte aligned", fn, name);              \
+      return fail_arg(BDSCAN_ERR_ARG, fn, name, "is not 16-byte aligned");              \
   } while (0)
 
 // Validates the dimensions and fills the geometry.
 int check(const bdscan_ssd_dims* d, bds::SsdGeo* g, const char* fn) {
   bds::api_begin();
-  if (d == nullptr) return failf(BDSCAN_ERR_ARG, "%s: dims is NULL", fn);
-  if (d->batch < 0 || d->len < 0 || d->heads < 0) return failf(BDSCAN_ERR_ARG, "%s: negative batch, len or heads", fn);
-  if (d->block <= 0) return failf(BDSCAN_ERR_ARG, "%s: block must be positive", fn);
-  if (d->len % d->block != 0) return failf(BDSCAN_ERR_ARG, "%s: len is not a multiple of block", fn);
-  if (d->dtype != BDSCAN_BF16) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: dtype must be bf16", fn);
-  if (d->head_dim != 64) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: head_dim must be 64", fn);
-  if (d->d_state != 64 && d->d_state != 128) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: d_state must be 64 or 128", fn);
-  if (d->block != 128 && d->block != 256) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: block must be 128 or 256", fn);
-  if (d->heads > 65535 * 8) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: too many heads", fn);
+  if (d == nullptr) return fail_msg(BDSCAN_ERR_ARG, fn, "dims is NULL");
+  if (d->batch < 0 || d->len < 0 || d->heads < 0) return fail_msg(BDSCAN_ERR_ARG, fn, "negative batch, len or heads");
+  if (d->block <= 0) return fail_msg(BDSCAN_ERR_ARG, fn, "block must be positive");
+  if (d->len % d->block != 0) return fail_msg(BDSCAN_ERR_ARG, fn, "len is not a multiple of block");
+  if (d->dtype != BDSCAN_BF16) return fail_msg(BDSCAN_ERR_UNSUPPORTED, fn, "dtype must be bf16");
+  if (d->head_dim != 64) return fail_msg(BDSCAN_ERR_UNSUPPORTED, fn, "head_dim must be 64");
+  if (d->d_state != 64 && d->d_state != 128) return fail_msg(BDSCAN_ERR_UNSUPPORTED, fn, "d_state must be 64 or 128");
+  if (d->block != 128 && d->block != 256) return fail_msg(BDSCAN_ERR_UNSUPPORTED, fn, "block must be 128 or 256");
+  if (d->heads > 65535 * 8) return fail_msg(BDSCAN_ERR_UNSUPPORTED, fn, "too many heads");
   const int64_t nb = d->len / d->block;
-  if (d->batch * nb * (d->block / 128) > 0x7fffffffLL) return failf(BDSCAN_ERR_UNSUPPORTED, "%s: too many blocks", fn);
+  if (d->batch * nb * (d->block / 128) > 0x7fffffffLL) return fail_msg(BDSCAN_ERR_UNSUPPORTED, fn, "too many blocks");
   g->Bt = d->batch;
   g->L = d->len;
   g->Bs = d->block;
@@ -91,7 +99,7 @@ size_t sumdt_bytes(const bds::SsdGeo& g) { return al256((size_t)g.Bt * g.nb * g.
 size_t states_bytes(const bds::SsdGeo& g) { return al256((size_t)g.Bt * g.nb * g.H * 64 * g.N * 4); }
 
 int check_clean(const bdscan_clean* c, const char* fn) {
-  if (c == nullptr) return failf(BDSCAN_ERR_ARG, "%s: clean is NULL", fn);
+  if (c == nullptr) return fail_msg(BDSCAN_ERR_ARG, fn, "clean is NULL");
   SSD_REQ(c->x, fn, "clean.x");
   SSD_REQ(c->dt, fn, "clean.dt");
   SSD_REQ(c->B, fn, "clean.B");
@@ -100,8 +108,8 @@ int check_clean(const bdscan_clean* c, const char* fn) {
 }
 
 int check_noisy(const bdscan_noisy* n, const bdscan_params* pr, const char* fn) {
-  if (n == nullptr) return failf(BDSCAN_ERR_ARG, "%s: noisy is NULL", fn);
-  if (pr == nullptr) return failf(BDSCAN_ERR_ARG, "%s: params is NULL", fn);
+  if (n == nullptr) return fail_msg(BDSCAN_ERR_ARG, fn, "noisy is NULL");
+  if (pr == nullptr) return fail_msg(BDSCAN_ERR_ARG, fn, "params is NULL");
   SSD_REQ(n->x, fn, "noisy.x");
   SSD_REQ(n->dt_f, fn, "noisy.dt_f");
   SSD_REQ(n->B_f, fn, "noisy.B_f");
@@ -215,7 +223,7 @@ int bdscan_ssd_forward(const bdscan_ssd_dims* dims, const bdscan_clean* clean, c
   SSD_REQ(y_n, fn, "y_n");
   SSD_REQ(states, fn, "states");
   SSD_REQ(workspace, fn, "workspace");
-  if (workspace_bytes < sumdt_bytes(g)) return failf(BDSCAN_ERR_ARG, "%s: workspace too small%s", fn);
+  if (workspace_bytes < sumdt_bytes(g)) return fail_msg(BDSCAN_ERR_ARG, fn, "workspace too small");
   int* flag = bds::ssd_wait_flag_ptr();
   if (flag == nullptr) return cuda_fail(cudaGetLastError(), fn);
   cudaStream_t s = (cudaStream_t)stream;
@@ -258,7 +266,7 @@ int bdscan_ssd_boundary_states(const bdscan_ssd_dims* dims, const bdscan_clean* 
   SSD_OPT(y_c, fn, "y_c");
   if (y_c != nullptr) SSD_REQ(D_f, fn, "D_f");
   if (workspace_bytes < sumdt_bytes(g) + (emit_all ? 0 : states_bytes(g)))
-    return failf(BDSCAN_ERR_ARG, "%s: workspace too small%s", fn);
+    return fail_msg(BDSCAN_ERR_ARG, fn, "workspace too small");
   int* flag = bds::ssd_wait_flag_ptr();
   if (flag == nullptr) return cuda_fail(cudaGetLastError(), fn);
   cudaStream_t s = (cudaStream_t)stream;
@@ -281,7 +289,7 @@ int bdscan_ssd_active_block(const bdscan_ssd_dims* dims, const float* seed, cons
   bds::SsdGeo g;
   int rc = check(dims, &g, fn);
   if (rc) return rc;
-  if (dims->len != dims->block) return failf(BDSCAN_ERR_ARG, "%s: len must equal block%s", fn);
+  if (dims->len != dims->block) return fail_msg(BDSCAN_ERR_ARG, fn, "len must equal block");
   if (g.Bt == 0 || g.H == 0) return bds::api_ok();
   if ((rc = check_noisy(noisy, params, fn))) return rc;
   SSD_OPT(seed, fn, "seed");
@@ -310,7 +318,7 @@ int bdscan_ssd_wait_flag(int reset) {
 int bdscan_ssd_wait_selftest(uint32_t polls) {
   const char* fn = "bdscan_ssd_wait_selftest";
   bds::api_begin();
-  if (polls == 0 || polls > (1u << 20)) return failf(BDSCAN_ERR_ARG, "%s: polls must be in 1..2^20%s", fn);
+  if (polls == 0 || polls > (1u << 20)) return fail_msg(BDSCAN_ERR_ARG, fn, "polls must be in 1..2^20");
   if (bdscan_ssd_wait_flag(1) < 0) return cuda_fail(cudaGetLastError(), fn);
   cudaError_t e = bds::api_launched(bds::launch_ssd_wait_probe(polls, nullptr), nullptr);
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -338,7 +346,7 @@ int bdscan_ssd_full_bidir_forward(const bdscan_ssd_dims* dims, const bdscan_nois
   SSD_REQ(y, fn, "y");
   SSD_REQ(workspace, fn, "workspace");
   const size_t need = sumdt_bytes(g) + states_bytes(g) + al256((size_t)g.Bt * g.L * g.H * 64 * 4);
-  if (workspace_bytes < need) return failf(BDSCAN_ERR_ARG, "%s: workspace too small%s", fn);
+  if (workspace_bytes < need) return fail_msg(BDSCAN_ERR_ARG, fn, "workspace too small");
   int* flag = bds::ssd_wait_flag_ptr();
   if (flag == nullptr) return cuda_fail(cudaGetLastError(), fn);
   cudaStream_t s = (cudaStream_t)stream;
