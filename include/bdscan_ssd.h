@@ -3,8 +3,9 @@
  * bidirectional scan in libbdscan (arXiv 2607.02805, sm_103a).
  *
  * The paper's trained BDLM Mamba-H layers are Mamba-2 mixers (Appendix C:
- * head dimension 64, state 64 or 128, chunk 128; block 256 in Appendix C's
- * hyperparameter table). In that form the decay is one scalar per head and
+ * state 64 or 128, chunk 128, expansion 2; block 256 in the hyperparameter
+ * table; the head dimension is not given for the Mamba mixers, 64 is the
+ * Mamba-2 default). In that form the decay is one scalar per head and
  * B_t, C_t are shared by every channel (one group): for channel p of head h,
  *   h_t[p, :] = exp(dt_t[h] A[h]) h_{t-1}[p, :] + dt_t[h] x_t[h, p] B_t
  *   y_t[h, p] = C_t . h_t[p, :] + D[h] x_t[h, p]
