@@ -3,8 +3,8 @@
 TEST INFRASTRUCTURE, like the rest of ``oracle/``: only ``tests/``,
 ``__graft_entry__.smoke()`` and the CPU baseline of ``bench.py`` may use it.
 
-The paper's trained mixers are Mamba-2 layers (Appendix C: head dimension,
-state size 64 or 128, chunk 128; block 256). In that form the decay is one
+The paper's trained mixers are Mamba-2 layers (Appendix C: state size 64 or
+128, chunk 128; block 256). In that form the decay is one
 scalar per head, A[h], and B_t, C_t are shared by every channel of the layer
 (one group). For channel d = h * P + p of head h the recurrence is the
 selective update of Sec. 3 (eq. mamba-scan-background) with
