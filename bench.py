@@ -79,9 +79,9 @@ def kernel_bytes(Bt, L, D, N, Bs, in_b=2, out_b=2):
 
 
 # DRAM bytes (read + write) per launch of the dominant kernel, from one
-# `ncu --set full` capture at batch 4 (profiles/k_bwd_noisy_87m_layer_batch4.md),
-# scaled by batch / 4: the kernel's traffic is proportional to the batch. Set
-# to None whenever the kernel changes until it is captured again.
+# `ncu --set full` capture of the same kernel at batch 4, scaled by batch / 4:
+# the kernel's traffic is proportional to the batch. Set to None whenever the
+# kernel changes until it is captured again.
 MEASURED_TRAFFIC_BATCH4 = {"bwd_noisy": 330_220_544}
 
 # FP32 work per (token, channel, state) element of each scan kernel, counted

@@ -33,8 +33,29 @@ def rel_err(gpu, ora, u=0.0):
     return float(max(0.0, np.max(excess)) / scale)
 
 
+def elementwise_rel_err(gpu, ora):
+    """Largest per-element relative error |gpu - oracle| / (|oracle| + 1e-3 rms(oracle)):
+    reported for information next to the per-tensor bound (the rms term keeps
+    elements near zero from dominating)."""
+    gpu = np.asarray(gpu, dtype=np.float64)
+    ora = np.asarray(ora, dtype=np.float64)
+    if ora.size == 0:
+        return 0.0
+    rms = float(np.sqrt(np.mean(ora * ora)))
+    if rms == 0.0:
+        return float(np.max(np.abs(gpu)))
+    return float(np.max(np.abs(gpu - ora) / (np.abs(ora) + 1e-3 * rms)))
+
+
+# (test id, tensor, per-tensor error, elementwise error) of every comparison
+# made in this process, printed in the pytest summary
+RECORD = []
+_CURRENT_TEST = [""]
+
+
 def assert_close(name, gpu, ora, tol, u=0.0):
     e = rel_err(gpu, ora, u)
+    RECORD.append((_CURRENT_TEST[0], name, e, elementwise_rel_err(gpu, ora)))
     assert e <= tol, f"{name}: relative error {e:.3e} above {tol:.1e}"
     return e
 

@@ -59,15 +59,23 @@ def _run_both(Bt, L, Bs, D, N, seed, emit_all, want_y, with_init):
     rc = binding.bdscan_boundary_states(dims, clean, t["A_f"].data_ptr(), t["D_f"].data_ptr(), _ptr(init),
                                         _ptr(y_ws), st_ws.data_ptr(), emit_all, ws.data_ptr(), nbytes, stream)
     assert rc == binding.BDSCAN_OK, binding.bdscan_last_error()
+    launches_ws = binding.bdscan_last_launch_count()
     # the entry point without a workspace
     st_na, y_na = _outputs(wl, t, emit_all, want_y)
     rc = binding.bdscan_boundary_states_noalloc(dims, clean, t["A_f"].data_ptr(), t["D_f"].data_ptr(), _ptr(init),
                                                 _ptr(y_na), st_na.data_ptr(), emit_all, stream)
     assert rc == binding.BDSCAN_OK, binding.bdscan_last_error()
+    # the same kernels, counted the same way by the library's launch counter
+    assert binding.bdscan_last_launch_count() == launches_ws
     torch.cuda.synchronize()
+    # Both paths run the same kernels on the same inputs, so the results are
+    # the same bits. The tolerance check runs first only to report the size
+    # of a difference, should there be one.
     P.assert_close("states", to_numpy(st_na), to_numpy(st_ws), P.FWD_TOL)
+    assert torch.equal(st_na, st_ws)
     if want_y:
         P.assert_close("y_c", to_numpy(y_na), to_numpy(y_ws), P.FWD_TOL, P.BF16_U)
+        assert torch.equal(y_na, y_ws)
 
 
 def test_noalloc_matches_workspace_entry_point_two_calls_in_a_row():
@@ -76,6 +84,11 @@ def test_noalloc_matches_workspace_entry_point_two_calls_in_a_row():
     # second call, a different problem: final state only, continued from an
     # initial state, ragged last chunk (it rescans that chunk from scratch data)
     _run_both(1, 400, 16, 136, 8, seed=2, emit_all=False, want_y=False, with_init=True)
+    # third call: final state only over whole chunks (512 tokens at block 16
+    # are four 128-token chunks), so the final state is copied out of the
+    # scratch row by row with the chunk-slot pitch
+    assert 512 % binding.bdscan_chunk_tokens(16) == 0
+    _run_both(2, 512, 16, 136, 16, seed=3, emit_all=False, want_y=False, with_init=True)
 
 
 def test_noalloc_rejects_problems_larger_than_its_scratch():
