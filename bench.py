@@ -84,14 +84,36 @@ def kernel_bytes(Bt, L, D, N, Bs, in_b=2, out_b=2):
 # kernel changes until it is captured again.
 MEASURED_TRAFFIC_BATCH4 = {"bwd_noisy": 330_220_544}
 
-# FP32 work per (token, channel, state) element of each scan kernel, counted
-# from the kernel's arithmetic (FMA = 2 flops; ex2, mul, add, reduction add = 1).
-KERNEL_FLOPS_PER_ELEM = {
-    "chunk_local": 6,     # dt*A, ex2, u*B, fma
-    "block_scan": 21,     # 3 directions x (dt*A, ex2, u*B, fma h, fma y)
-    "bwd_noisy": 47,      # clean local adjoint 5 + 2 directions x (recompute 7 + adjoint 14)
-    "bwd_clean": 21,      # recompute 7 + adjoint 14
+# FP32 operations per (token, channel, state) element of each pass the scan
+# kernels make, listed as the kernels write them (an FMA counts 2, ex2, mul,
+# add and a reduction add 1 each):
+#   scan       forward step with output: dt*A, ex2, u*B, a*h+uB, C*h+acc
+#   scan_state forward step without output: dt*A, ex2, u*B, a*h+uB
+#   recompute  backward recompute: dt*A, ex2, a*h, u*B+p, dy*h, channel add (dC)
+#   adjoint    backward adjoint: dt*A, ex2, C*dy+g, a*gb, gb*p, A*q+sa, dt*q+dA,
+#              gb*B+sg, gb*u, channel add (dB)
+#   half       the half-state scheme's rebuild of every other state, per
+#              element and token: (u*B + a*S) every second token
+#   local      chunk-local adjoint carry: dt*A, ex2, C*dy+carry, a*(...)
+PASS_FLOPS = {
+    "scan": 1 + 1 + 1 + 2 + 2,
+    "scan_state": 1 + 1 + 1 + 2,
+    "recompute": 1 + 1 + 1 + 2 + 1 + 1,
+    "adjoint": 1 + 1 + 2 + 1 + 1 + 2 + 2 + 2 + 1 + 1,
+    "half": (2 + 1) / 2,
+    "local": 1 + 1 + 2 + 1,
 }
+# The passes of each kernel per element (blocks of one 16-token segment).
+KERNEL_PASSES = {
+    "chunk_local": ["scan_state"],
+    "block_scan": ["scan", "scan", "scan"],                     # clean rescan, noisy forward, noisy reverse
+    "bwd_noisy": ["local"] + ["recompute", "adjoint"] * 2,      # clean local adjoint, both noisy directions
+    "bwd_clean": ["recompute", "adjoint", "half"],
+}
+
+
+def kernel_flops_per_elem(name):
+    return sum(PASS_FLOPS[q] for q in KERNEL_PASSES.get(name, []))
 
 
 def sample_clocks(stop, rows, bus_id):
@@ -321,6 +343,8 @@ def run_ours(args, rank, world, local_rank):
     # end-to-end through the public API with host buffers
     e2e = run_e2e(lay, wl, stream, dev, args)
     e2e["ms"] = max_over_ranks(e2e["ms"], dev, world)
+    e2e_full = run_e2e(lay, wl, stream, dev, args, full_readback=True)
+    e2e_full["ms"] = max_over_ranks(e2e_full["ms"], dev, world)
     stop.set()
 
     if rank != 0:
@@ -341,7 +365,11 @@ def run_ours(args, rank, world, local_rank):
     elems = Bt * L * D * N
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
     fp32_peak_tflops = 152 * 128 * 2 * sm_max * 1e6 / 1e12
-    dom_flops = KERNEL_FLOPS_PER_ELEM.get(dname, 0) * elems
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    dom_flops = kernel_flops_per_elem(dname) * elems
+    dom_gbs = kb[dname] / (avg_us[dom] * 1e-6) / 1e9
+    # the dominant kernel against the FP32 ALU roofline that binds it, with its
+    # algorithmic-byte HBM fraction beside it
     roofline = {"bound": "alu", "kernel": dname,
                 "achieved": round(dom_flops / (avg_us[dom] * 1e-6) / 1e12, 2),
                 "peak": round(fp32_peak_tflops, 1), "unit": "TFLOP/s",
@@ -349,13 +377,17 @@ def run_ours(args, rank, world, local_rank):
                 "traffic": (None if MEASURED_TRAFFIC_BATCH4.get(dname) is None
                             else int(MEASURED_TRAFFIC_BATCH4[dname] * Bt / 4)),
                 "peak_kind": "derived: 152 SMs x 128 FP32 lanes x 2 flop/FMA x max SM clock",
-                "flops_per_launch": dom_flops}
+                "flops_per_launch": dom_flops,
+                "flops_per_elem": {"passes": KERNEL_PASSES.get(dname, []), "total": kernel_flops_per_elem(dname)},
+                "hbm": {"achieved": round(dom_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                        "frac": round(dom_gbs / hbm_peak, 4), "alg_bytes_per_launch": kb[dname],
+                        "peak_kind": peak_kind}}
     hbm = {"bound": "hbm", "achieved": round((fb + bb) / (ms_step * 1e-3) / 1e9, 1),
            "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
-           "frac": round((fb + bb) / (ms_step * 1e-3) / 1e9 / float(peaks.get("hbm_gbs", 6800.0)), 4),
+           "frac": round((fb + bb) / (ms_step * 1e-3) / 1e9 / hbm_peak, 4),
            "frac_of_8tbs": round((fb + bb) / (ms_step * 1e-3) / 8e12, 4),
            "alg_bytes_per_step": fb + bb, "peak_kind": peak_kind,
-           "dominant_kernel_gbs": round(kb[dname] / (avg_us[dom] * 1e-6) / 1e9, 1)}
+           "dominant_kernel_gbs": round(dom_gbs, 1)}
 
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
@@ -371,7 +403,11 @@ def run_ours(args, rank, world, local_rank):
                        "l2": "inputs larger than L2 (about 0.36 GB of token tensors per step; no flush)"},
             "roofline": roofline, "hbm": hbm, "cpu_baseline": cpu,
             "e2e": {"value": job_tokens_per_s(Bt * L, world, e2e["ms"]), "unit": "tokens/s",
-                    "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"]},
+                    "h2d_bytes_per_step": e2e["h2d"], "d2h_bytes_per_step": e2e["d2h"],
+                    "readback": "the step's result: the parameter gradients (dA, dD of both directions)"},
+            "e2e_full_readback": {"value": job_tokens_per_s(Bt * L, world, e2e_full["ms"]), "unit": "tokens/s",
+                                  "h2d_bytes_per_step": e2e_full["h2d"], "d2h_bytes_per_step": e2e_full["d2h"],
+                                  "readback": "every output and every gradient (y_c, y_n and all 15 gradients)"},
             "gpu_launches": launches_per_step * args.steps, "clocks": clocks, "kernels": kernels}
     print(json.dumps(line), flush=True)
 
@@ -820,13 +856,15 @@ def run_prefill(args, L, Bs, calls):
         "bytes_per_call": blk_bytes}), flush=True)
 
 
-def run_e2e(lay, wl, stream, dev, args):
+def run_e2e(lay, wl, stream, dev, args, full_readback=False):
     """Forward + backward through the C ABI end to end: every step copies all
     of its inputs (both streams' x, dt, B, C and the upstream gradients) from
     pinned host memory to the device and reads the step's result back: the
     layer's parameter gradients (dA, dD of both directions), which is what a
     training step hands to its optimizer. The outputs and per-token gradients
-    stay on the device, where the neighbouring layers consume them. Copies run
+    stay on the device, where the neighbouring layers consume them; with
+    full_readback they are read back as well (y_c, y_n and every gradient),
+    the host-to-host reading of the same step. Copies run
     on their own streams and two device buffer sets alternate, so that step
     i+1's inputs go up and step i-1's result comes down while step i computes.
     The timed region covers all copies of every step."""
@@ -836,7 +874,10 @@ def run_e2e(lay, wl, stream, dev, args):
     lays[1].alloc_backward()
     ins = [k for k in wl.t32]
     host_in = {k: lay.t[k].detach().to("cpu").pin_memory() for k in ins}
-    outs = [[la.g[k] for k in ("A_f", "D_f", "A_r", "D_r")] for la in lays]
+    if full_readback:
+        outs = [[la.y_c, la.y_n] + [la.g[k] for k in la.g] for la in lays]
+    else:
+        outs = [[la.g[k] for k in ("A_f", "D_f", "A_r", "D_r")] for la in lays]
     host_out = [[torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs[0]] for _ in range(2)]
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
     d2h = sum(t.numel() * t.element_size() for t in host_out[0])

@@ -220,6 +220,34 @@ int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan
                         const bdscan_params* params, void* y_n, void* stream);
 
 /* ---------------------------------------------------------------------- */
+/* Timestep-modulated active block (Appendix E, AdaLN factorization,         */
+/* eq. cacheable-adaln): adaptive layer norm acts on the active block only,  */
+/* so the cached prefix state stays timestep-free.                          */
+/* ---------------------------------------------------------------------- */
+/* Modulation of one denoising step: shift, scale, gate [Bt][D] fp32 (the
+ * caller maps the timestep embedding e_t to them), eps of the layer norm. */
+typedef struct bdscan_adaln {
+  const float* shift;
+  const float* scale;
+  const float* gate;
+  float eps;
+} bdscan_adaln;
+
+/* Bt * block * 8 bytes: the per-token layer-norm statistics. */
+size_t bdscan_active_block_adaln_workspace_size(const bdscan_dims* dims);
+
+/* As bdscan_active_block, with noisy->x = h [Bt][Bs][D], the block's hidden
+ * input, normalised per token over the D channels (mean and biased variance;
+ * no affine of its own) and modulated, u = (1 + scale) LN(h) + shift. The
+ * block-restricted bidirectional scan runs on u from the read-only seed.
+ * Writes out [Bt][Bs][D] (out_dtype) = h + gate * y_n, the gated residual.
+ * Two launches: the statistics, then the scan. dt, B, C of the block are
+ * given by the caller; nothing here touches the seed or any other cache. */
+int bdscan_active_block_adaln(const bdscan_dims* dims, const float* seed, const bdscan_noisy* noisy,
+                              const bdscan_params* params, const bdscan_adaln* mod, void* out, void* workspace,
+                              size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------------- */
 /* Full-sequence bidirectional layer (Sec. 4: the fully bidirectional Mamba */
 /* denoiser of DiffuMamba, a forward scan and a reverse scan over the whole */
 /* sequence, which the block partial-reverse design replaces). A comparator */

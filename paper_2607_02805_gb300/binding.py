@@ -65,6 +65,10 @@ class bdscan_param_grads(ctypes.Structure):
     _fields_ = [("dA_f", c_void_p), ("dD_f", c_void_p), ("dA_r", c_void_p), ("dD_r", c_void_p)]
 
 
+class bdscan_adaln(ctypes.Structure):
+    _fields_ = [("shift", c_void_p), ("scale", c_void_p), ("gate", c_void_p), ("eps", ctypes.c_float)]
+
+
 # (name, restype, argtypes) of every exported function, in header order
 _P = ctypes.POINTER
 SIGNATURES = [
@@ -88,6 +92,10 @@ SIGNATURES = [
       c_void_p, ctypes.c_size_t, c_void_p]),
     ("bdscan_active_block", ctypes.c_int,
      [_P(bdscan_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
+    ("bdscan_active_block_adaln_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_active_block_adaln", ctypes.c_int,
+     [_P(bdscan_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), _P(bdscan_adaln), c_void_p, c_void_p,
+      ctypes.c_size_t, c_void_p]),
     ("bdscan_boundary_states_noalloc", ctypes.c_int,
      [_P(bdscan_dims), _P(bdscan_clean), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, ctypes.c_int, c_void_p]),
     ("bdscan_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
@@ -208,6 +216,15 @@ def bdscan_boundary_states(dims, clean, A_f, D_f, init_state, y_c, states, emit_
 def bdscan_active_block(dims, seed, noisy, params, y_n, stream):
     return load().bdscan_active_block(_ref(dims), seed, _ref(noisy), _ref(params),
                                       y_n, stream)
+
+
+def bdscan_active_block_adaln_workspace_size(dims) -> int:
+    return load().bdscan_active_block_adaln_workspace_size(_ref(dims))
+
+
+def bdscan_active_block_adaln(dims, seed, noisy, params, mod, out, workspace, workspace_bytes, stream):
+    return load().bdscan_active_block_adaln(_ref(dims), seed, _ref(noisy), _ref(params), _ref(mod), out,
+                                            workspace, workspace_bytes, stream)
 
 
 def bdscan_boundary_states_noalloc(dims, clean, A_f, D_f, init_state, y_c, states, emit_all, stream):
@@ -335,6 +352,15 @@ def boundary_states(dims, t, init_state, y_c, states, emit_all, workspace, strea
 def active_block(dims, seed, t, y_n, stream=None):
     _call("bdscan_active_block", ctypes.byref(dims), _ptr(seed), ctypes.byref(make_noisy(t)),
           ctypes.byref(make_params(t)), _ptr(y_n), _stream(stream))
+
+
+def active_block_adaln(dims, seed, t, shift, scale, gate, eps, out, workspace, stream=None):
+    """One timestep-modulated active block: t["x_n"] is the block's hidden input
+    h; out = h + gate * y_n of the modulated input."""
+    mod = bdscan_adaln(_ptr(shift), _ptr(scale), _ptr(gate), float(eps))
+    _call("bdscan_active_block_adaln", ctypes.byref(dims), _ptr(seed), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), ctypes.byref(mod), _ptr(out), _ptr(workspace),
+          0 if workspace is None else workspace.numel() * workspace.element_size(), _stream(stream))
 
 
 def full_bidir_forward(dims, t, y, workspace, stream=None):

@@ -369,6 +369,58 @@ int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan
   return ok();
 }
 
+size_t bdscan_active_block_adaln_workspace_size(const bdscan_dims* dims) {
+  Call c;
+  if (check_dims(dims, &c, "bdscan_active_block_adaln_workspace_size") != BDSCAN_OK) return 0;
+  return al256((size_t)c.g.Bt * c.g.L * sizeof(float2));
+}
+
+int bdscan_active_block_adaln(const bdscan_dims* dims, const float* seed, const bdscan_noisy* noisy,
+                              const bdscan_params* params, const bdscan_adaln* mod, void* out, void* workspace,
+                              size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_active_block_adaln";
+  Call c;
+  int rc = check_dims(dims, &c, fn);
+  if (rc) return rc;
+  if (dims->len != dims->block && dims->len != 0)
+    return fail(BDSCAN_ERR_ARG, "%s: len (%lld) must equal block (%lld)", fn, (long long)dims->len,
+                (long long)dims->block);
+  if ((rc = check_block_limits(c, false, fn))) return rc;
+  if (c.g.Bt == 0 || c.g.L == 0) return ok();
+  REQ(seed, fn, "seed");
+  if ((rc = check_noisy(noisy, fn)) || (rc = check_params(params, fn))) return rc;
+  if (mod == nullptr) return fail(BDSCAN_ERR_ARG, "%s: mod is NULL", fn);
+  REQ(mod->shift, fn, "mod.shift");
+  REQ(mod->scale, fn, "mod.scale");
+  REQ(mod->gate, fn, "mod.gate");
+  if (!(mod->eps >= 0.f)) return fail(BDSCAN_ERR_ARG, "%s: eps must be a non-negative number", fn);
+  REQ(out, fn, "out");
+  const size_t need = al256((size_t)c.g.Bt * c.g.L * sizeof(float2));
+  REQ(workspace, fn, "workspace");
+  if (workspace_bytes < need)
+    return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
+  cudaStream_t s = (cudaStream_t)stream;
+  bds::FwdParams p;
+  memset(&p, 0, sizeof(p));
+  p.g = c.g;
+  fill_noisy(p, noisy);
+  p.Af = params->A_f;
+  p.Df = params->D_f;
+  p.Ar = params->A_r;
+  p.Dr = params->D_r;
+  p.yn = out;
+  p.seed = seed;
+  p.shift = mod->shift;
+  p.scale = mod->scale;
+  p.gate = mod->gate;
+  p.ln_stats = (const float2*)workspace;
+  cudaError_t e = launched(
+      bds::launch_ln_stats(c.dt, noisy->x, c.g.Bt * c.g.L, c.g.D, mod->eps, (float2*)workspace, s), s);
+  if (e == cudaSuccess) e = launched(bds::launch_active_block_adaln(c.dt, c.N, p, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
 size_t bdscan_full_bidir_workspace_size(const bdscan_dims* dims) {
   Call c;
   if (check_dims(dims, &c, "bdscan_full_bidir_workspace_size") != BDSCAN_OK) return 0;

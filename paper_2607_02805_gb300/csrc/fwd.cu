@@ -309,9 +309,14 @@ struct ActiveLayout {
   static __host__ __device__ size_t bytes(int Bs) {
     return td_bytes(Bs) + raw_bytes(Bs) + rows_bytes(Bs) + (size_t)2 * Bs * kActW * 4;
   }
+  // with adaptive layer norm: the modulated input [Bs][32] fp32 after the outputs
+  static __host__ __device__ size_t bytes_ada(int Bs) { return bytes(Bs) + (size_t)Bs * kActW * 4; }
 };
 
-template <typename T, typename TO, int N>
+// ADA: adaptive layer norm on the block (Appendix E, eq. cacheable-adaln):
+// the scans read u = (1 + scale) (x - mean) rstd + shift instead of x, and
+// the output is x + gate * y_n. The seed, the cache, is never modulated.
+template <typename T, typename TO, int N, bool ADA = false>
 __global__ void __launch_bounds__(2 * kActW, 1) k_active_block(const FwdParams p) {
   using Ly = ActiveLayout<T, N>;
   extern __shared__ __align__(16) unsigned char smem[];
@@ -364,23 +369,41 @@ __global__ void __launch_bounds__(2 * kActW, 1) k_active_block(const FwdParams p
       reinterpret_cast<float2*>(rows)[q] = make_float2(cvt(raw[2 * q]), cvt(raw[2 * q + 1]));
     __syncthreads();
   }
+  float* xmod = ybuf + (size_t)2 * Bs * kActW;  // [Bs][32], ADA only
+  if (ADA) {
+    for (int q = threadIdx.x; q < Bs * kActW; q += 2 * kActW) {
+      const int i = q / kActW, c = q - i * kActW;
+      const int64_t dc = d0 + c;
+      float u = 0.f;
+      if (dc < g.D) {
+        const float2 st = p.ln_stats[b * Bs + i];
+        const float z = __fmul_rn(__fsub_rn(cvt(td[q]), st.x), st.y);
+        u = __fmaf_rn(__fadd_rn(1.f, p.scale[b * g.D + dc]), z, p.shift[b * g.D + dc]);
+      }
+      xmod[q] = u;
+    }
+    __syncthreads();
+  }
+  // this lane's input at token i: x as stored, or the modulated input
+  auto xin = [&](int i) { return ADA ? xmod[i * kActW + lane] : cvt(td[i * kActW + lane]); };
 
   const T* xs = td;
   const T* dts = td + (size_t)(1 + dir) * Bs * kActW;
   const float* Brow = rows + (size_t)(2 * dir) * Bs * N;
   const float* Crow = Brow + (size_t)Bs * N;
   float* yb = ybuf + (size_t)dir * Bs * kActW;
+  (void)xs;
   if (dir == 0) {
 #pragma unroll 4
     for (int i = 0; i < Bs; ++i) {
-      const float x = cvt(xs[i * kActW + lane]), dt = cvt(dts[i * kActW + lane]);
+      const float x = xin(i), dt = cvt(dts[i * kActW + lane]);
       const float y = scan_step<N>(h, A2, dt, x, Brow + i * N, Crow + i * N);
       yb[i * kActW + lane] = with_skip(y, Dd, x);
     }
   } else {
 #pragma unroll 4
     for (int i = Bs - 1; i >= 0; --i) {
-      const float x = cvt(xs[i * kActW + lane]), dt = cvt(dts[i * kActW + lane]);
+      const float x = xin(i), dt = cvt(dts[i * kActW + lane]);
       const float y = scan_step<N>(h, A2, dt, x, Brow + i * N, Crow + i * N);
       yb[i * kActW + lane] = with_skip(y, Dd, x);
     }
@@ -388,10 +411,36 @@ __global__ void __launch_bounds__(2 * kActW, 1) k_active_block(const FwdParams p
   __syncthreads();
   for (int q = threadIdx.x; q < Bs * kActW; q += 2 * kActW) {
     const int i = q / kActW, c = q - i * kActW;
-    if (d0 + c < g.D)
-      reinterpret_cast<TO*>(p.yn)[(row0 + i) * g.D + d0 + c] =
-          to_out<TO>(combine_dirs(ybuf[q], ybuf[(size_t)Bs * kActW + q]));
+    if (d0 + c < g.D) {
+      const float yv = combine_dirs(ybuf[q], ybuf[(size_t)Bs * kActW + q]);
+      // gated residual of the modulated step: x + gate * y_n
+      const float o = ADA ? __fmaf_rn(p.gate[b * g.D + d0 + c], yv, cvt(td[q])) : yv;
+      reinterpret_cast<TO*>(p.yn)[(row0 + i) * g.D + d0 + c] = to_out<TO>(o);
+    }
   }
+}
+
+// Layer-norm statistics of each token (one warp per row of D elements): the
+// mean, then 1/sqrt(var + eps) from the centred second moment, in fp32.
+template <typename T>
+__global__ void __launch_bounds__(256) k_ln_stats(const T* h, int64_t rows, int64_t D, float eps, float2* stats) {
+  const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const T* r = h + row * D;
+  float s = 0.f;
+  for (int64_t i = lane; i < D; i += 32) s = __fadd_rn(s, cvt(r[i]));
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) s = __fadd_rn(s, __shfl_xor_sync(0xffffffffu, s, o));
+  const float mu = __fdiv_rn(s, (float)D);
+  float v = 0.f;
+  for (int64_t i = lane; i < D; i += 32) {
+    const float e = __fsub_rn(cvt(r[i]), mu);
+    v = __fmaf_rn(e, e, v);
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+  if (lane == 0) stats[row] = make_float2(mu, __fdiv_rn(1.f, __fsqrt_rn(__fadd_rn(__fdiv_rn(v, (float)D), eps))));
 }
 
 // ---------------------------------------------------------------------------
@@ -483,15 +532,16 @@ cudaError_t block_scan_mode(int mode, int nchunks, const FwdParams& p, cudaStrea
   }
 }
 
-template <typename T, typename TO, int N>
+template <typename T, typename TO, int N, bool ADA = false>
 cudaError_t active_block_t(const FwdParams& p, cudaStream_t s) {
-  const size_t smem = ActiveLayout<T, N>::bytes((int)p.g.Bs);
+  const size_t smem = ADA ? ActiveLayout<T, N>::bytes_ada((int)p.g.Bs) : ActiveLayout<T, N>::bytes((int)p.g.Bs);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(k_active_block<T, TO, N>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(k_active_block<T, TO, N, ADA>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
   dim3 grid((unsigned)((p.g.D + kActW - 1) / kActW), (unsigned)p.g.Bt);
-  k_active_block<T, TO, N><<<grid, 2 * kActW, smem, s>>>(p);
+  k_active_block<T, TO, N, ADA><<<grid, 2 * kActW, smem, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -535,6 +585,25 @@ cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t 
     case 1: BDS_DISPATCH_N(N, return active_block_t<bf16, bf16, NN>(p, s);)
     default: BDS_DISPATCH_N(N, return active_block_t<bf16, float, NN>(p, s);)
   }
+}
+
+cudaError_t launch_active_block_adaln(int dt, int N, const FwdParams& p, cudaStream_t s) {
+  if (p.g.Bt == 0 || p.g.D == 0) return cudaSuccess;
+  switch (dt) {
+    case 0: BDS_DISPATCH_N(N, return active_block_t<float, float, NN, true>(p, s);)
+    case 1: BDS_DISPATCH_N(N, return active_block_t<bf16, bf16, NN, true>(p, s);)
+    default: BDS_DISPATCH_N(N, return active_block_t<bf16, float, NN, true>(p, s);)
+  }
+}
+
+cudaError_t launch_ln_stats(int dt, const void* h, int64_t rows, int64_t D, float eps, float2* stats, cudaStream_t s) {
+  if (rows == 0) return cudaSuccess;
+  const unsigned blocks = (unsigned)((rows + 7) / 8);
+  if (dt == 0)
+    k_ln_stats<float><<<blocks, 256, 0, s>>>(reinterpret_cast<const float*>(h), rows, D, eps, stats);
+  else
+    k_ln_stats<bf16><<<blocks, 256, 0, s>>>(reinterpret_cast<const bf16*>(h), rows, D, eps, stats);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_combine(int out_f32, const float* yf, const float* yr, void* y, int64_t n, cudaStream_t s) {

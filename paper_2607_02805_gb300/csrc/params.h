@@ -36,6 +36,10 @@ struct FwdParams {
   int c_begin;         // first chunk handled by a block-scan launch
   int stage_bufs;      // block scan: 2 = copy the next block while computing, 1 = synchronous
   int rev;             // chunk-local scan: right to left in time (with block-scan mode 2)
+  // active block with adaptive layer norm: per batch row shift, scale, gate
+  // [Bt][D] and per token (mean, 1/sqrt(var + eps)) of the block's input
+  const float *shift, *scale, *gate;
+  const float2* ln_stats;
 };
 
 // Backward-side kernels.
@@ -67,6 +71,11 @@ cudaError_t launch_chunk_carry(int N, const FwdParams& p, cudaStream_t s);
 cudaError_t launch_block_scan(int dt, int N, int mode, int nchunks, const FwdParams& p, cudaStream_t s);
 // One noisy block per batch row from p.seed (len == block).
 cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t s);
+// Per-token layer-norm statistics of rows x D elements (dt: 0 f32, else bf16).
+cudaError_t launch_ln_stats(int dt, const void* h, int64_t rows, int64_t D, float eps, float2* stats, cudaStream_t s);
+// The active block on the modulated input (1 + scale) LN(x) + shift, writing
+// x + gate * y_n (p.shift, p.scale, p.gate, p.ln_stats set).
+cudaError_t launch_active_block_adaln(int dt, int N, const FwdParams& p, cudaStream_t s);
 // y = yf + yr elementwise (n elements, a multiple of 4), rounded to f32 or bf16.
 cudaError_t launch_combine(int out_f32, const float* yf, const float* yr, void* y, int64_t n, cudaStream_t s);
 cudaError_t launch_bwd_noisy(int dt, int N, const BwdParams& p, cudaStream_t s);

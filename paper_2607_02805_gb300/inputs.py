@@ -15,6 +15,9 @@ layer, with the value ranges of a Mamba-1 style parameterisation):
 * A = -exp(U[ln 1, ln 16])          per channel and state index, [D, N], fp32
 * D ~ N(0, 0.1)                     per channel, [D], fp32 (0.1 is the std)
 * upstream gradients dy ~ N(0, 1)   [Bt, L, D]; dstates ~ N(0, 1) if used
+* timestep modulation of an active block (adaptive layer norm): shift,
+  scale ~ N(0, 0.3) and gate ~ N(1, 0.3) per batch row and channel, [Bt, D],
+  fp32; a separate draw (`part`) per denoising step
 
 Every tensor has its own stream id; the generator for tensor ``name`` is
 ``numpy.random.Generator(PCG64(SeedSequence([seed, stream_id])))``. Values are
@@ -36,6 +39,7 @@ STREAM_IDS = {
     "dt_r": 8, "B_r": 9, "C_r": 10,
     "A_f": 11, "D_f": 12, "A_r": 13, "D_r": 14,
     "dy_c": 15, "dy_n": 16, "dstates": 17, "init_state": 18,
+    "shift": 19, "scale": 20, "gate": 21,
 }
 
 TOKEN_D = ("x_c", "dt_c", "x_n", "dt_f", "dt_r")       # [Bt, L, D]
@@ -87,6 +91,10 @@ def draw(name: str, shape, seed: int, part: int = 0) -> np.ndarray:
         return (-np.exp(u)).astype(np.float32)
     if name in ("D_f", "D_r"):
         return g.normal(0.0, 0.1, size=shape).astype(np.float32)
+    if name in ("shift", "scale"):
+        return g.normal(0.0, 0.3, size=shape).astype(np.float32)
+    if name == "gate":
+        return g.normal(1.0, 0.3, size=shape).astype(np.float32)
     raise KeyError(name)
 
 

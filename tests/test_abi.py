@@ -130,6 +130,26 @@ def test_active_block_needs_one_block():
     assert rc == binding.BDSCAN_ERR_ARG and "must equal block" in binding.bdscan_last_error()
 
 
+def test_active_block_adaln_checks():
+    d = _dims(length=16, block=16)
+    _, n, p = _structs()
+    nbytes = binding.bdscan_active_block_adaln_workspace_size(d)
+    assert nbytes >= d.batch * 16 * 8 and nbytes % 256 == 0
+    mod = binding.bdscan_adaln(FAKE, FAKE, FAKE, 1e-5)
+    rc = binding.bdscan_active_block_adaln(_dims(length=32, block=16), FAKE, n, p, mod, FAKE, FAKE, 1 << 20, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "must equal block" in binding.bdscan_last_error()
+    rc = binding.bdscan_active_block_adaln(d, FAKE, n, p, None, FAKE, FAKE, 1 << 20, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "mod is NULL" in binding.bdscan_last_error()
+    bad = binding.bdscan_adaln(FAKE, None, FAKE, 1e-5)
+    rc = binding.bdscan_active_block_adaln(d, FAKE, n, p, bad, FAKE, FAKE, 1 << 20, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "mod.scale is NULL" in binding.bdscan_last_error()
+    neg = binding.bdscan_adaln(FAKE, FAKE, FAKE, -1.0)
+    rc = binding.bdscan_active_block_adaln(d, FAKE, n, p, neg, FAKE, FAKE, 1 << 20, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "eps" in binding.bdscan_last_error()
+    rc = binding.bdscan_active_block_adaln(d, FAKE, n, p, mod, FAKE, FAKE, nbytes - 1, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "workspace" in binding.bdscan_last_error()
+
+
 def test_boundary_states_checks():
     d = _dims()
     c, _, _ = _structs()
