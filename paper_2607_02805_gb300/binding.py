@@ -65,6 +65,14 @@ class bdscan_param_grads(ctypes.Structure):
     _fields_ = [("dA_f", c_void_p), ("dD_f", c_void_p), ("dA_r", c_void_p), ("dD_r", c_void_p)]
 
 
+class bdscan_mixer_params(ctypes.Structure):
+    _fields_ = [("conv_w", c_void_p), ("conv_b", c_void_p), ("dt_bias_f", c_void_p), ("dt_bias_r", c_void_p)]
+
+
+class bdscan_mixer_grads(ctypes.Structure):
+    _fields_ = [("dconv_w", c_void_p), ("dconv_b", c_void_p), ("ddt_bias_f", c_void_p), ("ddt_bias_r", c_void_p)]
+
+
 class bdscan_adaln(ctypes.Structure):
     _fields_ = [("shift", c_void_p), ("scale", c_void_p), ("gate", c_void_p), ("eps", ctypes.c_float)]
 
@@ -101,6 +109,24 @@ SIGNATURES = [
     ("bdscan_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
     ("bdscan_full_bidir_forward", ctypes.c_int,
      [_P(bdscan_dims), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_mixer_forward_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_mixer_forward", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_clean), c_void_p, _P(bdscan_noisy), c_void_p, _P(bdscan_params),
+      _P(bdscan_mixer_params), c_void_p, c_void_p, c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_mixer_backward_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_mixer_backward", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_clean), c_void_p, _P(bdscan_noisy), c_void_p, _P(bdscan_params),
+      _P(bdscan_mixer_params), c_void_p, c_void_p, c_void_p, _P(bdscan_clean_grads), c_void_p,
+      _P(bdscan_noisy_grads), c_void_p, _P(bdscan_param_grads), _P(bdscan_mixer_grads), c_void_p, ctypes.c_size_t,
+      c_void_p]),
+    ("bdscan_mixer_boundary_states_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_mixer_boundary_states", ctypes.c_int,
+     [_P(bdscan_dims), _P(bdscan_clean), c_void_p, c_void_p, c_void_p, _P(bdscan_mixer_params), c_void_p, c_void_p,
+      c_void_p, c_void_p, c_void_p, ctypes.c_int, c_void_p, ctypes.c_size_t, c_void_p]),
+    ("bdscan_mixer_active_block_workspace_size", ctypes.c_size_t, [_P(bdscan_dims)]),
+    ("bdscan_mixer_active_block", ctypes.c_int,
+     [_P(bdscan_dims), c_void_p, c_void_p, _P(bdscan_noisy), c_void_p, _P(bdscan_params), _P(bdscan_mixer_params),
+      c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
     ("bdscan_ssd_forward_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
     ("bdscan_ssd_forward", ctypes.c_int,
      [_P(bdscan_ssd_dims), _P(bdscan_clean), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, c_void_p,
@@ -239,6 +265,48 @@ def bdscan_full_bidir_workspace_size(dims) -> int:
 def bdscan_full_bidir_forward(dims, noisy, params, y, workspace, workspace_bytes, stream):
     return load().bdscan_full_bidir_forward(_ref(dims), _ref(noisy), _ref(params), y, workspace,
                                             workspace_bytes, stream)
+
+
+def bdscan_mixer_forward_workspace_size(dims) -> int:
+    return load().bdscan_mixer_forward_workspace_size(_ref(dims))
+
+
+def bdscan_mixer_forward(dims, clean, z_c, noisy, z_n, params, mparams, out_c, out_n, states, workspace,
+                         workspace_bytes, stream):
+    return load().bdscan_mixer_forward(_ref(dims), _ref(clean), z_c, _ref(noisy), z_n, _ref(params), _ref(mparams),
+                                       out_c, out_n, states, workspace, workspace_bytes, stream)
+
+
+def bdscan_mixer_backward_workspace_size(dims) -> int:
+    return load().bdscan_mixer_backward_workspace_size(_ref(dims))
+
+
+def bdscan_mixer_backward(dims, clean, z_c, noisy, z_n, params, mparams, dout_c, dout_n, dstates, gclean, dz_c,
+                          gnoisy, dz_n, gparams, gmparams, workspace, workspace_bytes, stream):
+    return load().bdscan_mixer_backward(_ref(dims), _ref(clean), z_c, _ref(noisy), z_n, _ref(params), _ref(mparams),
+                                        dout_c, dout_n, dstates, _ref(gclean), dz_c, _ref(gnoisy), dz_n,
+                                        _ref(gparams), _ref(gmparams), workspace, workspace_bytes, stream)
+
+
+def bdscan_mixer_boundary_states_workspace_size(dims) -> int:
+    return load().bdscan_mixer_boundary_states_workspace_size(_ref(dims))
+
+
+def bdscan_mixer_boundary_states(dims, clean, z_c, A_f, D_f, mparams, init_state, conv_init, out_c, states,
+                                 conv_states, emit_all, workspace, workspace_bytes, stream):
+    return load().bdscan_mixer_boundary_states(_ref(dims), _ref(clean), z_c, A_f, D_f, _ref(mparams), init_state,
+                                               conv_init, out_c, states, conv_states, int(emit_all), workspace,
+                                               workspace_bytes, stream)
+
+
+def bdscan_mixer_active_block_workspace_size(dims) -> int:
+    return load().bdscan_mixer_active_block_workspace_size(_ref(dims))
+
+
+def bdscan_mixer_active_block(dims, seed, conv_seed, noisy, z_n, params, mparams, out_n, workspace, workspace_bytes,
+                              stream):
+    return load().bdscan_mixer_active_block(_ref(dims), seed, conv_seed, _ref(noisy), z_n, _ref(params),
+                                            _ref(mparams), out_n, workspace, workspace_bytes, stream)
 
 
 def bdscan_ssd_forward_workspace_size(dims) -> int:
@@ -404,3 +472,56 @@ def ssd_full_bidir_forward(dims, t, y, workspace, stream=None):
     tensors in t; y [Bt][L][H][64]."""
     _call("bdscan_ssd_full_bidir_forward", ctypes.byref(dims), ctypes.byref(make_noisy(t)),
           ctypes.byref(make_params(t)), _ptr(y), _ptr(workspace), _nbytes(workspace), _stream(stream))
+
+
+# ---------------------------------------------------------------------------
+# mixer (include/bdscan_mixer.h): tensors keyed xr_c, dtr_c, B_c, C_c, z_c,
+# xr_n, dtr_f, B_f, C_f, dtr_r, B_r, C_r, z_n, A_f, D_f, A_r, D_r, conv_w,
+# conv_b, dt_bias_f, dt_bias_r
+# ---------------------------------------------------------------------------
+def make_mixer_params(t):
+    return bdscan_mixer_params(_ptr(t["conv_w"]), _ptr(t["conv_b"]), _ptr(t["dt_bias_f"]), _ptr(t["dt_bias_r"]))
+
+
+def _mix_clean(t):
+    return bdscan_clean(_ptr(t["xr_c"]), _ptr(t["dtr_c"]), _ptr(t["B_c"]), _ptr(t["C_c"]))
+
+
+def _mix_noisy(t):
+    return bdscan_noisy(_ptr(t["xr_n"]), _ptr(t["dtr_f"]), _ptr(t["B_f"]), _ptr(t["C_f"]), _ptr(t["dtr_r"]),
+                        _ptr(t["B_r"]), _ptr(t["C_r"]))
+
+
+def mixer_forward(dims, t, out_c, out_n, states, workspace, stream=None):
+    _call("bdscan_mixer_forward", ctypes.byref(dims), ctypes.byref(_mix_clean(t)), _ptr(t["z_c"]),
+          ctypes.byref(_mix_noisy(t)), _ptr(t["z_n"]), ctypes.byref(make_params(t)),
+          ctypes.byref(make_mixer_params(t)), _ptr(out_c), _ptr(out_n), _ptr(states), _ptr(workspace),
+          _nbytes(workspace), _stream(stream))
+
+
+def mixer_backward(dims, t, dout_c, dout_n, dstates, g, workspace, stream=None):
+    """g: gradient tensors keyed like t (xr_c ... z_n, A_f ... dt_bias_r)."""
+    gc = bdscan_clean_grads(_ptr(g["xr_c"]), _ptr(g["dtr_c"]), _ptr(g["B_c"]), _ptr(g["C_c"]))
+    gn = bdscan_noisy_grads(_ptr(g["xr_n"]), _ptr(g["dtr_f"]), _ptr(g["B_f"]), _ptr(g["C_f"]), _ptr(g["dtr_r"]),
+                            _ptr(g["B_r"]), _ptr(g["C_r"]))
+    gp = bdscan_param_grads(_ptr(g["A_f"]), _ptr(g["D_f"]), _ptr(g["A_r"]), _ptr(g["D_r"]))
+    gm = bdscan_mixer_grads(_ptr(g["conv_w"]), _ptr(g["conv_b"]), _ptr(g["dt_bias_f"]), _ptr(g["dt_bias_r"]))
+    _call("bdscan_mixer_backward", ctypes.byref(dims), ctypes.byref(_mix_clean(t)), _ptr(t["z_c"]),
+          ctypes.byref(_mix_noisy(t)), _ptr(t["z_n"]), ctypes.byref(make_params(t)),
+          ctypes.byref(make_mixer_params(t)), _ptr(dout_c), _ptr(dout_n), _ptr(dstates), ctypes.byref(gc),
+          _ptr(g["z_c"]), ctypes.byref(gn), _ptr(g["z_n"]), ctypes.byref(gp), ctypes.byref(gm), _ptr(workspace),
+          _nbytes(workspace), _stream(stream))
+
+
+def mixer_boundary_states(dims, t, init_state, conv_init, out_c, states, conv_states, emit_all, workspace,
+                          stream=None):
+    _call("bdscan_mixer_boundary_states", ctypes.byref(dims), ctypes.byref(_mix_clean(t)),
+          _ptr(t["z_c"]) if out_c is not None else None, _ptr(t["A_f"]), _ptr(t["D_f"]),
+          ctypes.byref(make_mixer_params(t)), _ptr(init_state), _ptr(conv_init), _ptr(out_c), _ptr(states),
+          _ptr(conv_states), int(emit_all), _ptr(workspace), _nbytes(workspace), _stream(stream))
+
+
+def mixer_active_block(dims, seed, conv_seed, t, out_n, workspace, stream=None):
+    _call("bdscan_mixer_active_block", ctypes.byref(dims), _ptr(seed), _ptr(conv_seed), ctypes.byref(_mix_noisy(t)),
+          _ptr(t["z_n"]), ctypes.byref(make_params(t)), ctypes.byref(make_mixer_params(t)), _ptr(out_n),
+          _ptr(workspace), _nbytes(workspace), _stream(stream))

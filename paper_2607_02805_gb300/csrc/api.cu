@@ -317,25 +317,7 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
   p.init = init_state;
   p.hst = (float*)workspace;
   p.sdt = (float*)((char*)workspace + al256((size_t)c.g.Bt * (c.g.nc + 1) * c.g.D * c.N * 4));
-  if ((rc = run_chunk_states(c, p, s, fn))) return rc;
-  cudaError_t e = cudaSuccess;
-  if (emit_all || y_c != nullptr) {
-    p.emit_all = emit_all ? 1 : 0;
-    p.states = emit_all ? states : nullptr;
-    p.final_state = emit_all ? nullptr : states;
-    e = launched(bds::launch_block_scan(c.dt, c.N, 1, c.g.nc, p, s), s);
-  } else if (c.g.nc_full == c.g.nc) {
-    // the state after the last chunk is the carry kernel's final value
-    const size_t row = (size_t)c.g.D * c.N * 4;
-    e = cudaMemcpy2DAsync(states, row, p.hst + (size_t)c.g.nc * c.g.D * c.N, (size_t)(c.g.nc + 1) * row, row,
-                          (size_t)c.g.Bt, cudaMemcpyDeviceToDevice, s);
-  } else {
-    // a partial last chunk: rescan it from its start state
-    p.emit_all = 0;
-    p.final_state = states;
-    p.c_begin = c.g.nc - 1;
-    e = launched(bds::launch_block_scan(c.dt, c.N, 1, 1, p, s), s);
-  }
+  cudaError_t e = bds::api_run_boundary(c.dt, c.N, p, states, emit_all, s);
   if (e != cudaSuccess) return cuda_fail(e, fn);
   return ok();
 }
@@ -516,13 +498,8 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
   REQ(workspace, fn, "workspace");
   if (workspace_bytes < need)
     return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
-  bds::Geo gb = c.g;  // the backward's own chunking of each batch row
-  gb.nc = bds::bwd_chunk_count(c.dt, c.N, c.g);
-  const BwdWs w = bwd_ws(gb, c.N);
-
   bds::BwdParams p;
   memset(&p, 0, sizeof(p));
-  p.g = gb;
   p.xc = clean->x;
   p.dtc = clean->dt;
   p.Bc = clean->B;
@@ -557,19 +534,8 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
   p.dDf = gparams->dD_f;
   p.dAr = gparams->dA_r;
   p.dDr = gparams->dD_r;
-  char* ws = (char*)workspace;
-  p.dS = (float*)(ws + w.dS);
-  p.Lc = (float*)(ws + w.Lc);
-  p.sdtc = (float*)(ws + w.sdtc);
-  p.part_tok = (float*)(ws + w.part_tok);
-  p.part_A = (float*)(ws + w.part_A);
-  p.part_D = (float*)(ws + w.part_D);
-
-  cudaError_t e = launched(bds::launch_bwd_noisy(c.dt, c.N, p, s), s);
-  if (e == cudaSuccess) e = launched(bds::launch_bwd_carry(c.N, p, s), s);
-  if (e == cudaSuccess) e = launched(bds::launch_bwd_clean(c.dt, c.N, p, s), s);
-  if (e == cudaSuccess) e = launched(bds::launch_bwd_reduce_tok(c.dt, c.N, p, s), s);
-  if (e == cudaSuccess) e = launched(bds::launch_bwd_reduce_par(c.N, p, s), s);
+  p.g = c.g;
+  cudaError_t e = bds::api_run_backward(c.dt, c.N, p, workspace, s);
   if (e != cudaSuccess) return cuda_fail(e, fn);
   return ok();
 }
@@ -646,5 +612,74 @@ int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char
 }
 
 size_t api_fwd_workspace(const Geo& g, int N) { return fwd_ws(g, N); }
+
+size_t api_bwd_workspace(const Geo& g, int N) {
+  Geo gm = g;
+  gm.nc = bwd_max_chunks(g);
+  return bwd_ws(gm, N).total;
+}
+
+// The cache build's launches with p's clean tensors, hst/sdt (the workspace)
+// and init set: every block-end state or the final one into `states`, and
+// p.yc if set.
+cudaError_t api_run_boundary(int dt, int N, FwdParams& p, float* states, int emit_all, cudaStream_t s) {
+  const Geo& g = p.g;
+  cudaError_t e = cudaSuccess;
+  if (g.nc_full > 0) e = launched(launch_chunk_local(dt, N, p, s), s);
+  if (e == cudaSuccess) e = launched(launch_chunk_carry(N, p, s), s);
+  if (e != cudaSuccess) return e;
+  if (emit_all || p.yc != nullptr) {
+    p.emit_all = emit_all ? 1 : 0;
+    p.states = emit_all ? states : nullptr;
+    p.final_state = emit_all ? nullptr : states;
+    return launched(launch_block_scan(dt, N, 1, g.nc, p, s), s);
+  }
+  if (g.nc_full == g.nc) {
+    // the state after the last chunk is the carry kernel's final value
+    const size_t row = (size_t)g.D * N * 4;
+    return cudaMemcpy2DAsync(states, row, p.hst + (size_t)g.nc * g.D * N, (size_t)(g.nc + 1) * row, row,
+                             (size_t)g.Bt, cudaMemcpyDeviceToDevice, s);
+  }
+  // a partial last chunk: rescan it from its start state
+  p.emit_all = 0;
+  p.final_state = states;
+  p.c_begin = g.nc - 1;
+  return launched(launch_block_scan(dt, N, 1, 1, p, s), s);
+}
+
+// The all-block forward's launches (chunk-local scan, chunk carry, block
+// scan) with p's tensors set; the workspace holds the chunk states.
+cudaError_t api_run_forward(int dt, int N, FwdParams& p, void* workspace, cudaStream_t s) {
+  p.hst = (float*)workspace;
+  p.sdt = (float*)((char*)workspace + al256((size_t)p.g.Bt * (p.g.nc + 1) * p.g.D * N * 4));
+  p.emit_all = 1;
+  cudaError_t e = cudaSuccess;
+  if (p.g.nc_full > 0) e = launched(launch_chunk_local(dt, N, p, s), s);
+  if (e == cudaSuccess) e = launched(launch_chunk_carry(N, p, s), s);
+  if (e == cudaSuccess) e = launched(launch_block_scan(dt, N, 0, p.g.nc, p, s), s);
+  return e;
+}
+
+// The backward's launches with p's tensors set (p.g the forward geometry):
+// its own chunking of each batch row, the workspace layout, five kernels.
+cudaError_t api_run_backward(int dt, int N, BwdParams& p, void* workspace, cudaStream_t s) {
+  Geo gb = p.g;
+  gb.nc = bwd_chunk_count(dt, N, p.g);
+  const BwdWs w = bwd_ws(gb, N);
+  p.g = gb;
+  char* ws = (char*)workspace;
+  p.dS = (float*)(ws + w.dS);
+  p.Lc = (float*)(ws + w.Lc);
+  p.sdtc = (float*)(ws + w.sdtc);
+  p.part_tok = (float*)(ws + w.part_tok);
+  p.part_A = (float*)(ws + w.part_A);
+  p.part_D = (float*)(ws + w.part_D);
+  cudaError_t e = launched(launch_bwd_noisy(dt, N, p, s), s);
+  if (e == cudaSuccess) e = launched(launch_bwd_carry(N, p, s), s);
+  if (e == cudaSuccess) e = launched(launch_bwd_clean(dt, N, p, s), s);
+  if (e == cudaSuccess) e = launched(launch_bwd_reduce_tok(dt, N, p, s), s);
+  if (e == cudaSuccess) e = launched(launch_bwd_reduce_par(N, p, s), s);
+  return e;
+}
 
 }  // namespace bds

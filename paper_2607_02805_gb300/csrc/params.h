@@ -94,6 +94,12 @@ cudaError_t set_smem_cached(const void* fn, int bytes, int carveout);  // carveo
 int sm_count_cached();  // 0 if unknown
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn);
 size_t api_fwd_workspace(const Geo& g, int N);
+size_t api_bwd_workspace(const Geo& g, int N);
+// Launch sequences of bdscan_forward / bdscan_backward (counted by the
+// launch hook) for other entry points of the library.
+cudaError_t api_run_forward(int dt, int N, FwdParams& p, void* workspace, cudaStream_t s);
+cudaError_t api_run_boundary(int dt, int N, FwdParams& p, float* states, int emit_all, cudaStream_t s);
+cudaError_t api_run_backward(int dt, int N, BwdParams& p, void* workspace, cudaStream_t s);
 int bwd_chunk_count(int dt, int N, const Geo& g);
 // Upper bound of the backward's chunks per batch row (sizes its workspace
 // independently of the device): twice the forward chunking, at most one

@@ -15,6 +15,10 @@ layer, with the value ranges of a Mamba-1 style parameterisation):
 * A = -exp(U[ln 1, ln 16])          per channel and state index, [D, N], fp32
 * D ~ N(0, 0.1)                     per channel, [D], fp32 (0.1 is the std)
 * upstream gradients dy ~ N(0, 1)   [Bt, L, D]; dstates ~ N(0, 1) if used
+* mixer around the scan (raw projections before the convolution, softplus
+  and gate): xr ~ N(0, 1), dt_raw ~ N(-2, 0.5), z ~ N(0, 1) per token and
+  channel; convolution taps ~ N(0, 0.5) [D, 4], convolution bias and both
+  step-size biases ~ N(0, 0.1) [D]
 * timestep modulation of an active block (adaptive layer norm): shift,
   scale ~ N(0, 0.3) and gate ~ N(1, 0.3) per batch row and channel, [Bt, D],
   fp32; a separate draw (`part`) per denoising step
@@ -40,6 +44,8 @@ STREAM_IDS = {
     "A_f": 11, "D_f": 12, "A_r": 13, "D_r": 14,
     "dy_c": 15, "dy_n": 16, "dstates": 17, "init_state": 18,
     "shift": 19, "scale": 20, "gate": 21,
+    "xr_c": 22, "xr_n": 23, "dtr_c": 24, "dtr_f": 25, "dtr_r": 26, "z_c": 27, "z_n": 28,
+    "conv_w": 29, "conv_b": 30, "dt_bias_f": 31, "dt_bias_r": 32,
 }
 
 TOKEN_D = ("x_c", "dt_c", "x_n", "dt_f", "dt_r")       # [Bt, L, D]
@@ -90,6 +96,14 @@ def draw(name: str, shape, seed: int, part: int = 0) -> np.ndarray:
         u = g.uniform(np.log(1.0), np.log(16.0), size=shape)
         return (-np.exp(u)).astype(np.float32)
     if name in ("D_f", "D_r"):
+        return g.normal(0.0, 0.1, size=shape).astype(np.float32)
+    if name in ("xr_c", "xr_n", "z_c", "z_n"):
+        return g.standard_normal(shape, dtype=np.float32)
+    if name in ("dtr_c", "dtr_f", "dtr_r"):
+        return g.normal(-2.0, 0.5, size=shape).astype(np.float32)
+    if name == "conv_w":
+        return g.normal(0.0, 0.5, size=shape).astype(np.float32)
+    if name in ("conv_b", "dt_bias_f", "dt_bias_r"):
         return g.normal(0.0, 0.1, size=shape).astype(np.float32)
     if name in ("shift", "scale"):
         return g.normal(0.0, 0.3, size=shape).astype(np.float32)
@@ -176,3 +190,48 @@ class SsdWorkload(Workload):
             if k not in PARAMS and k != "init_state":
                 a = bf16_bits_to_f32(f32_to_bf16_bits(a)).reshape(shp)
             self.t32[k] = a
+
+
+MIXER_PARAMS = ("A_f", "D_f", "A_r", "D_r", "conv_w", "conv_b", "dt_bias_f", "dt_bias_r")
+
+
+class MixerWorkload(Workload):
+    """A seeded problem instance of the mixer around the scan: the raw inputs
+    xr, dt_raw and gates z of both streams ([Bt, L, D]), B and C ([Bt, L, N]),
+    the scan parameters and the convolution and step-size parameters (fp32),
+    and the upstream gradients dout (drawn like dy) of both streams."""
+
+    TOKEN = ("xr_c", "dtr_c", "z_c", "xr_n", "dtr_f", "dtr_r", "z_n")
+
+    def __init__(self, batch, length, block, d_inner, d_state, dtype="bf16", seed=0, with_grads=True,
+                 parts=("clean", "noisy"), part=0, with_init=False):
+        if dtype not in ("bf16", "f32"):
+            raise ValueError(dtype)
+        self.batch, self.len, self.block = int(batch), int(length), int(block)
+        self.d_inner, self.d_state, self.dtype, self.seed = int(d_inner), int(d_state), dtype, int(seed)
+        Bt, L, D, N = self.batch, self.len, self.d_inner, self.d_state
+        shapes = {}
+        for k in self.TOKEN:
+            if ("clean" in parts and k.endswith("_c")) or ("noisy" in parts and not k.endswith("_c")):
+                shapes[k] = (Bt, L, D)
+        for k in TOKEN_N:
+            if ("clean" in parts and k.endswith("_c")) or ("noisy" in parts and not k.endswith("_c")):
+                shapes[k] = (Bt, L, N)
+        shapes.update({"A_f": (D, N), "A_r": (D, N), "D_f": (D,), "D_r": (D,), "conv_w": (D, 4), "conv_b": (D,),
+                       "dt_bias_f": (D,), "dt_bias_r": (D,)})
+        if with_grads:
+            shapes.update({"dy_c": (Bt, L, D), "dy_n": (Bt, L, D)})
+        if with_init:
+            shapes["init_state"] = (Bt, D, N)
+        self.t32 = {}
+        for k, shp in shapes.items():
+            a = draw(k, shp, self.seed, 0 if k in MIXER_PARAMS else part)
+            if dtype == "bf16" and k not in MIXER_PARAMS and k != "init_state":
+                a = bf16_bits_to_f32(f32_to_bf16_bits(a)).reshape(shp)
+            self.t32[k] = a
+
+    def dev_bits(self, name: str) -> np.ndarray:
+        a = self.t32[name]
+        if self.dtype == "bf16" and name not in MIXER_PARAMS and name != "init_state":
+            return f32_to_bf16_bits(a).reshape(a.shape)
+        return a

@@ -9,7 +9,7 @@ import pytest
 from paper_2607_02805_gb300 import binding
 
 INCLUDE = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
-HEADERS = [os.path.join(INCLUDE, h) for h in ("bdscan.h", "bdscan_ssd.h")]
+HEADERS = [os.path.join(INCLUDE, h) for h in ("bdscan.h", "bdscan_ssd.h", "bdscan_mixer.h")]
 
 
 def header_functions():
@@ -148,6 +148,42 @@ def test_active_block_adaln_checks():
     assert rc == binding.BDSCAN_ERR_ARG and "eps" in binding.bdscan_last_error()
     rc = binding.bdscan_active_block_adaln(d, FAKE, n, p, mod, FAKE, FAKE, nbytes - 1, None)
     assert rc == binding.BDSCAN_ERR_ARG and "workspace" in binding.bdscan_last_error()
+
+
+def test_mixer_checks_and_workspace():
+    d = _dims()
+    c, n, p = _structs()
+    mp = binding.bdscan_mixer_params(FAKE, FAKE, FAKE, FAKE)
+    fw = binding.bdscan_mixer_forward_workspace_size(d)
+    bw = binding.bdscan_mixer_backward_workspace_size(d)
+    assert fw > 0 and bw > fw and fw % 256 == 0
+    assert binding.bdscan_mixer_boundary_states_workspace_size(d) == fw
+    rc = binding.bdscan_mixer_forward(d, c, FAKE, n, FAKE, p, None, FAKE, FAKE, FAKE, FAKE, fw, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "mparams is NULL" in binding.bdscan_last_error()
+    bad = binding.bdscan_mixer_params(FAKE, None, FAKE, FAKE)
+    rc = binding.bdscan_mixer_forward(d, c, FAKE, n, FAKE, p, bad, FAKE, FAKE, FAKE, FAKE, fw, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "conv_b" in binding.bdscan_last_error()
+    rc = binding.bdscan_mixer_forward(d, c, FAKE, n, FAKE, p, mp, FAKE, FAKE, FAKE, FAKE, fw - 1, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "workspace" in binding.bdscan_last_error()
+    rc = binding.bdscan_mixer_forward(d, c, None, n, FAKE, p, mp, FAKE, FAKE, FAKE, FAKE, fw, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "z_c" in binding.bdscan_last_error()
+    # the cache build takes the gate and the clean output together or not at all
+    rc = binding.bdscan_mixer_boundary_states(d, c, FAKE, FAKE, FAKE, mp, None, None, None, FAKE, FAKE, 1, FAKE, fw,
+                                              None)
+    assert rc == binding.BDSCAN_ERR_ARG and "both z_c and out_c" in binding.bdscan_last_error()
+    # the active block needs its convolution state
+    da = _dims(length=16, block=16)
+    rc = binding.bdscan_mixer_active_block(da, FAKE, None, n, FAKE, p, mp, FAKE, FAKE, 1 << 30, None)
+    assert rc == binding.BDSCAN_ERR_ARG and "conv_seed" in binding.bdscan_last_error()
+    # backward block limits as for bdscan_backward
+    db = _dims(length=96, block=24)
+    gc = binding.bdscan_clean_grads(FAKE, FAKE, FAKE, FAKE)
+    gn = binding.bdscan_noisy_grads(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE)
+    gp = binding.bdscan_param_grads(FAKE, FAKE, FAKE, FAKE)
+    gm = binding.bdscan_mixer_grads(FAKE, FAKE, FAKE, FAKE)
+    rc = binding.bdscan_mixer_backward(db, c, FAKE, n, FAKE, p, mp, FAKE, FAKE, None, gc, FAKE, gn, FAKE, gp, gm, FAKE,
+                                       1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "multiple of 16" in binding.bdscan_last_error()
 
 
 def test_boundary_states_checks():
