@@ -123,6 +123,30 @@ size_t bdscan_ssd_full_bidir_workspace_size(const bdscan_ssd_dims* dims);
 int bdscan_ssd_full_bidir_forward(const bdscan_ssd_dims* dims, const bdscan_noisy* noisy, const bdscan_params* params,
                                   void* y, void* workspace, size_t workspace_bytes, void* stream);
 
+/* All-block backward of the SSD form (Sec. 4.1, eq. prefix-cache-gradient):
+ * gradients of <dy_c, y_c> + <dy_n, y_n> + <dstates, states> with respect to
+ * every input of bdscan_ssd_forward. `states` must be the states that
+ * bdscan_ssd_forward wrote for the same inputs; dy_c and dstates
+ * ([Bt][nb][H][P][N] fp32) are nullable (zero). Per-token gradients are bf16
+ * in the layouts of their inputs (gclean: dx [Bt][L][H][P], ddt [Bt][L][H],
+ * dB, dC [Bt][L][N]; gnoisy likewise, dx summing both directions); dA, dD
+ * [H] fp32. Gradients are overwritten.
+ *
+ * Per block, head and direction the products G = C B^T and Q = dy x^T and the
+ * transposed mixing products (dx = (G o decay dt)^T dy, dC = (Q o decay dt) B,
+ * dB = (Q o decay dt)^T C, and the seed term's) run on the tensor cores with
+ * bf16 operands and fp32 accumulation; the decay, row and column sums that
+ * give the dt and A gradients are fp32. A reverse pass carries the state
+ * gradients over the clean stream's blocks, and the transpose of each block's
+ * state product (the state gradient split into bf16 high and low parts)
+ * finishes the clean stream. Partial sums are combined in a fixed order:
+ * results are deterministic. */
+size_t bdscan_ssd_backward_workspace_size(const bdscan_ssd_dims* dims);
+int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
+                        const bdscan_params* params, const float* states, const void* dy_c, const void* dy_n,
+                        const float* dstates, const bdscan_clean_grads* gclean, const bdscan_noisy_grads* gnoisy,
+                        const bdscan_param_grads* gparams, void* workspace, size_t workspace_bytes, void* stream);
+
 /* The device flag set by a kernel whose bounded wait on its tensor-core work
  * gave up (0 = never). Synchronises the current device; reset != 0 clears it.
  * Returns -1 if the flag cannot be read. */

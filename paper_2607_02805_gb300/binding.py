@@ -137,6 +137,11 @@ SIGNATURES = [
       c_void_p, ctypes.c_size_t, c_void_p]),
     ("bdscan_ssd_active_block", ctypes.c_int,
      [_P(bdscan_ssd_dims), c_void_p, _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p]),
+    ("bdscan_ssd_backward_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
+    ("bdscan_ssd_backward", ctypes.c_int,
+     [_P(bdscan_ssd_dims), _P(bdscan_clean), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, c_void_p,
+      c_void_p, _P(bdscan_clean_grads), _P(bdscan_noisy_grads), _P(bdscan_param_grads), c_void_p, ctypes.c_size_t,
+      c_void_p]),
     ("bdscan_ssd_wait_flag", ctypes.c_int, [ctypes.c_int]),
     ("bdscan_ssd_wait_selftest", ctypes.c_int, [ctypes.c_uint32]),
     ("bdscan_ssd_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
@@ -332,6 +337,16 @@ def bdscan_ssd_active_block(dims, seed, noisy, params, y_n, stream):
     return load().bdscan_ssd_active_block(_ref(dims), seed, _ref(noisy), _ref(params), y_n, stream)
 
 
+def bdscan_ssd_backward_workspace_size(dims) -> int:
+    return load().bdscan_ssd_backward_workspace_size(_ref(dims))
+
+
+def bdscan_ssd_backward(dims, clean, noisy, params, states, dy_c, dy_n, dstates, gclean, gnoisy, gparams, workspace,
+                        workspace_bytes, stream):
+    return load().bdscan_ssd_backward(_ref(dims), _ref(clean), _ref(noisy), _ref(params), states, dy_c, dy_n, dstates,
+                                      _ref(gclean), _ref(gnoisy), _ref(gparams), workspace, workspace_bytes, stream)
+
+
 def bdscan_ssd_wait_flag(reset) -> int:
     return load().bdscan_ssd_wait_flag(int(reset))
 
@@ -525,3 +540,14 @@ def mixer_active_block(dims, seed, conv_seed, t, out_n, workspace, stream=None):
     _call("bdscan_mixer_active_block", ctypes.byref(dims), _ptr(seed), _ptr(conv_seed), ctypes.byref(_mix_noisy(t)),
           _ptr(t["z_n"]), ctypes.byref(make_params(t)), ctypes.byref(make_mixer_params(t)), _ptr(out_n),
           _ptr(workspace), _nbytes(workspace), _stream(stream))
+
+
+def ssd_backward(dims, t, states, dy_c, dy_n, dstates, g, workspace, stream=None):
+    """SSD-form backward; g holds the gradient tensors keyed like t."""
+    gc = bdscan_clean_grads(_ptr(g["x_c"]), _ptr(g["dt_c"]), _ptr(g["B_c"]), _ptr(g["C_c"]))
+    gn = bdscan_noisy_grads(_ptr(g["x_n"]), _ptr(g["dt_f"]), _ptr(g["B_f"]), _ptr(g["C_f"]), _ptr(g["dt_r"]),
+                            _ptr(g["B_r"]), _ptr(g["C_r"]))
+    gp = bdscan_param_grads(_ptr(g["A_f"]), _ptr(g["D_f"]), _ptr(g["A_r"]), _ptr(g["D_r"]))
+    _call("bdscan_ssd_backward", ctypes.byref(dims), ctypes.byref(make_clean(t)), ctypes.byref(make_noisy(t)),
+          ctypes.byref(make_params(t)), _ptr(states), _ptr(dy_c), _ptr(dy_n), _ptr(dstates), ctypes.byref(gc),
+          ctypes.byref(gn), ctypes.byref(gp), _ptr(workspace), _nbytes(workspace), _stream(stream))

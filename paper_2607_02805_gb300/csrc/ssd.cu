@@ -25,6 +25,7 @@
 #include "device.cuh"
 #include "params.h"
 #include "ssd.cuh"
+#include "ssd_common.cuh"
 #include "umma.cuh"
 
 namespace bds {
@@ -33,64 +34,6 @@ namespace {
 using umma::sw128;
 
 __device__ int g_ssd_wait_flag;
-
-constexpr uint32_t kTile16 = 16384;  // one atom column of a 128-row operand tile
-
-// Bounded wait shared by all threads of the CTA; a give-up sets the flag and
-// makes every thread see the failure.
-__device__ __forceinline__ bool cta_wait(uint64_t* bar, uint32_t parity, int* flag) {
-  const bool ok = umma::bar_wait(bar, parity);
-  const int bad = __syncthreads_or(ok ? 0 : 1);
-  if (bad && threadIdx.x == 0) atomicExch(flag, 1);
-  return bad == 0;
-}
-
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<const uint32_t*>(&v);
-}
-
-// Inclusive scan of dt over `n` tokens by one warp (n a multiple of 32):
-// lane l sums tokens [l*n/32, (l+1)*n/32) in order, then the lane totals are
-// scanned. REV = true scans from the last token (suffix sums).
-template <bool REV>
-__device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t stride, int n, float* out) {
-  const int lane = threadIdx.x & 31, per = n / 32;
-  float loc[8];
-  float s = 0.f;
-  for (int q = 0; q < per; ++q) {
-    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
-    s = __fadd_rn(s, __bfloat162float(dt[pos * stride]));
-    loc[q] = s;
-  }
-  float inc = s;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const float v = __shfl_up_sync(0xffffffffu, inc, o);
-    if (lane >= o) inc = __fadd_rn(inc, v);
-  }
-  float base = __shfl_up_sync(0xffffffffu, inc, 1);
-  if (lane == 0) base = 0.f;
-  for (int q = 0; q < per; ++q) {
-    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
-    out[pos] = __fadd_rn(base, loc[q]);
-  }
-  return __shfl_sync(0xffffffffu, inc, 31);  // total
-}
-
-
-// Token index of position s of block k in batch row b: left to right, or
-// right to left (position t of the reversed stream is token L-1-t).
-struct RowMap {
-  int64_t base, step;
-  __device__ __forceinline__ RowMap(int64_t b, int64_t L, int64_t k0, bool rev)
-      : base(rev ? b * L + L - 1 - k0 : b * L + k0), step(rev ? -1 : 1) {}
-  __device__ __forceinline__ int64_t operator()(int64_t s) const { return base + step * s; }
-};
-
-__device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
-  return reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~(uintptr_t)1023);
-}
 
 // Shared memory of k_ssd_block_state (offsets from a 1024-aligned base):
 //   b     the block's B rows as the MN-major A operand: two 64-wide halves of

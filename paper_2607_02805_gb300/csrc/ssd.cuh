@@ -62,6 +62,91 @@ struct SsdScanParams {
   const float* y32_add;  // non-null: add this fp32 array to the output before rounding to y
 };
 
+// Backward (ssd_bwd.cu). One stream and direction of the block-local
+// backward: per (batch row, block, 128-token tile i, head) the products
+// G = C B^T and Q = dy x^T against every s-tile of the block the direction
+// reaches, the masked decays, dC (complete for tile i), the contributions of
+// tile i to dx and dB of every s-tile (partials over i), the column sums of
+// R' = Q o G o decay (partials over i) and its row sums with dt, and for the
+// seeded forward direction the seed term's products (dC, the seed gradient
+// partial over i, the row dot dy_t . seed term_t).
+struct SsdBwdTileParams {
+  SsdGeo g;
+  const __nv_bfloat16 *x, *dy, *dt, *B, *C;  // x, dy [Bt][L][H][P] (dy null: zero); dt [Bt][L][H]; B, C [Bt][L][N]
+  const float* A;       // [H]
+  const float* states;  // seeded direction: block k reads states[b][k-1] ([Bt][nb][H][P][N])
+  float* dx_part;       // [Bt*nb][H][m][Bs][P]
+  float* dB_part;       // [Bt*nb][H][m][Bs][N]
+  float* dC_part;       // [Bt*nb][H][Bs][N]
+  float* col_part;      // [Bt*nb][H][m][Bs]
+  float* rowsum;        // [Bt*nb][H][Bs]
+  float* rowdot;        // [Bt*nb][H][Bs] (seeded direction)
+  float* dS_part;       // [Bt*nb][H][m][P][N] (seeded direction)
+  int* flag;
+};
+
+// The dt and A gradients of one stream and direction from the row and column
+// sums: dc = A (rowsum - dt colsum' + rowdot), then a scan inside the block.
+struct SsdBwdVecParams {
+  SsdGeo g;
+  const __nv_bfloat16* dt;
+  const float* A;
+  const float *col_part, *rowsum, *rowdot;  // rowdot null: zero
+  int upper;
+  float* ddt;    // [Bt][L][H]
+  float* dA;     // [Bt*nb][H]
+  float* sumdt;  // [Bt*nb][H] or null: the block's sum of dt
+};
+
+// Reverse pass over the clean stream's block-end states: gS_k = dstates_k +
+// seed gradients of block k+1 (both streams) + exp(A sumdt_{k+1}) gS_{k+1}.
+struct SsdBwdPassParams {
+  SsdGeo g;
+  const float* A;
+  const float *dS_c, *dS_f;  // [Bt*nb][H][m][P][N] seed gradient partials
+  const float* dstates;      // [Bt][nb][H][P][N] or null
+  const float* sumdt;        // [Bt*nb][H]
+  float* gS;                 // [Bt][nb][H][P][N]
+};
+
+// Transpose of the clean block-state product T_k = sum_s w_s x_s B_s^T, and
+// the gradient of the block decay exp(A sumdt_k) S_{k-1}.
+struct SsdBwdStateParams {
+  SsdGeo g;
+  const __nv_bfloat16 *x, *dt, *B;
+  const float* A;
+  const float* gS;      // [Bt][nb][H][P][N]
+  const float* states;  // [Bt][nb][H][P][N]
+  const float* sumdt;   // [Bt*nb][H]
+  float* dx_state;      // [Bt*nb][H][Bs][P]
+  float* dB_state;      // [Bt*nb][H][Bs][N]
+  float* ddt;           // [Bt][L][H]
+  float* dA;            // [Bt*nb][H]
+  int* flag;
+};
+
+cudaError_t launch_ssd_bwd_tile(bool upper, bool seeded, const SsdBwdTileParams& p, cudaStream_t s);
+cudaError_t launch_ssd_bwd_vec(const SsdBwdVecParams& p, cudaStream_t s);
+cudaError_t launch_ssd_bwd_pass(const SsdBwdPassParams& p, cudaStream_t s);
+cudaError_t launch_ssd_bwd_state(const SsdBwdStateParams& p, cudaStream_t s);
+// Fixed-order combines of the backward's partials into the outputs (bf16
+// per-token gradients, fp32 parameter gradients); see ssd_bwd.cu.
+cudaError_t launch_ssd_bwd_dx(const SsdGeo& g, const float* dxp_c, const float* dxs, const float* dxp_f,
+                              const float* dxp_r, const __nv_bfloat16* dyc, const __nv_bfloat16* dyn, const float* Df,
+                              const float* Dr, __nv_bfloat16* dxc, __nv_bfloat16* dxn, cudaStream_t s);
+cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, const float* dBp_c, const float* dBs, const float* dCp_c,
+                               const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
+                               __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
+                               __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s);
+cudaError_t launch_ssd_bwd_ddt(int64_t n, const float* vc, const float* vs, const float* vf, const float* vr,
+                               __nv_bfloat16* dc, __nv_bfloat16* df, __nv_bfloat16* dr, cudaStream_t s);
+// two launches: per-block sums of dy x, then the per-head sums (the first
+// launch is counted here, the second by the caller)
+cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
+                                  const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* dd, const float* dA_c,
+                                  const float* dA_f, const float* dA_s, const float* dA_r, float* dAf, float* dDf,
+                                  float* dAr, float* dDr, cudaStream_t s);
+
 cudaError_t launch_ssd_block_state(const SsdStateParams& p, cudaStream_t s);
 cudaError_t launch_ssd_state_pass(const SsdPassParams& p, cudaStream_t s);
 cudaError_t launch_ssd_block_scan(bool noisy, const SsdScanParams& p, cudaStream_t s);

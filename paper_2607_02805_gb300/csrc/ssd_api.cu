@@ -1,6 +1,7 @@
 // ssd_api.cu -- the C ABI of the SSD-form scan (include/bdscan_ssd.h):
 // argument validation, workspace layout and the launch sequence.
 #include <cstdio>
+#include <cstring>
 
 #include "bdscan_ssd.h"
 #include "params.h"
@@ -375,3 +376,214 @@ int bdscan_ssd_full_bidir_forward(const bdscan_ssd_dims* dims, const bdscan_nois
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// backward
+// ---------------------------------------------------------------------------
+namespace {
+
+// Workspace regions of the SSD backward (byte offsets), per stream s = clean,
+// noisy forward direction, noisy reverse direction: the tile partials of dx,
+// dB, dC, the column and row sums, the row dots and seed-gradient partials
+// (seeded directions), the dt and A gradients; then the block sums of dt,
+// the state gradients, the clean block-state terms and the dD partials.
+struct SsdBwdWs {
+  size_t dxp[3], dBp[3], dCp[3], colp[3], rows[3], rowdot[3], dSp[3], ddtv[3], dAv[3];
+  size_t sumdt, gS, dxs, dBs, ddts, dAs, dd, total;
+};
+SsdBwdWs ssd_bwd_ws(const bds::SsdGeo& g) {
+  SsdBwdWs w;
+  const size_t bkh = (size_t)g.Bt * g.nb * g.H, P = 64, N = (size_t)g.N, m = (size_t)g.m, Bs = (size_t)g.Bs;
+  size_t o = 0;
+  auto take = [&](size_t floats) {
+    const size_t at = o;
+    o += al256(floats * 4);
+    return at;
+  };
+  for (int s = 0; s < 3; ++s) {
+    w.dxp[s] = take(bkh * m * Bs * P);
+    w.dBp[s] = take(bkh * m * Bs * N);
+    w.dCp[s] = take(bkh * Bs * N);
+    w.colp[s] = take(bkh * m * Bs);
+    w.rows[s] = take(bkh * Bs);
+    w.rowdot[s] = s < 2 ? take(bkh * Bs) : 0;
+    w.dSp[s] = s < 2 ? take(bkh * m * P * N) : 0;
+    w.ddtv[s] = take((size_t)g.Bt * g.L * g.H);
+    w.dAv[s] = take(bkh);
+  }
+  w.sumdt = take(bkh);
+  w.gS = take(bkh * P * N);
+  w.dxs = take(bkh * Bs * P);
+  w.dBs = take(bkh * Bs * N);
+  w.ddts = take((size_t)g.Bt * g.L * g.H);
+  w.dAs = take(bkh);
+  w.dd = take(bkh * 2);
+  w.total = o;
+  return w;
+}
+
+}  // namespace
+
+extern "C" size_t bdscan_ssd_backward_workspace_size(const bdscan_ssd_dims* dims) {
+  bds::SsdGeo g;
+  if (check(dims, &g, "bdscan_ssd_backward_workspace_size") != BDSCAN_OK) return 0;
+  return ssd_bwd_ws(g).total;
+}
+
+extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_clean* clean, const bdscan_noisy* noisy,
+                                   const bdscan_params* params, const float* states, const void* dy_c, const void* dy_n,
+                                   const float* dstates, const bdscan_clean_grads* gclean,
+                                   const bdscan_noisy_grads* gnoisy, const bdscan_param_grads* gparams,
+                                   void* workspace, size_t workspace_bytes, void* stream) {
+  const char* fn = "bdscan_ssd_backward";
+  bds::SsdGeo g;
+  int rc = check(dims, &g, fn);
+  if (rc) return rc;
+  if (gparams == nullptr) return fail_msg(BDSCAN_ERR_ARG, fn, "gparams is NULL");
+  SSD_REQ(gparams->dA_f, fn, "gparams.dA_f");
+  SSD_REQ(gparams->dD_f, fn, "gparams.dD_f");
+  SSD_REQ(gparams->dA_r, fn, "gparams.dA_r");
+  SSD_REQ(gparams->dD_r, fn, "gparams.dD_r");
+  cudaStream_t s = (cudaStream_t)stream;
+  if (g.Bt == 0 || g.L == 0 || g.H == 0) {
+    cudaError_t e = cudaSuccess;
+    const size_t hb = (size_t)g.H * 4;
+    if (hb > 0) {
+      e = cudaMemsetAsync(gparams->dA_f, 0, hb, s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(gparams->dA_r, 0, hb, s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(gparams->dD_f, 0, hb, s);
+      if (e == cudaSuccess) e = cudaMemsetAsync(gparams->dD_r, 0, hb, s);
+    }
+    return e == cudaSuccess ? bds::api_ok() : cuda_fail(e, fn);
+  }
+  if ((rc = check_clean(clean, fn)) || (rc = check_noisy(noisy, params, fn))) return rc;
+  SSD_REQ(states, fn, "states");
+  SSD_OPT(dy_c, fn, "dy_c");
+  SSD_REQ(dy_n, fn, "dy_n");
+  SSD_OPT(dstates, fn, "dstates");
+  if (gclean == nullptr || gnoisy == nullptr) return fail_msg(BDSCAN_ERR_ARG, fn, "gradient struct is NULL");
+  SSD_REQ(gclean->dx, fn, "gclean.dx");
+  SSD_REQ(gclean->ddt, fn, "gclean.ddt");
+  SSD_REQ(gclean->dB, fn, "gclean.dB");
+  SSD_REQ(gclean->dC, fn, "gclean.dC");
+  SSD_REQ(gnoisy->dx, fn, "gnoisy.dx");
+  SSD_REQ(gnoisy->ddt_f, fn, "gnoisy.ddt_f");
+  SSD_REQ(gnoisy->dB_f, fn, "gnoisy.dB_f");
+  SSD_REQ(gnoisy->dC_f, fn, "gnoisy.dC_f");
+  SSD_REQ(gnoisy->ddt_r, fn, "gnoisy.ddt_r");
+  SSD_REQ(gnoisy->dB_r, fn, "gnoisy.dB_r");
+  SSD_REQ(gnoisy->dC_r, fn, "gnoisy.dC_r");
+  const SsdBwdWs w = ssd_bwd_ws(g);
+  SSD_REQ(workspace, fn, "workspace");
+  if (workspace_bytes < w.total) {
+    char msg[160];
+    snprintf(msg, sizeof(msg), "workspace of %zu bytes, %zu needed", workspace_bytes, w.total);
+    return fail_msg(BDSCAN_ERR_ARG, fn, msg);
+  }
+  int* flag = bds::ssd_wait_flag_ptr();
+  if (flag == nullptr) return fail_msg(BDSCAN_ERR_CUDA, fn, "cannot locate the device wait flag");
+  char* ws = (char*)workspace;
+  auto F = [&](size_t off) { return (float*)(ws + off); };
+  using bf = __nv_bfloat16;
+  const bf* xs[3] = {(const bf*)clean->x, (const bf*)noisy->x, (const bf*)noisy->x};
+  const bf* dys[3] = {(const bf*)dy_c, (const bf*)dy_n, (const bf*)dy_n};
+  const bf* dts[3] = {(const bf*)clean->dt, (const bf*)noisy->dt_f, (const bf*)noisy->dt_r};
+  const bf* Bsrc[3] = {(const bf*)clean->B, (const bf*)noisy->B_f, (const bf*)noisy->B_r};
+  const bf* Csrc[3] = {(const bf*)clean->C, (const bf*)noisy->C_f, (const bf*)noisy->C_r};
+  const float* As[3] = {params->A_f, params->A_f, params->A_r};
+  cudaError_t e = cudaSuccess;
+  // 1. block-local products of the three streams (clean and noisy forward
+  //    seeded with the clean state before each block, noisy reverse unseeded)
+  for (int st = 0; st < 3 && e == cudaSuccess; ++st) {
+    bds::SsdBwdTileParams p;
+    memset(&p, 0, sizeof(p));
+    p.g = g;
+    p.x = xs[st];
+    p.dy = dys[st];
+    p.dt = dts[st];
+    p.B = Bsrc[st];
+    p.C = Csrc[st];
+    p.A = As[st];
+    p.states = st < 2 ? states : nullptr;
+    p.dx_part = F(w.dxp[st]);
+    p.dB_part = F(w.dBp[st]);
+    p.dC_part = F(w.dCp[st]);
+    p.col_part = F(w.colp[st]);
+    p.rowsum = F(w.rows[st]);
+    p.rowdot = st < 2 ? F(w.rowdot[st]) : nullptr;
+    p.dS_part = st < 2 ? F(w.dSp[st]) : nullptr;
+    p.flag = flag;
+    e = bds::api_launched(bds::launch_ssd_bwd_tile(st == 2, st < 2, p, s), s);
+  }
+  // 2. dt and A gradients of each stream from the row and column sums
+  for (int st = 0; st < 3 && e == cudaSuccess; ++st) {
+    bds::SsdBwdVecParams v;
+    memset(&v, 0, sizeof(v));
+    v.g = g;
+    v.dt = dts[st];
+    v.A = As[st];
+    v.col_part = F(w.colp[st]);
+    v.rowsum = F(w.rows[st]);
+    v.rowdot = st < 2 ? F(w.rowdot[st]) : nullptr;
+    v.upper = st == 2;
+    v.ddt = F(w.ddtv[st]);
+    v.dA = F(w.dAv[st]);
+    v.sumdt = st == 0 ? F(w.sumdt) : nullptr;
+    e = bds::api_launched(bds::launch_ssd_bwd_vec(v, s), s);
+  }
+  // 3. reverse pass over the clean block-end states
+  if (e == cudaSuccess) {
+    bds::SsdBwdPassParams q;
+    memset(&q, 0, sizeof(q));
+    q.g = g;
+    q.A = params->A_f;
+    q.dS_c = F(w.dSp[0]);
+    q.dS_f = F(w.dSp[1]);
+    q.dstates = dstates;
+    q.sumdt = F(w.sumdt);
+    q.gS = F(w.gS);
+    e = bds::api_launched(bds::launch_ssd_bwd_pass(q, s), s);
+  }
+  // 4. transpose of the clean block-state products
+  if (e == cudaSuccess) {
+    bds::SsdBwdStateParams r;
+    memset(&r, 0, sizeof(r));
+    r.g = g;
+    r.x = xs[0];
+    r.dt = dts[0];
+    r.B = Bsrc[0];
+    r.A = params->A_f;
+    r.gS = F(w.gS);
+    r.states = states;
+    r.sumdt = F(w.sumdt);
+    r.dx_state = F(w.dxs);
+    r.dB_state = F(w.dBs);
+    r.ddt = F(w.ddts);
+    r.dA = F(w.dAs);
+    r.flag = flag;
+    e = bds::api_launched(bds::launch_ssd_bwd_state(r, s), s);
+  }
+  // 5. fixed-order combines into the outputs
+  if (e == cudaSuccess)
+    e = bds::api_launched(bds::launch_ssd_bwd_dx(g, F(w.dxp[0]), F(w.dxs), F(w.dxp[1]), F(w.dxp[2]), dys[0], dys[1],
+                                                 params->D_f, params->D_r, (bf*)gclean->dx, (bf*)gnoisy->dx, s),
+                          s);
+  if (e == cudaSuccess)
+    e = bds::api_launched(bds::launch_ssd_bwd_dbc(g, F(w.dBp[0]), F(w.dBs), F(w.dCp[0]), F(w.dBp[1]), F(w.dCp[1]),
+                                                  F(w.dBp[2]), F(w.dCp[2]), (bf*)gclean->dB, (bf*)gclean->dC,
+                                                  (bf*)gnoisy->dB_f, (bf*)gnoisy->dC_f, (bf*)gnoisy->dB_r,
+                                                  (bf*)gnoisy->dC_r, s),
+                          s);
+  if (e == cudaSuccess)
+    e = bds::api_launched(bds::launch_ssd_bwd_ddt(g.Bt * g.L * g.H, F(w.ddtv[0]), F(w.ddts), F(w.ddtv[1]),
+                                                  F(w.ddtv[2]), (bf*)gclean->ddt, (bf*)gnoisy->ddt_f,
+                                                  (bf*)gnoisy->ddt_r, s),
+                          s);
+  if (e == cudaSuccess)
+    e = bds::api_launched(bds::launch_ssd_bwd_params(g, xs[0], dys[0], xs[1], dys[1], F(w.dd), F(w.dAv[0]),
+                                                     F(w.dAv[1]), F(w.dAs), F(w.dAv[2]), gparams->dA_f,
+                                                     gparams->dD_f, gparams->dA_r, gparams->dD_r, s),
+                          s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return bds::api_ok();
+}

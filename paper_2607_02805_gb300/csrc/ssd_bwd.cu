@@ -1,0 +1,798 @@
+// ssd_bwd.cu -- backward of the SSD form (Mamba-2: one scalar decay per head,
+// B and C shared by the channels) of the block-restricted bidirectional scan,
+// on the tcgen05 tensor cores of sm_103a (Sec. 4.1, eq. prefix-cache-gradient;
+// Appendix C for the Mamba-2 mixers).
+//
+// Per block of Bs tokens, head h and direction (forward: lower-triangular,
+// seeded with the state before the block; reverse: upper-triangular), with
+// c the in-block cumulative dt (prefix sums forward, suffix sums reverse),
+// decay[t, s] = exp(A (c_t - c_s)) on the direction's triangle, G = C B^T,
+// Q = dy x^T, R' = Q o G o decay and R = R' diag(dt):
+//   dx  = (G o decay diag(dt))^T dy          dC = (Q o decay diag(dt)) B
+//   dB  = (Q o decay diag(dt))^T C           seed term y += diag(E) C S^T,
+//   E_t = exp(A c_t): dC += diag(E) dy S, dS = (diag(E) dy)^T C,
+//   dc_t = A (rowsum_t R - colsum_t R + E_t dy_t . (C S^T)_t),
+//   ddt_r = colsum_r R' + sum of dc over the tokens whose c includes dt_r,
+//   dA = sum_t c_t dc_t / A.
+// The clean stream adds the reverse pass over block-end states
+// (S_k = exp(A sumdt_k) S_{k-1} + T_k, T_k = sum_s w_s x_s B_s^T,
+// w_s = exp(A sum_{r>s} dt_r) dt_s) and the transpose of T_k.
+//
+// Kernels: k_ssd_bwd_tile (tcgen05: the products of one 128-token tile of a
+// block against every s-tile its direction reaches, one head per CTA),
+// k_ssd_bwd_vec (dt, A gradients from the row and column sums), k_ssd_bwd_pass
+// (reverse state pass), k_ssd_bwd_state (tcgen05: the block-state transpose),
+// and fixed-order combines in ssd_api.cu's launch sequence.
+#include "device.cuh"
+#include "params.h"
+#include "ssd.cuh"
+#include "ssd_common.cuh"
+#include "umma.cuh"
+
+namespace bds {
+namespace {
+
+using umma::sw128;
+
+constexpr int kBwdThreads = 128;
+
+// Copies `rows` rows of `ncols` (64 or 128) bf16 into 128-byte-swizzled atom
+// columns of rows * 128 bytes each; a null source stages zeros.
+__device__ __forceinline__ void stage_bf16(unsigned char* dst, const __nv_bfloat16* src, int64_t ld, int rows,
+                                           int ncols) {
+  const int cpr = ncols / 8;
+  for (int c = threadIdx.x; c < rows * cpr; c += kBwdThreads) {
+    const int r = c / cpr, ch = c % cpr;
+    unsigned char* d = dst + (uint32_t)(ch >> 3) * (uint32_t)rows * 128u + sw128((uint32_t)r, (uint32_t)(ch & 7));
+    if (src == nullptr)
+      *reinterpret_cast<uint4*>(d) = make_uint4(0u, 0u, 0u, 0u);
+    else
+      cp_async16(d, src + (int64_t)r * ld + ch * 8, 16);
+  }
+}
+
+// An fp32 [rows][ncols] matrix (row stride ncols) as bf16 atom columns (rows * 128
+// bytes each); `lo` selects the rounding residual v - bf16(v) instead of bf16(v).
+__device__ __forceinline__ void stage_f32_as_bf16(unsigned char* dst, const float* src, int rows, int ncols, bool lo) {
+  const int cpr = ncols / 8;
+  for (int c = threadIdx.x; c < rows * cpr; c += kBwdThreads) {
+    const int r = c / cpr, ch = c % cpr;
+    const float4 a = *reinterpret_cast<const float4*>(src + (int64_t)r * ncols + ch * 8);
+    const float4 b = *reinterpret_cast<const float4*>(src + (int64_t)r * ncols + ch * 8 + 4);
+    float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      float x0 = v[2 * e], x1 = v[2 * e + 1];
+      if (lo) {
+        x0 = __fsub_rn(x0, __bfloat162float(__float2bfloat16_rn(x0)));
+        x1 = __fsub_rn(x1, __bfloat162float(__float2bfloat16_rn(x1)));
+      }
+      w[e] = pack_bf16(x0, x1);
+    }
+    *reinterpret_cast<uint4*>(dst + (uint32_t)(ch >> 3) * (uint32_t)rows * 128u + sw128((uint32_t)r, (uint32_t)(ch & 7))) =
+        make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
+// Element `col` of row `row` of a bf16 tile in swizzled atom columns of 128 rows.
+__device__ __forceinline__ float tile_at(const unsigned char* tile, int row, int col) {
+  const uint32_t off = (uint32_t)(col >> 6) * kTile16 + sw128((uint32_t)row, (uint32_t)((col & 63) >> 3)) + (uint32_t)(col & 7) * 2u;
+  return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(tile + off));
+}
+
+__device__ __forceinline__ void store_row(float* dst, const float (&v)[32]) {
+#pragma unroll
+  for (int e = 0; e < 32; e += 4) *reinterpret_cast<float4*>(dst + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
+}
+
+// Shared memory of k_ssd_bwd_tile (offsets from a 1024-aligned base).
+//   DY  dy of tile i, [128 t][64 p]          C   C of tile i, [128 t][128 n] (n >= N zero)
+//   X   x of s-tile j, [128 s][64 p]         BT  B of s-tile j, [128 s][N]
+//   DG  Q o decay o dt, [128 t][128 s]       M   G o decay o dt, [128 t][128 s]
+//   COL R' of 64 columns, [128][65] fp32     VEC c and dt of the block, fp32
+// The seed phase reuses X for the seed ([64 p][N], atom columns of 8 KB) and
+// BT for E o dy ([128 t][64 p]).
+struct TileSmem {
+  static constexpr uint32_t DY = 0, C = 16384, X = 49152, BT = 65536, DG = 98304, M = 131072, COL = 163840;
+  static constexpr uint32_t VEC = COL + 128u * 65u * 4u;
+  static constexpr uint32_t total = VEC + 2u * 256u * 4u + 1024u;
+};
+
+// One CTA of 4 warps per (batch row, block, tile i) and head: thread t owns
+// token row t of tile i (TMEM lane t) for the row-side products and row s = t
+// of s-tile j for the column-side ones. TMEM: G at columns 0..127 and Q at
+// 128..255 (then dx_j at 0..63, dB_j at 64..64+N), dC at 256, C S^T at 384,
+// dS^T at 448.
+template <int N, bool UPPER, bool SEED>
+__global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTileParams p) {
+  extern __shared__ unsigned char smraw[];
+  unsigned char* sm = align1024(smraw);
+  __shared__ uint64_t bar;
+  __shared__ uint32_t tslot;
+  using S = TileSmem;
+  const SsdGeo& g = p.g;
+  const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x, w = t >> 5;
+  const int64_t idx = blockIdx.x;
+  const int i = (int)(idx % m);
+  const int64_t bk = idx / m, b = bk / g.nb;
+  const int k = (int)(bk % g.nb);
+  const int h = blockIdx.y;
+  const int64_t tok0 = b * g.L + (int64_t)k * Bs;  // the block's first token
+  const int64_t HP = (int64_t)H * kSsdP;
+  float* s_c = reinterpret_cast<float*>(sm + S::VEC);
+  float* s_dt = s_c + 256;
+  float* s_col = reinterpret_cast<float*>(sm + S::COL);
+
+  stage_bf16(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+  stage_bf16(sm + S::C, p.C + (tok0 + i * kSsdT) * N, N, 128, N);
+  if (N == 64)
+    for (int c = t; c < 128 * 8; c += kBwdThreads) *reinterpret_cast<uint4*>(sm + S::C + kTile16 + c * 16) = make_uint4(0u, 0u, 0u, 0u);
+  cp_async_commit();
+  for (int s = t; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
+  if (w == 0) warp_scan_dt<UPPER>(p.dt + tok0 * H + h, H, Bs, s_c);
+  if (t == 0) umma::bar_init(&bar, 1);
+  if (w == 0) tmem_alloc(&tslot, 512);
+  umma::fence_before_sync();
+  __syncthreads();
+  umma::fence_after_sync();
+  const uint32_t tm = tslot, lane_base = tm + ((uint32_t)(32 * w) << 16);
+  const float A2 = __fmul_rn(p.A[h], kLog2e);
+  const int tt = i * kSsdT + t;
+  const float ct = s_c[tt];
+  float rowsum = 0.f;
+  uint32_t phase = 0;
+  bool alive = true;
+  const uint32_t y0 = umma::smem_u32(sm + S::DY), c0 = umma::smem_u32(sm + S::C), x0 = umma::smem_u32(sm + S::X),
+                 b0 = umma::smem_u32(sm + S::BT), dg0 = umma::smem_u32(sm + S::DG), m0 = umma::smem_u32(sm + S::M);
+  constexpr uint32_t id_gq = umma::idesc_bf16(128, 128, false, false);
+  constexpr uint32_t id_dc = umma::idesc_bf16(128, N, false, true);
+  constexpr uint32_t id_dx = umma::idesc_bf16(128, 64, true, true);
+  constexpr uint32_t id_db = umma::idesc_bf16(128, N, true, true);
+  const int j0 = UPPER ? i : 0, j1 = UPPER ? m - 1 : i;
+  for (int j = j0; j <= j1; ++j) {
+    const int64_t sr0 = tok0 + (int64_t)j * kSsdT;
+    stage_bf16(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
+    stage_bf16(sm + S::BT, p.B + sr0 * N, N, 128, N);
+    cp_async_commit();
+    cp_async_wait_all();
+    umma::fence_async_smem();
+    umma::fence_before_sync();
+    __syncthreads();
+    if (t == 0) {
+      umma::fence_after_sync();
+#pragma unroll
+      for (int kk = 0; kk < N / 16; ++kk) {  // G = C_i B_j^T
+        const uint32_t off = (uint32_t)(kk >> 2) * kTile16 + (uint32_t)(kk & 3) * 32u;
+        umma::mma_bf16(tm, umma::sdesc(c0 + off, 16, 1024), umma::sdesc(b0 + off, 16, 1024), id_gq, kk > 0);
+      }
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)  // Q = dy_i x_j^T
+        umma::mma_bf16(tm + 128u, umma::sdesc(y0 + kk * 32u, 16, 1024), umma::sdesc(x0 + kk * 32u, 16, 1024), id_gq,
+                       kk > 0);
+      umma::mma_commit(&bar);
+    }
+    if (!cta_wait(&bar, phase, p.flag)) {
+      alive = false;
+      break;
+    }
+    phase ^= 1u;
+    umma::fence_after_sync();
+    // decay-weighted tiles of this row: dG = Q decay dt (DG) and M = G decay dt
+    // (M) in bf16, R' for the column sums and R for the row sum in fp32
+#pragma unroll 1
+    for (int c = 0; c < 4; ++c) {
+      float gv[32], qv[32];
+      umma::tmem_ld32(lane_base + 32u * (uint32_t)c, gv);
+      umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)c, qv);
+      uint32_t dgp[16], mp[16];
+#pragma unroll
+      for (int e = 0; e < 32; e += 2) {
+        float dgv[2], mv[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const int s = j * kSsdT + 32 * c + e + q;
+          const bool valid = UPPER ? (s >= tt) : (s <= tt);
+          const float L = valid ? ex2(__fmul_rn(A2, __fsub_rn(ct, s_c[s]))) : 0.f;
+          const float ds = s_dt[s];
+          const float gl = __fmul_rn(gv[e + q], L);
+          const float rp = __fmul_rn(qv[e + q], gl);
+          rowsum = __fmaf_rn(rp, ds, rowsum);
+          s_col[t * 65 + 32 * (c & 1) + e + q] = rp;
+          dgv[q] = __fmul_rn(__fmul_rn(qv[e + q], L), ds);
+          mv[q] = __fmul_rn(gl, ds);
+        }
+        dgp[e >> 1] = pack_bf16(dgv[0], dgv[1]);
+        mp[e >> 1] = pack_bf16(mv[0], mv[1]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int chunk = 4 * c + u;
+        const uint32_t off = (uint32_t)(chunk >> 3) * kTile16 + sw128((uint32_t)t, (uint32_t)(chunk & 7));
+        *reinterpret_cast<uint4*>(sm + S::DG + off) = make_uint4(dgp[4 * u], dgp[4 * u + 1], dgp[4 * u + 2], dgp[4 * u + 3]);
+        *reinterpret_cast<uint4*>(sm + S::M + off) = make_uint4(mp[4 * u], mp[4 * u + 1], mp[4 * u + 2], mp[4 * u + 3]);
+      }
+      if (c & 1) {  // column sums of R' over the tile's 128 rows, 64 columns at a time
+        __syncthreads();
+        if (t < 64) {
+          float sum = 0.f;
+          for (int r = 0; r < 128; ++r) sum = __fadd_rn(sum, s_col[r * 65 + t]);
+          p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + 64 * (c >> 1) + t] = sum;
+        }
+        __syncthreads();
+      }
+    }
+    umma::fence_async_smem();
+    umma::fence_before_sync();
+    __syncthreads();
+    if (t == 0) {
+      umma::fence_after_sync();
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t koff = (uint32_t)(kk >> 2) * kTile16 + (uint32_t)(kk & 3) * 32u, mn = (uint32_t)kk * 2048u;
+        // dC += dG_j B_j: dG K-major [t][s], B_j MN-major [s][n]
+        umma::mma_bf16(tm + 256u, umma::sdesc(dg0 + koff, 16, 1024), umma::sdesc(b0 + mn, kTile16, 1024), id_dc,
+                       j != j0 || kk > 0);
+        // dx_j = M_j^T dy_i: M read as an MN-major operand (M = s, K = t)
+        umma::mma_bf16(tm, umma::sdesc(m0 + mn, kTile16, 1024), umma::sdesc(y0 + mn, kTile16, 1024), id_dx, kk > 0);
+        // dB_j = dG_j^T C_i
+        umma::mma_bf16(tm + 64u, umma::sdesc(dg0 + mn, kTile16, 1024), umma::sdesc(c0 + mn, kTile16, 1024), id_db,
+                       kk > 0);
+      }
+      umma::mma_commit(&bar);
+    }
+    if (!cta_wait(&bar, phase, p.flag)) {
+      alive = false;
+      break;
+    }
+    phase ^= 1u;
+    umma::fence_after_sync();
+    {  // row s = j*128 + t of tile i's contributions to dx and dB
+      float v[32];
+      float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * kSsdP;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
+        store_row(dxo + 32 * q, v);
+      }
+      float* dbo = p.dB_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * N;
+#pragma unroll
+      for (int q = 0; q < N / 32; ++q) {
+        umma::tmem_ld32(lane_base + 64u + 32u * (uint32_t)q, v);
+        store_row(dbo + 32 * q, v);
+      }
+    }
+    umma::fence_before_sync();
+  }
+
+  if (alive) {
+    p.rowsum[(bk * H + h) * Bs + tt] = rowsum;
+    if (SEED) {
+      float rowdot = 0.f;
+      if (k > 0) {
+        // the seed (the clean state before the block) as bf16, E o dy
+        stage_f32_as_bf16(sm + S::X, p.states + ((b * g.nb + k - 1) * H + h) * (int64_t)kSsdP * N, 64, N, false);
+        const float E = ex2(__fmul_rn(A2, ct));
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) {
+          const uint4 u = *reinterpret_cast<const uint4*>(sm + S::DY + sw128((uint32_t)t, (uint32_t)ch));
+          const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&u);
+          uint32_t o[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(v2[e]);
+            o[e] = pack_bf16(__fmul_rn(E, f.x), __fmul_rn(E, f.y));
+          }
+          *reinterpret_cast<uint4*>(sm + S::BT + sw128((uint32_t)t, (uint32_t)ch)) = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+        umma::fence_async_smem();
+        umma::fence_before_sync();
+        __syncthreads();
+        if (t == 0) {
+          umma::fence_after_sync();
+          constexpr uint32_t id_cs = umma::idesc_bf16(128, 64, false, false);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)  // dC += (E o dy) S: S as MN-major [p][n], atom columns of 8 KB
+            umma::mma_bf16(tm + 256u, umma::sdesc(b0 + kk * 32u, 16, 1024), umma::sdesc(x0 + kk * 2048u, 8192, 1024),
+                           id_dc, true);
+#pragma unroll
+          for (int kk = 0; kk < N / 16; ++kk)  // C S^T: S as K-major [p][n]
+            umma::mma_bf16(tm + 384u, umma::sdesc(c0 + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
+                           umma::sdesc(x0 + (kk >> 2) * 8192u + (kk & 3) * 32u, 16, 1024), id_cs, kk > 0);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)  // dS^T = C_i^T (E o dy): C read as MN-major (M = n)
+            umma::mma_bf16(tm + 448u, umma::sdesc(c0 + kk * 2048u, kTile16, 1024),
+                           umma::sdesc(b0 + kk * 2048u, kTile16, 1024), id_dx, kk > 0);
+          umma::mma_commit(&bar);
+        }
+        if (cta_wait(&bar, phase, p.flag)) {
+          phase ^= 1u;
+          umma::fence_after_sync();
+          float v[32];
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {  // dy_t . (C_t S^T)
+            umma::tmem_ld32(lane_base + 384u + 32u * (uint32_t)q, v);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) rowdot = __fmaf_rn(tile_at(sm + S::DY, t, 32 * q + e), v[e], rowdot);
+          }
+          rowdot = __fmul_rn(E, rowdot);
+          if (32 * w < N) {  // row n = t of dS^T: the seed gradient partial [p][n]
+            float* dso = p.dS_part + ((bk * H + h) * m + i) * (int64_t)kSsdP * N + t;
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              umma::tmem_ld32(lane_base + 448u + 32u * (uint32_t)q, v);
+#pragma unroll
+              for (int e = 0; e < 32; ++e) dso[(int64_t)(32 * q + e) * N] = v[e];
+            }
+          }
+        } else {
+          alive = false;
+        }
+      }
+      p.rowdot[(bk * H + h) * Bs + tt] = rowdot;
+    }
+    if (alive) {  // dC of row t of tile i
+      float v[32];
+      float* dco = p.dC_part + ((bk * H + h) * Bs + tt) * N;
+#pragma unroll
+      for (int q = 0; q < N / 32; ++q) {
+        umma::tmem_ld32(lane_base + 256u + 32u * (uint32_t)q, v);
+        store_row(dco + 32 * q, v);
+      }
+    }
+  }
+  cp_async_wait_all();
+  umma::fence_before_sync();
+  __syncthreads();
+  if (w == 0) tmem_dealloc(tm, 512);
+}
+
+// In-place inclusive scan of n fp32 values (n a multiple of 32, at most 256)
+// by one warp; REV scans from the end (suffix sums).
+template <bool REV>
+__device__ __forceinline__ void warp_scan_f32(float* a, int n) {
+  const int lane = threadIdx.x & 31, per = n / 32;
+  float loc[8];
+  float s = 0.f;
+  for (int q = 0; q < per; ++q) {
+    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
+    s = __fadd_rn(s, a[pos]);
+    loc[q] = s;
+  }
+  float inc = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float v = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc = __fadd_rn(inc, v);
+  }
+  float base = __shfl_up_sync(0xffffffffu, inc, 1);
+  if (lane == 0) base = 0.f;
+  __syncwarp();
+  for (int q = 0; q < per; ++q) {
+    const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
+    a[pos] = __fadd_rn(base, loc[q]);
+  }
+  __syncwarp();
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// One warp per (batch row, block, head): dc_t = A (rowsum_t - dt_t colsum'_t +
+// rowdot_t), ddt_r = colsum'_r + sum of dc over the tokens whose cumulative dt
+// includes dt_r (t >= r forward, t <= r reverse), dA = sum_t c_t (dc_t / A).
+__global__ void __launch_bounds__(128) k_ssd_bwd_vec(const SsdBwdVecParams p) {
+  __shared__ float s_c[4][256], s_q[4][256];
+  const SsdGeo& g = p.g;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, Bs = (int)g.Bs, m = g.m, H = g.H;
+  const int64_t u = (int64_t)blockIdx.x * 4 + w;
+  if (u >= g.Bt * g.nb * H) return;  // whole warps
+  const int h = (int)(u % H);
+  const int64_t bk = u / H, b = bk / g.nb, k = bk % g.nb;
+  const int64_t tok0 = b * g.L + k * Bs;
+  const float total = p.upper ? warp_scan_dt<true>(p.dt + tok0 * H + h, H, Bs, s_c[w])
+                              : warp_scan_dt<false>(p.dt + tok0 * H + h, H, Bs, s_c[w]);
+  if (p.sumdt != nullptr && lane == 0) p.sumdt[bk * H + h] = total;
+  __syncwarp();
+  const float A = p.A[h];
+  float dA = 0.f;
+  const float* colp = p.col_part + (bk * H + h) * (int64_t)m * Bs;
+  for (int s = lane; s < Bs; s += 32) {
+    const int js = s / kSsdT;
+    float col = 0.f;
+    for (int i = p.upper ? 0 : js; i <= (p.upper ? js : m - 1); ++i) col = __fadd_rn(col, colp[(int64_t)i * Bs + s]);
+    const float dt = __bfloat162float(p.dt[(tok0 + s) * H + h]);
+    float q = __fsub_rn(p.rowsum[(bk * H + h) * Bs + s], __fmul_rn(dt, col));
+    if (p.rowdot != nullptr) q = __fadd_rn(q, p.rowdot[(bk * H + h) * Bs + s]);
+    dA = __fmaf_rn(s_c[w][s], q, dA);
+    s_q[w][s] = __fmul_rn(A, q);
+    p.ddt[(tok0 + s) * H + h] = col;
+  }
+  __syncwarp();
+  if (p.upper)
+    warp_scan_f32<false>(s_q[w], Bs);  // reverse: c_t sums dt over r >= t, so dt_r feeds every t <= r
+  else
+    warp_scan_f32<true>(s_q[w], Bs);   // forward: dt_r feeds every t >= r
+  for (int s = lane; s < Bs; s += 32) p.ddt[(tok0 + s) * H + h] = __fadd_rn(p.ddt[(tok0 + s) * H + h], s_q[w][s]);
+  dA = warp_sum(dA);
+  if (lane == 0) p.dA[bk * H + h] = dA;
+}
+
+// One thread per (batch row, head, channel, state index), blocks last to first.
+__global__ void __launch_bounds__(256) k_ssd_bwd_pass(const SsdBwdPassParams p) {
+  const SsdGeo& g = p.g;
+  const int64_t PN = (int64_t)kSsdP * g.N, per_b = (int64_t)g.H * PN;
+  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (idx >= g.Bt * per_b) return;
+  const int64_t b = idx / per_b, r = idx - b * per_b;
+  const int h = (int)(r / PN);
+  const int64_t pn = r - (int64_t)h * PN;
+  const float A2 = __fmul_rn(p.A[h], kLog2e);
+  float gS = 0.f;
+  for (int k = g.nb - 1; k >= 0; --k) {
+    const int64_t o = ((b * g.nb + k) * g.H + h) * PN + pn;
+    if (k + 1 < g.nb) {  // the seed gradients of block k+1 (forward noisy direction, then clean)
+      const int64_t base = ((b * g.nb + k + 1) * g.H + h) * (int64_t)g.m * PN + pn;
+      float inj = 0.f;
+      for (int i = 0; i < g.m; ++i) inj = __fadd_rn(inj, p.dS_f[base + i * PN]);
+      for (int i = 0; i < g.m; ++i) inj = __fadd_rn(inj, p.dS_c[base + i * PN]);
+      gS = __fadd_rn(gS, inj);
+    }
+    if (p.dstates != nullptr) gS = __fadd_rn(gS, p.dstates[o]);
+    p.gS[o] = gS;
+    gS = __fmul_rn(ex2(__fmul_rn(A2, p.sumdt[(b * g.nb + k) * g.H + h])), gS);
+  }
+}
+
+// Shared memory of k_ssd_bwd_state (from a 1024-aligned base): the state
+// gradient's bf16 high and low parts ([64 p][N], atom columns of 8 KB), x and
+// B of one s-tile, per-token vectors of the block.
+struct StateBwdSmem {
+  static constexpr uint32_t GH = 0, GL = 16384, X = 32768, BT = 49152, VEC = 81920;
+  static constexpr uint32_t total = VEC + 5u * 256u * 4u + 1024u;
+};
+
+// One CTA of 4 warps per (batch row, block, head) of the clean stream, with
+// gS = the gradient of the state after the block: U = B gS^T and V = x gS per
+// s-tile on the tensor core (gS split into bf16 high and low parts), then
+// dx += w U, dB += w V, dw = x . U, and the dt and A gradients of w and of
+// the block decay.
+template <int N>
+__global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdStateParams p) {
+  extern __shared__ unsigned char smraw[];
+  unsigned char* sm = align1024(smraw);
+  __shared__ uint64_t bar;
+  __shared__ uint32_t tslot;
+  __shared__ float red[4];
+  using S = StateBwdSmem;
+  const SsdGeo& g = p.g;
+  const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x, w = t >> 5, lane = t & 31;
+  const int64_t bk = blockIdx.x, b = bk / g.nb;
+  const int k = (int)(bk % g.nb), h = blockIdx.y;
+  const int64_t tok0 = b * g.L + (int64_t)k * Bs, HP = (int64_t)H * kSsdP, PN = (int64_t)kSsdP * N;
+  float* s_suf = reinterpret_cast<float*>(sm + S::VEC);  // inclusive suffix sums of dt, then exclusive
+  float* s_dt = s_suf + 256;
+  float* s_w = s_dt + 256;
+  float* s_dw = s_w + 256;
+  float* s_e = s_dw + 256;
+  const float* gS = p.gS + (bk * H + h) * PN;
+  stage_f32_as_bf16(sm + S::GH, gS, 64, N, false);
+  stage_f32_as_bf16(sm + S::GL, gS, 64, N, true);
+  for (int s = t; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
+  if (w == 0) warp_scan_dt<true>(p.dt + tok0 * H + h, H, Bs, s_suf);
+  // block decay: da = sum over (p, n) of gS o S_{k-1}
+  float da = 0.f;
+  if (k > 0) {
+    const float* prev = p.states + ((b * g.nb + k - 1) * H + h) * PN;
+    for (int64_t q = t; q < PN; q += kBwdThreads) da = __fmaf_rn(gS[q], prev[q], da);
+  }
+  da = warp_sum(da);
+  if (lane == 0) red[w] = da;
+  if (t == 0) umma::bar_init(&bar, 1);
+  if (w == 0) tmem_alloc(&tslot, 256);
+  umma::fence_before_sync();
+  __syncthreads();
+  umma::fence_after_sync();
+  da = __fadd_rn(__fadd_rn(red[0], red[1]), __fadd_rn(red[2], red[3]));
+  for (int s = t; s < Bs; s += kBwdThreads) s_suf[s] = __fsub_rn(s_suf[s], s_dt[s]);  // dt after s
+  const uint32_t tm = tslot, lane_base = tm + ((uint32_t)(32 * w) << 16);
+  const float A = p.A[h], A2 = __fmul_rn(A, kLog2e);
+  const uint32_t gh = umma::smem_u32(sm + S::GH), gl = umma::smem_u32(sm + S::GL), x0 = umma::smem_u32(sm + S::X),
+                 b0 = umma::smem_u32(sm + S::BT);
+  constexpr uint32_t id_u = umma::idesc_bf16(128, 64, false, false);
+  constexpr uint32_t id_v = umma::idesc_bf16(128, N, false, true);
+  uint32_t phase = 0;
+  bool alive = true;
+  for (int j = 0; j < m; ++j) {
+    const int64_t sr0 = tok0 + (int64_t)j * kSsdT;
+    stage_bf16(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
+    stage_bf16(sm + S::BT, p.B + sr0 * N, N, 128, N);
+    cp_async_commit();
+    cp_async_wait_all();
+    umma::fence_async_smem();
+    umma::fence_before_sync();
+    __syncthreads();
+    if (t == 0) {
+      umma::fence_after_sync();
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const uint32_t gs0 = half ? gl : gh;
+#pragma unroll
+        for (int kk = 0; kk < N / 16; ++kk)  // U = B_j gS^T: gS K-major [p][n]
+          umma::mma_bf16(tm, umma::sdesc(b0 + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
+                         umma::sdesc(gs0 + (kk >> 2) * 8192u + (kk & 3) * 32u, 16, 1024), id_u, half > 0 || kk > 0);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)  // V = x_j gS: gS MN-major [p][n]
+          umma::mma_bf16(tm + 64u, umma::sdesc(x0 + kk * 32u, 16, 1024), umma::sdesc(gs0 + kk * 2048u, 8192, 1024),
+                         id_v, half > 0 || kk > 0);
+      }
+      umma::mma_commit(&bar);
+    }
+    if (!cta_wait(&bar, phase, p.flag)) {
+      alive = false;
+      break;
+    }
+    phase ^= 1u;
+    umma::fence_after_sync();
+    {
+      const int s = j * kSsdT + t;
+      const float e = ex2(__fmul_rn(A2, s_suf[s])), ws = __fmul_rn(e, s_dt[s]);
+      float v[32], dw = 0.f;
+      float* dxo = p.dx_state + ((bk * H + h) * Bs + s) * kSsdP;
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
+#pragma unroll
+        for (int e2 = 0; e2 < 32; ++e2) {
+          dw = __fmaf_rn(tile_at(sm + S::X, t, 32 * q + e2), v[e2], dw);
+          v[e2] = __fmul_rn(ws, v[e2]);
+        }
+        store_row(dxo + 32 * q, v);
+      }
+      float* dbo = p.dB_state + ((bk * H + h) * Bs + s) * N;
+#pragma unroll
+      for (int q = 0; q < N / 32; ++q) {
+        umma::tmem_ld32(lane_base + 64u + 32u * (uint32_t)q, v);
+#pragma unroll
+        for (int e2 = 0; e2 < 32; ++e2) v[e2] = __fmul_rn(ws, v[e2]);
+        store_row(dbo + 32 * q, v);
+      }
+      s_w[s] = ws;
+      s_dw[s] = dw;
+      s_e[s] = e;
+    }
+    umma::fence_before_sync();
+  }
+  __syncthreads();
+  if (alive && w == 0) {
+    // the exponent of w_s is A times the dt after s: dt_r feeds every s < r
+    float dA = 0.f;
+    for (int s = lane; s < Bs; s += 32) {
+      const float wdw = __fmul_rn(s_w[s], s_dw[s]);
+      dA = __fmaf_rn(s_suf[s], wdw, dA);
+      s_suf[s] = __fmul_rn(A, wdw);
+    }
+    __syncwarp();
+    warp_scan_f32<false>(s_suf, Bs);  // inclusive prefix sums of A w dw
+    const float sd = p.sumdt[bk * H + h], ak = ex2(__fmul_rn(A2, sd));
+    const float blk = __fmul_rn(__fmul_rn(A, ak), da);  // block decay exp(A sumdt) of S_{k-1}
+    for (int r = lane; r < Bs; r += 32) {
+      const float before = r > 0 ? s_suf[r - 1] : 0.f;  // exclusive: s < r
+      p.ddt[(tok0 + r) * H + h] = __fadd_rn(__fadd_rn(__fmul_rn(s_e[r], s_dw[r]), before), blk);
+    }
+    dA = warp_sum(dA);
+    if (lane == 0) p.dA[bk * H + h] = __fadd_rn(dA, __fmul_rn(__fmul_rn(sd, ak), da));
+  }
+  cp_async_wait_all();
+  umma::fence_before_sync();
+  __syncthreads();
+  if (w == 0) tmem_dealloc(tm, 256);
+}
+
+}  // namespace
+
+namespace {
+
+// dx of both streams: the tile partials of every tile that reaches s (tiles
+// i >= j(s) forward, i <= j(s) reverse), the clean state term and the skip
+// terms.
+__global__ void __launch_bounds__(256) k_ssd_bwd_dx(const SsdGeo g, const float* dxp_c, const float* dxs,
+                                                    const float* dxp_f, const float* dxp_r, const __nv_bfloat16* dyc,
+                                                    const __nv_bfloat16* dyn, const float* Df, const float* Dr,
+                                                    __nv_bfloat16* dxc, __nv_bfloat16* dxn) {
+  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  const int64_t total = g.Bt * g.L * g.H * kSsdP;
+  if (idx >= total) return;
+  const int pp = (int)(idx % kSsdP);
+  const int h = (int)((idx / kSsdP) % g.H);
+  const int64_t bt = idx / ((int64_t)g.H * kSsdP), b = bt / g.L, tl = bt % g.L;
+  const int64_t k = tl / g.Bs, s = tl % g.Bs, bk = b * g.nb + k;
+  const int j = (int)(s / kSsdT), m = g.m;
+  auto at = [&](const float* a, int i) { return a[(((bk * g.H + h) * m + i) * g.Bs + s) * kSsdP + pp]; };
+  float c = 0.f, n = 0.f;
+  for (int i = j; i < m; ++i) c = __fadd_rn(c, at(dxp_c, i));
+  c = __fadd_rn(c, dxs[((bk * g.H + h) * g.Bs + s) * kSsdP + pp]);
+  if (dyc != nullptr) c = __fmaf_rn(Df[h], __bfloat162float(dyc[idx]), c);
+  for (int i = j; i < m; ++i) n = __fadd_rn(n, at(dxp_f, i));
+  for (int i = 0; i <= j; ++i) n = __fadd_rn(n, at(dxp_r, i));
+  n = __fmaf_rn(__fadd_rn(Df[h], Dr[h]), __bfloat162float(dyn[idx]), n);
+  dxc[idx] = __float2bfloat16_rn(c);
+  dxn[idx] = __float2bfloat16_rn(n);
+}
+
+// dB and dC of the three streams: per head the tile partials (and the clean
+// state term), summed over the heads in order.
+__global__ void __launch_bounds__(256) k_ssd_bwd_dbc(const SsdGeo g, const float* dBp_c, const float* dBs,
+                                                     const float* dCp_c, const float* dBp_f, const float* dCp_f,
+                                                     const float* dBp_r, const float* dCp_r, __nv_bfloat16* dBc,
+                                                     __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
+                                                     __nv_bfloat16* dBr, __nv_bfloat16* dCr) {
+  const int N = g.N, m = g.m;
+  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (idx >= g.Bt * g.L * N) return;
+  const int n = (int)(idx % N);
+  const int64_t bt = idx / N, b = bt / g.L, tl = bt % g.L;
+  const int64_t k = tl / g.Bs, s = tl % g.Bs, bk = b * g.nb + k;
+  const int j = (int)(s / kSsdT);
+  float bc = 0.f, cc = 0.f, bf = 0.f, cf = 0.f, br = 0.f, cr = 0.f;
+  for (int h = 0; h < g.H; ++h) {
+    const int64_t hb = bk * g.H + h;
+    auto tp = [&](const float* a, int i) { return a[((hb * m + i) * g.Bs + s) * N + n]; };
+    for (int i = j; i < m; ++i) bc = __fadd_rn(bc, tp(dBp_c, i));
+    bc = __fadd_rn(bc, dBs[(hb * g.Bs + s) * N + n]);
+    cc = __fadd_rn(cc, dCp_c[(hb * g.Bs + s) * N + n]);
+    for (int i = j; i < m; ++i) bf = __fadd_rn(bf, tp(dBp_f, i));
+    cf = __fadd_rn(cf, dCp_f[(hb * g.Bs + s) * N + n]);
+    for (int i = 0; i <= j; ++i) br = __fadd_rn(br, tp(dBp_r, i));
+    cr = __fadd_rn(cr, dCp_r[(hb * g.Bs + s) * N + n]);
+  }
+  dBc[idx] = __float2bfloat16_rn(bc);
+  dCc[idx] = __float2bfloat16_rn(cc);
+  dBf[idx] = __float2bfloat16_rn(bf);
+  dCf[idx] = __float2bfloat16_rn(cf);
+  dBr[idx] = __float2bfloat16_rn(br);
+  dCr[idx] = __float2bfloat16_rn(cr);
+}
+
+__global__ void __launch_bounds__(256) k_ssd_bwd_ddt(int64_t n, const float* vc, const float* vs, const float* vf,
+                                                     const float* vr, __nv_bfloat16* dc, __nv_bfloat16* df,
+                                                     __nv_bfloat16* dr) {
+  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (i >= n) return;
+  dc[i] = __float2bfloat16_rn(__fadd_rn(vc[i], vs[i]));
+  df[i] = __float2bfloat16_rn(vf[i]);
+  dr[i] = __float2bfloat16_rn(vr[i]);
+}
+
+// Per (batch row, block, head): sum of dy x of each stream (the skip terms' gradients).
+__global__ void __launch_bounds__(256) k_ssd_bwd_dd(const SsdGeo g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
+                                                    const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* part) {
+  __shared__ float red[2][8];
+  const int64_t bk = blockIdx.x, b = bk / g.nb, k = bk % g.nb;
+  const int h = blockIdx.y, t = threadIdx.x;
+  float sc = 0.f, sn = 0.f;
+  for (int64_t q = t; q < g.Bs * kSsdP; q += 256) {
+    const int64_t o = ((b * g.L + k * g.Bs + q / kSsdP) * g.H + h) * kSsdP + q % kSsdP;
+    if (dyc != nullptr) sc = __fmaf_rn(__bfloat162float(dyc[o]), __bfloat162float(xc[o]), sc);
+    sn = __fmaf_rn(__bfloat162float(dyn[o]), __bfloat162float(xn[o]), sn);
+  }
+  sc = warp_sum(sc);
+  sn = warp_sum(sn);
+  if ((t & 31) == 0) {
+    red[0][t >> 5] = sc;
+    red[1][t >> 5] = sn;
+  }
+  __syncthreads();
+  if (t < 2) {
+    float v = 0.f;
+    for (int q = 0; q < 8; ++q) v = __fadd_rn(v, red[t][q]);
+    part[(bk * g.H + h) * 2 + t] = v;
+  }
+}
+
+// Parameter gradients per head, summing the (batch row, block) partials in order.
+__global__ void __launch_bounds__(128) k_ssd_bwd_par(const SsdGeo g, const float* dA_c, const float* dA_f,
+                                                     const float* dA_s, const float* dA_r, const float* dd, float* dAf,
+                                                     float* dDf, float* dAr, float* dDr) {
+  const int h = blockIdx.x * 128 + threadIdx.x;
+  if (h >= g.H) return;
+  float af = 0.f, ar = 0.f, df = 0.f, dr = 0.f;
+  for (int64_t bk = 0; bk < g.Bt * g.nb; ++bk) {
+    const int64_t o = bk * g.H + h;
+    af = __fadd_rn(af, __fadd_rn(__fadd_rn(dA_c[o], dA_f[o]), dA_s[o]));
+    ar = __fadd_rn(ar, dA_r[o]);
+    df = __fadd_rn(df, __fadd_rn(dd[o * 2], dd[o * 2 + 1]));
+    dr = __fadd_rn(dr, dd[o * 2 + 1]);
+  }
+  dAf[h] = af;
+  dAr[h] = ar;
+  dDf[h] = df;
+  dDr[h] = dr;
+}
+
+template <int N, bool UPPER, bool SEED>
+cudaError_t bwd_tile_t(const SsdBwdTileParams& p, cudaStream_t s) {
+  const int smem = (int)TileSmem::total;
+  cudaError_t e = set_smem_cached((const void*)k_ssd_bwd_tile<N, UPPER, SEED>, smem, -1);
+  if (e != cudaSuccess) return e;
+  dim3 grid((unsigned)(p.g.Bt * p.g.nb * p.g.m), (unsigned)p.g.H);
+  k_ssd_bwd_tile<N, UPPER, SEED><<<grid, kBwdThreads, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <int N>
+cudaError_t bwd_state_t(const SsdBwdStateParams& p, cudaStream_t s) {
+  const int smem = (int)StateBwdSmem::total;
+  cudaError_t e = set_smem_cached((const void*)k_ssd_bwd_state<N>, smem, -1);
+  if (e != cudaSuccess) return e;
+  dim3 grid((unsigned)(p.g.Bt * p.g.nb), (unsigned)p.g.H);
+  k_ssd_bwd_state<N><<<grid, kBwdThreads, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_ssd_bwd_tile(bool upper, bool seeded, const SsdBwdTileParams& p, cudaStream_t s) {
+  if (p.g.N == 64) {
+    if (upper) return bwd_tile_t<64, true, false>(p, s);
+    return seeded ? bwd_tile_t<64, false, true>(p, s) : bwd_tile_t<64, false, false>(p, s);
+  }
+  if (upper) return bwd_tile_t<128, true, false>(p, s);
+  return seeded ? bwd_tile_t<128, false, true>(p, s) : bwd_tile_t<128, false, false>(p, s);
+}
+
+cudaError_t launch_ssd_bwd_vec(const SsdBwdVecParams& p, cudaStream_t s) {
+  const int64_t warps = p.g.Bt * p.g.nb * p.g.H;
+  k_ssd_bwd_vec<<<(unsigned)((warps + 3) / 4), 128, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ssd_bwd_pass(const SsdBwdPassParams& p, cudaStream_t s) {
+  const int64_t n = p.g.Bt * p.g.H * kSsdP * p.g.N;
+  k_ssd_bwd_pass<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ssd_bwd_state(const SsdBwdStateParams& p, cudaStream_t s) {
+  return p.g.N == 64 ? bwd_state_t<64>(p, s) : bwd_state_t<128>(p, s);
+}
+
+cudaError_t launch_ssd_bwd_dx(const SsdGeo& g, const float* dxp_c, const float* dxs, const float* dxp_f,
+                              const float* dxp_r, const __nv_bfloat16* dyc, const __nv_bfloat16* dyn, const float* Df,
+                              const float* Dr, __nv_bfloat16* dxc, __nv_bfloat16* dxn, cudaStream_t s) {
+  const int64_t n = g.Bt * g.L * g.H * kSsdP;
+  k_ssd_bwd_dx<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, dxp_c, dxs, dxp_f, dxp_r, dyc, dyn, Df, Dr, dxc, dxn);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, const float* dBp_c, const float* dBs, const float* dCp_c,
+                               const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
+                               __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
+                               __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s) {
+  const int64_t n = g.Bt * g.L * g.N;
+  k_ssd_bwd_dbc<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, dBp_c, dBs, dCp_c, dBp_f, dCp_f, dBp_r, dCp_r, dBc, dCc,
+                                                            dBf, dCf, dBr, dCr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ssd_bwd_ddt(int64_t n, const float* vc, const float* vs, const float* vf, const float* vr,
+                               __nv_bfloat16* dc, __nv_bfloat16* df, __nv_bfloat16* dr, cudaStream_t s) {
+  k_ssd_bwd_ddt<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(n, vc, vs, vf, vr, dc, df, dr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
+                                  const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* dd, const float* dA_c,
+                                  const float* dA_f, const float* dA_s, const float* dA_r, float* dAf, float* dDf,
+                                  float* dAr, float* dDr, cudaStream_t s) {
+  k_ssd_bwd_dd<<<dim3((unsigned)(g.Bt * g.nb), (unsigned)g.H), 256, 0, s>>>(g, xc, dyc, xn, dyn, dd);
+  cudaError_t e = api_launched(cudaGetLastError(), s);
+  if (e != cudaSuccess) return e;
+  k_ssd_bwd_par<<<(unsigned)((g.H + 127) / 128), 128, 0, s>>>(g, dA_c, dA_f, dA_s, dA_r, dd, dAf, dDf, dAr, dDr);
+  return cudaGetLastError();
+}
+
+}  // namespace bds

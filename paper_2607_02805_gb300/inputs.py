@@ -173,7 +173,8 @@ class SsdWorkload(Workload):
     [Bt, H, 64, N]. Same draws as the diagonal layer (same stream ids and value
     recipe), with these shapes; the forward-side tensors only."""
 
-    def __init__(self, batch, length, block, heads, d_state, seed=0, with_init=False, head_dim=64, part=0):
+    def __init__(self, batch, length, block, heads, d_state, seed=0, with_init=False, head_dim=64, part=0,
+                 with_grads=False, with_dstates=False):
         self.batch, self.len, self.block = int(batch), int(length), int(block)
         self.heads, self.head_dim, self.d_state = int(heads), int(head_dim), int(d_state)
         self.d_inner, self.dtype, self.seed = self.heads * self.head_dim, "bf16", int(seed)
@@ -184,10 +185,14 @@ class SsdWorkload(Workload):
                   "A_f": (H,), "A_r": (H,), "D_f": (H,), "D_r": (H,)}
         if with_init:
             shapes["init_state"] = (Bt, H, P, N)
+        if with_grads:
+            shapes.update({"dy_c": (Bt, L, H, P), "dy_n": (Bt, L, H, P)})
+        if with_dstates:
+            shapes["dstates"] = (Bt, L // self.block, H, P, N)
         self.t32 = {}
         for k, shp in shapes.items():
             a = draw(k, shp, self.seed, 0 if k in PARAMS else part)
-            if k not in PARAMS and k != "init_state":
+            if k not in PARAMS and k not in ("init_state", "dstates"):
                 a = bf16_bits_to_f32(f32_to_bf16_bits(a)).reshape(shp)
             self.t32[k] = a
 
