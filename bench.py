@@ -590,6 +590,120 @@ def run_ssd(args):
         torch.cuda.empty_cache()
 
 
+SSD_BWD_KERNELS = ("bwd_tile_clean", "bwd_tile_fwd", "bwd_tile_rev", "bwd_vec_clean", "bwd_vec_fwd", "bwd_vec_rev",
+                   "bwd_state_pass", "bwd_block_state", "bwd_dx", "bwd_dbc", "bwd_ddt", "bwd_dd", "bwd_par")
+
+
+def ssd_bwd_tile_flops(Bt, L, Bs, H, N, seeded):
+    """Tensor-core flops of one backward tile launch (one stream and
+    direction): per block, head and (tile i, s-tile j) pair the direction
+    reaches, G = C B^T (K = N), Q = dy x^T (K = 64), dC += dG B, dx = M^T dy,
+    dB = dG^T C (K = 128); per tile of a seeded block after the first, the
+    seed products (E dy) S, C S^T and C^T (E dy)."""
+    m, nb = Bs // 128, L // Bs
+    pairs = m * (m + 1) // 2
+    per_pair = 2.0 * 128 * 128 * (N + 64) + 2.0 * 128 * 128 * (2 * N + 64)
+    f = Bt * nb * H * pairs * per_pair
+    if seeded:
+        f += Bt * (nb - 1) * H * m * (2.0 * 128 * N * 64 * 2 + 2.0 * 128 * 64 * 128)
+    return f
+
+
+def run_ssd_train(args):
+    """Forward + backward of the SSD (Mamba-2) form at the paper's two model
+    sizes (training length 8192, block 256), one line each."""
+    import torch
+    from paper_2607_02805_gb300 import binding
+    from paper_2607_02805_gb300.inputs import SsdWorkload
+    from paper_2607_02805_gb300.layer import to_device
+    peaks, peak_kind = measured_peaks()
+    tc_peak = float(peaks.get("bf16_tflops", 1900.0))
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    for name, (Bt, L, Bs, H, N) in (("350M-class Mamba-2 layer: 26 heads of 64, state 128", (8, 8192, 256, 26, 128)),
+                                   ("87M-class Mamba-2 layer: 14 heads of 64, state 64", (8, 8192, 256, 14, 64))):
+        if args.batch:
+            Bt = args.batch
+        wl = SsdWorkload(Bt, L, Bs, H, N, seed=0, with_grads=True)
+        t = {k: to_device(wl.dev_bits(k), binding.BDSCAN_F32 if k in ("A_f", "A_r", "D_f", "D_r")
+                          else binding.BDSCAN_BF16, "cuda") for k in wl.t32}
+        d = binding.make_ssd_dims(Bt, L, Bs, H, N)
+        y_c = torch.empty((Bt, L, H, 64), dtype=torch.bfloat16, device="cuda")
+        y_n = torch.empty_like(y_c)
+        st = torch.empty((Bt, L // Bs, H, 64, N), dtype=torch.float32, device="cuda")
+        wsf = torch.empty(binding.bdscan_ssd_forward_workspace_size(d), dtype=torch.uint8, device="cuda")
+        wsb = torch.empty(binding.bdscan_ssd_backward_workspace_size(d), dtype=torch.uint8, device="cuda")
+        names = ("x_c", "dt_c", "B_c", "C_c", "x_n", "dt_f", "B_f", "C_f", "dt_r", "B_r", "C_r", "A_f", "D_f", "A_r",
+                 "D_r")
+        g = {k: torch.empty(t[k].shape, dtype=torch.float32 if k in ("A_f", "A_r", "D_f", "D_r") else torch.bfloat16,
+                            device="cuda") for k in names}
+        stream = torch.cuda.current_stream()
+
+        def step():
+            binding.ssd_forward(d, t, y_c, y_n, st, wsf)
+            binding.ssd_backward(d, t, st, t["dy_c"], t["dy_n"], None, g, wsb)
+
+        for _ in range(max(3, args.warmup)):
+            step()
+        steps = max(3, min(args.steps, 20))
+        nf, nb_ = len(SSD_KERNELS), len(SSD_BWD_KERNELS)
+        ev_s = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        ev_k = [[torch.cuda.Event(enable_timing=True) for _ in range(nf + nb_)] for _ in range(steps)]
+        for evs in ev_k:
+            for e in evs:
+                e.record(stream)
+        torch.cuda.synchronize()
+        arr_f = [(ctypes.c_void_p * nf)(*[e.cuda_event for e in evs[:nf]]) for evs in ev_k]
+        arr_b = [(ctypes.c_void_p * nb_)(*[e.cuda_event for e in evs[nf:]]) for evs in ev_k]
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        launches = 0
+        for i in range(steps):
+            ev_s[i].record(stream)
+            binding.bdscan_profile_events(arr_f[i], nf)
+            binding.ssd_forward(d, t, y_c, y_n, st, wsf)
+            launches = binding.bdscan_last_launch_count()
+            binding.bdscan_profile_events(arr_b[i], nb_)
+            binding.ssd_backward(d, t, st, t["dy_c"], t["dy_n"], None, g, wsb)
+            launches += binding.bdscan_last_launch_count()
+            binding.bdscan_profile_events(None, 0)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        flag = binding.bdscan_ssd_wait_flag(1)
+        ms = e0.elapsed_time(e1) / steps
+        allk = SSD_KERNELS + SSD_BWD_KERNELS
+        per = {k: [] for k in allk}
+        for i in range(steps):
+            prev = ev_s[i]
+            for j, k in enumerate(allk):
+                per[k].append(prev.elapsed_time(ev_k[i][j]))
+                prev = ev_k[i][j]
+        kern = []
+        for k in allk:
+            us = 1e3 * statistics.mean(per[k])
+            row = {"name": k, "avg_us": round(us, 2)}
+            if k.startswith("bwd_tile"):
+                fl = ssd_bwd_tile_flops(Bt, L, Bs, H, N, seeded=k != "bwd_tile_rev")
+                row["tflops"] = round(fl / (us * 1e-6) / 1e12, 1)
+                row["tensor_frac"] = round(fl / (us * 1e-6) / 1e12 / tc_peak, 4)
+            kern.append(row)
+        fwd_ms = sum(r["avg_us"] for r in kern[:nf]) / 1e3
+        bwd_ms = sum(r["avg_us"] for r in kern[nf:]) / 1e3
+        dom = max(kern, key=lambda r: r["avg_us"])
+        print(json.dumps({
+            "metric": "SSD-form block-bidirectional forward+backward tokens/s (clean + noisy stream pair counts once)",
+            "value": Bt * L / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": steps, "ms_per_step": ms,
+            "higher_is_better": True, "dtype": "bf16 operands, fp32 accumulate and state", "data": "synthetic",
+            "config": {"workload": f"{name}; batch {Bt}, {L} tokens per stream, block {Bs}; forward with every "
+                                   "block-end state, then the backward of every input", "batch": Bt, "seq_len": L,
+                       "block": Bs, "heads": H, "head_dim": 64, "d_state": N},
+            "forward_ms": round(fwd_ms, 4), "backward_ms": round(bwd_ms, 4),
+            "dominant": {"name": dom["name"], "avg_us": dom["avg_us"], "tensor_frac": dom.get("tensor_frac")},
+            "tensor_peak_tflops": tc_peak, "hbm_peak_gbs": hbm_peak, "peak_kind": peak_kind,
+            "gpu_launches": launches * steps, "wait_flag": flag, "kernels": kern}), flush=True)
+        del t, y_c, y_n, st, wsf, wsb, g
+        torch.cuda.empty_cache()
+
+
 def run_ssd_cache(args, L=65536, Bs=256, calls=16):
     """Inference cache path of the SSD form (350M-class Mamba-2 layer, 26 heads
     of 64, state 128, batch 1): cache build over an L-token prefix (final state
@@ -933,7 +1047,7 @@ def main():
     ap.add_argument("--warmup-seconds", type=float, default=1.0,
                     help="keep warming up for at least this long (clock sampling under load)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (smaller profiling case)")
-    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k", "ssd", "ssd_cache"],
+    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k", "ssd", "ssd_cache", "ssd_train"],
                     help="layer: the step line; others: extra lines on one GPU")
     args = ap.parse_args()
     if args.batch:
@@ -952,6 +1066,8 @@ def main():
                 run_ssd(args)
             elif args.workload == "ssd_cache":
                 run_ssd_cache(args)
+            elif args.workload == "ssd_train":
+                run_ssd_train(args)
             elif args.workload == "prefill65k":
                 run_prefill(args, 65536, 32, 1)
             else:
