@@ -63,25 +63,27 @@ struct SsdScanParams {
 };
 
 // Backward (ssd_bwd.cu). One stream and direction of the block-local
-// backward: per (batch row, block, 128-token tile i, head) the products
-// G = C B^T and Q = dy x^T against every s-tile of the block the direction
-// reaches, the masked decays, dC (complete for tile i), the contributions of
-// tile i to dx and dB of every s-tile (partials over i), the column sums of
-// R' = Q o G o decay (partials over i) and its row sums with dt, and for the
-// seeded forward direction the seed term's products (dC, the seed gradient
-// partial over i, the row dot dy_t . seed term_t).
+// backward: per (batch row, block, 128-token tile i, group of hg heads) the
+// products G = C B^T (shared by the heads) and Q = dy x^T against every
+// s-tile of the block the direction reaches, the masked decays, the
+// contributions of tile i to dx (per head) and to dB and dC (summed over the
+// group's heads) of every s-tile (partials over i and groups), the column
+// sums of R' = Q o G o decay (partials over i) and its row sums with dt, and
+// for the seeded forward direction the seed term's products (dC, the seed
+// gradient partial over i, the row dot dy_t . seed term_t).
 struct SsdBwdTileParams {
   SsdGeo g;
   const __nv_bfloat16 *x, *dy, *dt, *B, *C;  // x, dy [Bt][L][H][P] (dy null: zero); dt [Bt][L][H]; B, C [Bt][L][N]
   const float* A;       // [H]
   const float* states;  // seeded direction: block k reads states[b][k-1] ([Bt][nb][H][P][N])
   float* dx_part;       // [Bt*nb][H][m][Bs][P]
-  float* dB_part;       // [Bt*nb][H][m][Bs][N]
-  float* dC_part;       // [Bt*nb][H][Bs][N]
+  float* dB_part;       // [Bt*nb][groups][m][Bs][N]
+  float* dC_part;       // [Bt*nb][groups][Bs][N]
   float* col_part;      // [Bt*nb][H][m][Bs]
   float* rowsum;        // [Bt*nb][H][Bs]
   float* rowdot;        // [Bt*nb][H][Bs] (seeded direction)
   float* dS_part;       // [Bt*nb][H][m][P][N] (seeded direction)
+  int hg;               // heads per CTA (at most 16); groups = ceil(H / hg)
   int* flag;
 };
 
@@ -134,7 +136,7 @@ cudaError_t launch_ssd_bwd_state(const SsdBwdStateParams& p, cudaStream_t s);
 cudaError_t launch_ssd_bwd_dx(const SsdGeo& g, const float* dxp_c, const float* dxs, const float* dxp_f,
                               const float* dxp_r, const __nv_bfloat16* dyc, const __nv_bfloat16* dyn, const float* Df,
                               const float* Dr, __nv_bfloat16* dxc, __nv_bfloat16* dxn, cudaStream_t s);
-cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, const float* dBp_c, const float* dBs, const float* dCp_c,
+cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, const float* dBs, const float* dCp_c,
                                const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
                                __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s);

@@ -390,9 +390,25 @@ namespace {
 struct SsdBwdWs {
   size_t dxp[3], dBp[3], dCp[3], colp[3], rows[3], rowdot[3], dSp[3], ddtv[3], dAv[3];
   size_t sumdt, gS, dxs, dBs, ddts, dAs, dd, total;
+  int hg, ngrp;  // heads per tile CTA, head groups
 };
+// Head groups of the tile kernel: enough CTAs for about 1024 (several waves
+// over the SMs), at most 16 heads per CTA; a function of the dimensions only,
+// so the workspace size does not depend on the device.
+void ssd_bwd_groups(const bds::SsdGeo& g, int* hg, int* ngrp) {
+  const int64_t units = g.Bt * g.nb * g.m;
+  int64_t want = units > 0 ? (1024 + units - 1) / units : 1;
+  const int64_t lo = (g.H + 15) / 16;
+  if (want < lo) want = lo;
+  if (want > g.H) want = g.H;
+  if (want < 1) want = 1;
+  *hg = (int)((g.H + want - 1) / want);
+  *ngrp = g.H > 0 ? (g.H + *hg - 1) / *hg : 1;
+}
 SsdBwdWs ssd_bwd_ws(const bds::SsdGeo& g) {
   SsdBwdWs w;
+  ssd_bwd_groups(g, &w.hg, &w.ngrp);
+  const size_t bkg = (size_t)g.Bt * g.nb * w.ngrp;
   const size_t bkh = (size_t)g.Bt * g.nb * g.H, P = 64, N = (size_t)g.N, m = (size_t)g.m, Bs = (size_t)g.Bs;
   size_t o = 0;
   auto take = [&](size_t floats) {
@@ -402,8 +418,8 @@ SsdBwdWs ssd_bwd_ws(const bds::SsdGeo& g) {
   };
   for (int s = 0; s < 3; ++s) {
     w.dxp[s] = take(bkh * m * Bs * P);
-    w.dBp[s] = take(bkh * m * Bs * N);
-    w.dCp[s] = take(bkh * Bs * N);
+    w.dBp[s] = take(bkg * m * Bs * N);
+    w.dCp[s] = take(bkg * Bs * N);
     w.colp[s] = take(bkh * m * Bs);
     w.rows[s] = take(bkh * Bs);
     w.rowdot[s] = s < 2 ? take(bkh * Bs) : 0;
@@ -512,6 +528,7 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
     p.rowsum = F(w.rows[st]);
     p.rowdot = st < 2 ? F(w.rowdot[st]) : nullptr;
     p.dS_part = st < 2 ? F(w.dSp[st]) : nullptr;
+    p.hg = w.hg;
     p.flag = flag;
     e = bds::api_launched(bds::launch_ssd_bwd_tile(st == 2, st < 2, p, s), s);
   }
@@ -569,7 +586,7 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
                                                  params->D_f, params->D_r, (bf*)gclean->dx, (bf*)gnoisy->dx, s),
                           s);
   if (e == cudaSuccess)
-    e = bds::api_launched(bds::launch_ssd_bwd_dbc(g, F(w.dBp[0]), F(w.dBs), F(w.dCp[0]), F(w.dBp[1]), F(w.dCp[1]),
+    e = bds::api_launched(bds::launch_ssd_bwd_dbc(g, w.ngrp, F(w.dBp[0]), F(w.dBs), F(w.dCp[0]), F(w.dBp[1]), F(w.dCp[1]),
                                                   F(w.dBp[2]), F(w.dCp[2]), (bf*)gclean->dB, (bf*)gclean->dC,
                                                   (bf*)gnoisy->dB_f, (bf*)gnoisy->dC_f, (bf*)gnoisy->dB_r,
                                                   (bf*)gnoisy->dC_r, s),

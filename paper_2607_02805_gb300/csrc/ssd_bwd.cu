@@ -86,24 +86,50 @@ __device__ __forceinline__ void store_row(float* dst, const float (&v)[32]) {
   for (int e = 0; e < 32; e += 4) *reinterpret_cast<float4*>(dst + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
 }
 
-// Shared memory of k_ssd_bwd_tile (offsets from a 1024-aligned base).
-//   DY  dy of tile i, [128 t][64 p]          C   C of tile i, [128 t][128 n] (n >= N zero)
-//   X   x of s-tile j, [128 s][64 p]         BT  B of s-tile j, [128 s][N]
-//   DG  Q o decay o dt, [128 t][128 s]       M   G o decay o dt, [128 t][128 s]
-//   COL R' of 64 columns, [128][65] fp32     VEC c and dt of the block, fp32
-// The seed phase reuses X for the seed ([64 p][N], atom columns of 8 KB) and
-// BT for E o dy ([128 t][64 p]).
-struct TileSmem {
-  static constexpr uint32_t DY = 0, C = 16384, X = 49152, BT = 65536, DG = 98304, M = 131072, COL = 163840;
-  static constexpr uint32_t VEC = COL + 128u * 65u * 4u;
-  static constexpr uint32_t total = VEC + 2u * 256u * 4u + 1024u;
-};
+// 32 consecutive fp32 columns of this thread's TMEM lane, written (the
+// counterpart of umma::tmem_ld32); tmem_wait_st() orders them before later loads.
+__device__ __forceinline__ void tmem_st32(uint32_t ta, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};\n" ::"r"(ta),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])), "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])), "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])), "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])), "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])), "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])), "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31])));
+}
 
-// One CTA of 4 warps per (batch row, block, tile i) and head: thread t owns
-// token row t of tile i (TMEM lane t) for the row-side products and row s = t
-// of s-tile j for the column-side ones. TMEM: G at columns 0..127 and Q at
-// 128..255 (then dx_j at 0..63, dB_j at 64..64+N), dC at 256, C S^T at 384,
-// dS^T at 448.
+// Shared memory of k_ssd_bwd_tile (offsets from a 1024-aligned base).
+//   C    C of tile i, [128 t][128 n] (n >= N zero)    BT  B of s-tile j, [128 s][N]
+//   X    x of s-tile j, one head, [128 s][64 p]       DY  dy of tile i, one head, [128 t][64 p]
+//   M    one head's G o decay o dt, [128 t][128 s]
+//   COL  R' of 64 columns, [128][65] fp32             VEC c and dt of one head's block
+//   ROWS row sums and row dots per head of the group, [16][128] fp32 each
+// After a s-tile's heads, the head-summed dG goes to M (bf16 high part) and
+// X + DY (low part). The seed phase uses DY, BT for E o dy, M for the seed's
+// bf16 high and low parts.
+struct TileSmem {
+  static constexpr uint32_t C = 0, BT = 32768, X = 65536, DY = 81920, M = 98304, COL = 131072;
+  static constexpr uint32_t VEC = COL + 128u * 65u * 4u;
+  static constexpr uint32_t ROWS = VEC + 2u * 256u * 4u;
+  static constexpr uint32_t total = ROWS + 2u * 16u * 128u * 4u + 1024u;
+};
+constexpr int kMaxBwdHeads = 16;  // heads per tile CTA
+
+// dt of head h over the block into s_dt, and its in-block cumulative sums
+// (inclusive; suffix sums for the reverse direction) into s_c by warp 0.
+template <bool UPPER>
+__device__ __forceinline__ void block_dt(const __nv_bfloat16* dt, int64_t tok0, int H, int h, int Bs, float* s_dt,
+                                         float* s_c) {
+  for (int s = threadIdx.x; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(dt[(tok0 + s) * H + h]);
+  if ((threadIdx.x >> 5) == 0) warp_scan_dt<UPPER>(dt + tok0 * H + h, H, Bs, s_c);
+}
+
+// One CTA of 4 warps per (batch row, block, tile i) and group of heads: thread
+// t owns token row t of tile i (TMEM lane t) for the row-side products and
+// row s = t of s-tile j for the column-side ones. Per s-tile j the Gram tile
+// G = C_i B_j^T is shared by the group's heads; per head, Q = dy x^T, the
+// masked decays, the column sums of R', dx_j = M^T dy, and dG = Q o decay o dt
+// summed over the heads in fp32 in TMEM. dC and dB_j then take the
+// head-summed dG once (B and C are shared by the heads), split into bf16 high
+// and low parts. TMEM: G, then dB_j (and the seed products) at 0; Q, then
+// dx_j at 128; the head sum of dG at 256; dC at 384.
 template <int N, bool UPPER, bool SEED>
 __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTileParams p) {
   extern __shared__ unsigned char smraw[];
@@ -117,42 +143,48 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
   const int i = (int)(idx % m);
   const int64_t bk = idx / m, b = bk / g.nb;
   const int k = (int)(bk % g.nb);
-  const int h = blockIdx.y;
+  const int grp = blockIdx.y, ngrp = gridDim.y;
+  const int h0 = grp * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
   const int64_t tok0 = b * g.L + (int64_t)k * Bs;  // the block's first token
   const int64_t HP = (int64_t)H * kSsdP;
   float* s_c = reinterpret_cast<float*>(sm + S::VEC);
   float* s_dt = s_c + 256;
   float* s_col = reinterpret_cast<float*>(sm + S::COL);
+  float* s_rows = reinterpret_cast<float*>(sm + S::ROWS);  // [hh][128]
+  float* s_dots = s_rows + kMaxBwdHeads * 128;
 
-  stage_bf16(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
   stage_bf16(sm + S::C, p.C + (tok0 + i * kSsdT) * N, N, 128, N);
   if (N == 64)
     for (int c = t; c < 128 * 8; c += kBwdThreads) *reinterpret_cast<uint4*>(sm + S::C + kTile16 + c * 16) = make_uint4(0u, 0u, 0u, 0u);
   cp_async_commit();
-  for (int s = t; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
-  if (w == 0) warp_scan_dt<UPPER>(p.dt + tok0 * H + h, H, Bs, s_c);
+  for (int hh = 0; hh < kMaxBwdHeads; ++hh) {
+    s_rows[hh * 128 + t] = 0.f;
+    s_dots[hh * 128 + t] = 0.f;
+  }
   if (t == 0) umma::bar_init(&bar, 1);
   if (w == 0) tmem_alloc(&tslot, 512);
   umma::fence_before_sync();
   __syncthreads();
   umma::fence_after_sync();
   const uint32_t tm = tslot, lane_base = tm + ((uint32_t)(32 * w) << 16);
-  const float A2 = __fmul_rn(p.A[h], kLog2e);
   const int tt = i * kSsdT + t;
-  const float ct = s_c[tt];
-  float rowsum = 0.f;
   uint32_t phase = 0;
   bool alive = true;
   const uint32_t y0 = umma::smem_u32(sm + S::DY), c0 = umma::smem_u32(sm + S::C), x0 = umma::smem_u32(sm + S::X),
-                 b0 = umma::smem_u32(sm + S::BT), dg0 = umma::smem_u32(sm + S::DG), m0 = umma::smem_u32(sm + S::M);
+                 b0 = umma::smem_u32(sm + S::BT), m0 = umma::smem_u32(sm + S::M);
   constexpr uint32_t id_gq = umma::idesc_bf16(128, 128, false, false);
   constexpr uint32_t id_dc = umma::idesc_bf16(128, N, false, true);
   constexpr uint32_t id_dx = umma::idesc_bf16(128, 64, true, true);
   constexpr uint32_t id_db = umma::idesc_bf16(128, N, true, true);
+  auto wait_mma = [&]() {
+    if (!cta_wait(&bar, phase, p.flag)) return false;
+    phase ^= 1u;
+    umma::fence_after_sync();
+    return true;
+  };
   const int j0 = UPPER ? i : 0, j1 = UPPER ? m - 1 : i;
-  for (int j = j0; j <= j1; ++j) {
+  for (int j = j0; j <= j1 && alive; ++j) {
     const int64_t sr0 = tok0 + (int64_t)j * kSsdT;
-    stage_bf16(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
     stage_bf16(sm + S::BT, p.B + sr0 * N, N, 128, N);
     cp_async_commit();
     cp_async_wait_all();
@@ -162,64 +194,121 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
     if (t == 0) {
       umma::fence_after_sync();
 #pragma unroll
-      for (int kk = 0; kk < N / 16; ++kk) {  // G = C_i B_j^T
+      for (int kk = 0; kk < N / 16; ++kk) {  // G = C_i B_j^T, shared by the heads
         const uint32_t off = (uint32_t)(kk >> 2) * kTile16 + (uint32_t)(kk & 3) * 32u;
         umma::mma_bf16(tm, umma::sdesc(c0 + off, 16, 1024), umma::sdesc(b0 + off, 16, 1024), id_gq, kk > 0);
       }
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk)  // Q = dy_i x_j^T
-        umma::mma_bf16(tm + 128u, umma::sdesc(y0 + kk * 32u, 16, 1024), umma::sdesc(x0 + kk * 32u, 16, 1024), id_gq,
-                       kk > 0);
       umma::mma_commit(&bar);
     }
-    if (!cta_wait(&bar, phase, p.flag)) {
-      alive = false;
-      break;
-    }
-    phase ^= 1u;
-    umma::fence_after_sync();
-    // decay-weighted tiles of this row: dG = Q decay dt (DG) and M = G decay dt
-    // (M) in bf16, R' for the column sums and R for the row sum in fp32
-#pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
-      float gv[32], qv[32];
-      umma::tmem_ld32(lane_base + 32u * (uint32_t)c, gv);
-      umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)c, qv);
-      uint32_t dgp[16], mp[16];
+    if (!(alive = wait_mma())) break;
+    for (int hh = 0; hh < hg; ++hh) {
+      const int h = h0 + hh;
+      stage_bf16(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
+      stage_bf16(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+      cp_async_commit();
+      block_dt<UPPER>(p.dt, tok0, H, h, Bs, s_dt, s_c);
+      cp_async_wait_all();
+      umma::fence_async_smem();
+      umma::fence_before_sync();
+      __syncthreads();
+      if (t == 0) {
+        umma::fence_after_sync();
 #pragma unroll
-      for (int e = 0; e < 32; e += 2) {
-        float dgv[2], mv[2];
+        for (int kk = 0; kk < 4; ++kk)  // Q = dy_i x_j^T
+          umma::mma_bf16(tm + 128u, umma::sdesc(y0 + kk * 32u, 16, 1024), umma::sdesc(x0 + kk * 32u, 16, 1024),
+                         id_gq, kk > 0);
+        umma::mma_commit(&bar);
+      }
+      if (!(alive = wait_mma())) break;
+      const float A2 = __fmul_rn(p.A[h], kLog2e), ct = s_c[tt];
+      float rowsum = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float gv[32], qv[32], dgs[32];
+        umma::tmem_ld32(lane_base + 32u * (uint32_t)c, gv);
+        umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)c, qv);
+        if (hh > 0) umma::tmem_ld32(lane_base + 256u + 32u * (uint32_t)c, dgs);
+        uint32_t mp[16];
+#pragma unroll
+        for (int e = 0; e < 32; e += 2) {
+          float mv[2];
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            const int s = j * kSsdT + 32 * c + e + q;
+            const bool valid = UPPER ? (s >= tt) : (s <= tt);
+            const float L = valid ? ex2(__fmul_rn(A2, __fsub_rn(ct, s_c[s]))) : 0.f;
+            const float ds = s_dt[s];
+            const float gl = __fmul_rn(gv[e + q], L);
+            const float rp = __fmul_rn(qv[e + q], gl);
+            rowsum = __fmaf_rn(rp, ds, rowsum);
+            s_col[t * 65 + 32 * (c & 1) + e + q] = rp;
+            const float dg = __fmul_rn(__fmul_rn(qv[e + q], L), ds);
+            dgs[e + q] = hh > 0 ? __fadd_rn(dgs[e + q], dg) : dg;
+            mv[q] = __fmul_rn(gl, ds);
+          }
+          mp[e >> 1] = pack_bf16(mv[0], mv[1]);
+        }
+        tmem_st32(lane_base + 256u + 32u * (uint32_t)c, dgs);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int chunk = 4 * c + u;
+          const uint32_t off = (uint32_t)(chunk >> 3) * kTile16 + sw128((uint32_t)t, (uint32_t)(chunk & 7));
+          *reinterpret_cast<uint4*>(sm + S::M + off) = make_uint4(mp[4 * u], mp[4 * u + 1], mp[4 * u + 2], mp[4 * u + 3]);
+        }
+        if (c & 1) {  // column sums of R' over the tile's 128 rows, 64 columns at a time
+          __syncthreads();
+          if (t < 64) {
+            float sum = 0.f;
+            for (int r = 0; r < 128; ++r) sum = __fadd_rn(sum, s_col[r * 65 + t]);
+            p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + 64 * (c >> 1) + t] = sum;
+          }
+          __syncthreads();
+        }
+      }
+      s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);
+      tmem_wait_st();
+      umma::fence_async_smem();
+      umma::fence_before_sync();
+      __syncthreads();
+      if (t == 0) {
+        umma::fence_after_sync();
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)  // dx_j = M^T dy_i: M read as an MN-major operand (M = s, K = t)
+          umma::mma_bf16(tm + 128u, umma::sdesc(m0 + kk * 2048u, kTile16, 1024), umma::sdesc(y0 + kk * 2048u, kTile16, 1024),
+                         id_dx, kk > 0);
+        umma::mma_commit(&bar);
+      }
+      if (!(alive = wait_mma())) break;
+      {  // row s = j*128 + t of head h's dx contribution from tile i
+        float v[32];
+        float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * kSsdP;
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
-          const int s = j * kSsdT + 32 * c + e + q;
-          const bool valid = UPPER ? (s >= tt) : (s <= tt);
-          const float L = valid ? ex2(__fmul_rn(A2, __fsub_rn(ct, s_c[s]))) : 0.f;
-          const float ds = s_dt[s];
-          const float gl = __fmul_rn(gv[e + q], L);
-          const float rp = __fmul_rn(qv[e + q], gl);
-          rowsum = __fmaf_rn(rp, ds, rowsum);
-          s_col[t * 65 + 32 * (c & 1) + e + q] = rp;
-          dgv[q] = __fmul_rn(__fmul_rn(qv[e + q], L), ds);
-          mv[q] = __fmul_rn(gl, ds);
+          umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)q, v);
+          store_row(dxo + 32 * q, v);
         }
-        dgp[e >> 1] = pack_bf16(dgv[0], dgv[1]);
-        mp[e >> 1] = pack_bf16(mv[0], mv[1]);
+      }
+      umma::fence_before_sync();
+    }
+    if (!alive) break;
+    // the head-summed dG as bf16 high (M) and low (X + DY) parts
+#pragma unroll 1
+    for (int c = 0; c < 4; ++c) {
+      float dgs[32];
+      umma::tmem_ld32(lane_base + 256u + 32u * (uint32_t)c, dgs);
+      uint32_t hi[16], lo[16];
+#pragma unroll
+      for (int e = 0; e < 32; e += 2) {
+        const __nv_bfloat162 hv = __floats2bfloat162_rn(dgs[e], dgs[e + 1]);
+        hi[e >> 1] = *reinterpret_cast<const uint32_t*>(&hv);
+        lo[e >> 1] = pack_bf16(__fsub_rn(dgs[e], __low2float(hv)), __fsub_rn(dgs[e + 1], __high2float(hv)));
       }
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const int chunk = 4 * c + u;
         const uint32_t off = (uint32_t)(chunk >> 3) * kTile16 + sw128((uint32_t)t, (uint32_t)(chunk & 7));
-        *reinterpret_cast<uint4*>(sm + S::DG + off) = make_uint4(dgp[4 * u], dgp[4 * u + 1], dgp[4 * u + 2], dgp[4 * u + 3]);
-        *reinterpret_cast<uint4*>(sm + S::M + off) = make_uint4(mp[4 * u], mp[4 * u + 1], mp[4 * u + 2], mp[4 * u + 3]);
-      }
-      if (c & 1) {  // column sums of R' over the tile's 128 rows, 64 columns at a time
-        __syncthreads();
-        if (t < 64) {
-          float sum = 0.f;
-          for (int r = 0; r < 128; ++r) sum = __fadd_rn(sum, s_col[r * 65 + t]);
-          p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + 64 * (c >> 1) + t] = sum;
-        }
-        __syncthreads();
+        *reinterpret_cast<uint4*>(sm + S::M + off) = make_uint4(hi[4 * u], hi[4 * u + 1], hi[4 * u + 2], hi[4 * u + 3]);
+        *reinterpret_cast<uint4*>(sm + S::X + off) = make_uint4(lo[4 * u], lo[4 * u + 1], lo[4 * u + 2], lo[4 * u + 3]);
       }
     }
     umma::fence_async_smem();
@@ -228,117 +317,120 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
     if (t == 0) {
       umma::fence_after_sync();
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t koff = (uint32_t)(kk >> 2) * kTile16 + (uint32_t)(kk & 3) * 32u, mn = (uint32_t)kk * 2048u;
-        // dC += dG_j B_j: dG K-major [t][s], B_j MN-major [s][n]
-        umma::mma_bf16(tm + 256u, umma::sdesc(dg0 + koff, 16, 1024), umma::sdesc(b0 + mn, kTile16, 1024), id_dc,
-                       j != j0 || kk > 0);
-        // dx_j = M_j^T dy_i: M read as an MN-major operand (M = s, K = t)
-        umma::mma_bf16(tm, umma::sdesc(m0 + mn, kTile16, 1024), umma::sdesc(y0 + mn, kTile16, 1024), id_dx, kk > 0);
-        // dB_j = dG_j^T C_i
-        umma::mma_bf16(tm + 64u, umma::sdesc(dg0 + mn, kTile16, 1024), umma::sdesc(c0 + mn, kTile16, 1024), id_db,
-                       kk > 0);
+      for (int part = 0; part < 2; ++part) {
+        const uint32_t dg0 = part ? x0 : m0;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t koff = (uint32_t)(kk >> 2) * kTile16 + (uint32_t)(kk & 3) * 32u, mn = (uint32_t)kk * 2048u;
+          // dC += dG B_j: dG K-major [t][s], B_j MN-major [s][n]
+          umma::mma_bf16(tm + 384u, umma::sdesc(dg0 + koff, 16, 1024), umma::sdesc(b0 + mn, kTile16, 1024), id_dc,
+                         j != j0 || part > 0 || kk > 0);
+          // dB_j = dG^T C_i: dG read as MN-major (M = s)
+          umma::mma_bf16(tm, umma::sdesc(dg0 + mn, kTile16, 1024), umma::sdesc(c0 + mn, kTile16, 1024), id_db,
+                         part > 0 || kk > 0);
+        }
       }
       umma::mma_commit(&bar);
     }
-    if (!cta_wait(&bar, phase, p.flag)) {
-      alive = false;
-      break;
-    }
-    phase ^= 1u;
-    umma::fence_after_sync();
-    {  // row s = j*128 + t of tile i's contributions to dx and dB
+    if (!(alive = wait_mma())) break;
+    {  // row s = j*128 + t of the group's dB contribution from tile i
       float v[32];
-      float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * kSsdP;
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
-        store_row(dxo + 32 * q, v);
-      }
-      float* dbo = p.dB_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * N;
+      float* dbo = p.dB_part + (((bk * ngrp + grp) * m + i) * Bs + j * kSsdT + t) * N;
 #pragma unroll
       for (int q = 0; q < N / 32; ++q) {
-        umma::tmem_ld32(lane_base + 64u + 32u * (uint32_t)q, v);
+        umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
         store_row(dbo + 32 * q, v);
       }
     }
     umma::fence_before_sync();
   }
 
-  if (alive) {
-    p.rowsum[(bk * H + h) * Bs + tt] = rowsum;
-    if (SEED) {
-      float rowdot = 0.f;
-      if (k > 0) {
-        // the seed (the clean state before the block) as bf16, E o dy
-        stage_f32_as_bf16(sm + S::X, p.states + ((b * g.nb + k - 1) * H + h) * (int64_t)kSsdP * N, 64, N, false);
-        const float E = ex2(__fmul_rn(A2, ct));
+  if (alive && SEED && k > 0) {
+    // seed products per head: dC += (E o dy) S, the row dot dy_t . E_t (C_t S^T)
+    // and the seed gradient (E o dy)^T C; the seed as bf16 high and low parts
+    constexpr uint32_t id_cs = umma::idesc_bf16(128, 64, false, false);
+    for (int hh = 0; hh < hg && alive; ++hh) {
+      const int h = h0 + hh;
+      stage_bf16(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+      cp_async_commit();
+      const float* seed = p.states + ((b * g.nb + k - 1) * H + h) * (int64_t)kSsdP * N;
+      stage_f32_as_bf16(sm + S::M, seed, 64, N, false);
+      stage_f32_as_bf16(sm + S::M + 16384u, seed, 64, N, true);
+      block_dt<false>(p.dt, tok0, H, h, Bs, s_dt, s_c);
+      cp_async_wait_all();
+      __syncthreads();
+      const float E = ex2(__fmul_rn(__fmul_rn(p.A[h], kLog2e), s_c[tt]));
 #pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-          const uint4 u = *reinterpret_cast<const uint4*>(sm + S::DY + sw128((uint32_t)t, (uint32_t)ch));
-          const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&u);
-          uint32_t o[4];
+      for (int ch = 0; ch < 8; ++ch) {
+        const uint4 u = *reinterpret_cast<const uint4*>(sm + S::DY + sw128((uint32_t)t, (uint32_t)ch));
+        const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&u);
+        uint32_t o[4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 f = __bfloat1622float2(v2[e]);
-            o[e] = pack_bf16(__fmul_rn(E, f.x), __fmul_rn(E, f.y));
-          }
-          *reinterpret_cast<uint4*>(sm + S::BT + sw128((uint32_t)t, (uint32_t)ch)) = make_uint4(o[0], o[1], o[2], o[3]);
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(v2[e]);
+          o[e] = pack_bf16(__fmul_rn(E, f.x), __fmul_rn(E, f.y));
         }
-        umma::fence_async_smem();
-        umma::fence_before_sync();
-        __syncthreads();
-        if (t == 0) {
-          umma::fence_after_sync();
-          constexpr uint32_t id_cs = umma::idesc_bf16(128, 64, false, false);
+        *reinterpret_cast<uint4*>(sm + S::BT + sw128((uint32_t)t, (uint32_t)ch)) = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+      umma::fence_async_smem();
+      umma::fence_before_sync();
+      __syncthreads();
+      if (t == 0) {
+        umma::fence_after_sync();
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)  // dC += (E o dy) S: S as MN-major [p][n], atom columns of 8 KB
-            umma::mma_bf16(tm + 256u, umma::sdesc(b0 + kk * 32u, 16, 1024), umma::sdesc(x0 + kk * 2048u, 8192, 1024),
+        for (int part = 0; part < 2; ++part) {
+          const uint32_t s0 = m0 + (part ? 16384u : 0u);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)  // dC += (E o dy) S: S MN-major [p][n], atom columns of 8 KB
+            umma::mma_bf16(tm + 384u, umma::sdesc(b0 + kk * 32u, 16, 1024), umma::sdesc(s0 + kk * 2048u, 8192, 1024),
                            id_dc, true);
 #pragma unroll
-          for (int kk = 0; kk < N / 16; ++kk)  // C S^T: S as K-major [p][n]
-            umma::mma_bf16(tm + 384u, umma::sdesc(c0 + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
-                           umma::sdesc(x0 + (kk >> 2) * 8192u + (kk & 3) * 32u, 16, 1024), id_cs, kk > 0);
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk)  // dS^T = C_i^T (E o dy): C read as MN-major (M = n)
-            umma::mma_bf16(tm + 448u, umma::sdesc(c0 + kk * 2048u, kTile16, 1024),
-                           umma::sdesc(b0 + kk * 2048u, kTile16, 1024), id_dx, kk > 0);
-          umma::mma_commit(&bar);
+          for (int kk = 0; kk < N / 16; ++kk)  // C S^T: S K-major [p][n]
+            umma::mma_bf16(tm, umma::sdesc(c0 + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
+                           umma::sdesc(s0 + (kk >> 2) * 8192u + (kk & 3) * 32u, 16, 1024), id_cs, part > 0 || kk > 0);
         }
-        if (cta_wait(&bar, phase, p.flag)) {
-          phase ^= 1u;
-          umma::fence_after_sync();
-          float v[32];
 #pragma unroll
-          for (int q = 0; q < 2; ++q) {  // dy_t . (C_t S^T)
-            umma::tmem_ld32(lane_base + 384u + 32u * (uint32_t)q, v);
+        for (int kk = 0; kk < 8; ++kk)  // dS^T = C_i^T (E o dy): C read as MN-major (M = n)
+          umma::mma_bf16(tm + 64u, umma::sdesc(c0 + kk * 2048u, kTile16, 1024), umma::sdesc(b0 + kk * 2048u, kTile16, 1024),
+                         id_dx, kk > 0);
+        umma::mma_commit(&bar);
+      }
+      if (!(alive = wait_mma())) break;
+      float v[32], rowdot = 0.f;
 #pragma unroll
-            for (int e = 0; e < 32; ++e) rowdot = __fmaf_rn(tile_at(sm + S::DY, t, 32 * q + e), v[e], rowdot);
-          }
-          rowdot = __fmul_rn(E, rowdot);
-          if (32 * w < N) {  // row n = t of dS^T: the seed gradient partial [p][n]
-            float* dso = p.dS_part + ((bk * H + h) * m + i) * (int64_t)kSsdP * N + t;
+      for (int q = 0; q < 2; ++q) {
+        umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
 #pragma unroll
-            for (int q = 0; q < 2; ++q) {
-              umma::tmem_ld32(lane_base + 448u + 32u * (uint32_t)q, v);
+        for (int e = 0; e < 32; ++e) rowdot = __fmaf_rn(tile_at(sm + S::DY, t, 32 * q + e), v[e], rowdot);
+      }
+      s_dots[hh * 128 + t] = __fmul_rn(E, rowdot);
+      if (32 * w < N) {  // row n = t of dS^T: the seed gradient partial [p][n]
+        float* dso = p.dS_part + ((bk * H + h) * m + i) * (int64_t)kSsdP * N + t;
 #pragma unroll
-              for (int e = 0; e < 32; ++e) dso[(int64_t)(32 * q + e) * N] = v[e];
-            }
-          }
-        } else {
-          alive = false;
+        for (int q = 0; q < 2; ++q) {
+          umma::tmem_ld32(lane_base + 64u + 32u * (uint32_t)q, v);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) dso[(int64_t)(32 * q + e) * N] = v[e];
         }
       }
-      p.rowdot[(bk * H + h) * Bs + tt] = rowdot;
+      umma::fence_before_sync();
+      __syncthreads();  // DY, BT and M are restaged for the next head
     }
-    if (alive) {  // dC of row t of tile i
+  }
+  if (alive) {
+    {  // dC of row t of tile i, summed over the group's heads
       float v[32];
-      float* dco = p.dC_part + ((bk * H + h) * Bs + tt) * N;
+      float* dco = p.dC_part + ((bk * ngrp + grp) * Bs + tt) * N;
 #pragma unroll
       for (int q = 0; q < N / 32; ++q) {
-        umma::tmem_ld32(lane_base + 256u + 32u * (uint32_t)q, v);
+        umma::tmem_ld32(lane_base + 384u + 32u * (uint32_t)q, v);
         store_row(dco + 32 * q, v);
       }
+    }
+    for (int hh = 0; hh < hg; ++hh) {
+      const int h = h0 + hh;
+      p.rowsum[(bk * H + h) * Bs + tt] = s_rows[hh * 128 + t];
+      if (SEED) p.rowdot[(bk * H + h) * Bs + tt] = s_dots[hh * 128 + t];
     }
   }
   cp_async_wait_all();
@@ -623,9 +715,9 @@ __global__ void __launch_bounds__(256) k_ssd_bwd_dx(const SsdGeo g, const float*
   dxn[idx] = __float2bfloat16_rn(n);
 }
 
-// dB and dC of the three streams: per head the tile partials (and the clean
-// state term), summed over the heads in order.
-__global__ void __launch_bounds__(256) k_ssd_bwd_dbc(const SsdGeo g, const float* dBp_c, const float* dBs,
+// dB and dC of the three streams: the tile partials of every head group (and
+// the clean state term of every head), summed in order.
+__global__ void __launch_bounds__(256) k_ssd_bwd_dbc(const SsdGeo g, int ngrp, const float* dBp_c, const float* dBs,
                                                      const float* dCp_c, const float* dBp_f, const float* dCp_f,
                                                      const float* dBp_r, const float* dCp_r, __nv_bfloat16* dBc,
                                                      __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
@@ -638,17 +730,17 @@ __global__ void __launch_bounds__(256) k_ssd_bwd_dbc(const SsdGeo g, const float
   const int64_t k = tl / g.Bs, s = tl % g.Bs, bk = b * g.nb + k;
   const int j = (int)(s / kSsdT);
   float bc = 0.f, cc = 0.f, bf = 0.f, cf = 0.f, br = 0.f, cr = 0.f;
-  for (int h = 0; h < g.H; ++h) {
-    const int64_t hb = bk * g.H + h;
-    auto tp = [&](const float* a, int i) { return a[((hb * m + i) * g.Bs + s) * N + n]; };
+  for (int q = 0; q < ngrp; ++q) {
+    const int64_t gb = bk * ngrp + q;
+    auto tp = [&](const float* a, int i) { return a[((gb * m + i) * g.Bs + s) * N + n]; };
     for (int i = j; i < m; ++i) bc = __fadd_rn(bc, tp(dBp_c, i));
-    bc = __fadd_rn(bc, dBs[(hb * g.Bs + s) * N + n]);
-    cc = __fadd_rn(cc, dCp_c[(hb * g.Bs + s) * N + n]);
+    cc = __fadd_rn(cc, dCp_c[(gb * g.Bs + s) * N + n]);
     for (int i = j; i < m; ++i) bf = __fadd_rn(bf, tp(dBp_f, i));
-    cf = __fadd_rn(cf, dCp_f[(hb * g.Bs + s) * N + n]);
+    cf = __fadd_rn(cf, dCp_f[(gb * g.Bs + s) * N + n]);
     for (int i = 0; i <= j; ++i) br = __fadd_rn(br, tp(dBp_r, i));
-    cr = __fadd_rn(cr, dCp_r[(hb * g.Bs + s) * N + n]);
+    cr = __fadd_rn(cr, dCp_r[(gb * g.Bs + s) * N + n]);
   }
+  for (int h = 0; h < g.H; ++h) bc = __fadd_rn(bc, dBs[((bk * g.H + h) * g.Bs + s) * N + n]);
   dBc[idx] = __float2bfloat16_rn(bc);
   dCc[idx] = __float2bfloat16_rn(cc);
   dBf[idx] = __float2bfloat16_rn(bf);
@@ -718,7 +810,7 @@ cudaError_t bwd_tile_t(const SsdBwdTileParams& p, cudaStream_t s) {
   const int smem = (int)TileSmem::total;
   cudaError_t e = set_smem_cached((const void*)k_ssd_bwd_tile<N, UPPER, SEED>, smem, -1);
   if (e != cudaSuccess) return e;
-  dim3 grid((unsigned)(p.g.Bt * p.g.nb * p.g.m), (unsigned)p.g.H);
+  dim3 grid((unsigned)(p.g.Bt * p.g.nb * p.g.m), (unsigned)((p.g.H + p.hg - 1) / p.hg));
   k_ssd_bwd_tile<N, UPPER, SEED><<<grid, kBwdThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
@@ -768,12 +860,12 @@ cudaError_t launch_ssd_bwd_dx(const SsdGeo& g, const float* dxp_c, const float* 
   return cudaGetLastError();
 }
 
-cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, const float* dBp_c, const float* dBs, const float* dCp_c,
+cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, const float* dBs, const float* dCp_c,
                                const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
                                __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s) {
   const int64_t n = g.Bt * g.L * g.N;
-  k_ssd_bwd_dbc<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, dBp_c, dBs, dCp_c, dBp_f, dCp_f, dBp_r, dCp_r, dBc, dCc,
+  k_ssd_bwd_dbc<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, ngrp, dBp_c, dBs, dCp_c, dBp_f, dCp_f, dBp_r, dCp_r, dBc, dCc,
                                                             dBf, dCf, dBr, dCr);
   return cudaGetLastError();
 }
