@@ -524,18 +524,44 @@ __global__ void __launch_bounds__(256) k_ssd_bwd_pass(const SsdBwdPassParams p) 
   const int64_t pn = r - (int64_t)h * PN;
   const float A2 = __fmul_rn(p.A[h], kLog2e);
   float gS = 0.f;
-  for (int k = g.nb - 1; k >= 0; --k) {
-    const int64_t o = ((b * g.nb + k) * g.H + h) * PN + pn;
-    if (k + 1 < g.nb) {  // the seed gradients of block k+1 (forward noisy direction, then clean)
-      const int64_t base = ((b * g.nb + k + 1) * g.H + h) * (int64_t)g.m * PN + pn;
-      float inj = 0.f;
-      for (int i = 0; i < g.m; ++i) inj = __fadd_rn(inj, p.dS_f[base + i * PN]);
-      for (int i = 0; i < g.m; ++i) inj = __fadd_rn(inj, p.dS_c[base + i * PN]);
-      gS = __fadd_rn(gS, inj);
+  // m is 1 or 2 (blocks of 128 or 256 tokens). The loads of U blocks are
+  // issued before the reverse recurrence uses them: they do not depend on gS.
+  const bool two = g.m > 1;
+  constexpr int U = 8;
+  for (int k0 = g.nb - 1; k0 >= 0; k0 -= U) {
+    float f0[U], f1[U], c0[U], c1[U], ext[U], sdt[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int k = k0 - u;
+      f0[u] = f1[u] = c0[u] = c1[u] = ext[u] = sdt[u] = 0.f;
+      if (k < 0) continue;
+      if (k + 1 < g.nb) {  // the seed gradients of block k+1 (forward noisy direction, then clean)
+        const int64_t base = ((b * g.nb + k + 1) * g.H + h) * (int64_t)g.m * PN + pn;
+        f0[u] = p.dS_f[base];
+        c0[u] = p.dS_c[base];
+        if (two) {
+          f1[u] = p.dS_f[base + PN];
+          c1[u] = p.dS_c[base + PN];
+        }
+      }
+      if (p.dstates != nullptr) ext[u] = p.dstates[((b * g.nb + k) * g.H + h) * PN + pn];
+      sdt[u] = p.sumdt[(b * g.nb + k) * g.H + h];
     }
-    if (p.dstates != nullptr) gS = __fadd_rn(gS, p.dstates[o]);
-    p.gS[o] = gS;
-    gS = __fmul_rn(ex2(__fmul_rn(A2, p.sumdt[(b * g.nb + k) * g.H + h])), gS);
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int k = k0 - u;
+      if (k < 0) break;
+      if (k + 1 < g.nb) {
+        float inj = f0[u];
+        if (two) inj = __fadd_rn(inj, f1[u]);
+        inj = __fadd_rn(inj, c0[u]);
+        if (two) inj = __fadd_rn(inj, c1[u]);
+        gS = __fadd_rn(gS, inj);
+      }
+      if (p.dstates != nullptr) gS = __fadd_rn(gS, ext[u]);
+      p.gS[((b * g.nb + k) * g.H + h) * PN + pn] = gS;
+      gS = __fmul_rn(ex2(__fmul_rn(A2, sdt[u])), gS);
+    }
   }
 }
 
@@ -690,57 +716,80 @@ namespace {
 
 // dx of both streams: the tile partials of every tile that reaches s (tiles
 // i >= j(s) forward, i <= j(s) reverse), the clean state term and the skip
-// terms.
+// terms. One CTA row (blockIdx.x) per token, threads over (head, channel).
 __global__ void __launch_bounds__(256) k_ssd_bwd_dx(const SsdGeo g, const float* dxp_c, const float* dxs,
                                                     const float* dxp_f, const float* dxp_r, const __nv_bfloat16* dyc,
                                                     const __nv_bfloat16* dyn, const float* Df, const float* Dr,
                                                     __nv_bfloat16* dxc, __nv_bfloat16* dxn) {
-  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  const int64_t total = g.Bt * g.L * g.H * kSsdP;
-  if (idx >= total) return;
-  const int pp = (int)(idx % kSsdP);
-  const int h = (int)((idx / kSsdP) % g.H);
-  const int64_t bt = idx / ((int64_t)g.H * kSsdP), b = bt / g.L, tl = bt % g.L;
-  const int64_t k = tl / g.Bs, s = tl % g.Bs, bk = b * g.nb + k;
-  const int j = (int)(s / kSsdT), m = g.m;
-  auto at = [&](const float* a, int i) { return a[(((bk * g.H + h) * m + i) * g.Bs + s) * kSsdP + pp]; };
-  float c = 0.f, n = 0.f;
-  for (int i = j; i < m; ++i) c = __fadd_rn(c, at(dxp_c, i));
-  c = __fadd_rn(c, dxs[((bk * g.H + h) * g.Bs + s) * kSsdP + pp]);
-  if (dyc != nullptr) c = __fmaf_rn(Df[h], __bfloat162float(dyc[idx]), c);
-  for (int i = j; i < m; ++i) n = __fadd_rn(n, at(dxp_f, i));
-  for (int i = 0; i <= j; ++i) n = __fadd_rn(n, at(dxp_r, i));
-  n = __fmaf_rn(__fadd_rn(Df[h], Dr[h]), __bfloat162float(dyn[idx]), n);
+  const int hp = blockIdx.y * 256 + threadIdx.x;
+  if (hp >= g.H * kSsdP) return;
+  const int h = hp / kSsdP, pp = hp - h * kSsdP;
+  const int64_t bt = blockIdx.x, b = bt / g.L;
+  const int tl = (int)(bt - b * g.L), k = tl / (int)g.Bs, s = tl - k * (int)g.Bs, j = s / kSsdT, m = g.m;
+  const int64_t hb = (b * g.nb + k) * g.H + h, idx = bt * g.H * kSsdP + hp;
+  const int64_t stride_i = (int64_t)g.Bs * kSsdP;  // between the tile partials of one head
+  const float* pc = dxp_c + (hb * m * g.Bs + s) * kSsdP + pp;
+  const float* pf = dxp_f + (hb * m * g.Bs + s) * kSsdP + pp;
+  const float* pr = dxp_r + (hb * m * g.Bs + s) * kSsdP + pp;
+  // m is 1 or 2: every load is issued before the sums (in the order i = j..m-1
+  // forward, 0..j reverse)
+  const bool two = m > 1;
+  const float c0 = pc[0], f0 = pf[0], r0 = pr[0];
+  const float c1 = two ? pc[stride_i] : 0.f, f1 = two ? pf[stride_i] : 0.f, r1 = two ? pr[stride_i] : 0.f;
+  const float st = dxs[(hb * g.Bs + s) * kSsdP + pp];
+  const float yc = dyc != nullptr ? __bfloat162float(dyc[idx]) : 0.f, yn = __bfloat162float(dyn[idx]);
+  float c = j == 0 ? c0 : 0.f, n = j == 0 ? f0 : 0.f;
+  if (two) {
+    c = j == 0 ? __fadd_rn(c, c1) : c1;
+    n = j == 0 ? __fadd_rn(n, f1) : f1;
+  }
+  c = __fadd_rn(c, st);
+  if (dyc != nullptr) c = __fmaf_rn(Df[h], yc, c);
+  n = __fadd_rn(n, r0);
+  if (j == 1) n = __fadd_rn(n, r1);
+  n = __fmaf_rn(__fadd_rn(Df[h], Dr[h]), yn, n);
   dxc[idx] = __float2bfloat16_rn(c);
   dxn[idx] = __float2bfloat16_rn(n);
 }
 
 // dB and dC of the three streams: the tile partials of every head group (and
-// the clean state term of every head), summed in order.
-__global__ void __launch_bounds__(256) k_ssd_bwd_dbc(const SsdGeo g, int ngrp, const float* dBp_c, const float* dBs,
+// the clean state term of every head), summed in order. One CTA per token,
+// one thread per state index.
+__global__ void __launch_bounds__(128) k_ssd_bwd_dbc(const SsdGeo g, int ngrp, const float* dBp_c, const float* dBs,
                                                      const float* dCp_c, const float* dBp_f, const float* dCp_f,
                                                      const float* dBp_r, const float* dCp_r, __nv_bfloat16* dBc,
                                                      __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                                      __nv_bfloat16* dBr, __nv_bfloat16* dCr) {
-  const int N = g.N, m = g.m;
-  const int64_t idx = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (idx >= g.Bt * g.L * N) return;
-  const int n = (int)(idx % N);
-  const int64_t bt = idx / N, b = bt / g.L, tl = bt % g.L;
-  const int64_t k = tl / g.Bs, s = tl % g.Bs, bk = b * g.nb + k;
-  const int j = (int)(s / kSsdT);
+  const int N = g.N, m = g.m, n = threadIdx.x;
+  if (n >= N) return;
+  const int64_t bt = blockIdx.x, b = bt / g.L;
+  const int tl = (int)(bt - b * g.L), k = tl / (int)g.Bs, s = tl - k * (int)g.Bs, j = s / kSsdT;
+  const int64_t bk = b * g.nb + k, idx = bt * N + n;
   float bc = 0.f, cc = 0.f, bf = 0.f, cf = 0.f, br = 0.f, cr = 0.f;
   for (int q = 0; q < ngrp; ++q) {
     const int64_t gb = bk * ngrp + q;
-    auto tp = [&](const float* a, int i) { return a[((gb * m + i) * g.Bs + s) * N + n]; };
-    for (int i = j; i < m; ++i) bc = __fadd_rn(bc, tp(dBp_c, i));
-    cc = __fadd_rn(cc, dCp_c[(gb * g.Bs + s) * N + n]);
-    for (int i = j; i < m; ++i) bf = __fadd_rn(bf, tp(dBp_f, i));
-    cf = __fadd_rn(cf, dCp_f[(gb * g.Bs + s) * N + n]);
-    for (int i = 0; i <= j; ++i) br = __fadd_rn(br, tp(dBp_r, i));
-    cr = __fadd_rn(cr, dCp_r[(gb * g.Bs + s) * N + n]);
+    const int64_t tp = (gb * m * g.Bs + s) * N + n, ti = (int64_t)g.Bs * N, c1 = (gb * g.Bs + s) * N + n;
+    // m is 1 or 2: the loads first, then the sums in the order i = j..m-1
+    // (forward), 0..j (reverse)
+    const float bc0 = dBp_c[tp], bf0 = dBp_f[tp], br0 = dBp_r[tp];
+    const float bc1 = m > 1 ? dBp_c[tp + ti] : 0.f, bf1 = m > 1 ? dBp_f[tp + ti] : 0.f, br1 = m > 1 ? dBp_r[tp + ti] : 0.f;
+    const float cc0 = dCp_c[c1], cf0 = dCp_f[c1], cr0 = dCp_r[c1];
+    if (j == 0) {
+      bc = __fadd_rn(bc, bc0);
+      bf = __fadd_rn(bf, bf0);
+    }
+    if (m > 1) {
+      bc = __fadd_rn(bc, bc1);
+      bf = __fadd_rn(bf, bf1);
+    }
+    br = __fadd_rn(br, br0);
+    if (j == 1) br = __fadd_rn(br, br1);
+    cc = __fadd_rn(cc, cc0);
+    cf = __fadd_rn(cf, cf0);
+    cr = __fadd_rn(cr, cr0);
   }
-  for (int h = 0; h < g.H; ++h) bc = __fadd_rn(bc, dBs[((bk * g.H + h) * g.Bs + s) * N + n]);
+  const float* st = dBs + (bk * g.H * g.Bs + s) * N + n;
+  for (int h = 0; h < g.H; ++h) bc = __fadd_rn(bc, st[(int64_t)h * g.Bs * N]);
   dBc[idx] = __float2bfloat16_rn(bc);
   dCc[idx] = __float2bfloat16_rn(cc);
   dBf[idx] = __float2bfloat16_rn(bf);
@@ -855,8 +904,8 @@ cudaError_t launch_ssd_bwd_state(const SsdBwdStateParams& p, cudaStream_t s) {
 cudaError_t launch_ssd_bwd_dx(const SsdGeo& g, const float* dxp_c, const float* dxs, const float* dxp_f,
                               const float* dxp_r, const __nv_bfloat16* dyc, const __nv_bfloat16* dyn, const float* Df,
                               const float* Dr, __nv_bfloat16* dxc, __nv_bfloat16* dxn, cudaStream_t s) {
-  const int64_t n = g.Bt * g.L * g.H * kSsdP;
-  k_ssd_bwd_dx<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, dxp_c, dxs, dxp_f, dxp_r, dyc, dyn, Df, Dr, dxc, dxn);
+  const dim3 grid((unsigned)(g.Bt * g.L), (unsigned)((g.H * kSsdP + 255) / 256));
+  k_ssd_bwd_dx<<<grid, 256, 0, s>>>(g, dxp_c, dxs, dxp_f, dxp_r, dyc, dyn, Df, Dr, dxc, dxn);
   return cudaGetLastError();
 }
 
@@ -864,8 +913,7 @@ cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, co
                                const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
                                __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s) {
-  const int64_t n = g.Bt * g.L * g.N;
-  k_ssd_bwd_dbc<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, ngrp, dBp_c, dBs, dCp_c, dBp_f, dCp_f, dBp_r, dCp_r, dBc, dCc,
+  k_ssd_bwd_dbc<<<(unsigned)(g.Bt * g.L), 128, 0, s>>>(g, ngrp, dBp_c, dBs, dCp_c, dBp_f, dCp_f, dBp_r, dCp_r, dBc, dCc,
                                                             dBf, dCf, dBr, dCr);
   return cudaGetLastError();
 }
