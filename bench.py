@@ -594,18 +594,32 @@ SSD_BWD_KERNELS = ("bwd_tile_clean", "bwd_tile_fwd", "bwd_tile_rev", "bwd_vec_cl
                    "bwd_state_pass", "bwd_block_state", "bwd_dx", "bwd_dbc", "bwd_ddt", "bwd_dd", "bwd_par")
 
 
+def ssd_bwd_head_groups(Bt, L, Bs, H):
+    """Heads per tile CTA and the number of head groups the backward picks
+    (about 1024 CTAs per launch, at most 16 heads per CTA)."""
+    units = Bt * (L // Bs) * (Bs // 128)
+    want = -(-1024 // units) if units > 0 else 1
+    want = min(max(want, -(-H // 16)), H)
+    want = max(want, 1)
+    hg = -(-H // want)
+    return hg, -(-H // hg)
+
+
 def ssd_bwd_tile_flops(Bt, L, Bs, H, N, seeded):
-    """Tensor-core flops of one backward tile launch (one stream and
-    direction): per block, head and (tile i, s-tile j) pair the direction
-    reaches, G = C B^T (K = N), Q = dy x^T (K = 64), dC += dG B, dx = M^T dy,
-    dB = dG^T C (K = 128); per tile of a seeded block after the first, the
-    seed products (E dy) S, C S^T and C^T (E dy)."""
+    """Tensor-core flops one backward tile launch (one stream and direction)
+    issues. Per block and (tile i, s-tile j) pair the direction reaches: per
+    head group G = C B^T (K = N) and, with the head-summed dG split into bf16
+    high and low parts, dC += dG B and dB = dG^T C (K = 128, twice each); per
+    head Q = dy x^T (K = 64) and dx = M^T dy (K = 128). Per head and tile of a
+    seeded block after the first: (E dy) S (K = 64) and C S^T (K = N) with the
+    seed's two parts, and C^T (E dy) (K = 128, C padded to 128 rows)."""
     m, nb = Bs // 128, L // Bs
+    _, ngrp = ssd_bwd_head_groups(Bt, L, Bs, H)
     pairs = m * (m + 1) // 2
-    per_pair = 2.0 * 128 * 128 * (N + 64) + 2.0 * 128 * 128 * (2 * N + 64)
-    f = Bt * nb * H * pairs * per_pair
+    per_pair = ngrp * (2.0 * 128 * 128 * N + 2 * 2 * (2.0 * 128 * N * 128)) + H * 2 * (2.0 * 128 * 128 * 64)
+    f = Bt * nb * pairs * per_pair
     if seeded:
-        f += Bt * (nb - 1) * H * m * (2.0 * 128 * N * 64 * 2 + 2.0 * 128 * 64 * 128)
+        f += Bt * (nb - 1) * m * H * (2 * (2.0 * 128 * N * 64) + 2 * (2.0 * 128 * 64 * N) + 2.0 * 128 * 64 * 128)
     return f
 
 

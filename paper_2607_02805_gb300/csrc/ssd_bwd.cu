@@ -34,14 +34,16 @@ namespace {
 
 using umma::sw128;
 
-constexpr int kBwdThreads = 128;
+constexpr int kBwdThreads = 128;   // k_ssd_bwd_state
+constexpr int kTileThreads = 256;  // k_ssd_bwd_tile: two threads per token row
 
 // Copies `rows` rows of `ncols` (64 or 128) bf16 into 128-byte-swizzled atom
-// columns of rows * 128 bytes each; a null source stages zeros.
+// columns of rows * 128 bytes each, by NT threads; a null source stages zeros.
+template <int NT>
 __device__ __forceinline__ void stage_bf16(unsigned char* dst, const __nv_bfloat16* src, int64_t ld, int rows,
                                            int ncols) {
   const int cpr = ncols / 8;
-  for (int c = threadIdx.x; c < rows * cpr; c += kBwdThreads) {
+  for (int c = threadIdx.x; c < rows * cpr; c += NT) {
     const int r = c / cpr, ch = c % cpr;
     unsigned char* d = dst + (uint32_t)(ch >> 3) * (uint32_t)rows * 128u + sw128((uint32_t)r, (uint32_t)(ch & 7));
     if (src == nullptr)
@@ -52,10 +54,12 @@ __device__ __forceinline__ void stage_bf16(unsigned char* dst, const __nv_bfloat
 }
 
 // An fp32 [rows][ncols] matrix (row stride ncols) as bf16 atom columns (rows * 128
-// bytes each); `lo` selects the rounding residual v - bf16(v) instead of bf16(v).
+// bytes each) by NT threads; `lo` selects the rounding residual v - bf16(v)
+// instead of bf16(v).
+template <int NT>
 __device__ __forceinline__ void stage_f32_as_bf16(unsigned char* dst, const float* src, int rows, int ncols, bool lo) {
   const int cpr = ncols / 8;
-  for (int c = threadIdx.x; c < rows * cpr; c += kBwdThreads) {
+  for (int c = threadIdx.x; c < rows * cpr; c += NT) {
     const int r = c / cpr, ch = c % cpr;
     const float4 a = *reinterpret_cast<const float4*>(src + (int64_t)r * ncols + ch * 8);
     const float4 b = *reinterpret_cast<const float4*>(src + (int64_t)r * ncols + ch * 8 + 4);
@@ -100,45 +104,52 @@ __device__ __forceinline__ void tmem_st32(uint32_t ta, const float (&v)[32]) {
 //   X    x of s-tile j, one head, [128 s][64 p]       DY  dy of tile i, one head, [128 t][64 p]
 //   M    one head's G o decay o dt, [128 t][128 s]
 //   COL  R' of 64 columns, [128][65] fp32             VEC c and dt of one head's block
-//   ROWS row sums and row dots per head of the group, [16][128] fp32 each
+//   CP   column-sum partials of four row quarters, [4][64] fp32
+//   ROWS row sums and row dots per column half and head of the group, [2][16][128] fp32 each
 // After a s-tile's heads, the head-summed dG goes to M (bf16 high part) and
 // X + DY (low part). The seed phase uses DY, BT for E o dy, M for the seed's
 // bf16 high and low parts.
 struct TileSmem {
   static constexpr uint32_t C = 0, BT = 32768, X = 65536, DY = 81920, M = 98304, COL = 131072;
   static constexpr uint32_t VEC = COL + 128u * 65u * 4u;
-  static constexpr uint32_t ROWS = VEC + 2u * 256u * 4u;
-  static constexpr uint32_t total = ROWS + 2u * 16u * 128u * 4u + 1024u;
+  static constexpr uint32_t CP = VEC + 2u * 256u * 4u;
+  static constexpr uint32_t ROWS = CP + 4u * 64u * 4u;
+  static constexpr uint32_t total = ROWS + 2u * 2u * 16u * 128u * 4u + 1024u;
 };
 constexpr int kMaxBwdHeads = 16;  // heads per tile CTA
 
-// dt of head h over the block into s_dt, and its in-block cumulative sums
-// (inclusive; suffix sums for the reverse direction) into s_c by warp 0.
-template <bool UPPER>
+// dt of head h over the block into s_dt (by NT threads), and its in-block
+// cumulative sums (inclusive; suffix sums for the reverse direction) into s_c
+// by warp 0.
+template <bool UPPER, int NT>
 __device__ __forceinline__ void block_dt(const __nv_bfloat16* dt, int64_t tok0, int H, int h, int Bs, float* s_dt,
                                          float* s_c) {
-  for (int s = threadIdx.x; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(dt[(tok0 + s) * H + h]);
+  for (int s = threadIdx.x; s < Bs; s += NT) s_dt[s] = __bfloat162float(dt[(tok0 + s) * H + h]);
   if ((threadIdx.x >> 5) == 0) warp_scan_dt<UPPER>(dt + tok0 * H + h, H, Bs, s_c);
 }
 
-// One CTA of 4 warps per (batch row, block, tile i) and group of heads: thread
-// t owns token row t of tile i (TMEM lane t) for the row-side products and
-// row s = t of s-tile j for the column-side ones. Per s-tile j the Gram tile
-// G = C_i B_j^T is shared by the group's heads; per head, Q = dy x^T, the
-// masked decays, the column sums of R', dx_j = M^T dy, and dG = Q o decay o dt
-// summed over the heads in fp32 in TMEM. dC and dB_j then take the
-// head-summed dG once (B and C are shared by the heads), split into bf16 high
-// and low parts. TMEM: G, then dB_j (and the seed products) at 0; Q, then
-// dx_j at 128; the head sum of dG at 256; dC at 384.
+// One CTA of 8 warps per (batch row, block, tile i) and group of heads. Token
+// row t of tile i (TMEM lane t) has two threads, t and t + 128: the first
+// takes columns 0..63 of every 128-column product, the second 64..127 (a
+// warp reaches the TMEM lanes 32 (warp mod 4) onward). Row s = t of s-tile j
+// is the column-side row. Per s-tile j the Gram tile G = C_i B_j^T is shared
+// by the group's heads; per head, Q = dy x^T, the masked decays, the column
+// sums of R', dx_j = M^T dy, and dG = Q o decay o dt summed over the heads in
+// fp32 in TMEM. dC and dB_j then take the head-summed dG once (B and C are
+// shared by the heads), split into bf16 high and low parts. TMEM: G, then
+// dB_j (and the seed products) at 0; Q, then dx_j at 128; the head sum of dG
+// at 256; dC at 384.
 template <int N, bool UPPER, bool SEED>
-__global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTileParams p) {
+__global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTileParams p) {
   extern __shared__ unsigned char smraw[];
   unsigned char* sm = align1024(smraw);
   __shared__ uint64_t bar;
   __shared__ uint32_t tslot;
   using S = TileSmem;
+  constexpr int NT = kTileThreads;
   const SsdGeo& g = p.g;
-  const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x, w = t >> 5;
+  const int Bs = (int)g.Bs, H = g.H, m = g.m, tid = threadIdx.x, w = tid >> 5;
+  const int t = tid & 127, half = tid >> 7;  // token row, column half
   const int64_t idx = blockIdx.x;
   const int i = (int)(idx % m);
   const int64_t bk = idx / m, b = bk / g.nb;
@@ -150,23 +161,24 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
   float* s_c = reinterpret_cast<float*>(sm + S::VEC);
   float* s_dt = s_c + 256;
   float* s_col = reinterpret_cast<float*>(sm + S::COL);
-  float* s_rows = reinterpret_cast<float*>(sm + S::ROWS);  // [hh][128]
-  float* s_dots = s_rows + kMaxBwdHeads * 128;
+  float* s_cp = reinterpret_cast<float*>(sm + S::CP);
+  float* s_rows = reinterpret_cast<float*>(sm + S::ROWS) + half * kMaxBwdHeads * 128;  // [hh][128] of this half
+  float* s_dots = s_rows + 2 * kMaxBwdHeads * 128;
 
-  stage_bf16(sm + S::C, p.C + (tok0 + i * kSsdT) * N, N, 128, N);
+  stage_bf16<NT>(sm + S::C, p.C + (tok0 + i * kSsdT) * N, N, 128, N);
   if (N == 64)
-    for (int c = t; c < 128 * 8; c += kBwdThreads) *reinterpret_cast<uint4*>(sm + S::C + kTile16 + c * 16) = make_uint4(0u, 0u, 0u, 0u);
+    for (int c = tid; c < 128 * 8; c += NT) *reinterpret_cast<uint4*>(sm + S::C + kTile16 + c * 16) = make_uint4(0u, 0u, 0u, 0u);
   cp_async_commit();
   for (int hh = 0; hh < kMaxBwdHeads; ++hh) {
     s_rows[hh * 128 + t] = 0.f;
     s_dots[hh * 128 + t] = 0.f;
   }
-  if (t == 0) umma::bar_init(&bar, 1);
+  if (tid == 0) umma::bar_init(&bar, 1);
   if (w == 0) tmem_alloc(&tslot, 512);
   umma::fence_before_sync();
   __syncthreads();
   umma::fence_after_sync();
-  const uint32_t tm = tslot, lane_base = tm + ((uint32_t)(32 * w) << 16);
+  const uint32_t tm = tslot, lane_base = tm + ((uint32_t)(32 * (w & 3)) << 16);
   const int tt = i * kSsdT + t;
   uint32_t phase = 0;
   bool alive = true;
@@ -185,13 +197,13 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
   const int j0 = UPPER ? i : 0, j1 = UPPER ? m - 1 : i;
   for (int j = j0; j <= j1 && alive; ++j) {
     const int64_t sr0 = tok0 + (int64_t)j * kSsdT;
-    stage_bf16(sm + S::BT, p.B + sr0 * N, N, 128, N);
+    stage_bf16<NT>(sm + S::BT, p.B + sr0 * N, N, 128, N);
     cp_async_commit();
     cp_async_wait_all();
     umma::fence_async_smem();
     umma::fence_before_sync();
     __syncthreads();
-    if (t == 0) {
+    if (tid == 0) {
       umma::fence_after_sync();
 #pragma unroll
       for (int kk = 0; kk < N / 16; ++kk) {  // G = C_i B_j^T, shared by the heads
@@ -203,15 +215,15 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
     if (!(alive = wait_mma())) break;
     for (int hh = 0; hh < hg; ++hh) {
       const int h = h0 + hh;
-      stage_bf16(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
-      stage_bf16(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+      stage_bf16<NT>(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
+      stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
       cp_async_commit();
-      block_dt<UPPER>(p.dt, tok0, H, h, Bs, s_dt, s_c);
+      block_dt<UPPER, NT>(p.dt, tok0, H, h, Bs, s_dt, s_c);
       cp_async_wait_all();
       umma::fence_async_smem();
       umma::fence_before_sync();
       __syncthreads();
-      if (t == 0) {
+      if (tid == 0) {
         umma::fence_after_sync();
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)  // Q = dy_i x_j^T
@@ -222,8 +234,11 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
       if (!(alive = wait_mma())) break;
       const float A2 = __fmul_rn(p.A[h], kLog2e), ct = s_c[tt];
       float rowsum = 0.f;
+      // two rounds: round r takes 32-column chunk r (first half) and 2 + r
+      // (second half), then the column sums of those 64 columns
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
+      for (int r = 0; r < 2; ++r) {
+        const int c = 2 * half + r;
         float gv[32], qv[32], dgs[32];
         umma::tmem_ld32(lane_base + 32u * (uint32_t)c, gv);
         umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)c, qv);
@@ -241,7 +256,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
             const float gl = __fmul_rn(gv[e + q], L);
             const float rp = __fmul_rn(qv[e + q], gl);
             rowsum = __fmaf_rn(rp, ds, rowsum);
-            s_col[t * 65 + 32 * (c & 1) + e + q] = rp;
+            s_col[t * 65 + 32 * half + e + q] = rp;
             const float dg = __fmul_rn(__fmul_rn(qv[e + q], L), ds);
             dgs[e + q] = hh > 0 ? __fadd_rn(dgs[e + q], dg) : dg;
             mv[q] = __fmul_rn(gl, ds);
@@ -255,14 +270,23 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
           const uint32_t off = (uint32_t)(chunk >> 3) * kTile16 + sw128((uint32_t)t, (uint32_t)(chunk & 7));
           *reinterpret_cast<uint4*>(sm + S::M + off) = make_uint4(mp[4 * u], mp[4 * u + 1], mp[4 * u + 2], mp[4 * u + 3]);
         }
-        if (c & 1) {  // column sums of R' over the tile's 128 rows, 64 columns at a time
-          __syncthreads();
-          if (t < 64) {
-            float sum = 0.f;
-            for (int r = 0; r < 128; ++r) sum = __fadd_rn(sum, s_col[r * 65 + t]);
-            p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + 64 * (c >> 1) + t] = sum;
-          }
-          __syncthreads();
+        // column sums of R' over the tile's 128 rows: four row quarters of 32
+        // (four interleaved sums each), then the quarters in order
+        __syncthreads();
+        {
+          const int col = tid & 63, qr = tid >> 6;
+          float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int rr = 0; rr < 32; rr += 4)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) a[q] = __fadd_rn(a[q], s_col[(32 * qr + rr + q) * 65 + col]);
+          s_cp[qr * 64 + col] = __fadd_rn(__fadd_rn(a[0], a[1]), __fadd_rn(a[2], a[3]));
+        }
+        __syncthreads();
+        if (tid < 64) {  // s_col column cc is tile column 32 (2 (cc / 32) + r) + cc % 32
+          const float sum = __fadd_rn(__fadd_rn(s_cp[tid], s_cp[64 + tid]), __fadd_rn(s_cp[128 + tid], s_cp[192 + tid]));
+          const int tc = 32 * (2 * (tid >> 5) + r) + (tid & 31);
+          p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + tc] = sum;
         }
       }
       s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);
@@ -270,7 +294,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
       umma::fence_async_smem();
       umma::fence_before_sync();
       __syncthreads();
-      if (t == 0) {
+      if (tid == 0) {
         umma::fence_after_sync();
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)  // dx_j = M^T dy_i: M read as an MN-major operand (M = s, K = t)
@@ -279,21 +303,19 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
         umma::mma_commit(&bar);
       }
       if (!(alive = wait_mma())) break;
-      {  // row s = j*128 + t of head h's dx contribution from tile i
+      {  // row s = j*128 + t of head h's dx contribution from tile i, 32 channels per half
         float v[32];
-        float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * kSsdP;
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)q, v);
-          store_row(dxo + 32 * q, v);
-        }
+        float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * kSsdP + 32 * half;
+        umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)half, v);
+        store_row(dxo, v);
       }
       umma::fence_before_sync();
     }
     if (!alive) break;
     // the head-summed dG as bf16 high (M) and low (X + DY) parts
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
+    for (int r = 0; r < 2; ++r) {
+      const int c = 2 * half + r;
       float dgs[32];
       umma::tmem_ld32(lane_base + 256u + 32u * (uint32_t)c, dgs);
       uint32_t hi[16], lo[16];
@@ -314,7 +336,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
     umma::fence_async_smem();
     umma::fence_before_sync();
     __syncthreads();
-    if (t == 0) {
+    if (tid == 0) {
       umma::fence_after_sync();
 #pragma unroll
       for (int part = 0; part < 2; ++part) {
@@ -333,11 +355,11 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
       umma::mma_commit(&bar);
     }
     if (!(alive = wait_mma())) break;
-    {  // row s = j*128 + t of the group's dB contribution from tile i
+    {  // row s = j*128 + t of the group's dB contribution from tile i, N/2 columns per half
       float v[32];
       float* dbo = p.dB_part + (((bk * ngrp + grp) * m + i) * Bs + j * kSsdT + t) * N;
 #pragma unroll
-      for (int q = 0; q < N / 32; ++q) {
+      for (int q = half * (N / 64); q < (half + 1) * (N / 64); ++q) {
         umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
         store_row(dbo + 32 * q, v);
       }
@@ -351,17 +373,18 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
     constexpr uint32_t id_cs = umma::idesc_bf16(128, 64, false, false);
     for (int hh = 0; hh < hg && alive; ++hh) {
       const int h = h0 + hh;
-      stage_bf16(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+      stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
       cp_async_commit();
       const float* seed = p.states + ((b * g.nb + k - 1) * H + h) * (int64_t)kSsdP * N;
-      stage_f32_as_bf16(sm + S::M, seed, 64, N, false);
-      stage_f32_as_bf16(sm + S::M + 16384u, seed, 64, N, true);
-      block_dt<false>(p.dt, tok0, H, h, Bs, s_dt, s_c);
+      stage_f32_as_bf16<NT>(sm + S::M, seed, 64, N, false);
+      stage_f32_as_bf16<NT>(sm + S::M + 16384u, seed, 64, N, true);
+      block_dt<false, NT>(p.dt, tok0, H, h, Bs, s_dt, s_c);
       cp_async_wait_all();
       __syncthreads();
       const float E = ex2(__fmul_rn(__fmul_rn(p.A[h], kLog2e), s_c[tt]));
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) {
+      for (int cq = 0; cq < 4; ++cq) {  // 16-byte chunks 4 half .. 4 half + 3 of row t
+        const int ch = 4 * half + cq;
         const uint4 u = *reinterpret_cast<const uint4*>(sm + S::DY + sw128((uint32_t)t, (uint32_t)ch));
         const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&u);
         uint32_t o[4];
@@ -375,7 +398,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
       umma::fence_async_smem();
       umma::fence_before_sync();
       __syncthreads();
-      if (t == 0) {
+      if (tid == 0) {
         umma::fence_after_sync();
 #pragma unroll
         for (int part = 0; part < 2; ++part) {
@@ -396,41 +419,38 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_tile(const SsdBwdTil
         umma::mma_commit(&bar);
       }
       if (!(alive = wait_mma())) break;
-      float v[32], rowdot = 0.f;
+      float v[32], rowdot = 0.f;  // channels 32 half .. 32 half + 31 of the row dot
+      umma::tmem_ld32(lane_base + 32u * (uint32_t)half, v);
 #pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) rowdot = __fmaf_rn(tile_at(sm + S::DY, t, 32 * q + e), v[e], rowdot);
-      }
+      for (int e = 0; e < 32; ++e) rowdot = __fmaf_rn(tile_at(sm + S::DY, t, 32 * half + e), v[e], rowdot);
       s_dots[hh * 128 + t] = __fmul_rn(E, rowdot);
-      if (32 * w < N) {  // row n = t of dS^T: the seed gradient partial [p][n]
+      if (32 * (w & 3) < N) {  // row n = t of dS^T, channels 32 half ..: the seed gradient partial [p][n]
         float* dso = p.dS_part + ((bk * H + h) * m + i) * (int64_t)kSsdP * N + t;
+        umma::tmem_ld32(lane_base + 64u + 32u * (uint32_t)half, v);
 #pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          umma::tmem_ld32(lane_base + 64u + 32u * (uint32_t)q, v);
-#pragma unroll
-          for (int e = 0; e < 32; ++e) dso[(int64_t)(32 * q + e) * N] = v[e];
-        }
+        for (int e = 0; e < 32; ++e) dso[(int64_t)(32 * half + e) * N] = v[e];
       }
       umma::fence_before_sync();
       __syncthreads();  // DY, BT and M are restaged for the next head
     }
   }
-  if (alive) {
-    {  // dC of row t of tile i, summed over the group's heads
-      float v[32];
-      float* dco = p.dC_part + ((bk * ngrp + grp) * Bs + tt) * N;
+  if (alive) {  // dC of row t of tile i, summed over the group's heads, N/2 columns per half
+    float v[32];
+    float* dco = p.dC_part + ((bk * ngrp + grp) * Bs + tt) * N;
 #pragma unroll
-      for (int q = 0; q < N / 32; ++q) {
-        umma::tmem_ld32(lane_base + 384u + 32u * (uint32_t)q, v);
-        store_row(dco + 32 * q, v);
-      }
+    for (int q = half * (N / 64); q < (half + 1) * (N / 64); ++q) {
+      umma::tmem_ld32(lane_base + 384u + 32u * (uint32_t)q, v);
+      store_row(dco + 32 * q, v);
     }
-    for (int hh = 0; hh < hg; ++hh) {
+  }
+  __syncthreads();  // both halves' row sums and dots are in shared memory
+  if (alive) {
+    const float* rows = reinterpret_cast<const float*>(sm + S::ROWS);  // [half][hh][128]
+    const float* dots = rows + 2 * kMaxBwdHeads * 128;
+    for (int hh = half; hh < hg; hh += 2) {
       const int h = h0 + hh;
-      p.rowsum[(bk * H + h) * Bs + tt] = s_rows[hh * 128 + t];
-      if (SEED) p.rowdot[(bk * H + h) * Bs + tt] = s_dots[hh * 128 + t];
+      p.rowsum[(bk * H + h) * Bs + tt] = __fadd_rn(rows[hh * 128 + t], rows[(kMaxBwdHeads + hh) * 128 + t]);
+      if (SEED) p.rowdot[(bk * H + h) * Bs + tt] = __fadd_rn(dots[hh * 128 + t], dots[(kMaxBwdHeads + hh) * 128 + t]);
     }
   }
   cp_async_wait_all();
@@ -597,8 +617,8 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
   float* s_dw = s_w + 256;
   float* s_e = s_dw + 256;
   const float* gS = p.gS + (bk * H + h) * PN;
-  stage_f32_as_bf16(sm + S::GH, gS, 64, N, false);
-  stage_f32_as_bf16(sm + S::GL, gS, 64, N, true);
+  stage_f32_as_bf16<kBwdThreads>(sm + S::GH, gS, 64, N, false);
+  stage_f32_as_bf16<kBwdThreads>(sm + S::GL, gS, 64, N, true);
   for (int s = t; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
   if (w == 0) warp_scan_dt<true>(p.dt + tok0 * H + h, H, Bs, s_suf);
   // block decay: da = sum over (p, n) of gS o S_{k-1}
@@ -626,8 +646,8 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
   bool alive = true;
   for (int j = 0; j < m; ++j) {
     const int64_t sr0 = tok0 + (int64_t)j * kSsdT;
-    stage_bf16(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
-    stage_bf16(sm + S::BT, p.B + sr0 * N, N, 128, N);
+    stage_bf16<kBwdThreads>(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
+    stage_bf16<kBwdThreads>(sm + S::BT, p.B + sr0 * N, N, 128, N);
     cp_async_commit();
     cp_async_wait_all();
     umma::fence_async_smem();
@@ -860,7 +880,7 @@ cudaError_t bwd_tile_t(const SsdBwdTileParams& p, cudaStream_t s) {
   cudaError_t e = set_smem_cached((const void*)k_ssd_bwd_tile<N, UPPER, SEED>, smem, -1);
   if (e != cudaSuccess) return e;
   dim3 grid((unsigned)(p.g.Bt * p.g.nb * p.g.m), (unsigned)((p.g.H + p.hg - 1) / p.hg));
-  k_ssd_bwd_tile<N, UPPER, SEED><<<grid, kBwdThreads, smem, s>>>(p);
+  k_ssd_bwd_tile<N, UPPER, SEED><<<grid, kTileThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 
