@@ -72,6 +72,7 @@ extern "C" {
 #define BDSCAN_ERR_ARG (-1)         /* null/misaligned pointer, bad size, len % block != 0, small workspace */
 #define BDSCAN_ERR_UNSUPPORTED (-2) /* valid arguments outside the supported set above */
 #define BDSCAN_ERR_CUDA (-3)        /* a CUDA launch or runtime call failed */
+#define BDSCAN_ERR_DEVICE (-4)      /* debug build only: a device-side check failed (see bdscan_debug_build) */
 
 #define BDSCAN_F32 0
 #define BDSCAN_BF16 1
@@ -159,6 +160,26 @@ int bdscan_profile_events(void* const* events, int n);
 
 /* Number of kernels the last successful call of this host thread launched. */
 int bdscan_last_launch_count(void);
+
+/* Debug build (lib/libbdscan_debug.so, the same sources compiled with
+ * BDSCAN_DEBUG=1; same symbols). Each kernel first checks, from its block
+ * index and the call's sizes alone, that the last element its CTA touches in
+ * every buffer lies inside that buffer's extent; a failed check writes a
+ * device status word and the CTA skips its work (no out-of-range access is
+ * made, nothing traps). The cached boundary states and the parameter
+ * gradients are also checked for NaN and infinity. Every entry point of the
+ * debug build then synchronizes the device before it returns (so it cannot
+ * be captured into a CUDA graph) and returns BDSCAN_ERR_DEVICE, with the
+ * kernel and offset in bdscan_last_error(), if any check failed; the status
+ * words are cleared for the next call.
+ * bdscan_debug_build() returns 1 in the debug build and 0 otherwise.
+ * bdscan_debug_set_slack(e): every extent is taken e >= 0 elements shorter
+ * than the sizes give, so a test can make the checks fail on in-range
+ * accesses (the flagged CTAs then skip their work and the outputs are
+ * incomplete); 0 restores the exact extents. Needs a CUDA device; returns
+ * BDSCAN_ERR_UNSUPPORTED in the release build, BDSCAN_ERR_ARG for e < 0. */
+int bdscan_debug_build(void);
+int bdscan_debug_set_slack(long long elements);
 
 /* ---------------------------------------------------------------------- */
 /* All-block forward (Sec. 4 eqs. boundary-state and partial-reverse, all  */

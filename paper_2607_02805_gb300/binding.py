@@ -5,7 +5,8 @@ same arguments; the ctypes structures mirror the C structs field by field.
 The tensor helpers at the bottom turn torch tensors into those structs (data
 pointers, the current CUDA stream) and raise on a non-zero return code. All
 computation happens in the CUDA library; if it cannot be loaded, every call
-raises.
+raises. use_debug_build() routes every later call to the debug build of the
+same library (device status words, BDSCAN_ERR_DEVICE).
 """
 
 from __future__ import annotations
@@ -16,11 +17,13 @@ import threading
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "lib", "libbdscan.so")
+LIB_DEBUG_PATH = os.path.join(_HERE, "lib", "libbdscan_debug.so")
 
 BDSCAN_OK = 0
 BDSCAN_ERR_ARG = -1
 BDSCAN_ERR_UNSUPPORTED = -2
 BDSCAN_ERR_CUDA = -3
+BDSCAN_ERR_DEVICE = -4
 BDSCAN_F32 = 0
 BDSCAN_BF16 = 1
 
@@ -143,6 +146,8 @@ SIGNATURES = [
       c_void_p, _P(bdscan_clean_grads), _P(bdscan_noisy_grads), _P(bdscan_param_grads), c_void_p, ctypes.c_size_t,
       c_void_p]),
     ("bdscan_ssd_wait_flag", ctypes.c_int, [ctypes.c_int]),
+    ("bdscan_debug_build", ctypes.c_int, []),
+    ("bdscan_debug_set_slack", ctypes.c_int, [ctypes.c_longlong]),
     ("bdscan_ssd_wait_selftest", ctypes.c_int, [ctypes.c_uint32]),
     ("bdscan_ssd_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
     ("bdscan_ssd_full_bidir_forward", ctypes.c_int,
@@ -152,26 +157,38 @@ SIGNATURES = [
 BDSCAN_NOALLOC_SCRATCH_BYTES = 32 << 20
 
 _lock = threading.Lock()
-_lib = None
+_libs = {False: None, True: None}
+_use_debug = False
 
 
-def load(build_if_missing: bool = True):
-    """Load the CUDA library (building it in-tree first if it is missing or stale)."""
-    global _lib
+def load(build_if_missing: bool = True, debug=None):
+    """Load the CUDA library (building it in-tree first if it is missing or
+    stale): the release build, or the debug build when `debug` is true (by
+    default the one use_debug_build() selected)."""
+    dbg = _use_debug if debug is None else bool(debug)
+    path = LIB_DEBUG_PATH if dbg else LIB_PATH
     with _lock:
-        if _lib is None:
+        if _libs[dbg] is None:
             if build_if_missing:
                 from . import build as _build
-                _build.build()
-            if not os.path.exists(LIB_PATH):
-                raise RuntimeError(f"libbdscan is not built ({LIB_PATH} missing); run paper_2607_02805_gb300/build.py")
-            lib = ctypes.CDLL(LIB_PATH)
+                _build.build(debug=dbg)
+            if not os.path.exists(path):
+                raise RuntimeError(f"libbdscan is not built ({path} missing); run paper_2607_02805_gb300/build.py")
+            lib = ctypes.CDLL(path)
             for name, res, args in SIGNATURES:
                 f = getattr(lib, name)
                 f.restype = res
                 f.argtypes = args
-            _lib = lib
-    return _lib
+            _libs[dbg] = lib
+    return _libs[dbg]
+
+
+def use_debug_build(on: bool = True) -> None:
+    """Route every later call of this module to the debug build (or back)."""
+    global _use_debug
+    if on:
+        load(debug=True)
+    _use_debug = bool(on)
 
 
 class BdscanError(RuntimeError):
@@ -195,6 +212,14 @@ def _ref(x):
 # raw functions, same names and arguments as the C ABI
 def bdscan_last_error() -> str:
     return load().bdscan_last_error().decode()
+
+
+def bdscan_debug_build() -> int:
+    return load().bdscan_debug_build()
+
+
+def bdscan_debug_set_slack(elements) -> int:
+    return load().bdscan_debug_set_slack(elements)
 
 
 def bdscan_version() -> int:

@@ -4,6 +4,11 @@ Each .cu file is compiled to an object in parallel, then linked into
 ``paper_2607_02805_gb300/lib/libbdscan.so``. The CUDA runtime is linked
 statically, so the library needs only the driver at run time. A rebuild
 happens when any source or header is newer than the library.
+
+The debug build, ``lib/libbdscan_debug.so``, is the same sources compiled
+with ``-DBDSCAN_DEBUG=1``: its kernels check their extents and write device
+status words, and its entry points return BDSCAN_ERR_DEVICE when a check
+failed (include/bdscan.h). ``build_all()`` compiles both variants at once.
 """
 
 from __future__ import annotations
@@ -22,6 +27,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIBDIR = os.path.join(HERE, "lib")
 LIB = os.path.join(LIBDIR, "libbdscan.so")
+LIB_DEBUG = os.path.join(LIBDIR, "libbdscan_debug.so")
+DEBUG_FLAGS = ["-DBDSCAN_DEBUG=1"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
@@ -44,45 +51,75 @@ def _deps():
                                + glob.glob(os.path.join(INCLUDE, "*.h")) + [os.path.abspath(__file__)])
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(debug: bool = False) -> bool:
+    lib = LIB_DEBUG if debug else LIB
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    if not force and up_to_date():
-        return LIB
-    os.makedirs(BUILD, exist_ok=True)
+def _variants(debug_list, force):
+    return [d for d in debug_list if force or not up_to_date(d)]
+
+
+def _build_variants(debug_list, verbose=False, extra_flags=()):
+    """Compiles every (variant, source) pair in one process pool, then links."""
     os.makedirs(LIBDIR, exist_ok=True)
     cc = nvcc()
     srcs = _sources()
-    objs = [os.path.join(BUILD, os.path.basename(s)[:-3] + ".o") for s in srcs]
+    jobs = []
+    for dbg in debug_list:
+        bdir = os.path.join(BUILD, "debug") if dbg else BUILD
+        os.makedirs(bdir, exist_ok=True)
+        flags = list(extra_flags) + (DEBUG_FLAGS if dbg else [])
+        for src in srcs:
+            jobs.append((dbg, src, os.path.join(bdir, os.path.basename(src)[:-3] + ".o"), flags))
 
-    def compile_one(src, obj):
-        cmd = [cc] + ARCH + NVCC_FLAGS + list(extra_flags) + ["-c", src, "-o", obj]
+    def compile_one(job):
+        _, src, obj, flags = job
+        cmd = [cc] + ARCH + NVCC_FLAGS + flags + ["-c", src, "-o", obj]
         if verbose:
             cmd.insert(1, "-Xptxas=-v")
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
-            raise RuntimeError(f"nvcc failed for {os.path.basename(src)}:\n{r.stdout}\n{r.stderr}")
+            raise RuntimeError(f"nvcc failed for {os.path.basename(src)} {' '.join(flags)}:\n{r.stdout}\n{r.stderr}")
         return r.stdout + r.stderr
 
-    with concurrent.futures.ThreadPoolExecutor(max_workers=max(1, len(srcs))) as ex:
-        logs = list(ex.map(compile_one, srcs, objs))
+    with concurrent.futures.ThreadPoolExecutor(max_workers=max(1, len(jobs))) as ex:
+        logs = list(ex.map(compile_one, jobs))
     if verbose:
-        for src, log in zip(srcs, logs):
-            sys.stdout.write(f"== {os.path.basename(src)}\n{log}")
-    tmp = LIB + f".tmp{os.getpid()}"
-    cmd = [cc] + ARCH + ["-shared", "-o", tmp] + objs
-    r = subprocess.run(cmd, capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+        for job, log in zip(jobs, logs):
+            sys.stdout.write(f"== {os.path.basename(job[1])} {' '.join(job[3])}\n{log}")
+    out = []
+    for dbg in debug_list:
+        lib = LIB_DEBUG if dbg else LIB
+        objs = [j[2] for j in jobs if j[0] == dbg]
+        tmp = lib + f".tmp{os.getpid()}"
+        cmd = [cc] + ARCH + ["-shared", "-o", tmp] + objs
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, lib)
+        out.append(lib)
+    return out
+
+
+def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: bool = False) -> str:
+    """Builds one variant (the release library, or the debug one) if stale."""
+    if _variants([debug], force):
+        _build_variants([debug], verbose, extra_flags)
+    return LIB_DEBUG if debug else LIB
+
+
+def build_all(force: bool = False, verbose: bool = False) -> list:
+    """Builds the release and the debug library (whichever is stale) in one pool."""
+    todo = _variants([False, True], force)
+    if todo:
+        _build_variants(todo, verbose)
+    return [LIB, LIB_DEBUG]
 
 
 if __name__ == "__main__":
-    build(force="--force" in sys.argv, verbose="-v" in sys.argv)
-    print(LIB)
+    for p in build_all(force="--force" in sys.argv, verbose="-v" in sys.argv):
+        print(p)

@@ -6,9 +6,32 @@
 #include <cstring>
 #include <atomic>
 #include <mutex>
+#include <vector>
 
 #include "bdscan.h"
+#include "debug.cuh"
 #include "params.h"
+
+namespace bds {
+namespace dbg {
+// Status words of the translation units of the debug build (registered at
+// load time, before any call).
+std::vector<StatusIo>& status_ios() {
+  static std::vector<StatusIo> v;
+  return v;
+}
+std::mutex& status_mu() {
+  static std::mutex mu;
+  return mu;
+}
+int add_status_io(StatusIo io) {
+  std::lock_guard<std::mutex> lk(status_mu());
+  status_ios().push_back(io);
+  return (int)status_ios().size();
+}
+long long g_slack = 0;
+}  // namespace dbg
+}  // namespace bds
 
 namespace {
 
@@ -28,7 +51,40 @@ thread_local int g_prof_n = 0;
 thread_local int g_launches = 0;
 thread_local int g_last_launches = 0;
 
+const char* site_name(int site) {
+  static const char* names[] = {"?", "k_chunk_local", "k_chunk_carry", "k_block_scan", "k_active_block",
+                                "k_bwd_noisy", "k_bwd_carry", "k_bwd_clean", "k_reduce_tok", "k_reduce_par",
+                                "k_ssd_block_state", "k_ssd_state_pass", "k_ssd_block_scan", "k_ssd_bwd_tile",
+                                "k_ssd_bwd_state"};
+  static_assert(sizeof(names) / sizeof(names[0]) == bds::kSiteCount, "one name per debug site");
+  return site > 0 && site < bds::kSiteCount ? names[site] : names[0];
+}
+
+// Debug build: after an entry point's launches, wait for them and read every
+// translation unit's status word (clearing it). Returns BDSCAN_OK or the code.
+int debug_check(int launches) {
+  if (!BDSCAN_DEBUG || launches == 0) return BDSCAN_OK;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return fail(BDSCAN_ERR_CUDA, "debug status check: %s", cudaGetErrorString(e));
+  bds::DevStatus first = {0, 0, 0, 0};
+  std::lock_guard<std::mutex> lk(bds::dbg::status_mu());
+  for (bds::dbg::StatusIo io : bds::dbg::status_ios()) {
+    bds::DevStatus st;
+    const int r = io(&st, 1, bds::dbg::g_slack);
+    if (r != 0) return fail(BDSCAN_ERR_CUDA, "debug status read: %s", cudaGetErrorString((cudaError_t)r));
+    if (st.code != 0 && first.code == 0) first = st;
+  }
+  if (first.code == bds::kStatusRange)
+    return fail(BDSCAN_ERR_DEVICE, "device status: %s: offset %lld outside the extent %lld its sizes give (the CTA skipped its work)",
+                site_name(first.site), first.value, first.limit);
+  if (first.code != 0)
+    return fail(BDSCAN_ERR_DEVICE, "device status: %s: non-finite value at index %lld", site_name(first.site), first.value);
+  return BDSCAN_OK;
+}
+
 int ok() {
+  const int rc = debug_check(g_launches);
+  if (rc != BDSCAN_OK) return rc;
   g_err[0] = '\0';
   g_last_launches = g_launches;
   return BDSCAN_OK;
@@ -215,6 +271,23 @@ int bdscan_profile_events(void* const* events, int n) {
 }
 
 int bdscan_last_launch_count(void) { return g_last_launches; }
+
+int bdscan_debug_build(void) { return BDSCAN_DEBUG; }
+
+int bdscan_debug_set_slack(long long elements) {
+  const char* fn = "bdscan_debug_set_slack";
+  if (!BDSCAN_DEBUG) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: this is the release build (no device checks)", fn);
+  if (elements < 0) return fail(BDSCAN_ERR_ARG, "%s: negative slack %lld", fn, elements);
+  std::lock_guard<std::mutex> lk(bds::dbg::status_mu());
+  bds::dbg::g_slack = elements;
+  for (bds::dbg::StatusIo io : bds::dbg::status_ios()) {
+    bds::DevStatus st;
+    const int r = io(&st, 0, elements);
+    if (r != 0) return fail(BDSCAN_ERR_CUDA, "%s: %s", fn, cudaGetErrorString((cudaError_t)r));
+  }
+  g_err[0] = '\0';
+  return BDSCAN_OK;
+}
 
 int64_t bdscan_chunk_tokens(int64_t block) { return block <= 0 ? 0 : blocks_per_chunk(block) * block; }
 

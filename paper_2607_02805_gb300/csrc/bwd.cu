@@ -16,6 +16,8 @@ __global__ void __launch_bounds__(256) k_bwd_carry(const BwdParams p) {
   if (idx >= g.Bt * g.D * N) return;
   const int n = (int)(idx % N);
   const int64_t d = (idx / N) % g.D, b = idx / ((int64_t)N * g.D);
+  // debug build: the last seed gradient this thread reads (no barrier follows)
+  if (!dguard(kSiteBwdCarry, ((b * g.nb + g.nb - 1) * g.D + d) * N + n, g.Bt * g.nb * g.D * N)) return;
   const float A2 = __fmul_rn(p.Af[d * N + n], kLog2e);
   const float* dS = p.dS + (b * g.nb * g.D + d) * N + n;  // block k at [k * D * N]
   const float* ext = p.dstates != nullptr ? p.dstates + (b * g.nb * g.D + d) * N + n : nullptr;
@@ -75,6 +77,8 @@ __global__ void __launch_bounds__(256) k_reduce_tok(const BwdParams p) {
   const int64_t row = idx / (N / 4);
   const int tensor = (int)(row / rows);
   const int64_t bt = row - (int64_t)tensor * rows;
+  // debug build: the last channel-group partial this thread reads (no barrier follows)
+  if (!dguard(kSiteReduceTok, (row * g.G + g.G - 1) * N + n + 3, 6 * rows * g.G * N)) return;
   const float* src = p.part_tok + row * g.G * N + n;
   float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int gi = 0; gi < g.G; ++gi) {
@@ -106,6 +110,8 @@ __global__ void __launch_bounds__(32 * kParSlices) k_reduce_par(const BwdParams 
   const int64_t DN = g.D * N;
   const int lane = threadIdx.x & 31, slice = threadIdx.x >> 5;
   const int64_t col = ((int64_t)blockIdx.x * 32 + lane) * 4;  // D and D*N are multiples of 4
+  // debug build: the CTA's first column lies inside the parameter columns
+  if (!dguard(kSiteReducePar, (int64_t)blockIdx.x * 128, DN + g.D)) return;
   float4 s0 = make_float4(0.f, 0.f, 0.f, 0.f), s1 = s0, s2 = s0;
   auto acc = [](float4& s, const float* src) {
     const float4 v = *reinterpret_cast<const float4*>(src);
@@ -144,6 +150,12 @@ __global__ void __launch_bounds__(32 * kParSlices) k_reduce_par(const BwdParams 
       t0 = make_float4(t0.x + v0.x, t0.y + v0.y, t0.z + v0.z, t0.w + v0.w);
       t1 = make_float4(t1.x + v1.x, t1.y + v1.y, t1.z + v1.z, t1.w + v1.w);
       t2 = make_float4(t2.x + v2.x, t2.y + v2.y, t2.z + v2.z, t2.w + v2.w);
+    }
+    // debug build: a non-finite parameter gradient
+    if (BDSCAN_DEBUG) {
+      const float v[12] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w, t2.x, t2.y, t2.z, t2.w};
+#pragma unroll
+      for (int q = 0; q < 12; ++q) dfinite(kSiteReducePar, v[q], col + (q & 3));
     }
     if (col < DN) {
       // noisy forward direction + clean stream

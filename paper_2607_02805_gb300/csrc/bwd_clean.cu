@@ -36,6 +36,10 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   const bool act = d < g.D;
   const int Bs = (int)g.Bs, TS = Bs < 16 ? Bs : 16, NSEG = Bs / TS;
   const int k_lo = chunk_lo(g, c), k_hi = chunk_lo(g, c + 1) - 1;
+  // debug build: the chunk's last token and the channel group lie inside the sizes
+  if (!(dguard(kSiteBwdClean, b, g.Bt) && dguard(kSiteBwdClean, (int64_t)(k_hi + 1) * Bs - 1, g.L) &&
+        dguard(kSiteBwdClean, d0, g.D)))
+    return;
 
   enum { XC = 0, DTC = 1, DYC = 2 };
   enum { BC = 0, CC = 1 };

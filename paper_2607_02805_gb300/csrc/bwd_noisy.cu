@@ -41,6 +41,10 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   const bool act = d < g.D;
   const int Bs = (int)g.Bs, TS = Bs < 16 ? Bs : 16, NSEG = Bs / TS;
   const int k_lo = chunk_lo(g, c), k_hi = chunk_lo(g, c + 1) - 1;
+  // debug build: the chunk's last token and the channel group lie inside the sizes
+  if (!(dguard(kSiteBwdNoisy, b, g.Bt) && dguard(kSiteBwdNoisy, (int64_t)(k_hi + 1) * Bs - 1, g.L) &&
+        dguard(kSiteBwdNoisy, d0, g.D)))
+    return;
 
   enum { XN = 0, DTF = 1, DTR = 2, DYN = 3, DTC = 4, DYC = 5 };
   enum { BF = 0, CF = 1, BR = 2, CR = 3, CC = 4 };

@@ -44,6 +44,13 @@ __global__ void __launch_bounds__(kCta) k_chunk_local(const FwdParams p) {
   const int c = blockIdx.y;
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
   const bool act = d < g.D;
+  {  // debug build: the chunk's tokens, channels and state slot lie inside the sizes
+    const int64_t tc = (int64_t)g.m * g.Bs, dl = (d0 + kCta < g.D ? d0 + kCta : g.D) - 1;
+    if (!(dguard(kSiteChunkLocal, b, g.Bt) && dguard(kSiteChunkLocal, (c + 1) * tc - 1, g.L) &&
+          dguard(kSiteChunkLocal, d0, g.D) &&
+          dguard(kSiteChunkLocal, ((b * (g.nc + 1) + c) * g.D + dl) * N + N - 1, g.Bt * (g.nc + 1) * g.D * N)))
+      return;
+  }
   Stage<T, N, 2, 1, 2, 0, REV> st;
   st.carve(smem, kLocalSpan);
   auto prow = [&](int64_t t) { return b * g.L + (REV ? g.L - 1 - t : t); };  // row of logical token t
@@ -93,6 +100,8 @@ __global__ void __launch_bounds__(256) k_chunk_carry(const FwdParams p) {
   if (idx >= g.Bt * g.D * N) return;
   const int n = (int)(idx % N);
   const int64_t d = (idx / N) % g.D, b = idx / ((int64_t)N * g.D);
+  // debug build: the last state slot this thread writes (no barrier follows)
+  if (!dguard(kSiteChunkCarry, ((b * (g.nc + 1) + g.nc_full) * g.D + d) * N + n, g.Bt * (g.nc + 1) * g.D * N)) return;
   const float A2 = __fmul_rn(p.Af[d * N + n], kLog2e);
   float H = p.init ? p.init[(b * g.D + d) * N + n] : 0.f;
   const int64_t hstride = g.D * N;
@@ -119,6 +128,7 @@ __global__ void __launch_bounds__(256) k_chunk_carry(const FwdParams p) {
     H = __fmaf_rn(ex2(__fmul_rn(A2, s)), H, hl);
   }
   hs[(int64_t)g.nc_full * hstride] = H;
+  dfinite(kSiteChunkCarry, H, idx);  // debug build: a non-finite cached state
 }
 
 // MODE 0: all-block forward (clean + noisy). MODE 1: clean scan only (cache
@@ -150,6 +160,10 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
   const int c = p.c_begin + blockIdx.y;
   const int64_t d0 = (int64_t)blockIdx.x * kCta, d = d0 + threadIdx.x;
   const bool act = d < g.D;
+  // debug build: the chunk's first token and the channel group lie inside the sizes
+  if (!(dguard(kSiteBlockScan, b, g.Bt) && dguard(kSiteBlockScan, (int64_t)c * g.m * g.Bs, g.L) &&
+        dguard(kSiteBlockScan, d0, g.D)))
+    return;
   const int Bs = (int)g.Bs;
   const int SEG = Bs < kScanSeg ? Bs : kScanSeg, NSEG = (Bs + SEG - 1) / SEG;
   // blocks shorter than kScanSeg are staged TB at a time (one tile of at most
@@ -326,6 +340,8 @@ __global__ void __launch_bounds__(2 * kActW, 1) k_active_block(const FwdParams p
   const int lane = threadIdx.x & 31, dir = threadIdx.x >> 5;  // dir 0: forward, 1: reverse
   const int64_t d = d0 + lane;
   const bool act = d < g.D;
+  // debug build: the batch row and the channel group lie inside the sizes
+  if (!(dguard(kSiteActiveBlock, b, g.Bt) && dguard(kSiteActiveBlock, d0, g.D))) return;
   T* td = reinterpret_cast<T*>(smem);
   float* rows = reinterpret_cast<float*>(smem + Ly::td_bytes(Bs) + Ly::raw_bytes(Bs));
   T* raw = is_f32<T>::value ? reinterpret_cast<T*>(rows) : reinterpret_cast<T*>(smem + Ly::td_bytes(Bs));

@@ -74,6 +74,10 @@ __global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdS
   const int64_t bk = blockIdx.x, b = bk / g.nb;
   const int k = (int)(bk % g.nb);
   const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
+  // debug build: the block, the head group and its last state slot lie inside the sizes
+  if (!(dguard(kSiteSsdBlockState, bk, g.Bt * g.nb) && dguard(kSiteSsdBlockState, h0, H) &&
+        dguard(kSiteSsdBlockState, ((bk * H + h1 - 1) * kSsdP + kSsdP - 1) * N + N - 1, g.Bt * g.nb * H * kSsdP * N)))
+    return;
   const RowMap tok(b, g.L, (int64_t)k * Bs, p.rev != 0);
   float* s_w = reinterpret_cast<float*>(sm + S.w);  // [hg][256]
   // B rows: chunk c of 8 state indices of token s goes to half c / 8
@@ -203,6 +207,8 @@ __global__ void __launch_bounds__(256) k_ssd_state_pass(const SsdPassParams p) {
   if (idx >= g.Bt * per_b) return;
   const int64_t b = idx / per_b, r = idx - b * per_b;
   const int h = (int)(r / ((int64_t)kSsdP * g.N));
+  // debug build: the last block-state slot this thread reads (no barrier follows)
+  if (!dguard(kSiteSsdStatePass, (b * g.nb + g.nb - 1) * per_b + r, g.Bt * g.nb * per_b)) return;
   const float A2 = __fmul_rn(p.A[h], kLog2e);
   float S = p.init != nullptr ? p.init[idx] : 0.f;
   const float* T = p.T + b * g.nb * per_b + r;
@@ -225,6 +231,7 @@ __global__ void __launch_bounds__(256) k_ssd_state_pass(const SsdPassParams p) {
   }
   if (!p.emit_all) p.states[b * per_b + r] = S;
   if (p.final_state != nullptr) p.final_state[b * per_b + r] = S;
+  dfinite(kSiteSsdStatePass, S, idx);  // debug build: a non-finite cached state
 }
 
 // Copies one 128-token tile of a [tokens][N] bf16 tensor into K-major
@@ -353,6 +360,8 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   const int64_t bk = idx / m, b = bk / g.nb;
   const int k = (int)(bk % g.nb);
   const int h0 = blockIdx.y * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
+  // debug build: the tile and the head group lie inside the sizes
+  if (!(dguard(kSiteSsdBlockScan, idx, g.Bt * g.nb * m) && dguard(kSiteSsdBlockScan, h0, H))) return;
   const RowMap tok(b, g.L, (int64_t)k * Bs, p.rev != 0);
   const int row = 32 * q4 + lane, tt = i * kSsdT + row;  // token row in the tile / in the block
   const int rg = 4 * i + q4;                              // 32-token row group in the block

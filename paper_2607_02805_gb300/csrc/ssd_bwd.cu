@@ -156,6 +156,11 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
   const int k = (int)(bk % g.nb);
   const int grp = blockIdx.y, ngrp = gridDim.y;
   const int h0 = grp * p.hg, h1 = min(H, h0 + p.hg), hg = h1 - h0;
+  // debug build: the tile, the head group and its last dx partial lie inside the sizes
+  if (!(dguard(kSiteSsdBwdTile, idx, g.Bt * g.nb * m) && dguard(kSiteSsdBwdTile, h0, H) &&
+        dguard(kSiteSsdBwdTile, (((bk * H + h1 - 1) * m + i) * Bs + Bs - 1) * kSsdP + kSsdP - 1,
+               g.Bt * g.nb * H * m * g.Bs * kSsdP)))
+    return;
   const int64_t tok0 = b * g.L + (int64_t)k * Bs;  // the block's first token
   const int64_t HP = (int64_t)H * kSsdP;
   float* s_c = reinterpret_cast<float*>(sm + S::VEC);
@@ -610,6 +615,8 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
   const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x, w = t >> 5, lane = t & 31;
   const int64_t bk = blockIdx.x, b = bk / g.nb;
   const int k = (int)(bk % g.nb), h = blockIdx.y;
+  // debug build: the block and the head lie inside the sizes
+  if (!(dguard(kSiteSsdBwdState, bk, g.Bt * g.nb) && dguard(kSiteSsdBwdState, h, H))) return;
   const int64_t tok0 = b * g.L + (int64_t)k * Bs, HP = (int64_t)H * kSsdP, PN = (int64_t)kSsdP * N;
   float* s_suf = reinterpret_cast<float*>(sm + S::VEC);  // inclusive suffix sums of dt, then exclusive
   float* s_dt = s_suf + 256;

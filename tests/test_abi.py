@@ -1,6 +1,7 @@
 """The C ABI on the host: the library builds and loads, exports every function
 include/bdscan.h declares, and rejects bad arguments before touching a GPU."""
 
+import ctypes
 import os
 import re
 
@@ -307,3 +308,24 @@ def test_binding_argument_counts_match_the_headers():
     assert set(protos) == set(header_functions())
     for name, _, args in binding.SIGNATURES:
         assert len(args) == protos[name], (name, len(args), protos[name])
+
+
+def test_release_build_has_no_device_checks():
+    assert binding.bdscan_debug_build() == 0
+    rc = binding.bdscan_debug_set_slack(1)
+    assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "release build" in binding.bdscan_last_error()
+
+
+def test_debug_build_exports_the_same_functions():
+    """The debug build (BDSCAN_DEBUG=1) builds, loads, exports every declared
+    function, says it is the debug build, and validates on the host exactly
+    like the release build (no GPU is touched before a launch)."""
+    lib = binding.load(debug=True)
+    for name in header_functions():
+        assert hasattr(lib, name), name
+    assert lib.bdscan_debug_build() == 1
+    assert lib.bdscan_debug_set_slack(-1) == binding.BDSCAN_ERR_ARG
+    assert b"negative slack" in lib.bdscan_last_error()
+    d = binding.make_dims(1, 64, 16, 32, 3, binding.BDSCAN_F32)
+    rc = lib.bdscan_forward(ctypes.byref(d), None, None, None, None, None, None, None, 0, None)
+    assert rc == binding.BDSCAN_ERR_UNSUPPORTED and b"d_state 3" in lib.bdscan_last_error()
