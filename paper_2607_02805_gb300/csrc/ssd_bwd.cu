@@ -79,6 +79,37 @@ __device__ __forceinline__ void stage_f32_as_bf16(unsigned char* dst, const floa
   }
 }
 
+// An fp32 [ROWS][NC] matrix (row stride NC) as bf16 high parts bf16(v) at
+// `dhi` and low parts bf16(v - bf16(v)) at `dlo` (atom columns of ROWS * 128
+// bytes each), by NT threads; every load is issued before the first store.
+template <int NT, int ROWS, int NC>
+__device__ __forceinline__ void stage_f32_hilo(unsigned char* dhi, unsigned char* dlo, const float* src) {
+  constexpr int cpr = NC / 8, per = ROWS * cpr / NT;
+  static_assert(ROWS * cpr % NT == 0, "whole chunks per thread");
+  float4 a[per], b[per];
+#pragma unroll
+  for (int q = 0; q < per; ++q) {
+    const int c = (int)threadIdx.x + q * NT, r = c / cpr, ch = c % cpr;
+    a[q] = *reinterpret_cast<const float4*>(src + (int64_t)r * NC + ch * 8);
+    b[q] = *reinterpret_cast<const float4*>(src + (int64_t)r * NC + ch * 8 + 4);
+  }
+#pragma unroll
+  for (int q = 0; q < per; ++q) {
+    const int c = (int)threadIdx.x + q * NT, r = c / cpr, ch = c % cpr;
+    const float v[8] = {a[q].x, a[q].y, a[q].z, a[q].w, b[q].x, b[q].y, b[q].z, b[q].w};
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+      hi[e] = *reinterpret_cast<const uint32_t*>(&hv);
+      lo[e] = pack_bf16(__fsub_rn(v[2 * e], __low2float(hv)), __fsub_rn(v[2 * e + 1], __high2float(hv)));
+    }
+    const uint32_t off = (uint32_t)(ch >> 3) * (uint32_t)ROWS * 128u + sw128((uint32_t)r, (uint32_t)(ch & 7));
+    *reinterpret_cast<uint4*>(dhi + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    *reinterpret_cast<uint4*>(dlo + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+  }
+}
+
 // Element `col` of row `row` of a bf16 tile in swizzled atom columns of 128 rows.
 __device__ __forceinline__ float tile_at(const unsigned char* tile, int row, int col) {
   const uint32_t off = (uint32_t)(col >> 6) * kTile16 + sw128((uint32_t)row, (uint32_t)((col & 63) >> 3)) + (uint32_t)(col & 7) * 2u;
@@ -103,30 +134,21 @@ __device__ __forceinline__ void tmem_st32(uint32_t ta, const float (&v)[32]) {
 //   C    C of tile i, [128 t][128 n] (n >= N zero)    BT  B of s-tile j, [128 s][N]
 //   X    x of s-tile j, one head, [128 s][64 p]       DY  dy of tile i, one head, [128 t][64 p]
 //   M    one head's G o decay o dt, [128 t][128 s]
-//   COL  R' of 64 columns, [128][65] fp32             VEC c and dt of one head's block
+//   COL  R' of 64 columns, [128][65] fp32
+//   VEC  c and dt of the block for every head of the group, [2][16][256] fp32
 //   CP   column-sum partials of four row quarters, [4][64] fp32
-//   ROWS row sums and row dots per column half and head of the group, [2][16][128] fp32 each
+//   ROWS row sums per head of the group [16][128], row dots per column half [2][16][128]
 // After a s-tile's heads, the head-summed dG goes to M (bf16 high part) and
 // X + DY (low part). The seed phase uses DY, BT for E o dy, M for the seed's
 // bf16 high and low parts.
 struct TileSmem {
   static constexpr uint32_t C = 0, BT = 32768, X = 65536, DY = 81920, M = 98304, COL = 131072;
   static constexpr uint32_t VEC = COL + 128u * 65u * 4u;
-  static constexpr uint32_t CP = VEC + 2u * 256u * 4u;
+  static constexpr uint32_t CP = VEC + 2u * 16u * 256u * 4u;
   static constexpr uint32_t ROWS = CP + 4u * 64u * 4u;
-  static constexpr uint32_t total = ROWS + 2u * 2u * 16u * 128u * 4u + 1024u;
+  static constexpr uint32_t total = ROWS + 3u * 16u * 128u * 4u + 1024u;
 };
 constexpr int kMaxBwdHeads = 16;  // heads per tile CTA
-
-// dt of head h over the block into s_dt (by NT threads), and its in-block
-// cumulative sums (inclusive; suffix sums for the reverse direction) into s_c
-// by warp 0.
-template <bool UPPER, int NT>
-__device__ __forceinline__ void block_dt(const __nv_bfloat16* dt, int64_t tok0, int H, int h, int Bs, float* s_dt,
-                                         float* s_c) {
-  for (int s = threadIdx.x; s < Bs; s += NT) s_dt[s] = __bfloat162float(dt[(tok0 + s) * H + h]);
-  if ((threadIdx.x >> 5) == 0) warp_scan_dt<UPPER>(dt + tok0 * H + h, H, Bs, s_c);
-}
 
 // One CTA of 8 warps per (batch row, block, tile i) and group of heads. Token
 // row t of tile i (TMEM lane t) has two threads, t and t + 128: the first
@@ -163,20 +185,27 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     return;
   const int64_t tok0 = b * g.L + (int64_t)k * Bs;  // the block's first token
   const int64_t HP = (int64_t)H * kSsdP;
-  float* s_c = reinterpret_cast<float*>(sm + S::VEC);
-  float* s_dt = s_c + 256;
+  float* s_cv = reinterpret_cast<float*>(sm + S::VEC);  // [hh][256]: c of every head of the group
+  float* s_dtv = s_cv + kMaxBwdHeads * 256;              // [hh][256]: dt
   float* s_col = reinterpret_cast<float*>(sm + S::COL);
   float* s_cp = reinterpret_cast<float*>(sm + S::CP);
-  float* s_rows = reinterpret_cast<float*>(sm + S::ROWS) + half * kMaxBwdHeads * 128;  // [hh][128] of this half
-  float* s_dots = s_rows + 2 * kMaxBwdHeads * 128;
+  float* s_rows = reinterpret_cast<float*>(sm + S::ROWS);                              // [hh][128]
+  float* s_dots = s_rows + kMaxBwdHeads * 128 + half * kMaxBwdHeads * 128;             // [hh][128] of this half
 
   stage_bf16<NT>(sm + S::C, p.C + (tok0 + i * kSsdT) * N, N, 128, N);
   if (N == 64)
     for (int c = tid; c < 128 * 8; c += NT) *reinterpret_cast<uint4*>(sm + S::C + kTile16 + c * 16) = make_uint4(0u, 0u, 0u, 0u);
   cp_async_commit();
   for (int hh = 0; hh < kMaxBwdHeads; ++hh) {
-    s_rows[hh * 128 + t] = 0.f;
+    if (half == 0) s_rows[hh * 128 + t] = 0.f;
     s_dots[hh * 128 + t] = 0.f;
+  }
+  // dt and its in-block cumulative sums of every head of the group, once per
+  // CTA: warp w takes heads w, w + 8
+  for (int hh = w; hh < hg; hh += NT / 32) {
+    const int h = h0 + hh;
+    for (int q = tid & 31; q < Bs; q += 32) s_dtv[hh * 256 + q] = __bfloat162float(p.dt[(tok0 + q) * H + h]);
+    warp_scan_dt<UPPER>(p.dt + tok0 * H + h, H, Bs, s_cv + hh * 256);
   }
   if (tid == 0) umma::bar_init(&bar, 1);
   if (w == 0) tmem_alloc(&tslot, 512);
@@ -202,7 +231,15 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
   const int j0 = UPPER ? i : 0, j1 = UPPER ? m - 1 : i;
   for (int j = j0; j <= j1 && alive; ++j) {
     const int64_t sr0 = tok0 + (int64_t)j * kSsdT;
+    // x and dy of head hh are staged after head hh-1's dx products (head 0's
+    // with B_j): the copies run during the previous head's epilogue
+    auto stage_head = [&](int hh) {
+      const int h = h0 + hh;
+      stage_bf16<NT>(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
+      stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+    };
     stage_bf16<NT>(sm + S::BT, p.B + sr0 * N, N, 128, N);
+    stage_head(0);
     cp_async_commit();
     cp_async_wait_all();
     umma::fence_async_smem();
@@ -220,10 +257,6 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     if (!(alive = wait_mma())) break;
     for (int hh = 0; hh < hg; ++hh) {
       const int h = h0 + hh;
-      stage_bf16<NT>(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
-      stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
-      cp_async_commit();
-      block_dt<UPPER, NT>(p.dt, tok0, H, h, Bs, s_dt, s_c);
       cp_async_wait_all();
       umma::fence_async_smem();
       umma::fence_before_sync();
@@ -237,6 +270,8 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
         umma::mma_commit(&bar);
       }
       if (!(alive = wait_mma())) break;
+      const float* s_c = s_cv + hh * 256;
+      const float* s_dt = s_dtv + hh * 256;
       const float A2 = __fmul_rn(p.A[h], kLog2e), ct = s_c[tt];
       float rowsum = 0.f;
       // two rounds: round r takes 32-column chunk r (first half) and 2 + r
@@ -294,7 +329,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
           p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + tc] = sum;
         }
       }
-      s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);
+      if (half == 0) s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);  // the second half after the barrier
       tmem_wait_st();
       umma::fence_async_smem();
       umma::fence_before_sync();
@@ -307,12 +342,32 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
                          id_dx, kk > 0);
         umma::mma_commit(&bar);
       }
+      if (half == 1) s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);
       if (!(alive = wait_mma())) break;
-      {  // row s = j*128 + t of head h's dx contribution from tile i, 32 channels per half
+      if (hh + 1 < hg) {  // X and DY are free: the next head's copies start now
+        stage_head(hh + 1);
+        cp_async_commit();
+      }
+      {  // head h's dx contribution from tile i, rows j*128 + 32 (w mod 4) .. of
+         // channels 32 half ..: the warp's 32 x 32 block is transposed through
+         // COL (float pairs, XOR-swizzled by row) so that each store writes
+         // two 128-byte row segments
         float v[32];
-        float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + t) * kSsdP + 32 * half;
         umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)half, v);
-        store_row(dxo, v);
+        float* tb = s_col + w * 1024;
+        const int r = tid & 31;
+#pragma unroll
+        for (int c2 = 0; c2 < 16; ++c2)
+          *reinterpret_cast<float2*>(tb + r * 32 + 2 * (c2 ^ (r & 15))) = make_float2(v[2 * c2], v[2 * c2 + 1]);
+        __syncwarp();
+        const int c2 = r & 15;
+        float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + 32 * (w & 3)) * kSsdP + 32 * half + 2 * c2;
+#pragma unroll 4
+        for (int rr = 0; rr < 32; rr += 2) {
+          const int row = rr + (r >> 4);
+          *reinterpret_cast<float2*>(dxo + row * kSsdP) =
+              *reinterpret_cast<const float2*>(tb + row * 32 + 2 * (c2 ^ (row & 15)));
+        }
       }
       umma::fence_before_sync();
     }
@@ -381,12 +436,11 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
       cp_async_commit();
       const float* seed = p.states + ((b * g.nb + k - 1) * H + h) * (int64_t)kSsdP * N;
-      stage_f32_as_bf16<NT>(sm + S::M, seed, 64, N, false);
-      stage_f32_as_bf16<NT>(sm + S::M + 16384u, seed, 64, N, true);
-      block_dt<false, NT>(p.dt, tok0, H, h, Bs, s_dt, s_c);
+      stage_f32_hilo<NT, 64, N>(sm + S::M, sm + S::M + 16384u, seed);
       cp_async_wait_all();
       __syncthreads();
-      const float E = ex2(__fmul_rn(__fmul_rn(p.A[h], kLog2e), s_c[tt]));
+      // the seeded direction is the forward one: s_cv holds prefix sums
+      const float E = ex2(__fmul_rn(__fmul_rn(p.A[h], kLog2e), s_cv[hh * 256 + tt]));
 #pragma unroll
       for (int cq = 0; cq < 4; ++cq) {  // 16-byte chunks 4 half .. 4 half + 3 of row t
         const int ch = 4 * half + cq;
@@ -450,11 +504,10 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
   }
   __syncthreads();  // both halves' row sums and dots are in shared memory
   if (alive) {
-    const float* rows = reinterpret_cast<const float*>(sm + S::ROWS);  // [half][hh][128]
-    const float* dots = rows + 2 * kMaxBwdHeads * 128;
+    const float* dots = s_rows + kMaxBwdHeads * 128;  // [half][hh][128]
     for (int hh = half; hh < hg; hh += 2) {
       const int h = h0 + hh;
-      p.rowsum[(bk * H + h) * Bs + tt] = __fadd_rn(rows[hh * 128 + t], rows[(kMaxBwdHeads + hh) * 128 + t]);
+      p.rowsum[(bk * H + h) * Bs + tt] = s_rows[hh * 128 + t];
       if (SEED) p.rowdot[(bk * H + h) * Bs + tt] = __fadd_rn(dots[hh * 128 + t], dots[(kMaxBwdHeads + hh) * 128 + t]);
     }
   }

@@ -34,10 +34,16 @@ template <bool REV>
 __device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t stride, int n, float* out) {
   const int lane = threadIdx.x & 31, per = n / 32;
   float loc[8];
-  float s = 0.f;
-  for (int q = 0; q < per; ++q) {
+  // all of the lane's loads are issued before the first add (n <= 256)
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
     const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
-    s = __fadd_rn(s, __bfloat162float(dt[pos * stride]));
+    loc[q] = q < per ? __bfloat162float(dt[pos * stride]) : 0.f;
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    s = q < per ? __fadd_rn(s, loc[q]) : s;
     loc[q] = s;
   }
   float inc = s;
@@ -48,9 +54,10 @@ __device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t s
   }
   float base = __shfl_up_sync(0xffffffffu, inc, 1);
   if (lane == 0) base = 0.f;
-  for (int q = 0; q < per; ++q) {
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
     const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
-    out[pos] = __fadd_rn(base, loc[q]);
+    if (q < per) out[pos] = __fadd_rn(base, loc[q]);
   }
   return __shfl_sync(0xffffffffu, inc, 31);  // total
 }
