@@ -53,32 +53,6 @@ __device__ __forceinline__ void stage_bf16(unsigned char* dst, const __nv_bfloat
   }
 }
 
-// An fp32 [rows][ncols] matrix (row stride ncols) as bf16 atom columns (rows * 128
-// bytes each) by NT threads; `lo` selects the rounding residual v - bf16(v)
-// instead of bf16(v).
-template <int NT>
-__device__ __forceinline__ void stage_f32_as_bf16(unsigned char* dst, const float* src, int rows, int ncols, bool lo) {
-  const int cpr = ncols / 8;
-  for (int c = threadIdx.x; c < rows * cpr; c += NT) {
-    const int r = c / cpr, ch = c % cpr;
-    const float4 a = *reinterpret_cast<const float4*>(src + (int64_t)r * ncols + ch * 8);
-    const float4 b = *reinterpret_cast<const float4*>(src + (int64_t)r * ncols + ch * 8 + 4);
-    float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-    uint32_t w[4];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      float x0 = v[2 * e], x1 = v[2 * e + 1];
-      if (lo) {
-        x0 = __fsub_rn(x0, __bfloat162float(__float2bfloat16_rn(x0)));
-        x1 = __fsub_rn(x1, __bfloat162float(__float2bfloat16_rn(x1)));
-      }
-      w[e] = pack_bf16(x0, x1);
-    }
-    *reinterpret_cast<uint4*>(dst + (uint32_t)(ch >> 3) * (uint32_t)rows * 128u + sw128((uint32_t)r, (uint32_t)(ch & 7))) =
-        make_uint4(w[0], w[1], w[2], w[3]);
-  }
-}
-
 // An fp32 [ROWS][NC] matrix (row stride NC) as bf16 high parts bf16(v) at
 // `dhi` and low parts bf16(v - bf16(v)) at `dlo` (atom columns of ROWS * 128
 // bytes each), by NT threads; every load is issued before the first store.
@@ -648,8 +622,27 @@ __global__ void __launch_bounds__(256) k_ssd_bwd_pass(const SsdBwdPassParams p) 
 // B of one s-tile, per-token vectors of the block.
 struct StateBwdSmem {
   static constexpr uint32_t GH = 0, GL = 16384, X = 32768, BT = 49152, VEC = 81920;
-  static constexpr uint32_t total = VEC + 5u * 256u * 4u + 1024u;
+  static constexpr uint32_t TR = VEC + 5u * 256u * 4u;  // per-warp 32 x 32 fp32 transposition blocks
+  static constexpr uint32_t total = TR + 4u * 4096u + 1024u;
 };
+
+// Stores a warp's 32 x 32 fp32 block (lane r holds row r in v) to rows
+// dst + r * ld, through a warp-private XOR-swizzled buffer `tb` so that each
+// store instruction writes two 128-byte row segments.
+__device__ __forceinline__ void store_block32(float* dst, int64_t ld, const float (&v)[32], float* tb) {
+  const int r = threadIdx.x & 31;
+#pragma unroll
+  for (int c2 = 0; c2 < 16; ++c2)
+    *reinterpret_cast<float2*>(tb + r * 32 + 2 * (c2 ^ (r & 15))) = make_float2(v[2 * c2], v[2 * c2 + 1]);
+  __syncwarp();
+  const int c2 = r & 15;
+#pragma unroll 4
+  for (int rr = 0; rr < 32; rr += 2) {
+    const int row = rr + (r >> 4);
+    *reinterpret_cast<float2*>(dst + row * ld + 2 * c2) = *reinterpret_cast<const float2*>(tb + row * 32 + 2 * (c2 ^ (row & 15)));
+  }
+  __syncwarp();
+}
 
 // One CTA of 4 warps per (batch row, block, head) of the clean stream, with
 // gS = the gradient of the state after the block: U = B gS^T and V = x gS per
@@ -677,15 +670,41 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
   float* s_dw = s_w + 256;
   float* s_e = s_dw + 256;
   const float* gS = p.gS + (bk * H + h) * PN;
-  stage_f32_as_bf16<kBwdThreads>(sm + S::GH, gS, 64, N, false);
-  stage_f32_as_bf16<kBwdThreads>(sm + S::GL, gS, 64, N, true);
   for (int s = t; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
   if (w == 0) warp_scan_dt<true>(p.dt + tok0 * H + h, H, Bs, s_suf);
-  // block decay: da = sum over (p, n) of gS o S_{k-1}
+  // gS as bf16 high and low parts, and the block decay's da = sum over (p, n)
+  // of gS o S_{k-1}: the loads of both matrices are issued first
   float da = 0.f;
-  if (k > 0) {
-    const float* prev = p.states + ((b * g.nb + k - 1) * H + h) * PN;
-    for (int64_t q = t; q < PN; q += kBwdThreads) da = __fmaf_rn(gS[q], prev[q], da);
+  {
+    constexpr int cpr = N / 8, per = 64 * cpr / kBwdThreads;
+    const float* prev = k > 0 ? p.states + ((b * g.nb + k - 1) * H + h) * PN : nullptr;
+    float4 ga[per], gb[per], pa[per], pb[per];
+#pragma unroll
+    for (int q = 0; q < per; ++q) {
+      const int c = t + q * kBwdThreads, r = c / cpr, ch = c % cpr;
+      ga[q] = *reinterpret_cast<const float4*>(gS + r * N + ch * 8);
+      gb[q] = *reinterpret_cast<const float4*>(gS + r * N + ch * 8 + 4);
+      pa[q] = prev != nullptr ? *reinterpret_cast<const float4*>(prev + r * N + ch * 8) : make_float4(0.f, 0.f, 0.f, 0.f);
+      pb[q] = prev != nullptr ? *reinterpret_cast<const float4*>(prev + r * N + ch * 8 + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int q = 0; q < per; ++q) {
+      const int c = t + q * kBwdThreads, r = c / cpr, ch = c % cpr;
+      const float v[8] = {ga[q].x, ga[q].y, ga[q].z, ga[q].w, gb[q].x, gb[q].y, gb[q].z, gb[q].w};
+      const float u[8] = {pa[q].x, pa[q].y, pa[q].z, pa[q].w, pb[q].x, pb[q].y, pb[q].z, pb[q].w};
+      uint32_t hi[4], lo[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+        hi[e] = *reinterpret_cast<const uint32_t*>(&hv);
+        lo[e] = pack_bf16(__fsub_rn(v[2 * e], __low2float(hv)), __fsub_rn(v[2 * e + 1], __high2float(hv)));
+      }
+#pragma unroll
+      for (int e = 0; e < 8; ++e) da = __fmaf_rn(v[e], u[e], da);
+      const uint32_t off = (uint32_t)(ch >> 3) * 64u * 128u + sw128((uint32_t)r, (uint32_t)(ch & 7));
+      *reinterpret_cast<uint4*>(sm + S::GH + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+      *reinterpret_cast<uint4*>(sm + S::GL + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    }
   }
   da = warp_sum(da);
   if (lane == 0) red[w] = da;
@@ -739,7 +758,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
       const int s = j * kSsdT + t;
       const float e = ex2(__fmul_rn(A2, s_suf[s])), ws = __fmul_rn(e, s_dt[s]);
       float v[32], dw = 0.f;
-      float* dxo = p.dx_state + ((bk * H + h) * Bs + s) * kSsdP;
+      float* tb = reinterpret_cast<float*>(sm + S::TR) + w * 1024;
+      const int s0 = j * kSsdT + 32 * w;  // the warp's first row
+      float* dxo = p.dx_state + ((bk * H + h) * Bs + s0) * kSsdP;
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
         umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
@@ -748,15 +769,15 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
           dw = __fmaf_rn(tile_at(sm + S::X, t, 32 * q + e2), v[e2], dw);
           v[e2] = __fmul_rn(ws, v[e2]);
         }
-        store_row(dxo + 32 * q, v);
+        store_block32(dxo + 32 * q, kSsdP, v, tb);
       }
-      float* dbo = p.dB_state + ((bk * H + h) * Bs + s) * N;
+      float* dbo = p.dB_state + ((bk * H + h) * Bs + s0) * N;
 #pragma unroll
       for (int q = 0; q < N / 32; ++q) {
         umma::tmem_ld32(lane_base + 64u + 32u * (uint32_t)q, v);
 #pragma unroll
         for (int e2 = 0; e2 < 32; ++e2) v[e2] = __fmul_rn(ws, v[e2]);
-        store_row(dbo + 32 * q, v);
+        store_block32(dbo + 32 * q, N, v, tb);
       }
       s_w[s] = ws;
       s_dw[s] = dw;
