@@ -307,17 +307,29 @@ __device__ __forceinline__ void issue_head_loads(unsigned char* sm, const ScanSm
   cp_async_commit();
 }
 
-// Inclusive scan over the block of one head's dt held in shared memory
-// (stride `hs` floats between tokens), by one warp; REV scans from the end.
+// Decay vectors of one direction of a head, by one warp, from the head's dt
+// column in shared memory (bf16, stride `hs` between tokens): va = A2 times
+// the inclusive cumulative dt (prefix sums forward, suffix sums reverse: each
+// lane sums its tokens in order, then the lane totals are scanned), vw = dt,
+// and the column factors
+// vc = exp2(va_ref - va_s) vw_s with the reference at the last (forward) or
+// first (reverse) token of s's 32-token column group. Lane l holds the
+// tokens at scan positions l * per .. l * per + per - 1 in registers, so the
+// reference is one shuffle away and every load is issued at once.
 template <bool REV, typename T>
-__device__ __forceinline__ void warp_scan_smem(const T* dt, int hs, int n, float* out) {
-  const int lane = threadIdx.x & 31, per = n / 32;
-  float loc[8];
-  float s = 0.f;
-  for (int q = 0; q < per; ++q) {
+__device__ __forceinline__ void setup_dir(const T* dt, int hs, int n, float A2, float* va, float* vw, float* vc) {
+  const int lane = threadIdx.x & 31, per = n / 32;  // 4 or 8
+  float d[8], a[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
     const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
-    s = __fadd_rn(s, cvt(dt[pos * hs]));
-    loc[q] = s;
+    d[q] = q < per ? cvt(dt[pos * hs]) : 0.f;
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    s = q < per ? __fadd_rn(s, d[q]) : s;
+    a[q] = s;
   }
   float inc = s;
 #pragma unroll
@@ -327,9 +339,17 @@ __device__ __forceinline__ void warp_scan_smem(const T* dt, int hs, int n, float
   }
   float base = __shfl_up_sync(0xffffffffu, inc, 1);
   if (lane == 0) base = 0.f;
-  for (int q = 0; q < per; ++q) {
+#pragma unroll
+  for (int q = 0; q < 8; ++q) a[q] = __fmul_rn(A2, __fadd_rn(base, a[q]));
+  // the group's reference token is scan position 32 g + 31: lane (l | (32/per - 1)), slot per - 1
+  const float ref = __shfl_sync(0xffffffffu, per == 8 ? a[7] : a[3], lane | (32 / per - 1));
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    if (q >= per) break;
     const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
-    out[pos] = __fadd_rn(base, loc[q]);
+    va[pos] = a[q];
+    vw[pos] = d[q];
+    vc[pos] = __fmul_rn(ex2(__fsub_rn(ref, a[q])), d[q]);
   }
 }
 
@@ -434,28 +454,10 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   // forward referenced to the column group's last token, reverse to its first)
   auto setup = [&](int hh, int buf) {
     float* v = vec0 + buf * 1536;
-    if (w == 0) {
-      warp_scan_smem<false>(s_dtf + hh, hg, Bs, v);
-      __syncwarp();
-      const float A2 = __fmul_rn(s_prm[hh], kLog2e);
-      for (int s = lane; s < Bs; s += 32) {
-        v[s] = __fmul_rn(A2, v[s]);
-        v[256 + s] = __bfloat162float(s_dtf[s * hg + hh]);
-      }
-      __syncwarp();
-      for (int s = lane; s < Bs; s += 32) v[512 + s] = __fmul_rn(ex2(__fsub_rn(v[(s & ~31) + 31], v[s])), v[256 + s]);
-    } else if (NOISY && w == 1) {
-      warp_scan_smem<true>(s_dtr + hh, hg, Bs, v + 768);
-      __syncwarp();
-      const float A2 = __fmul_rn(s_prm[32 + hh], kLog2e);
-      for (int s = lane; s < Bs; s += 32) {
-        v[768 + s] = __fmul_rn(A2, v[768 + s]);
-        v[1024 + s] = __bfloat162float(s_dtr[s * hg + hh]);
-      }
-      __syncwarp();
-      for (int s = lane; s < Bs; s += 32)
-        v[1280 + s] = __fmul_rn(ex2(__fsub_rn(v[768 + (s & ~31)], v[768 + s])), v[1024 + s]);
-    }
+    if (w == 0)
+      setup_dir<false>(s_dtf + hh, hg, Bs, __fmul_rn(s_prm[hh], kLog2e), v, v + 256, v + 512);
+    else if (NOISY && w == 1)
+      setup_dir<true>(s_dtr + hh, hg, Bs, __fmul_rn(s_prm[32 + hh], kLog2e), v + 768, v + 1024, v + 1280);
   };
   if (alive && h0 < h1) setup(0, 0);
   // mixing tile j of head hh into shared buffer mt: this warp's two 32-column
@@ -625,7 +627,11 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       const float Dd = NOISY ? __fadd_rn(s_prm[16 + hh], s_prm[48 + hh]) : s_prm[16 + hh];
       const int64_t off = (tok(tt) * H + h) * kSsdP + 32 * hf;
       const unsigned char* xr = sm + xcur + (uint32_t)i * 16384u;
-      uint4* yg = reinterpret_cast<uint4*>(p.y + off);
+      // bf16 output: the warp's 32 rows x 64 bytes go through a 2 KB block of
+      // m0 (free until the next head's mixing tile; 16-byte chunks XOR-swizzled
+      // by row pair) and are stored as 64-byte row segments, 8 rows per store
+      unsigned char* yb = sm + L.m0 + w * 2048u;
+      const int lr = row & 31;
 #pragma unroll
       for (int ch = 0; ch < 4; ++ch) {
         const uint4 xv = *reinterpret_cast<const uint4*>(xr + sw128(row, 4 * hf + ch));
@@ -650,7 +656,18 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
           o[3] = __fadd_rn(u0.w, o[3]); o[4] = __fadd_rn(u1.x, o[4]); o[5] = __fadd_rn(u1.y, o[5]);
           o[6] = __fadd_rn(u1.z, o[6]); o[7] = __fadd_rn(u1.w, o[7]);
         }
-        yg[ch] = make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]), pack_bf16(o[6], o[7]));
+        *reinterpret_cast<uint4*>(yb + lr * 64 + 16 * (ch ^ ((lr >> 1) & 3))) =
+            make_uint4(pack_bf16(o[0], o[1]), pack_bf16(o[2], o[3]), pack_bf16(o[4], o[5]), pack_bf16(o[6], o[7]));
+      }
+      if (p.y32 == nullptr) {
+        __syncwarp();
+        const int ch = lane & 3;
+#pragma unroll
+        for (int rr = 0; rr < 32; rr += 8) {
+          const int r2 = rr + (lane >> 2), tr = i * kSsdT + 32 * q4 + r2;  // row of the warp, token of the block
+          *reinterpret_cast<uint4*>(p.y + (tok(tr) * H + h) * kSsdP + 32 * hf + 8 * ch) =
+              *reinterpret_cast<const uint4*>(yb + r2 * 64 + 16 * (ch ^ ((r2 >> 1) & 3)));
+        }
       }
     }
     umma::fence_before_sync();
