@@ -844,6 +844,86 @@ def run_ssd_cache(args, L=65536, Bs=256, calls=16):
         "graph_replay_us_per_call": graph_us, "wait_flag": flag}), flush=True)
 
 
+def run_mixer(args):
+    """The mixer around the scan (conv1d of width 4 with SiLU, softplus step
+    size, SiLU gate) at the benchmark layer's geometry: all-block forward then
+    the backward of every input, against the bare scan's forward + backward on
+    the same sizes."""
+    import torch
+    from paper_2607_02805_gb300 import binding
+    from paper_2607_02805_gb300.inputs import MixerWorkload, Workload
+    from paper_2607_02805_gb300.layer import Layer, to_device
+    Bt, L, Bs, D, N = (args.batch or 8), 2048, 16, 1536, 16
+    code = binding.BDSCAN_BF16
+    wl = MixerWorkload(Bt, L, Bs, D, N, dtype="bf16", seed=0)
+    t = {k: to_device(wl.dev_bits(k), code, "cuda") for k in wl.t32}
+    dims = binding.make_dims(Bt, L, Bs, D, N, code)
+    out_c = torch.empty((Bt, L, D), dtype=torch.bfloat16, device="cuda")
+    out_n = torch.empty_like(out_c)
+    st = torch.empty((Bt, L // Bs, D, N), dtype=torch.float32, device="cuda")
+    wsf = torch.empty(binding.bdscan_mixer_forward_workspace_size(dims), dtype=torch.uint8, device="cuda")
+    wsb = torch.empty(binding.bdscan_mixer_backward_workspace_size(dims), dtype=torch.uint8, device="cuda")
+    per_ch = ("A_f", "D_f", "A_r", "D_r", "conv_w", "conv_b", "dt_bias_f", "dt_bias_r")
+    g = {k: torch.empty(v.shape, dtype=torch.float32 if k in per_ch else torch.bfloat16, device="cuda")
+         for k, v in t.items() if k not in ("dy_c", "dy_n")}
+    stream = torch.cuda.current_stream()
+
+    def step_mixer():
+        binding.mixer_forward(dims, t, out_c, out_n, st, wsf, stream)
+        binding.mixer_backward(dims, t, t["dy_c"], t["dy_n"], None, g, wsb, stream)
+
+    lay = Layer(Workload(Bt, L, Bs, D, N, dtype="bf16", seed=0, with_grads=True), device="cuda")
+    lay.alloc_backward()
+
+    def step_scan():
+        lay.forward(stream)
+        lay.backward(stream, use_dstates=False)
+
+    res = {}
+    for name, fn in (("mixer", step_mixer), ("scan", step_scan)):
+        for _ in range(max(3, args.warmup)):
+            fn()
+        reps = max(3, min(args.steps, 50))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        res[name] = e0.elapsed_time(e1) / reps
+    # per-launch times of one forward and one backward (the events hook records
+    # an event after each launch)
+    per_launch = {}
+    for name, fn in (("forward", lambda: binding.mixer_forward(dims, t, out_c, out_n, st, wsf, stream)),
+                     ("backward", lambda: binding.mixer_backward(dims, t, t["dy_c"], t["dy_n"], None, g, wsb,
+                                                                 stream))):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(33)]
+        for e in evs:
+            e.record(stream)
+        torch.cuda.synchronize()
+        arr = (ctypes.c_void_p * 32)(*[e.cuda_event for e in evs[1:]])
+        evs[0].record(stream)
+        binding.bdscan_profile_events(arr, 32)
+        fn()
+        n = binding.bdscan_last_launch_count()
+        binding.bdscan_profile_events(None, 0)
+        torch.cuda.synchronize()
+        per_launch[name] = [round(1e3 * evs[j].elapsed_time(evs[j + 1]), 1) for j in range(min(n, 32))]
+    print(json.dumps({
+        "metric": "mixer (conv1d + softplus + gate around the block-bidirectional scan) forward+backward tokens/s",
+        "value": Bt * L / (res["mixer"] * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": reps,
+        "ms_per_step": res["mixer"], "higher_is_better": True, "dtype": "bf16 I/O, fp32 scan inputs and state",
+        "data": "synthetic",
+        "config": {"workload": f"87M-scale layer geometry with the mixer around the scan: batch {Bt}, {L} tokens "
+                               f"per stream, block {Bs}, d_inner {D}, d_state {N}; all-block forward then the "
+                               "backward of every input", "batch": Bt, "seq_len": L, "block": Bs, "d_inner": D,
+                   "d_state": N},
+        "scan_only_ms_per_step": round(res["scan"], 4),
+        "mixer_overhead_ms": round(res["mixer"] - res["scan"], 4),
+        "launch_us": per_launch}), flush=True)
+
+
 def run_prefill(args, L, Bs, calls):
     """Inference cache path at d_inner 2048, d_state 16, batch 1: the cache
     build over an L-token clean prefix (final state only, and every block-end
@@ -944,6 +1024,43 @@ def run_prefill(args, L, Bs, calls):
         graph_us = 1e3 * e0.elapsed_time(e1) / (reps * calls)
     except Exception as exc:  # report the failure in the line, keep the rest
         graph_us = f"capture failed: {exc}"
+    # the same calls with AdaLN on the block (a fresh modulation per step),
+    # replayed as one CUDA graph
+    adaln_us = None
+    try:
+        from paper_2607_02805_gb300.inputs import draw
+        mods = [{k: torch.from_numpy(draw(k, (1, D), 5, j + 1)).cuda() for k in ("shift", "scale", "gate")}
+                for j in range(calls)]
+        ws_ad = torch.empty(max(1, (binding.bdscan_active_block_adaln_workspace_size(bdims) + 3) // 4),
+                            dtype=torch.float32, device="cuda")
+
+        def call_ad(j, s):
+            m = mods[j]
+            binding.active_block_adaln(bdims, seed, blocks[j][0], m["shift"], m["scale"], m["gate"], 1e-5,
+                                       blocks[j][1], ws_ad, s)
+
+        for j in range(calls):
+            call_ad(j, stream)
+        torch.cuda.synchronize()
+        g2 = torch.cuda.CUDAGraph()
+        side2 = torch.cuda.Stream()
+        side2.wait_stream(stream)
+        with torch.cuda.graph(g2, stream=side2):
+            for j in range(calls):
+                call_ad(j, side2)
+        torch.cuda.synchronize()
+        g2.replay()
+        torch.cuda.synchronize()
+        reps = 20
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            g2.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        adaln_us = 1e3 * e0.elapsed_time(e1) / (reps * calls)
+    except Exception as exc:
+        adaln_us = f"capture failed: {exc}"
     # the same layer step without the cache: a full-sequence bidirectional
     # layer (DiffuMamba) rescans the whole sequence in both directions at every
     # denoising step, because its reverse states depend on the active block
@@ -981,7 +1098,7 @@ def run_prefill(args, L, Bs, calls):
         "config": {"workload": f"active block of {Bs} tokens from the cached state of a {L}-token prefix, "
                                "d_inner 2048, d_state 16, batch 1, bf16", "calls": calls},
         "per_call_us": [round(u, 2) for u in per_call], "graph_replay_us_per_call": graph_us,
-        "bytes_per_call": blk_bytes}), flush=True)
+        "adaln_graph_replay_us_per_call": adaln_us, "bytes_per_call": blk_bytes}), flush=True)
 
 
 def run_e2e(lay, wl, stream, dev, args, full_readback=False):
@@ -1061,7 +1178,8 @@ def main():
     ap.add_argument("--warmup-seconds", type=float, default=1.0,
                     help="keep warming up for at least this long (clock sampling under load)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (smaller profiling case)")
-    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k", "ssd", "ssd_cache", "ssd_train"],
+    ap.add_argument("--workload", default="layer", choices=["layer", "sweep", "prefill65k", "prefill262k", "ssd", "ssd_cache", "ssd_train",
+                             "mixer"],
                     help="layer: the step line; others: extra lines on one GPU")
     args = ap.parse_args()
     if args.batch:
@@ -1082,6 +1200,8 @@ def main():
                 run_ssd_cache(args)
             elif args.workload == "ssd_train":
                 run_ssd_train(args)
+            elif args.workload == "mixer":
+                run_mixer(args)
             elif args.workload == "prefill65k":
                 run_prefill(args, 65536, 32, 1)
             else:

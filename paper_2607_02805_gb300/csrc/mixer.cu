@@ -24,14 +24,20 @@ namespace {
 constexpr int kW = 4;           // convolution width
 constexpr int kParSplit = 64;   // token slices of the parameter-gradient reduction
 
-__device__ __forceinline__ float sigm(float z) { return __fdiv_rn(1.f, __fadd_rn(1.f, expf(-z))); }
+// The logistic function and softplus on the fast hardware paths (__expf,
+// __logf, __fdividef): relative errors of order 1e-6, far inside the
+// tolerance of the path, and the same functions serve every entry point, so
+// the cache paths stay bit-identical to the all-block ones.
+__device__ __forceinline__ float sigm(float z) { return __fdividef(1.f, __fadd_rn(1.f, __expf(-z))); }
 __device__ __forceinline__ float silu(float z) { return __fmul_rn(z, sigm(z)); }
 // d SiLU / dz = s (1 + z (1 - s))
 __device__ __forceinline__ float dsilu(float z) {
   const float s = sigm(z);
   return __fmul_rn(s, __fmaf_rn(z, __fsub_rn(1.f, s), 1.f));
 }
-__device__ __forceinline__ float softplus(float z) { return __fadd_rn(fmaxf(z, 0.f), log1pf(expf(-fabsf(z)))); }
+__device__ __forceinline__ float softplus(float z) {
+  return __fadd_rn(fmaxf(z, 0.f), __logf(__fadd_rn(1.f, __expf(-fabsf(z)))));
+}
 
 // Arguments of the input-side kernels. Token-by-channel tensors [Bt][L][D].
 template <typename T>
@@ -73,12 +79,15 @@ __device__ __forceinline__ float pre_n(const MixIn<T>& a, int64_t b, int64_t t, 
 
 // Scan inputs in fp32: x = SiLU(conv), dt = softplus(dt_raw + bias), for the
 // clean stream (if x_c) and the noisy stream (if x_n).
+// Grid of the token-by-channel kernels: one CTA row per token (blockIdx.x,
+// batch row b = token / L), 256 channels per CTA (blockIdx.y); no per-element
+// division.
 template <typename T>
 __global__ void __launch_bounds__(256) k_mix_prep(const MixIn<T> a, float* x_c, float* dt_c, float* x_n, float* dt_f,
                                                   float* dt_r) {
-  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (i >= a.Bt * a.L * a.D) return;
-  const int64_t d = i % a.D, bt = i / a.D, t = bt % a.L, b = bt / a.L;
+  const int64_t d = (int64_t)blockIdx.y * 256 + threadIdx.x;
+  if (d >= a.D) return;
+  const int64_t bt = blockIdx.x, b = bt / a.L, t = bt - b * a.L, i = bt * a.D + d;
   if (x_c != nullptr) {
     x_c[i] = silu(pre_c(a, b, t, d));
     dt_c[i] = softplus(__fadd_rn(cvt(a.dtr_c[i]), a.bias_f[d]));
@@ -96,9 +105,9 @@ __global__ void __launch_bounds__(256) k_mix_prep(const MixIn<T> a, float* x_c, 
 template <typename T, typename TO>
 __global__ void __launch_bounds__(256) k_mix_dpre(const MixIn<T> a, float* gx_c, float* gdt_c, float* gx_n,
                                                   float* gdt_f, float* gdt_r, TO* ddtr_c, TO* ddtr_f, TO* ddtr_r) {
-  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (i >= a.Bt * a.L * a.D) return;
-  const int64_t d = i % a.D, bt = i / a.D, t = bt % a.L, b = bt / a.L;
+  const int64_t d = (int64_t)blockIdx.y * 256 + threadIdx.x;
+  if (d >= a.D) return;
+  const int64_t bt = blockIdx.x, b = bt / a.L, t = bt - b * a.L, i = bt * a.D + d;
   gx_c[i] = __fmul_rn(gx_c[i], dsilu(pre_c(a, b, t, d)));
   gx_n[i] = __fmul_rn(gx_n[i], dsilu(pre_n(a, b, t, d)));
   const float vc = __fmul_rn(gdt_c[i], sigm(__fadd_rn(cvt(a.dtr_c[i]), a.bias_f[d])));
@@ -118,9 +127,9 @@ __global__ void __launch_bounds__(256) k_mix_dpre(const MixIn<T> a, float* gx_c,
 template <typename TO>
 __global__ void __launch_bounds__(256) k_mix_dxr(int64_t Bt, int64_t L, int64_t D, int64_t Bs, const float* w,
                                                  const float* gp_c, const float* gp_n, TO* dxr_c, TO* dxr_n) {
-  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (i >= Bt * L * D) return;
-  const int64_t d = i % D, bt = i / D, u = bt % L, b = bt / L;
+  const int64_t d = (int64_t)blockIdx.y * 256 + threadIdx.x;
+  if (d >= D) return;
+  const int64_t bt = blockIdx.x, b = bt / L, u = bt - b * L, i = bt * D + d;
   float ac = 0.f, an = 0.f;
 #pragma unroll
   for (int j = 0; j < kW; ++j) {
@@ -150,8 +159,9 @@ __global__ void __launch_bounds__(128) k_mix_par_part(const MixIn<T> a, const fl
   float s[kW + 3];
 #pragma unroll
   for (int v = 0; v < kW + 3; ++v) s[v] = 0.f;
+  int64_t b = slice / a.L, t = slice - b * a.L;  // batch row and token of `row`, stepped without division
   for (int64_t row = slice; row < a.Bt * a.L; row += kParSplit) {
-    const int64_t b = row / a.L, t = row % a.L, o = row * a.D + d;
+    const int64_t o = row * a.D + d;
     const float pc = gp_c[o], pn = gp_n[o];
     const int64_t k0 = t - t % a.Bs;
 #pragma unroll
@@ -163,6 +173,11 @@ __global__ void __launch_bounds__(128) k_mix_par_part(const MixIn<T> a, const fl
     s[kW] = __fadd_rn(s[kW], __fadd_rn(pc, pn));
     s[kW + 1] = __fadd_rn(s[kW + 1], __fadd_rn(gdt_c[o], gdt_f[o]));
     s[kW + 2] = __fadd_rn(s[kW + 2], gdt_r[o]);
+    t += kParSplit;
+    while (t >= a.L) {
+      t -= a.L;
+      ++b;
+    }
   }
 #pragma unroll
   for (int v = 0; v < kW + 3; ++v) part[((int64_t)slice * (kW + 3) + v) * a.D + d] = s[v];
@@ -297,6 +312,8 @@ int check_mparams(const bdscan_mixer_params* m, const char* fn) {
 }
 
 unsigned blocks_of(int64_t n) { return (unsigned)((n + 255) / 256); }
+// one CTA row per token, 256 channels per CTA
+dim3 rows_grid(const Geo& g) { return dim3((unsigned)(g.Bt * g.L), (unsigned)((g.D + 255) / 256)); }
 
 template <typename T>
 MixIn<T> mix_in(const Geo& g, const bdscan_clean* c, const bdscan_noisy* n, const bdscan_mixer_params* m,
@@ -342,10 +359,10 @@ cudaError_t mix_forward_core(const Geo& g, int N, const bdscan_clean* cl, const 
                              const bdscan_params* pr, const bdscan_mixer_params* mp, float* states, char* ws,
                              const MixWs& w, cudaStream_t s) {
   const MixIn<T> a = mix_in<T>(g, cl, nz, mp, nullptr);
-  const int64_t n = g.Bt * g.L * g.D, nn = g.Bt * g.L * N;
+  const int64_t nn = g.Bt * g.L * N;
   float* X[5];
   for (int i = 0; i < 5; ++i) X[i] = (float*)(ws + w.x[i]);
-  k_mix_prep<T><<<blocks_of(n), 256, 0, s>>>(a, X[0], X[1], X[2], X[3], X[4]);
+  k_mix_prep<T><<<rows_grid(g), 256, 0, s>>>(a, X[0], X[1], X[2], X[3], X[4]);
   cudaError_t e = api_launched(cudaGetLastError(), s);
   const void* bc[6] = {cl->B, cl->C, nz->B_f, nz->C_f, nz->B_r, nz->C_r};
   if (e == cudaSuccess) e = to_f32<T>(bc, w.bc, 6, ws, nn, s);
@@ -456,11 +473,11 @@ cudaError_t mix_backward_t(const Geo& g, int N, const bdscan_clean* cl, const vo
   if (e != cudaSuccess) return e;
   // through SiLU, softplus and the convolution
   const MixIn<T> a = mix_in<T>(g, cl, nz, mp, nullptr);
-  k_mix_dpre<T, TO><<<blocks_of(n), 256, 0, s>>>(a, G[0], G[1], G[2], G[3], G[4], (TO*)gc->ddt, (TO*)gn->ddt_f,
+  k_mix_dpre<T, TO><<<rows_grid(g), 256, 0, s>>>(a, G[0], G[1], G[2], G[3], G[4], (TO*)gc->ddt, (TO*)gn->ddt_f,
                                                  (TO*)gn->ddt_r);
   e = api_launched(cudaGetLastError(), s);
   if (e != cudaSuccess) return e;
-  k_mix_dxr<TO><<<blocks_of(n), 256, 0, s>>>(g.Bt, g.L, g.D, g.Bs, mp->conv_w, G[0], G[2], (TO*)gc->dx, (TO*)gn->dx);
+  k_mix_dxr<TO><<<rows_grid(g), 256, 0, s>>>(g.Bt, g.L, g.D, g.Bs, mp->conv_w, G[0], G[2], (TO*)gc->dx, (TO*)gn->dx);
   e = api_launched(cudaGetLastError(), s);
   if (e != cudaSuccess) return e;
   void* gbc_out[6] = {gc->dB, gc->dC, gn->dB_f, gn->dC_f, gn->dB_r, gn->dC_r};
@@ -487,7 +504,7 @@ cudaError_t mix_boundary_t(const Geo& g, int N, const bdscan_clean* cl, const vo
   const MixWs w = mix_ws(g, N);
   const MixIn<T> a = mix_in<T>(g, cl, nullptr, mp, conv_init);
   const int64_t n = g.Bt * g.L * g.D, nn = g.Bt * g.L * N;
-  k_mix_prep<T><<<blocks_of(n), 256, 0, s>>>(a, (float*)(ws + w.x[0]), (float*)(ws + w.x[1]), nullptr, nullptr,
+  k_mix_prep<T><<<rows_grid(g), 256, 0, s>>>(a, (float*)(ws + w.x[0]), (float*)(ws + w.x[1]), nullptr, nullptr,
                                              nullptr);
   cudaError_t e = api_launched(cudaGetLastError(), s);
   const void* bc[2] = {cl->B, cl->C};
@@ -523,7 +540,7 @@ cudaError_t mix_active_t(const Geo& g, int N, const float* seed, const float* co
   // convolution state
   const MixIn<T> a = mix_in<T>(g, nullptr, nz, mp, conv_seed);
   const int64_t n = g.Bt * g.L * g.D, nn = g.Bt * g.L * N;
-  k_mix_prep<T><<<blocks_of(n), 256, 0, s>>>(a, nullptr, nullptr, (float*)(ws + w.x[2]), (float*)(ws + w.x[3]),
+  k_mix_prep<T><<<rows_grid(g), 256, 0, s>>>(a, nullptr, nullptr, (float*)(ws + w.x[2]), (float*)(ws + w.x[3]),
                                              (float*)(ws + w.x[4]));
   cudaError_t e = api_launched(cudaGetLastError(), s);
   const void* bc[4] = {nz->B_f, nz->C_f, nz->B_r, nz->C_r};
