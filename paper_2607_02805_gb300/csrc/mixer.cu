@@ -22,7 +22,7 @@ namespace bds {
 namespace {
 
 constexpr int kW = 4;           // convolution width
-constexpr int kParSplit = 64;   // token slices of the parameter-gradient reduction
+constexpr int kParSplit = 256;  // token slices of the parameter-gradient reduction
 
 // The logistic function and softplus on the fast hardware paths (__expf,
 // __logf, __fdividef): relative errors of order 1e-6, far inside the
@@ -77,6 +77,81 @@ __device__ __forceinline__ float pre_n(const MixIn<T>& a, int64_t b, int64_t t, 
   return pre;
 }
 
+// Vector access: V = 16 / sizeof(T) consecutive channels per thread (8 for
+// bf16, 4 for fp32; d_inner is a multiple of V), so every token-by-channel
+// load is 16 bytes per thread.
+template <typename T>
+struct Vec {
+  static constexpr int V = 16 / (int)sizeof(T);
+};
+__device__ __forceinline__ void ld16(const bf16* p, float (&v)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 f = __bfloat1622float2(h[e]);
+    v[2 * e] = f.x;
+    v[2 * e + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void ld16(const float* p, float (&v)[4]) {
+  const float4 u = *reinterpret_cast<const float4*>(p);
+  v[0] = u.x;
+  v[1] = u.y;
+  v[2] = u.z;
+  v[3] = u.w;
+}
+template <int V>
+__device__ __forceinline__ void ldf(const float* p, float (&v)[V]) {
+#pragma unroll
+  for (int q = 0; q < V / 4; ++q) {
+    const float4 u = *reinterpret_cast<const float4*>(p + 4 * q);
+    v[4 * q] = u.x;
+    v[4 * q + 1] = u.y;
+    v[4 * q + 2] = u.z;
+    v[4 * q + 3] = u.w;
+  }
+}
+template <int V>
+__device__ __forceinline__ void stv(float* p, const float (&v)[V]) {
+#pragma unroll
+  for (int q = 0; q < V / 4; ++q)
+    *reinterpret_cast<float4*>(p + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+}
+template <int V>
+__device__ __forceinline__ void stv(bf16* p, const float (&v)[V]) {
+#pragma unroll
+  for (int q = 0; q < V / 4; ++q) {
+    const __nv_bfloat162 a = __floats2bfloat162_rn(v[4 * q], v[4 * q + 1]);
+    const __nv_bfloat162 c = __floats2bfloat162_rn(v[4 * q + 2], v[4 * q + 3]);
+    *reinterpret_cast<uint2*>(p + 4 * q) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&a), *reinterpret_cast<const uint32_t*>(&c));
+  }
+}
+
+// Raw inputs of window tap j (position u) for V channels from d: the clean
+// stream, or the initial convolution state before token 0. u is the same for
+// the whole CTA (one token row per CTA), so the branches are uniform.
+template <typename T, int V>
+__device__ __forceinline__ void raw_cv(const MixIn<T>& a, int64_t b, int64_t u, int64_t d, float (&r)[V]) {
+  if (u >= 0) {
+    ld16(a.xr_c + (b * a.L + u) * a.D + d, r);
+  } else if (a.conv_init != nullptr) {
+    ldf<V>(a.conv_init + (b * (kW - 1) + (kW - 1) + u) * a.D + d, r);
+  } else {
+#pragma unroll
+    for (int v = 0; v < V; ++v) r[v] = 0.f;
+  }
+}
+// The same for a noisy token of the block starting at k0: the noisy stream
+// inside the block, the clean one (or the initial state) before it.
+template <typename T, int V>
+__device__ __forceinline__ void raw_nv(const MixIn<T>& a, int64_t b, int64_t u, int64_t k0, int64_t d, float (&r)[V]) {
+  if (u >= k0)
+    ld16(a.xr_n + (b * a.L + u) * a.D + d, r);
+  else
+    raw_cv<T, V>(a, b, u, d, r);
+}
 // Scan inputs in fp32: x = SiLU(conv), dt = softplus(dt_raw + bias), for the
 // clean stream (if x_c) and the noisy stream (if x_n).
 // Grid of the token-by-channel kernels: one CTA row per token (blockIdx.x,
@@ -123,56 +198,84 @@ __global__ void __launch_bounds__(256) k_mix_dpre(const MixIn<T> a, float* gx_c,
 
 // Gradients of the raw inputs from the pre-activation gradients (the
 // convolution's transpose): raw position u feeds tap j of token u + 3 - j; a
-// noisy token's taps before its block feed the clean stream.
-template <typename TO>
+// noisy token's taps before its block feed the clean stream. V channels per
+// thread (V = 16 / sizeof(TI), TI the input type).
+template <typename TO, int V>
 __global__ void __launch_bounds__(256) k_mix_dxr(int64_t Bt, int64_t L, int64_t D, int64_t Bs, const float* w,
                                                  const float* gp_c, const float* gp_n, TO* dxr_c, TO* dxr_n) {
-  const int64_t d = (int64_t)blockIdx.y * 256 + threadIdx.x;
+  const int64_t d = ((int64_t)blockIdx.y * 256 + threadIdx.x) * V;
   if (d >= D) return;
   const int64_t bt = blockIdx.x, b = bt / L, u = bt - b * L, i = bt * D + d;
-  float ac = 0.f, an = 0.f;
+  float wv[kW * V], ac[V], an[V];
+  ldf<kW * V>(w + d * kW, wv);
+#pragma unroll
+  for (int v = 0; v < V; ++v) ac[v] = an[v] = 0.f;
 #pragma unroll
   for (int j = 0; j < kW; ++j) {
     const int64_t t = u + (kW - 1) - j;
     if (t >= L) continue;
-    const float wj = w[d * kW + j];
     const int64_t o = (b * L + t) * D + d;
-    ac = __fmaf_rn(wj, gp_c[o], ac);
-    if (u >= t - t % Bs)
-      an = __fmaf_rn(wj, gp_n[o], an);
-    else
-      ac = __fmaf_rn(wj, gp_n[o], ac);
+    float pc[V], pn[V];
+    ldf<V>(gp_c + o, pc);
+    ldf<V>(gp_n + o, pn);
+    const bool inside = u >= t - t % Bs;  // the same block as the consuming noisy token
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      const float wj = wv[v * kW + j];
+      ac[v] = __fmaf_rn(wj, pc[v], ac[v]);
+      if (inside)
+        an[v] = __fmaf_rn(wj, pn[v], an[v]);
+      else
+        ac[v] = __fmaf_rn(wj, pn[v], ac[v]);
+    }
   }
-  dxr_c[i] = to_out<TO>(ac);
-  dxr_n[i] = to_out<TO>(an);
+  stv<V>(dxr_c + i, ac);
+  stv<V>(dxr_n + i, an);
 }
 
 // Partial sums of the parameter gradients over a slice of the token rows:
-// part[slice][v][d] for v = tap 0..3, conv bias, dt_bias_f, dt_bias_r.
+// part[slice][v][d] for v = tap 0..3, conv bias, dt_bias_f, dt_bias_r; V
+// channels per thread.
 template <typename T>
 __global__ void __launch_bounds__(128) k_mix_par_part(const MixIn<T> a, const float* gp_c, const float* gp_n,
                                                       const float* gdt_c, const float* gdt_f, const float* gdt_r,
                                                       float* part) {
-  const int64_t d = (int64_t)blockIdx.x * 128 + threadIdx.x;
+  constexpr int V = Vec<T>::V;
+  const int64_t d = ((int64_t)blockIdx.x * 128 + threadIdx.x) * V;
   const int slice = blockIdx.y;
   if (d >= a.D) return;
-  float s[kW + 3];
+  float s[kW + 3][V];
 #pragma unroll
-  for (int v = 0; v < kW + 3; ++v) s[v] = 0.f;
+  for (int q = 0; q < kW + 3; ++q)
+#pragma unroll
+    for (int v = 0; v < V; ++v) s[q][v] = 0.f;
   int64_t b = slice / a.L, t = slice - b * a.L;  // batch row and token of `row`, stepped without division
   for (int64_t row = slice; row < a.Bt * a.L; row += kParSplit) {
-    const int64_t o = row * a.D + d;
-    const float pc = gp_c[o], pn = gp_n[o];
-    const int64_t k0 = t - t % a.Bs;
+    const int64_t o = row * a.D + d, k0 = t - t % a.Bs;
+    float pc[V], pn[V], g1[V], g2[V], g3[V];
+    ldf<V>(gp_c + o, pc);
+    ldf<V>(gp_n + o, pn);
+    ldf<V>(gdt_c + o, g1);
+    ldf<V>(gdt_f + o, g2);
+    ldf<V>(gdt_r + o, g3);
 #pragma unroll
     for (int j = 0; j < kW; ++j) {
       const int64_t u = t - (kW - 1) + j;
-      s[j] = __fmaf_rn(pc, raw_c(a, b, u, d), s[j]);
-      s[j] = __fmaf_rn(pn, raw_n(a, b, u, k0, d), s[j]);
+      float rc[V], rn[V];
+      raw_cv<T, V>(a, b, u, d, rc);
+      raw_nv<T, V>(a, b, u, k0, d, rn);
+#pragma unroll
+      for (int v = 0; v < V; ++v) {
+        s[j][v] = __fmaf_rn(pc[v], rc[v], s[j][v]);
+        s[j][v] = __fmaf_rn(pn[v], rn[v], s[j][v]);
+      }
     }
-    s[kW] = __fadd_rn(s[kW], __fadd_rn(pc, pn));
-    s[kW + 1] = __fadd_rn(s[kW + 1], __fadd_rn(gdt_c[o], gdt_f[o]));
-    s[kW + 2] = __fadd_rn(s[kW + 2], gdt_r[o]);
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      s[kW][v] = __fadd_rn(s[kW][v], __fadd_rn(pc[v], pn[v]));
+      s[kW + 1][v] = __fadd_rn(s[kW + 1][v], __fadd_rn(g1[v], g2[v]));
+      s[kW + 2][v] = __fadd_rn(s[kW + 2][v], g3[v]);
+    }
     t += kParSplit;
     while (t >= a.L) {
       t -= a.L;
@@ -180,7 +283,7 @@ __global__ void __launch_bounds__(128) k_mix_par_part(const MixIn<T> a, const fl
     }
   }
 #pragma unroll
-  for (int v = 0; v < kW + 3; ++v) part[((int64_t)slice * (kW + 3) + v) * a.D + d] = s[v];
+  for (int q = 0; q < kW + 3; ++q) stv<V>(part + ((int64_t)slice * (kW + 3) + q) * a.D + d, s[q]);
 }
 
 // The slices summed in order: dconv_w [D][4], dconv_b, ddt_bias_f, ddt_bias_r [D].
@@ -202,24 +305,44 @@ __global__ void __launch_bounds__(256) k_mix_par_red(int64_t D, const float* par
     dbr[d] = s;
 }
 
-// out = y * SiLU(z).
+// out = y * SiLU(z), V elements per thread.
 template <typename T, typename TO>
 __global__ void __launch_bounds__(256) k_mix_gate(int64_t n, const float* y, const T* z, TO* out) {
-  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  constexpr int V = Vec<T>::V;
+  const int64_t i = ((int64_t)blockIdx.x * 256 + threadIdx.x) * V;
   if (i >= n) return;
-  out[i] = to_out<TO>(__fmul_rn(y[i], silu(cvt(z[i]))));
+  float yv[V], zv[V];
+  ldf<V>(y + i, yv);
+  ld16(z + i, zv);
+#pragma unroll
+  for (int v = 0; v < V; ++v) yv[v] = __fmul_rn(yv[v], silu(zv[v]));
+  stv<V>(out + i, yv);
 }
 
 // The gate's backward: dy = dout * SiLU(z), dz = dout * y * SiLU'(z) (zero
-// without dout).
+// without dout), V elements per thread.
 template <typename T, typename TO>
 __global__ void __launch_bounds__(256) k_mix_gate_bwd(int64_t n, const float* y, const T* z, const T* dout, float* dy,
                                                       TO* dz) {
-  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  constexpr int V = Vec<T>::V;
+  const int64_t i = ((int64_t)blockIdx.x * 256 + threadIdx.x) * V;
   if (i >= n) return;
-  const float g = dout != nullptr ? cvt(dout[i]) : 0.f, zz = cvt(z[i]);
-  dy[i] = __fmul_rn(g, silu(zz));
-  dz[i] = to_out<TO>(__fmul_rn(__fmul_rn(g, y[i]), dsilu(zz)));
+  float yv[V], zv[V], gv[V], a[V], c[V];
+  ldf<V>(y + i, yv);
+  ld16(z + i, zv);
+  if (dout != nullptr) {
+    ld16(dout + i, gv);
+  } else {
+#pragma unroll
+    for (int v = 0; v < V; ++v) gv[v] = 0.f;
+  }
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    a[v] = __fmul_rn(gv[v], silu(zv[v]));
+    c[v] = __fmul_rn(__fmul_rn(gv[v], yv[v]), dsilu(zv[v]));
+  }
+  stv<V>(dy + i, a);
+  stv<V>(dz + i, c);
 }
 
 // Element type conversion (B, C to fp32 for the scan; their gradients back).
@@ -312,8 +435,16 @@ int check_mparams(const bdscan_mixer_params* m, const char* fn) {
 }
 
 unsigned blocks_of(int64_t n) { return (unsigned)((n + 255) / 256); }
-// one CTA row per token, 256 channels per CTA
-dim3 rows_grid(const Geo& g) { return dim3((unsigned)(g.Bt * g.L), (unsigned)((g.D + 255) / 256)); }
+// one CTA row per token, 256 threads of V channels per CTA
+dim3 rows_grid(const Geo& g, int V) {
+  const int64_t span = 256 * (int64_t)V;
+  return dim3((unsigned)(g.Bt * g.L), (unsigned)((g.D + span - 1) / span));
+}
+template <typename T>
+unsigned vec_blocks(int64_t n) {
+  constexpr int64_t span = 256 * Vec<T>::V;
+  return (unsigned)((n + span - 1) / span);
+}
 
 template <typename T>
 MixIn<T> mix_in(const Geo& g, const bdscan_clean* c, const bdscan_noisy* n, const bdscan_mixer_params* m,
@@ -362,7 +493,7 @@ cudaError_t mix_forward_core(const Geo& g, int N, const bdscan_clean* cl, const 
   const int64_t nn = g.Bt * g.L * N;
   float* X[5];
   for (int i = 0; i < 5; ++i) X[i] = (float*)(ws + w.x[i]);
-  k_mix_prep<T><<<rows_grid(g), 256, 0, s>>>(a, X[0], X[1], X[2], X[3], X[4]);
+  k_mix_prep<T><<<rows_grid(g, 1), 256, 0, s>>>(a, X[0], X[1], X[2], X[3], X[4]);
   cudaError_t e = api_launched(cudaGetLastError(), s);
   const void* bc[6] = {cl->B, cl->C, nz->B_f, nz->C_f, nz->B_r, nz->C_r};
   if (e == cudaSuccess) e = to_f32<T>(bc, w.bc, 6, ws, nn, s);
@@ -393,7 +524,7 @@ cudaError_t mix_forward_core(const Geo& g, int N, const bdscan_clean* cl, const 
 
 template <typename T, typename TO>
 cudaError_t gate(int64_t n, const char* ws, size_t yslot, const void* z, void* out, cudaStream_t s) {
-  k_mix_gate<T, TO><<<blocks_of(n), 256, 0, s>>>(n, (const float*)(ws + yslot), (const T*)z, (TO*)out);
+  k_mix_gate<T, TO><<<vec_blocks<T>(n), 256, 0, s>>>(n, (const float*)(ws + yslot), (const T*)z, (TO*)out);
   return api_launched(cudaGetLastError(), s);
 }
 
@@ -422,11 +553,11 @@ cudaError_t mix_backward_t(const Geo& g, int N, const bdscan_clean* cl, const vo
   if (e != cudaSuccess) return e;
   const int64_t n = g.Bt * g.L * g.D, nn = g.Bt * g.L * N;
   float* dy[2] = {(float*)(ws + w.dy[0]), (float*)(ws + w.dy[1])};
-  k_mix_gate_bwd<T, TO><<<blocks_of(n), 256, 0, s>>>(n, (const float*)(ws + w.y[0]), (const T*)z_c, (const T*)dout_c,
+  k_mix_gate_bwd<T, TO><<<vec_blocks<T>(n), 256, 0, s>>>(n, (const float*)(ws + w.y[0]), (const T*)z_c, (const T*)dout_c,
                                                      dy[0], (TO*)dz_c);
   e = api_launched(cudaGetLastError(), s);
   if (e != cudaSuccess) return e;
-  k_mix_gate_bwd<T, TO><<<blocks_of(n), 256, 0, s>>>(n, (const float*)(ws + w.y[1]), (const T*)z_n, (const T*)dout_n,
+  k_mix_gate_bwd<T, TO><<<vec_blocks<T>(n), 256, 0, s>>>(n, (const float*)(ws + w.y[1]), (const T*)z_n, (const T*)dout_n,
                                                      dy[1], (TO*)dz_n);
   e = api_launched(cudaGetLastError(), s);
   if (e != cudaSuccess) return e;
@@ -473,11 +604,11 @@ cudaError_t mix_backward_t(const Geo& g, int N, const bdscan_clean* cl, const vo
   if (e != cudaSuccess) return e;
   // through SiLU, softplus and the convolution
   const MixIn<T> a = mix_in<T>(g, cl, nz, mp, nullptr);
-  k_mix_dpre<T, TO><<<rows_grid(g), 256, 0, s>>>(a, G[0], G[1], G[2], G[3], G[4], (TO*)gc->ddt, (TO*)gn->ddt_f,
+  k_mix_dpre<T, TO><<<rows_grid(g, 1), 256, 0, s>>>(a, G[0], G[1], G[2], G[3], G[4], (TO*)gc->ddt, (TO*)gn->ddt_f,
                                                  (TO*)gn->ddt_r);
   e = api_launched(cudaGetLastError(), s);
   if (e != cudaSuccess) return e;
-  k_mix_dxr<TO><<<rows_grid(g), 256, 0, s>>>(g.Bt, g.L, g.D, g.Bs, mp->conv_w, G[0], G[2], (TO*)gc->dx, (TO*)gn->dx);
+  k_mix_dxr<TO, Vec<T>::V><<<rows_grid(g, Vec<T>::V), 256, 0, s>>>(g.Bt, g.L, g.D, g.Bs, mp->conv_w, G[0], G[2], (TO*)gc->dx, (TO*)gn->dx);
   e = api_launched(cudaGetLastError(), s);
   if (e != cudaSuccess) return e;
   void* gbc_out[6] = {gc->dB, gc->dC, gn->dB_f, gn->dC_f, gn->dB_r, gn->dC_r};
@@ -487,7 +618,7 @@ cudaError_t mix_backward_t(const Geo& g, int N, const bdscan_clean* cl, const vo
   }
   if (e != cudaSuccess) return e;
   float* part = (float*)(ws + w.part);
-  k_mix_par_part<T><<<dim3((unsigned)((g.D + 127) / 128), kParSplit), 128, 0, s>>>(a, G[0], G[2], G[1], G[3], G[4],
+  k_mix_par_part<T><<<dim3((unsigned)((g.D + 128 * Vec<T>::V - 1) / (128 * Vec<T>::V)), kParSplit), 128, 0, s>>>(a, G[0], G[2], G[1], G[3], G[4],
                                                                                   part);
   e = api_launched(cudaGetLastError(), s);
   if (e != cudaSuccess) return e;
@@ -504,7 +635,7 @@ cudaError_t mix_boundary_t(const Geo& g, int N, const bdscan_clean* cl, const vo
   const MixWs w = mix_ws(g, N);
   const MixIn<T> a = mix_in<T>(g, cl, nullptr, mp, conv_init);
   const int64_t n = g.Bt * g.L * g.D, nn = g.Bt * g.L * N;
-  k_mix_prep<T><<<rows_grid(g), 256, 0, s>>>(a, (float*)(ws + w.x[0]), (float*)(ws + w.x[1]), nullptr, nullptr,
+  k_mix_prep<T><<<rows_grid(g, 1), 256, 0, s>>>(a, (float*)(ws + w.x[0]), (float*)(ws + w.x[1]), nullptr, nullptr,
                                              nullptr);
   cudaError_t e = api_launched(cudaGetLastError(), s);
   const void* bc[2] = {cl->B, cl->C};
@@ -540,7 +671,7 @@ cudaError_t mix_active_t(const Geo& g, int N, const float* seed, const float* co
   // convolution state
   const MixIn<T> a = mix_in<T>(g, nullptr, nz, mp, conv_seed);
   const int64_t n = g.Bt * g.L * g.D, nn = g.Bt * g.L * N;
-  k_mix_prep<T><<<rows_grid(g), 256, 0, s>>>(a, nullptr, nullptr, (float*)(ws + w.x[2]), (float*)(ws + w.x[3]),
+  k_mix_prep<T><<<rows_grid(g, 1), 256, 0, s>>>(a, nullptr, nullptr, (float*)(ws + w.x[2]), (float*)(ws + w.x[3]),
                                              (float*)(ws + w.x[4]));
   cudaError_t e = api_launched(cudaGetLastError(), s);
   const void* bc[4] = {nz->B_f, nz->C_f, nz->B_r, nz->C_r};
