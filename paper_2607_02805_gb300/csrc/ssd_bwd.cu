@@ -112,6 +112,7 @@ __device__ __forceinline__ void tmem_st32(uint32_t ta, const float (&v)[32]) {
 //   VEC  c and dt of the block for every head of the group, [2][16][256] fp32
 //   CP   column-sum partials of four row quarters, [4][64] fp32
 //   ROWS row sums per head of the group [16][128], row dots per column half [2][16][128]
+//   CF   the current head's column factors exp(A (c_ref - c_s)) and their products with dt_s
 // After a s-tile's heads, the head-summed dG goes to M (bf16 high part) and
 // X + DY (low part). The seed phase uses DY, BT for E o dy, M for the seed's
 // bf16 high and low parts.
@@ -120,7 +121,8 @@ struct TileSmem {
   static constexpr uint32_t VEC = COL + 128u * 65u * 4u;
   static constexpr uint32_t CP = VEC + 2u * 16u * 256u * 4u;
   static constexpr uint32_t ROWS = CP + 4u * 64u * 4u;
-  static constexpr uint32_t total = ROWS + 3u * 16u * 128u * 4u + 1024u;
+  static constexpr uint32_t CF = ROWS + 3u * 16u * 128u * 4u;  // one head's column factors, and times dt [2][256]
+  static constexpr uint32_t total = CF + 2u * 256u * 4u + 1024u;
 };
 constexpr int kMaxBwdHeads = 16;  // heads per tile CTA
 
@@ -163,6 +165,8 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
   float* s_dtv = s_cv + kMaxBwdHeads * 256;              // [hh][256]: dt
   float* s_col = reinterpret_cast<float*>(sm + S::COL);
   float* s_cp = reinterpret_cast<float*>(sm + S::CP);
+  float* s_cf = reinterpret_cast<float*>(sm + S::CF);  // [256]
+  float* s_cfd = s_cf + 256;                           // [256]
   float* s_rows = reinterpret_cast<float*>(sm + S::ROWS);                              // [hh][128]
   float* s_dots = s_rows + kMaxBwdHeads * 128 + half * kMaxBwdHeads * 128;             // [hh][128] of this half
 
@@ -231,6 +235,16 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     if (!(alive = wait_mma())) break;
     for (int hh = 0; hh < hg; ++hh) {
       const int h = h0 + hh;
+      // column factors of this head: exp(A (c_ref - c_s)), with c_ref the
+      // cumulative dt at the last (forward) or first (reverse) token of s's
+      // 32-token group, and their products with dt_s (the previous head's
+      // element-wise phase is past the barrier before its dx products)
+      if (tid < Bs) {
+        const float* c = s_cv + hh * 256;
+        const float cf = ex2(__fmul_rn(__fmul_rn(p.A[h], kLog2e), __fsub_rn(c[UPPER ? (tid & ~31) : (tid | 31)], c[tid])));
+        s_cf[tid] = cf;
+        s_cfd[tid] = __fmul_rn(cf, s_dtv[hh * 256 + tid]);
+      }
       cp_async_wait_all();
       umma::fence_async_smem();
       umma::fence_before_sync();
@@ -258,24 +272,64 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
         umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)c, qv);
         if (hh > 0) umma::tmem_ld32(lane_base + 256u + 32u * (uint32_t)c, dgs);
         uint32_t mp[16];
+        // the chunk's 32 columns against this warp's 32 rows: entirely inside
+        // the direction's triangle (the decay factors into a row factor times
+        // the column factors, both at most 1), the diagonal 32 x 32 block
+        // (one ex2 per element, masked), or entirely outside (zero)
+        const int rq = w & 3;  // the warp's row group in the tile
+        const int mode = UPPER ? (j > i || c > rq ? 1 : (c == rq ? 2 : 0)) : (j < i || c < rq ? 1 : (c == rq ? 2 : 0));
+        const int s0 = j * kSsdT + 32 * c;
+        if (mode == 1) {
+          const float rf = ex2(__fmul_rn(A2, __fsub_rn(ct, s_c[UPPER ? s0 : s0 + 31])));
+          const float2 rf2 = f2(rf);
+          float2 rs2 = f2(0.f);
 #pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          float mv[2];
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            const int s = j * kSsdT + 32 * c + e + q;
-            const bool valid = UPPER ? (s >= tt) : (s <= tt);
-            const float L = valid ? ex2(__fmul_rn(A2, __fsub_rn(ct, s_c[s]))) : 0.f;
-            const float ds = s_dt[s];
-            const float gl = __fmul_rn(gv[e + q], L);
-            const float rp = __fmul_rn(qv[e + q], gl);
-            rowsum = __fmaf_rn(rp, ds, rowsum);
-            s_col[t * 65 + 32 * half + e + q] = rp;
-            const float dg = __fmul_rn(__fmul_rn(qv[e + q], L), ds);
-            dgs[e + q] = hh > 0 ? __fadd_rn(dgs[e + q], dg) : dg;
-            mv[q] = __fmul_rn(gl, ds);
+          for (int e = 0; e < 32; e += 2) {
+            const float2 cf = *reinterpret_cast<const float2*>(s_cf + s0 + e);
+            const float2 cfd = *reinterpret_cast<const float2*>(s_cfd + s0 + e);
+            const float2 g2 = make_float2(gv[e], gv[e + 1]), q2 = make_float2(qv[e], qv[e + 1]);
+            const float2 L = mul2(rf2, cf), Ld = mul2(rf2, cfd);
+            const float2 rp = mul2(q2, mul2(g2, L));
+            s_col[t * 65 + 32 * half + e] = rp.x;  // row stride 65: scalar stores
+            s_col[t * 65 + 32 * half + e + 1] = rp.y;
+            const float2 dg = mul2(q2, Ld);
+            rs2 = fma2(g2, dg, rs2);
+            const float2 old2 = make_float2(dgs[e], dgs[e + 1]);
+            const float2 nd = hh > 0 ? add2(old2, dg) : dg;
+            dgs[e] = nd.x;
+            dgs[e + 1] = nd.y;
+            const float2 mv = mul2(g2, Ld);
+            mp[e >> 1] = pack_bf16(mv.x, mv.y);
           }
-          mp[e >> 1] = pack_bf16(mv[0], mv[1]);
+          rowsum = __fadd_rn(rowsum, __fadd_rn(rs2.x, rs2.y));
+        } else if (mode == 2) {
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            float mv[2];
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const int s = s0 + e + q;
+              const bool valid = UPPER ? (s >= tt) : (s <= tt);
+              const float L = valid ? ex2(__fmul_rn(A2, __fsub_rn(ct, s_c[s]))) : 0.f;
+              const float ds = s_dt[s];
+              const float gl = __fmul_rn(gv[e + q], L);
+              const float rp = __fmul_rn(qv[e + q], gl);
+              rowsum = __fmaf_rn(rp, ds, rowsum);
+              s_col[t * 65 + 32 * half + e + q] = rp;
+              const float dg = __fmul_rn(__fmul_rn(qv[e + q], L), ds);
+              dgs[e + q] = hh > 0 ? __fadd_rn(dgs[e + q], dg) : dg;
+              mv[q] = __fmul_rn(gl, ds);
+            }
+            mp[e >> 1] = pack_bf16(mv[0], mv[1]);
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            s_col[t * 65 + 32 * half + e] = 0.f;
+            s_col[t * 65 + 32 * half + e + 1] = 0.f;
+            if (hh == 0) dgs[e] = dgs[e + 1] = 0.f;
+            mp[e >> 1] = 0u;
+          }
         }
         tmem_st32(lane_base + 256u + 32u * (uint32_t)c, dgs);
 #pragma unroll
