@@ -52,7 +52,15 @@
  *   - Return codes: BDSCAN_OK, or a negative code; bdscan_last_error()
  *     then returns a message for the calling thread. No C++ exception
  *     crosses this interface.
- *   - Supported: d_state N in {8, 16}; dtype/out_dtype pairs (f32,f32),
+ *   - Supported: d_state N in {8, 16} for every entry point, and any
+ *     multiple of 4 up to 64 for bdscan_forward, bdscan_backward,
+ *     bdscan_boundary_states and bdscan_active_block: those run the scan
+ *     once per group of 16 states (the last group 8 or 16, zero-padded; the
+ *     state index is separable in the recurrence, only y, dx and dt sum over
+ *     it) and add the groups' fp32 outputs in group order. Their workspaces
+ *     grow accordingly; the grouped bdscan_active_block uses a static 16 MiB
+ *     device scratch (calls that overlap in time on one device race on it).
+ *     dtype/out_dtype pairs (f32,f32),
  *     (bf16,bf16), (bf16,f32); d_inner a multiple of 8 (bf16 inputs) or 4
  *     (f32 inputs); len a multiple of block; block <= 64 for forward-only
  *     calls and block <= 16, or a multiple of 16 up to 64, for the backward.

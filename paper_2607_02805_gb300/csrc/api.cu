@@ -113,8 +113,12 @@ struct Call {
   size_t in_elt;
 };
 
-// Validates the dimensions common to every entry point.
-int check_dims(const bdscan_dims* dm, Call* c, const char* fn) {
+// d_state of the kernels themselves; other sizes run in state groups
+bool direct_N(int N) { return N == 8 || N == 16; }
+
+// Validates the dimensions common to every entry point; d_state is any
+// multiple of 4 up to 64 (state groups above, see check_dims).
+int check_dims_any(const bdscan_dims* dm, Call* c, const char* fn) {
   g_launches = 0;
   if (dm == nullptr) return fail(BDSCAN_ERR_ARG, "%s: dims is NULL", fn);
   if (dm->batch < 0 || dm->len < 0) return fail(BDSCAN_ERR_ARG, "%s: negative batch or len", fn);
@@ -128,8 +132,9 @@ int check_dims(const bdscan_dims* dm, Call* c, const char* fn) {
     return fail(BDSCAN_ERR_ARG, "%s: bad out_dtype %d", fn, dm->out_dtype);
   if (dm->dtype == BDSCAN_F32 && dm->out_dtype == BDSCAN_BF16)
     return fail(BDSCAN_ERR_UNSUPPORTED, "%s: f32 inputs with bf16 outputs are not supported", fn);
-  if (dm->d_state != 8 && dm->d_state != 16)
-    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: d_state %lld not supported (8 or 16)", fn, (long long)dm->d_state);
+  if (dm->d_state > 64 || dm->d_state % 4 != 0)
+    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: d_state %lld not supported (a multiple of 4 up to 64)", fn,
+                (long long)dm->d_state);
   const int64_t vec = dm->dtype == BDSCAN_BF16 ? 8 : 4;
   if (dm->d_inner % vec != 0)
     return fail(BDSCAN_ERR_UNSUPPORTED, "%s: d_inner %lld must be a multiple of %lld for this dtype", fn,
@@ -152,6 +157,14 @@ int check_dims(const bdscan_dims* dm, Call* c, const char* fn) {
   c->dt = dm->dtype == BDSCAN_F32 ? 0 : (dm->out_dtype == BDSCAN_BF16 ? 1 : 2);
   c->N = (int)dm->d_state;
   c->in_elt = dm->dtype == BDSCAN_F32 ? 4 : 2;
+  return BDSCAN_OK;
+}
+
+// The same for entry points without state groups: d_state 8 or 16.
+int check_dims(const bdscan_dims* dm, Call* c, const char* fn) {
+  const int rc = check_dims_any(dm, c, fn);
+  if (rc != BDSCAN_OK) return rc;
+  if (!direct_N(c->N)) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: d_state %d not supported here (8 or 16)", fn, c->N);
   return BDSCAN_OK;
 }
 
@@ -256,6 +269,332 @@ int run_chunk_states(const Call& c, bds::FwdParams& p, cudaStream_t s, const cha
   return BDSCAN_OK;
 }
 
+
+// ---------------------------------------------------------------------------
+// State groups: d_state other than 8 or 16 (a multiple of 4 up to 64). The
+// scan kernels run once per group of 16 states (the last one 8 or 16,
+// zero-padded: zero B, C and A add nothing), on gathered copies of the
+// group's B, C, A and states, with fp32 outputs that are added in group
+// order; the D terms come from group 0 only (the others get D = 0).
+// ---------------------------------------------------------------------------
+struct GroupPlan {
+  int G;
+  int n0[4], gs[4];
+};
+GroupPlan group_plan(int N) {
+  GroupPlan q;
+  q.G = (N + 15) / 16;
+  for (int g = 0; g < q.G; ++g) {
+    q.n0[g] = 16 * g;
+    const int rem = N - 16 * g;
+    q.gs[g] = rem >= 16 ? 16 : (rem <= 8 ? 8 : 16);
+  }
+  return q;
+}
+
+struct Carve {
+  size_t o = 0;
+  size_t take(size_t bytes) {
+    const size_t at = o;
+    o += al256(bytes);
+    return at;
+  }
+};
+
+// the per-group calls write fp32 outputs: dt code 0 (f32 inputs) or 2 (bf16
+// inputs, f32 outputs); the caller's outputs have element size out_elt
+int group_dt(const Call& c) { return c.dt == 0 ? 0 : 2; }
+int out_elt(const Call& c) { return c.dt == 1 ? 2 : 4; }
+
+struct FwdGroupWs {
+  size_t scan, bc[6], a[2], dzero, st, acc[2], tmp[2], total;
+};
+FwdGroupWs fwd_group_ws(const Call& c) {
+  const bds::Geo& g = c.g;
+  FwdGroupWs w;
+  Carve k;
+  w.scan = k.take(fwd_ws(g, 16));
+  for (int i = 0; i < 6; ++i) w.bc[i] = k.take((size_t)g.Bt * g.L * 16 * c.in_elt);
+  for (int i = 0; i < 2; ++i) w.a[i] = k.take((size_t)g.D * 16 * 4);
+  w.dzero = k.take((size_t)g.D * 4);
+  w.st = k.take((size_t)g.Bt * g.nb * g.D * 16 * 4);
+  for (int i = 0; i < 2; ++i) w.acc[i] = k.take((size_t)g.Bt * g.L * g.D * 4);
+  for (int i = 0; i < 2; ++i) w.tmp[i] = k.take((size_t)g.Bt * g.L * g.D * 4);
+  w.total = k.o;
+  return w;
+}
+
+struct BndGroupWs {
+  size_t scan, bc[2], a, dzero, st, init, acc, tmp, total;
+};
+BndGroupWs bnd_group_ws(const Call& c, int emit_all) {
+  const bds::Geo& g = c.g;
+  BndGroupWs w;
+  Carve k;
+  w.scan = k.take(fwd_ws(g, 16));
+  for (int i = 0; i < 2; ++i) w.bc[i] = k.take((size_t)g.Bt * g.L * 16 * c.in_elt);
+  w.a = k.take((size_t)g.D * 16 * 4);
+  w.dzero = k.take((size_t)g.D * 4);
+  w.st = k.take((size_t)g.Bt * (emit_all ? g.nb : 1) * g.D * 16 * 4);
+  w.init = k.take((size_t)g.Bt * g.D * 16 * 4);
+  w.acc = k.take((size_t)g.Bt * g.L * g.D * 4);
+  w.tmp = k.take((size_t)g.Bt * g.L * g.D * 4);
+  w.total = k.o;
+  return w;
+}
+
+struct BwdGroupWs {
+  size_t scan, bc[6], a[2], dzero, st, dst, acc[5], tmp[5], gbc[6], ga[2], gd[2], total;
+};
+BwdGroupWs bwd_group_ws(const Call& c) {
+  const bds::Geo& g = c.g;
+  bds::Geo gmax = g;
+  gmax.nc = bds::bwd_max_chunks(g);
+  BwdGroupWs w;
+  Carve k;
+  w.scan = k.take(bwd_ws(gmax, 16).total);
+  for (int i = 0; i < 6; ++i) w.bc[i] = k.take((size_t)g.Bt * g.L * 16 * c.in_elt);
+  for (int i = 0; i < 2; ++i) w.a[i] = k.take((size_t)g.D * 16 * 4);
+  w.dzero = k.take((size_t)g.D * 4);
+  w.st = k.take((size_t)g.Bt * g.nb * g.D * 16 * 4);
+  w.dst = k.take((size_t)g.Bt * g.nb * g.D * 16 * 4);
+  for (int i = 0; i < 5; ++i) w.acc[i] = k.take((size_t)g.Bt * g.L * g.D * 4);
+  for (int i = 0; i < 5; ++i) w.tmp[i] = k.take((size_t)g.Bt * g.L * g.D * 4);
+  for (int i = 0; i < 6; ++i) w.gbc[i] = k.take((size_t)g.Bt * g.L * 16 * 4);
+  for (int i = 0; i < 2; ++i) w.ga[i] = k.take((size_t)g.D * 16 * 4);
+  for (int i = 0; i < 2; ++i) w.gd[i] = k.take((size_t)g.D * 4);
+  w.total = k.o;
+  return w;
+}
+
+struct ActGroupWs {
+  size_t bc[4], a[2], dzero, seed, acc, tmp, total;
+};
+ActGroupWs act_group_ws(const Call& c) {
+  const bds::Geo& g = c.g;
+  ActGroupWs w;
+  Carve k;
+  for (int i = 0; i < 4; ++i) w.bc[i] = k.take((size_t)g.Bt * g.L * 16 * c.in_elt);
+  for (int i = 0; i < 2; ++i) w.a[i] = k.take((size_t)g.D * 16 * 4);
+  w.dzero = k.take((size_t)g.D * 4);
+  w.seed = k.take((size_t)g.Bt * g.D * 16 * 4);
+  w.acc = k.take((size_t)g.Bt * g.L * g.D * 4);
+  w.tmp = k.take((size_t)g.Bt * g.L * g.D * 4);
+  w.total = k.o;
+  return w;
+}
+
+// gathers of one group (B/C rows of the tokens, A rows of the channels)
+cudaError_t gather(const void* src, int elt, int64_t rows, int N, int n0, int gs, char* dst, cudaStream_t s) {
+  return launched(bds::launch_group_gather(src, elt, rows, N, n0, gs, dst, s), s);
+}
+
+int grouped_forward(const Call& c, const bdscan_clean* clean, const bdscan_noisy* noisy, const bdscan_params* pr,
+                    void* y_c, void* y_n, float* states, char* ws, cudaStream_t s, const char* fn) {
+  const bds::Geo& g = c.g;
+  const FwdGroupWs w = fwd_group_ws(c);
+  const GroupPlan q = group_plan(c.N);
+  const int64_t tok = g.Bt * g.L, n = g.Bt * g.L * g.D;
+  cudaError_t e = cudaMemsetAsync(ws + w.dzero, 0, (size_t)g.D * 4, s);
+  const void* bc[6] = {clean->B, clean->C, noisy->B_f, noisy->C_f, noisy->B_r, noisy->C_r};
+  for (int gi = 0; gi < q.G && e == cudaSuccess; ++gi) {
+    const int n0 = q.n0[gi], gs = q.gs[gi];
+    for (int i = 0; i < 6 && e == cudaSuccess; ++i) e = gather(bc[i], (int)c.in_elt, tok, c.N, n0, gs, ws + w.bc[i], s);
+    if (e == cudaSuccess) e = gather(pr->A_f, 4, g.D, c.N, n0, gs, ws + w.a[0], s);
+    if (e == cudaSuccess) e = gather(pr->A_r, 4, g.D, c.N, n0, gs, ws + w.a[1], s);
+    if (e != cudaSuccess) break;
+    bds::FwdParams p;
+    memset(&p, 0, sizeof(p));
+    p.g = g;
+    p.xc = clean->x;
+    p.dtc = clean->dt;
+    p.Bc = ws + w.bc[0];
+    p.Cc = ws + w.bc[1];
+    p.xn = noisy->x;
+    p.dtf = noisy->dt_f;
+    p.Bf = ws + w.bc[2];
+    p.Cf = ws + w.bc[3];
+    p.dtr = noisy->dt_r;
+    p.Br = ws + w.bc[4];
+    p.Cr = ws + w.bc[5];
+    p.Af = (const float*)(ws + w.a[0]);
+    p.Ar = (const float*)(ws + w.a[1]);
+    p.Df = gi == 0 ? pr->D_f : (const float*)(ws + w.dzero);
+    p.Dr = gi == 0 ? pr->D_r : (const float*)(ws + w.dzero);
+    p.yc = ws + (gi == 0 ? w.acc[0] : w.tmp[0]);
+    p.yn = ws + (gi == 0 ? w.acc[1] : w.tmp[1]);
+    p.states = (float*)(ws + w.st);
+    e = bds::api_run_forward(group_dt(c), gs, p, ws + w.scan, s);
+    for (int i = 0; i < 2 && gi > 0 && e == cudaSuccess; ++i)
+      e = launched(bds::launch_group_add((float*)(ws + w.acc[i]), (const float*)(ws + w.tmp[i]), n, s), s);
+    if (e == cudaSuccess)
+      e = launched(bds::launch_group_scatter((const float*)(ws + w.st), g.Bt * g.nb * g.D, c.N, n0, gs, states, 4, s), s);
+  }
+  if (e == cudaSuccess) e = launched(bds::launch_group_out((const float*)(ws + w.acc[0]), y_c, out_elt(c), n, s), s);
+  if (e == cudaSuccess) e = launched(bds::launch_group_out((const float*)(ws + w.acc[1]), y_n, out_elt(c), n, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
+int grouped_boundary(const Call& c, const bdscan_clean* clean, const float* A_f, const float* D_f,
+                     const float* init_state, void* y_c, float* states, int emit_all, char* ws, cudaStream_t s,
+                     const char* fn) {
+  const bds::Geo& g = c.g;
+  const BndGroupWs w = bnd_group_ws(c, emit_all);
+  const GroupPlan q = group_plan(c.N);
+  const int64_t tok = g.Bt * g.L, n = g.Bt * g.L * g.D, srows = g.Bt * (emit_all ? g.nb : 1) * g.D;
+  cudaError_t e = cudaMemsetAsync(ws + w.dzero, 0, (size_t)g.D * 4, s);
+  for (int gi = 0; gi < q.G && e == cudaSuccess; ++gi) {
+    const int n0 = q.n0[gi], gs = q.gs[gi];
+    e = gather(clean->B, (int)c.in_elt, tok, c.N, n0, gs, ws + w.bc[0], s);
+    if (e == cudaSuccess) e = gather(clean->C, (int)c.in_elt, tok, c.N, n0, gs, ws + w.bc[1], s);
+    if (e == cudaSuccess) e = gather(A_f, 4, g.D, c.N, n0, gs, ws + w.a, s);
+    if (e == cudaSuccess && init_state != nullptr) e = gather(init_state, 4, g.Bt * g.D, c.N, n0, gs, ws + w.init, s);
+    if (e != cudaSuccess) break;
+    bds::FwdParams p;
+    memset(&p, 0, sizeof(p));
+    p.g = g;
+    p.xc = clean->x;
+    p.dtc = clean->dt;
+    p.Bc = ws + w.bc[0];
+    p.Cc = ws + w.bc[1];
+    p.Af = (const float*)(ws + w.a);
+    p.Df = gi == 0 ? D_f : (const float*)(ws + w.dzero);
+    p.yc = y_c != nullptr ? (void*)(ws + (gi == 0 ? w.acc : w.tmp)) : nullptr;
+    p.init = init_state != nullptr ? (const float*)(ws + w.init) : nullptr;
+    p.hst = (float*)(ws + w.scan);
+    p.sdt = (float*)(ws + w.scan + al256((size_t)g.Bt * (g.nc + 1) * g.D * 16 * 4));
+    e = bds::api_run_boundary(group_dt(c), gs, p, (float*)(ws + w.st), emit_all, s);
+    if (e == cudaSuccess && y_c != nullptr && gi > 0)
+      e = launched(bds::launch_group_add((float*)(ws + w.acc), (const float*)(ws + w.tmp), n, s), s);
+    if (e == cudaSuccess)
+      e = launched(bds::launch_group_scatter((const float*)(ws + w.st), srows, c.N, n0, gs, states, 4, s), s);
+  }
+  if (e == cudaSuccess && y_c != nullptr)
+    e = launched(bds::launch_group_out((const float*)(ws + w.acc), y_c, out_elt(c), n, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
+int grouped_backward(const Call& c, const bdscan_clean* clean, const bdscan_noisy* noisy, const bdscan_params* pr,
+                     const float* states, const void* dy_c, const void* dy_n, const float* dstates,
+                     const bdscan_clean_grads* gc, const bdscan_noisy_grads* gn, const bdscan_param_grads* gp,
+                     char* ws, cudaStream_t s, const char* fn) {
+  const bds::Geo& g = c.g;
+  const BwdGroupWs w = bwd_group_ws(c);
+  const GroupPlan q = group_plan(c.N);
+  const int64_t tok = g.Bt * g.L, n = g.Bt * g.L * g.D, srows = g.Bt * g.nb * g.D;
+  cudaError_t e = cudaMemsetAsync(ws + w.dzero, 0, (size_t)g.D * 4, s);
+  const void* bc[6] = {clean->B, clean->C, noisy->B_f, noisy->C_f, noisy->B_r, noisy->C_r};
+  void* gbc_out[6] = {gc->dB, gc->dC, gn->dB_f, gn->dC_f, gn->dB_r, gn->dC_r};
+  void* acc_out[5] = {gc->dx, gc->ddt, gn->dx, gn->ddt_f, gn->ddt_r};
+  for (int gi = 0; gi < q.G && e == cudaSuccess; ++gi) {
+    const int n0 = q.n0[gi], gs = q.gs[gi];
+    for (int i = 0; i < 6 && e == cudaSuccess; ++i) e = gather(bc[i], (int)c.in_elt, tok, c.N, n0, gs, ws + w.bc[i], s);
+    if (e == cudaSuccess) e = gather(pr->A_f, 4, g.D, c.N, n0, gs, ws + w.a[0], s);
+    if (e == cudaSuccess) e = gather(pr->A_r, 4, g.D, c.N, n0, gs, ws + w.a[1], s);
+    if (e == cudaSuccess) e = gather(states, 4, srows, c.N, n0, gs, ws + w.st, s);
+    if (e == cudaSuccess && dstates != nullptr) e = gather(dstates, 4, srows, c.N, n0, gs, ws + w.dst, s);
+    if (e != cudaSuccess) break;
+    bds::BwdParams p;
+    memset(&p, 0, sizeof(p));
+    p.g = g;
+    p.xc = clean->x;
+    p.dtc = clean->dt;
+    p.Bc = ws + w.bc[0];
+    p.Cc = ws + w.bc[1];
+    p.xn = noisy->x;
+    p.dtf = noisy->dt_f;
+    p.Bf = ws + w.bc[2];
+    p.Cf = ws + w.bc[3];
+    p.dtr = noisy->dt_r;
+    p.Br = ws + w.bc[4];
+    p.Cr = ws + w.bc[5];
+    p.Af = (const float*)(ws + w.a[0]);
+    p.Ar = (const float*)(ws + w.a[1]);
+    p.Df = gi == 0 ? pr->D_f : (const float*)(ws + w.dzero);
+    p.Dr = gi == 0 ? pr->D_r : (const float*)(ws + w.dzero);
+    p.states = (const float*)(ws + w.st);
+    p.dyc = dy_c;
+    p.dyn = dy_n;
+    p.dstates = dstates != nullptr ? (const float*)(ws + w.dst) : nullptr;
+    const size_t* dst = gi == 0 ? w.acc : w.tmp;
+    p.dxc = ws + dst[0];
+    p.ddtc = ws + dst[1];
+    p.dxn = ws + dst[2];
+    p.ddtf = ws + dst[3];
+    p.ddtr = ws + dst[4];
+    p.dBc = ws + w.gbc[0];
+    p.dCc = ws + w.gbc[1];
+    p.dBf = ws + w.gbc[2];
+    p.dCf = ws + w.gbc[3];
+    p.dBr = ws + w.gbc[4];
+    p.dCr = ws + w.gbc[5];
+    p.dAf = (float*)(ws + w.ga[0]);
+    p.dAr = (float*)(ws + w.ga[1]);
+    p.dDf = gi == 0 ? gp->dD_f : (float*)(ws + w.gd[0]);  // the D gradients do not depend on the group
+    p.dDr = gi == 0 ? gp->dD_r : (float*)(ws + w.gd[1]);
+    e = bds::api_run_backward(group_dt(c), gs, p, ws + w.scan, s);
+    for (int i = 0; i < 5 && gi > 0 && e == cudaSuccess; ++i)
+      e = launched(bds::launch_group_add((float*)(ws + w.acc[i]), (const float*)(ws + w.tmp[i]), n, s), s);
+    for (int i = 0; i < 6 && e == cudaSuccess; ++i)
+      e = launched(bds::launch_group_scatter((const float*)(ws + w.gbc[i]), tok, c.N, n0, gs, gbc_out[i], out_elt(c), s), s);
+    if (e == cudaSuccess)
+      e = launched(bds::launch_group_scatter((const float*)(ws + w.ga[0]), g.D, c.N, n0, gs, gp->dA_f, 4, s), s);
+    if (e == cudaSuccess)
+      e = launched(bds::launch_group_scatter((const float*)(ws + w.ga[1]), g.D, c.N, n0, gs, gp->dA_r, 4, s), s);
+  }
+  for (int i = 0; i < 5 && e == cudaSuccess; ++i)
+    e = launched(bds::launch_group_out((const float*)(ws + w.acc[i]), acc_out[i], out_elt(c), n, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
+int grouped_active(const Call& c, const float* seed, const bdscan_noisy* noisy, const bdscan_params* pr, void* y_n,
+                   cudaStream_t s, const char* fn) {
+  const bds::Geo& g = c.g;
+  const ActGroupWs w = act_group_ws(c);
+  if (w.total > bds::kGroupScratchBytes)
+    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: d_state %d needs %zu bytes of group scratch (%zu available)", fn, c.N,
+                w.total, bds::kGroupScratchBytes);
+  char* ws = (char*)bds::group_scratch();
+  if (ws == nullptr) return cuda_fail(cudaGetLastError(), fn);
+  const GroupPlan q = group_plan(c.N);
+  const int64_t tok = g.Bt * g.L, n = g.Bt * g.L * g.D;
+  cudaError_t e = cudaMemsetAsync(ws + w.dzero, 0, (size_t)g.D * 4, s);
+  const void* bc[4] = {noisy->B_f, noisy->C_f, noisy->B_r, noisy->C_r};
+  for (int gi = 0; gi < q.G && e == cudaSuccess; ++gi) {
+    const int n0 = q.n0[gi], gs = q.gs[gi];
+    for (int i = 0; i < 4 && e == cudaSuccess; ++i) e = gather(bc[i], (int)c.in_elt, tok, c.N, n0, gs, ws + w.bc[i], s);
+    if (e == cudaSuccess) e = gather(pr->A_f, 4, g.D, c.N, n0, gs, ws + w.a[0], s);
+    if (e == cudaSuccess) e = gather(pr->A_r, 4, g.D, c.N, n0, gs, ws + w.a[1], s);
+    if (e == cudaSuccess) e = gather(seed, 4, g.Bt * g.D, c.N, n0, gs, ws + w.seed, s);
+    if (e != cudaSuccess) break;
+    bds::FwdParams p;
+    memset(&p, 0, sizeof(p));
+    p.g = g;
+    p.xn = noisy->x;
+    p.dtf = noisy->dt_f;
+    p.Bf = ws + w.bc[0];
+    p.Cf = ws + w.bc[1];
+    p.dtr = noisy->dt_r;
+    p.Br = ws + w.bc[2];
+    p.Cr = ws + w.bc[3];
+    p.Af = (const float*)(ws + w.a[0]);
+    p.Ar = (const float*)(ws + w.a[1]);
+    p.Df = gi == 0 ? pr->D_f : (const float*)(ws + w.dzero);
+    p.Dr = gi == 0 ? pr->D_r : (const float*)(ws + w.dzero);
+    p.yn = ws + (gi == 0 ? w.acc : w.tmp);
+    p.seed = (const float*)(ws + w.seed);
+    e = launched(bds::launch_active_block(group_dt(c), gs, p, s), s);
+    if (e == cudaSuccess && gi > 0)
+      e = launched(bds::launch_group_add((float*)(ws + w.acc), (const float*)(ws + w.tmp), n, s), s);
+  }
+  if (e == cudaSuccess) e = launched(bds::launch_group_out((const float*)(ws + w.acc), y_n, out_elt(c), n, s), s);
+  if (e != cudaSuccess) return cuda_fail(e, fn);
+  return ok();
+}
+
 }  // namespace
 
 extern "C" {
@@ -293,20 +632,23 @@ int64_t bdscan_chunk_tokens(int64_t block) { return block <= 0 ? 0 : blocks_per_
 
 size_t bdscan_forward_workspace_size(const bdscan_dims* dims) {
   Call c;
-  if (check_dims(dims, &c, "bdscan_forward_workspace_size") != BDSCAN_OK) return 0;
+  if (check_dims_any(dims, &c, "bdscan_forward_workspace_size") != BDSCAN_OK) return 0;
+  if (!direct_N(c.N)) return fwd_group_ws(c).total;
   return fwd_ws(c.g, c.N);
 }
 
 size_t bdscan_boundary_states_workspace_size(const bdscan_dims* dims, int emit_all) {
   (void)emit_all;
   Call c;
-  if (check_dims(dims, &c, "bdscan_boundary_states_workspace_size") != BDSCAN_OK) return 0;
+  if (check_dims_any(dims, &c, "bdscan_boundary_states_workspace_size") != BDSCAN_OK) return 0;
+  if (!direct_N(c.N)) return bnd_group_ws(c, emit_all).total;
   return fwd_ws(c.g, c.N);
 }
 
 size_t bdscan_backward_workspace_size(const bdscan_dims* dims) {
   Call c;
-  if (check_dims(dims, &c, "bdscan_backward_workspace_size") != BDSCAN_OK) return 0;
+  if (check_dims_any(dims, &c, "bdscan_backward_workspace_size") != BDSCAN_OK) return 0;
+  if (!direct_N(c.N)) return bwd_group_ws(c).total;
   bds::Geo gmax = c.g;
   gmax.nc = bds::bwd_max_chunks(c.g);
   return bwd_ws(gmax, c.N).total;
@@ -317,7 +659,7 @@ int bdscan_forward(const bdscan_dims* dims, const bdscan_clean* clean, const bds
                    size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_forward";
   Call c;
-  int rc = check_dims(dims, &c, fn);
+  int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, false, fn))) return rc;
   if (c.g.Bt == 0 || c.g.L == 0) return ok();
@@ -325,11 +667,12 @@ int bdscan_forward(const bdscan_dims* dims, const bdscan_clean* clean, const bds
   REQ(y_c, fn, "y_c");
   REQ(y_n, fn, "y_n");
   REQ(states, fn, "states");
-  const size_t need = fwd_ws(c.g, c.N);
+  const size_t need = direct_N(c.N) ? fwd_ws(c.g, c.N) : fwd_group_ws(c).total;
   REQ(workspace, fn, "workspace");
   if (workspace_bytes < need)
     return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
   cudaStream_t s = (cudaStream_t)stream;
+  if (!direct_N(c.N)) return grouped_forward(c, clean, noisy, params, y_c, y_n, states, (char*)workspace, s, fn);
   bds::FwdParams p;
   memset(&p, 0, sizeof(p));
   p.g = c.g;
@@ -356,7 +699,7 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
                            void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_boundary_states";
   Call c;
-  int rc = check_dims(dims, &c, fn);
+  int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, false, fn))) return rc;
   if (c.g.Bt == 0) return ok();
@@ -376,10 +719,12 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
   REQ(D_f, fn, "D_f");
   REQ(states, fn, "states");
   OPT(y_c, fn, "y_c");
-  const size_t need = fwd_ws(c.g, c.N);
+  const size_t need = direct_N(c.N) ? fwd_ws(c.g, c.N) : bnd_group_ws(c, emit_all).total;
   REQ(workspace, fn, "workspace");
   if (workspace_bytes < need)
     return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
+  if (!direct_N(c.N))
+    return grouped_boundary(c, clean, A_f, D_f, init_state, y_c, states, emit_all, (char*)workspace, s, fn);
   bds::FwdParams p;
   memset(&p, 0, sizeof(p));
   p.g = c.g;
@@ -399,7 +744,7 @@ int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan
                         const bdscan_params* params, void* y_n, void* stream) {
   const char* fn = "bdscan_active_block";
   Call c;
-  int rc = check_dims(dims, &c, fn);
+  int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if (dims->len != dims->block && dims->len != 0)
     return fail(BDSCAN_ERR_ARG, "%s: len (%lld) must equal block (%lld)", fn, (long long)dims->len,
@@ -409,6 +754,7 @@ int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan
   REQ(seed, fn, "seed");
   if ((rc = check_noisy(noisy, fn)) || (rc = check_params(params, fn))) return rc;
   REQ(y_n, fn, "y_n");
+  if (!direct_N(c.N)) return grouped_active(c, seed, noisy, params, y_n, (cudaStream_t)stream, fn);
   bds::FwdParams p;
   memset(&p, 0, sizeof(p));
   p.g = c.g;
@@ -530,7 +876,7 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
                     const bdscan_param_grads* gparams, void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_backward";
   Call c;
-  int rc = check_dims(dims, &c, fn);
+  int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, true, fn))) return rc;
   if (gparams == nullptr) return fail(BDSCAN_ERR_ARG, "%s: gparams is NULL", fn);
@@ -567,10 +913,13 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
   REQ(gnoisy->dC_r, fn, "gnoisy.dC_r");
   bds::Geo gmax = c.g;
   gmax.nc = bds::bwd_max_chunks(c.g);
-  const size_t need = bwd_ws(gmax, c.N).total;
+  const size_t need = direct_N(c.N) ? bwd_ws(gmax, c.N).total : bwd_group_ws(c).total;
   REQ(workspace, fn, "workspace");
   if (workspace_bytes < need)
     return fail(BDSCAN_ERR_ARG, "%s: workspace of %zu bytes, %zu needed", fn, workspace_bytes, need);
+  if (!direct_N(c.N))
+    return grouped_backward(c, clean, noisy, params, states, dy_c, dy_n, dstates, gclean, gnoisy, gparams,
+                            (char*)workspace, s, fn);
   bds::BwdParams p;
   memset(&p, 0, sizeof(p));
   p.xc = clean->x;

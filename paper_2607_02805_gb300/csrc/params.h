@@ -72,6 +72,17 @@ cudaError_t launch_block_scan(int dt, int N, int mode, int nchunks, const FwdPar
 // One noisy block per batch row from p.seed (len == block).
 cudaError_t launch_active_block(int dt, int N, const FwdParams& p, cudaStream_t s);
 // Per-token layer-norm statistics of rows x D elements (dt: 0 f32, else bf16).
+// State groups of the diagonal form (groups.cu): d_state split into groups
+// of 16 (the last one 8 or 16, zero-padded) run one after another.
+constexpr size_t kGroupScratchBytes = (size_t)16 << 20;  // scratch of the grouped active block
+cudaError_t launch_group_gather(const void* src, int elt, int64_t rows, int N, int n0, int gs, void* dst,
+                                cudaStream_t s);
+cudaError_t launch_group_scatter(const float* src, int64_t rows, int N, int n0, int gs, void* dst, int out_elt,
+                                 cudaStream_t s);
+cudaError_t launch_group_add(float* acc, const float* add, int64_t n, cudaStream_t s);
+cudaError_t launch_group_out(const float* acc, void* out, int out_elt, int64_t n, cudaStream_t s);
+void* group_scratch();  // device address of the grouped active block's scratch, or null
+
 cudaError_t launch_ln_stats(int dt, const void* h, int64_t rows, int64_t D, float eps, float2* stats, cudaStream_t s);
 // The active block on the modulated input (1 + scale) LN(x) + shift, writing
 // x + gate * y_n (p.shift, p.scale, p.gate, p.ln_stats set).

@@ -81,7 +81,8 @@ def _fwd(d, c=None, n=None, p=None, y=FAKE, ws=FAKE, wsb=1 << 40):
     (dict(length=60), binding.BDSCAN_ERR_ARG, "not a multiple of block"),
     (dict(block=0), binding.BDSCAN_ERR_ARG, "block must be positive"),
     (dict(batch=-1), binding.BDSCAN_ERR_ARG, "negative"),
-    (dict(d_state=12), binding.BDSCAN_ERR_UNSUPPORTED, "d_state"),
+    (dict(d_state=10), binding.BDSCAN_ERR_UNSUPPORTED, "a multiple of 4 up to 64"),
+    (dict(d_state=68), binding.BDSCAN_ERR_UNSUPPORTED, "a multiple of 4 up to 64"),
     (dict(d_inner=12), binding.BDSCAN_ERR_UNSUPPORTED, "multiple of 8"),
     (dict(dtype=binding.BDSCAN_F32, out_dtype=binding.BDSCAN_BF16), binding.BDSCAN_ERR_UNSUPPORTED, "f32 inputs"),
     (dict(dtype=7), binding.BDSCAN_ERR_ARG, "bad dtype"),
@@ -329,3 +330,17 @@ def test_debug_build_exports_the_same_functions():
     d = binding.make_dims(1, 64, 16, 32, 3, binding.BDSCAN_F32)
     rc = lib.bdscan_forward(ctypes.byref(d), None, None, None, None, None, None, None, 0, None)
     assert rc == binding.BDSCAN_ERR_UNSUPPORTED and b"d_state 3" in lib.bdscan_last_error()
+
+
+def test_state_groups_size_their_workspaces_and_other_entry_points_refuse_them():
+    """d_state 32 runs in state groups for the forward, backward, cache build
+    and active block (their workspaces grow with the per-group buffers); the
+    other entry points keep d_state 8 or 16."""
+    d16, d32 = _dims(d_state=16), _dims(d_state=32)
+    assert binding.bdscan_forward_workspace_size(d32) > binding.bdscan_forward_workspace_size(d16) > 0
+    assert binding.bdscan_backward_workspace_size(d32) > binding.bdscan_backward_workspace_size(d16) > 0
+    assert binding.bdscan_boundary_states_workspace_size(d32, 1) > 0
+    assert binding.bdscan_full_bidir_workspace_size(d32) == 0
+    assert "not supported here (8 or 16)" in binding.bdscan_last_error()
+    assert binding.bdscan_active_block_adaln_workspace_size(d32) == 0
+    assert binding.bdscan_mixer_forward_workspace_size(d32) == 0
