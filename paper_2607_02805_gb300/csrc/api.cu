@@ -207,8 +207,12 @@ BwdWs bwd_ws(const bds::Geo& g, int N) {
   return w;
 }
 
+// Blocks up to 256 tokens for the forward-side kernels (the paper's block,
+// hyperparameter table), up to 64 for the backward (its per-block dx buffer
+// and segment checkpoints live in shared memory).
 int check_block_limits(const Call& c, bool backward, const char* fn) {
-  if (c.g.Bs > 64) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: block %lld above 64", fn, (long long)c.g.Bs);
+  if (backward && c.g.Bs > 64) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward block %lld above 64", fn, (long long)c.g.Bs);
+  if (c.g.Bs > 256) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: block %lld above 256", fn, (long long)c.g.Bs);
   if (backward && c.g.Bs > 16 && c.g.Bs % 16 != 0)
     return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward needs block <= 16 or a multiple of 16", fn);
   return BDSCAN_OK;
@@ -787,6 +791,8 @@ int bdscan_active_block_adaln(const bdscan_dims* dims, const float* seed, const 
     return fail(BDSCAN_ERR_ARG, "%s: len (%lld) must equal block (%lld)", fn, (long long)dims->len,
                 (long long)dims->block);
   if ((rc = check_block_limits(c, false, fn))) return rc;
+  if (c.g.Bs > 128)  // the modulated block is kept in shared memory next to the scan's
+    return fail(BDSCAN_ERR_UNSUPPORTED, "%s: block %lld above 128", fn, (long long)c.g.Bs);
   if (c.g.Bt == 0 || c.g.L == 0) return ok();
   REQ(seed, fn, "seed");
   if ((rc = check_noisy(noisy, fn)) || (rc = check_params(params, fn))) return rc;

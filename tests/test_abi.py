@@ -86,7 +86,7 @@ def _fwd(d, c=None, n=None, p=None, y=FAKE, ws=FAKE, wsb=1 << 40):
     (dict(d_inner=12), binding.BDSCAN_ERR_UNSUPPORTED, "multiple of 8"),
     (dict(dtype=binding.BDSCAN_F32, out_dtype=binding.BDSCAN_BF16), binding.BDSCAN_ERR_UNSUPPORTED, "f32 inputs"),
     (dict(dtype=7), binding.BDSCAN_ERR_ARG, "bad dtype"),
-    (dict(block=128, length=256), binding.BDSCAN_ERR_UNSUPPORTED, "above 64"),
+    (dict(block=512, length=1024), binding.BDSCAN_ERR_UNSUPPORTED, "above 256"),
 ])
 def test_forward_rejects_bad_dims(kw, code, msg):
     assert _fwd(_dims(**kw)) == code
@@ -120,6 +120,9 @@ def test_backward_block_limits():
     gp = binding.bdscan_param_grads(FAKE, FAKE, FAKE, FAKE)
     rc = binding.bdscan_backward(d, c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE, 1 << 40, None)
     assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "multiple of 16" in binding.bdscan_last_error()
+    rc = binding.bdscan_backward(_dims(block=128, length=256), c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE,
+                                 1 << 40, None)
+    assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "backward block 128 above 64" in binding.bdscan_last_error()
     gn.dB_r = None
     rc = binding.bdscan_backward(_dims(), c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE, 1 << 40, None)
     assert rc == binding.BDSCAN_ERR_ARG and "gnoisy.dB_r is NULL" in binding.bdscan_last_error()

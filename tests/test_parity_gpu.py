@@ -318,3 +318,31 @@ def test_config_very_long_context_262k():
     """Cache build over 262,144 tokens (block 16), then 16 active-block calls
     reusing the same read-only cached state."""
     _long_context(262144, 16, 16, seed=5)
+
+
+# ---------------------------------------------------------------------------
+# the forward side at the paper's block sizes (128 and 256 tokens)
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("Bt,L,Bs,D,N,dt,seed", [
+    (2, 512, 128, 136, 16, "bf16", 41),   # one block per chunk, ragged channel group
+    (1, 768, 256, 64, 8, "f32", 42),
+    (1, 512, 256, 64, 32, "bf16", 43),    # with state groups
+])
+def test_long_block_forward_parity_and_cache(Bt, L, Bs, D, N, dt, seed):
+    """All-block forward against the oracle; cache build and the cached
+    active block reproduce it bit for bit."""
+    wl = Workload(Bt, L, Bs, D, N, dtype=dt, seed=seed, with_grads=False)
+    lay = Layer(wl)
+    lay.forward()
+    torch.cuda.synchronize()
+    y_c, y_n, st = P.oracle_forward(wl)
+    _check_forward(lay, y_c, y_n, st)
+    pre = _sub_workload(wl, 0, L - Bs)
+    fin, _ = _boundary(pre, emit_all=False)
+    allst, y_pre = _boundary(pre, emit_all=True, want_y=True)
+    y = _active(_sub_workload(wl, L - Bs, L), fin[:, 0])
+    torch.cuda.synchronize()
+    assert torch.equal(allst, lay.states[:, :-1])
+    assert torch.equal(fin[:, 0], lay.states[:, -2])
+    assert torch.equal(y_pre, lay.y_c[:, : L - Bs])
+    assert torch.equal(y, lay.y_n[:, L - Bs:])
