@@ -208,10 +208,10 @@ BwdWs bwd_ws(const bds::Geo& g, int N) {
 }
 
 // Blocks up to 256 tokens for the forward-side kernels (the paper's block,
-// hyperparameter table), up to 64 for the backward (its per-block dx buffer
+// hyperparameter table), up to 128 for the backward (its per-block dx buffer
 // and segment checkpoints live in shared memory).
 int check_block_limits(const Call& c, bool backward, const char* fn) {
-  if (backward && c.g.Bs > 64) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward block %lld above 64", fn, (long long)c.g.Bs);
+  if (backward && c.g.Bs > 128) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward block %lld above 128", fn, (long long)c.g.Bs);
   if (c.g.Bs > 256) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: block %lld above 256", fn, (long long)c.g.Bs);
   if (backward && c.g.Bs > 16 && c.g.Bs % 16 != 0)
     return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward needs block <= 16 or a multiple of 16", fn);

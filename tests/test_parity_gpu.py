@@ -56,6 +56,9 @@ SMALL = [  # (Bt, L, Bs, D, N, dtype, out_dtype, seed)
     (2, 96, 1, 40, 16, "f32", None, 6),           # block size 1
     (1, 288, 48, 48, 16, "f32", None, 7),         # 3 segments, 2-block chunks, ragged chunk
     (3, 256, 8, 256, 8, "bf16", binding.BDSCAN_F32, 8),
+    (1, 384, 128, 136, 16, "bf16", None, 9),     # 8 segments per block, one block per chunk
+    (2, 256, 128, 64, 8, "f32", None, 10),
+    (1, 384, 96, 64, 16, "bf16", binding.BDSCAN_F32, 14),  # 6 segments, 96-token chunks
 ]
 
 
