@@ -64,7 +64,8 @@
  *     (bf16,bf16), (bf16,f32); d_inner a multiple of 8 (bf16 inputs) or 4
  *     (f32 inputs); len a multiple of block; block <= 256 for forward-only
  *     calls (<= 128 with AdaLN) and block <= 16, or a multiple of 16 up to
- *     128, for the backward.
+ *     256, for the backward (above 128 tokens its segment checkpoints are
+ *     kept in the workspace).
  *     Any batch and len >= 0 (zero-size problems are no-ops).
  */
 #ifndef BDSCAN_H

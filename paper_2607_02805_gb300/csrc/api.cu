@@ -186,7 +186,7 @@ size_t fwd_ws(const bds::Geo& g, int N) {
 }
 
 struct BwdWs {
-  size_t dS, Lc, sdtc, part_tok, part_A, part_D, total;
+  size_t dS, Lc, sdtc, part_tok, part_A, part_D, ck, total;
 };
 BwdWs bwd_ws(const bds::Geo& g, int N) {
   BwdWs w;
@@ -203,15 +203,19 @@ BwdWs bwd_ws(const bds::Geo& g, int N) {
   o += al256((size_t)3 * g.Bt * g.nc * g.D * N * 4);
   w.part_D = o;
   o += al256((size_t)2 * g.Bt * g.nc * g.D * 4);
+  // segment checkpoints of long blocks: one region per CTA of each TMEM kernel
+  // (grid G x nc x Bt), (Bs/16 - 1) x N x 128 floats each
+  w.ck = o;
+  if (g.Bs > bds::kCkSmemMaxBs) o += 2 * al256((size_t)g.G * g.nc * g.Bt * (g.Bs / 16 - 1) * N * bds::kCtaHost * 4);
   w.total = o;
   return w;
 }
 
-// Blocks up to 256 tokens for the forward-side kernels (the paper's block,
-// hyperparameter table), up to 128 for the backward (its per-block dx buffer
-// and segment checkpoints live in shared memory).
+// Blocks up to 256 tokens (the paper's block, hyperparameter table); the
+// backward keeps the segment checkpoints of blocks above kCkSmemMaxBs in
+// global memory.
 int check_block_limits(const Call& c, bool backward, const char* fn) {
-  if (backward && c.g.Bs > 128) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward block %lld above 128", fn, (long long)c.g.Bs);
+  if (backward && c.g.Bs > 256) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward block %lld above 256", fn, (long long)c.g.Bs);
   if (c.g.Bs > 256) return fail(BDSCAN_ERR_UNSUPPORTED, "%s: block %lld above 256", fn, (long long)c.g.Bs);
   if (backward && c.g.Bs > 16 && c.g.Bs % 16 != 0)
     return fail(BDSCAN_ERR_UNSUPPORTED, "%s: backward needs block <= 16 or a multiple of 16", fn);
@@ -1102,6 +1106,11 @@ cudaError_t api_run_backward(int dt, int N, BwdParams& p, void* workspace, cudaS
   p.part_tok = (float*)(ws + w.part_tok);
   p.part_A = (float*)(ws + w.part_A);
   p.part_D = (float*)(ws + w.part_D);
+  if (gb.Bs > kCkSmemMaxBs) {
+    const size_t ckb = al256((size_t)gb.G * gb.nc * gb.Bt * (gb.Bs / 16 - 1) * N * kCtaHost * 4);
+    p.ck_noisy = (float*)(ws + w.ck);
+    p.ck_clean = (float*)(ws + w.ck + ckb);
+  }
   cudaError_t e = launched(launch_bwd_noisy(dt, N, p, s), s);
   if (e == cudaSuccess) e = launched(launch_bwd_carry(N, p, s), s);
   if (e == cudaSuccess) e = launched(launch_bwd_clean(dt, N, p, s), s);

@@ -13,8 +13,9 @@ struct CleanBwdSmem {
   // `bufs` staging buffers, as for the noisy kernel
   static __host__ __device__ size_t red_off(int bufs) { return align16(St::buf_bytes(kBwdTS) * bufs); }
   static __host__ __device__ size_t ck_off(int bufs) { return red_off(bufs) + (size_t)2 * kBwdTS * kRedRow * 4; }
+  // checkpoints in shared memory up to kCkSmemMaxBs tokens, else in global memory
   static __host__ __device__ size_t slot_off(int bufs, int TS, int Bs) {
-    return ck_off(bufs) + (size_t)(Bs / TS - 1) * N * kCta * 4;
+    return ck_off(bufs) + (Bs > kCkSmemMaxBs ? 0 : (size_t)(Bs / TS - 1) * N * kCta * 4);
   }
   // one-segment blocks: the seeds of the current and the next block
   static __host__ __device__ size_t seed_off(int bufs, int TS, int Bs) { return slot_off(bufs, TS, Bs) + 16; }
@@ -54,7 +55,10 @@ __global__ void __launch_bounds__(kCta, 3) k_bwd_clean(const BwdParams p) {
   const int bufs = NSEG == 1 ? 2 : (resident ? NSEG : 1);
   float* red = reinterpret_cast<float*>(smem + L::red_off(bufs));
   float* mine = red_slot<N>(red);
-  float* ck = reinterpret_cast<float*>(smem + L::ck_off(bufs));
+  float* ck = Bs > kCkSmemMaxBs
+                  ? p.ck_clean + (((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x) *
+                                     (size_t)(NSEG - 1) * N * kCta
+                  : reinterpret_cast<float*>(smem + L::ck_off(bufs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(bufs, TS, Bs));
   float* seedb = reinterpret_cast<float*>(smem + L::seed_off(bufs, TS, Bs));  // [2][kCta][N]
 

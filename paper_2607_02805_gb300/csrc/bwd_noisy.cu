@@ -21,8 +21,9 @@ struct NoisyBwdSmem {
   // direction's segment at a time otherwise
   static __host__ __device__ int red_slots(int Bs) { return Bs < kBwdTS ? 4 : 2; }
   static __host__ __device__ size_t ck_off(int bufs, int Bs) { return red_off(bufs, Bs) + (size_t)red_slots(Bs) * kBwdTS * kRedRow * 4; }
+  // checkpoints in shared memory up to kCkSmemMaxBs tokens, else in global memory
   static __host__ __device__ size_t slot_off(int bufs, int TS, int Bs) {
-    return ck_off(bufs, Bs) + (size_t)(Bs / TS - 1) * N * kCta * 4;
+    return ck_off(bufs, Bs) + (Bs > kCkSmemMaxBs ? 0 : (size_t)(Bs / TS - 1) * N * kCta * 4);
   }
   static __host__ __device__ size_t bytes(int bufs, int TS, int Bs) { return slot_off(bufs, TS, Bs) + 16; }
 };
@@ -66,7 +67,10 @@ __global__ void __launch_bounds__(kCta, 1) k_bwd_noisy(const BwdParams p) {
   float* dxbuf = reinterpret_cast<float*>(smem + L::dx_off(bufs));
   float* red = reinterpret_cast<float*>(smem + L::red_off(bufs, Bs));
   float* mine = red_slot<N>(red);
-  float* ck = reinterpret_cast<float*>(smem + L::ck_off(bufs, Bs));
+  float* ck = Bs > kCkSmemMaxBs
+                  ? p.ck_noisy + (((size_t)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x) *
+                                     (size_t)(NSEG - 1) * N * kCta
+                  : reinterpret_cast<float*>(smem + L::ck_off(bufs, Bs));
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + L::slot_off(bufs, TS, Bs));
 
   const uint32_t tcols = full_cols(TS, N);

@@ -822,8 +822,8 @@ int bdscan_mixer_backward(const bdscan_dims* dims, const bdscan_clean* clean, co
   int dt = 0, N = 0;
   int rc = bds::api_check_forward_dims(dims, &g, &dt, &N, fn);
   if (rc) return rc;
-  if (g.Bs > 128)
-    return bds::api_fail(BDSCAN_ERR_UNSUPPORTED, "bdscan_mixer_backward: backward block above 128");
+  if (g.Bs > 256)
+    return bds::api_fail(BDSCAN_ERR_UNSUPPORTED, "bdscan_mixer_backward: backward block above 256");
   if (g.Bs > 16 && g.Bs % 16 != 0)
     return bds::api_fail(BDSCAN_ERR_UNSUPPORTED, "bdscan_mixer_backward: backward needs block <= 16 or a multiple of 16");
   if (gparams == nullptr || gmparams == nullptr) return bds::bad_arg(fn, "gparams or gmparams is NULL");

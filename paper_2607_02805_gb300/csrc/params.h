@@ -8,6 +8,8 @@
 namespace bds {
 
 constexpr int kCtaHost = 128;  // channels per CTA (one per thread); equals kCta in device.cuh
+// Longest block whose backward segment checkpoints stay in shared memory.
+constexpr int kCkSmemMaxBs = 128;
 
 // Geometry shared by all kernels of one call.
 struct Geo {
@@ -62,6 +64,10 @@ struct BwdParams {
   float* part_A;    // [3][Bt*nc][D][N] dA partial sums: noisy fwd, noisy rev, clean
   float* part_D;    // [2][Bt*nc][D]    dD partial sums: noisy, clean
   int seg_resident;  // set per launch: blocks of several segments staged whole
+  // segment checkpoints of blocks above kCkSmemMaxBs tokens, in global memory:
+  // per CTA (linear block index) (Bs/16 - 1) x N x 128 floats; null otherwise
+  float* ck_noisy;
+  float* ck_clean;
 };
 
 // Launchers (fwd.cu / bwd.cu). dt: 0 = f32 in/out, 1 = bf16 in/out, 2 = bf16 in, f32 out.

@@ -120,9 +120,12 @@ def test_backward_block_limits():
     gp = binding.bdscan_param_grads(FAKE, FAKE, FAKE, FAKE)
     rc = binding.bdscan_backward(d, c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE, 1 << 40, None)
     assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "multiple of 16" in binding.bdscan_last_error()
-    rc = binding.bdscan_backward(_dims(block=256, length=512), c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE,
+    rc = binding.bdscan_backward(_dims(block=512, length=1024), c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE,
                                  1 << 40, None)
-    assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "backward block 256 above 128" in binding.bdscan_last_error()
+    assert rc == binding.BDSCAN_ERR_UNSUPPORTED and "backward block 512 above 256" in binding.bdscan_last_error()
+    # blocks above 128 tokens keep their segment checkpoints in the workspace
+    assert binding.bdscan_backward_workspace_size(_dims(block=256, length=512)) > \
+        binding.bdscan_backward_workspace_size(_dims(block=128, length=512))
     gn.dB_r = None
     rc = binding.bdscan_backward(_dims(), c, n, p, FAKE, FAKE, FAKE, None, gc, gn, gp, FAKE, 1 << 40, None)
     assert rc == binding.BDSCAN_ERR_ARG and "gnoisy.dB_r is NULL" in binding.bdscan_last_error()

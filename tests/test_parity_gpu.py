@@ -59,6 +59,8 @@ SMALL = [  # (Bt, L, Bs, D, N, dtype, out_dtype, seed)
     (1, 384, 128, 136, 16, "bf16", None, 9),     # 8 segments per block, one block per chunk
     (2, 256, 128, 64, 8, "f32", None, 10),
     (1, 384, 96, 64, 16, "bf16", binding.BDSCAN_F32, 14),  # 6 segments, 96-token chunks
+    (2, 512, 256, 136, 16, "bf16", None, 15),    # 16 segments: checkpoints in global memory
+    (1, 512, 256, 64, 8, "f32", None, 16),
 ]
 
 
