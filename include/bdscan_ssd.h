@@ -159,6 +159,11 @@ int bdscan_ssd_wait_flag(int reset);
  * up and was reported) after clearing it, or a negative BDSCAN_ERR_* code. */
 int bdscan_ssd_wait_selftest(uint32_t polls);
 
+/* 1 if the kernels load their operand tiles with the tensor memory
+ * accelerator (TMA: the driver provides the tensor-map encoder), 0 if they
+ * fall back to cp.async. Left-to-right streams use TMA when available. */
+int bdscan_ssd_tma_enabled(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -149,6 +149,7 @@ SIGNATURES = [
     ("bdscan_debug_build", ctypes.c_int, []),
     ("bdscan_debug_set_slack", ctypes.c_int, [ctypes.c_longlong]),
     ("bdscan_ssd_wait_selftest", ctypes.c_int, [ctypes.c_uint32]),
+    ("bdscan_ssd_tma_enabled", ctypes.c_int, []),
     ("bdscan_ssd_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
     ("bdscan_ssd_full_bidir_forward", ctypes.c_int,
      [_P(bdscan_ssd_dims), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
@@ -378,6 +379,10 @@ def bdscan_ssd_wait_flag(reset) -> int:
 
 def bdscan_ssd_wait_selftest(polls) -> int:
     return load().bdscan_ssd_wait_selftest(int(polls))
+
+
+def bdscan_ssd_tma_enabled() -> int:
+    return load().bdscan_ssd_tma_enabled()
 
 
 def bdscan_ssd_full_bidir_workspace_size(dims) -> int:

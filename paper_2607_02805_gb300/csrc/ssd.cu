@@ -21,6 +21,11 @@
 //     parts); the epilogue adds the decayed seed term and D x.
 #include <atomic>
 #include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
 
 #include "device.cuh"
 #include "params.h"
@@ -366,10 +371,11 @@ __device__ __forceinline__ void setup_dir(const T* dt, int hs, int n, float A2, 
 // the forward direction and its first token for the reverse one); only the
 // 32 x 32 blocks on the diagonal take one exp per element.
 template <int N, bool NOISY>
-__global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdScanParams p) {
+__global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdScanParams p,
+                                                                    const __grid_constant__ CUtensorMap xmap) {
   extern __shared__ unsigned char smraw[];
   unsigned char* sm = align1024(smraw);
-  __shared__ uint64_t bar[2];  // [0]: a head's MMAs, [1]: the Gram products
+  __shared__ uint64_t bar[3];  // [0]: a head's MMAs, [1]: the Gram products, [2]: a head's loads (TMA)
   __shared__ uint32_t tslot;
   const SsdGeo& g = p.g;
   const int Bs = (int)g.Bs, H = g.H, m = g.m, t = threadIdx.x;
@@ -429,6 +435,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   if (t == 0) {
     umma::bar_init(&bar[0], 1);
     umma::bar_init(&bar[1], 1);
+    umma::bar_init(&bar[2], 1);
   }
   if (t < 32) tmem_alloc(&tslot, 512);
   cp_async_wait_all();
@@ -446,9 +453,25 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   }
   bool alive = cta_wait(&bar[1], 0, p.flag);
   umma::fence_after_sync();
+  // one head's x tiles and raw seed into buffer xbuf: by TMA (thread 0; a
+  // 128-token x tile is one box of the [tokens][heads][64] map, the seed one
+  // contiguous run) when the launcher set up the map, else by cp.async
+  auto load_head = [&](int hd, uint32_t xbuf) {
+    const float* seed_h = has_seed ? seed_src + (int64_t)hd * kSsdP * N : nullptr;
+    if (p.tma) {
+      if (t == 0) {
+        umma::fence_async_smem();  // the buffers' earlier generic accesses before the async writes
+        bar_expect_tx(&bar[2], (uint32_t)ntile * 16384u + (seed_h != nullptr ? (uint32_t)(kSsdP * N * 4) : 0u));
+        const int row0 = (int)(b * g.L + (int64_t)k * Bs);
+        for (int j = 0; j < ntile; ++j) tma_load_3d(sm + xbuf + (uint32_t)j * 16384u, &xmap, 0, hd, row0 + 128 * j, &bar[2]);
+        if (seed_h != nullptr) bulk_load(sm + L.raw, seed_h, (uint32_t)(kSsdP * N * 4), &bar[2]);
+      }
+    } else {
+      issue_head_loads<N>(sm, L, p.x, tok, H, hd, ntile, seed_h, xbuf);
+    }
+  };
   // the first head's x and seed (the B tiles are no longer read)
-  if (alive && h0 < h1)
-    issue_head_loads<N>(sm, L, p.x, tok, H, h0, ntile, has_seed ? seed_src + (int64_t)h0 * kSsdP * N : nullptr, L.x);
+  if (alive && h0 < h1) load_head(h0, L.x);
   // decay vectors of head hh into buffer `buf`: warp 0 the forward direction,
   // warp 1 the reverse one (each scans, then fills its column factors;
   // forward referenced to the column group's last token, reverse to its first)
@@ -569,7 +592,14 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     const int h = h0 + hh;
     const uint32_t xcur = L.x + (hh & 1) * L.xsz;  // this head's x tiles
     const float* v = vec0 + (hh & 1) * 1536;       // this head's decay vectors
-    cp_async_wait_all();
+    if (p.tma) {  // head hh's loads complete phase hh of the load barrier
+      if (!cta_wait(&bar[2], (uint32_t)(hh & 1), p.flag)) {
+        alive = false;
+        break;
+      }
+    } else {
+      cp_async_wait_all();
+    }
     __syncthreads();  // the head's x and raw seed have landed, its decay vectors are ready
     if (has_seed) {   // seed (fp32, staged in m1) -> bf16 high + low parts, K-major
       for (int c = t; c < kSsdP * N / 8; c += kScanThreads) {
@@ -614,9 +644,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     }
     umma::fence_after_sync();
     // the next head's loads run under this head's epilogue
-    if (hh + 1 < hg)
-      issue_head_loads<N>(sm, L, p.x, tok, H, h + 1, ntile, has_seed ? seed_src + (int64_t)(h + 1) * kSsdP * N : nullptr,
-                          L.x + ((hh + 1) & 1) * L.xsz);
+    if (hh + 1 < hg) load_head(h + 1, L.x + ((hh + 1) & 1) * L.xsz);
     // --- epilogue: y = mixing term + decayed seed term + D x, bf16 out;
     // this warp's 32 channels of its token row
     {
@@ -752,16 +780,52 @@ cudaError_t launch_ssd_state_pass(const SsdPassParams& p, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+// The driver's tensor-map encoder, looked up once through the runtime (no
+// link against the driver library); null if unavailable.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+bool ssd_tma_enabled() { return tensor_map_encoder() != nullptr; }
+
+// x [rows][H][64] bf16 as a 3-D map with boxes of 64 channels x 1 head x 128
+// tokens, 128-byte swizzle (the layout the MMA descriptors read).
+bool encode_x_map(CUtensorMap* m, const __nv_bfloat16* x, int64_t rows, int H) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (enc == nullptr || rows >= ((int64_t)1 << 31) || ((uintptr_t)x & 15u) != 0) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)kSsdP, (cuuint64_t)H, (cuuint64_t)rows};
+  const cuuint64_t strides[2] = {(cuuint64_t)kSsdP * 2, (cuuint64_t)H * kSsdP * 2};  // bytes, dims 1 and 2
+  const cuuint32_t box[3] = {(cuuint32_t)kSsdP, 1u, (cuuint32_t)kSsdT};
+  const cuuint32_t estr[3] = {1u, 1u, 1u};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<__nv_bfloat16*>(x), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int N, bool NOISY>
-cudaError_t scan_t(const SsdScanParams& p, cudaStream_t s) {
-  const int64_t tiles = p.g.Bt * p.g.nb * p.g.m;
-  if (tiles == 0 || p.g.H == 0) return cudaSuccess;
-  if (p.hg < 1 || p.hg > kMaxHeadsPerCta) return cudaErrorInvalidValue;
-  const ScanSmem L(N, p.g.m);
+cudaError_t scan_t(const SsdScanParams& p_in, cudaStream_t s) {
+  const int64_t tiles = p_in.g.Bt * p_in.g.nb * p_in.g.m;
+  if (tiles == 0 || p_in.g.H == 0) return cudaSuccess;
+  if (p_in.hg < 1 || p_in.hg > kMaxHeadsPerCta) return cudaErrorInvalidValue;
+  const ScanSmem L(N, p_in.g.m);
   cudaError_t e = set_smem(k_ssd_block_scan<N, NOISY>, L.total);
   if (e != cudaSuccess) return e;
+  SsdScanParams p = p_in;
+  CUtensorMap xmap;
+  memset(&xmap, 0, sizeof(xmap));
+  // streams read right to left keep the cp.async path (a box cannot reverse rows)
+  p.tma = !p.rev && encode_x_map(&xmap, p.x, p.g.Bt * p.g.L, p.g.H) ? 1 : 0;
   const dim3 grid((unsigned)tiles, (unsigned)((p.g.H + p.hg - 1) / p.hg));
-  k_ssd_block_scan<N, NOISY><<<grid, kScanThreads, L.total, s>>>(p);
+  k_ssd_block_scan<N, NOISY><<<grid, kScanThreads, L.total, s>>>(p, xmap);
   return cudaGetLastError();
 }
 

@@ -60,6 +60,7 @@ struct SsdScanParams {
   int rev;            // 1: the stream is read right to left (as in SsdStateParams)
   float* y32;         // non-null: write the output in fp32 here instead of y
   const float* y32_add;  // non-null: add this fp32 array to the output before rounding to y
+  int tma;            // set by the launcher: x tiles and seeds arrive by TMA (left-to-right streams)
 };
 
 // Backward (ssd_bwd.cu). One stream and direction of the block-local
@@ -153,6 +154,7 @@ cudaError_t launch_ssd_block_state(const SsdStateParams& p, cudaStream_t s);
 cudaError_t launch_ssd_state_pass(const SsdPassParams& p, cudaStream_t s);
 cudaError_t launch_ssd_block_scan(bool noisy, const SsdScanParams& p, cudaStream_t s);
 int* ssd_wait_flag_ptr();  // device address of the wait flag (current device), or null
+bool ssd_tma_enabled();    // the tensor-map encoder is available (TMA operand loads)
 cudaError_t launch_ssd_wait_probe(uint32_t polls, cudaStream_t s);
 
 }  // namespace bds

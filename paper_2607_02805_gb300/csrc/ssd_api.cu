@@ -316,6 +316,8 @@ int bdscan_ssd_wait_flag(int reset) {
   return v;
 }
 
+int bdscan_ssd_tma_enabled(void) { return bds::ssd_tma_enabled() ? 1 : 0; }
+
 int bdscan_ssd_wait_selftest(uint32_t polls) {
   const char* fn = "bdscan_ssd_wait_selftest";
   bds::api_begin();

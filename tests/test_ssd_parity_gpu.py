@@ -178,3 +178,10 @@ def test_ssd_full_bidir_matches_oracle(cfg):
     args = [z[k] if k in z else wl.f64(k) for k in NAMES]
     _, y_ref, _ = ssd.forward(wl.len, *args)
     P.assert_close("y (full bidirectional)", to_numpy(y), y_ref, P.FWD_TOL, P.BF16_U)
+
+
+def test_operand_tiles_arrive_by_tma():
+    """On GB300 the left-to-right scans take their x tiles and seeds through
+    the tensor memory accelerator (the parity tests above then cover that
+    path); right-to-left streams keep cp.async."""
+    assert binding.bdscan_ssd_tma_enabled() == 1
