@@ -456,9 +456,13 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
   // one head's x tiles and raw seed into buffer xbuf: by TMA (thread 0; a
   // 128-token x tile is one box of the [tokens][heads][64] map, the seed one
   // contiguous run) when the launcher set up the map, else by cp.async
+  bool ld_pending = false;  // a TMA phase issued and not yet waited for
+  uint32_t ld_parity = 0;
   auto load_head = [&](int hd, uint32_t xbuf) {
     const float* seed_h = has_seed ? seed_src + (int64_t)hd * kSsdP * N : nullptr;
     if (p.tma) {
+      ld_pending = true;
+      ld_parity = (uint32_t)((hd - h0) & 1);
       if (t == 0) {
         umma::fence_async_smem();  // the buffers' earlier generic accesses before the async writes
         bar_expect_tx(&bar[2], (uint32_t)ntile * 16384u + (seed_h != nullptr ? (uint32_t)(kSsdP * N * 4) : 0u));
@@ -597,6 +601,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
         alive = false;
         break;
       }
+      ld_pending = false;
     } else {
       cp_async_wait_all();
     }
@@ -703,6 +708,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     umma::fence_after_sync();
   }
   cp_async_wait_all();
+  if (ld_pending) umma::bar_wait(&bar[2], ld_parity);  // after a give-up: the copies in flight, bounded
   umma::fence_before_sync();
   __syncthreads();
   if (t < 32) tmem_dealloc(tm, 512);
@@ -799,7 +805,7 @@ bool ssd_tma_enabled() { return tensor_map_encoder() != nullptr; }
 
 // x [rows][H][64] bf16 as a 3-D map with boxes of 64 channels x 1 head x 128
 // tokens, 128-byte swizzle (the layout the MMA descriptors read).
-bool encode_x_map(CUtensorMap* m, const __nv_bfloat16* x, int64_t rows, int H) {
+bool encode_head_map(CUtensorMap* m, const __nv_bfloat16* x, int64_t rows, int H) {
   PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
   if (enc == nullptr || rows >= ((int64_t)1 << 31) || ((uintptr_t)x & 15u) != 0) return false;
   const cuuint64_t dims[3] = {(cuuint64_t)kSsdP, (cuuint64_t)H, (cuuint64_t)rows};
@@ -823,7 +829,7 @@ cudaError_t scan_t(const SsdScanParams& p_in, cudaStream_t s) {
   CUtensorMap xmap;
   memset(&xmap, 0, sizeof(xmap));
   // streams read right to left keep the cp.async path (a box cannot reverse rows)
-  p.tma = !p.rev && encode_x_map(&xmap, p.x, p.g.Bt * p.g.L, p.g.H) ? 1 : 0;
+  p.tma = !p.rev && encode_head_map(&xmap, p.x, p.g.Bt * p.g.L, p.g.H) ? 1 : 0;
   const dim3 grid((unsigned)tiles, (unsigned)((p.g.H + p.hg - 1) / p.hg));
   k_ssd_block_scan<N, NOISY><<<grid, kScanThreads, L.total, s>>>(p, xmap);
   return cudaGetLastError();

@@ -3,6 +3,7 @@
 // documented in include/bdscan_ssd.h.
 #pragma once
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -86,6 +87,7 @@ struct SsdBwdTileParams {
   float* dS_part;       // [Bt*nb][H][m][P][N] (seeded direction)
   int hg;               // heads per CTA (at most 16); groups = ceil(H / hg)
   int* flag;
+  int tma;              // set by the launcher: x and dy tiles arrive by TMA
 };
 
 // The dt and A gradients of one stream and direction from the row and column
@@ -155,6 +157,9 @@ cudaError_t launch_ssd_state_pass(const SsdPassParams& p, cudaStream_t s);
 cudaError_t launch_ssd_block_scan(bool noisy, const SsdScanParams& p, cudaStream_t s);
 int* ssd_wait_flag_ptr();  // device address of the wait flag (current device), or null
 bool ssd_tma_enabled();    // the tensor-map encoder is available (TMA operand loads)
+// A [rows][H][64] bf16 tensor (x, dy) as a 3-D tensor map with boxes of 64
+// channels x 1 head x 128 tokens and 128-byte swizzle; false if unavailable.
+bool encode_head_map(CUtensorMap* m, const __nv_bfloat16* base, int64_t rows, int H);
 cudaError_t launch_ssd_wait_probe(uint32_t polls, cudaStream_t s);
 
 }  // namespace bds

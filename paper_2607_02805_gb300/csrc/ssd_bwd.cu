@@ -23,6 +23,8 @@
 // k_ssd_bwd_vec (dt, A gradients from the row and column sums), k_ssd_bwd_pass
 // (reverse state pass), k_ssd_bwd_state (tcgen05: the block-state transpose),
 // and fixed-order combines in ssd_api.cu's launch sequence.
+#include <cstring>
+
 #include "device.cuh"
 #include "params.h"
 #include "ssd.cuh"
@@ -138,10 +140,12 @@ constexpr int kMaxBwdHeads = 16;  // heads per tile CTA
 // dB_j (and the seed products) at 0; Q, then dx_j at 128; the head sum of dG
 // at 256; dC at 384.
 template <int N, bool UPPER, bool SEED>
-__global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTileParams p) {
+__global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTileParams p,
+                                                                  const __grid_constant__ CUtensorMap xmap,
+                                                                  const __grid_constant__ CUtensorMap dymap) {
   extern __shared__ unsigned char smraw[];
   unsigned char* sm = align1024(smraw);
-  __shared__ uint64_t bar;
+  __shared__ uint64_t bar, bar_ld;  // MMAs; a head's x and dy tiles (TMA)
   __shared__ uint32_t tslot;
   using S = TileSmem;
   constexpr int NT = kTileThreads;
@@ -185,15 +189,18 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     for (int q = tid & 31; q < Bs; q += 32) s_dtv[hh * 256 + q] = __bfloat162float(p.dt[(tok0 + q) * H + h]);
     warp_scan_dt<UPPER>(p.dt + tok0 * H + h, H, Bs, s_cv + hh * 256);
   }
-  if (tid == 0) umma::bar_init(&bar, 1);
+  if (tid == 0) {
+    umma::bar_init(&bar, 1);
+    umma::bar_init(&bar_ld, 1);
+  }
   if (w == 0) tmem_alloc(&tslot, 512);
   umma::fence_before_sync();
   __syncthreads();
   umma::fence_after_sync();
   const uint32_t tm = tslot, lane_base = tm + ((uint32_t)(32 * (w & 3)) << 16);
   const int tt = i * kSsdT + t;
-  uint32_t phase = 0;
-  bool alive = true;
+  uint32_t phase = 0, ldphase = 0;
+  bool alive = true, ld_pending = false;  // a TMA phase issued and not yet waited for
   const uint32_t y0 = umma::smem_u32(sm + S::DY), c0 = umma::smem_u32(sm + S::C), x0 = umma::smem_u32(sm + S::X),
                  b0 = umma::smem_u32(sm + S::BT), m0 = umma::smem_u32(sm + S::M);
   constexpr uint32_t id_gq = umma::idesc_bf16(128, 128, false, false);
@@ -211,10 +218,24 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     const int64_t sr0 = tok0 + (int64_t)j * kSsdT;
     // x and dy of head hh are staged after head hh-1's dx products (head 0's
     // with B_j): the copies run during the previous head's epilogue
+    // (by TMA, thread 0, when the launcher set up the maps; a missing dy is
+    // zero-filled by the threads)
     auto stage_head = [&](int hh) {
       const int h = h0 + hh;
-      stage_bf16<NT>(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
-      stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+      if (p.tma) {
+        if (tid == 0) {
+          umma::fence_async_smem();  // earlier generic accesses of X and DY before the async writes
+          bar_expect_tx(&bar_ld, p.dy != nullptr ? 32768u : 16384u);
+          tma_load_3d(sm + S::X, &xmap, 0, h, (int)sr0, &bar_ld);
+          if (p.dy != nullptr) tma_load_3d(sm + S::DY, &dymap, 0, h, (int)(tok0 + i * kSsdT), &bar_ld);
+        }
+        ld_pending = true;
+        if (p.dy == nullptr) stage_bf16<NT>(sm + S::DY, nullptr, HP, 128, 64);
+      } else {
+        stage_bf16<NT>(sm + S::X, p.x + (sr0 * H + h) * kSsdP, HP, 128, 64);
+        stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128,
+                       64);
+      }
     };
     stage_bf16<NT>(sm + S::BT, p.B + sr0 * N, N, 128, N);
     stage_head(0);
@@ -245,7 +266,16 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
         s_cf[tid] = cf;
         s_cfd[tid] = __fmul_rn(cf, s_dtv[hh * 256 + tid]);
       }
-      cp_async_wait_all();
+      if (p.tma) {  // every staged head completes one phase of the load barrier
+        if (!cta_wait(&bar_ld, ldphase, p.flag)) {
+          alive = false;
+          break;
+        }
+        ldphase ^= 1u;
+        ld_pending = false;
+      } else {
+        cp_async_wait_all();
+      }
       umma::fence_async_smem();
       umma::fence_before_sync();
       __syncthreads();
@@ -540,6 +570,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     }
   }
   cp_async_wait_all();
+  if (ld_pending) umma::bar_wait(&bar_ld, ldphase);  // after a give-up: the copies in flight, bounded
   umma::fence_before_sync();
   __syncthreads();
   if (w == 0) tmem_dealloc(tm, 512);
@@ -1010,12 +1041,20 @@ __global__ void __launch_bounds__(128) k_ssd_bwd_par(const SsdGeo g, const float
 }
 
 template <int N, bool UPPER, bool SEED>
-cudaError_t bwd_tile_t(const SsdBwdTileParams& p, cudaStream_t s) {
+cudaError_t bwd_tile_t(const SsdBwdTileParams& p_in, cudaStream_t s) {
   const int smem = (int)TileSmem::total;
   cudaError_t e = set_smem_cached((const void*)k_ssd_bwd_tile<N, UPPER, SEED>, smem, -1);
   if (e != cudaSuccess) return e;
+  SsdBwdTileParams p = p_in;
+  CUtensorMap xmap, dymap;
+  memset(&xmap, 0, sizeof(xmap));
+  memset(&dymap, 0, sizeof(dymap));
+  const int64_t rows = p.g.Bt * p.g.L;
+  p.tma = encode_head_map(&xmap, p.x, rows, p.g.H) && (p.dy == nullptr || encode_head_map(&dymap, p.dy, rows, p.g.H))
+              ? 1
+              : 0;
   dim3 grid((unsigned)(p.g.Bt * p.g.nb * p.g.m), (unsigned)((p.g.H + p.hg - 1) / p.hg));
-  k_ssd_bwd_tile<N, UPPER, SEED><<<grid, kTileThreads, smem, s>>>(p);
+  k_ssd_bwd_tile<N, UPPER, SEED><<<grid, kTileThreads, smem, s>>>(p, xmap, dymap);
   return cudaGetLastError();
 }
 
