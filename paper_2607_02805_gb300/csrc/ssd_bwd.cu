@@ -487,22 +487,47 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
 
   if (alive && SEED && k > 0) {
     // seed products per head: dC += (E o dy) S, the row dot dy_t . E_t (C_t S^T)
-    // and the seed gradient (E o dy)^T C; the seed as bf16 high and low parts
+    // and the seed gradient (E o dy)^T C; the seed as bf16 high and low parts.
+    // With TMA the next head's dy tile (DY and X alternate) and raw seed (into
+    // COL, free here) arrive under the current head's MMAs and epilogue.
     constexpr uint32_t id_cs = umma::idesc_bf16(128, 64, false, false);
+    const float* seeds = p.states + (b * g.nb + k - 1) * H * (int64_t)kSsdP * N;  // head h at h * 64 N
+    auto seed_loads = [&](int hh) {
+      if (tid == 0) {
+        umma::fence_async_smem();  // earlier generic accesses of the buffers before the async writes
+        bar_expect_tx(&bar_ld, (p.dy != nullptr ? 16384u : 0u) + (uint32_t)(kSsdP * N * 4));
+        if (p.dy != nullptr)
+          tma_load_3d(sm + ((hh & 1) ? S::X : S::DY), &dymap, 0, h0 + hh, (int)(tok0 + i * kSsdT), &bar_ld);
+        bulk_load(sm + S::COL, seeds + (int64_t)(h0 + hh) * kSsdP * N, (uint32_t)(kSsdP * N * 4), &bar_ld);
+      }
+      ld_pending = true;
+    };
+    if (p.tma) seed_loads(0);
     for (int hh = 0; hh < hg && alive; ++hh) {
       const int h = h0 + hh;
-      stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
-      cp_async_commit();
-      const float* seed = p.states + ((b * g.nb + k - 1) * H + h) * (int64_t)kSsdP * N;
-      stage_f32_hilo<NT, 64, N>(sm + S::M, sm + S::M + 16384u, seed);
-      cp_async_wait_all();
+      const uint32_t dyo = (p.tma && (hh & 1)) ? S::X : S::DY;  // this head's dy tile
+      if (p.tma) {
+        if (p.dy == nullptr) stage_bf16<NT>(sm + dyo, nullptr, HP, 128, 64);
+        if (!cta_wait(&bar_ld, ldphase, p.flag)) {
+          alive = false;
+          break;
+        }
+        ldphase ^= 1u;
+        ld_pending = false;
+        stage_f32_hilo<NT, 64, N>(sm + S::M, sm + S::M + 16384u, reinterpret_cast<const float*>(sm + S::COL));
+      } else {
+        stage_bf16<NT>(sm + S::DY, p.dy != nullptr ? p.dy + ((tok0 + i * kSsdT) * H + h) * kSsdP : nullptr, HP, 128, 64);
+        cp_async_commit();
+        stage_f32_hilo<NT, 64, N>(sm + S::M, sm + S::M + 16384u, seeds + (int64_t)h * kSsdP * N);
+        cp_async_wait_all();
+      }
       __syncthreads();
       // the seeded direction is the forward one: s_cv holds prefix sums
       const float E = ex2(__fmul_rn(__fmul_rn(p.A[h], kLog2e), s_cv[hh * 256 + tt]));
 #pragma unroll
       for (int cq = 0; cq < 4; ++cq) {  // 16-byte chunks 4 half .. 4 half + 3 of row t
         const int ch = 4 * half + cq;
-        const uint4 u = *reinterpret_cast<const uint4*>(sm + S::DY + sw128((uint32_t)t, (uint32_t)ch));
+        const uint4 u = *reinterpret_cast<const uint4*>(sm + dyo + sw128((uint32_t)t, (uint32_t)ch));
         const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&u);
         uint32_t o[4];
 #pragma unroll
@@ -535,11 +560,21 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
                          id_dx, kk > 0);
         umma::mma_commit(&bar);
       }
+      if (p.tma && hh + 1 < hg) seed_loads(hh + 1);  // COL and the other dy buffer are free
       if (!(alive = wait_mma())) break;
-      float v[32], rowdot = 0.f;  // channels 32 half .. 32 half + 31 of the row dot
+      float v[32], rowdot = 0.f;  // channels 32 half .. 32 half + 31 of the row dot, in order
       umma::tmem_ld32(lane_base + 32u * (uint32_t)half, v);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) rowdot = __fmaf_rn(tile_at(sm + S::DY, t, 32 * half + e), v[e], rowdot);
+      for (int cq = 0; cq < 4; ++cq) {
+        const uint4 u = *reinterpret_cast<const uint4*>(sm + dyo + sw128((uint32_t)t, (uint32_t)(4 * half + cq)));
+        const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(v2[e]);
+          rowdot = __fmaf_rn(f.x, v[8 * cq + 2 * e], rowdot);
+          rowdot = __fmaf_rn(f.y, v[8 * cq + 2 * e + 1], rowdot);
+        }
+      }
       s_dots[hh * 128 + t] = __fmul_rn(E, rowdot);
       if (32 * (w & 3) < N) {  // row n = t of dS^T, channels 32 half ..: the seed gradient partial [p][n]
         float* dso = p.dS_part + ((bk * H + h) * m + i) * (int64_t)kSsdP * N + t;
@@ -548,7 +583,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
         for (int e = 0; e < 32; ++e) dso[(int64_t)(32 * half + e) * N] = v[e];
       }
       umma::fence_before_sync();
-      __syncthreads();  // DY, BT and M are restaged for the next head
+      __syncthreads();  // BT, M and this head's dy buffer are restaged for the next heads
     }
   }
   if (alive) {  // dC of row t of tile i, summed over the group's heads, N/2 columns per half
