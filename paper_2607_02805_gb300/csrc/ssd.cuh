@@ -98,9 +98,10 @@ struct SsdBwdVecParams {
   const float* A;
   const float *col_part, *rowsum, *rowdot;  // rowdot null: zero
   int upper;
-  float* ddt;    // [Bt][L][H]
-  float* dA;     // [Bt*nb][H]
-  float* sumdt;  // [Bt*nb][H] or null: the block's sum of dt
+  float* ddt;                // [Bt][L][H] fp32, used when ddt_out is null
+  __nv_bfloat16* ddt_out;    // [Bt][L][H] or null: the stream's final dt gradient (no other term adds to it)
+  float* dA;                 // [Bt*nb][H]
+  float* sumdt;              // [Bt*nb][H] or null: the block's sum of dt
 };
 
 // Reverse pass over the clean stream's block-end states: gS_k = dstates_k +
@@ -123,10 +124,11 @@ struct SsdBwdStateParams {
   const float* gS;      // [Bt][nb][H][P][N]
   const float* states;  // [Bt][nb][H][P][N]
   const float* sumdt;   // [Bt*nb][H]
-  float* dx_state;      // [Bt*nb][H][Bs][P]
-  float* dB_state;      // [Bt*nb][H][Bs][N]
-  float* ddt;           // [Bt][L][H]
-  float* dA;            // [Bt*nb][H]
+  float* dx_state;          // [Bt*nb][H][Bs][P]
+  float* dB_state;          // [Bt*nb][H][Bs][N]
+  const float* ddt_tile;    // [Bt][L][H] the tile side of the clean dt gradient
+  __nv_bfloat16* ddt;       // [Bt][L][H] output: ddt_tile + this kernel's terms
+  float* dA;                // [Bt*nb][H]
   int* flag;
 };
 
@@ -143,8 +145,6 @@ cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, co
                                const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
                                __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s);
-cudaError_t launch_ssd_bwd_ddt(int64_t n, const float* vc, const float* vs, const float* vf, const float* vr,
-                               __nv_bfloat16* dc, __nv_bfloat16* df, __nv_bfloat16* dr, cudaStream_t s);
 // two launches: per-block sums of dy x, then the per-head sums (the first
 // launch is counted here, the second by the caller)
 cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,

@@ -391,7 +391,7 @@ namespace {
 // the state gradients, the clean block-state terms and the dD partials.
 struct SsdBwdWs {
   size_t dxp[3], dBp[3], dCp[3], colp[3], rows[3], rowdot[3], dSp[3], ddtv[3], dAv[3];
-  size_t sumdt, gS, dxs, dBs, ddts, dAs, dd, total;
+  size_t sumdt, gS, dxs, dBs, dAs, dd, total;
   int hg, ngrp;  // heads per tile CTA, head groups
 };
 // Head groups of the tile kernel: enough CTAs for about 1024 (several waves
@@ -426,14 +426,13 @@ SsdBwdWs ssd_bwd_ws(const bds::SsdGeo& g) {
     w.rows[s] = take(bkh * Bs);
     w.rowdot[s] = s < 2 ? take(bkh * Bs) : 0;
     w.dSp[s] = s < 2 ? take(bkh * m * P * N) : 0;
-    w.ddtv[s] = take((size_t)g.Bt * g.L * g.H);
+    w.ddtv[s] = s == 0 ? take((size_t)g.Bt * g.L * g.H) : 0;  // the noisy directions write their outputs
     w.dAv[s] = take(bkh);
   }
   w.sumdt = take(bkh);
   w.gS = take(bkh * P * N);
   w.dxs = take(bkh * Bs * P);
   w.dBs = take(bkh * Bs * N);
-  w.ddts = take((size_t)g.Bt * g.L * g.H);
   w.dAs = take(bkh);
   w.dd = take(bkh * 2);
   w.total = o;
@@ -545,7 +544,8 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
     v.rowsum = F(w.rows[st]);
     v.rowdot = st < 2 ? F(w.rowdot[st]) : nullptr;
     v.upper = st == 2;
-    v.ddt = F(w.ddtv[st]);
+    v.ddt = st == 0 ? F(w.ddtv[0]) : nullptr;
+    v.ddt_out = st == 1 ? (bf*)gnoisy->ddt_f : st == 2 ? (bf*)gnoisy->ddt_r : nullptr;
     v.dA = F(w.dAv[st]);
     v.sumdt = st == 0 ? F(w.sumdt) : nullptr;
     e = bds::api_launched(bds::launch_ssd_bwd_vec(v, s), s);
@@ -577,7 +577,8 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
     r.sumdt = F(w.sumdt);
     r.dx_state = F(w.dxs);
     r.dB_state = F(w.dBs);
-    r.ddt = F(w.ddts);
+    r.ddt_tile = F(w.ddtv[0]);
+    r.ddt = (bf*)gclean->ddt;
     r.dA = F(w.dAs);
     r.flag = flag;
     e = bds::api_launched(bds::launch_ssd_bwd_state(r, s), s);
@@ -592,11 +593,6 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
                                                   F(w.dBp[2]), F(w.dCp[2]), (bf*)gclean->dB, (bf*)gclean->dC,
                                                   (bf*)gnoisy->dB_f, (bf*)gnoisy->dC_f, (bf*)gnoisy->dB_r,
                                                   (bf*)gnoisy->dC_r, s),
-                          s);
-  if (e == cudaSuccess)
-    e = bds::api_launched(bds::launch_ssd_bwd_ddt(g.Bt * g.L * g.H, F(w.ddtv[0]), F(w.ddts), F(w.ddtv[1]),
-                                                  F(w.ddtv[2]), (bf*)gclean->ddt, (bf*)gnoisy->ddt_f,
-                                                  (bf*)gnoisy->ddt_r, s),
                           s);
   if (e == cudaSuccess)
     e = bds::api_launched(bds::launch_ssd_bwd_params(g, xs[0], dys[0], xs[1], dys[1], F(w.dd), F(w.dAv[0]),

@@ -649,7 +649,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 // rowdot_t), ddt_r = colsum'_r + sum of dc over the tokens whose cumulative dt
 // includes dt_r (t >= r forward, t <= r reverse), dA = sum_t c_t (dc_t / A).
 __global__ void __launch_bounds__(128) k_ssd_bwd_vec(const SsdBwdVecParams p) {
-  __shared__ float s_c[4][256], s_q[4][256];
+  __shared__ float s_c[4][256], s_q[4][256], s_col[4][256];
   const SsdGeo& g = p.g;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, Bs = (int)g.Bs, m = g.m, H = g.H;
   const int64_t u = (int64_t)blockIdx.x * 4 + w;
@@ -673,14 +673,20 @@ __global__ void __launch_bounds__(128) k_ssd_bwd_vec(const SsdBwdVecParams p) {
     if (p.rowdot != nullptr) q = __fadd_rn(q, p.rowdot[(bk * H + h) * Bs + s]);
     dA = __fmaf_rn(s_c[w][s], q, dA);
     s_q[w][s] = __fmul_rn(A, q);
-    p.ddt[(tok0 + s) * H + h] = col;
+    s_col[w][s] = col;
   }
   __syncwarp();
   if (p.upper)
     warp_scan_f32<false>(s_q[w], Bs);  // reverse: c_t sums dt over r >= t, so dt_r feeds every t <= r
   else
     warp_scan_f32<true>(s_q[w], Bs);   // forward: dt_r feeds every t >= r
-  for (int s = lane; s < Bs; s += 32) p.ddt[(tok0 + s) * H + h] = __fadd_rn(p.ddt[(tok0 + s) * H + h], s_q[w][s]);
+  for (int s = lane; s < Bs; s += 32) {
+    const float v = __fadd_rn(s_col[w][s], s_q[w][s]);
+    if (p.ddt_out != nullptr)
+      p.ddt_out[(tok0 + s) * H + h] = __float2bfloat16_rn(v);
+    else
+      p.ddt[(tok0 + s) * H + h] = v;
+  }
   dA = warp_sum(dA);
   if (lane == 0) p.dA[bk * H + h] = dA;
 }
@@ -742,7 +748,7 @@ __global__ void __launch_bounds__(256) k_ssd_bwd_pass(const SsdBwdPassParams p) 
 // B of one s-tile, per-token vectors of the block.
 struct StateBwdSmem {
   static constexpr uint32_t GH = 0, GL = 16384, X = 32768, BT = 49152, VEC = 81920;
-  static constexpr uint32_t TR = VEC + 5u * 256u * 4u;  // per-warp 32 x 32 fp32 transposition blocks
+  static constexpr uint32_t TR = VEC + 6u * 256u * 4u;  // per-warp 32 x 32 fp32 transposition blocks
   static constexpr uint32_t total = TR + 4u * 4096u + 1024u;
 };
 
@@ -789,8 +795,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
   float* s_w = s_dt + 256;
   float* s_dw = s_w + 256;
   float* s_e = s_dw + 256;
+  float* s_vt = s_e + 256;  // the tile side of the dt gradient, added at the end
   const float* gS = p.gS + (bk * H + h) * PN;
-  for (int s = t; s < Bs; s += kBwdThreads) s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
+  for (int s = t; s < Bs; s += kBwdThreads) {
+    cp_async4(s_vt + s, p.ddt_tile + (tok0 + s) * H + h);  // completes with the first tile's staging
+    s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
+  }
   if (w == 0) warp_scan_dt<true>(p.dt + tok0 * H + h, H, Bs, s_suf);
   // gS as bf16 high and low parts, and the block decay's da = sum over (p, n)
   // of gS o S_{k-1}: the loads of both matrices are issued first
@@ -920,7 +930,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
     const float blk = __fmul_rn(__fmul_rn(A, ak), da);  // block decay exp(A sumdt) of S_{k-1}
     for (int r = lane; r < Bs; r += 32) {
       const float before = r > 0 ? s_suf[r - 1] : 0.f;  // exclusive: s < r
-      p.ddt[(tok0 + r) * H + h] = __fadd_rn(__fadd_rn(__fmul_rn(s_e[r], s_dw[r]), before), blk);
+      const float vs = __fadd_rn(__fadd_rn(__fmul_rn(s_e[r], s_dw[r]), before), blk);
+      const int64_t o = (tok0 + r) * H + h;
+      p.ddt[o] = __float2bfloat16_rn(__fadd_rn(s_vt[r], vs));
     }
     dA = warp_sum(dA);
     if (lane == 0) p.dA[bk * H + h] = __fadd_rn(dA, __fmul_rn(__fmul_rn(sd, ak), da));
@@ -935,42 +947,62 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
 
 namespace {
 
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+  return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z), __fadd_rn(a.w, b.w));
+}
+__device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 bf4(const __nv_bfloat16* p) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+  const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+  return make_float4(a.x, a.y, b.x, b.y);
+}
+__device__ __forceinline__ void st_bf4(__nv_bfloat16* p, float4 v) {
+  const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  *reinterpret_cast<uint2*>(p) = make_uint2(*reinterpret_cast<const uint32_t*>(&a), *reinterpret_cast<const uint32_t*>(&b));
+}
+
 // dx of both streams: the tile partials of every tile that reaches s (tiles
 // i >= j(s) forward, i <= j(s) reverse), the clean state term and the skip
-// terms. One CTA row (blockIdx.x) per token, threads over (head, channel).
+// terms. One thread per (token, head, 4 channels).
 __global__ void __launch_bounds__(256) k_ssd_bwd_dx(const SsdGeo g, const float* dxp_c, const float* dxs,
                                                     const float* dxp_f, const float* dxp_r, const __nv_bfloat16* dyc,
                                                     const __nv_bfloat16* dyn, const float* Df, const float* Dr,
                                                     __nv_bfloat16* dxc, __nv_bfloat16* dxn) {
-  const int hp = blockIdx.y * 256 + threadIdx.x;
-  if (hp >= g.H * kSsdP) return;
-  const int h = hp / kSsdP, pp = hp - h * kSsdP;
-  const int64_t bt = blockIdx.x, b = bt / g.L;
+  constexpr int Q = kSsdP / 4;  // 4-channel groups per head
+  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (i >= g.Bt * g.L * g.H * Q) return;
+  const int64_t bt = i / (g.H * Q);
+  const int hq = (int)(i - bt * g.H * Q), h = hq / Q, pp = (hq - h * Q) * 4;
+  const int64_t b = bt / g.L;
   const int tl = (int)(bt - b * g.L), k = tl / (int)g.Bs, s = tl - k * (int)g.Bs, j = s / kSsdT, m = g.m;
-  const int64_t hb = (b * g.nb + k) * g.H + h, idx = bt * g.H * kSsdP + hp;
+  const int64_t hb = (b * g.nb + k) * g.H + h, idx = (bt * g.H + h) * kSsdP + pp;
   const int64_t stride_i = (int64_t)g.Bs * kSsdP;  // between the tile partials of one head
-  const float* pc = dxp_c + (hb * m * g.Bs + s) * kSsdP + pp;
-  const float* pf = dxp_f + (hb * m * g.Bs + s) * kSsdP + pp;
-  const float* pr = dxp_r + (hb * m * g.Bs + s) * kSsdP + pp;
-  // m is 1 or 2: every load is issued before the sums (in the order i = j..m-1
-  // forward, 0..j reverse)
+  const int64_t po = (hb * m * g.Bs + s) * kSsdP + pp;
+  // m is 1 or 2: every load is issued before the sums (in the order
+  // i = j..m-1 forward, 0..j reverse); a slab that does not reach s is read
+  // and dropped, which keeps the loads independent of j
   const bool two = m > 1;
-  const float c0 = pc[0], f0 = pf[0], r0 = pr[0];
-  const float c1 = two ? pc[stride_i] : 0.f, f1 = two ? pf[stride_i] : 0.f, r1 = two ? pr[stride_i] : 0.f;
-  const float st = dxs[(hb * g.Bs + s) * kSsdP + pp];
-  const float yc = dyc != nullptr ? __bfloat162float(dyc[idx]) : 0.f, yn = __bfloat162float(dyn[idx]);
-  float c = j == 0 ? c0 : 0.f, n = j == 0 ? f0 : 0.f;
+  const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  const float4 c0 = ld4(dxp_c + po), f0 = ld4(dxp_f + po), r0 = ld4(dxp_r + po);
+  const float4 c1 = two ? ld4(dxp_c + po + stride_i) : z, f1 = two ? ld4(dxp_f + po + stride_i) : z,
+               r1 = two ? ld4(dxp_r + po + stride_i) : z;
+  const float4 st = ld4(dxs + (hb * g.Bs + s) * kSsdP + pp);
+  const float4 yc = dyc != nullptr ? bf4(dyc + idx) : z, yn = bf4(dyn + idx);
+  float4 c = j == 0 ? c0 : z, n = j == 0 ? f0 : z;
   if (two) {
-    c = j == 0 ? __fadd_rn(c, c1) : c1;
-    n = j == 0 ? __fadd_rn(n, f1) : f1;
+    c = j == 0 ? add4(c, c1) : c1;
+    n = j == 0 ? add4(n, f1) : f1;
   }
-  c = __fadd_rn(c, st);
-  if (dyc != nullptr) c = __fmaf_rn(Df[h], yc, c);
-  n = __fadd_rn(n, r0);
-  if (j == 1) n = __fadd_rn(n, r1);
-  n = __fmaf_rn(__fadd_rn(Df[h], Dr[h]), yn, n);
-  dxc[idx] = __float2bfloat16_rn(c);
-  dxn[idx] = __float2bfloat16_rn(n);
+  c = add4(c, st);
+  const float dc = Df[h], dn = __fadd_rn(Df[h], Dr[h]);
+  if (dyc != nullptr)
+    c = make_float4(__fmaf_rn(dc, yc.x, c.x), __fmaf_rn(dc, yc.y, c.y), __fmaf_rn(dc, yc.z, c.z), __fmaf_rn(dc, yc.w, c.w));
+  n = add4(n, r0);
+  if (j == 1) n = add4(n, r1);
+  n = make_float4(__fmaf_rn(dn, yn.x, n.x), __fmaf_rn(dn, yn.y, n.y), __fmaf_rn(dn, yn.z, n.z), __fmaf_rn(dn, yn.w, n.w));
+  st_bf4(dxc + idx, c);
+  st_bf4(dxn + idx, n);
 }
 
 // dB and dC of the three streams: the tile partials of every head group (and
@@ -1019,60 +1051,103 @@ __global__ void __launch_bounds__(128) k_ssd_bwd_dbc(const SsdGeo g, int ngrp, c
   dCr[idx] = __float2bfloat16_rn(cr);
 }
 
-__global__ void __launch_bounds__(256) k_ssd_bwd_ddt(int64_t n, const float* vc, const float* vs, const float* vf,
-                                                     const float* vr, __nv_bfloat16* dc, __nv_bfloat16* df,
-                                                     __nv_bfloat16* dr) {
-  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
-  if (i >= n) return;
-  dc[i] = __float2bfloat16_rn(__fadd_rn(vc[i], vs[i]));
-  df[i] = __float2bfloat16_rn(vf[i]);
-  dr[i] = __float2bfloat16_rn(vr[i]);
+// sum of dy x over 8 bf16 pairs of two 16-byte vectors, added to acc in order
+__device__ __forceinline__ float dot8(uint4 a, uint4 b, float acc) {
+  const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
+  const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 u = __bfloat1622float2(pa[e]), v = __bfloat1622float2(pb[e]);
+    acc = __fmaf_rn(u.x, v.x, acc);
+    acc = __fmaf_rn(u.y, v.y, acc);
+  }
+  return acc;
 }
 
-// Per (batch row, block, head): sum of dy x of each stream (the skip terms' gradients).
+// Per (batch row, block, head): sum of dy x of each stream (the skip terms'
+// gradients). Two items per CTA, item = (row * nb + block) * H + head, so
+// that neighbouring warps read neighbouring heads of the same tokens; the
+// four warps of an item take a quarter of its tokens each, and lane l reads
+// the 16-byte vector l % 8 of the tokens l / 8, l / 8 + 4, ..., four
+// tokens' loads at a time. The quarters are added in order. CLEAN: the
+// clean stream has a dy.
+template <bool CLEAN>
 __global__ void __launch_bounds__(256) k_ssd_bwd_dd(const SsdGeo g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
                                                     const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* part) {
-  __shared__ float red[2][8];
-  const int64_t bk = blockIdx.x, b = bk / g.nb, k = bk % g.nb;
-  const int h = blockIdx.y, t = threadIdx.x;
+  __shared__ float red[2][4][2];
+  const int half = threadIdx.x >> 7, wq = (threadIdx.x >> 5) & 3, lane = threadIdx.x & 31;
+  const int64_t item = (int64_t)blockIdx.x * 2 + half;
+  const bool valid = item < g.Bt * g.nb * g.H;
   float sc = 0.f, sn = 0.f;
-  for (int64_t q = t; q < g.Bs * kSsdP; q += 256) {
-    const int64_t o = ((b * g.L + k * g.Bs + q / kSsdP) * g.H + h) * kSsdP + q % kSsdP;
-    if (dyc != nullptr) sc = __fmaf_rn(__bfloat162float(dyc[o]), __bfloat162float(xc[o]), sc);
-    sn = __fmaf_rn(__bfloat162float(dyn[o]), __bfloat162float(xn[o]), sn);
+  if (valid) {
+    const int64_t bk = item / g.H, b = bk / g.nb, k = bk % g.nb;
+    const int h = (int)(item % g.H);
+    const int64_t rs = (int64_t)g.H * kSsdP;  // between tokens
+    const int qt = (int)(g.Bs / 4);             // tokens per quarter, a multiple of 16
+    const int64_t o0 = ((b * g.L + k * g.Bs + wq * qt + (lane >> 3)) * g.H + h) * kSsdP + (lane & 7) * 8;
+    for (int j0 = 0; j0 < qt; j0 += 16) {
+      uint4 an[4], bn[4], ac[4], bc[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int64_t o = o0 + (int64_t)(j0 + 4 * u) * rs;
+        an[u] = __ldg(reinterpret_cast<const uint4*>(dyn + o));
+        bn[u] = __ldg(reinterpret_cast<const uint4*>(xn + o));
+        if (CLEAN) {
+          ac[u] = __ldg(reinterpret_cast<const uint4*>(dyc + o));
+          bc[u] = __ldg(reinterpret_cast<const uint4*>(xc + o));
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        sn = dot8(an[u], bn[u], sn);
+        if (CLEAN) sc = dot8(ac[u], bc[u], sc);
+      }
+    }
   }
   sc = warp_sum(sc);
   sn = warp_sum(sn);
-  if ((t & 31) == 0) {
-    red[0][t >> 5] = sc;
-    red[1][t >> 5] = sn;
+  if (lane == 0) {
+    red[half][wq][0] = sc;
+    red[half][wq][1] = sn;
   }
   __syncthreads();
-  if (t < 2) {
-    float v = 0.f;
-    for (int q = 0; q < 8; ++q) v = __fadd_rn(v, red[t][q]);
-    part[(bk * g.H + h) * 2 + t] = v;
-  }
+  if (valid && wq == 0 && lane < 2)
+    part[item * 2 + lane] = __fadd_rn(__fadd_rn(__fadd_rn(red[half][0][lane], red[half][1][lane]), red[half][2][lane]),
+                                      red[half][3][lane]);
 }
 
-// Parameter gradients per head, summing the (batch row, block) partials in order.
-__global__ void __launch_bounds__(128) k_ssd_bwd_par(const SsdGeo g, const float* dA_c, const float* dA_f,
+// Parameter gradients per head: one CTA per head; thread t sums the (batch
+// row, block) partials t, t + 256, ... in order, then a fixed tree over the
+// threads, so the result does not depend on scheduling.
+__global__ void __launch_bounds__(256) k_ssd_bwd_par(const SsdGeo g, const float* dA_c, const float* dA_f,
                                                      const float* dA_s, const float* dA_r, const float* dd, float* dAf,
                                                      float* dDf, float* dAr, float* dDr) {
-  const int h = blockIdx.x * 128 + threadIdx.x;
-  if (h >= g.H) return;
+  __shared__ float4 red[256];
+  const int h = blockIdx.x, t = threadIdx.x;
   float af = 0.f, ar = 0.f, df = 0.f, dr = 0.f;
-  for (int64_t bk = 0; bk < g.Bt * g.nb; ++bk) {
+  for (int64_t bk = t; bk < g.Bt * g.nb; bk += 256) {
     const int64_t o = bk * g.H + h;
     af = __fadd_rn(af, __fadd_rn(__fadd_rn(dA_c[o], dA_f[o]), dA_s[o]));
     ar = __fadd_rn(ar, dA_r[o]);
     df = __fadd_rn(df, __fadd_rn(dd[o * 2], dd[o * 2 + 1]));
     dr = __fadd_rn(dr, dd[o * 2 + 1]);
   }
-  dAf[h] = af;
-  dAr[h] = ar;
-  dDf[h] = df;
-  dDr[h] = dr;
+  red[t] = make_float4(af, ar, df, dr);
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (t < w) {
+      const float4 u = red[t], v = red[t + w];
+      red[t] = make_float4(__fadd_rn(u.x, v.x), __fadd_rn(u.y, v.y), __fadd_rn(u.z, v.z), __fadd_rn(u.w, v.w));
+    }
+    __syncthreads();
+  }
+  if (t == 0) {
+    const float4 r = red[0];
+    dAf[h] = r.x;
+    dAr[h] = r.y;
+    dDf[h] = r.z;
+    dDr[h] = r.w;
+  }
 }
 
 template <int N, bool UPPER, bool SEED>
@@ -1133,8 +1208,9 @@ cudaError_t launch_ssd_bwd_state(const SsdBwdStateParams& p, cudaStream_t s) {
 cudaError_t launch_ssd_bwd_dx(const SsdGeo& g, const float* dxp_c, const float* dxs, const float* dxp_f,
                               const float* dxp_r, const __nv_bfloat16* dyc, const __nv_bfloat16* dyn, const float* Df,
                               const float* Dr, __nv_bfloat16* dxc, __nv_bfloat16* dxn, cudaStream_t s) {
-  const dim3 grid((unsigned)(g.Bt * g.L), (unsigned)((g.H * kSsdP + 255) / 256));
-  k_ssd_bwd_dx<<<grid, 256, 0, s>>>(g, dxp_c, dxs, dxp_f, dxp_r, dyc, dyn, Df, Dr, dxc, dxn);
+  const int64_t n = g.Bt * g.L * g.H * (kSsdP / 4);
+  if (n == 0) return cudaSuccess;
+  k_ssd_bwd_dx<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, dxp_c, dxs, dxp_f, dxp_r, dyc, dyn, Df, Dr, dxc, dxn);
   return cudaGetLastError();
 }
 
@@ -1147,20 +1223,20 @@ cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, co
   return cudaGetLastError();
 }
 
-cudaError_t launch_ssd_bwd_ddt(int64_t n, const float* vc, const float* vs, const float* vf, const float* vr,
-                               __nv_bfloat16* dc, __nv_bfloat16* df, __nv_bfloat16* dr, cudaStream_t s) {
-  k_ssd_bwd_ddt<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(n, vc, vs, vf, vr, dc, df, dr);
-  return cudaGetLastError();
-}
-
 cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
                                   const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* dd, const float* dA_c,
                                   const float* dA_f, const float* dA_s, const float* dA_r, float* dAf, float* dDf,
                                   float* dAr, float* dDr, cudaStream_t s) {
-  k_ssd_bwd_dd<<<dim3((unsigned)(g.Bt * g.nb), (unsigned)g.H), 256, 0, s>>>(g, xc, dyc, xn, dyn, dd);
-  cudaError_t e = api_launched(cudaGetLastError(), s);
-  if (e != cudaSuccess) return e;
-  k_ssd_bwd_par<<<(unsigned)((g.H + 127) / 128), 128, 0, s>>>(g, dA_c, dA_f, dA_s, dA_r, dd, dAf, dDf, dAr, dDr);
+  const int64_t items = g.Bt * g.nb * g.H;
+  if (items > 0) {
+    if (dyc != nullptr)
+      k_ssd_bwd_dd<true><<<(unsigned)((items + 1) / 2), 256, 0, s>>>(g, xc, dyc, xn, dyn, dd);
+    else
+      k_ssd_bwd_dd<false><<<(unsigned)((items + 1) / 2), 256, 0, s>>>(g, xc, dyc, xn, dyn, dd);
+    cudaError_t e = api_launched(cudaGetLastError(), s);
+    if (e != cudaSuccess) return e;
+  }
+  k_ssd_bwd_par<<<(unsigned)g.H, 256, 0, s>>>(g, dA_c, dA_f, dA_s, dA_r, dd, dAf, dDf, dAr, dDr);
   return cudaGetLastError();
 }
 
