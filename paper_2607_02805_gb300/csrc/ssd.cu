@@ -427,10 +427,25 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       s_prm[48 + t] = p.Dr[h0 + t];
     }
   }
-  for (int e = t; e < Bs * hg; e += kScanThreads) {  // dt of the CTA's heads, bf16 as stored
-    const int s = e / hg, hh = e - s * hg;
-    s_dtf[s * hg + hh] = p.dtf[tok(s) * H + h0 + hh];
-    if (NOISY) s_dtr[s * hg + hh] = p.dtr[tok(s) * H + h0 + hh];
+  {  // dt of the CTA's heads, bf16 as stored (Bs hg <= 256 * 16): every load issued before the stores
+    __nv_bfloat16 vf[kMaxHeadsPerCta], vr[kMaxHeadsPerCta];
+    const int ne = Bs * hg;
+#pragma unroll
+    for (int q = 0; q < kMaxHeadsPerCta; ++q) {
+      const int e = t + q * kScanThreads, s = e / hg, hh = e - s * hg;
+      if (e < ne) {
+        vf[q] = p.dtf[tok(s) * H + h0 + hh];
+        if (NOISY) vr[q] = p.dtr[tok(s) * H + h0 + hh];
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kMaxHeadsPerCta; ++q) {
+      const int e = t + q * kScanThreads;
+      if (e < ne) {
+        s_dtf[e] = vf[q];
+        if (NOISY) s_dtr[e] = vr[q];
+      }
+    }
   }
   if (t == 0) {
     umma::bar_init(&bar[0], 1);

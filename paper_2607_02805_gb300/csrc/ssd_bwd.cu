@@ -186,8 +186,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
   // CTA: warp w takes heads w, w + 8
   for (int hh = w; hh < hg; hh += NT / 32) {
     const int h = h0 + hh;
-    for (int q = tid & 31; q < Bs; q += 32) s_dtv[hh * 256 + q] = __bfloat162float(p.dt[(tok0 + q) * H + h]);
-    warp_scan_dt<UPPER>(p.dt + tok0 * H + h, H, Bs, s_cv + hh * 256);
+    warp_scan_dt<UPPER>(p.dt + tok0 * H + h, H, Bs, s_cv + hh * 256, s_dtv + hh * 256);
   }
   if (tid == 0) {
     umma::bar_init(&bar, 1);
@@ -797,11 +796,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
   float* s_e = s_dw + 256;
   float* s_vt = s_e + 256;  // the tile side of the dt gradient, added at the end
   const float* gS = p.gS + (bk * H + h) * PN;
-  for (int s = t; s < Bs; s += kBwdThreads) {
+  for (int s = t; s < Bs; s += kBwdThreads)
     cp_async4(s_vt + s, p.ddt_tile + (tok0 + s) * H + h);  // completes with the first tile's staging
-    s_dt[s] = __bfloat162float(p.dt[(tok0 + s) * H + h]);
-  }
-  if (w == 0) warp_scan_dt<true>(p.dt + tok0 * H + h, H, Bs, s_suf);
+  if (w == 0) warp_scan_dt<true>(p.dt + tok0 * H + h, H, Bs, s_suf, s_dt);
   // gS as bf16 high and low parts, and the block decay's da = sum over (p, n)
   // of gS o S_{k-1}: the loads of both matrices are issued first
   float da = 0.f;

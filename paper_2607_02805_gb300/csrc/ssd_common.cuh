@@ -51,9 +51,11 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 
 // Inclusive scan of dt over `n` tokens by one warp (n a multiple of 32):
 // lane l sums tokens [l*n/32, (l+1)*n/32) in order, then the lane totals are
-// scanned. REV = true scans from the last token (suffix sums).
+// scanned. REV = true scans from the last token (suffix sums). `raw`, if not
+// null, receives dt itself (fp32) at the same positions.
 template <bool REV>
-__device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t stride, int n, float* out) {
+__device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t stride, int n, float* out,
+                                              float* raw = nullptr) {
   const int lane = threadIdx.x & 31, per = n / 32;
   float loc[8];
   // all of the lane's loads are issued before the first add (n <= 256)
@@ -61,6 +63,13 @@ __device__ __forceinline__ float warp_scan_dt(const __nv_bfloat16* dt, int64_t s
   for (int q = 0; q < 8; ++q) {
     const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
     loc[q] = q < per ? __bfloat162float(dt[pos * stride]) : 0.f;
+  }
+  if (raw != nullptr) {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int pos = REV ? n - 1 - (lane * per + q) : lane * per + q;
+      if (q < per) raw[pos] = loc[q];
+    }
   }
   float s = 0.f;
 #pragma unroll
