@@ -182,10 +182,12 @@ __global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdS
       const uint32_t a0 = umma::smem_u32(sm + S.b), x0 = umma::smem_u32(sm + S.xs);
       constexpr uint32_t id = umma::idesc_bf16(128, 64, true, true);
       const uint32_t d = tm + 64u * (uint32_t)(hh & 1);
+      const uint64_t da = umma::sdesc(a0, half, 1024), dh = umma::sdesc(x0, 1024, 1024),
+                     dl = umma::sdesc(x0 + half, 1024, 1024);
       for (int kk = 0; kk < Bs / 16; ++kk) {
-        const uint64_t a = umma::sdesc(a0 + kk * 2048u, half, 1024);
-        umma::mma_bf16(d, a, umma::sdesc(x0 + kk * 2048u, 1024, 1024), id, kk > 0);
-        umma::mma_bf16(d, a, umma::sdesc(x0 + half + kk * 2048u, 1024, 1024), id, true);
+        const uint64_t a = umma::sdesc_adv(da, kk * 2048u);
+        umma::mma_bf16(d, a, umma::sdesc_adv(dh, kk * 2048u), id, kk > 0);
+        umma::mma_bf16(d, a, umma::sdesc_adv(dl, kk * 2048u), id, true);
       }
       umma::mma_commit(&bar[hh & 1]);
     }
@@ -253,10 +255,11 @@ __device__ __forceinline__ void stage_rows(unsigned char* dst, const __nv_bfloat
 template <int N>
 __device__ __forceinline__ void mma_gram(uint32_t d, uint32_t a, uint32_t b) {
   constexpr uint32_t id = umma::idesc_bf16(128, 128, false, false);
+  const uint64_t da = umma::sdesc(a, 16, 1024), db = umma::sdesc(b, 16, 1024);
 #pragma unroll
   for (int kk = 0; kk < N / 16; ++kk) {
     const uint32_t off = (kk >> 2) * kTile16 + (kk & 3) * 32u;
-    umma::mma_bf16(d, umma::sdesc(a + off, 16, 1024), umma::sdesc(b + off, 16, 1024), id, kk > 0);
+    umma::mma_bf16(d, umma::sdesc_adv(da, off), umma::sdesc_adv(db, off), id, kk > 0);
   }
 }
 
@@ -591,21 +594,24 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     const uint32_t base = umma::smem_u32(sm);
     if (seed_term) {  // C^f . seed^T into columns 448..511
       constexpr uint32_t id = umma::idesc_bf16(128, 64, false, false);
+      const uint64_t dc = umma::sdesc(base + L.cf, 16, 1024), dh = umma::sdesc(base + L.seed, 16, 1024),
+                     dl = umma::sdesc(base + L.seed + 128u * N, 16, 1024);
 #pragma unroll
       for (int kk = 0; kk < N / 16; ++kk) {
         const uint32_t offc = (kk >> 2) * kTile16 + (kk & 3) * 32u;
         const uint32_t offs = (kk >> 2) * 8192u + (kk & 3) * 32u;
-        const uint64_t a = umma::sdesc(base + L.cf + offc, 16, 1024);
-        umma::mma_bf16(tm + 448, a, umma::sdesc(base + L.seed + offs, 16, 1024), id, kk > 0);
-        umma::mma_bf16(tm + 448, a, umma::sdesc(base + L.seed + 128u * N + offs, 16, 1024), id, true);
+        const uint64_t a = umma::sdesc_adv(dc, offc);
+        umma::mma_bf16(tm + 448, a, umma::sdesc_adv(dh, offs), id, kk > 0);
+        umma::mma_bf16(tm + 448, a, umma::sdesc_adv(dl, offs), id, true);
       }
     }
-    const uint32_t ma = base + (j ? L.m1 : L.m0), xb = base + xcur + (uint32_t)j * 16384u;
+    const uint64_t dm = umma::sdesc(base + (j ? L.m1 : L.m0), 16, 1024),
+                   dx = umma::sdesc(base + xcur + (uint32_t)j * 16384u, 1024, 1024);
     constexpr uint32_t id = umma::idesc_bf16(128, 64, false, true);
 #pragma unroll
     for (int kk = 0; kk < 8; ++kk)
-      umma::mma_bf16(tm + 384, umma::sdesc(ma + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
-                     umma::sdesc(xb + kk * 2048u, 1024, 1024), id, j > 0 || kk > 0);
+      umma::mma_bf16(tm + 384, umma::sdesc_adv(dm, (kk >> 2) * kTile16 + (kk & 3) * 32u),
+                     umma::sdesc_adv(dx, kk * 2048u), id, j > 0 || kk > 0);
   };
   for (int hh = 0; hh < hg && alive; ++hh) {
     const int h = h0 + hh;

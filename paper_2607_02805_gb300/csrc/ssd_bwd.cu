@@ -245,10 +245,11 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     __syncthreads();
     if (tid == 0) {
       umma::fence_after_sync();
+      const uint64_t dc = umma::sdesc(c0, 16, 1024), db = umma::sdesc(b0, 16, 1024);
 #pragma unroll
       for (int kk = 0; kk < N / 16; ++kk) {  // G = C_i B_j^T, shared by the heads
         const uint32_t off = (uint32_t)(kk >> 2) * kTile16 + (uint32_t)(kk & 3) * 32u;
-        umma::mma_bf16(tm, umma::sdesc(c0 + off, 16, 1024), umma::sdesc(b0 + off, 16, 1024), id_gq, kk > 0);
+        umma::mma_bf16(tm, umma::sdesc_adv(dc, off), umma::sdesc_adv(db, off), id_gq, kk > 0);
       }
       umma::mma_commit(&bar);
     }
@@ -280,10 +281,10 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       __syncthreads();
       if (tid == 0) {
         umma::fence_after_sync();
+        const uint64_t dy = umma::sdesc(y0, 16, 1024), dx = umma::sdesc(x0, 16, 1024);
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)  // Q = dy_i x_j^T
-          umma::mma_bf16(tm + 128u, umma::sdesc(y0 + kk * 32u, 16, 1024), umma::sdesc(x0 + kk * 32u, 16, 1024),
-                         id_gq, kk > 0);
+          umma::mma_bf16(tm + 128u, umma::sdesc_adv(dy, kk * 32u), umma::sdesc_adv(dx, kk * 32u), id_gq, kk > 0);
         umma::mma_commit(&bar);
       }
       if (!(alive = wait_mma())) break;
@@ -393,10 +394,10 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       __syncthreads();
       if (tid == 0) {
         umma::fence_after_sync();
+        const uint64_t dm = umma::sdesc(m0, kTile16, 1024), dy = umma::sdesc(y0, kTile16, 1024);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)  // dx_j = M^T dy_i: M read as an MN-major operand (M = s, K = t)
-          umma::mma_bf16(tm + 128u, umma::sdesc(m0 + kk * 2048u, kTile16, 1024), umma::sdesc(y0 + kk * 2048u, kTile16, 1024),
-                         id_dx, kk > 0);
+          umma::mma_bf16(tm + 128u, umma::sdesc_adv(dm, kk * 2048u), umma::sdesc_adv(dy, kk * 2048u), id_dx, kk > 0);
         umma::mma_commit(&bar);
       }
       if (half == 1) s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);
@@ -455,18 +456,19 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
     __syncthreads();
     if (tid == 0) {
       umma::fence_after_sync();
+      const uint64_t db = umma::sdesc(b0, kTile16, 1024), dc = umma::sdesc(c0, kTile16, 1024);
 #pragma unroll
       for (int part = 0; part < 2; ++part) {
         const uint32_t dg0 = part ? x0 : m0;
+        const uint64_t dgk = umma::sdesc(dg0, 16, 1024), dgm = umma::sdesc(dg0, kTile16, 1024);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
           const uint32_t koff = (uint32_t)(kk >> 2) * kTile16 + (uint32_t)(kk & 3) * 32u, mn = (uint32_t)kk * 2048u;
           // dC += dG B_j: dG K-major [t][s], B_j MN-major [s][n]
-          umma::mma_bf16(tm + 384u, umma::sdesc(dg0 + koff, 16, 1024), umma::sdesc(b0 + mn, kTile16, 1024), id_dc,
+          umma::mma_bf16(tm + 384u, umma::sdesc_adv(dgk, koff), umma::sdesc_adv(db, mn), id_dc,
                          j != j0 || part > 0 || kk > 0);
           // dB_j = dG^T C_i: dG read as MN-major (M = s)
-          umma::mma_bf16(tm, umma::sdesc(dg0 + mn, kTile16, 1024), umma::sdesc(c0 + mn, kTile16, 1024), id_db,
-                         part > 0 || kk > 0);
+          umma::mma_bf16(tm, umma::sdesc_adv(dgm, mn), umma::sdesc_adv(dc, mn), id_db, part > 0 || kk > 0);
         }
       }
       umma::mma_commit(&bar);
@@ -541,22 +543,23 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       __syncthreads();
       if (tid == 0) {
         umma::fence_after_sync();
+        const uint64_t dbk = umma::sdesc(b0, 16, 1024), dck = umma::sdesc(c0, 16, 1024);
+        const uint64_t dbm = umma::sdesc(b0, kTile16, 1024), dcm = umma::sdesc(c0, kTile16, 1024);
 #pragma unroll
         for (int part = 0; part < 2; ++part) {
           const uint32_t s0 = m0 + (part ? 16384u : 0u);
+          const uint64_t dsm = umma::sdesc(s0, 8192, 1024), dsk = umma::sdesc(s0, 16, 1024);
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)  // dC += (E o dy) S: S MN-major [p][n], atom columns of 8 KB
-            umma::mma_bf16(tm + 384u, umma::sdesc(b0 + kk * 32u, 16, 1024), umma::sdesc(s0 + kk * 2048u, 8192, 1024),
-                           id_dc, true);
+            umma::mma_bf16(tm + 384u, umma::sdesc_adv(dbk, kk * 32u), umma::sdesc_adv(dsm, kk * 2048u), id_dc, true);
 #pragma unroll
           for (int kk = 0; kk < N / 16; ++kk)  // C S^T: S K-major [p][n]
-            umma::mma_bf16(tm, umma::sdesc(c0 + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
-                           umma::sdesc(s0 + (kk >> 2) * 8192u + (kk & 3) * 32u, 16, 1024), id_cs, part > 0 || kk > 0);
+            umma::mma_bf16(tm, umma::sdesc_adv(dck, (kk >> 2) * kTile16 + (kk & 3) * 32u),
+                           umma::sdesc_adv(dsk, (kk >> 2) * 8192u + (kk & 3) * 32u), id_cs, part > 0 || kk > 0);
         }
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)  // dS^T = C_i^T (E o dy): C read as MN-major (M = n)
-          umma::mma_bf16(tm + 64u, umma::sdesc(c0 + kk * 2048u, kTile16, 1024), umma::sdesc(b0 + kk * 2048u, kTile16, 1024),
-                         id_dx, kk > 0);
+          umma::mma_bf16(tm + 64u, umma::sdesc_adv(dcm, kk * 2048u), umma::sdesc_adv(dbm, kk * 2048u), id_dx, kk > 0);
         umma::mma_commit(&bar);
       }
       if (p.tma && hh + 1 < hg) seed_loads(hh + 1);  // COL and the other dy buffer are free
@@ -861,17 +864,19 @@ __global__ void __launch_bounds__(kBwdThreads, 1) k_ssd_bwd_state(const SsdBwdSt
     __syncthreads();
     if (t == 0) {
       umma::fence_after_sync();
+      const uint64_t db = umma::sdesc(b0, 16, 1024), dx = umma::sdesc(x0, 16, 1024);
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         const uint32_t gs0 = half ? gl : gh;
+        const uint64_t dgk = umma::sdesc(gs0, 16, 1024), dgm = umma::sdesc(gs0, 8192, 1024);
 #pragma unroll
         for (int kk = 0; kk < N / 16; ++kk)  // U = B_j gS^T: gS K-major [p][n]
-          umma::mma_bf16(tm, umma::sdesc(b0 + (kk >> 2) * kTile16 + (kk & 3) * 32u, 16, 1024),
-                         umma::sdesc(gs0 + (kk >> 2) * 8192u + (kk & 3) * 32u, 16, 1024), id_u, half > 0 || kk > 0);
+          umma::mma_bf16(tm, umma::sdesc_adv(db, (kk >> 2) * kTile16 + (kk & 3) * 32u),
+                         umma::sdesc_adv(dgk, (kk >> 2) * 8192u + (kk & 3) * 32u), id_u, half > 0 || kk > 0);
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)  // V = x_j gS: gS MN-major [p][n]
-          umma::mma_bf16(tm + 64u, umma::sdesc(x0 + kk * 32u, 16, 1024), umma::sdesc(gs0 + kk * 2048u, 8192, 1024),
-                         id_v, half > 0 || kk > 0);
+          umma::mma_bf16(tm + 64u, umma::sdesc_adv(dx, kk * 32u), umma::sdesc_adv(dgm, kk * 2048u), id_v,
+                         half > 0 || kk > 0);
       }
       umma::mma_commit(&bar);
     }

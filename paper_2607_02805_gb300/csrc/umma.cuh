@@ -36,6 +36,11 @@ __host__ __device__ constexpr uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint3
          ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
+// The descriptor d with its start address advanced by `bytes` (a multiple of
+// 16; the advanced address stays below 256 KB, so the 14-bit field does not
+// carry): one add in the MMA issue loops instead of rebuilding every field.
+__host__ __device__ constexpr uint64_t sdesc_adv(uint64_t d, uint32_t bytes) { return d + (uint64_t)(bytes >> 4); }
+
 // Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator (bits
 // 4-5 = 1), bf16 A and B (7-9 = 1, 10-12 = 1), A/B major (15, 16: 0 = K-major,
 // 1 = MN-major), N >> 3 (17-22), M >> 4 (24-28).
