@@ -675,8 +675,10 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     // this warp's 32 channels of its token row
     {
       float ya[32], yo[32];
-      umma::tmem_ld32(lane_base + 384u + 32u * hf, ya);
-      if (has_seed) umma::tmem_ld32(lane_base + 448u + 32u * hf, yo);
+      if (has_seed)
+        umma::tmem_ld32x2(lane_base + 384u + 32u * hf, ya, lane_base + 448u + 32u * hf, yo);
+      else
+        umma::tmem_ld32(lane_base + 384u + 32u * hf, ya);
       const float dec = has_seed ? ex2(v[tt]) : 0.f;
       const float Dd = NOISY ? __fadd_rn(s_prm[16 + hh], s_prm[48 + hh]) : s_prm[16 + hh];
       const int64_t off = (tok(tt) * H + h) * kSsdP + 32 * hf;

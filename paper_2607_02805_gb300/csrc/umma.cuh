@@ -99,8 +99,10 @@ __device__ __forceinline__ void fence_before_sync() { asm volatile("tcgen05.fenc
 
 // 32 consecutive fp32 columns of this thread's TMEM lane (warp w reads lanes
 // 32w..32w+31; `ta` carries the warp's lane base in bits 16-31).
-__device__ __forceinline__ void tmem_ld32(uint32_t ta, float (&v)[32]) {
-  uint32_t r[32];
+// 32 consecutive fp32 columns of this thread's TMEM lane, without the wait:
+// the registers are ready after tmem_ld_wait (on one of the loads issued
+// since the last wait) and tmem_ld_after (on each of the others).
+__device__ __forceinline__ void tmem_ld32_issue(uint32_t ta, uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
       "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n"
@@ -109,6 +111,9 @@ __device__ __forceinline__ void tmem_ld32(uint32_t ta, float (&v)[32]) {
         "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
         "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(ta));
+}
+// Waits for every TMEM load this thread issued; r's registers are used only after it.
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;\n"
                : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
                  "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
@@ -116,8 +121,37 @@ __device__ __forceinline__ void tmem_ld32(uint32_t ta, float (&v)[32]) {
                  "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
                  "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
                :);
+}
+// No instruction: orders the uses of r after the preceding tmem_ld_wait
+// (volatile statements keep their order), for a second load of the same wait.
+__device__ __forceinline__ void tmem_ld_after(uint32_t (&r)[32]) {
+  asm volatile(""
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :);
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t ta, float (&v)[32]) {
+  uint32_t r[32];
+  tmem_ld32_issue(ta, r);
+  tmem_ld_wait(r);
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+// Two loads under one wait.
+__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, float (&v)[32], uint32_t tb, float (&u)[32]) {
+  uint32_t r[32], q[32];
+  tmem_ld32_issue(ta, r);
+  tmem_ld32_issue(tb, q);
+  tmem_ld_wait(r);
+  tmem_ld_after(q);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    v[i] = __uint_as_float(r[i]);
+    u[i] = __uint_as_float(q[i]);
+  }
 }
 #endif  // __CUDACC__
 
