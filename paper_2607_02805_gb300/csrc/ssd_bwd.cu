@@ -106,13 +106,27 @@ __device__ __forceinline__ void tmem_st32(uint32_t ta, const float (&v)[32]) {
       "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])), "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])), "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])), "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])), "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])), "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])), "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31])));
 }
 
+// Barrier of the warp pair q, q + 4 of a k_ssd_bwd_tile CTA (the two column
+// halves of the same 32 token rows): named barrier 1 + q over 64 threads.
+__device__ __forceinline__ void pair_sync(int q) {
+  asm volatile("bar.sync %0, 64;\n" ::"r"(1 + q) : "memory");
+}
+
+// bf16 high parts bf16(v) and low parts bf16(v - bf16(v)) of a pair
+__device__ __forceinline__ void split_pair(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 hv = __floats2bfloat162_rn(a, b);
+  hi = *reinterpret_cast<const uint32_t*>(&hv);
+  lo = pack_bf16(__fsub_rn(a, __low2float(hv)), __fsub_rn(b, __high2float(hv)));
+}
+
 // Shared memory of k_ssd_bwd_tile (offsets from a 1024-aligned base).
 //   C    C of tile i, [128 t][128 n] (n >= N zero)    BT  B of s-tile j, [128 s][N]
 //   X    x of s-tile j, one head, [128 s][64 p]       DY  dy of tile i, one head, [128 t][64 p]
-//   M    one head's G o decay o dt, [128 t][128 s]
-//   COL  R' of 64 columns, [128][65] fp32
+//   M    one head's M' = G o decay, bf16 high part, [128 t][128 s]
+//   COL  its low part (same layout); after the head's D product, per-warp
+//        32 x 32 fp32 transposition blocks of the dx stores
 //   VEC  c and dt of the block for every head of the group, [2][16][256] fp32
-//   CP   column-sum partials of four row quarters, [4][64] fp32
+//   CP   the second column half's partial of the column sums, [128] fp32
 //   ROWS row sums per head of the group [16][128], row dots per column half [2][16][128]
 //   CF   the current head's column factors exp(A (c_ref - c_s)) and their products with dt_s
 // After a s-tile's heads, the head-summed dG goes to M (bf16 high part) and
@@ -133,11 +147,12 @@ constexpr int kMaxBwdHeads = 16;  // heads per tile CTA
 // takes columns 0..63 of every 128-column product, the second 64..127 (a
 // warp reaches the TMEM lanes 32 (warp mod 4) onward). Row s = t of s-tile j
 // is the column-side row. Per s-tile j the Gram tile G = C_i B_j^T is shared
-// by the group's heads; per head, Q = dy x^T, the masked decays, the column
-// sums of R', dx_j = M^T dy, and dG = Q o decay o dt summed over the heads in
-// fp32 in TMEM. dC and dB_j then take the head-summed dG once (B and C are
+// by the group's heads; per head, Q = dy x^T, the masked decays M' = G o
+// decay (bf16 high and low parts), D = M'^T dy (then dx_j = diag(dt) D and
+// the column sums of R' as x_s . D_s, since R'[t, s] = (dy_t . x_s)
+// M'[t, s]), and dG = Q o decay o dt summed over the heads in fp32 in TMEM. dC and dB_j then take the head-summed dG once (B and C are
 // shared by the heads), split into bf16 high and low parts. TMEM: G, then
-// dB_j (and the seed products) at 0; Q, then dx_j at 128; the head sum of dG
+// dB_j (and the seed products) at 0; Q, then D at 128; the head sum of dG
 // at 256; dC at 384.
 template <int N, bool UPPER, bool SEED>
 __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTileParams p,
@@ -301,7 +316,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
         umma::tmem_ld32(lane_base + 32u * (uint32_t)c, gv);
         umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)c, qv);
         if (hh > 0) umma::tmem_ld32(lane_base + 256u + 32u * (uint32_t)c, dgs);
-        uint32_t mp[16];
+        uint32_t mp[16], ml[16];  // M' as bf16 high and low parts, column pairs
         // the chunk's 32 columns against this warp's 32 rows: entirely inside
         // the direction's triangle (the decay factors into a row factor times
         // the column factors, both at most 1), the diagonal 32 x 32 block
@@ -319,17 +334,14 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
             const float2 cfd = *reinterpret_cast<const float2*>(s_cfd + s0 + e);
             const float2 g2 = make_float2(gv[e], gv[e + 1]), q2 = make_float2(qv[e], qv[e + 1]);
             const float2 L = mul2(rf2, cf), Ld = mul2(rf2, cfd);
-            const float2 rp = mul2(q2, mul2(g2, L));
-            s_col[t * 65 + 32 * half + e] = rp.x;  // row stride 65: scalar stores
-            s_col[t * 65 + 32 * half + e + 1] = rp.y;
             const float2 dg = mul2(q2, Ld);
             rs2 = fma2(g2, dg, rs2);
             const float2 old2 = make_float2(dgs[e], dgs[e + 1]);
             const float2 nd = hh > 0 ? add2(old2, dg) : dg;
             dgs[e] = nd.x;
             dgs[e + 1] = nd.y;
-            const float2 mv = mul2(g2, Ld);
-            mp[e >> 1] = pack_bf16(mv.x, mv.y);
+            const float2 mv = mul2(g2, L);
+            split_pair(mv.x, mv.y, mp[e >> 1], ml[e >> 1]);
           }
           rowsum = __fadd_rn(rowsum, __fadd_rn(rs2.x, rs2.y));
         } else if (mode == 2) {
@@ -343,22 +355,18 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
               const float L = valid ? ex2(__fmul_rn(A2, __fsub_rn(ct, s_c[s]))) : 0.f;
               const float ds = s_dt[s];
               const float gl = __fmul_rn(gv[e + q], L);
-              const float rp = __fmul_rn(qv[e + q], gl);
-              rowsum = __fmaf_rn(rp, ds, rowsum);
-              s_col[t * 65 + 32 * half + e + q] = rp;
+              rowsum = __fmaf_rn(__fmul_rn(qv[e + q], gl), ds, rowsum);
               const float dg = __fmul_rn(__fmul_rn(qv[e + q], L), ds);
               dgs[e + q] = hh > 0 ? __fadd_rn(dgs[e + q], dg) : dg;
-              mv[q] = __fmul_rn(gl, ds);
+              mv[q] = gl;
             }
-            mp[e >> 1] = pack_bf16(mv[0], mv[1]);
+            split_pair(mv[0], mv[1], mp[e >> 1], ml[e >> 1]);
           }
         } else {
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
-            s_col[t * 65 + 32 * half + e] = 0.f;
-            s_col[t * 65 + 32 * half + e + 1] = 0.f;
             if (hh == 0) dgs[e] = dgs[e + 1] = 0.f;
-            mp[e >> 1] = 0u;
+            mp[e >> 1] = ml[e >> 1] = 0u;
           }
         }
         tmem_st32(lane_base + 256u + 32u * (uint32_t)c, dgs);
@@ -367,24 +375,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
           const int chunk = 4 * c + u;
           const uint32_t off = (uint32_t)(chunk >> 3) * kTile16 + sw128((uint32_t)t, (uint32_t)(chunk & 7));
           *reinterpret_cast<uint4*>(sm + S::M + off) = make_uint4(mp[4 * u], mp[4 * u + 1], mp[4 * u + 2], mp[4 * u + 3]);
-        }
-        // column sums of R' over the tile's 128 rows: four row quarters of 32
-        // (four interleaved sums each), then the quarters in order
-        __syncthreads();
-        {
-          const int col = tid & 63, qr = tid >> 6;
-          float a[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-          for (int rr = 0; rr < 32; rr += 4)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) a[q] = __fadd_rn(a[q], s_col[(32 * qr + rr + q) * 65 + col]);
-          s_cp[qr * 64 + col] = __fadd_rn(__fadd_rn(a[0], a[1]), __fadd_rn(a[2], a[3]));
-        }
-        __syncthreads();
-        if (tid < 64) {  // s_col column cc is tile column 32 (2 (cc / 32) + r) + cc % 32
-          const float sum = __fadd_rn(__fadd_rn(s_cp[tid], s_cp[64 + tid]), __fadd_rn(s_cp[128 + tid], s_cp[192 + tid]));
-          const int tc = 32 * (2 * (tid >> 5) + r) + (tid & 31);
-          p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + tc] = sum;
+          *reinterpret_cast<uint4*>(sm + S::COL + off) = make_uint4(ml[4 * u], ml[4 * u + 1], ml[4 * u + 2], ml[4 * u + 3]);
         }
       }
       if (half == 0) s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);  // the second half after the barrier
@@ -394,24 +385,49 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       __syncthreads();
       if (tid == 0) {
         umma::fence_after_sync();
-        const uint64_t dm = umma::sdesc(m0, kTile16, 1024), dy = umma::sdesc(y0, kTile16, 1024);
+        const uint64_t dy = umma::sdesc(y0, kTile16, 1024);
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk)  // dx_j = M^T dy_i: M read as an MN-major operand (M = s, K = t)
-          umma::mma_bf16(tm + 128u, umma::sdesc_adv(dm, kk * 2048u), umma::sdesc_adv(dy, kk * 2048u), id_dx, kk > 0);
+        for (int part = 0; part < 2; ++part) {  // D = M'^T dy_i: M' read as an MN-major operand (M = s, K = t)
+          const uint64_t dm = umma::sdesc(part ? umma::smem_u32(sm + S::COL) : m0, kTile16, 1024);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            umma::mma_bf16(tm + 128u, umma::sdesc_adv(dm, kk * 2048u), umma::sdesc_adv(dy, kk * 2048u), id_dx,
+                           part > 0 || kk > 0);
+        }
         umma::mma_commit(&bar);
       }
       if (half == 1) s_rows[hh * 128 + t] = __fadd_rn(s_rows[hh * 128 + t], rowsum);
       if (!(alive = wait_mma())) break;
-      if (hh + 1 < hg) {  // X and DY are free: the next head's copies start now
-        stage_head(hh + 1);
-        cp_async_commit();
-      }
-      {  // head h's dx contribution from tile i, rows j*128 + 32 (w mod 4) .. of
-         // channels 32 half ..: the warp's 32 x 32 block is transposed through
-         // COL (float pairs, XOR-swizzled by row) so that each store writes
-         // two 128-byte row segments
+      {  // row s = j*128 + t of D, channels 32 half ..: the column sum of R'
+         // is x_s . D_s, this half's 32 channels in order and then the two
+         // halves; head h's dx contribution from tile i is dt_s D_s
         float v[32];
         umma::tmem_ld32(lane_base + 128u + 32u * (uint32_t)half, v);
+        float cs = 0.f;
+#pragma unroll
+        for (int cq = 0; cq < 4; ++cq) {
+          const uint4 u = *reinterpret_cast<const uint4*>(sm + S::X + sw128((uint32_t)t, (uint32_t)(4 * half + cq)));
+          const __nv_bfloat162* x2 = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(x2[e]);
+            cs = __fmaf_rn(f.x, v[8 * cq + 2 * e], cs);
+            cs = __fmaf_rn(f.y, v[8 * cq + 2 * e + 1], cs);
+          }
+        }
+        if (half == 1) s_cp[t] = cs;
+        pair_sync(w & 3);  // warps w and w + 4 hold the two halves of the same rows
+        if (half == 0) p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + t] = __fadd_rn(cs, s_cp[t]);
+        if (hh + 1 < hg) {  // X and DY are free: the next head's copies start now
+          stage_head(hh + 1);
+          cp_async_commit();
+        }
+        const float ds = s_dtv[hh * 256 + j * kSsdT + t];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) v[e] = __fmul_rn(ds, v[e]);
+        // the warp's 32 x 32 block is transposed through COL (float pairs,
+        // XOR-swizzled by row) so that each store writes two 128-byte row
+        // segments
         float* tb = s_col + w * 1024;
         const int r = tid & 31;
 #pragma unroll
