@@ -92,11 +92,26 @@ __device__ __forceinline__ float tile_at(const unsigned char* tile, int row, int
   return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(tile + off));
 }
 
-__device__ __forceinline__ void store_row(float* dst, const float (&v)[32]) {
+// Stores a warp's 32 x 32 fp32 block (lane r holds row r in v) to rows
+// dst + r * ld (16-byte aligned, ld a multiple of 4), through a warp-private
+// buffer tb of 1024 floats (16-byte chunks XOR-swizzled by row), so that each
+// store instruction writes four 128-byte row segments.
+__device__ __forceinline__ void store_block32(float* dst, int64_t ld, const float (&v)[32], float* tb) {
+  const int r = threadIdx.x & 31;
 #pragma unroll
-  for (int e = 0; e < 32; e += 4) *reinterpret_cast<float4*>(dst + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
+  for (int c4 = 0; c4 < 8; ++c4)
+    *reinterpret_cast<float4*>(tb + r * 32 + 4 * (c4 ^ (r & 7))) =
+        make_float4(v[4 * c4], v[4 * c4 + 1], v[4 * c4 + 2], v[4 * c4 + 3]);
+  __syncwarp();
+  const int c4 = r & 7;
+#pragma unroll
+  for (int rr = 0; rr < 32; rr += 4) {
+    const int row = rr + (r >> 3);
+    *reinterpret_cast<float4*>(dst + row * ld + 4 * c4) =
+        *reinterpret_cast<const float4*>(tb + row * 32 + 4 * (c4 ^ (row & 7)));
+  }
+  __syncwarp();
 }
-
 // 32 consecutive fp32 columns of this thread's TMEM lane, written (the
 // counterpart of umma::tmem_ld32); tmem_wait_st() orders them before later loads.
 __device__ __forceinline__ void tmem_st32(uint32_t ta, const float (&v)[32]) {
@@ -425,23 +440,9 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
         const float ds = s_dtv[hh * 256 + j * kSsdT + t];
 #pragma unroll
         for (int e = 0; e < 32; ++e) v[e] = __fmul_rn(ds, v[e]);
-        // the warp's 32 x 32 block is transposed through COL (float pairs,
-        // XOR-swizzled by row) so that each store writes two 128-byte row
-        // segments
-        float* tb = s_col + w * 1024;
-        const int r = tid & 31;
-#pragma unroll
-        for (int c2 = 0; c2 < 16; ++c2)
-          *reinterpret_cast<float2*>(tb + r * 32 + 2 * (c2 ^ (r & 15))) = make_float2(v[2 * c2], v[2 * c2 + 1]);
-        __syncwarp();
-        const int c2 = r & 15;
-        float* dxo = p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + 32 * (w & 3)) * kSsdP + 32 * half + 2 * c2;
-#pragma unroll 4
-        for (int rr = 0; rr < 32; rr += 2) {
-          const int row = rr + (r >> 4);
-          *reinterpret_cast<float2*>(dxo + row * kSsdP) =
-              *reinterpret_cast<const float2*>(tb + row * 32 + 2 * (c2 ^ (row & 15)));
-        }
+        // the warp's 32 x 32 block goes out through COL (free after the D product)
+        store_block32(p.dx_part + (((bk * H + h) * m + i) * Bs + j * kSsdT + 32 * (w & 3)) * kSsdP + 32 * half, kSsdP,
+                      v, s_col + w * 1024);
       }
       umma::fence_before_sync();
     }
@@ -490,13 +491,14 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       umma::mma_commit(&bar);
     }
     if (!(alive = wait_mma())) break;
-    {  // row s = j*128 + t of the group's dB contribution from tile i, N/2 columns per half
+    {  // rows s = j*128 + 32 (w mod 4) .. of the group's dB contribution from
+       // tile i, N/2 columns per half, through the warp's block of COL
       float v[32];
-      float* dbo = p.dB_part + (((bk * ngrp + grp) * m + i) * Bs + j * kSsdT + t) * N;
+      float* dbo = p.dB_part + (((bk * ngrp + grp) * m + i) * Bs + j * kSsdT + 32 * (w & 3)) * N;
 #pragma unroll
       for (int q = half * (N / 64); q < (half + 1) * (N / 64); ++q) {
         umma::tmem_ld32(lane_base + 32u * (uint32_t)q, v);
-        store_row(dbo + 32 * q, v);
+        store_block32(dbo + 32 * q, N, v, s_col + w * 1024);
       }
     }
     umma::fence_before_sync();
@@ -519,6 +521,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       }
       ld_pending = true;
     };
+    __syncthreads();  // the last dB stores went through COL
     if (p.tma) seed_loads(0);
     for (int hh = 0; hh < hg && alive; ++hh) {
       const int h = h0 + hh;
@@ -604,13 +607,13 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
       __syncthreads();  // BT, M and this head's dy buffer are restaged for the next heads
     }
   }
-  if (alive) {  // dC of row t of tile i, summed over the group's heads, N/2 columns per half
+  if (alive) {  // dC of rows 32 (w mod 4) .. of tile i, summed over the group's heads, N/2 columns per half
     float v[32];
-    float* dco = p.dC_part + ((bk * ngrp + grp) * Bs + tt) * N;
+    float* dco = p.dC_part + ((bk * ngrp + grp) * Bs + i * kSsdT + 32 * (w & 3)) * N;
 #pragma unroll
     for (int q = half * (N / 64); q < (half + 1) * (N / 64); ++q) {
       umma::tmem_ld32(lane_base + 384u + 32u * (uint32_t)q, v);
-      store_row(dco + 32 * q, v);
+      store_block32(dco + 32 * q, N, v, s_col + w * 1024);
     }
   }
   __syncthreads();  // both halves' row sums and dots are in shared memory
@@ -769,24 +772,6 @@ struct StateBwdSmem {
   static constexpr uint32_t TR = VEC + 6u * 256u * 4u;  // per-warp 32 x 32 fp32 transposition blocks
   static constexpr uint32_t total = TR + 4u * 4096u + 1024u;
 };
-
-// Stores a warp's 32 x 32 fp32 block (lane r holds row r in v) to rows
-// dst + r * ld, through a warp-private XOR-swizzled buffer `tb` so that each
-// store instruction writes two 128-byte row segments.
-__device__ __forceinline__ void store_block32(float* dst, int64_t ld, const float (&v)[32], float* tb) {
-  const int r = threadIdx.x & 31;
-#pragma unroll
-  for (int c2 = 0; c2 < 16; ++c2)
-    *reinterpret_cast<float2*>(tb + r * 32 + 2 * (c2 ^ (r & 15))) = make_float2(v[2 * c2], v[2 * c2 + 1]);
-  __syncwarp();
-  const int c2 = r & 15;
-#pragma unroll 4
-  for (int rr = 0; rr < 32; rr += 2) {
-    const int row = rr + (r >> 4);
-    *reinterpret_cast<float2*>(dst + row * ld + 2 * c2) = *reinterpret_cast<const float2*>(tb + row * 32 + 2 * (c2 ^ (row & 15)));
-  }
-  __syncwarp();
-}
 
 // One CTA of 4 warps per (batch row, block, head) of the clean stream, with
 // gS = the gradient of the state after the block: U = B gS^T and V = x gS per
