@@ -591,7 +591,7 @@ def run_ssd(args):
 
 
 SSD_BWD_KERNELS = ("bwd_tile_clean", "bwd_tile_fwd", "bwd_tile_rev", "bwd_vec_clean", "bwd_vec_fwd", "bwd_vec_rev",
-                   "bwd_state_pass", "bwd_block_state", "bwd_dx", "bwd_dbc", "bwd_dd", "bwd_par")
+                   "bwd_state_pass", "bwd_block_state", "bwd_dx", "bwd_dbc", "bwd_par")
 
 
 def ssd_bwd_head_groups(Bt, L, Bs, H):

@@ -85,6 +85,7 @@ struct SsdBwdTileParams {
   float* rowsum;        // [Bt*nb][H][Bs]
   float* rowdot;        // [Bt*nb][H][Bs] (seeded direction)
   float* dS_part;       // [Bt*nb][H][m][P][N] (seeded direction)
+  float* dd_part;       // [Bt*nb][H][m][8] or null: per warp, sum of dy . x over its rows of tile i
   int hg;               // heads per CTA (at most 16); groups = ceil(H / hg)
   int* flag;
   int tma;              // set by the launcher: x and dy tiles arrive by TMA
@@ -145,10 +146,10 @@ cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, co
                                const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
                                __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s);
-// two launches: per-block sums of dy x, then the per-head sums (the first
-// launch is counted here, the second by the caller)
-cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
-                                  const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* dd, const float* dA_c,
+// per-head sums of the partials: dA of both directions (clean, seeded,
+// state and reverse terms), dD from the dy . x partials of both streams
+// ([Bt*nb][H][m][8] each, from the tile kernels)
+cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const float* dd_c, const float* dd_n, const float* dA_c,
                                   const float* dA_f, const float* dA_s, const float* dA_r, float* dAf, float* dDf,
                                   float* dAr, float* dDr, cudaStream_t s);
 

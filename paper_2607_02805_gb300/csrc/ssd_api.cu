@@ -434,7 +434,7 @@ SsdBwdWs ssd_bwd_ws(const bds::SsdGeo& g) {
   w.dxs = take(bkh * Bs * P);
   w.dBs = take(bkh * Bs * N);
   w.dAs = take(bkh);
-  w.dd = take(bkh * 2);
+  w.dd = take(bkh * m * 8 * 2);  // dy . x partials of the clean, then the noisy stream
   w.total = o;
   return w;
 }
@@ -529,6 +529,7 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
     p.rowsum = F(w.rows[st]);
     p.rowdot = st < 2 ? F(w.rowdot[st]) : nullptr;
     p.dS_part = st < 2 ? F(w.dSp[st]) : nullptr;
+    p.dd_part = st < 2 ? F(w.dd) + (size_t)st * g.Bt * g.nb * g.H * g.m * 8 : nullptr;
     p.hg = w.hg;
     p.flag = flag;
     e = bds::api_launched(bds::launch_ssd_bwd_tile(st == 2, st < 2, p, s), s);
@@ -595,8 +596,8 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
                                                   (bf*)gnoisy->dC_r, s),
                           s);
   if (e == cudaSuccess)
-    e = bds::api_launched(bds::launch_ssd_bwd_params(g, xs[0], dys[0], xs[1], dys[1], F(w.dd), F(w.dAv[0]),
-                                                     F(w.dAv[1]), F(w.dAs), F(w.dAv[2]), gparams->dA_f,
+    e = bds::api_launched(bds::launch_ssd_bwd_params(g, F(w.dd), F(w.dd) + (size_t)g.Bt * g.nb * g.H * g.m * 8,
+                                                     F(w.dAv[0]), F(w.dAv[1]), F(w.dAs), F(w.dAv[2]), gparams->dA_f,
                                                      gparams->dD_f, gparams->dA_r, gparams->dD_r, s),
                           s);
   if (e != cudaSuccess) return cuda_fail(e, fn);

@@ -121,6 +121,12 @@ __device__ __forceinline__ void tmem_st32(uint32_t ta, const float (&v)[32]) {
       "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])), "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])), "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])), "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])), "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])), "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])), "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31])));
 }
 
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
 // Barrier of the warp pair q, q + 4 of a k_ssd_bwd_tile CTA (the two column
 // halves of the same 32 token rows): named barrier 1 + q over 64 threads.
 __device__ __forceinline__ void pair_sync(int q) {
@@ -430,6 +436,25 @@ __global__ void __launch_bounds__(kTileThreads, 1) k_ssd_bwd_tile(const SsdBwdTi
             cs = __fmaf_rn(f.y, v[8 * cq + 2 * e + 1], cs);
           }
         }
+        if (p.dd_part != nullptr && j == i) {  // x and dy tiles of the same tokens: the skip term's dy . x
+          float dd = 0.f;
+#pragma unroll
+          for (int cq = 0; cq < 4; ++cq) {
+            const uint32_t off = sw128((uint32_t)t, (uint32_t)(4 * half + cq));
+            const uint4 ux = *reinterpret_cast<const uint4*>(sm + S::X + off);
+            const uint4 uy = *reinterpret_cast<const uint4*>(sm + S::DY + off);
+            const __nv_bfloat162* x2 = reinterpret_cast<const __nv_bfloat162*>(&ux);
+            const __nv_bfloat162* y2 = reinterpret_cast<const __nv_bfloat162*>(&uy);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 fx = __bfloat1622float2(x2[e]), fy = __bfloat1622float2(y2[e]);
+              dd = __fmaf_rn(fy.x, fx.x, dd);
+              dd = __fmaf_rn(fy.y, fx.y, dd);
+            }
+          }
+          dd = warp_sum(dd);
+          if ((tid & 31) == 0) p.dd_part[((bk * H + h) * m + i) * 8 + w] = dd;
+        }
         if (half == 1) s_cp[t] = cs;
         pair_sync(w & 3);  // warps w and w + 4 hold the two halves of the same rows
         if (half == 0) p.col_part[((bk * H + h) * m + i) * Bs + j * kSsdT + t] = __fadd_rn(cs, s_cp[t]);
@@ -660,11 +685,6 @@ __device__ __forceinline__ void warp_scan_f32(float* a, int n) {
   __syncwarp();
 }
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
 
 // One warp per (batch row, block, head): dc_t = A (rowsum_t - dt_t colsum'_t +
 // rowdot_t), ddt_r = colsum'_r + sum of dc over the tokens whose cumulative dt
@@ -1054,86 +1074,28 @@ __global__ void __launch_bounds__(128) k_ssd_bwd_dbc(const SsdGeo g, int ngrp, c
   dCr[idx] = __float2bfloat16_rn(cr);
 }
 
-// sum of dy x over 8 bf16 pairs of two 16-byte vectors, added to acc in order
-__device__ __forceinline__ float dot8(uint4 a, uint4 b, float acc) {
-  const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
-  const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const float2 u = __bfloat1622float2(pa[e]), v = __bfloat1622float2(pb[e]);
-    acc = __fmaf_rn(u.x, v.x, acc);
-    acc = __fmaf_rn(u.y, v.y, acc);
-  }
-  return acc;
-}
-
-// Per (batch row, block, head): sum of dy x of each stream (the skip terms'
-// gradients). Two items per CTA, item = (row * nb + block) * H + head, so
-// that neighbouring warps read neighbouring heads of the same tokens; the
-// four warps of an item take a quarter of its tokens each, and lane l reads
-// the 16-byte vector l % 8 of the tokens l / 8, l / 8 + 4, ..., four
-// tokens' loads at a time. The quarters are added in order. CLEAN: the
-// clean stream has a dy.
-template <bool CLEAN>
-__global__ void __launch_bounds__(256) k_ssd_bwd_dd(const SsdGeo g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
-                                                    const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* part) {
-  __shared__ float red[2][4][2];
-  const int half = threadIdx.x >> 7, wq = (threadIdx.x >> 5) & 3, lane = threadIdx.x & 31;
-  const int64_t item = (int64_t)blockIdx.x * 2 + half;
-  const bool valid = item < g.Bt * g.nb * g.H;
-  float sc = 0.f, sn = 0.f;
-  if (valid) {
-    const int64_t bk = item / g.H, b = bk / g.nb, k = bk % g.nb;
-    const int h = (int)(item % g.H);
-    const int64_t rs = (int64_t)g.H * kSsdP;  // between tokens
-    const int qt = (int)(g.Bs / 4);             // tokens per quarter, a multiple of 16
-    const int64_t o0 = ((b * g.L + k * g.Bs + wq * qt + (lane >> 3)) * g.H + h) * kSsdP + (lane & 7) * 8;
-    for (int j0 = 0; j0 < qt; j0 += 16) {
-      uint4 an[4], bn[4], ac[4], bc[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int64_t o = o0 + (int64_t)(j0 + 4 * u) * rs;
-        an[u] = __ldg(reinterpret_cast<const uint4*>(dyn + o));
-        bn[u] = __ldg(reinterpret_cast<const uint4*>(xn + o));
-        if (CLEAN) {
-          ac[u] = __ldg(reinterpret_cast<const uint4*>(dyc + o));
-          bc[u] = __ldg(reinterpret_cast<const uint4*>(xc + o));
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        sn = dot8(an[u], bn[u], sn);
-        if (CLEAN) sc = dot8(ac[u], bc[u], sc);
-      }
-    }
-  }
-  sc = warp_sum(sc);
-  sn = warp_sum(sn);
-  if (lane == 0) {
-    red[half][wq][0] = sc;
-    red[half][wq][1] = sn;
-  }
-  __syncthreads();
-  if (valid && wq == 0 && lane < 2)
-    part[item * 2 + lane] = __fadd_rn(__fadd_rn(__fadd_rn(red[half][0][lane], red[half][1][lane]), red[half][2][lane]),
-                                      red[half][3][lane]);
-}
-
 // Parameter gradients per head: one CTA per head; thread t sums the (batch
-// row, block) partials t, t + 256, ... in order, then a fixed tree over the
-// threads, so the result does not depend on scheduling.
-__global__ void __launch_bounds__(256) k_ssd_bwd_par(const SsdGeo g, const float* dA_c, const float* dA_f,
-                                                     const float* dA_s, const float* dA_r, const float* dd, float* dAf,
-                                                     float* dDf, float* dAr, float* dDr) {
+// row, block) partials t, t + 256, ... in order (the dy . x partials of a
+// block in tile and warp order), then a fixed tree over the threads, so the
+// result does not depend on scheduling.
+__global__ void __launch_bounds__(256) k_ssd_bwd_par(const SsdGeo g, const float* dd_c, const float* dd_n,
+                                                     const float* dA_c, const float* dA_f, const float* dA_s,
+                                                     const float* dA_r, float* dAf, float* dDf, float* dAr,
+                                                     float* dDr) {
   __shared__ float4 red[256];
-  const int h = blockIdx.x, t = threadIdx.x;
+  const int h = blockIdx.x, t = threadIdx.x, nd = g.m * 8;
   float af = 0.f, ar = 0.f, df = 0.f, dr = 0.f;
   for (int64_t bk = t; bk < g.Bt * g.nb; bk += 256) {
     const int64_t o = bk * g.H + h;
     af = __fadd_rn(af, __fadd_rn(__fadd_rn(dA_c[o], dA_f[o]), dA_s[o]));
     ar = __fadd_rn(ar, dA_r[o]);
-    df = __fadd_rn(df, __fadd_rn(dd[o * 2], dd[o * 2 + 1]));
-    dr = __fadd_rn(dr, dd[o * 2 + 1]);
+    float sc = 0.f, sn = 0.f;
+    for (int q = 0; q < nd; ++q) {
+      sc = __fadd_rn(sc, dd_c[o * nd + q]);
+      sn = __fadd_rn(sn, dd_n[o * nd + q]);
+    }
+    df = __fadd_rn(df, __fadd_rn(sc, sn));
+    dr = __fadd_rn(dr, sn);
   }
   red[t] = make_float4(af, ar, df, dr);
   __syncthreads();
@@ -1226,20 +1188,10 @@ cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, co
   return cudaGetLastError();
 }
 
-cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const __nv_bfloat16* xc, const __nv_bfloat16* dyc,
-                                  const __nv_bfloat16* xn, const __nv_bfloat16* dyn, float* dd, const float* dA_c,
+cudaError_t launch_ssd_bwd_params(const SsdGeo& g, const float* dd_c, const float* dd_n, const float* dA_c,
                                   const float* dA_f, const float* dA_s, const float* dA_r, float* dAf, float* dDf,
                                   float* dAr, float* dDr, cudaStream_t s) {
-  const int64_t items = g.Bt * g.nb * g.H;
-  if (items > 0) {
-    if (dyc != nullptr)
-      k_ssd_bwd_dd<true><<<(unsigned)((items + 1) / 2), 256, 0, s>>>(g, xc, dyc, xn, dyn, dd);
-    else
-      k_ssd_bwd_dd<false><<<(unsigned)((items + 1) / 2), 256, 0, s>>>(g, xc, dyc, xn, dyn, dd);
-    cudaError_t e = api_launched(cudaGetLastError(), s);
-    if (e != cudaSuccess) return e;
-  }
-  k_ssd_bwd_par<<<(unsigned)g.H, 256, 0, s>>>(g, dA_c, dA_f, dA_s, dA_r, dd, dAf, dDf, dAr, dDr);
+  k_ssd_bwd_par<<<(unsigned)g.H, 256, 0, s>>>(g, dd_c, dd_n, dA_c, dA_f, dA_s, dA_r, dAf, dDf, dAr, dDr);
   return cudaGetLastError();
 }
 
