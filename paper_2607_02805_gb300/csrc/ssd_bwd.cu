@@ -1002,14 +1002,14 @@ __global__ void __launch_bounds__(256) k_ssd_bwd_dx(const SsdGeo g, const float*
   const int64_t hb = (b * g.nb + k) * g.H + h, idx = (bt * g.H + h) * kSsdP + pp;
   const int64_t stride_i = (int64_t)g.Bs * kSsdP;  // between the tile partials of one head
   const int64_t po = (hb * m * g.Bs + s) * kSsdP + pp;
-  // m is 1 or 2: every load is issued before the sums (in the order
-  // i = j..m-1 forward, 0..j reverse); a slab that does not reach s is read
-  // and dropped, which keeps the loads independent of j
+  // m is 1 or 2: only the tiles that reach s are read (j is the same for a
+  // warp's threads but at the ends of 128-token tiles), every load before
+  // the sums (in the order i = j..m-1 forward, 0..j reverse)
   const bool two = m > 1;
   const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-  const float4 c0 = ld4(dxp_c + po), f0 = ld4(dxp_f + po), r0 = ld4(dxp_r + po);
+  const float4 c0 = j == 0 ? ld4(dxp_c + po) : z, f0 = j == 0 ? ld4(dxp_f + po) : z, r0 = ld4(dxp_r + po);
   const float4 c1 = two ? ld4(dxp_c + po + stride_i) : z, f1 = two ? ld4(dxp_f + po + stride_i) : z,
-               r1 = two ? ld4(dxp_r + po + stride_i) : z;
+               r1 = j == 1 ? ld4(dxp_r + po + stride_i) : z;
   const float4 st = ld4(dxs + (hb * g.Bs + s) * kSsdP + pp);
   const float4 yc = dyc != nullptr ? bf4(dyc + idx) : z, yn = bf4(dyn + idx);
   float4 c = j == 0 ? c0 : z, n = j == 0 ? f0 : z;
