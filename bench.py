@@ -610,13 +610,14 @@ def ssd_bwd_tile_flops(Bt, L, Bs, H, N, seeded):
     issues. Per block and (tile i, s-tile j) pair the direction reaches: per
     head group G = C B^T (K = N) and, with the head-summed dG split into bf16
     high and low parts, dC += dG B and dB = dG^T C (K = 128, twice each); per
-    head Q = dy x^T (K = 64) and dx = M^T dy (K = 128). Per head and tile of a
+    head Q = dy x^T (K = 64) and D = M'^T dy (K = 128) with M' split into its
+    two bf16 parts (dx and the column sums come from D). Per head and tile of a
     seeded block after the first: (E dy) S (K = 64) and C S^T (K = N) with the
     seed's two parts, and C^T (E dy) (K = 128, C padded to 128 rows)."""
     m, nb = Bs // 128, L // Bs
     _, ngrp = ssd_bwd_head_groups(Bt, L, Bs, H)
     pairs = m * (m + 1) // 2
-    per_pair = ngrp * (2.0 * 128 * 128 * N + 2 * 2 * (2.0 * 128 * N * 128)) + H * 2 * (2.0 * 128 * 128 * 64)
+    per_pair = ngrp * (2.0 * 128 * 128 * N + 2 * 2 * (2.0 * 128 * N * 128)) + H * 3 * (2.0 * 128 * 128 * 64)
     f = Bt * nb * pairs * per_pair
     if seeded:
         f += Bt * (nb - 1) * m * H * (2 * (2.0 * 128 * N * 64) + 2 * (2.0 * 128 * 64 * N) + 2.0 * 128 * 64 * 128)
