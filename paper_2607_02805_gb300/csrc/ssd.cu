@@ -298,6 +298,7 @@ struct ScanSmem {
 };
 
 constexpr int kScanThreads = 256;
+constexpr int kScanIssuer = 128;  // the thread that issues a head's MMAs
 constexpr int kMaxHeadsPerCta = 16;
 
 // Issues the cp.async copies of one head's x tiles (MN-major) and its seed
@@ -649,7 +650,11 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
     umma::fence_async_smem();
     umma::fence_before_sync();
     __syncthreads();
-    if (t == 0) {
+    // The issuing thread is held while the tensor pipe takes the MMAs, so it
+    // is thread 128: warp 4 (rows 0..31, right column half) has the least
+    // mixing work on a diagonal tile (nothing for a clean block's, one term
+    // per column group for a noisy block's)
+    if (t == kScanIssuer) {
       issue(0, xcur, has_seed);
       if (ntile == 1) umma::mma_commit(&bar[0]);
     }
@@ -658,7 +663,7 @@ __global__ void __launch_bounds__(kScanThreads, 1) k_ssd_block_scan(const SsdSca
       umma::fence_async_smem();
       umma::fence_before_sync();
       __syncthreads();
-      if (t == 0) {
+      if (t == kScanIssuer) {
         issue(1, xcur, false);
         umma::mma_commit(&bar[0]);
       }
