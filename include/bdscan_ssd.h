@@ -164,6 +164,14 @@ int bdscan_ssd_wait_selftest(uint32_t polls);
  * fall back to cp.async. Left-to-right streams use TMA when available. */
 int bdscan_ssd_tma_enabled(void);
 
+/* Allows (enable != 0, the default) or forbids TMA operand loads for the
+ * calls that follow, process-wide; forbidden, every kernel stages its tiles
+ * with cp.async, the path taken where the driver has no tensor-map encoder.
+ * The results are the same bits either way (the arithmetic does not depend
+ * on how tiles arrive). Returns bdscan_ssd_tma_enabled() afterwards. Not to
+ * be changed while calls are in flight on another thread. */
+int bdscan_ssd_set_tma(int enable);
+
 #ifdef __cplusplus
 }
 #endif

@@ -150,6 +150,7 @@ SIGNATURES = [
     ("bdscan_debug_set_slack", ctypes.c_int, [ctypes.c_longlong]),
     ("bdscan_ssd_wait_selftest", ctypes.c_int, [ctypes.c_uint32]),
     ("bdscan_ssd_tma_enabled", ctypes.c_int, []),
+    ("bdscan_ssd_set_tma", ctypes.c_int, [ctypes.c_int]),
     ("bdscan_ssd_full_bidir_workspace_size", ctypes.c_size_t, [_P(bdscan_ssd_dims)]),
     ("bdscan_ssd_full_bidir_forward", ctypes.c_int,
      [_P(bdscan_ssd_dims), _P(bdscan_noisy), _P(bdscan_params), c_void_p, c_void_p, ctypes.c_size_t, c_void_p]),
@@ -383,6 +384,10 @@ def bdscan_ssd_wait_selftest(polls) -> int:
 
 def bdscan_ssd_tma_enabled() -> int:
     return load().bdscan_ssd_tma_enabled()
+
+
+def bdscan_ssd_set_tma(enable) -> int:
+    return load().bdscan_ssd_set_tma(int(enable))
 
 
 def bdscan_ssd_full_bidir_workspace_size(dims) -> int:

@@ -829,13 +829,19 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-bool ssd_tma_enabled() { return tensor_map_encoder() != nullptr; }
+// Whether the launchers may use TMA at all (bdscan_ssd_set_tma): the
+// cp.async path stays callable on hardware that has TMA, for its tests.
+static std::atomic<int> g_tma_allowed{1};
+void ssd_set_tma(bool on) { g_tma_allowed.store(on ? 1 : 0); }
+
+bool ssd_tma_enabled() { return g_tma_allowed.load() != 0 && tensor_map_encoder() != nullptr; }
 
 // x [rows][H][64] bf16 as a 3-D map with boxes of 64 channels x 1 head x 128
 // tokens, 128-byte swizzle (the layout the MMA descriptors read).
 bool encode_head_map(CUtensorMap* m, const __nv_bfloat16* x, int64_t rows, int H) {
   PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
-  if (enc == nullptr || rows >= ((int64_t)1 << 31) || ((uintptr_t)x & 15u) != 0) return false;
+  if (enc == nullptr || g_tma_allowed.load() == 0 || rows >= ((int64_t)1 << 31) || ((uintptr_t)x & 15u) != 0)
+    return false;
   const cuuint64_t dims[3] = {(cuuint64_t)kSsdP, (cuuint64_t)H, (cuuint64_t)rows};
   const cuuint64_t strides[2] = {(cuuint64_t)kSsdP * 2, (cuuint64_t)H * kSsdP * 2};  // bytes, dims 1 and 2
   const cuuint32_t box[3] = {(cuuint32_t)kSsdP, 1u, (cuuint32_t)kSsdT};

@@ -157,7 +157,8 @@ cudaError_t launch_ssd_block_state(const SsdStateParams& p, cudaStream_t s);
 cudaError_t launch_ssd_state_pass(const SsdPassParams& p, cudaStream_t s);
 cudaError_t launch_ssd_block_scan(bool noisy, const SsdScanParams& p, cudaStream_t s);
 int* ssd_wait_flag_ptr();  // device address of the wait flag (current device), or null
-bool ssd_tma_enabled();    // the tensor-map encoder is available (TMA operand loads)
+bool ssd_tma_enabled();    // the tensor-map encoder is available and TMA is allowed
+void ssd_set_tma(bool on);  // allow (default) or forbid TMA operand loads
 // A [rows][H][64] bf16 tensor (x, dy) as a 3-D tensor map with boxes of 64
 // channels x 1 head x 128 tokens and 128-byte swizzle; false if unavailable.
 bool encode_head_map(CUtensorMap* m, const __nv_bfloat16* base, int64_t rows, int H);

@@ -318,6 +318,11 @@ int bdscan_ssd_wait_flag(int reset) {
 
 int bdscan_ssd_tma_enabled(void) { return bds::ssd_tma_enabled() ? 1 : 0; }
 
+int bdscan_ssd_set_tma(int enable) {
+  bds::ssd_set_tma(enable != 0);
+  return bds::ssd_tma_enabled() ? 1 : 0;
+}
+
 int bdscan_ssd_wait_selftest(uint32_t polls) {
   const char* fn = "bdscan_ssd_wait_selftest";
   bds::api_begin();

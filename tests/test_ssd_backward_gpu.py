@@ -124,6 +124,34 @@ def test_ssd_backward_is_deterministic():
         assert torch.equal(first[k], g[k]), k
 
 
+def test_ssd_cp_async_path_matches_tma_bit_exact():
+    """The cp.async staging (taken where the driver has no tensor-map encoder)
+    gives the same bits as the TMA path, forward and backward: the arithmetic
+    does not depend on how the tiles arrive."""
+    wl = SsdWorkload(2, 512, 256, 3, 128, seed=74, with_grads=True)
+
+    def both():
+        t, st, g, (d, _) = _run(wl)
+        y_c = torch.empty((wl.batch, wl.len, wl.heads, 64), dtype=torch.bfloat16, device="cuda")
+        y_n = torch.empty_like(y_c)
+        ws = torch.empty(binding.bdscan_ssd_forward_workspace_size(d), dtype=torch.uint8, device="cuda")
+        binding.ssd_forward(d, t, y_c, y_n, torch.empty_like(st), ws)
+        torch.cuda.synchronize()
+        return st, dict(g, y_c=y_c, y_n=y_n)
+
+    assert binding.bdscan_ssd_set_tma(1) == 1
+    st_tma, out_tma = both()
+    try:
+        assert binding.bdscan_ssd_set_tma(0) == 0
+        st_cp, out_cp = both()
+    finally:
+        binding.bdscan_ssd_set_tma(1)
+    assert binding.bdscan_ssd_wait_flag(1) == 0
+    assert torch.equal(st_tma, st_cp)
+    for k in out_tma:
+        assert torch.equal(out_tma[k], out_cp[k]), k
+
+
 @pytest.mark.parametrize("cfg,heads,rows", [
     ((8, 8192, 256, 26, 128), [0, 25], [3]),   # 350M-class layer
     ((8, 8192, 256, 14, 64), [7], [0]),        # 87M-class layer
