@@ -261,15 +261,17 @@ def _full_size_check(Bt, L, Bs, D, N, seed, sub, sums_row):
 
 
 def test_config_87m_layer_full_size():
-    """batch 8, 2048 tokens per stream, block 16, d_inner 1536, d_state 16, bf16."""
-    sub = [0, 1, 2, 31, 127, 128, 129, 700, 1023, 1024, 1534, 1535]
+    """batch 8, 2048 tokens per stream, block 16, d_inner 1536, d_state 16, bf16:
+    every channel of one 128-channel group (one CTA's channels: all warps and
+    lanes) plus the edges of others, and dB, dC over all channels of a batch row."""
+    sub = sorted({0, 1, 2, 31, 127, 128, 129, 700, 1023, 1024, 1534, 1535} | set(range(384, 512)))
     _full_size_check(8, 2048, 16, 1536, 16, 0, sub, sums_row=3)
 
 
 @pytest.mark.parametrize("Bs", [4, 8, 16, 32, 64])
 def test_config_350m_block_sweep_full_size(Bs):
     """batch 8, 2048 tokens, d_inner 2048, d_state 16, bf16, block size sweep."""
-    sub = [0, 5, 255, 256, 1337, 2047]
+    sub = sorted({0, 5, 255, 256, 1337, 2047} | set(range(1536, 1664)))  # edges and one 128-channel group
     _full_size_check(8, 2048, Bs, 2048, 16, 1, sub, sums_row={4: 0, 8: 2, 16: 5, 32: 6, 64: 7}[Bs])
 
 
