@@ -1029,49 +1029,56 @@ __global__ void __launch_bounds__(256) k_ssd_bwd_dx(const SsdGeo g, const float*
 }
 
 // dB and dC of the three streams: the tile partials of every head group (and
-// the clean state term of every head), summed in order. One CTA per token,
-// one thread per state index.
-__global__ void __launch_bounds__(128) k_ssd_bwd_dbc(const SsdGeo g, int ngrp, const float* dBp_c, const float* dBs,
+// the clean state term of every head), summed in order. One thread per
+// (token, 4 state indices); the tile index j of a token is the same across
+// a warp but at the ends of 128-token tiles, and only the tile partials that
+// reach the token are read.
+__global__ void __launch_bounds__(256) k_ssd_bwd_dbc(const SsdGeo g, int ngrp, const float* dBp_c, const float* dBs,
                                                      const float* dCp_c, const float* dBp_f, const float* dCp_f,
                                                      const float* dBp_r, const float* dCp_r, __nv_bfloat16* dBc,
                                                      __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                                      __nv_bfloat16* dBr, __nv_bfloat16* dCr) {
-  const int N = g.N, m = g.m, n = threadIdx.x;
-  if (n >= N) return;
-  const int64_t bt = blockIdx.x, b = bt / g.L;
+  const int N = g.N, m = g.m, Q = N / 4;
+  const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  if (i >= g.Bt * g.L * Q) return;
+  const int64_t bt = i / Q, b = bt / g.L;
+  const int n = (int)(i - bt * Q) * 4;
   const int tl = (int)(bt - b * g.L), k = tl / (int)g.Bs, s = tl - k * (int)g.Bs, j = s / kSsdT;
   const int64_t bk = b * g.nb + k, idx = bt * N + n;
-  float bc = 0.f, cc = 0.f, bf = 0.f, cf = 0.f, br = 0.f, cr = 0.f;
+  const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  float4 bc = z, cc = z, bf = z, cf = z, br = z, cr = z;
+  const bool two = m > 1;
   for (int q = 0; q < ngrp; ++q) {
     const int64_t gb = bk * ngrp + q;
     const int64_t tp = (gb * m * g.Bs + s) * N + n, ti = (int64_t)g.Bs * N, c1 = (gb * g.Bs + s) * N + n;
     // m is 1 or 2: the loads first, then the sums in the order i = j..m-1
     // (forward), 0..j (reverse)
-    const float bc0 = dBp_c[tp], bf0 = dBp_f[tp], br0 = dBp_r[tp];
-    const float bc1 = m > 1 ? dBp_c[tp + ti] : 0.f, bf1 = m > 1 ? dBp_f[tp + ti] : 0.f, br1 = m > 1 ? dBp_r[tp + ti] : 0.f;
-    const float cc0 = dCp_c[c1], cf0 = dCp_f[c1], cr0 = dCp_r[c1];
+    const float4 bc0 = j == 0 ? ld4(dBp_c + tp) : z, bf0 = j == 0 ? ld4(dBp_f + tp) : z, br0 = ld4(dBp_r + tp);
+    const float4 bc1 = two ? ld4(dBp_c + tp + ti) : z, bf1 = two ? ld4(dBp_f + tp + ti) : z,
+                 br1 = j == 1 ? ld4(dBp_r + tp + ti) : z;
+    const float4 cc0 = ld4(dCp_c + c1), cf0 = ld4(dCp_f + c1), cr0 = ld4(dCp_r + c1);
     if (j == 0) {
-      bc = __fadd_rn(bc, bc0);
-      bf = __fadd_rn(bf, bf0);
+      bc = add4(bc, bc0);
+      bf = add4(bf, bf0);
     }
-    if (m > 1) {
-      bc = __fadd_rn(bc, bc1);
-      bf = __fadd_rn(bf, bf1);
+    if (two) {
+      bc = add4(bc, bc1);
+      bf = add4(bf, bf1);
     }
-    br = __fadd_rn(br, br0);
-    if (j == 1) br = __fadd_rn(br, br1);
-    cc = __fadd_rn(cc, cc0);
-    cf = __fadd_rn(cf, cf0);
-    cr = __fadd_rn(cr, cr0);
+    br = add4(br, br0);
+    if (j == 1) br = add4(br, br1);
+    cc = add4(cc, cc0);
+    cf = add4(cf, cf0);
+    cr = add4(cr, cr0);
   }
   const float* st = dBs + (bk * g.H * g.Bs + s) * N + n;
-  for (int h = 0; h < g.H; ++h) bc = __fadd_rn(bc, st[(int64_t)h * g.Bs * N]);
-  dBc[idx] = __float2bfloat16_rn(bc);
-  dCc[idx] = __float2bfloat16_rn(cc);
-  dBf[idx] = __float2bfloat16_rn(bf);
-  dCf[idx] = __float2bfloat16_rn(cf);
-  dBr[idx] = __float2bfloat16_rn(br);
-  dCr[idx] = __float2bfloat16_rn(cr);
+  for (int h = 0; h < g.H; ++h) bc = add4(bc, ld4(st + (int64_t)h * g.Bs * N));
+  st_bf4(dBc + idx, bc);
+  st_bf4(dCc + idx, cc);
+  st_bf4(dBf + idx, bf);
+  st_bf4(dCf + idx, cf);
+  st_bf4(dBr + idx, br);
+  st_bf4(dCr + idx, cr);
 }
 
 // Parameter gradients per head: one CTA per head; thread t sums the (batch
@@ -1183,8 +1190,10 @@ cudaError_t launch_ssd_bwd_dbc(const SsdGeo& g, int ngrp, const float* dBp_c, co
                                const float* dBp_f, const float* dCp_f, const float* dBp_r, const float* dCp_r,
                                __nv_bfloat16* dBc, __nv_bfloat16* dCc, __nv_bfloat16* dBf, __nv_bfloat16* dCf,
                                __nv_bfloat16* dBr, __nv_bfloat16* dCr, cudaStream_t s) {
-  k_ssd_bwd_dbc<<<(unsigned)(g.Bt * g.L), 128, 0, s>>>(g, ngrp, dBp_c, dBs, dCp_c, dBp_f, dCp_f, dBp_r, dCp_r, dBc, dCc,
-                                                            dBf, dCf, dBr, dCr);
+  const int64_t n = g.Bt * g.L * (g.N / 4);
+  if (n == 0) return cudaSuccess;
+  k_ssd_bwd_dbc<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(g, ngrp, dBp_c, dBs, dCp_c, dBp_f, dCp_f, dBp_r, dCp_r, dBc,
+                                                              dCc, dBf, dCf, dBr, dCr);
   return cudaGetLastError();
 }
 
