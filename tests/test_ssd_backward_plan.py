@@ -1,9 +1,11 @@
 """CPU check of the decomposition the SSD-form backward kernels follow (fp64
 numpy, small sizes): per block and head, the products Q = dy x^T and
-G = C B^T, the masked decays, row and column sums turned into dt and A
-gradients by a cumulative sum inside the block, the seed terms, a reverse pass
-over block-end states, and the transpose of the block-state product. Its
-gradients must equal the oracle's (tied diagonal backward) for every input.
+G = C B^T, the masked decays M' = G o decay, D = M'^T dy (dx = diag(dt) D,
+and the column sums of R' = Q o M' as x_s . D_s), row and column sums turned
+into dt and A gradients by a cumulative sum inside the block, the seed terms,
+a reverse pass over block-end states, and the transpose of the block-state
+product. Its gradients must equal the oracle's (tied diagonal backward) for
+every input.
 Everything here is written from the matrix form of Sec. 4 (eqs.
 boundary-state and partial-reverse) with scalar decays per head."""
 
@@ -24,12 +26,13 @@ def _direction(dy, x, dt, B, C, A, seed, upper):
     mask = np.triu(np.ones((T, T))) if upper else np.tril(np.ones((T, T)))
     dec = np.exp(A * np.where(mask > 0, diff, 0.0)) * mask
     G = C @ B.T
-    M = G * dec * dt[None, :]
+    Mp = G * dec                                               # M' (without dt_s)
     Q = dy @ x.T                                               # dy_t . x_s
-    Rp = Q * G * dec                                           # without dt_s
-    R = Rp * dt[None, :]
+    R = Q * Mp * dt[None, :]                                   # R = R' diag(dt), R' = Q o M'
     dG = Q * dec * dt[None, :]
-    dx = M.T @ dy
+    D = Mp.T @ dy                                              # D_s = sum_t M'[t, s] dy_t
+    dx = dt[:, None] * D
+    colsum = np.sum(x * D, axis=1)                             # colsum_s R' = x_s . D_s
     dC = dG @ B
     dB = dG.T @ C
     rowdot = np.zeros(T)
@@ -40,9 +43,9 @@ def _direction(dy, x, dt, B, C, A, seed, upper):
         rowdot = np.sum(dy * Ys, axis=1)                       # dy_t . seed term_t
         dC = dC + E[:, None] * (dy @ seed)
         dseed = (E[:, None] * dy).T @ C
-    dc = A * (R.sum(axis=1) - R.sum(axis=0) + rowdot)
+    dc = A * (R.sum(axis=1) - dt * colsum + rowdot)
     # c_t = sum of dt over q <= t (forward) or q >= t (reverse)
-    ddt = Rp.sum(axis=0) + (np.cumsum(dc[::-1])[::-1] if not upper else np.cumsum(dc))
+    ddt = colsum + (np.cumsum(dc[::-1])[::-1] if not upper else np.cumsum(dc))
     dA = float(np.sum(c * dc)) / A
     return dx, dB, dC, ddt, dA, dseed
 
