@@ -60,6 +60,7 @@ struct StateSmem {
 };
 
 constexpr int kStateThreads = 256;
+constexpr int kStateIssuer = 64;  // the thread that issues a head's MMAs (k_ssd_block_state)
 
 // One CTA of 8 warps per (batch row, block) and group of at most 8 heads.
 // T^T[n][p] = sum_s B_s[n] (w_s x_s[p]): M = 128 state rows, N = 64
@@ -177,7 +178,10 @@ __global__ void __launch_bounds__(kStateThreads, 1) k_ssd_block_state(const SsdS
     umma::fence_async_smem();
     umma::fence_before_sync();
     __syncthreads();
-    if (t == 0) {
+    // the issuing thread is held while the tensor pipe takes the MMAs: thread
+    // 64's warp writes no output rows when N is 64 (only warps with
+    // 32 (w mod 4) < N do), so the previous head's write-out runs beside it
+    if (t == kStateIssuer) {
       umma::fence_after_sync();
       const uint32_t a0 = umma::smem_u32(sm + S.b), x0 = umma::smem_u32(sm + S.xs);
       constexpr uint32_t id = umma::idesc_bf16(128, 64, true, true);
