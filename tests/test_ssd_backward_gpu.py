@@ -152,6 +152,32 @@ def test_ssd_cp_async_path_matches_tma_bit_exact():
         assert torch.equal(out_tma[k], out_cp[k]), k
 
 
+def test_bench_event_lists_match_launches():
+    """bench.py times every SSD kernel with one CUDA event per launch, so its
+    kernel lists must name each launch of a forward and of a backward call."""
+    import importlib.util
+    import os
+    path = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "bench.py")
+    spec = importlib.util.spec_from_file_location("bench_lists", path)
+    bench = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(bench)
+    wl = SsdWorkload(2, 512, 256, 3, 128, seed=75, with_grads=True)
+    t = _dev(wl)
+    d = binding.make_ssd_dims(wl.batch, wl.len, wl.block, wl.heads, wl.d_state)
+    y_c = torch.empty((wl.batch, wl.len, wl.heads, 64), dtype=torch.bfloat16, device="cuda")
+    y_n = torch.empty_like(y_c)
+    st = torch.empty((wl.batch, wl.len // wl.block, wl.heads, 64, wl.d_state), dtype=torch.float32, device="cuda")
+    ws = torch.empty(binding.bdscan_ssd_forward_workspace_size(d), dtype=torch.uint8, device="cuda")
+    binding.ssd_forward(d, t, y_c, y_n, st, ws)
+    assert binding.bdscan_last_launch_count() == len(bench.SSD_KERNELS)
+    g = {k: torch.empty(v.shape, dtype=torch.float32 if k in P.PARAMS else torch.bfloat16, device="cuda")
+         for k, v in t.items() if k in NAMES}
+    wsb = torch.empty(binding.bdscan_ssd_backward_workspace_size(d), dtype=torch.uint8, device="cuda")
+    binding.ssd_backward(d, t, st, t["dy_c"], t["dy_n"], None, g, wsb)
+    assert binding.bdscan_last_launch_count() == len(bench.SSD_BWD_KERNELS)
+    torch.cuda.synchronize()
+
+
 @pytest.mark.parametrize("cfg,heads,rows", [
     ((8, 8192, 256, 26, 128), [0, 25], [3]),   # 350M-class layer
     ((8, 8192, 256, 14, 64), [7], [0]),        # 87M-class layer
