@@ -240,7 +240,7 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
       for (int sg = 0; sg < NSEG; ++sg) {  // segments left to right
         const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
         if (NSEG > 1) st.load(prow(row0 + i0), ns, g.D, d0);
-#pragma unroll 4
+#pragma unroll 2
         for (int ii = 0; ii < ns; ++ii) {
           const int i = i0 + ii;
           const int64_t o = prow(row0 + i) * g.D + d;
@@ -272,7 +272,7 @@ __global__ void __launch_bounds__(kCta, 4) k_block_scan(const FwdParams p) {
         for (int sg = NSEG - 1; sg >= 0; --sg) {  // segments right to left; the last is still staged
           const int i0 = sg * SEG, ns = Bs - i0 < SEG ? Bs - i0 : SEG;
           if (sg < NSEG - 1) st.load(prow(row0 + i0), ns, g.D, d0);
-#pragma unroll 4
+#pragma unroll 2
           for (int ii = ns - 1; ii >= 0; --ii) {
             const int i = i0 + ii;
             const int64_t o = prow(row0 + i) * g.D + d;
