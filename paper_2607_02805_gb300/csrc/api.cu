@@ -639,7 +639,7 @@ int bdscan_debug_set_slack(long long elements) {
 int64_t bdscan_chunk_tokens(int64_t block) { return block <= 0 ? 0 : blocks_per_chunk(block) * block; }
 
 size_t bdscan_forward_workspace_size(const bdscan_dims* dims) {
-  Call c;
+  Call c{};
   if (check_dims_any(dims, &c, "bdscan_forward_workspace_size") != BDSCAN_OK) return 0;
   if (!direct_N(c.N)) return fwd_group_ws(c).total;
   return fwd_ws(c.g, c.N);
@@ -647,14 +647,14 @@ size_t bdscan_forward_workspace_size(const bdscan_dims* dims) {
 
 size_t bdscan_boundary_states_workspace_size(const bdscan_dims* dims, int emit_all) {
   (void)emit_all;
-  Call c;
+  Call c{};
   if (check_dims_any(dims, &c, "bdscan_boundary_states_workspace_size") != BDSCAN_OK) return 0;
   if (!direct_N(c.N)) return bnd_group_ws(c, emit_all).total;
   return fwd_ws(c.g, c.N);
 }
 
 size_t bdscan_backward_workspace_size(const bdscan_dims* dims) {
-  Call c;
+  Call c{};
   if (check_dims_any(dims, &c, "bdscan_backward_workspace_size") != BDSCAN_OK) return 0;
   if (!direct_N(c.N)) return bwd_group_ws(c).total;
   bds::Geo gmax = c.g;
@@ -666,7 +666,7 @@ int bdscan_forward(const bdscan_dims* dims, const bdscan_clean* clean, const bds
                    const bdscan_params* params, void* y_c, void* y_n, float* states, void* workspace,
                    size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_forward";
-  Call c;
+  Call c{};
   int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, false, fn))) return rc;
@@ -706,7 +706,7 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
                            const float* D_f, const float* init_state, void* y_c, float* states, int emit_all,
                            void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_boundary_states";
-  Call c;
+  Call c{};
   int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, false, fn))) return rc;
@@ -751,7 +751,7 @@ int bdscan_boundary_states(const bdscan_dims* dims, const bdscan_clean* clean, c
 int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan_noisy* noisy,
                         const bdscan_params* params, void* y_n, void* stream) {
   const char* fn = "bdscan_active_block";
-  Call c;
+  Call c{};
   int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if (dims->len != dims->block && dims->len != 0)
@@ -779,7 +779,7 @@ int bdscan_active_block(const bdscan_dims* dims, const float* seed, const bdscan
 }
 
 size_t bdscan_active_block_adaln_workspace_size(const bdscan_dims* dims) {
-  Call c;
+  Call c{};
   if (check_dims(dims, &c, "bdscan_active_block_adaln_workspace_size") != BDSCAN_OK) return 0;
   return al256((size_t)c.g.Bt * c.g.L * sizeof(float2));
 }
@@ -788,7 +788,7 @@ int bdscan_active_block_adaln(const bdscan_dims* dims, const float* seed, const 
                               const bdscan_params* params, const bdscan_adaln* mod, void* out, void* workspace,
                               size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_active_block_adaln";
-  Call c;
+  Call c{};
   int rc = check_dims(dims, &c, fn);
   if (rc) return rc;
   if (dims->len != dims->block && dims->len != 0)
@@ -833,7 +833,7 @@ int bdscan_active_block_adaln(const bdscan_dims* dims, const float* seed, const 
 }
 
 size_t bdscan_full_bidir_workspace_size(const bdscan_dims* dims) {
-  Call c;
+  Call c{};
   if (check_dims(dims, &c, "bdscan_full_bidir_workspace_size") != BDSCAN_OK) return 0;
   const size_t y32 = al256((size_t)c.g.Bt * c.g.L * c.g.D * 4);
   return fwd_ws(c.g, c.N) + 2 * y32;
@@ -842,7 +842,7 @@ size_t bdscan_full_bidir_workspace_size(const bdscan_dims* dims) {
 int bdscan_full_bidir_forward(const bdscan_dims* dims, const bdscan_noisy* noisy, const bdscan_params* params,
                               void* y, void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_full_bidir_forward";
-  Call c;
+  Call c{};
   int rc = check_dims(dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, false, fn))) return rc;
@@ -885,7 +885,7 @@ int bdscan_backward(const bdscan_dims* dims, const bdscan_clean* clean, const bd
                     const float* dstates, const bdscan_clean_grads* gclean, const bdscan_noisy_grads* gnoisy,
                     const bdscan_param_grads* gparams, void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_backward";
-  Call c;
+  Call c{};
   int rc = check_dims_any(dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, true, fn))) return rc;
@@ -1033,7 +1033,7 @@ int sm_count_cached() {
 
 // Validation shared with other entry points that take forward-side dims.
 int api_check_forward_dims(const void* dims, Geo* g, int* dt, int* N, const char* fn) {
-  Call c;
+  Call c{};
   int rc = check_dims((const bdscan_dims*)dims, &c, fn);
   if (rc) return rc;
   if ((rc = check_block_limits(c, false, fn))) return rc;

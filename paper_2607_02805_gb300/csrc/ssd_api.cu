@@ -206,7 +206,7 @@ cudaError_t build_states(const bds::SsdGeo& g, const bdscan_clean* c, const floa
 extern "C" {
 
 size_t bdscan_ssd_forward_workspace_size(const bdscan_ssd_dims* dims) {
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   if (check(dims, &g, "bdscan_ssd_forward_workspace_size") != BDSCAN_OK) return 0;
   return sumdt_bytes(g);
 }
@@ -215,7 +215,7 @@ int bdscan_ssd_forward(const bdscan_ssd_dims* dims, const bdscan_clean* clean, c
                        const bdscan_params* params, void* y_c, void* y_n, float* states, void* workspace,
                        size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_ssd_forward";
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   int rc = check(dims, &g, fn);
   if (rc) return rc;
   if (g.Bt == 0 || g.nb == 0 || g.H == 0) return bds::api_ok();
@@ -246,7 +246,7 @@ int bdscan_ssd_forward(const bdscan_ssd_dims* dims, const bdscan_clean* clean, c
 }
 
 size_t bdscan_ssd_boundary_states_workspace_size(const bdscan_ssd_dims* dims, int emit_all) {
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   if (check(dims, &g, "bdscan_ssd_boundary_states_workspace_size") != BDSCAN_OK) return 0;
   return sumdt_bytes(g) + (emit_all ? 0 : states_bytes(g));
 }
@@ -255,7 +255,7 @@ int bdscan_ssd_boundary_states(const bdscan_ssd_dims* dims, const bdscan_clean* 
                                const float* D_f, const float* init_state, void* y_c, float* states,
                                int emit_all, void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_ssd_boundary_states";
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   int rc = check(dims, &g, fn);
   if (rc) return rc;
   if (g.Bt == 0 || g.nb == 0 || g.H == 0) return bds::api_ok();
@@ -287,7 +287,7 @@ int bdscan_ssd_boundary_states(const bdscan_ssd_dims* dims, const bdscan_clean* 
 int bdscan_ssd_active_block(const bdscan_ssd_dims* dims, const float* seed, const bdscan_noisy* noisy,
                             const bdscan_params* params, void* y_n, void* stream) {
   const char* fn = "bdscan_ssd_active_block";
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   int rc = check(dims, &g, fn);
   if (rc) return rc;
   if (dims->len != dims->block) return fail_msg(BDSCAN_ERR_ARG, fn, "len must equal block");
@@ -338,7 +338,7 @@ int bdscan_ssd_wait_selftest(uint32_t polls) {
 }
 
 size_t bdscan_ssd_full_bidir_workspace_size(const bdscan_ssd_dims* dims) {
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   if (check(dims, &g, "bdscan_ssd_full_bidir_workspace_size") != BDSCAN_OK) return 0;
   return sumdt_bytes(g) + states_bytes(g) + al256((size_t)g.Bt * g.L * g.H * 64 * 4);
 }
@@ -346,7 +346,7 @@ size_t bdscan_ssd_full_bidir_workspace_size(const bdscan_ssd_dims* dims) {
 int bdscan_ssd_full_bidir_forward(const bdscan_ssd_dims* dims, const bdscan_noisy* noisy, const bdscan_params* params,
                                   void* y, void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_ssd_full_bidir_forward";
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   int rc = check(dims, &g, fn);
   if (rc) return rc;
   if (g.Bt == 0 || g.nb == 0 || g.H == 0) return bds::api_ok();
@@ -447,7 +447,7 @@ SsdBwdWs ssd_bwd_ws(const bds::SsdGeo& g) {
 }  // namespace
 
 extern "C" size_t bdscan_ssd_backward_workspace_size(const bdscan_ssd_dims* dims) {
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   if (check(dims, &g, "bdscan_ssd_backward_workspace_size") != BDSCAN_OK) return 0;
   return ssd_bwd_ws(g).total;
 }
@@ -458,7 +458,7 @@ extern "C" int bdscan_ssd_backward(const bdscan_ssd_dims* dims, const bdscan_cle
                                    const bdscan_noisy_grads* gnoisy, const bdscan_param_grads* gparams,
                                    void* workspace, size_t workspace_bytes, void* stream) {
   const char* fn = "bdscan_ssd_backward";
-  bds::SsdGeo g;
+  bds::SsdGeo g{};
   int rc = check(dims, &g, fn);
   if (rc) return rc;
   if (gparams == nullptr) return fail_msg(BDSCAN_ERR_ARG, fn, "gparams is NULL");
